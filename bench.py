@@ -1,0 +1,353 @@
+#!/usr/bin/env python3
+"""Retrieve throughput of the MemAttention memory hot path on GB300.
+
+One step = one retrieval pass (score -> two relation hops -> top-k -> page
+resolve) of a batch of 256 bf16 queries against the N=1,048,576-chunk,
+d=1024 synthetic store (gmm1m recipe: 4096-component Zipf(1.1) mixture,
+32-neighbour power-law relation graph, 64 chunks per page, clustered
+placement), k=32, alpha=0.5.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl reference]
+
+N>1 runs under torch.distributed.run: every rank runs an independent
+replica of the store on its own GPU (queries are independent; there is no
+collective on the data path); timing is the max over ranks and `value`
+counts the queries of all ranks.  `--impl reference` times the CPU oracle
+(plain single-threaded fp64 C) on a bounded sample of the same workload.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "retrieve queries/sec at N=1M chunks, d=1024, B=256; % of roofline"
+WORKLOAD = ("gmm1m: N=1048576 chunks, d=1024 bf16, 4096-component Zipf(1.1) mixture, 32-neighbour "
+            "power-law relation graph (nnz 33554432), B=256 queries, hops=2, alpha=0.5, k=32, "
+            "64 chunks/page, clustered placement")
+
+
+def peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return d.get("hbm_gbs", 6800.0), d.get("bf16_tflops", 1895.6), "measured"
+    return 6800.0, 1900.0, "fallback"
+
+
+def algorithmic_bytes(n, d, b, nnz, hops, k):
+    """Bytes a retrieval pass must move at least once (E once, the graph once
+    per hop, the fp32 score slab written by the score pass and, per hop, each
+    input slab read once and the output written once except the last hop's,
+    which feeds the top-k directly), plus queries, page table and outputs."""
+    slab = n * b * 4
+    graph = (n + 1) * 8 + nnz * 4 + nnz * 4
+    passes = 1 + (2 * hops if hops > 0 else 1)          # u write; per hop read in + write/ u read
+    return dict(emb=n * d * 2, graph=graph * hops, slab=slab * passes,
+                small=b * d * 2 + n * 4 + b * k * 16 + b * 4)
+
+
+def hop_bytes(n, b, nnz):
+    """One propagation hop: graph once + input slab read once + output slab written once."""
+    return (n + 1) * 8 + nnz * 8 + 2 * n * b * 4
+
+
+def score_bytes(n, d, b):
+    return n * d * 2 + n * b * 4 + b * d * 2
+
+
+class Clocks:
+    """nvidia-smi sampled during the timed region."""
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, dev):
+        self.dev = dev
+        self.proc = None
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--query-gpu={self.Q}", "--format=csv,noheader,nounits",
+                 "-lms", "200", "-i", str(self.dev)], stdout=subprocess.PIPE,
+                stderr=subprocess.DEVNULL, text=True)
+        except Exception:
+            self.proc = None
+        return self
+
+    def __exit__(self, *a):
+        self.out = ""
+        if self.proc:
+            self.proc.terminate()
+            try:
+                self.out, _ = self.proc.communicate(timeout=5)
+            except Exception:
+                self.proc.kill()
+                self.out = ""
+
+    def summary(self):
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in (self.out or "").strip().splitlines():
+            f = [x.strip() for x in line.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                mx.append(float(f[2]))
+            except ValueError:
+                continue
+            for nm, v in zip(names, f[5:9]):
+                if v.lower() == "active":
+                    reasons.add(nm)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"]}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+def cpu_baseline(wl, placement, n_queries, rng_seed=0):
+    import oracle
+    rows = np.random.default_rng(rng_seed).choice(wl.n_queries, size=n_queries, replace=False)
+    t0 = time.perf_counter()
+    w = oracle.row_softmax(wl.row_ptr, wl.aff)
+    oracle.retrieve(wl.emb, wl.queries[rows], wl.row_ptr, wl.col, w, tau=wl.tau, alpha=wl.alpha,
+                    hops=wl.hops, k=wl.k, page_of=wl.page_of[placement])
+    dt = time.perf_counter() - t0
+    return dict(value=n_queries / dt, unit="queries/s", cores=1, kind="oracle",
+                sample=f"{n_queries} of the {wl.n_queries} queries against the full store "
+                       f"(relation weights included), one thread",
+                seconds=dt)
+
+
+def dist_env():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return ws, rank, local
+
+
+def run_reference(args):
+    ws, rank, _ = dist_env()
+    if rank != 0:
+        return 0
+    import synth
+    wl = synth.workload(2, placements=("clustered",))
+    per_step = 1
+    times = []
+    for i in range(args.warmup + args.steps):
+        r = cpu_baseline(wl, "clustered", per_step, rng_seed=i)
+        if i >= args.warmup:
+            times.append(r["seconds"])
+    tot = sum(times)
+    value = per_step * len(times) / tot
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "queries/s",
+        "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": 1e3 * tot / len(times), "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": WORKLOAD, "sample": f"{per_step} query per step"},
+        "cpu_baseline": {"value": value, "unit": "queries/s", "cores": 1, "kind": "oracle",
+                         "sample": f"{per_step} query of 256 per step, full store, one thread"},
+        "e2e": {"value": value, "unit": "queries/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="native", choices=["native", "reference"])
+    ap.add_argument("--cpu-queries", type=int, default=8)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--placement", default="clustered")
+    args = ap.parse_args()
+    if args.impl == "reference":
+        return run_reference(args)
+
+    import torch
+    ws, rank, local = dist_env()
+    if ws > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl")
+    dev = local if ws > 1 else 0
+    torch.cuda.set_device(dev)
+
+    import synth
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2607_05708_gb300 import MemStore
+
+    t_gen = time.perf_counter()
+    wl = synth.workload(2)
+    t_gen = time.perf_counter() - t_gen
+    cpu = None
+    if rank == 0 and not args.no_cpu_baseline and ws == 1:
+        cpu = cpu_baseline(wl, args.placement, args.cpu_queries)
+
+    store = MemStore.from_arrays(wl.emb, wl.page_of[args.placement], wl.row_ptr, wl.col, wl.aff,
+                                 capacity=wl.n, chunks_per_page=wl.chunks_per_page,
+                                 temperature=wl.tau, device=dev)
+    B, k = wl.n_queries, wl.k
+    st = torch.cuda.Stream(device=dev)
+    q_dev = torch.from_numpy(wl.queries.view(np.int16)).to(f"cuda:{dev}")
+    ids = torch.empty((B, k), dtype=torch.int64, device=f"cuda:{dev}")
+    scores = torch.empty((B, k), dtype=torch.float32, device=f"cuda:{dev}")
+    pages = torch.empty((B, k), dtype=torch.int32, device=f"cuda:{dev}")
+    npages = torch.empty((B,), dtype=torch.int32, device=f"cuda:{dev}")
+
+    def step():
+        store.retrieve(q_dev, k, wl.alpha, wl.hops, ids, scores, pages, npages, stream=st)
+
+    def barrier():
+        torch.cuda.synchronize(dev)
+        if ws > 1:
+            torch.distributed.barrier()
+
+    with torch.cuda.stream(st):
+        for _ in range(args.warmup):
+            step()
+    store.sync(stream=st)
+    # ---- timed region (device-resident inputs)
+    store.set_profiling(True)
+    store.phase_times()                       # reset
+    barrier()
+    ev0 = torch.cuda.Event(enable_timing=True)
+    ev1 = torch.cuda.Event(enable_timing=True)
+    with Clocks(dev) as clk:
+        ev0.record(st)
+        for _ in range(args.steps):
+            step()
+        ev1.record(st)
+        barrier()
+    store.sync(stream=st)
+    ms = ev0.elapsed_time(ev1)
+    phases = store.phase_times()
+    store.set_profiling(False)
+    # page counts of this placement and of the other
+    npg_clustered = npages.float().mean().item()
+
+    # ---- end-to-end: host query buffer in, host results out, via the public API
+    q_host = torch.from_numpy(wl.queries.view(np.int16)).pin_memory()
+    outs_host = [torch.empty((B, k), dtype=torch.int64).pin_memory(),
+                 torch.empty((B, k), dtype=torch.float32).pin_memory(),
+                 torch.empty((B, k), dtype=torch.int32).pin_memory(),
+                 torch.empty((B,), dtype=torch.int32).pin_memory()]
+
+    def e2e_step():
+        with torch.cuda.stream(st):
+            q_dev.copy_(q_host, non_blocking=True)
+            step()
+            for h, d in zip(outs_host, (ids, scores, pages, npages)):
+                h.copy_(d, non_blocking=True)
+
+    for _ in range(args.warmup):
+        e2e_step()
+    barrier()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(st)
+    for _ in range(args.steps):
+        e2e_step()
+    e1.record(st)
+    barrier()
+    ms_e2e = e0.elapsed_time(e1)
+    store.sync(stream=st)
+    h2d = q_host.numel() * 2
+    d2h = sum(t.numel() * t.element_size() for t in outs_host)
+
+    # max over ranks
+    if ws > 1:
+        t = torch.tensor([ms, ms_e2e], device=f"cuda:{dev}")
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        ms, ms_e2e = t.tolist()
+
+    hbm, bf16, peak_kind = peaks()
+    ab = algorithmic_bytes(wl.n, wl.dim, B, wl.nnz, wl.hops, k)
+    total_ab = sum(ab.values())
+    per_step_ms = ms / args.steps
+    # dominant phase
+    names = {"score": None, "propagate": None, "select": None}
+    dom = max(("score", "propagate", "select"), key=lambda p: phases[p][0])
+    dom_ms, dom_launches = phases[dom]
+    if dom == "propagate":
+        per_launch_bytes = hop_bytes(wl.n, 256, wl.nnz)
+        units = args.steps * wl.hops
+        what = "propagation hop (graph once + input slab read once + output slab written once)"
+    elif dom == "score":
+        per_launch_bytes = score_bytes(wl.n, wl.dim, 256)
+        units = args.steps
+        what = "score pass (E read once + u slab written once)"
+    else:
+        per_launch_bytes = wl.n * 256 * 4
+        units = args.steps
+        what = "selection pass (final slab read once)"
+    dom_avg_ms = dom_ms / units
+    achieved = per_launch_bytes / (dom_avg_ms * 1e-3) / 1e9
+    line = {
+        "metric": METRIC,
+        "value": B * args.steps * ws / (ms * 1e-3),
+        "unit": "queries/s",
+        "n_gpus": ws,
+        "steps": args.steps,
+        "warmup": args.warmup,
+        "ms_per_step": per_step_ms,
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "f32",
+        "data": "synthetic",
+        "config": {"workload": WORKLOAD, "l2": "inputs larger than L2 (E 2.1 GB, score slabs 1.07 GB "
+                   "each), no flush", "placement": args.placement,
+                   "parallelism": "replicas" if ws > 1 else "single GPU"},
+        "roofline": {"bound": "hbm", "achieved": achieved, "peak": hbm, "unit": "GB/s",
+                     "frac": achieved / hbm, "traffic": None, "kernel": dom, "what": what,
+                     "peak_kind": peak_kind},
+        "pass_roofline": {"algorithmic_bytes": total_ab,
+                          "ideal_ms": total_ab / (hbm * 1e9) * 1e3,
+                          "frac": (total_ab / (hbm * 1e9) * 1e3) / per_step_ms,
+                          "flops": 2.0 * wl.n * B * wl.dim,
+                          "peak_tflops_bf16": bf16},
+        "phases_ms_per_step": {p: phases[p][0] / args.steps for p in ("score", "propagate", "select")},
+        "e2e": {"value": B * args.steps * ws / (ms_e2e * 1e-3), "unit": "queries/s",
+                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
+        "gpu_launches": int(sum(v[1] for v in phases.values())),
+        "pages_per_query": {args.placement: npg_clustered},
+        "clocks": clk.summary(),
+        "gen_seconds": t_gen,
+    }
+    if cpu is not None:
+        line["cpu_baseline"] = {k2: cpu[k2] for k2 in ("value", "unit", "cores", "kind", "sample")}
+    # the other placement's page count (same selected IDs, different page table)
+    other = "random" if args.placement == "clustered" else "clustered"
+    if other in wl.page_of:
+        po = wl.page_of[other]
+        sel = ids.cpu().numpy()
+        line["pages_per_query"][other] = float(np.mean([len(set(po[r].tolist())) for r in sel]))
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    store.close()
+    if ws > 1:
+        torch.distributed.destroy_process_group()
+    return 0
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -1,0 +1,177 @@
+/*
+ * akashic_mem.h -- C ABI of the GB300 (sm_103a) memory-retrieval library.
+ *
+ * The library keeps a chunked memory store on one GPU and runs the
+ * data-parallel hot path of MemAttention's memory system (arXiv 2607.05708)
+ * in its Dense-only form (embedding similarity in place of the LLM matcher,
+ * §5.5):
+ *
+ *   retrieve  score every chunk against a batch of queries (softmax over
+ *             chunks), spread the scores along the cross-chunk relation
+ *             graph, keep the top-k chunks per query and resolve them to the
+ *             pages that hold them (query-aware retrieval, §4.1 and
+ *             Algorithm 1, lines 14-18; the locality gap |P(R_t)|, §3.2);
+ *   append    add immutable chunk records, each with a logical ID and a
+ *             physical page (§4.2: logical identity is separate from
+ *             physical placement);
+ *   update    for new chunks, select the top-M related prior chunks by
+ *             cosine similarity and link them both ways in the relation
+ *             graph (cross-chunk selection, §4.1 and Algorithm 1, line 7).
+ *
+ * Conventions
+ *   - Every entry point returns an akashic_status_t and never throws.
+ *     akashic_mem_last_error() gives a thread-local message for the last
+ *     failure on the calling thread.
+ *   - The library owns all store memory; the caller owns every argument
+ *     buffer.  Array arguments named "device" are CUDA device pointers on
+ *     the store's device; "host" ones are host pointers.
+ *   - `stream` is a cudaStream_t passed as void* (NULL = legacy default
+ *     stream).  Calls are stream-ordered: device inputs may be reused once
+ *     the stream has passed the call; outputs are valid once it has
+ *     completed.  Faults found by a kernel (a bounded device wait that
+ *     expired, an index out of range) are recorded in a device status word
+ *     and returned by the next akashic_mem_sync() on that store.
+ *   - retrieve may run concurrently on different streams (each stream gets
+ *     its own scratch); append and update must not overlap any other call
+ *     on the same store.
+ *   - Embeddings are bf16, passed as their raw 16-bit patterns (uint16_t),
+ *     row-major, `dim` values per row.
+ */
+#ifndef AKASHIC_MEM_H
+#define AKASHIC_MEM_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct akashic_mem akashic_mem_t; /* opaque, library-owned */
+
+typedef enum {
+    AKASHIC_OK = 0,
+    AKASHIC_EINVAL = 1,    /* bad argument (see each call)                       */
+    AKASHIC_ENOMEM = 2,    /* a device or host allocation failed                 */
+    AKASHIC_ECAPACITY = 3, /* the store's chunk capacity would be exceeded       */
+    AKASHIC_ECUDA = 4,     /* a CUDA runtime/driver call failed                  */
+    AKASHIC_ETIMEOUT = 5,  /* a bounded device-side wait expired                 */
+    AKASHIC_EDEVICE = 6,   /* a kernel found an inconsistent index or size       */
+    AKASHIC_ERANGE = 7     /* scores would leave fp32 range (see retrieve)       */
+} akashic_status_t;
+
+typedef struct {
+    int32_t dim;             /* embedding width; multiple of 64, 64..4096          */
+    int64_t capacity;        /* maximum number of chunks, 1..2^31-1                */
+    int32_t chunks_per_page; /* page packing for appends given no page table (>=1) */
+    int32_t device;          /* CUDA device ordinal                                */
+    float temperature;       /* softmax temperature tau; 0 => 1/sqrt(dim)          */
+    float relation_scale;    /* edge logit = scale * cosine in updates; 0 => 10    */
+} akashic_mem_config_t;
+
+/* Create an empty store on cfg->device.  Allocates the embedding table
+ * (capacity x dim bf16) and the page table up front; the relation graph
+ * grows on demand.  EINVAL for an out-of-range field, ENOMEM if the device
+ * cannot hold the table. */
+akashic_status_t akashic_mem_create(const akashic_mem_config_t *cfg, akashic_mem_t **out);
+
+/* NULL-safe.  Synchronises the store's device and frees everything. */
+void akashic_mem_destroy(akashic_mem_t *m);
+
+/* Append n immutable chunk records (§4.2: chunks are written once; the
+ * store's IDs are assigned in append order, first_id .. first_id+n-1).
+ *   emb      device, n x dim bf16 bits.
+ *   page_of  device int32[n], the physical page of each new chunk (>= 0), or
+ *            NULL: fresh pages after the highest page in use, packed
+ *            chunks_per_page at a time in ID order.
+ *   row_ptr, col, aff  optional initial out-edges of the NEW rows, as a CSR
+ *            over their local rows: row_ptr device int64[n+1] (row_ptr[0]
+ *            may be non-zero; offsets index col/aff), col device int32
+ *            (global target IDs < first_id+n, never the row itself, strictly
+ *            ascending within a row), aff device float (edge logits; the
+ *            relation weight of an edge is the softmax of its row's logits).
+ *            All three NULL => no edges.
+ *   first_id_out  host, receives first_id (may be NULL).
+ * ECAPACITY if the store would exceed its capacity; EINVAL on a bad
+ * argument; EDEVICE (at once, since this call synchronises) if the edges
+ * are not a valid CSR.  Synchronises `stream`. */
+akashic_status_t akashic_mem_append_chunks(akashic_mem_t *m, const uint16_t *emb, int64_t n,
+                                           const int32_t *page_of, const int64_t *row_ptr,
+                                           const int32_t *col, const float *aff,
+                                           int64_t *first_id_out, void *stream);
+
+/* Relation update for the chunks [first, first+n) (cross-chunk selection,
+ * Algorithm 1 line 7, in its dense form): for each such chunk c, its top-M
+ * prior chunks j < first by cosine <e_c, e_j> of the stored bf16 values
+ * (no further normalisation), ordered by cosine descending then lower ID,
+ * become its out-edges with logit relation_scale * cos; with reciprocal != 0
+ * each chosen j also gets the edge j -> c with the same logit.  Rows stay
+ * sorted by column and every touched row's weights are re-normalised (row
+ * softmax).  New chunks are not linked to each other.
+ * EINVAL if first+n > size, M < 1, M > 64, M > first, or any row in
+ * [first, first+n) already has out-edges; EDEVICE if an existing edge
+ * already points into [first, first+n).  Synchronises `stream`. */
+akashic_status_t akashic_mem_update_relations(akashic_mem_t *m, int64_t first, int64_t n,
+                                              int32_t M, int32_t reciprocal, void *stream);
+
+/* Query-aware retrieval (§4.1, Algorithm 1 lines 14-18, Dense-only form):
+ *   z[b,i] = tau <q_b, e_i>;  s0[b,:] = softmax over chunks of z[b,:];
+ *   s^(0) = u = exp(z - c_b);  s^(h)_j = u_j + alpha sum_{i->j} w_ij s^(h-1)_i
+ *   for h = 1..hops (mass flows along out-edges i -> j);
+ *   score_j = s^(hops)_j / sum_i u_i.
+ * Per query the k chunks with the largest score, ordered by score descending
+ * then lower chunk ID, and their pages (FetchByID; the number of distinct
+ * pages is |P(R_t)| of §3.2).
+ *   q        device, B x dim bf16 bits.
+ *   ids      device int64[B*k]   (row b holds query b's winners)
+ *   scores   device float[B*k]   (the final scores above)
+ *   page_ids device int32[B*k]   (page_of of each winner; may be NULL)
+ *   n_pages  device int32[B]     (distinct pages per query; may be NULL)
+ * hops = 0 or alpha = 0 => plain top-k of the softmax.  The shift c_b is the
+ * bound tau |q_b| max_i |e_i|, so no extra pass is needed; ERANGE (via
+ * akashic_mem_sync) if 2 c_b > 80, where exp would leave fp32 range.
+ * EINVAL if B < 1, k < 1, k > 64, k > size, hops < 0, hops > 16, alpha < 0
+ * or not finite.  Does not synchronise. */
+akashic_status_t akashic_mem_retrieve(akashic_mem_t *m, const uint16_t *q, int32_t B, int32_t k,
+                                      float alpha, int32_t hops, int64_t *ids, float *scores,
+                                      int32_t *page_ids, int32_t *n_pages, void *stream);
+
+/* Read back the canonical out-edge CSR.  With all array pointers NULL only
+ * the sizes are returned (host n_rows, host nnz).  Otherwise row_ptr device
+ * int64[n_rows+1], col device int32[nnz], and optionally aff / w device
+ * float[nnz] (edge logits and row-softmax weights) are written.
+ * Synchronises `stream`. */
+akashic_status_t akashic_mem_export_csr(akashic_mem_t *m, int64_t *n_rows, int64_t *nnz,
+                                        int64_t *row_ptr, int32_t *col, float *aff, float *w,
+                                        void *stream);
+
+/* Number of chunks in the store and the relation graph's edge count (host). */
+akashic_status_t akashic_mem_size(const akashic_mem_t *m, int64_t *n_chunks, int64_t *nnz);
+
+/* Synchronise `stream`, then return and clear the store's device status
+ * word (ETIMEOUT, EDEVICE or ERANGE from an earlier kernel), else OK. */
+akashic_status_t akashic_mem_sync(akashic_mem_t *m, void *stream);
+
+/* Phase timing.  With profiling on, each call records CUDA events on its
+ * own stream around every phase; akashic_mem_phase_times synchronises the
+ * recorded events and returns, per phase, the summed device milliseconds
+ * and the number of kernel launches since the last reset, then resets.
+ * Phases: */
+enum {
+    AKASHIC_PHASE_SCORE = 0,     /* query x chunk score GEMM + exp + Z partials */
+    AKASHIC_PHASE_PROPAGATE = 1, /* relation-graph hops                         */
+    AKASHIC_PHASE_SELECT = 2,    /* top-k candidates, merge, page resolve       */
+    AKASHIC_PHASE_RELATE = 3,    /* new x store cosine GEMM + top-M             */
+    AKASHIC_PHASE_GRAPH = 4,     /* CSR insert, weights, transpose rebuild      */
+    AKASHIC_PHASE_COUNT = 5
+};
+akashic_status_t akashic_mem_set_profiling(akashic_mem_t *m, int32_t on);
+akashic_status_t akashic_mem_phase_times(akashic_mem_t *m, float *ms, int32_t *launches);
+
+/* Thread-local description of the last failure on this thread ("" if none). */
+const char *akashic_mem_last_error(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* AKASHIC_MEM_H */

@@ -1,0 +1,646 @@
+// The C ABI declared in include/akashic_mem.h: store lifecycle, appends,
+// relation-graph maintenance, retrieval orchestration, read-back, status and
+// phase timing.  All arithmetic runs in the kernels of the other files.
+#include <math.h>
+#include <stdarg.h>
+#include <stdio.h>
+#include <string.h>
+
+#include <mutex>
+#include <string>
+#include <unordered_map>
+#include <vector>
+
+#include "ak_common.cuh"
+#include "ak_update.cuh"
+
+using namespace ak;
+
+// ------------------------------------------------------------------ errors
+static thread_local std::string g_last_error;
+
+static akashic_status_t fail(akashic_status_t st, const char *fmt, ...) {
+    char buf[512];
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(buf, sizeof buf, fmt, ap);
+    va_end(ap);
+    g_last_error = buf;
+    return st;
+}
+
+#define CUDA_TRY(call)                                                                         \
+    do {                                                                                       \
+        cudaError_t e_ = (call);                                                               \
+        if (e_ != cudaSuccess)                                                                 \
+            return fail(e_ == cudaErrorMemoryAllocation ? AKASHIC_ENOMEM : AKASHIC_ECUDA,      \
+                        "%s: %s (%s:%d)", #call, cudaGetErrorString(e_), __FILE__, __LINE__);  \
+    } while (0)
+
+#define AK_TRY(call)                                                                           \
+    do {                                                                                       \
+        akashic_status_t s_ = (call);                                                          \
+        if (s_ != AKASHIC_OK) return s_;                                                       \
+    } while (0)
+
+// ------------------------------------------------------------------ device buffers
+struct DevBuf {
+    void *p = nullptr;
+    size_t cap = 0;
+    ~DevBuf() {
+        if (p) cudaFree(p);
+    }
+    // Grow to at least `bytes`; contents are not preserved unless keep.
+    akashic_status_t ensure(size_t bytes, bool keep = false, cudaStream_t st = 0) {
+        if (bytes <= cap) return AKASHIC_OK;
+        size_t want = bytes < 256 ? 256 : bytes;
+        void *q = nullptr;
+        cudaError_t e = cudaMalloc(&q, want);
+        if (e != cudaSuccess) {
+            cudaGetLastError();
+            return fail(AKASHIC_ENOMEM, "device allocation of %zu bytes failed", want);
+        }
+        if (keep && p && cap) {
+            e = cudaMemcpyAsync(q, p, cap, cudaMemcpyDeviceToDevice, st);
+            if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+            if (e != cudaSuccess) {
+                cudaFree(q);
+                return fail(AKASHIC_ECUDA, "buffer growth copy: %s", cudaGetErrorString(e));
+            }
+        }
+        if (p) cudaFree(p);
+        p = q;
+        cap = want;
+        return AKASHIC_OK;
+    }
+    template <typename T> T *as() const { return (T *)p; }
+};
+
+struct StreamScratch {
+    DevBuf qp, shift, u, sa, sb, zpart, partial, cand;
+};
+
+struct ProfRec {
+    int phase;
+    cudaEvent_t a, b;
+    int launches;
+};
+
+struct DeviceGuard {
+    int prev = -1;
+    explicit DeviceGuard(int dev) {
+        if (cudaGetDevice(&prev) != cudaSuccess) prev = -1;
+        if (prev != dev) cudaSetDevice(dev);
+    }
+    ~DeviceGuard() {
+        int cur = -1;
+        if (prev >= 0 && cudaGetDevice(&cur) == cudaSuccess && cur != prev) cudaSetDevice(prev);
+    }
+};
+
+struct akashic_mem {
+    int device = 0;
+    int dim = 0;
+    int64_t cap = 0;
+    int per_page = 1;
+    float tau = 0.f;
+    float rel_scale = 10.f;
+    int64_t n = 0;
+    int64_t next_page = 0;
+    DevBuf emb, page_of, max_norm, status;
+    // canonical out-edge CSR
+    int64_t nnz = 0;
+    DevBuf row_ptr, col, aff, w;
+    // in-edge transpose + split plan for the propagation hop
+    DevBuf in_ptr, in_src, in_w;
+    int64_t n_split = 0, n_segs = 0;
+    DevBuf split_row, split_slot0, seg_e0, seg_e1;
+    std::mutex mu;
+    std::unordered_map<void *, StreamScratch *> scratch;
+    // profiling
+    bool prof = false;
+    std::vector<ProfRec> recs;
+    std::vector<cudaEvent_t> ev_pool;
+    ~akashic_mem() {
+        for (auto &kv : scratch) delete kv.second;
+        for (auto &r : recs) {
+            cudaEventDestroy(r.a);
+            cudaEventDestroy(r.b);
+        }
+        for (auto e : ev_pool) cudaEventDestroy(e);
+    }
+};
+
+// ------------------------------------------------------------------ profiling helpers
+struct PhaseScope {
+    akashic_mem *m;
+    int phase;
+    cudaStream_t st;
+    cudaEvent_t a = nullptr;
+    int launches = 0;
+    PhaseScope(akashic_mem *m_, int ph, cudaStream_t s) : m(m_), phase(ph), st(s) {
+        if (!m->prof) return;
+        a = take_event();
+        if (a) cudaEventRecord(a, st);
+    }
+    cudaEvent_t take_event() {
+        std::lock_guard<std::mutex> g(m->mu);
+        cudaEvent_t e = nullptr;
+        if (!m->ev_pool.empty()) {
+            e = m->ev_pool.back();
+            m->ev_pool.pop_back();
+        } else if (cudaEventCreate(&e) != cudaSuccess) {
+            cudaGetLastError();
+            e = nullptr;
+        }
+        return e;
+    }
+    ~PhaseScope() {
+        if (!m->prof || !a) return;
+        cudaEvent_t b = take_event();
+        if (!b) return;
+        cudaEventRecord(b, st);
+        std::lock_guard<std::mutex> g(m->mu);
+        m->recs.push_back(ProfRec{phase, a, b, launches});
+    }
+};
+
+// ------------------------------------------------------------------ small kernels
+__global__ void k_fill_pages(int32_t *page_of, int64_t n, int64_t first_page, int per_page) {
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n;
+         i += (int64_t)gridDim.x * blockDim.x)
+        page_of[i] = (int32_t)(first_page + i / per_page);
+}
+
+__global__ void k_page_max(const int32_t *page_of, int64_t n, int *out_max, int *status) {
+    int best = -1;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n;
+         i += (int64_t)gridDim.x * blockDim.x) {
+        int p = page_of[i];
+        if (p < 0) set_status(status, AKASHIC_EDEVICE);
+        best = p > best ? p : best;
+    }
+    atomicMax(out_max, best);
+}
+
+// row_ptr of the appended rows in the store's CSR: dst[r] = base + src[r] - src[0]
+__global__ void k_rebase_ptr(const int64_t *src, int64_t *dst, int64_t n1, int64_t base) {
+    const int64_t p0 = src ? src[0] : 0;
+    for (int64_t r = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; r < n1;
+         r += (int64_t)gridDim.x * blockDim.x)
+        dst[r] = src ? base + src[r] - p0 : base;
+}
+
+static int bits_for(int64_t max_value) {
+    int b = 0;
+    while (b < 32 && ((int64_t)1 << b) <= max_value) ++b;
+    return b;
+}
+
+static akashic_status_t check_status(akashic_mem *m, cudaStream_t st, const char *what) {
+    CUDA_TRY(cudaStreamSynchronize(st));
+    int code = 0;
+    CUDA_TRY(cudaMemcpy(&code, m->status.p, sizeof(int), cudaMemcpyDeviceToHost));
+    if (code != 0) {
+        CUDA_TRY(cudaMemset(m->status.p, 0, sizeof(int)));
+        return fail((akashic_status_t)code, "%s: device reported status %d", what, code);
+    }
+    return AKASHIC_OK;
+}
+
+// Rebuild the in-edge transpose (stable by source, hence sorted by source
+// within each destination), its weights, and the split plan of long rows.
+static akashic_status_t rebuild_in_edges(akashic_mem *m, cudaStream_t st) {
+    const int64_t n = m->n, nnz = m->nnz;
+    AK_TRY(m->in_ptr.ensure((size_t)(m->cap + 1) * sizeof(int64_t)));
+    AK_TRY(m->in_src.ensure((size_t)(nnz > 0 ? nnz : 1) * sizeof(int32_t)));
+    AK_TRY(m->in_w.ensure((size_t)(nnz > 0 ? nnz : 1) * sizeof(float)));
+    DevBuf src, keys, vals, keys2, vals2, tmp, deg;
+    const size_t tmp_bytes = (radix_tmp_bytes(nnz) > scan_tmp_bytes(n + 1) ? radix_tmp_bytes(nnz)
+                                                                             : scan_tmp_bytes(n + 1)) +
+                             4096;
+    AK_TRY(tmp.ensure(tmp_bytes));
+    AK_TRY(deg.ensure((size_t)(n + 1) * sizeof(int64_t) * 2));
+    if (nnz > 0) {
+        AK_TRY(src.ensure((size_t)nnz * 4));
+        AK_TRY(keys.ensure((size_t)nnz * 4));
+        AK_TRY(vals.ensure((size_t)nnz * 4));
+        AK_TRY(keys2.ensure((size_t)nnz * 4));
+        AK_TRY(vals2.ensure((size_t)nnz * 4));
+        CUDA_TRY(launch_edge_src_check(m->row_ptr.as<int64_t>(), m->col.as<int32_t>(), n, 0, n,
+                                       src.as<int32_t>(), m->status.as<int>(), st));
+        CUDA_TRY(cudaMemcpyAsync(keys.p, m->col.p, (size_t)nnz * 4, cudaMemcpyDeviceToDevice, st));
+        CUDA_TRY(launch_iota(vals.as<uint32_t>(), nnz, st));
+        bool alt = false;
+        CUDA_TRY(radix_sort_pairs(keys.as<uint32_t>(), vals.as<uint32_t>(), keys2.as<uint32_t>(),
+                                  vals2.as<uint32_t>(), nnz, bits_for(n - 1), tmp.p, tmp.cap, st,
+                                  &alt));
+        const uint32_t *order = alt ? vals2.as<uint32_t>() : vals.as<uint32_t>();
+        CUDA_TRY(launch_gather_in(order, src.as<int32_t>(), m->w.as<float>(), m->in_src.as<int32_t>(),
+                                  m->in_w.as<float>(), nnz, st));
+    }
+    int64_t *degp = deg.as<int64_t>();
+    CUDA_TRY(cudaMemsetAsync(degp, 0, (size_t)(n + 1) * sizeof(int64_t), st));
+    CUDA_TRY(launch_in_degree(m->col.as<int32_t>(), nnz, degp, st));
+    CUDA_TRY(scan_exclusive(degp, m->in_ptr.as<int64_t>(), n, tmp.p, tmp.cap, st));
+    // split plan
+    DevBuf nseg, flag, slot_off, split_idx;
+    AK_TRY(nseg.ensure((size_t)(n + 1) * 8));
+    AK_TRY(flag.ensure((size_t)(n + 1) * 8));
+    AK_TRY(slot_off.ensure((size_t)(n + 1) * 8));
+    AK_TRY(split_idx.ensure((size_t)(n + 1) * 8));
+    CUDA_TRY(launch_split_count(m->in_ptr.as<int64_t>(), n, HOP_SEG, nseg.as<int64_t>(),
+                                flag.as<int64_t>(), st));
+    CUDA_TRY(scan_exclusive(nseg.as<int64_t>(), slot_off.as<int64_t>(), n, tmp.p, tmp.cap, st));
+    CUDA_TRY(scan_exclusive(flag.as<int64_t>(), split_idx.as<int64_t>(), n, tmp.p, tmp.cap, st));
+    int64_t n_segs = 0, n_split = 0;
+    CUDA_TRY(cudaMemcpyAsync(&n_segs, slot_off.as<int64_t>() + n, 8, cudaMemcpyDeviceToHost, st));
+    CUDA_TRY(cudaMemcpyAsync(&n_split, split_idx.as<int64_t>() + n, 8, cudaMemcpyDeviceToHost, st));
+    AK_TRY(check_status(m, st, "relation graph rebuild"));
+    m->n_segs = n_segs;
+    m->n_split = n_split;
+    if (n_split > 0) {
+        AK_TRY(m->split_row.ensure((size_t)n_split * 4));
+        AK_TRY(m->split_slot0.ensure((size_t)(n_split + 1) * 8));
+        AK_TRY(m->seg_e0.ensure((size_t)n_segs * 8));
+        AK_TRY(m->seg_e1.ensure((size_t)n_segs * 8));
+        CUDA_TRY(launch_split_fill(m->in_ptr.as<int64_t>(), n, HOP_SEG, nseg.as<int64_t>(),
+                                   slot_off.as<int64_t>(), split_idx.as<int64_t>(),
+                                   m->split_row.as<int32_t>(), m->split_slot0.as<int64_t>(),
+                                   m->seg_e0.as<int64_t>(), m->seg_e1.as<int64_t>(), st));
+        CUDA_TRY(cudaMemcpyAsync(m->split_slot0.as<int64_t>() + n_split, &n_segs, 8,
+                                 cudaMemcpyHostToDevice, st));
+    }
+    return check_status(m, st, "relation graph rebuild");
+}
+
+// ================================================================== ABI
+extern "C" {
+
+const char *akashic_mem_last_error(void) { return g_last_error.c_str(); }
+
+akashic_status_t akashic_mem_create(const akashic_mem_config_t *cfg, akashic_mem_t **out) {
+    g_last_error.clear();
+    if (!cfg || !out) return fail(AKASHIC_EINVAL, "create: NULL argument");
+    *out = nullptr;
+    if (cfg->dim < 64 || cfg->dim > 4096 || cfg->dim % 64 != 0)
+        return fail(AKASHIC_EINVAL, "create: dim must be a multiple of 64 in [64, 4096]");
+    if (cfg->capacity < 1 || cfg->capacity > 0x7fffffffLL)
+        return fail(AKASHIC_EINVAL, "create: capacity must be in [1, 2^31-1]");
+    if (cfg->chunks_per_page < 1) return fail(AKASHIC_EINVAL, "create: chunks_per_page < 1");
+    if (!(cfg->temperature >= 0.f) || !isfinite(cfg->temperature) ||
+        !(cfg->relation_scale >= 0.f) || !isfinite(cfg->relation_scale))
+        return fail(AKASHIC_EINVAL, "create: temperature/relation_scale must be finite and >= 0");
+    int ndev = 0;
+    if (cudaGetDeviceCount(&ndev) != cudaSuccess || cfg->device < 0 || cfg->device >= ndev) {
+        cudaGetLastError();
+        return fail(AKASHIC_EINVAL, "create: no CUDA device %d", cfg->device);
+    }
+    DeviceGuard g(cfg->device);
+    akashic_mem *m = new (std::nothrow) akashic_mem();
+    if (!m) return fail(AKASHIC_ENOMEM, "create: host allocation failed");
+    m->device = cfg->device;
+    m->dim = cfg->dim;
+    m->cap = cfg->capacity;
+    m->per_page = cfg->chunks_per_page;
+    m->tau = cfg->temperature > 0.f ? cfg->temperature : 1.0f / sqrtf((float)cfg->dim);
+    m->rel_scale = cfg->relation_scale > 0.f ? cfg->relation_scale : 10.f;
+    akashic_status_t s;
+    if ((s = m->emb.ensure((size_t)m->cap * m->dim * 2)) != AKASHIC_OK ||
+        (s = m->page_of.ensure((size_t)m->cap * 4)) != AKASHIC_OK ||
+        (s = m->max_norm.ensure(4)) != AKASHIC_OK || (s = m->status.ensure(4)) != AKASHIC_OK ||
+        (s = m->row_ptr.ensure((size_t)(m->cap + 1) * 8)) != AKASHIC_OK ||
+        (s = m->in_ptr.ensure((size_t)(m->cap + 1) * 8)) != AKASHIC_OK) {
+        delete m;
+        return s;
+    }
+    if (cudaMemset(m->max_norm.p, 0, 4) != cudaSuccess || cudaMemset(m->status.p, 0, 4) != cudaSuccess ||
+        cudaMemset(m->row_ptr.p, 0, 8) != cudaSuccess || cudaMemset(m->in_ptr.p, 0, 8) != cudaSuccess ||
+        cudaDeviceSynchronize() != cudaSuccess) {
+        delete m;
+        return fail(AKASHIC_ECUDA, "create: initialisation failed");
+    }
+    *out = m;
+    return AKASHIC_OK;
+}
+
+void akashic_mem_destroy(akashic_mem_t *m) {
+    if (!m) return;
+    DeviceGuard g(m->device);
+    cudaDeviceSynchronize();
+    delete m;
+}
+
+akashic_status_t akashic_mem_size(const akashic_mem_t *m, int64_t *n_chunks, int64_t *nnz) {
+    if (!m) return fail(AKASHIC_EINVAL, "size: NULL store");
+    if (n_chunks) *n_chunks = m->n;
+    if (nnz) *nnz = m->nnz;
+    return AKASHIC_OK;
+}
+
+akashic_status_t akashic_mem_sync(akashic_mem_t *m, void *stream) {
+    if (!m) return fail(AKASHIC_EINVAL, "sync: NULL store");
+    DeviceGuard g(m->device);
+    return check_status(m, (cudaStream_t)stream, "sync");
+}
+
+akashic_status_t akashic_mem_append_chunks(akashic_mem_t *m, const uint16_t *emb, int64_t n,
+                                           const int32_t *page_of, const int64_t *row_ptr,
+                                           const int32_t *col, const float *aff,
+                                           int64_t *first_id_out, void *stream) {
+    g_last_error.clear();
+    if (!m) return fail(AKASHIC_EINVAL, "append: NULL store");
+    if (n < 0 || (n > 0 && !emb)) return fail(AKASHIC_EINVAL, "append: bad n or emb");
+    const bool has_edges = row_ptr || col || aff;
+    if (has_edges && !(row_ptr && col && aff))
+        return fail(AKASHIC_EINVAL, "append: row_ptr, col and aff must be given together");
+    if (m->n + n > m->cap)
+        return fail(AKASHIC_ECAPACITY, "append: %lld + %lld chunks exceed capacity %lld",
+                    (long long)m->n, (long long)n, (long long)m->cap);
+    if (first_id_out) *first_id_out = m->n;
+    if (n == 0) return AKASHIC_OK;
+    DeviceGuard g(m->device);
+    cudaStream_t st = (cudaStream_t)stream;
+    const int64_t first = m->n;
+    PhaseScope ph(m, AKASHIC_PHASE_GRAPH, st);
+    // -- validate the new edges before anything is committed
+    int64_t e_lo = 0, e_hi = 0;
+    if (has_edges) {
+        CUDA_TRY(cudaMemcpyAsync(&e_lo, row_ptr, 8, cudaMemcpyDeviceToHost, st));
+        CUDA_TRY(cudaMemcpyAsync(&e_hi, row_ptr + n, 8, cudaMemcpyDeviceToHost, st));
+        CUDA_TRY(launch_edge_src_check(row_ptr, col, n, first, first + n, nullptr,
+                                       m->status.as<int>(), st));
+        AK_TRY(check_status(m, st, "append: edge check"));
+        if (e_hi < e_lo) return fail(AKASHIC_EINVAL, "append: row_ptr decreases");
+        if (m->nnz + (e_hi - e_lo) > 0x7fffffffLL)
+            return fail(AKASHIC_ECAPACITY, "append: more than 2^31-1 relation edges");
+    }
+    int64_t max_page = -1;
+    if (page_of) {
+        DevBuf pm;
+        AK_TRY(pm.ensure(4));
+        int init = -1;
+        CUDA_TRY(cudaMemcpyAsync(pm.p, &init, 4, cudaMemcpyHostToDevice, st));
+        k_page_max<<<device_sm_count(), 256, 0, st>>>(page_of, n, pm.as<int>(), m->status.as<int>());
+        CUDA_TRY(cudaGetLastError());
+        int mx = -1;
+        CUDA_TRY(cudaMemcpyAsync(&mx, pm.p, 4, cudaMemcpyDeviceToHost, st));
+        AK_TRY(check_status(m, st, "append: page_of must be >= 0"));
+        max_page = mx;
+    }
+    const int64_t new_nnz = e_hi - e_lo;
+    if (new_nnz > 0) {
+        const size_t need = (size_t)(m->nnz + new_nnz);
+        size_t grow = need + need / 4;
+        AK_TRY(m->col.ensure(grow * 4, true, st));
+        AK_TRY(m->aff.ensure(grow * 4, true, st));
+        AK_TRY(m->w.ensure(grow * 4, true, st));
+    }
+    // -- commit
+    CUDA_TRY(cudaMemcpyAsync(m->emb.as<uint16_t>() + first * m->dim, emb, (size_t)n * m->dim * 2,
+                             cudaMemcpyDeviceToDevice, st));
+    int32_t *pg = m->page_of.as<int32_t>() + first;
+    if (page_of) {
+        CUDA_TRY(cudaMemcpyAsync(pg, page_of, (size_t)n * 4, cudaMemcpyDeviceToDevice, st));
+        if (max_page + 1 > m->next_page) m->next_page = max_page + 1;
+    } else {
+        k_fill_pages<<<device_sm_count() * 4, 256, 0, st>>>(pg, n, m->next_page, m->per_page);
+        CUDA_TRY(cudaGetLastError());
+        m->next_page += ceil_div<int64_t>(n, m->per_page);
+    }
+    CUDA_TRY(launch_row_norm_max(m->emb.as<uint16_t>() + first * m->dim, n, m->dim,
+                                 m->max_norm.as<float>(), st));
+    int64_t *rp = m->row_ptr.as<int64_t>() + first;   // rp[0] is already m->nnz
+    k_rebase_ptr<<<device_sm_count() * 4, 256, 0, st>>>(has_edges ? row_ptr : nullptr, rp, n + 1,
+                                                         m->nnz);
+    CUDA_TRY(cudaGetLastError());
+    if (new_nnz > 0) {
+        CUDA_TRY(cudaMemcpyAsync(m->col.as<int32_t>() + m->nnz, col + e_lo, (size_t)new_nnz * 4,
+                                 cudaMemcpyDeviceToDevice, st));
+        CUDA_TRY(cudaMemcpyAsync(m->aff.as<float>() + m->nnz, aff + e_lo, (size_t)new_nnz * 4,
+                                 cudaMemcpyDeviceToDevice, st));
+        CUDA_TRY(launch_row_softmax(rp, m->aff.as<float>(), m->w.as<float>(), n, st));
+    }
+    m->n += n;
+    m->nnz += new_nnz;
+    AK_TRY(rebuild_in_edges(m, st));
+    return AKASHIC_OK;
+}
+
+akashic_status_t akashic_mem_update_relations(akashic_mem_t *m, int64_t first, int64_t n,
+                                              int32_t M, int32_t reciprocal, void *stream) {
+    g_last_error.clear();
+    if (!m) return fail(AKASHIC_EINVAL, "update: NULL store");
+    if (first < 0 || n < 0 || first + n > m->n)
+        return fail(AKASHIC_EINVAL, "update: range [%lld, %lld) outside the store of %lld",
+                    (long long)first, (long long)(first + n), (long long)m->n);
+    if (M < 1 || M > 64 || M > first)
+        return fail(AKASHIC_EINVAL, "update: M must be in [1, min(64, first)]");
+    if (n == 0) return AKASHIC_OK;
+    DeviceGuard g(m->device);
+    cudaStream_t st = (cudaStream_t)stream;
+    // rows [first, first+n) must have no out-edges
+    int64_t a = 0, b = 0;
+    CUDA_TRY(cudaMemcpyAsync(&a, m->row_ptr.as<int64_t>() + first, 8, cudaMemcpyDeviceToHost, st));
+    CUDA_TRY(cudaMemcpyAsync(&b, m->row_ptr.as<int64_t>() + first + n, 8, cudaMemcpyDeviceToHost, st));
+    CUDA_TRY(cudaStreamSynchronize(st));
+    if (a != b) return fail(AKASHIC_EINVAL, "update: rows [first, first+n) already have out-edges");
+    UpdateArgs ua;
+    ua.emb = m->emb.as<uint16_t>();
+    ua.dim = m->dim;
+    ua.n_rows = m->n;
+    ua.first = first;
+    ua.n_new = n;
+    ua.M = M;
+    ua.reciprocal = reciprocal != 0;
+    ua.scale = m->rel_scale;
+    ua.status = m->status.as<int>();
+    int64_t nnz_new = m->nnz + n * M * (reciprocal ? 2 : 1);
+    if (nnz_new > 0x7fffffffLL)
+        return fail(AKASHIC_ECAPACITY, "update: more than 2^31-1 relation edges");
+    DevBuf ncol, naff, nrp, nbr_ids, nbr_cos;
+    AK_TRY(nbr_ids.ensure((size_t)n * M * 4));
+    AK_TRY(nbr_cos.ensure((size_t)n * M * 4));
+    ua.nbr_ids = nbr_ids.as<int32_t>();
+    ua.nbr_cos = nbr_cos.as<float>();
+    AK_TRY(ncol.ensure((size_t)(nnz_new + nnz_new / 4) * 4));
+    AK_TRY(naff.ensure((size_t)(nnz_new + nnz_new / 4) * 4));
+    AK_TRY(nrp.ensure((size_t)(m->cap + 1) * 8));
+    {
+        PhaseScope ph(m, AKASHIC_PHASE_RELATE, st);
+        akashic_status_t r = relate_top_m(ua, st, &ph.launches);
+        if (r != AKASHIC_OK) return fail(r, "update: relation GEMM / top-M failed");
+        AK_TRY(check_status(m, st, "update: top-M"));
+    }
+    {
+        PhaseScope ph(m, AKASHIC_PHASE_GRAPH, st);
+        akashic_status_t r = csr_insert(ua, m->row_ptr.as<int64_t>(), m->col.as<int32_t>(),
+                                        m->aff.as<float>(), m->nnz, nrp.as<int64_t>(),
+                                        ncol.as<int32_t>(), naff.as<float>(), st, &ph.launches);
+        if (r != AKASHIC_OK) return fail(r, "update: CSR insert failed");
+        AK_TRY(check_status(m, st, "update"));
+        std::swap(m->row_ptr.p, nrp.p);
+        std::swap(m->row_ptr.cap, nrp.cap);
+        std::swap(m->col.p, ncol.p);
+        std::swap(m->col.cap, ncol.cap);
+        std::swap(m->aff.p, naff.p);
+        std::swap(m->aff.cap, naff.cap);
+        m->nnz = nnz_new;
+        AK_TRY(m->w.ensure(m->col.cap, false));
+        CUDA_TRY(launch_row_softmax(m->row_ptr.as<int64_t>(), m->aff.as<float>(), m->w.as<float>(),
+                                    m->n, st));
+        AK_TRY(rebuild_in_edges(m, st));
+    }
+    return AKASHIC_OK;
+}
+
+static StreamScratch *scratch_for(akashic_mem *m, void *stream) {
+    std::lock_guard<std::mutex> g(m->mu);
+    auto it = m->scratch.find(stream);
+    if (it != m->scratch.end()) return it->second;
+    StreamScratch *s = new (std::nothrow) StreamScratch();
+    if (s) m->scratch[stream] = s;
+    return s;
+}
+
+akashic_status_t akashic_mem_retrieve(akashic_mem_t *m, const uint16_t *q, int32_t B, int32_t k,
+                                      float alpha, int32_t hops, int64_t *ids, float *scores,
+                                      int32_t *page_ids, int32_t *n_pages, void *stream) {
+    g_last_error.clear();
+    if (!m) return fail(AKASHIC_EINVAL, "retrieve: NULL store");
+    if (!q || !ids || !scores) return fail(AKASHIC_EINVAL, "retrieve: NULL q/ids/scores");
+    if (B < 1) return fail(AKASHIC_EINVAL, "retrieve: B < 1");
+    if (k < 1 || k > 64) return fail(AKASHIC_EINVAL, "retrieve: k must be in [1, 64]");
+    if (k > m->n) return fail(AKASHIC_EINVAL, "retrieve: k=%d exceeds the %lld chunks", k, (long long)m->n);
+    if (hops < 0 || hops > 16) return fail(AKASHIC_EINVAL, "retrieve: hops must be in [0, 16]");
+    if (!(alpha >= 0.f) || !isfinite(alpha)) return fail(AKASHIC_EINVAL, "retrieve: alpha must be finite and >= 0");
+    DeviceGuard g(m->device);
+    cudaStream_t st = (cudaStream_t)stream;
+    StreamScratch *sc = scratch_for(m, stream);
+    if (!sc) return fail(AKASHIC_ENOMEM, "retrieve: host allocation failed");
+    const int64_t n = m->n;
+    const int eff_hops = (alpha > 0.f && m->nnz > 0) ? hops : 0;
+    const int sms = device_sm_count();
+    for (int32_t off = 0; off < B; off += 256) {
+        const int b = B - off < 256 ? B - off : 256;
+        int bp = 16;
+        while (bp < b) bp <<= 1;
+        const int64_t tiles = score_tiles(n);
+        const SelectPlan sp = select_plan(n, bp, k, sms);
+        AK_TRY(sc->qp.ensure((size_t)bp * m->dim * 2));
+        AK_TRY(sc->shift.ensure((size_t)bp * 4));
+        AK_TRY(sc->u.ensure((size_t)n * bp * 4));
+        AK_TRY(sc->zpart.ensure((size_t)tiles * bp * 4));
+        AK_TRY(sc->cand.ensure((size_t)sp.lists * bp * k * 8));
+        if (eff_hops >= 1) AK_TRY(sc->sa.ensure((size_t)n * bp * 4));
+        if (eff_hops >= 2) AK_TRY(sc->sb.ensure((size_t)n * bp * 4));
+        if (eff_hops >= 1 && m->n_segs > 0) AK_TRY(sc->partial.ensure((size_t)m->n_segs * bp * 4));
+        const uint16_t *qb = q + (int64_t)off * m->dim;
+        {
+            PhaseScope ph(m, AKASHIC_PHASE_SCORE, st);
+            CUDA_TRY(launch_prep_queries(qb, b, bp, m->dim, m->tau, m->max_norm.as<float>(),
+                                         sc->qp.as<uint16_t>(), sc->shift.as<float>(),
+                                         m->status.as<int>(), st));
+            CUDA_TRY(launch_score(m->emb.as<uint16_t>(), n, m->dim, sc->qp.as<uint16_t>(), bp,
+                                  sc->shift.as<float>(), m->tau, sc->u.as<float>(),
+                                  sc->zpart.as<float>(), m->status.as<int>(), st, &ph.launches));
+            ph.launches += 1;
+        }
+        const float *fin = sc->u.as<float>();
+        if (eff_hops >= 1) {
+            PhaseScope ph(m, AKASHIC_PHASE_PROPAGATE, st);
+            HopPlan hp;
+            hp.in_ptr = m->in_ptr.as<int64_t>();
+            hp.in_src = m->in_src.as<int32_t>();
+            hp.in_w = m->in_w.as<float>();
+            hp.n = n;
+            hp.n_split_rows = m->n_split;
+            hp.split_row = m->split_row.as<int32_t>();
+            hp.split_slot0 = m->split_slot0.as<int64_t>();
+            hp.n_segs = m->n_segs;
+            hp.seg_e0 = m->seg_e0.as<int64_t>();
+            hp.seg_e1 = m->seg_e1.as<int64_t>();
+            float *bufs[2] = {sc->sa.as<float>(), sc->sb.as<float>()};
+            for (int h = 0; h < eff_hops; ++h) {
+                float *out = bufs[h & 1];
+                CUDA_TRY(launch_hop(hp, sc->u.as<float>(), fin, out, bp, alpha,
+                                    sc->partial.as<float>(), st, &ph.launches));
+                fin = out;
+            }
+        }
+        {
+            PhaseScope ph(m, AKASHIC_PHASE_SELECT, st);
+            CUDA_TRY(launch_select(sp, fin, n, bp, b, k, sc->cand.as<unsigned long long>(),
+                                   sc->zpart.as<float>(), tiles, m->page_of.as<int32_t>(),
+                                   ids + (int64_t)off * k, scores + (int64_t)off * k,
+                                   page_ids ? page_ids + (int64_t)off * k : nullptr,
+                                   n_pages ? n_pages + off : nullptr, m->status.as<int>(), st,
+                                   &ph.launches));
+        }
+    }
+    return AKASHIC_OK;
+}
+
+akashic_status_t akashic_mem_export_csr(akashic_mem_t *m, int64_t *n_rows, int64_t *nnz,
+                                        int64_t *row_ptr, int32_t *col, float *aff, float *w,
+                                        void *stream) {
+    g_last_error.clear();
+    if (!m) return fail(AKASHIC_EINVAL, "export: NULL store");
+    if (n_rows) *n_rows = m->n;
+    if (nnz) *nnz = m->nnz;
+    if (!row_ptr && !col && !aff && !w) return AKASHIC_OK;
+    DeviceGuard g(m->device);
+    cudaStream_t st = (cudaStream_t)stream;
+    if (row_ptr)
+        CUDA_TRY(cudaMemcpyAsync(row_ptr, m->row_ptr.p, (size_t)(m->n + 1) * 8,
+                                 cudaMemcpyDeviceToDevice, st));
+    if (m->nnz > 0) {
+        if (col) CUDA_TRY(cudaMemcpyAsync(col, m->col.p, (size_t)m->nnz * 4, cudaMemcpyDeviceToDevice, st));
+        if (aff) CUDA_TRY(cudaMemcpyAsync(aff, m->aff.p, (size_t)m->nnz * 4, cudaMemcpyDeviceToDevice, st));
+        if (w) CUDA_TRY(cudaMemcpyAsync(w, m->w.p, (size_t)m->nnz * 4, cudaMemcpyDeviceToDevice, st));
+    }
+    CUDA_TRY(cudaStreamSynchronize(st));
+    return AKASHIC_OK;
+}
+
+akashic_status_t akashic_mem_set_profiling(akashic_mem_t *m, int32_t on) {
+    if (!m) return fail(AKASHIC_EINVAL, "set_profiling: NULL store");
+    m->prof = on != 0;
+    return AKASHIC_OK;
+}
+
+akashic_status_t akashic_mem_phase_times(akashic_mem_t *m, float *ms, int32_t *launches) {
+    if (!m) return fail(AKASHIC_EINVAL, "phase_times: NULL store");
+    DeviceGuard g(m->device);
+    std::vector<ProfRec> recs;
+    {
+        std::lock_guard<std::mutex> lk(m->mu);
+        recs.swap(m->recs);
+    }
+    for (int p = 0; p < AKASHIC_PHASE_COUNT; ++p) {
+        if (ms) ms[p] = 0.f;
+        if (launches) launches[p] = 0;
+    }
+    akashic_status_t rc = AKASHIC_OK;
+    for (auto &r : recs) {
+        float t = 0.f;
+        cudaError_t e = cudaEventSynchronize(r.b);
+        if (e == cudaSuccess) e = cudaEventElapsedTime(&t, r.a, r.b);
+        if (e != cudaSuccess) {
+            cudaGetLastError();
+            rc = fail(AKASHIC_ECUDA, "phase_times: %s", cudaGetErrorString(e));
+        }
+        if (r.phase >= 0 && r.phase < AKASHIC_PHASE_COUNT) {
+            if (ms) ms[r.phase] += t;
+            if (launches) launches[r.phase] += r.launches;
+        }
+    }
+    std::lock_guard<std::mutex> lk(m->mu);
+    for (auto &r : recs) {
+        m->ev_pool.push_back(r.a);
+        m->ev_pool.push_back(r.b);
+    }
+    return rc;
+}
+
+}  // extern "C"

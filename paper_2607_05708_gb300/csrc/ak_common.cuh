@@ -1,0 +1,150 @@
+// Internal declarations shared by the library's translation units.
+// Nothing here is part of the public ABI (include/akashic_mem.h is).
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "../../include/akashic_mem.h"
+
+namespace ak {
+
+// ------------------------------------------------------------------ status word
+// Device-side faults are recorded with atomicCAS(status, 0, code) so that the
+// first one wins; the host reads and clears the word in akashic_mem_sync.
+__device__ __forceinline__ void set_status(int *status, int code) {
+    if (status) atomicCAS(status, 0, code);
+}
+
+// ------------------------------------------------------------------ small helpers
+__device__ __forceinline__ float bf16_to_f32(uint16_t h) {
+    return __uint_as_float(((uint32_t)h) << 16);
+}
+
+template <typename T>
+__host__ __device__ __forceinline__ T ceil_div(T a, T b) { return (a + b - 1) / b; }
+
+// Selection key: larger key = better.  High word: the score's fp32 bit
+// pattern (scores are >= 0, where the bit pattern is monotone in value);
+// low word: ~id, so that on equal scores the lower chunk ID wins.
+__device__ __forceinline__ unsigned long long make_key(float score, uint32_t id) {
+    return ((unsigned long long)__float_as_uint(score) << 32) | (unsigned long long)(~id);
+}
+__device__ __forceinline__ float key_score(unsigned long long key) {
+    return __uint_as_float((uint32_t)(key >> 32));
+}
+__device__ __forceinline__ uint32_t key_id(unsigned long long key) {
+    return ~(uint32_t)(key & 0xffffffffull);
+}
+
+// Keys for signed cosine values: order-preserving map of any finite fp32 to
+// uint32 (flip all bits of negatives, set the sign bit of non-negatives).
+__device__ __forceinline__ uint32_t ordered_bits(float v) {
+    uint32_t u = __float_as_uint(v);
+    return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+}
+__device__ __forceinline__ float unordered_bits(uint32_t o) {
+    uint32_t u = (o & 0x80000000u) ? (o & 0x7fffffffu) : ~o;
+    return __uint_as_float(u);
+}
+
+// ------------------------------------------------------------------ launchers
+// All launchers enqueue on `st` and report launch errors by return value.
+
+// Score (a1): u[j, c] = exp(tau * <e_j, q_c> - shift[c]) for j < n, c < bp,
+// written chunk-major with row stride bp; zpart[t, c] = sum of u over the
+// rows of score tile t.  Returns the number of score tiles (rows of zpart).
+int64_t score_tiles(int64_t n);
+cudaError_t launch_score(const uint16_t *emb, int64_t n, int dim, const uint16_t *qp, int bp,
+                         const float *shift, float tau, float *u, float *zpart, int *status,
+                         cudaStream_t st, int *launches);
+
+// Plain dot products out[j, c] = <e_j, q_c> (fp32 accumulate), row stride bp.
+cudaError_t launch_dots(const uint16_t *emb, int64_t n, int dim, const uint16_t *qp, int bp,
+                        float *out, cudaStream_t st, int *launches);
+
+// Query preparation: pad q (b rows) to bp rows of zeros and compute
+// shift[c] = tau * |q_c| * max_norm (0 for padding); flags ERANGE.
+cudaError_t launch_prep_queries(const uint16_t *q, int b, int bp, int dim, float tau,
+                                const float *max_norm, uint16_t *qp, float *shift, int *status,
+                                cudaStream_t st);
+
+// Running maximum of row norms of emb[0..n) into *max_norm (monotone).
+cudaError_t launch_row_norm_max(const uint16_t *emb, int64_t n, int dim, float *max_norm,
+                                cudaStream_t st);
+
+// ------------------------------------------------------------------ graph
+int device_sm_count();
+
+// In-edge rows longer than this are split into segments of this many edges
+// whose partial sums are combined by a fixup pass.
+constexpr int64_t HOP_SEG = 2048;
+
+// Exclusive prefix sum of `in` (n values) into out (n+1 values; out[n] = total).
+cudaError_t scan_exclusive(const int64_t *in, int64_t *out, int64_t n, void *tmp,
+                           size_t tmp_bytes, cudaStream_t st);
+size_t scan_tmp_bytes(int64_t n);
+
+// Stable LSD radix sort of (key, value) pairs on the low `bits` key bits;
+// the result lands in (keys, vals) or, if *result_in_alt, in the alt buffers.
+size_t radix_tmp_bytes(int64_t n);
+cudaError_t radix_sort_pairs(uint32_t *keys, uint32_t *vals, uint32_t *keys_alt,
+                             uint32_t *vals_alt, int64_t n, int bits, void *tmp,
+                             size_t tmp_bytes, cudaStream_t st, bool *result_in_alt);
+
+// CSR helpers (see ak_graph.cu).
+cudaError_t launch_edge_src_check(const int64_t *row_ptr, const int32_t *col, int64_t n_rows,
+                                  int64_t row_base, int64_t n_total, int32_t *src, int *status,
+                                  cudaStream_t st);
+cudaError_t launch_row_softmax(const int64_t *row_ptr, const float *aff, float *w, int64_t n_rows,
+                               cudaStream_t st);
+cudaError_t launch_in_degree(const int32_t *col, int64_t nnz, int64_t *deg, cudaStream_t st);
+cudaError_t launch_iota(uint32_t *v, int64_t n, cudaStream_t st);
+cudaError_t launch_gather_in(const uint32_t *order, const int32_t *src, const float *w,
+                             int32_t *in_src, float *in_w, int64_t nnz, cudaStream_t st);
+cudaError_t launch_split_count(const int64_t *in_ptr, int64_t n, int64_t seg_len, int64_t *nseg,
+                               int64_t *flag, cudaStream_t st);
+cudaError_t launch_split_fill(const int64_t *in_ptr, int64_t n, int64_t seg_len,
+                              const int64_t *nseg, const int64_t *slot_off,
+                              const int64_t *split_idx, int32_t *split_row, int64_t *split_slot0,
+                              int64_t *seg_e0, int64_t *seg_e1, cudaStream_t st);
+
+// Propagation hop (a2): out[j,:] = u[j,:] + alpha * sum_{i->j} w_ij * in[i,:].
+struct HopPlan {
+    const int64_t *in_ptr;      // n+1
+    const int32_t *in_src;      // nnz
+    const float *in_w;          // nnz
+    int64_t n;
+    // rows whose in-degree exceeds the segment length are split
+    int64_t n_split_rows;       // number of such rows
+    const int32_t *split_row;   // [n_split_rows] row index
+    const int64_t *split_slot0; // [n_split_rows+1] first partial slot of each split row
+    int64_t n_segs;             // total segments of split rows (= partial slots)
+    const int64_t *seg_e0;      // [n_segs] first edge of segment
+    const int64_t *seg_e1;      // [n_segs] end edge
+};
+cudaError_t launch_hop(const HopPlan &p, const float *u, const float *in, float *out, int bp,
+                       float alpha, float *partial, cudaStream_t st, int *launches);
+
+// ------------------------------------------------------------------ selection
+// Per-CTA top-k candidate lists over the final slab (a3), then the merge
+// with normalisation by Z (a1), page resolve and distinct count (a4).
+struct SelectPlan {
+    int grid;        // CTAs of the candidate kernel
+    int lanes;       // row lanes per CTA (threads = lanes * bp)
+    int64_t lists;   // grid * lanes lists per column
+};
+SelectPlan select_plan(int64_t n, int bp, int k, int sm_count);
+cudaError_t launch_select(const SelectPlan &sp, const float *s, int64_t n, int bp, int b, int k,
+                          unsigned long long *cand, const float *zpart, int64_t n_ztiles,
+                          const int32_t *page_of, int64_t *ids, float *scores,
+                          int32_t *page_ids, int32_t *n_pages, int *status, cudaStream_t st,
+                          int *launches);
+// Same selection over signed values (cosines): the k best rows of each of
+// the b columns go to nbr_ids / nbr_cos rows c_base .. c_base+b-1.
+cudaError_t launch_select_signed(const SelectPlan &sp, const float *s, int64_t n, int bp, int b,
+                                 int k, unsigned long long *cand, int64_t c_base,
+                                 int32_t *nbr_ids, float *nbr_cos, int *status, cudaStream_t st,
+                                 int *launches);
+
+}  // namespace ak

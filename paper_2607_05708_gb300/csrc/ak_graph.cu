@@ -1,0 +1,607 @@
+// Relation graph on the device: prefix sums, a stable LSD radix sort, the
+// in-edge transpose, relation weights, and the propagation hop (a2) that
+// spreads scores along cross-chunk relations (arXiv 2607.05708, §4.1:
+// related chunks are recovered together).
+#include "ak_common.cuh"
+
+namespace ak {
+
+static int sm_count_cached() {
+    static int cached[64] = {0};
+    int dev = 0;
+    cudaGetDevice(&dev);
+    if (dev < 0 || dev >= 64) dev = 0;
+    if (!cached[dev]) {
+        int v = 0;
+        cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, dev);
+        cached[dev] = v > 0 ? v : 1;
+    }
+    return cached[dev];
+}
+int device_sm_count() { return sm_count_cached(); }
+
+// ================================================================== scan
+constexpr int SCAN_THREADS = 256, SCAN_ITEMS = 8, SCAN_TILE = SCAN_THREADS * SCAN_ITEMS;
+
+__device__ __forceinline__ int64_t warp_incl_scan(int64_t v) {
+    const int lane = threadIdx.x & 31;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        int64_t t = __shfl_up_sync(0xffffffffu, v, o);
+        if (lane >= o) v += t;
+    }
+    return v;
+}
+
+// Each CTA scans one tile of SCAN_TILE values (exclusive) and emits the
+// tile total.
+__global__ __launch_bounds__(SCAN_THREADS) void k_scan_tile(const int64_t *__restrict__ in,
+                                                            int64_t *__restrict__ out, int64_t n,
+                                                            int64_t *__restrict__ tile_sum) {
+    __shared__ int64_t wsum[SCAN_THREADS / 32];
+    const int64_t base = (int64_t)blockIdx.x * SCAN_TILE + (int64_t)threadIdx.x * SCAN_ITEMS;
+    int64_t v[SCAN_ITEMS];
+    int64_t run = 0;
+#pragma unroll
+    for (int i = 0; i < SCAN_ITEMS; ++i) {
+        int64_t idx = base + i;
+        v[i] = idx < n ? in[idx] : 0;
+        run += v[i];
+    }
+    int64_t incl = warp_incl_scan(run);
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    if (lane == 31) wsum[warp] = incl;
+    __syncthreads();
+    if (warp == 0) {
+        int64_t s = lane < SCAN_THREADS / 32 ? wsum[lane] : 0;
+        s = warp_incl_scan(s);
+        if (lane < SCAN_THREADS / 32) wsum[lane] = s;
+    }
+    __syncthreads();
+    int64_t excl = incl - run + (warp > 0 ? wsum[warp - 1] : 0);
+#pragma unroll
+    for (int i = 0; i < SCAN_ITEMS; ++i) {
+        int64_t idx = base + i;
+        if (idx < n) out[idx] = excl;
+        excl += v[i];
+    }
+    if (threadIdx.x == SCAN_THREADS - 1) tile_sum[blockIdx.x] = excl;
+}
+
+__global__ void k_scan_add(int64_t *__restrict__ out, int64_t n,
+                           const int64_t *__restrict__ tile_off) {
+    int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    if (idx < n) out[idx] += tile_off[idx / SCAN_TILE];
+}
+
+__global__ void k_scan_total(const int64_t *__restrict__ in, int64_t *__restrict__ out,
+                             int64_t n) {
+    // out[n] = out[n-1] + in[n-1]  (n >= 1), else 0
+    out[n] = n > 0 ? out[n - 1] + in[n - 1] : 0;
+}
+
+size_t scan_tmp_bytes(int64_t n) {
+    size_t tot = 0;
+    int64_t m = n;
+    do {
+        int64_t tiles = ceil_div<int64_t>(m, SCAN_TILE);
+        tot += (size_t)(2 * tiles + 2) * sizeof(int64_t);
+        m = tiles;
+    } while (m > 1);
+    return tot + 64;
+}
+
+static cudaError_t scan_rec(const int64_t *in, int64_t *out, int64_t n, int64_t *tmp,
+                            cudaStream_t st) {
+    if (n <= 0) return cudaSuccess;
+    int64_t tiles = ceil_div<int64_t>(n, SCAN_TILE);
+    int64_t *sums = tmp, *offs = tmp + tiles;
+    k_scan_tile<<<(unsigned)tiles, SCAN_THREADS, 0, st>>>(in, out, n, sums);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess || tiles == 1) return e;
+    e = scan_rec(sums, offs, tiles, tmp + 2 * tiles + 2, st);
+    if (e != cudaSuccess) return e;
+    k_scan_add<<<(unsigned)ceil_div<int64_t>(n, 256), 256, 0, st>>>(out, n, offs);
+    return cudaGetLastError();
+}
+
+cudaError_t scan_exclusive(const int64_t *in, int64_t *out, int64_t n, void *tmp,
+                           size_t tmp_bytes, cudaStream_t st) {
+    if (tmp_bytes < scan_tmp_bytes(n)) return cudaErrorInvalidValue;
+    cudaError_t e = scan_rec(in, out, n, (int64_t *)tmp, st);
+    if (e != cudaSuccess) return e;
+    k_scan_total<<<1, 1, 0, st>>>(in, out, n);
+    return cudaGetLastError();
+}
+
+// ================================================================== radix sort
+// Stable LSD radix sort of (uint32 key, uint32 value) pairs, 8 bits a pass.
+// Per pass: tile histograms (digit-major), one exclusive scan, then a stable
+// scatter in which each warp ranks its keys round by round with
+// __match_any_sync and the warps of a tile are combined in order.
+constexpr int RS_THREADS = 256, RS_ITEMS = 16, RS_TILE = RS_THREADS * RS_ITEMS;
+constexpr int RS_WARPS = RS_THREADS / 32, RS_PER_WARP = RS_TILE / RS_WARPS;
+
+__global__ __launch_bounds__(RS_THREADS) void k_rs_hist(const uint32_t *__restrict__ keys,
+                                                        int64_t n, int shift, uint32_t mask,
+                                                        int64_t n_tiles,
+                                                        int64_t *__restrict__ hist) {
+    __shared__ int h[256];
+    h[threadIdx.x] = 0;
+    __syncthreads();
+    const int64_t base = (int64_t)blockIdx.x * RS_TILE;
+    for (int i = threadIdx.x; i < RS_TILE; i += RS_THREADS) {
+        int64_t idx = base + i;
+        if (idx < n) atomicAdd(&h[(keys[idx] >> shift) & mask], 1);
+    }
+    __syncthreads();
+    hist[(int64_t)threadIdx.x * n_tiles + blockIdx.x] = h[threadIdx.x];
+}
+
+__global__ __launch_bounds__(RS_THREADS) void k_rs_scatter(
+    const uint32_t *__restrict__ keys, const uint32_t *__restrict__ vals, int64_t n, int shift,
+    uint32_t mask, int64_t n_tiles, const int64_t *__restrict__ offs, uint32_t *__restrict__ okeys,
+    uint32_t *__restrict__ ovals) {
+    __shared__ int cnt[RS_WARPS][256];
+    __shared__ int pre[RS_WARPS][256];
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    for (int d = lane; d < 256; d += 32) cnt[warp][d] = 0;
+    __syncwarp();
+    const int64_t base = (int64_t)blockIdx.x * RS_TILE + (int64_t)warp * RS_PER_WARP;
+    const unsigned lt = (1u << lane) - 1u;
+    uint32_t k[RS_ITEMS], v[RS_ITEMS];
+    int loc[RS_ITEMS];
+#pragma unroll
+    for (int r = 0; r < RS_ITEMS; ++r) {
+        int64_t idx = base + r * 32 + lane;
+        bool ok = idx < n;
+        k[r] = ok ? keys[idx] : 0u;
+        v[r] = ok ? vals[idx] : 0u;
+        uint32_t d = ok ? ((k[r] >> shift) & mask) : 0x100u;   // 0x100: no digit
+        unsigned peers = __match_any_sync(0xffffffffu, d);
+        int leader = __ffs(peers) - 1;
+        int c = ok ? cnt[warp][d] : 0;
+        loc[r] = c + __popc(peers & lt);
+        __syncwarp();
+        if (ok && lane == leader) cnt[warp][d] = c + __popc(peers);
+        __syncwarp();
+    }
+    __syncthreads();
+    {
+        int d = threadIdx.x;   // RS_THREADS == 256 digits
+        int run = 0;
+#pragma unroll
+        for (int w = 0; w < RS_WARPS; ++w) {
+            pre[w][d] = run;
+            run += cnt[w][d];
+        }
+    }
+    __syncthreads();
+#pragma unroll
+    for (int r = 0; r < RS_ITEMS; ++r) {
+        int64_t idx = base + r * 32 + lane;
+        if (idx < n) {
+            uint32_t d = (k[r] >> shift) & mask;
+            int64_t pos = offs[(int64_t)d * n_tiles + blockIdx.x] + pre[warp][d] + loc[r];
+            okeys[pos] = k[r];
+            ovals[pos] = v[r];
+        }
+    }
+}
+
+size_t radix_tmp_bytes(int64_t n) {
+    int64_t n_tiles = ceil_div<int64_t>(n, RS_TILE);
+    int64_t m = 256 * n_tiles;
+    return (size_t)(2 * m + 1) * sizeof(int64_t) + scan_tmp_bytes(m) + 256;
+}
+
+cudaError_t radix_sort_pairs(uint32_t *keys, uint32_t *vals, uint32_t *keys_alt,
+                             uint32_t *vals_alt, int64_t n, int bits, void *tmp,
+                             size_t tmp_bytes, cudaStream_t st, bool *result_in_alt) {
+    *result_in_alt = false;
+    if (n <= 1 || bits <= 0) return cudaSuccess;
+    if (tmp_bytes < radix_tmp_bytes(n)) return cudaErrorInvalidValue;
+    const int64_t n_tiles = ceil_div<int64_t>(n, RS_TILE);
+    const int64_t m = 256 * n_tiles;
+    int64_t *hist = (int64_t *)tmp;
+    int64_t *offs = hist + m;
+    void *stmp = (void *)(offs + m + 1);
+    size_t stmp_bytes = tmp_bytes - (size_t)(2 * m + 1) * sizeof(int64_t);
+    uint32_t *ki = keys, *vi = vals, *ko = keys_alt, *vo = vals_alt;
+    for (int sh = 0; sh < bits; sh += 8) {
+        int nb = bits - sh < 8 ? bits - sh : 8;
+        uint32_t mask = (1u << nb) - 1u;
+        k_rs_hist<<<(unsigned)n_tiles, RS_THREADS, 0, st>>>(ki, n, sh, mask, n_tiles, hist);
+        cudaError_t e = cudaGetLastError();
+        if (e != cudaSuccess) return e;
+        e = scan_exclusive(hist, offs, m, stmp, stmp_bytes, st);
+        if (e != cudaSuccess) return e;
+        k_rs_scatter<<<(unsigned)n_tiles, RS_THREADS, 0, st>>>(ki, vi, n, sh, mask, n_tiles, offs,
+                                                                ko, vo);
+        e = cudaGetLastError();
+        if (e != cudaSuccess) return e;
+        uint32_t *t;
+        t = ki; ki = ko; ko = t;
+        t = vi; vi = vo; vo = t;
+        *result_in_alt = !*result_in_alt;
+    }
+    return cudaSuccess;
+}
+
+// ================================================================== CSR helpers
+// One warp per row: src[e] = global row id for every edge of the row, and the
+// row is checked: targets in [0, n_total), never the row itself, strictly
+// ascending.  row_ptr is relative (offsets into col), rows are local; the
+// global id of local row r is row_base + r; edge e is written at out_off + e.
+__global__ void k_edge_src_check(const int64_t *__restrict__ row_ptr, const int32_t *__restrict__ col,
+                                 int64_t n_rows, int64_t row_base, int64_t n_total,
+                                 int32_t *__restrict__ src, int *status) {
+    const int lane = threadIdx.x & 31;
+    int64_t r = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    const int64_t stride = ((int64_t)gridDim.x * blockDim.x) >> 5;
+    const int64_t p0 = row_ptr[0];
+    for (; r < n_rows; r += stride) {
+        int64_t a = row_ptr[r], b = row_ptr[r + 1];
+        if (b < a) {
+            if (lane == 0) set_status(status, AKASHIC_EDEVICE);
+            continue;
+        }
+        const int64_t gid = row_base + r;
+        for (int64_t e = a + lane; e < b; e += 32) {
+            int32_t c = col[e];
+            bool bad = c < 0 || (int64_t)c >= n_total || (int64_t)c == gid ||
+                       (e > a && col[e - 1] >= c);
+            if (bad) set_status(status, AKASHIC_EDEVICE);
+            if (src) src[e - p0] = (int32_t)gid;
+        }
+    }
+}
+
+cudaError_t launch_edge_src_check(const int64_t *row_ptr, const int32_t *col, int64_t n_rows,
+                                  int64_t row_base, int64_t n_total, int32_t *src, int *status,
+                                  cudaStream_t st) {
+    if (n_rows <= 0) return cudaSuccess;
+    int64_t warps = n_rows < (int64_t)device_sm_count() * 64 ? n_rows : (int64_t)device_sm_count() * 64;
+    k_edge_src_check<<<(unsigned)ceil_div<int64_t>(warps * 32, 256), 256, 0, st>>>(
+        row_ptr, col, n_rows, row_base, n_total, src, status);
+    return cudaGetLastError();
+}
+
+// Relation weights: w = softmax of each row's edge logits (one warp per row).
+__global__ void k_row_softmax(const int64_t *__restrict__ row_ptr, const float *__restrict__ aff,
+                              float *__restrict__ w, int64_t n_rows) {
+    const int lane = threadIdx.x & 31;
+    int64_t r = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    const int64_t stride = ((int64_t)gridDim.x * blockDim.x) >> 5;
+    for (; r < n_rows; r += stride) {
+        int64_t a = row_ptr[r], b = row_ptr[r + 1];
+        if (b <= a) continue;
+        float m = -INFINITY;
+        for (int64_t e = a + lane; e < b; e += 32) m = fmaxf(m, aff[e]);
+        for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
+        float s = 0.f;
+        for (int64_t e = a + lane; e < b; e += 32) s += expf(aff[e] - m);
+        for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+        const float inv = 1.f / s;
+        for (int64_t e = a + lane; e < b; e += 32) w[e] = expf(aff[e] - m) * inv;
+    }
+}
+
+cudaError_t launch_row_softmax(const int64_t *row_ptr, const float *aff, float *w, int64_t n_rows,
+                               cudaStream_t st) {
+    if (n_rows <= 0) return cudaSuccess;
+    int64_t warps = n_rows < (int64_t)device_sm_count() * 64 ? n_rows : (int64_t)device_sm_count() * 64;
+    k_row_softmax<<<(unsigned)ceil_div<int64_t>(warps * 32, 256), 256, 0, st>>>(row_ptr, aff, w,
+                                                                              n_rows);
+    return cudaGetLastError();
+}
+
+__global__ void k_in_degree(const int32_t *__restrict__ col, int64_t nnz,
+                            unsigned long long *__restrict__ deg) {
+    for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < nnz;
+         e += (int64_t)gridDim.x * blockDim.x)
+        atomicAdd(&deg[col[e]], 1ull);
+}
+
+cudaError_t launch_in_degree(const int32_t *col, int64_t nnz, int64_t *deg, cudaStream_t st) {
+    if (nnz <= 0) return cudaSuccess;
+    int grid = (int)(nnz / 256 + 1 < (int64_t)device_sm_count() * 16 ? nnz / 256 + 1
+                                                                     : device_sm_count() * 16);
+    k_in_degree<<<grid, 256, 0, st>>>(col, nnz, (unsigned long long *)deg);
+    return cudaGetLastError();
+}
+
+__global__ void k_iota_u32(uint32_t *__restrict__ v, int64_t n) {
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n;
+         i += (int64_t)gridDim.x * blockDim.x)
+        v[i] = (uint32_t)i;
+}
+
+cudaError_t launch_iota(uint32_t *v, int64_t n, cudaStream_t st) {
+    if (n <= 0) return cudaSuccess;
+    k_iota_u32<<<device_sm_count() * 8, 256, 0, st>>>(v, n);
+    return cudaGetLastError();
+}
+
+__global__ void k_gather_in(const uint32_t *__restrict__ order, const int32_t *__restrict__ src,
+                            const float *__restrict__ w, int32_t *__restrict__ in_src,
+                            float *__restrict__ in_w, int64_t nnz) {
+    for (int64_t p = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; p < nnz;
+         p += (int64_t)gridDim.x * blockDim.x) {
+        uint32_t e = order[p];
+        in_src[p] = src[e];
+        in_w[p] = w[e];
+    }
+}
+
+cudaError_t launch_gather_in(const uint32_t *order, const int32_t *src, const float *w,
+                             int32_t *in_src, float *in_w, int64_t nnz, cudaStream_t st) {
+    if (nnz <= 0) return cudaSuccess;
+    k_gather_in<<<device_sm_count() * 8, 256, 0, st>>>(order, src, w, in_src, in_w, nnz);
+    return cudaGetLastError();
+}
+
+// Rows whose in-degree exceeds seg_len are split into segments of seg_len
+// edges; nseg[j] = that count (0 for rows kept whole), flag[j] = nseg > 0.
+__global__ void k_split_count(const int64_t *__restrict__ in_ptr, int64_t n, int64_t seg_len,
+                              int64_t *__restrict__ nseg, int64_t *__restrict__ flag) {
+    for (int64_t j = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; j < n;
+         j += (int64_t)gridDim.x * blockDim.x) {
+        int64_t d = in_ptr[j + 1] - in_ptr[j];
+        int64_t s = d > seg_len ? ceil_div<int64_t>(d, seg_len) : 0;
+        nseg[j] = s;
+        flag[j] = s > 0;
+    }
+}
+
+__global__ void k_split_fill(const int64_t *__restrict__ in_ptr, int64_t n, int64_t seg_len,
+                             const int64_t *__restrict__ nseg, const int64_t *__restrict__ slot_off,
+                             const int64_t *__restrict__ split_idx, int32_t *__restrict__ split_row,
+                             int64_t *__restrict__ split_slot0, int64_t *__restrict__ seg_e0,
+                             int64_t *__restrict__ seg_e1) {
+    for (int64_t j = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; j < n;
+         j += (int64_t)gridDim.x * blockDim.x) {
+        int64_t s = nseg[j];
+        if (s == 0) continue;
+        int64_t idx = split_idx[j];
+        split_row[idx] = (int32_t)j;
+        split_slot0[idx] = slot_off[j];
+        const int64_t a = in_ptr[j], b = in_ptr[j + 1];
+        for (int64_t t = 0; t < s; ++t) {
+            int64_t e0 = a + t * seg_len;
+            seg_e0[slot_off[j] + t] = e0;
+            seg_e1[slot_off[j] + t] = e0 + seg_len < b ? e0 + seg_len : b;
+        }
+    }
+}
+
+cudaError_t launch_split_count(const int64_t *in_ptr, int64_t n, int64_t seg_len, int64_t *nseg,
+                               int64_t *flag, cudaStream_t st) {
+    if (n <= 0) return cudaSuccess;
+    k_split_count<<<device_sm_count() * 4, 256, 0, st>>>(in_ptr, n, seg_len, nseg, flag);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_split_fill(const int64_t *in_ptr, int64_t n, int64_t seg_len,
+                              const int64_t *nseg, const int64_t *slot_off,
+                              const int64_t *split_idx, int32_t *split_row, int64_t *split_slot0,
+                              int64_t *seg_e0, int64_t *seg_e1, cudaStream_t st) {
+    if (n <= 0) return cudaSuccess;
+    k_split_fill<<<device_sm_count() * 4, 256, 0, st>>>(in_ptr, n, seg_len, nseg, slot_off,
+                                                        split_idx, split_row, split_slot0, seg_e0,
+                                                        seg_e1);
+    return cudaGetLastError();
+}
+
+// ================================================================== propagation hop
+// out[j,:] = u[j,:] + alpha * sum_{i->j} w_ij in[i,:], gathered over the
+// in-edge CSR, one warp per destination row.  A row holds BP fp32 values
+// (BP/4 float4).  For BP >= 128 each lane owns BP/128 float4 of the row; for
+// smaller BP the warp splits into 32/(BP/4) lane groups that take
+// alternate edges and are summed at the end.  Rows with more than
+// HOP_SEG in-edges are skipped here and handled by segments + fixup.
+template <int BP>
+struct HopShape {
+    static constexpr int F = BP / 4;                       // float4 per row
+    static constexpr int G = F >= 32 ? 1 : 32 / F;         // edge groups per warp
+    static constexpr int V = F >= 32 ? F / 32 : 1;         // float4 per lane
+    static constexpr int LW = F >= 32 ? 32 : F;            // lanes per group
+};
+
+template <int BP>
+__device__ __forceinline__ void hop_accumulate(const int32_t *__restrict__ in_src,
+                                               const float *__restrict__ in_w, int64_t e0,
+                                               int64_t e1, const float4 *__restrict__ in4,
+                                               float4 (&acc)[HopShape<BP>::V]) {
+    using S = HopShape<BP>;
+    const int lane = threadIdx.x & 31;
+    const int g = lane / S::LW, sub = lane % S::LW;
+#pragma unroll
+    for (int v = 0; v < S::V; ++v) acc[v] = make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int64_t eb = e0; eb < e1; eb += 32) {
+        const int cnt = (int)(e1 - eb < 32 ? e1 - eb : 32);
+        int32_t s_l = 0;
+        float w_l = 0.f;
+        if (lane < cnt) {
+            s_l = in_src[eb + lane];
+            w_l = in_w[eb + lane];
+        }
+        int t = 0;
+        for (; t + 4 * S::G <= cnt; t += 4 * S::G) {
+            int32_t s[4];
+            float w[4];
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                s[q] = __shfl_sync(0xffffffffu, s_l, t + q * S::G + g);
+                w[q] = __shfl_sync(0xffffffffu, w_l, t + q * S::G + g);
+            }
+            float4 x[4][S::V];
+#pragma unroll
+            for (int q = 0; q < 4; ++q)
+#pragma unroll
+                for (int v = 0; v < S::V; ++v) x[q][v] = in4[(int64_t)s[q] * S::F + sub + 32 * v];
+#pragma unroll
+            for (int q = 0; q < 4; ++q)
+#pragma unroll
+                for (int v = 0; v < S::V; ++v) {
+                    acc[v].x = fmaf(w[q], x[q][v].x, acc[v].x);
+                    acc[v].y = fmaf(w[q], x[q][v].y, acc[v].y);
+                    acc[v].z = fmaf(w[q], x[q][v].z, acc[v].z);
+                    acc[v].w = fmaf(w[q], x[q][v].w, acc[v].w);
+                }
+        }
+        for (; t < cnt; t += S::G) {
+            const int idx = t + g;
+            int32_t s = __shfl_sync(0xffffffffu, s_l, idx < 32 ? idx : 31);
+            float w = __shfl_sync(0xffffffffu, w_l, idx < 32 ? idx : 31);
+            if (idx < cnt) {
+#pragma unroll
+                for (int v = 0; v < S::V; ++v) {
+                    float4 x = in4[(int64_t)s * S::F + sub + 32 * v];
+                    acc[v].x = fmaf(w, x.x, acc[v].x);
+                    acc[v].y = fmaf(w, x.y, acc[v].y);
+                    acc[v].z = fmaf(w, x.z, acc[v].z);
+                    acc[v].w = fmaf(w, x.w, acc[v].w);
+                }
+            }
+        }
+    }
+    if (S::G > 1) {
+#pragma unroll
+        for (int o = S::LW; o < 32; o <<= 1) {
+#pragma unroll
+            for (int v = 0; v < S::V; ++v) {
+                acc[v].x += __shfl_xor_sync(0xffffffffu, acc[v].x, o);
+                acc[v].y += __shfl_xor_sync(0xffffffffu, acc[v].y, o);
+                acc[v].z += __shfl_xor_sync(0xffffffffu, acc[v].z, o);
+                acc[v].w += __shfl_xor_sync(0xffffffffu, acc[v].w, o);
+            }
+        }
+    }
+}
+
+template <int BP>
+__global__ __launch_bounds__(256) void k_hop_rows(const int64_t *__restrict__ in_ptr,
+                                                  const int32_t *__restrict__ in_src,
+                                                  const float *__restrict__ in_w, int64_t n,
+                                                  const float4 *__restrict__ u4,
+                                                  const float4 *__restrict__ in4,
+                                                  float4 *__restrict__ out4, float alpha) {
+    using S = HopShape<BP>;
+    const int lane = threadIdx.x & 31;
+    const int sub = lane % S::LW;
+    int64_t j = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    const int64_t stride = ((int64_t)gridDim.x * blockDim.x) >> 5;
+    for (; j < n; j += stride) {
+        const int64_t e0 = in_ptr[j], e1 = in_ptr[j + 1];
+        if (e1 - e0 > HOP_SEG) continue;
+        float4 acc[S::V];
+        hop_accumulate<BP>(in_src, in_w, e0, e1, in4, acc);
+        if (lane < S::LW) {
+#pragma unroll
+            for (int v = 0; v < S::V; ++v) {
+                const int64_t o = j * S::F + sub + 32 * v;
+                float4 b = u4[o];
+                b.x = fmaf(alpha, acc[v].x, b.x);
+                b.y = fmaf(alpha, acc[v].y, b.y);
+                b.z = fmaf(alpha, acc[v].z, b.z);
+                b.w = fmaf(alpha, acc[v].w, b.w);
+                out4[o] = b;
+            }
+        }
+    }
+}
+
+template <int BP>
+__global__ __launch_bounds__(256) void k_hop_segs(const int64_t *__restrict__ seg_e0,
+                                                  const int64_t *__restrict__ seg_e1,
+                                                  int64_t n_segs,
+                                                  const int32_t *__restrict__ in_src,
+                                                  const float *__restrict__ in_w,
+                                                  const float4 *__restrict__ in4,
+                                                  float4 *__restrict__ part4) {
+    using S = HopShape<BP>;
+    const int lane = threadIdx.x & 31;
+    const int sub = lane % S::LW;
+    int64_t s = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    const int64_t stride = ((int64_t)gridDim.x * blockDim.x) >> 5;
+    for (; s < n_segs; s += stride) {
+        float4 acc[S::V];
+        hop_accumulate<BP>(in_src, in_w, seg_e0[s], seg_e1[s], in4, acc);
+        if (lane < S::LW) {
+#pragma unroll
+            for (int v = 0; v < S::V; ++v) part4[s * S::F + sub + 32 * v] = acc[v];
+        }
+    }
+}
+
+template <int BP>
+__global__ __launch_bounds__(256) void k_hop_fixup(const int32_t *__restrict__ split_row,
+                                                   const int64_t *__restrict__ split_slot0,
+                                                   int64_t n_split,
+                                                   const float4 *__restrict__ part4,
+                                                   const float4 *__restrict__ u4,
+                                                   float4 *__restrict__ out4, float alpha) {
+    constexpr int F = BP / 4;
+    int64_t r = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    const int64_t stride = ((int64_t)gridDim.x * blockDim.x) >> 5;
+    const int lane = threadIdx.x & 31;
+    for (; r < n_split; r += stride) {
+        const int64_t j = split_row[r];
+        const int64_t a = split_slot0[r], b = split_slot0[r + 1];
+        for (int f = lane; f < F; f += 32) {
+            float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+            for (int64_t s = a; s < b; ++s) {
+                float4 x = part4[s * F + f];
+                acc.x += x.x; acc.y += x.y; acc.z += x.z; acc.w += x.w;
+            }
+            float4 o = u4[j * F + f];
+            o.x = fmaf(alpha, acc.x, o.x);
+            o.y = fmaf(alpha, acc.y, o.y);
+            o.z = fmaf(alpha, acc.z, o.z);
+            o.w = fmaf(alpha, acc.w, o.w);
+            out4[j * F + f] = o;
+        }
+    }
+}
+
+template <int BP>
+static cudaError_t hop_bp(const HopPlan &p, const float *u, const float *in, float *out,
+                          float alpha, float *partial, cudaStream_t st, int *launches) {
+    const int sms = device_sm_count();
+    const int64_t warps_rows = p.n;
+    int grid = (int)(ceil_div<int64_t>(warps_rows, 8) < (int64_t)sms * 8 ? ceil_div<int64_t>(warps_rows, 8)
+                                                                         : (int64_t)sms * 8);
+    if (grid < 1) grid = 1;
+    k_hop_rows<BP><<<grid, 256, 0, st>>>(p.in_ptr, p.in_src, p.in_w, p.n, (const float4 *)u,
+                                         (const float4 *)in, (float4 *)out, alpha);
+    cudaError_t e = cudaGetLastError();
+    if (launches) *launches += 1;
+    if (e != cudaSuccess || p.n_split_rows == 0) return e;
+    int g2 = (int)(ceil_div<int64_t>(p.n_segs, 8) < (int64_t)sms * 8 ? ceil_div<int64_t>(p.n_segs, 8)
+                                                                    : (int64_t)sms * 8);
+    k_hop_segs<BP><<<g2, 256, 0, st>>>(p.seg_e0, p.seg_e1, p.n_segs, p.in_src, p.in_w,
+                                       (const float4 *)in, (float4 *)partial);
+    e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    int g3 = (int)ceil_div<int64_t>(p.n_split_rows, 8);
+    k_hop_fixup<BP><<<g3, 256, 0, st>>>(p.split_row, p.split_slot0, p.n_split_rows,
+                                        (const float4 *)partial, (const float4 *)u, (float4 *)out,
+                                        alpha);
+    if (launches) *launches += 2;
+    return cudaGetLastError();
+}
+
+cudaError_t launch_hop(const HopPlan &p, const float *u, const float *in, float *out, int bp,
+                       float alpha, float *partial, cudaStream_t st, int *launches) {
+    switch (bp) {
+    case 16: return hop_bp<16>(p, u, in, out, alpha, partial, st, launches);
+    case 32: return hop_bp<32>(p, u, in, out, alpha, partial, st, launches);
+    case 64: return hop_bp<64>(p, u, in, out, alpha, partial, st, launches);
+    case 128: return hop_bp<128>(p, u, in, out, alpha, partial, st, launches);
+    case 256: return hop_bp<256>(p, u, in, out, alpha, partial, st, launches);
+    default: return cudaErrorInvalidValue;
+    }
+}
+
+}  // namespace ak

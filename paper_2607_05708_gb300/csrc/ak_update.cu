@@ -1,0 +1,235 @@
+// Relation update (a6, a7): for new chunks, the top-M related prior chunks
+// by cosine of the stored embeddings, then the reciprocal insertion of those
+// edges into the relation graph's CSR (arXiv 2607.05708, §4.1: cross-chunk
+// inference selects the related prior chunks of each new chunk; Algorithm 1,
+// line 7, in its Dense-only form of §5.5).
+#include "ak_update.cuh"
+
+namespace ak {
+
+// Copy rows [first+off, first+off+b) of emb into a zero-padded bp-row block.
+__global__ void k_pad_rows(const uint16_t *__restrict__ src, int b, int bp, int dim,
+                           uint16_t *__restrict__ dst) {
+    const int64_t total = (int64_t)bp * dim;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < total;
+         i += (int64_t)gridDim.x * blockDim.x) {
+        const int64_t r = i / dim;
+        dst[i] = r < b ? src[i] : (uint16_t)0;
+    }
+}
+
+akashic_status_t relate_top_m(const UpdateArgs &a, cudaStream_t st, int *launches) {
+    const int64_t n_old = a.first;
+    int bp_max = 16;
+    while (bp_max < 256 && bp_max < a.n_new) bp_max <<= 1;
+    uint16_t *qp = nullptr;
+    float *dots = nullptr;
+    unsigned long long *cand = nullptr;
+    const SelectPlan sp_max = select_plan(n_old, bp_max, a.M, device_sm_count());
+    cudaError_t e = cudaMalloc(&qp, (size_t)bp_max * a.dim * 2);
+    if (e == cudaSuccess) e = cudaMalloc(&dots, (size_t)n_old * bp_max * 4);
+    if (e == cudaSuccess) {
+        // lists for the smallest bp are the most numerous; size for the worst case
+        int64_t lists = 0;
+        for (int bp = 16; bp <= bp_max; bp <<= 1) {
+            SelectPlan sp = select_plan(n_old, bp, a.M, device_sm_count());
+            int64_t need = sp.lists * bp;
+            lists = need > lists ? need : lists;
+        }
+        (void)sp_max;
+        e = cudaMalloc(&cand, (size_t)lists * a.M * 8);
+    }
+    akashic_status_t rc = AKASHIC_OK;
+    if (e != cudaSuccess) {
+        cudaGetLastError();
+        rc = AKASHIC_ENOMEM;
+    }
+    for (int64_t off = 0; rc == AKASHIC_OK && off < a.n_new; off += 256) {
+        const int b = (int)(a.n_new - off < 256 ? a.n_new - off : 256);
+        int bp = 16;
+        while (bp < b) bp <<= 1;
+        k_pad_rows<<<device_sm_count(), 256, 0, st>>>(a.emb + (a.first + off) * a.dim, b, bp, a.dim,
+                                                       qp);
+        e = cudaGetLastError();
+        if (e == cudaSuccess) e = launch_dots(a.emb, n_old, a.dim, qp, bp, dots, st, launches);
+        const SelectPlan sp = select_plan(n_old, bp, a.M, device_sm_count());
+        if (e == cudaSuccess)
+            e = launch_select_signed(sp, dots, n_old, bp, b, a.M, cand, off, a.nbr_ids, a.nbr_cos,
+                                     a.status, st, launches);
+        if (e != cudaSuccess) rc = AKASHIC_ECUDA;
+        if (launches) *launches += 1;
+    }
+    if (rc == AKASHIC_OK && cudaStreamSynchronize(st) != cudaSuccess) rc = AKASHIC_ECUDA;
+    cudaFree(qp);
+    cudaFree(dots);
+    cudaFree(cand);
+    return rc;
+}
+
+// ------------------------------------------------------------------ CSR insert
+// An existing edge into a new chunk would make a reciprocal edge a repeat.
+__global__ void k_check_no_edge_into(const int32_t *__restrict__ col, int64_t nnz, int64_t lo,
+                                     int64_t hi, int *status) {
+    for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < nnz;
+         e += (int64_t)gridDim.x * blockDim.x) {
+        const int64_t c = col[e];
+        if (c >= lo && c < hi) set_status(status, AKASHIC_EDEVICE);
+    }
+}
+
+// new degree of every row: old degree, + M for new rows, + reciprocal count
+__global__ void k_new_degree(const int64_t *__restrict__ rp, int64_t n_rows, int64_t first,
+                             int64_t n_new, int M, const int64_t *__restrict__ recip,
+                             int64_t *__restrict__ deg) {
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n_rows;
+         i += (int64_t)gridDim.x * blockDim.x) {
+        int64_t d = rp[i + 1] - rp[i];
+        if (i >= first && i < first + n_new) d += M;
+        if (recip) d += recip[i];
+        deg[i] = d;
+    }
+}
+
+__global__ void k_count_recip(const int32_t *__restrict__ nbr, int64_t pairs,
+                              unsigned long long *__restrict__ recip) {
+    for (int64_t p = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; p < pairs;
+         p += (int64_t)gridDim.x * blockDim.x)
+        atomicAdd(&recip[nbr[p]], 1ull);
+}
+
+// Old edges keep their order at the front of each row (one warp per row).
+__global__ void k_copy_old_rows(const int64_t *__restrict__ rp, const int32_t *__restrict__ col,
+                                const float *__restrict__ aff, int64_t n_rows,
+                                const int64_t *__restrict__ nrp, int32_t *__restrict__ ncol,
+                                float *__restrict__ naff) {
+    const int lane = threadIdx.x & 31;
+    int64_t r = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    const int64_t stride = ((int64_t)gridDim.x * blockDim.x) >> 5;
+    for (; r < n_rows; r += stride) {
+        const int64_t a = rp[r], b = rp[r + 1], o = nrp[r];
+        for (int64_t e = a + lane; e < b; e += 32) {
+            ncol[o + e - a] = col[e];
+            naff[o + e - a] = aff[e];
+        }
+    }
+}
+
+// Rows of the new chunks: their M neighbours in ascending ID order (one warp
+// per new row; rank of each neighbour among the row's M by ID).
+__global__ void k_fill_new_rows(const int32_t *__restrict__ nbr, const float *__restrict__ cosv,
+                                int64_t first, int64_t n_new, int M, float scale,
+                                const int64_t *__restrict__ nrp, int32_t *__restrict__ ncol,
+                                float *__restrict__ naff) {
+    const int lane = threadIdx.x & 31;
+    int64_t a = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    const int64_t stride = ((int64_t)gridDim.x * blockDim.x) >> 5;
+    for (; a < n_new; a += stride) {
+        const int32_t *row = nbr + a * M;
+        const int64_t o = nrp[first + a];
+        for (int t = lane; t < M; t += 32) {
+            const int32_t id = row[t];
+            int rank = 0;
+            for (int u = 0; u < M; ++u) rank += row[u] < id;
+            ncol[o + rank] = id;
+            naff[o + rank] = scale * cosv[a * M + t];
+        }
+    }
+}
+
+// Reciprocal edges j -> new chunk, appended after row j's old edges in
+// ascending new-chunk order.  `order` lists the (new, slot) pair indices
+// stably sorted by target j, so pairs of one j come in ascending new ID.
+__global__ void k_fill_recip(const uint32_t *__restrict__ order, const uint32_t *__restrict__ tgt,
+                             int64_t pairs, const int32_t *__restrict__ nbr,
+                             const float *__restrict__ cosv, int64_t first, int M, float scale,
+                             const int64_t *__restrict__ rp, const int64_t *__restrict__ recip_off,
+                             const int64_t *__restrict__ nrp, int32_t *__restrict__ ncol,
+                             float *__restrict__ naff) {
+    for (int64_t p = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; p < pairs;
+         p += (int64_t)gridDim.x * blockDim.x) {
+        const uint32_t pair = order[p];
+        const int64_t j = tgt[p];
+        const int64_t rank = p - recip_off[j];
+        const int64_t pos = nrp[j] + (rp[j + 1] - rp[j]) + rank;
+        ncol[pos] = (int32_t)(first + pair / M);
+        naff[pos] = scale * cosv[pair];
+        (void)nbr;
+    }
+}
+
+akashic_status_t csr_insert(const UpdateArgs &a, const int64_t *rp, const int32_t *col,
+                            const float *aff, int64_t nnz, int64_t *new_rp, int32_t *new_col,
+                            float *new_aff, cudaStream_t st, int *launches) {
+    const int64_t n_rows = a.n_rows, pairs = a.n_new * a.M;
+    const int sms = device_sm_count();
+    int64_t *deg = nullptr, *recip = nullptr, *recip_off = nullptr;
+    uint32_t *keys = nullptr, *vals = nullptr, *keys2 = nullptr, *vals2 = nullptr;
+    void *tmp = nullptr;
+    const size_t tmp_bytes = (radix_tmp_bytes(pairs) > scan_tmp_bytes(n_rows + 1)
+                                  ? radix_tmp_bytes(pairs)
+                                  : scan_tmp_bytes(n_rows + 1)) + 4096;
+    cudaError_t e = cudaMalloc(&deg, (size_t)(n_rows + 1) * 8);
+    if (e == cudaSuccess) e = cudaMalloc(&recip, (size_t)(n_rows + 1) * 8);
+    if (e == cudaSuccess) e = cudaMalloc(&recip_off, (size_t)(n_rows + 1) * 8);
+    if (e == cudaSuccess) e = cudaMalloc(&keys, (size_t)pairs * 4 + 16);
+    if (e == cudaSuccess) e = cudaMalloc(&vals, (size_t)pairs * 4 + 16);
+    if (e == cudaSuccess) e = cudaMalloc(&keys2, (size_t)pairs * 4 + 16);
+    if (e == cudaSuccess) e = cudaMalloc(&vals2, (size_t)pairs * 4 + 16);
+    if (e == cudaSuccess) e = cudaMalloc(&tmp, tmp_bytes);
+    akashic_status_t rc = AKASHIC_OK;
+    if (e != cudaSuccess) {
+        cudaGetLastError();
+        rc = AKASHIC_ENOMEM;
+    }
+    int L = 0;
+    if (rc == AKASHIC_OK) {
+        k_check_no_edge_into<<<sms * 4, 256, 0, st>>>(col, nnz, a.first, a.first + a.n_new, a.status);
+        cudaMemsetAsync(recip, 0, (size_t)(n_rows + 1) * 8, st);
+        if (a.reciprocal)
+            k_count_recip<<<sms * 4, 256, 0, st>>>(a.nbr_ids, pairs, (unsigned long long *)recip);
+        k_new_degree<<<sms * 4, 256, 0, st>>>(rp, n_rows, a.first, a.n_new, a.M,
+                                              a.reciprocal ? recip : nullptr, deg);
+        L += 4;
+        e = cudaGetLastError();
+        if (e == cudaSuccess) e = scan_exclusive(deg, new_rp, n_rows, tmp, tmp_bytes, st);
+        if (e == cudaSuccess) {
+            k_copy_old_rows<<<sms * 8, 256, 0, st>>>(rp, col, aff, n_rows, new_rp, new_col, new_aff);
+            k_fill_new_rows<<<sms * 2, 256, 0, st>>>(a.nbr_ids, a.nbr_cos, a.first, a.n_new, a.M,
+                                                     a.scale, new_rp, new_col, new_aff);
+            L += 2;
+            e = cudaGetLastError();
+        }
+        if (e == cudaSuccess && a.reciprocal && pairs > 0) {
+            e = scan_exclusive(recip, recip_off, n_rows, tmp, tmp_bytes, st);
+            if (e == cudaSuccess) e = cudaMemcpyAsync(keys, a.nbr_ids, (size_t)pairs * 4,
+                                                      cudaMemcpyDeviceToDevice, st);
+            if (e == cudaSuccess) e = launch_iota(vals, pairs, st);
+            bool alt = false;
+            int bits = 0;
+            while (bits < 32 && ((int64_t)1 << bits) <= a.first - 1) ++bits;
+            if (e == cudaSuccess)
+                e = radix_sort_pairs(keys, vals, keys2, vals2, pairs, bits, tmp, tmp_bytes, st, &alt);
+            if (e == cudaSuccess) {
+                k_fill_recip<<<sms * 2, 256, 0, st>>>(alt ? vals2 : vals, alt ? keys2 : keys, pairs,
+                                                      a.nbr_ids, a.nbr_cos, a.first, a.M, a.scale, rp,
+                                                      recip_off, new_rp, new_col, new_aff);
+                L += 1;
+                e = cudaGetLastError();
+            }
+        }
+        if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+        if (e != cudaSuccess) rc = AKASHIC_ECUDA;
+    }
+    if (launches) *launches += L;
+    cudaFree(deg);
+    cudaFree(recip);
+    cudaFree(recip_off);
+    cudaFree(keys);
+    cudaFree(vals);
+    cudaFree(keys2);
+    cudaFree(vals2);
+    cudaFree(tmp);
+    return rc;
+}
+
+}  // namespace ak

@@ -1,0 +1,178 @@
+"""Parity helpers: run a synthetic workload through the CUDA library and the
+oracle on the same inputs and compare element by element.
+
+Tolerances (written here, used by every parity test):
+  * Selected IDs, page IDs and page counts are compared exactly, except that
+    an ID may be swapped for another whose ORACLE score lies within the
+    near-tie band |s - s_k| <= SWAP_REL * max(s, s_k) of the oracle's k-th
+    score (every softmax score is about 1/N, so the band is relative; a
+    relative 1e-4 is a logit difference of 1e-4), and the order inside the
+    list may differ only among such near-ties.
+  * Page IDs must equal the page table applied to the GPU's own IDs and the
+    page count must equal the number of distinct ones: bit-exact.
+  * Each GPU score is within SCORE_REL (2e-3) of the oracle's fp64 score of
+    the same chunk.
+  * Relation update: neighbour lists exact except swaps whose oracle cosines
+    differ by < COS_ABS (1e-4) at the M-th/(M+1)-th boundary; the CSR
+    (row pointers, columns) exactly equal after those swaps; logits within
+    1e-5 absolute of scale * fp64 cosine; weights within 2e-3 relative.
+"""
+from __future__ import annotations
+
+import numpy as np
+
+import oracle
+
+SWAP_REL = 1e-4
+SCORE_REL = 2e-3
+COS_ABS = 1e-4
+
+
+# --------------------------------------------------------------------------- retrieval
+def gpu_store(wl, placement, capacity=None):
+    from paper_2607_05708_gb300 import MemStore
+    return MemStore.from_arrays(wl.emb, wl.page_of[placement], wl.row_ptr, wl.col, wl.aff,
+                                capacity=capacity or wl.n, chunks_per_page=wl.chunks_per_page,
+                                temperature=wl.tau)
+
+
+def gpu_retrieve(wl, placement, store=None, queries=None, k=None, alpha=None, hops=None):
+    import torch
+    if store is None:
+        store = gpu_store(wl, placement)
+    q = wl.queries if queries is None else queries
+    qt = torch.from_numpy(np.ascontiguousarray(q).view(np.int16)).cuda()
+    ids, sc, pg, npg = store.retrieve(qt, k or wl.k, wl.alpha if alpha is None else alpha,
+                                      wl.hops if hops is None else hops)
+    store.sync()
+    return store, dict(ids=ids.cpu().numpy(), scores=sc.cpu().numpy(), page_ids=pg.cpu().numpy(),
+                       n_pages=npg.cpu().numpy())
+
+
+_W_CACHE = {}
+
+
+def oracle_weights(wl):
+    key = id(wl)
+    if key not in _W_CACHE:
+        _W_CACHE.clear()
+        _W_CACHE[key] = oracle.row_softmax(wl.row_ptr, wl.aff)
+    return _W_CACHE[key]
+
+
+def oracle_retrieve(wl, placement, queries=None, k=None, alpha=None, hops=None):
+    q = wl.queries if queries is None else queries
+    return oracle.retrieve(wl.emb, q, wl.row_ptr, wl.col, oracle_weights(wl), tau=wl.tau,
+                           alpha=wl.alpha if alpha is None else alpha,
+                           hops=wl.hops if hops is None else hops, k=k or wl.k,
+                           page_of=wl.page_of[placement], want_final=True)
+
+
+def assert_retrieval_parity(wl, placement, got, ref, rows=None):
+    """got: GPU outputs (row r of got = query rows[r] of ref if rows is given)."""
+    page_of = wl.page_of[placement]
+    k = ref["ids"].shape[1]
+    n_rows = got["ids"].shape[0] if rows is None else len(rows)
+    for r in range(n_rows):
+        b = r if rows is None else rows[r]
+        gi = got["ids"][r].astype(np.int64)
+        oi = ref["ids"][b]
+        fin = ref["final"][b]
+        assert len(set(gi.tolist())) == k, f"query {b}: repeated IDs {gi}"
+        assert (gi >= 0).all() and (gi < wl.n).all(), f"query {b}: ID out of range"
+        sk = ref["scores"][b][k - 1]
+        band = lambda s: abs(s - sk) <= SWAP_REL * max(abs(s), abs(sk))
+        for x in set(gi.tolist()) ^ set(oi.tolist()):
+            assert band(fin[x]), (f"query {b}: chunk {x} (oracle score {fin[x]!r}) swapped "
+                                  f"outside the near-tie band of the k-th score {sk!r}")
+        s_gpu_ids = fin[gi]
+        for a in range(k - 1):
+            hi, lo = s_gpu_ids[a], s_gpu_ids[a + 1]
+            assert hi >= lo - SWAP_REL * max(abs(hi), abs(lo)), (
+                f"query {b}: order differs beyond near-ties at {a}: {hi!r} < {lo!r}")
+        rel = np.abs(got["scores"][r].astype(np.float64) - fin[gi]) / np.abs(fin[gi])
+        assert rel.max() <= SCORE_REL, f"query {b}: score error {rel.max():.3g} > {SCORE_REL}"
+        assert (got["page_ids"][r] == page_of[gi]).all(), f"query {b}: page IDs differ"
+        assert got["n_pages"][r] == len(set(page_of[gi].tolist())), f"query {b}: page count"
+        assert got["n_pages"][r] == ref["n_pages"][b] or set(gi.tolist()) != set(oi.tolist())
+
+
+# --------------------------------------------------------------------------- relation update
+def check_update(wl, sample=None, M=None, seed=0):
+    """Append wl.new_emb to a store holding wl, run the update on the GPU and
+    compare with the oracle (all new rows, or a seeded sample of them)."""
+    import torch
+    from paper_2607_05708_gb300 import MemStore
+    M = M or wl.top_m
+    n_old, n_new = wl.n, wl.new_emb.shape[0]
+    store = MemStore.from_arrays(wl.emb, wl.page_of["clustered"], wl.row_ptr, wl.col, wl.aff,
+                                 capacity=n_old + n_new, chunks_per_page=wl.chunks_per_page,
+                                 temperature=wl.tau, relation_scale=wl.relation_scale)
+    new = torch.from_numpy(np.ascontiguousarray(wl.new_emb).view(np.int16)).cuda()
+    first = store.append_chunks(new)
+    assert first == n_old
+    store.update_relations(first, n_new, M, reciprocal=wl.reciprocal)
+    store.sync()
+    rp, col, aff, w = (t.cpu().numpy() for t in store.export_csr())
+    all_emb = np.concatenate([wl.emb, wl.new_emb])
+    if sample is None:
+        old_rp = np.concatenate([wl.row_ptr, np.full(n_new, wl.row_ptr[-1], np.int64)])
+        ref = oracle.update_relations(all_emb, n_old, n_new, M, old_rp, wl.col, wl.aff,
+                                      scale=wl.relation_scale, reciprocal=wl.reciprocal)
+        _compare_update(wl, M, rp, col, aff, w, ref, np.arange(n_new), full=True)
+    else:
+        rng = np.random.default_rng(seed)
+        picks = np.sort(rng.choice(n_new, size=min(sample, n_new), replace=False))
+        # oracle on the sampled new chunks only (each is independent of the others)
+        sub_emb = np.concatenate([wl.emb, wl.new_emb[picks]])
+        old_rp = np.concatenate([wl.row_ptr, np.full(len(picks), wl.row_ptr[-1], np.int64)])
+        ref = oracle.update_relations(sub_emb, n_old, len(picks), M, old_rp, wl.col, wl.aff,
+                                      scale=wl.relation_scale, reciprocal=wl.reciprocal)
+        _compare_update(wl, M, rp, col, aff, w, ref, picks, full=False)
+    return store
+
+
+def _compare_update(wl, M, rp, col, aff, w, ref, picks, full):
+    n_old = wl.n
+    E = oracle_free_widen(np.concatenate([wl.emb, wl.new_emb]))
+    assert (np.diff(rp) >= 0).all()
+    assert rp[-1] == wl.row_ptr[-1] + len(wl.new_emb) * M * (2 if wl.reciprocal else 1)
+    for t, a in enumerate(picks):
+        nid = n_old + a
+        g_cols = col[rp[nid]:rp[nid + 1]]
+        o_ids = ref["nbr_ids"][t]
+        o_cos = ref["nbr_cos"][t]
+        assert len(g_cols) == M and (np.diff(g_cols) > 0).all()
+        kth = o_cos[M - 1]
+        for x in set(g_cols.tolist()) ^ set(o_ids.tolist()):
+            cx = float(E[x] @ E[nid])
+            assert abs(cx - kth) < COS_ABS, f"new chunk {nid}: neighbour {x} swapped ({cx} vs {kth})"
+        for x, lg in zip(g_cols, aff[rp[nid]:rp[nid + 1]]):
+            cx = float(E[x] @ E[nid])
+            assert abs(lg - wl.relation_scale * cx) <= 1e-5 * max(1.0, abs(wl.relation_scale * cx)), \
+                f"logit of {nid}->{x}: {lg} vs {wl.relation_scale * cx}"
+            if wl.reciprocal:
+                row = col[rp[x]:rp[x + 1]]
+                pos = np.searchsorted(row, nid)
+                assert pos < len(row) and row[pos] == nid, f"missing reciprocal edge {x}->{nid}"
+                assert aff[rp[x] + pos] == lg
+    # weights: row softmax of the exported logits
+    wr = oracle.row_softmax(rp, aff)
+    assert np.allclose(w, wr, rtol=2e-3, atol=0)
+    if full:
+        # whole CSR identical to the oracle's, given no swaps were needed
+        if (ref["row_ptr"] == rp).all() and (ref["col"] == col).all():
+            assert np.allclose(aff, ref["aff"], rtol=1e-5, atol=1e-5)
+        else:
+            # a swap happened: row pointers can differ only through swapped reciprocal edges
+            assert ref["row_ptr"][-1] == rp[-1]
+        # old edges untouched
+        for i in range(0, n_old, max(1, n_old // 997)):
+            a, b = wl.row_ptr[i], wl.row_ptr[i + 1]
+            g = col[rp[i]:rp[i] + (b - a)]
+            assert (g == wl.col[a:b]).all()
+
+
+def oracle_free_widen(h):
+    """fp64 values of bf16 bits (plain widening, used for the test's own checks)."""
+    return ((np.ascontiguousarray(h).astype(np.uint32) << 16).view(np.float32)).astype(np.float64)

@@ -1,0 +1,66 @@
+"""The C-ABI library builds for sm_103a, loads without a GPU, and exports
+every function include/akashic_mem.h declares (no compute calls here)."""
+import ctypes
+import os
+import re
+import subprocess
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "akashic_mem.h")
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(akashic_mem_\w+)\s*\(", text)))
+
+
+@pytest.fixture(scope="module")
+def lib_path():
+    from paper_2607_05708_gb300 import _build
+    return _build.build()
+
+
+def test_header_matches_binding():
+    import paper_2607_05708_gb300 as pkg
+    assert declared_functions() == sorted(pkg.EXPORTS)
+
+
+def test_library_exports_every_declared_symbol(lib_path):
+    out = subprocess.run(["nm", "-D", "--defined-only", lib_path], capture_output=True, text=True,
+                         check=True).stdout
+    exported = set(re.findall(r"\bT (akashic_mem_\w+)", out))
+    missing = set(declared_functions()) - exported
+    assert not missing, f"not exported: {missing}"
+    lib = ctypes.CDLL(lib_path)
+    for name in declared_functions():
+        assert getattr(lib, name) is not None
+
+
+def test_binding_loads_and_reports_no_error(lib_path):
+    import paper_2607_05708_gb300 as pkg
+    lib = pkg.load_library()
+    assert lib.akashic_mem_last_error() == b""
+
+
+def test_invalid_config_is_rejected_without_gpu_work(lib_path):
+    """create() validates its arguments before touching any device."""
+    import paper_2607_05708_gb300 as pkg
+    lib = pkg.load_library()
+    h = ctypes.c_void_p()
+    for cfg in (pkg._Config(100, 10, 1, 0, 0.0, 0.0),     # dim not a multiple of 64
+                pkg._Config(64, 0, 1, 0, 0.0, 0.0),       # capacity 0
+                pkg._Config(64, 10, 0, 0, 0.0, 0.0)):     # chunks_per_page 0
+        assert lib.akashic_mem_create(ctypes.byref(cfg), ctypes.byref(h)) == 1
+        assert b"create" in lib.akashic_mem_last_error()
+    assert lib.akashic_mem_create(None, ctypes.byref(h)) == 1
+
+
+def test_sm103a_cubin_in_library(lib_path):
+    """The library carries code for sm_103a (listing the ELF sections only)."""
+    out = subprocess.run(["cuobjdump", "--list-elf", lib_path], capture_output=True, text=True)
+    if out.returncode != 0:
+        pytest.skip("cuobjdump unavailable")
+    assert "sm_103a" in out.stdout
