@@ -89,7 +89,8 @@ void akashic_mem_destroy(akashic_mem_t *m);
  *            (global target IDs < first_id+n, never the row itself, strictly
  *            ascending within a row), aff device float (edge logits; the
  *            relation weight of an edge is the softmax of its row's logits).
- *            All three NULL => no edges.
+ *            row_ptr NULL => no edges (col and aff must then be NULL too);
+ *            col and aff may be NULL when row_ptr describes no edges.
  *   first_id_out  host, receives first_id (may be NULL).
  * ECAPACITY if the store would exceed its capacity; EINVAL on a bad
  * argument; EDEVICE (at once, since this call synchronises) if the edges

@@ -351,9 +351,9 @@ akashic_status_t akashic_mem_append_chunks(akashic_mem_t *m, const uint16_t *emb
     g_last_error.clear();
     if (!m) return fail(AKASHIC_EINVAL, "append: NULL store");
     if (n < 0 || (n > 0 && !emb)) return fail(AKASHIC_EINVAL, "append: bad n or emb");
-    const bool has_edges = row_ptr || col || aff;
-    if (has_edges && !(row_ptr && col && aff))
-        return fail(AKASHIC_EINVAL, "append: row_ptr, col and aff must be given together");
+    const bool has_edges = row_ptr != nullptr;
+    if (!row_ptr && (col || aff))
+        return fail(AKASHIC_EINVAL, "append: col/aff given without row_ptr");
     if (m->n + n > m->cap)
         return fail(AKASHIC_ECAPACITY, "append: %lld + %lld chunks exceed capacity %lld",
                     (long long)m->n, (long long)n, (long long)m->cap);
@@ -372,6 +372,8 @@ akashic_status_t akashic_mem_append_chunks(akashic_mem_t *m, const uint16_t *emb
                                        m->status.as<int>(), st));
         AK_TRY(check_status(m, st, "append: edge check"));
         if (e_hi < e_lo) return fail(AKASHIC_EINVAL, "append: row_ptr decreases");
+        if (e_hi > e_lo && !(col && aff))
+            return fail(AKASHIC_EINVAL, "append: edges given without col or aff");
         if (m->nnz + (e_hi - e_lo) > 0x7fffffffLL)
             return fail(AKASHIC_ECAPACITY, "append: more than 2^31-1 relation edges");
     }
