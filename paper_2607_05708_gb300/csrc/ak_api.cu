@@ -525,9 +525,10 @@ akashic_status_t akashic_mem_retrieve(akashic_mem_t *m, const uint16_t *q, int32
     const int sms = device_sm_count();
     for (int32_t off = 0; off < B; off += 256) {
         const int b = B - off < 256 ? B - off : 256;
-        int bp = 16;
+        int bp = 32;
         while (bp < b) bp <<= 1;
         const int64_t tiles = score_tiles(n);
+        int zrows = 0;
         const SelectPlan sp = select_plan(n, bp, k, sms);
         AK_TRY(sc->qp.ensure((size_t)bp * m->dim * 2));
         AK_TRY(sc->shift.ensure((size_t)bp * 4));
@@ -545,7 +546,8 @@ akashic_status_t akashic_mem_retrieve(akashic_mem_t *m, const uint16_t *q, int32
                                          m->status.as<int>(), st));
             CUDA_TRY(launch_score(m->emb.as<uint16_t>(), n, m->dim, sc->qp.as<uint16_t>(), bp,
                                   sc->shift.as<float>(), m->tau, sc->u.as<float>(),
-                                  sc->zpart.as<float>(), m->status.as<int>(), st, &ph.launches));
+                                  sc->zpart.as<float>(), m->status.as<int>(), st, &ph.launches,
+                                  &zrows));
             ph.launches += 1;
         }
         const float *fin = sc->u.as<float>();
@@ -573,7 +575,7 @@ akashic_status_t akashic_mem_retrieve(akashic_mem_t *m, const uint16_t *q, int32
         {
             PhaseScope ph(m, AKASHIC_PHASE_SELECT, st);
             CUDA_TRY(launch_select(sp, fin, n, bp, b, k, sc->cand.as<unsigned long long>(),
-                                   sc->zpart.as<float>(), tiles, m->page_of.as<int32_t>(),
+                                   sc->zpart.as<float>(), zrows, m->page_of.as<int32_t>(),
                                    ids + (int64_t)off * k, scores + (int64_t)off * k,
                                    page_ids ? page_ids + (int64_t)off * k : nullptr,
                                    n_pages ? n_pages + off : nullptr, m->status.as<int>(), st,

@@ -51,17 +51,19 @@ __device__ __forceinline__ float unordered_bits(uint32_t o) {
 // ------------------------------------------------------------------ launchers
 // All launchers enqueue on `st` and report launch errors by return value.
 
-// Score (a1): u[j, c] = exp(tau * <e_j, q_c> - shift[c]) for j < n, c < bp,
-// written chunk-major with row stride bp; zpart[t, c] = sum of u over the
-// rows of score tile t.  Returns the number of score tiles (rows of zpart).
+// Score (a1) on the tensor cores: u[j, c] = exp(tau * <e_j, q_c> - shift[c])
+// for j < n, c < bp (bp = 32, 64, 128 or 256), written chunk-major with row
+// stride bp; zpart[r, c] = sum of u over the rows handled by score CTA r,
+// for r < *zrows.  score_tiles(n) bounds *zrows.
 int64_t score_tiles(int64_t n);
 cudaError_t launch_score(const uint16_t *emb, int64_t n, int dim, const uint16_t *qp, int bp,
                          const float *shift, float tau, float *u, float *zpart, int *status,
-                         cudaStream_t st, int *launches);
+                         cudaStream_t st, int *launches, int *zrows);
 
-// Plain dot products out[j, c] = <e_j, q_c> (fp32 accumulate), row stride bp.
+// Plain dot products out[j, c] = <e_j, q_c> (bf16 tensor cores, fp32
+// accumulate), row stride bp.
 cudaError_t launch_dots(const uint16_t *emb, int64_t n, int dim, const uint16_t *qp, int bp,
-                        float *out, cudaStream_t st, int *launches);
+                        float *out, int *status, cudaStream_t st, int *launches);
 
 // Query preparation: pad q (b rows) to bp rows of zeros and compute
 // shift[c] = tau * |q_c| * max_norm (0 for padding); flags ERANGE.

@@ -2,7 +2,9 @@
 // with per-tile partial sums toward Z = sum_i u (arXiv 2607.05708, §4.1,
 // Dense-only form of §5.5).  Also the query preparation and the running
 // maximum of chunk-embedding norms used for the shift bound c.
-#include "ak_common.cuh"
+#include <cudaTypedefs.h>
+
+#include "ak_sm100.cuh"
 
 namespace ak {
 
@@ -71,106 +73,309 @@ cudaError_t launch_row_norm_max(const uint16_t *emb, int64_t n, int dim, float *
     return cudaGetLastError();
 }
 
-// ------------------------------------------------------------------ score GEMM
-// Tiled SIMT GEMM: a 64-row x 64-query tile per CTA, K in steps of 32,
-// each thread a 4 x 4 block of outputs, fp32 accumulation of exactly
-// widened bf16 values.  The epilogue applies exp(tau*acc - shift) and sums
-// each query column over the tile's rows.
-constexpr int SM_TM = 64, SM_TN = 64, SM_TK = 32;
-
-int64_t score_tiles(int64_t n) { return ceil_div<int64_t>(n, SM_TM); }
-
-template <bool EXP>
-__global__ __launch_bounds__(256) void k_score_simt(const uint16_t *__restrict__ emb, int64_t n,
-                                                    int dim, const uint16_t *__restrict__ qp,
-                                                    int bp, const float *__restrict__ shift,
-                                                    float tau, float *__restrict__ u,
-                                                    float *__restrict__ zpart) {
-    __shared__ float As[SM_TK][SM_TM + 4];
-    __shared__ float Bs[SM_TK][SM_TN + 4];
-    __shared__ float zs[16][SM_TN];
-    const int64_t tile = blockIdx.x;
-    const int64_t r0 = tile * SM_TM;
-    const int c0 = blockIdx.y * SM_TN;
-    const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
-    float acc[4][4];
-#pragma unroll
-    for (int i = 0; i < 4; ++i)
-#pragma unroll
-        for (int j = 0; j < 4; ++j) acc[i][j] = 0.f;
-
-    for (int k0 = 0; k0 < dim; k0 += SM_TK) {
-        for (int i = threadIdx.x; i < SM_TM * SM_TK; i += 256) {
-            int r = i / SM_TK, kk = i % SM_TK;
-            int64_t row = r0 + r;
-            As[kk][r] = row < n ? bf16_to_f32(emb[row * dim + k0 + kk]) : 0.f;
-        }
-        for (int i = threadIdx.x; i < SM_TN * SM_TK; i += 256) {
-            int c = i / SM_TK, kk = i % SM_TK;
-            int col = c0 + c;
-            Bs[kk][c] = col < bp ? bf16_to_f32(qp[(int64_t)col * dim + k0 + kk]) : 0.f;
-        }
-        __syncthreads();
-#pragma unroll 8
-        for (int kk = 0; kk < SM_TK; ++kk) {
-            float a[4], b[4];
-#pragma unroll
-            for (int i = 0; i < 4; ++i) a[i] = As[kk][ty * 4 + i];
-#pragma unroll
-            for (int j = 0; j < 4; ++j) b[j] = Bs[kk][tx * 4 + j];
-#pragma unroll
-            for (int i = 0; i < 4; ++i)
-#pragma unroll
-                for (int j = 0; j < 4; ++j) acc[i][j] = fmaf(a[i], b[j], acc[i][j]);
-        }
-        __syncthreads();
+// ------------------------------------------------------------------ tensor maps
+static PFN_cuTensorMapEncodeTiled_v12000 tmap_encoder() {
+    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+    if (!fn) {
+        void *p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                             &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = (PFN_cuTensorMapEncodeTiled_v12000)p;
+        else
+            cudaGetLastError();
     }
-    float colsum[4] = {0.f, 0.f, 0.f, 0.f};
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-        int64_t row = r0 + ty * 4 + i;
-        if (row >= n) continue;
-#pragma unroll
-        for (int j = 0; j < 4; ++j) {
-            int col = c0 + tx * 4 + j;
-            if (col < bp) {
-                float v = EXP ? expf(tau * acc[i][j] - shift[col]) : acc[i][j];
-                u[row * bp + col] = v;
-                colsum[j] += v;
+    return fn;
+}
+
+cudaError_t make_tmap_2d(CUtensorMap *map, const void *base, CUtensorMapDataType dtype,
+                         int elem_bytes, uint64_t inner, uint64_t outer, uint64_t row_bytes,
+                         uint32_t box_inner, uint32_t box_outer) {
+    auto fn = tmap_encoder();
+    if (!fn) return cudaErrorNotSupported;
+    (void)elem_bytes;
+    cuuint64_t dims[2] = {inner, outer};
+    cuuint64_t strides[1] = {row_bytes};
+    cuuint32_t box[2] = {box_inner, box_outer};
+    cuuint32_t es[2] = {1, 1};
+    CUresult r = fn(map, dtype, 2, const_cast<void *>(base), dims, strides, box, es,
+                    CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                    CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
+}
+
+// ------------------------------------------------------------------ tcgen05 GEMM
+// C[j, c] = <e_j, q_c> for a 128-row tile of E against all BP (<= 256)
+// query rows, on the 5th-generation tensor cores: bf16 operands staged by
+// TMA in the 128-byte swizzle layout, fp32 accumulator in tensor memory
+// (two accumulators, so the epilogue of one tile overlaps the MMAs of the
+// next), persistent CTAs walking the tiles round-robin.
+//   warp 0     TMA producer (one thread)
+//   warp 1     TMEM owner and MMA issuer (one thread)
+//   warps 2-5  epilogue: TMEM -> registers -> (EXP: exp(tau*acc - shift),
+//              column sums toward Z) -> swizzled staging -> TMA store
+template <int BP>
+struct GemmCfg {
+    static constexpr int BM = 128, BK = 64;
+    static constexpr int A_BYTES = BM * BK * 2;
+    static constexpr int B_BYTES = BP * BK * 2;
+    static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
+    static constexpr int OUT_BYTES = BM * 32 * 4;
+    static constexpr int MISC = 4096;   // shift, Z sums, flags, barriers
+    static constexpr int BUDGET = 227 * 1024 - 1024;
+    static constexpr int S_FIT = (BUDGET - 2 * OUT_BYTES - MISC) / STAGE_BYTES;
+    static constexpr int STAGES = S_FIT > 8 ? 8 : S_FIT;
+    static constexpr int TMEM_COLS = 2 * BP < 32 ? 32 : 2 * BP;
+    static constexpr int SMEM = 1024 + STAGES * STAGE_BYTES + 2 * OUT_BYTES + MISC;
+    static_assert(BP >= 32 && BP <= 256 && (BP & (BP - 1)) == 0, "BP must be 32..256, a power of 2");
+    static_assert(STAGES >= 2, "not enough shared memory for two stages");
+};
+
+template <int BP, bool EXP>
+__global__ __launch_bounds__(192, 1) void k_gemm_umma(const __grid_constant__ CUtensorMap tmA,
+                                                      const __grid_constant__ CUtensorMap tmB,
+                                                      const __grid_constant__ CUtensorMap tmC,
+                                                      int64_t n_rows, int dim,
+                                                      const float *__restrict__ shift_g, float tau,
+                                                      float *__restrict__ zpart, int *status) {
+    using C = GemmCfg<BP>;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *smem = (uint8_t *)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+    uint8_t *sA = smem;
+    uint8_t *sB = smem + C::STAGES * C::A_BYTES;
+    float *sOut = (float *)(smem + C::STAGES * C::STAGE_BYTES);     // 2 x [128][32], swizzled
+    uint8_t *misc = smem + C::STAGES * C::STAGE_BYTES + 2 * C::OUT_BYTES;
+    float *shift_s = (float *)misc;                  // [BP]
+    float *zacc = shift_s + BP;                      // [BP]
+    float *zq = zacc + BP;                           // [4][32]  (ends below misc + 2560)
+    int *go = (int *)(misc + 2560);                  // epilogue: the tile's accumulator is ready
+    uint64_t *bars = (uint64_t *)(misc + 3072);      // full[S], empty[S], tfull[2], tempty[2]
+    uint64_t *full = bars, *empty = bars + C::STAGES;
+    uint64_t *tfull = bars + 2 * C::STAGES, *tempty = tfull + 2;
+    uint32_t *tmem_slot = (uint32_t *)(tempty + 2);
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int64_t n_tiles = (n_rows + C::BM - 1) / C::BM;
+    const int kb_n = dim / C::BK;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < C::STAGES; ++s) {
+            mbar_init(&full[s], 1);
+            mbar_init(&empty[s], 1);
+        }
+        for (int a = 0; a < 2; ++a) {
+            mbar_init(&tfull[a], 1);
+            mbar_init(&tempty[a], 1);
+        }
+        mbar_fence_init();
+    }
+    if (warp == 1) {
+        tmem_alloc(tmem_slot, C::TMEM_COLS);
+        tmem_relinquish();
+    }
+    for (int i = threadIdx.x; i < BP; i += blockDim.x) {
+        shift_s[i] = EXP ? shift_g[i] : 0.f;
+        zacc[i] = 0.f;
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem_base = *tmem_slot;
+
+    if (warp == 0) {
+        if (lane == 0) {
+            // ---------------- TMA producer
+            uint32_t stage = 0, phase = 0;
+            int last_par[8];
+            for (int s = 0; s < 8; ++s) last_par[s] = -1;
+            bool ok = true;
+            for (int64_t t = blockIdx.x; t < n_tiles && ok; t += gridDim.x) {
+                for (int kb = 0; kb < kb_n; ++kb) {
+                    if (!mbar_wait(&empty[stage], phase ^ 1u, status)) {
+                        ok = false;
+                        break;
+                    }
+                    mbar_expect_tx(&full[stage], C::STAGE_BYTES);
+                    tma_load_2d(sA + stage * C::A_BYTES, &tmA, &full[stage], kb * C::BK,
+                                (int)(t * C::BM));
+                    tma_load_2d(sB + stage * C::B_BYTES, &tmB, &full[stage], kb * C::BK, 0);
+                    last_par[stage] = (int)phase;
+                    if (++stage == (uint32_t)C::STAGES) {
+                        stage = 0;
+                        phase ^= 1u;
+                    }
+                }
+            }
+            if (!ok) {
+                // let every copy this thread issued land before the CTA exits
+                for (int s = 0; s < C::STAGES; ++s)
+                    if (last_par[s] >= 0) mbar_wait(&full[s], (uint32_t)last_par[s], status);
             }
         }
-    }
+    } else if (warp == 1) {
+        if (lane == 0) {
+            // ---------------- MMA issuer
+            const uint32_t idesc = idesc_bf16_m128(BP);
+            uint32_t stage = 0, phase = 0;
+            int it = 0;
+            bool ok = true;
+            for (int64_t t = blockIdx.x; t < n_tiles && ok; t += gridDim.x, ++it) {
+                const int acc = it & 1;
+                const uint32_t aph = (uint32_t)(it >> 1) & 1u;
+                if (!mbar_wait(&tempty[acc], aph ^ 1u, status)) break;
+                tc_fence_after();
+                const uint32_t d = tmem_base + (uint32_t)(acc * BP);
+                for (int kb = 0; kb < kb_n; ++kb) {
+                    if (!mbar_wait(&full[stage], phase, status)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    const uint64_t ad = sdesc_sw128(smem_u32(sA + stage * C::A_BYTES));
+                    const uint64_t bd = sdesc_sw128(smem_u32(sB + stage * C::B_BYTES));
 #pragma unroll
-    for (int j = 0; j < 4; ++j) zs[ty][tx * 4 + j] = colsum[j];
-    if (!EXP) return;
-    __syncthreads();
-    if (threadIdx.x < SM_TN) {
-        int col = c0 + threadIdx.x;
-        if (col < bp) {
-            float s = 0.f;
-#pragma unroll
-            for (int r = 0; r < 16; ++r) s += zs[r][threadIdx.x];
-            zpart[tile * bp + col] = s;
+                    for (int k = 0; k < C::BK / 16; ++k)
+                        umma_bf16(d, ad + (uint64_t)(2 * k), bd + (uint64_t)(2 * k), idesc,
+                                  (kb | k) != 0 ? 1u : 0u);
+                    umma_commit(&empty[stage]);
+                    if (++stage == (uint32_t)C::STAGES) {
+                        stage = 0;
+                        phase ^= 1u;
+                    }
+                }
+                if (ok) umma_commit(&tfull[acc]);
+            }
         }
+    } else {
+        // ---------------- epilogue (128 threads; warp w reads TMEM lanes 32*(w%4)..)
+        const int q = warp & 3;
+        const int row = q * 32 + lane;                   // row inside the tile
+        const int et = threadIdx.x - 64;                 // 0..127
+        int it = 0, cc = 0;
+        for (int64_t t = blockIdx.x; t < n_tiles; t += gridDim.x, ++it) {
+            const int acc = it & 1;
+            const uint32_t aph = (uint32_t)(it >> 1) & 1u;
+            // one thread polls, the barrier makes the outcome uniform
+            if (et == 0) *go = mbar_wait(&tfull[acc], aph, status) ? 1 : 0;
+            named_bar(1, 128);
+            if (!*go) break;
+            tc_fence_after();
+            const bool valid = t * C::BM + row < n_rows;
+#pragma unroll 1
+            for (int ch = 0; ch < BP / 32; ++ch, ++cc) {
+                const int buf = cc & 1;
+                uint32_t r[32];
+                tmem_ld32(tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * BP + ch * 32), r);
+                tmem_ld_wait();
+                float v[32];
+#pragma unroll
+                for (int i = 0; i < 32; ++i) {
+                    const float x = __uint_as_float(r[i]);
+                    v[i] = valid ? (EXP ? expf(tau * x - shift_s[ch * 32 + i]) : x) : 0.f;
+                }
+                named_bar(1, 128);                       // staging[buf] free again
+                float4 *dst = (float4 *)(sOut + buf * (C::OUT_BYTES / 4) + row * 32);
+#pragma unroll
+                for (int j = 0; j < 8; ++j)
+                    dst[j ^ (row & 7)] = make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
+                fence_async_smem();
+                named_bar(1, 128);                       // staging[buf] complete
+                if (EXP) {
+                    const int c = et & 31, g = et >> 5;
+                    const float *so = sOut + buf * (C::OUT_BYTES / 4);
+                    float s = 0.f;
+#pragma unroll 8
+                    for (int rr = g * 32; rr < g * 32 + 32; ++rr)
+                        s += so[rr * 32 + ((((c >> 2) ^ (rr & 7))) << 2) + (c & 3)];
+                    zq[g * 32 + c] = s;
+                }
+                if (et == 0) {
+                    tma_store_2d(&tmC, sOut + buf * (C::OUT_BYTES / 4), ch * 32, (int)(t * C::BM));
+                    bulk_commit();
+                }
+                if (EXP) {
+                    named_bar(1, 128);
+                    if (et < 32) zacc[ch * 32 + et] += (zq[et] + zq[32 + et]) + (zq[64 + et] + zq[96 + et]);
+                }
+                if (et == 0) bulk_wait_read<1>();
+            }
+            tc_fence_before();
+            named_bar(1, 128);
+            if (et == 0) mbar_arrive(&tempty[acc]);
+        }
+        if (et == 0) bulk_wait_all();
+        named_bar(1, 128);
+        if (EXP && zpart)
+            for (int c = et; c < BP; c += 128) zpart[(int64_t)blockIdx.x * BP + c] = zacc[c];
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    if (warp == 1) tmem_dealloc(tmem_base, C::TMEM_COLS);
+}
+
+int64_t score_tiles(int64_t n) { return ceil_div<int64_t>(n, 128); }
+
+template <int BP, bool EXP>
+static cudaError_t gemm_bp(const uint16_t *emb, int64_t n, int dim, const uint16_t *qp,
+                           const float *shift, float tau, float *out, float *zpart, int *status,
+                           cudaStream_t st, int *zrows) {
+    using C = GemmCfg<BP>;
+    static bool attr[64] = {false};
+    int dev = 0;
+    cudaGetDevice(&dev);
+    if (dev >= 0 && dev < 64 && !attr[dev]) {
+        cudaError_t e = cudaFuncSetAttribute(k_gemm_umma<BP, EXP>,
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
+        if (e != cudaSuccess) return e;
+        attr[dev] = true;
+    }
+    CUtensorMap ta, tb, tc;
+    cudaError_t e = make_tmap_2d(&ta, emb, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, (uint64_t)dim,
+                                 (uint64_t)n, (uint64_t)dim * 2, 64, 128);
+    if (e == cudaSuccess)
+        e = make_tmap_2d(&tb, qp, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, (uint64_t)dim, (uint64_t)BP,
+                         (uint64_t)dim * 2, 64, BP);
+    if (e == cudaSuccess)
+        e = make_tmap_2d(&tc, out, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, (uint64_t)BP, (uint64_t)n,
+                         (uint64_t)BP * 4, 32, 128);
+    if (e != cudaSuccess) return e;
+    const int64_t tiles = ceil_div<int64_t>(n, 128);
+    const int grid = (int)(tiles < device_sm_count() ? tiles : device_sm_count());
+    k_gemm_umma<BP, EXP><<<grid, 192, C::SMEM, st>>>(ta, tb, tc, n, dim, shift, tau, zpart, status);
+    if (zrows) *zrows = grid;
+    return cudaGetLastError();
+}
+
+template <bool EXP>
+static cudaError_t gemm_dispatch(const uint16_t *emb, int64_t n, int dim, const uint16_t *qp,
+                                 int bp, const float *shift, float tau, float *out, float *zpart,
+                                 int *status, cudaStream_t st, int *zrows) {
+    if (n <= 0 || dim % 64 != 0) return cudaErrorInvalidValue;
+    switch (bp) {
+    case 32: return gemm_bp<32, EXP>(emb, n, dim, qp, shift, tau, out, zpart, status, st, zrows);
+    case 64: return gemm_bp<64, EXP>(emb, n, dim, qp, shift, tau, out, zpart, status, st, zrows);
+    case 128: return gemm_bp<128, EXP>(emb, n, dim, qp, shift, tau, out, zpart, status, st, zrows);
+    case 256: return gemm_bp<256, EXP>(emb, n, dim, qp, shift, tau, out, zpart, status, st, zrows);
+    default: return cudaErrorInvalidValue;
     }
 }
 
 cudaError_t launch_score(const uint16_t *emb, int64_t n, int dim, const uint16_t *qp, int bp,
                          const float *shift, float tau, float *u, float *zpart, int *status,
-                         cudaStream_t st, int *launches) {
-    (void)status;
-    dim3 grid((unsigned)score_tiles(n), (unsigned)ceil_div(bp, SM_TN));
-    k_score_simt<true><<<grid, 256, 0, st>>>(emb, n, dim, qp, bp, shift, tau, u, zpart);
+                         cudaStream_t st, int *launches, int *zrows) {
+    cudaError_t e = gemm_dispatch<true>(emb, n, dim, qp, bp, shift, tau, u, zpart, status, st, zrows);
     if (launches) *launches += 1;
-    return cudaGetLastError();
+    return e;
 }
 
 cudaError_t launch_dots(const uint16_t *emb, int64_t n, int dim, const uint16_t *qp, int bp,
-                        float *out, cudaStream_t st, int *launches) {
-    dim3 grid((unsigned)score_tiles(n), (unsigned)ceil_div(bp, SM_TN));
-    k_score_simt<false><<<grid, 256, 0, st>>>(emb, n, dim, qp, bp, nullptr, 1.f, out, nullptr);
+                        float *out, int *status, cudaStream_t st, int *launches) {
+    cudaError_t e = gemm_dispatch<false>(emb, n, dim, qp, bp, nullptr, 1.f, out, nullptr, status,
+                                         st, nullptr);
     if (launches) *launches += 1;
-    return cudaGetLastError();
+    return e;
 }
 
 }  // namespace ak

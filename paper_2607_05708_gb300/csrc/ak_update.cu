@@ -20,7 +20,7 @@ __global__ void k_pad_rows(const uint16_t *__restrict__ src, int b, int bp, int 
 
 akashic_status_t relate_top_m(const UpdateArgs &a, cudaStream_t st, int *launches) {
     const int64_t n_old = a.first;
-    int bp_max = 16;
+    int bp_max = 32;
     while (bp_max < 256 && bp_max < a.n_new) bp_max <<= 1;
     uint16_t *qp = nullptr;
     float *dots = nullptr;
@@ -31,7 +31,7 @@ akashic_status_t relate_top_m(const UpdateArgs &a, cudaStream_t st, int *launche
     if (e == cudaSuccess) {
         // lists for the smallest bp are the most numerous; size for the worst case
         int64_t lists = 0;
-        for (int bp = 16; bp <= bp_max; bp <<= 1) {
+        for (int bp = 32; bp <= bp_max; bp <<= 1) {
             SelectPlan sp = select_plan(n_old, bp, a.M, device_sm_count());
             int64_t need = sp.lists * bp;
             lists = need > lists ? need : lists;
@@ -46,12 +46,13 @@ akashic_status_t relate_top_m(const UpdateArgs &a, cudaStream_t st, int *launche
     }
     for (int64_t off = 0; rc == AKASHIC_OK && off < a.n_new; off += 256) {
         const int b = (int)(a.n_new - off < 256 ? a.n_new - off : 256);
-        int bp = 16;
+        int bp = 32;
         while (bp < b) bp <<= 1;
         k_pad_rows<<<device_sm_count(), 256, 0, st>>>(a.emb + (a.first + off) * a.dim, b, bp, a.dim,
                                                        qp);
         e = cudaGetLastError();
-        if (e == cudaSuccess) e = launch_dots(a.emb, n_old, a.dim, qp, bp, dots, st, launches);
+        if (e == cudaSuccess)
+            e = launch_dots(a.emb, n_old, a.dim, qp, bp, dots, a.status, st, launches);
         const SelectPlan sp = select_plan(n_old, bp, a.M, device_sm_count());
         if (e == cudaSuccess)
             e = launch_select_signed(sp, dots, n_old, bp, b, a.M, cand, off, a.nbr_ids, a.nbr_cos,
