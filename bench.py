@@ -177,6 +177,8 @@ def main():
     ap.add_argument("--cpu-queries", type=int, default=8)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--placement", default="clustered")
+    ap.add_argument("--scale", type=float, default=1.0,
+                    help="shrink N (profiling captures of a smaller case); 1.0 = the benchmark")
     args = ap.parse_args()
     if args.impl == "reference":
         return run_reference(args)
@@ -196,7 +198,7 @@ def main():
     from paper_2607_05708_gb300 import MemStore
 
     t_gen = time.perf_counter()
-    wl = synth.workload(2)
+    wl = synth.workload(2, scale=args.scale)
     t_gen = time.perf_counter() - t_gen
     cpu = None
     if rank == 0 and not args.no_cpu_baseline and ws == 1:
@@ -314,7 +316,8 @@ def main():
         "vs_baseline": None,
         "dtype": "f32",
         "data": "synthetic",
-        "config": {"workload": WORKLOAD, "l2": "inputs larger than L2 (E 2.1 GB, score slabs 1.07 GB "
+        "config": {"workload": WORKLOAD if args.scale == 1.0 else f"{WORKLOAD} scaled by {args.scale}",
+                   "l2": "inputs larger than L2 (E 2.1 GB, score slabs 1.07 GB "
                    "each), no flush", "placement": args.placement,
                    "parallelism": "replicas" if ws > 1 else "single GPU"},
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": hbm, "unit": "GB/s",
