@@ -79,7 +79,10 @@ void akashic_mem_destroy(akashic_mem_t *m);
 
 /* Append n immutable chunk records (§4.2: chunks are written once; the
  * store's IDs are assigned in append order, first_id .. first_id+n-1).
- *   emb      device, n x dim bf16 bits.
+ * In device memory the batch is laid out in page order (ID order within a
+ * page), so that chunks the placement co-locates are adjacent rows; IDs
+ * are unaffected.
+ *   emb      device, n x dim bf16 bits, 16-byte aligned.
  *   page_of  device int32[n], the physical page of each new chunk (>= 0), or
  *            NULL: fresh pages after the highest page in use, packed
  *            chunks_per_page at a time in ID order.

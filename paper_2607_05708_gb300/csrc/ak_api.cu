@@ -4,6 +4,7 @@
 #include <math.h>
 #include <stdarg.h>
 #include <stdio.h>
+#include <stdlib.h>
 #include <string.h>
 
 #include <mutex>
@@ -77,7 +78,7 @@ struct DevBuf {
 };
 
 struct StreamScratch {
-    DevBuf qp, shift, u, sa, sb, zpart, partial, cand;
+    DevBuf qp, shift, u, sa, sb, zpart, partial, cand, counters;
 };
 
 struct ProfRec {
@@ -107,14 +108,17 @@ struct akashic_mem {
     float rel_scale = 10.f;
     int64_t n = 0;
     int64_t next_page = 0;
-    DevBuf emb, page_of, max_norm, status;
+    // chunks live in HBM in page order: row r holds chunk ext_of[r], chunk c
+    // is in row row_of[c]; page_of is indexed by row
+    DevBuf emb, page_of, ext_of, row_of, max_norm, status;
     // canonical out-edge CSR
     int64_t nnz = 0;
     DevBuf row_ptr, col, aff, w;
     // in-edge transpose + split plan for the propagation hop
     DevBuf in_ptr, in_src, in_w;
+    SplitParams split;
     int64_t n_split = 0, n_segs = 0;
-    DevBuf split_row, split_slot0, seg_e0, seg_e1;
+    DevBuf split_row, split_slot0, seg_e0, seg_e1, seg_slot;
     std::mutex mu;
     std::unordered_map<void *, StreamScratch *> scratch;
     // profiling
@@ -166,12 +170,6 @@ struct PhaseScope {
 };
 
 // ------------------------------------------------------------------ small kernels
-__global__ void k_fill_pages(int32_t *page_of, int64_t n, int64_t first_page, int per_page) {
-    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n;
-         i += (int64_t)gridDim.x * blockDim.x)
-        page_of[i] = (int32_t)(first_page + i / per_page);
-}
-
 __global__ void k_page_max(const int32_t *page_of, int64_t n, int *out_max, int *status) {
     int best = -1;
     for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n;
@@ -227,49 +225,80 @@ static akashic_status_t rebuild_in_edges(akashic_mem *m, cudaStream_t st) {
         AK_TRY(vals.ensure((size_t)nnz * 4));
         AK_TRY(keys2.ensure((size_t)nnz * 4));
         AK_TRY(vals2.ensure((size_t)nnz * 4));
+        const int32_t *row_of = m->row_of.as<int32_t>();
         CUDA_TRY(launch_edge_src_check(m->row_ptr.as<int64_t>(), m->col.as<int32_t>(), n, 0, n,
                                        src.as<int32_t>(), m->status.as<int>(), st));
-        CUDA_TRY(cudaMemcpyAsync(keys.p, m->col.p, (size_t)nnz * 4, cudaMemcpyDeviceToDevice, st));
+        // edges ordered by (target row, source row): sort by source row, then
+        // stably by target row
+        CUDA_TRY(launch_map_keys(nullptr, src.as<int32_t>(), row_of, keys.as<uint32_t>(), nnz, st));
         CUDA_TRY(launch_iota(vals.as<uint32_t>(), nnz, st));
         bool alt = false;
         CUDA_TRY(radix_sort_pairs(keys.as<uint32_t>(), vals.as<uint32_t>(), keys2.as<uint32_t>(),
                                   vals2.as<uint32_t>(), nnz, bits_for(n - 1), tmp.p, tmp.cap, st,
                                   &alt));
-        const uint32_t *order = alt ? vals2.as<uint32_t>() : vals.as<uint32_t>();
-        CUDA_TRY(launch_gather_in(order, src.as<int32_t>(), m->w.as<float>(), m->in_src.as<int32_t>(),
-                                  m->in_w.as<float>(), nnz, st));
+        uint32_t *k1 = alt ? keys2.as<uint32_t>() : keys.as<uint32_t>();
+        uint32_t *v1 = alt ? vals2.as<uint32_t>() : vals.as<uint32_t>();
+        uint32_t *k2 = alt ? keys.as<uint32_t>() : keys2.as<uint32_t>();
+        uint32_t *v2 = alt ? vals.as<uint32_t>() : vals2.as<uint32_t>();
+        CUDA_TRY(launch_map_keys(v1, m->col.as<int32_t>(), row_of, k1, nnz, st));
+        bool alt2 = false;
+        CUDA_TRY(radix_sort_pairs(k1, v1, k2, v2, nnz, bits_for(n - 1), tmp.p, tmp.cap, st, &alt2));
+        const uint32_t *order = alt2 ? v2 : v1;
+        CUDA_TRY(launch_gather_in(order, src.as<int32_t>(), row_of, m->w.as<float>(),
+                                  m->in_src.as<int32_t>(), m->in_w.as<float>(), nnz, st));
     }
     int64_t *degp = deg.as<int64_t>();
     CUDA_TRY(cudaMemsetAsync(degp, 0, (size_t)(n + 1) * sizeof(int64_t), st));
-    CUDA_TRY(launch_in_degree(m->col.as<int32_t>(), nnz, degp, st));
+    CUDA_TRY(launch_in_degree(m->col.as<int32_t>(), m->row_of.as<int32_t>(), nnz, degp, st));
     CUDA_TRY(scan_exclusive(degp, m->in_ptr.as<int64_t>(), n, tmp.p, tmp.cap, st));
-    // split plan
+    // split plan: hub rows cut into window segments, segments in window-major order
     DevBuf nseg, flag, slot_off, split_idx;
     AK_TRY(nseg.ensure((size_t)(n + 1) * 8));
     AK_TRY(flag.ensure((size_t)(n + 1) * 8));
     AK_TRY(slot_off.ensure((size_t)(n + 1) * 8));
     AK_TRY(split_idx.ensure((size_t)(n + 1) * 8));
-    CUDA_TRY(launch_split_count(m->in_ptr.as<int64_t>(), n, HOP_SEG, nseg.as<int64_t>(),
-                                flag.as<int64_t>(), st));
+    CUDA_TRY(launch_split_count(m->split, m->in_ptr.as<int64_t>(), m->in_src.as<int32_t>(), n,
+                                nseg.as<int64_t>(), flag.as<int64_t>(), st));
     CUDA_TRY(scan_exclusive(nseg.as<int64_t>(), slot_off.as<int64_t>(), n, tmp.p, tmp.cap, st));
     CUDA_TRY(scan_exclusive(flag.as<int64_t>(), split_idx.as<int64_t>(), n, tmp.p, tmp.cap, st));
     int64_t n_segs = 0, n_split = 0;
     CUDA_TRY(cudaMemcpyAsync(&n_segs, slot_off.as<int64_t>() + n, 8, cudaMemcpyDeviceToHost, st));
     CUDA_TRY(cudaMemcpyAsync(&n_split, split_idx.as<int64_t>() + n, 8, cudaMemcpyDeviceToHost, st));
     AK_TRY(check_status(m, st, "relation graph rebuild"));
+    if (n_segs > 0x7fffffffLL) return fail(AKASHIC_ECAPACITY, "too many hub segments");
     m->n_segs = n_segs;
     m->n_split = n_split;
     if (n_split > 0) {
+        DevBuf e0, e1, win, order, win2, order2, rtmp;
         AK_TRY(m->split_row.ensure((size_t)n_split * 4));
         AK_TRY(m->split_slot0.ensure((size_t)(n_split + 1) * 8));
         AK_TRY(m->seg_e0.ensure((size_t)n_segs * 8));
         AK_TRY(m->seg_e1.ensure((size_t)n_segs * 8));
-        CUDA_TRY(launch_split_fill(m->in_ptr.as<int64_t>(), n, HOP_SEG, nseg.as<int64_t>(),
-                                   slot_off.as<int64_t>(), split_idx.as<int64_t>(),
-                                   m->split_row.as<int32_t>(), m->split_slot0.as<int64_t>(),
-                                   m->seg_e0.as<int64_t>(), m->seg_e1.as<int64_t>(), st));
+        AK_TRY(m->seg_slot.ensure((size_t)n_segs * 4));
+        AK_TRY(e0.ensure((size_t)n_segs * 8));
+        AK_TRY(e1.ensure((size_t)n_segs * 8));
+        AK_TRY(win.ensure((size_t)n_segs * 4));
+        AK_TRY(order.ensure((size_t)n_segs * 4));
+        AK_TRY(win2.ensure((size_t)n_segs * 4));
+        AK_TRY(order2.ensure((size_t)n_segs * 4));
+        AK_TRY(rtmp.ensure(radix_tmp_bytes(n_segs) + 4096));
+        CUDA_TRY(launch_split_fill(m->split, m->in_ptr.as<int64_t>(), m->in_src.as<int32_t>(), n,
+                                   nseg.as<int64_t>(), slot_off.as<int64_t>(),
+                                   split_idx.as<int64_t>(), m->split_row.as<int32_t>(),
+                                   m->split_slot0.as<int64_t>(), e0.as<int64_t>(),
+                                   e1.as<int64_t>(), win.as<uint32_t>(), st));
         CUDA_TRY(cudaMemcpyAsync(m->split_slot0.as<int64_t>() + n_split, &n_segs, 8,
                                  cudaMemcpyHostToDevice, st));
+        CUDA_TRY(launch_iota(order.as<uint32_t>(), n_segs, st));
+        bool alt = false;
+        CUDA_TRY(radix_sort_pairs(win.as<uint32_t>(), order.as<uint32_t>(), win2.as<uint32_t>(),
+                                  order2.as<uint32_t>(), n_segs, bits_for((n - 1) / m->split.win_rows),
+                                  rtmp.p, rtmp.cap, st, &alt));
+        CUDA_TRY(launch_seg_permute(alt ? order2.as<uint32_t>() : order.as<uint32_t>(),
+                                    e0.as<int64_t>(), e1.as<int64_t>(), n_segs,
+                                    m->seg_e0.as<int64_t>(), m->seg_e1.as<int64_t>(),
+                                    m->seg_slot.as<int32_t>(), st));
+        AK_TRY(check_status(m, st, "relation graph rebuild"));
     }
     return check_status(m, st, "relation graph rebuild");
 }
@@ -305,9 +334,16 @@ akashic_status_t akashic_mem_create(const akashic_mem_config_t *cfg, akashic_mem
     m->per_page = cfg->chunks_per_page;
     m->tau = cfg->temperature > 0.f ? cfg->temperature : 1.0f / sqrtf((float)cfg->dim);
     m->rel_scale = cfg->relation_scale > 0.f ? cfg->relation_scale : 10.f;
+    // propagation plan knobs (tuning only; results do not depend on them
+    // beyond fp32 summation order)
+    if (const char *v = getenv("AKASHIC_SPLIT_T")) m->split.split_t = atoll(v) > 0 ? atoll(v) : m->split.split_t;
+    if (const char *v = getenv("AKASHIC_SEG_LEN")) m->split.seg_len = atoll(v) > 0 ? atoll(v) : m->split.seg_len;
+    if (const char *v = getenv("AKASHIC_WIN_ROWS")) m->split.win_rows = atoll(v) > 0 ? atoll(v) : m->split.win_rows;
     akashic_status_t s;
     if ((s = m->emb.ensure((size_t)m->cap * m->dim * 2)) != AKASHIC_OK ||
         (s = m->page_of.ensure((size_t)m->cap * 4)) != AKASHIC_OK ||
+        (s = m->ext_of.ensure((size_t)m->cap * 4)) != AKASHIC_OK ||
+        (s = m->row_of.ensure((size_t)m->cap * 4)) != AKASHIC_OK ||
         (s = m->max_norm.ensure(4)) != AKASHIC_OK || (s = m->status.ensure(4)) != AKASHIC_OK ||
         (s = m->row_ptr.ensure((size_t)(m->cap + 1) * 8)) != AKASHIC_OK ||
         (s = m->in_ptr.ensure((size_t)(m->cap + 1) * 8)) != AKASHIC_OK) {
@@ -351,6 +387,7 @@ akashic_status_t akashic_mem_append_chunks(akashic_mem_t *m, const uint16_t *emb
     g_last_error.clear();
     if (!m) return fail(AKASHIC_EINVAL, "append: NULL store");
     if (n < 0 || (n > 0 && !emb)) return fail(AKASHIC_EINVAL, "append: bad n or emb");
+    if (((uintptr_t)emb & 15u) != 0) return fail(AKASHIC_EINVAL, "append: emb must be 16-byte aligned");
     const bool has_edges = row_ptr != nullptr;
     if (!row_ptr && (col || aff))
         return fail(AKASHIC_EINVAL, "append: col/aff given without row_ptr");
@@ -398,16 +435,30 @@ akashic_status_t akashic_mem_append_chunks(akashic_mem_t *m, const uint16_t *emb
         AK_TRY(m->aff.ensure(grow * 4, true, st));
         AK_TRY(m->w.ensure(grow * 4, true, st));
     }
+    // -- the batch's rows in page order (stable: ID order within a page)
+    DevBuf okeys, ovals, okeys2, ovals2, otmp;
+    const uint32_t *order = nullptr;
+    if (page_of && max_page > 0 && n > 1) {
+        AK_TRY(okeys.ensure((size_t)n * 4));
+        AK_TRY(ovals.ensure((size_t)n * 4));
+        AK_TRY(okeys2.ensure((size_t)n * 4));
+        AK_TRY(ovals2.ensure((size_t)n * 4));
+        AK_TRY(otmp.ensure(radix_tmp_bytes(n) + 4096));
+        CUDA_TRY(cudaMemcpyAsync(okeys.p, page_of, (size_t)n * 4, cudaMemcpyDeviceToDevice, st));
+        CUDA_TRY(launch_iota(ovals.as<uint32_t>(), n, st));
+        bool alt = false;
+        CUDA_TRY(radix_sort_pairs(okeys.as<uint32_t>(), ovals.as<uint32_t>(), okeys2.as<uint32_t>(),
+                                  ovals2.as<uint32_t>(), n, bits_for(max_page), otmp.p, otmp.cap,
+                                  st, &alt));
+        order = alt ? ovals2.as<uint32_t>() : ovals.as<uint32_t>();
+    }
     // -- commit
-    CUDA_TRY(cudaMemcpyAsync(m->emb.as<uint16_t>() + first * m->dim, emb, (size_t)n * m->dim * 2,
-                             cudaMemcpyDeviceToDevice, st));
-    int32_t *pg = m->page_of.as<int32_t>() + first;
+    CUDA_TRY(launch_batch_layout(order, first, n, m->dim, emb, m->emb.as<uint16_t>(), page_of,
+                                 m->next_page, m->per_page, m->page_of.as<int32_t>(),
+                                 m->ext_of.as<int32_t>(), m->row_of.as<int32_t>(), st));
     if (page_of) {
-        CUDA_TRY(cudaMemcpyAsync(pg, page_of, (size_t)n * 4, cudaMemcpyDeviceToDevice, st));
         if (max_page + 1 > m->next_page) m->next_page = max_page + 1;
     } else {
-        k_fill_pages<<<device_sm_count() * 4, 256, 0, st>>>(pg, n, m->next_page, m->per_page);
-        CUDA_TRY(cudaGetLastError());
         m->next_page += ceil_div<int64_t>(n, m->per_page);
     }
     CUDA_TRY(launch_row_norm_max(m->emb.as<uint16_t>() + first * m->dim, n, m->dim,
@@ -457,6 +508,8 @@ akashic_status_t akashic_mem_update_relations(akashic_mem_t *m, int64_t first, i
     ua.reciprocal = reciprocal != 0;
     ua.scale = m->rel_scale;
     ua.status = m->status.as<int>();
+    ua.ext_of = m->ext_of.as<int32_t>();
+    ua.row_of = m->row_of.as<int32_t>();
     int64_t nnz_new = m->nnz + n * M * (reciprocal ? 2 : 1);
     if (nnz_new > 0x7fffffffLL)
         return fail(AKASHIC_ECAPACITY, "update: more than 2^31-1 relation edges");
@@ -538,6 +591,7 @@ akashic_status_t akashic_mem_retrieve(akashic_mem_t *m, const uint16_t *q, int32
         if (eff_hops >= 1) AK_TRY(sc->sa.ensure((size_t)n * bp * 4));
         if (eff_hops >= 2) AK_TRY(sc->sb.ensure((size_t)n * bp * 4));
         if (eff_hops >= 1 && m->n_segs > 0) AK_TRY(sc->partial.ensure((size_t)m->n_segs * bp * 4));
+        if (eff_hops >= 1) AK_TRY(sc->counters.ensure(64));
         const uint16_t *qb = q + (int64_t)off * m->dim;
         {
             PhaseScope ph(m, AKASHIC_PHASE_SCORE, st);
@@ -554,6 +608,7 @@ akashic_status_t akashic_mem_retrieve(akashic_mem_t *m, const uint16_t *q, int32
         if (eff_hops >= 1) {
             PhaseScope ph(m, AKASHIC_PHASE_PROPAGATE, st);
             HopPlan hp;
+            hp.split = m->split;
             hp.in_ptr = m->in_ptr.as<int64_t>();
             hp.in_src = m->in_src.as<int32_t>();
             hp.in_w = m->in_w.as<float>();
@@ -564,18 +619,21 @@ akashic_status_t akashic_mem_retrieve(akashic_mem_t *m, const uint16_t *q, int32
             hp.n_segs = m->n_segs;
             hp.seg_e0 = m->seg_e0.as<int64_t>();
             hp.seg_e1 = m->seg_e1.as<int64_t>();
+            hp.seg_slot = m->seg_slot.as<int32_t>();
             float *bufs[2] = {sc->sa.as<float>(), sc->sb.as<float>()};
             for (int h = 0; h < eff_hops; ++h) {
                 float *out = bufs[h & 1];
                 CUDA_TRY(launch_hop(hp, sc->u.as<float>(), fin, out, bp, alpha,
-                                    sc->partial.as<float>(), st, &ph.launches));
+                                    sc->partial.as<float>(), sc->counters.as<int>(), st,
+                                    &ph.launches));
                 fin = out;
             }
         }
         {
             PhaseScope ph(m, AKASHIC_PHASE_SELECT, st);
             CUDA_TRY(launch_select(sp, fin, n, bp, b, k, sc->cand.as<unsigned long long>(),
-                                   sc->zpart.as<float>(), zrows, m->page_of.as<int32_t>(),
+                                   sc->zpart.as<float>(), zrows, m->ext_of.as<int32_t>(),
+                                   m->row_of.as<int32_t>(), m->page_of.as<int32_t>(),
                                    ids + (int64_t)off * k, scores + (int64_t)off * k,
                                    page_ids ? page_ids + (int64_t)off * k : nullptr,
                                    n_pages ? n_pages + off : nullptr, m->status.as<int>(), st,

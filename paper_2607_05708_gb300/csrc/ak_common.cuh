@@ -78,9 +78,17 @@ cudaError_t launch_row_norm_max(const uint16_t *emb, int64_t n, int dim, float *
 // ------------------------------------------------------------------ graph
 int device_sm_count();
 
-// In-edge rows longer than this are split into segments of this many edges
-// whose partial sums are combined by a fixup pass.
-constexpr int64_t HOP_SEG = 2048;
+// Propagation work plan.  Rows with more than SPLIT_T in-edges (the hubs of
+// a power-law relation graph) are cut into segments of at most SEG_LEN
+// edges that never cross a source window of WIN_ROWS rows; segments are
+// processed window by window so that the source rows they gather stay in L2,
+// and a fixup pass sums each hub's segment partials in order.
+struct SplitParams {
+    int64_t split_t = 256;      // in-degree above which a row is split
+    int64_t seg_len = 512;      // edges per segment at most
+    int64_t win_rows = 16384;   // source window (rows); 16 MB of slab at 256 queries
+};
+constexpr int ROWS_PER_GRAB = 8;     // rows a warp claims at a time (dynamic scheduling)
 
 // Exclusive prefix sum of `in` (n values) into out (n+1 values; out[n] = total).
 cudaError_t scan_exclusive(const int64_t *in, int64_t *out, int64_t n, void *tmp,
@@ -100,19 +108,39 @@ cudaError_t launch_edge_src_check(const int64_t *row_ptr, const int32_t *col, in
                                   cudaStream_t st);
 cudaError_t launch_row_softmax(const int64_t *row_ptr, const float *aff, float *w, int64_t n_rows,
                                cudaStream_t st);
-cudaError_t launch_in_degree(const int32_t *col, int64_t nnz, int64_t *deg, cudaStream_t st);
+// The store keeps chunks in HBM in page order: row r holds chunk ext_of[r],
+// chunk c lives in row row_of[c].  The out-edge CSR stays in chunk IDs; the
+// in-edge transpose used by propagation is in rows.
+cudaError_t launch_in_degree(const int32_t *col, const int32_t *row_of, int64_t nnz, int64_t *deg,
+                             cudaStream_t st);
 cudaError_t launch_iota(uint32_t *v, int64_t n, cudaStream_t st);
-cudaError_t launch_gather_in(const uint32_t *order, const int32_t *src, const float *w,
-                             int32_t *in_src, float *in_w, int64_t nnz, cudaStream_t st);
-cudaError_t launch_split_count(const int64_t *in_ptr, int64_t n, int64_t seg_len, int64_t *nseg,
-                               int64_t *flag, cudaStream_t st);
-cudaError_t launch_split_fill(const int64_t *in_ptr, int64_t n, int64_t seg_len,
+cudaError_t launch_map_keys(const uint32_t *sel, const int32_t *ids, const int32_t *row_of,
+                            uint32_t *keys, int64_t n, cudaStream_t st);
+cudaError_t launch_gather_in(const uint32_t *order, const int32_t *src, const int32_t *row_of,
+                             const float *w, int32_t *in_src, float *in_w, int64_t nnz,
+                             cudaStream_t st);
+cudaError_t launch_batch_layout(const uint32_t *order, int64_t first, int64_t n, int dim,
+                                const uint16_t *emb_in, uint16_t *emb, const int32_t *page_in,
+                                int64_t first_page, int per_page, int32_t *page_row,
+                                int32_t *ext_of, int32_t *row_of, cudaStream_t st);
+// Split plan (see SPLIT_T): per row the number of segments (0 for rows kept
+// whole) and a split flag; then the segments themselves with their window.
+cudaError_t launch_split_count(const SplitParams &sp, const int64_t *in_ptr, const int32_t *in_src,
+                               int64_t n, int64_t *nseg, int64_t *flag, cudaStream_t st);
+cudaError_t launch_split_fill(const SplitParams &sp, const int64_t *in_ptr, const int32_t *in_src,
+                              int64_t n,
                               const int64_t *nseg, const int64_t *slot_off,
                               const int64_t *split_idx, int32_t *split_row, int64_t *split_slot0,
-                              int64_t *seg_e0, int64_t *seg_e1, cudaStream_t st);
+                              int64_t *seg_e0, int64_t *seg_e1, uint32_t *seg_win,
+                              cudaStream_t st);
+// Permute segments into window-major order: dst[i] = src[order[i]], slot[i] = order[i].
+cudaError_t launch_seg_permute(const uint32_t *order, const int64_t *e0, const int64_t *e1,
+                               int64_t n_segs, int64_t *e0s, int64_t *e1s, int32_t *slot,
+                               cudaStream_t st);
 
 // Propagation hop (a2): out[j,:] = u[j,:] + alpha * sum_{i->j} w_ij * in[i,:].
 struct HopPlan {
+    SplitParams split;
     const int64_t *in_ptr;      // n+1
     const int32_t *in_src;      // nnz
     const float *in_w;          // nnz
@@ -122,11 +150,14 @@ struct HopPlan {
     const int32_t *split_row;   // [n_split_rows] row index
     const int64_t *split_slot0; // [n_split_rows+1] first partial slot of each split row
     int64_t n_segs;             // total segments of split rows (= partial slots)
-    const int64_t *seg_e0;      // [n_segs] first edge of segment
+    const int64_t *seg_e0;      // [n_segs] first edge, window-major order
     const int64_t *seg_e1;      // [n_segs] end edge
+    const int32_t *seg_slot;    // [n_segs] partial slot (segments of a row are contiguous)
 };
+// `counters` = 2 device ints, zeroed by the launcher (work queues).
 cudaError_t launch_hop(const HopPlan &p, const float *u, const float *in, float *out, int bp,
-                       float alpha, float *partial, cudaStream_t st, int *launches);
+                       float alpha, float *partial, int *counters, cudaStream_t st,
+                       int *launches);
 
 // ------------------------------------------------------------------ selection
 // Per-CTA top-k candidate lists over the final slab (a3), then the merge
@@ -137,16 +168,19 @@ struct SelectPlan {
     int64_t lists;   // grid * lanes lists per column
 };
 SelectPlan select_plan(int64_t n, int bp, int k, int sm_count);
+// Rows are store rows; keys and outputs carry chunk IDs (ext_of), so ties
+// resolve to the lower chunk ID; page_row is indexed by row (row_of).
 cudaError_t launch_select(const SelectPlan &sp, const float *s, int64_t n, int bp, int b, int k,
                           unsigned long long *cand, const float *zpart, int64_t n_ztiles,
-                          const int32_t *page_of, int64_t *ids, float *scores,
-                          int32_t *page_ids, int32_t *n_pages, int *status, cudaStream_t st,
-                          int *launches);
-// Same selection over signed values (cosines): the k best rows of each of
-// the b columns go to nbr_ids / nbr_cos rows c_base .. c_base+b-1.
+                          const int32_t *ext_of, const int32_t *row_of, const int32_t *page_row,
+                          int64_t *ids, float *scores, int32_t *page_ids, int32_t *n_pages,
+                          int *status, cudaStream_t st, int *launches);
+// Same selection over signed values (cosines) among rows whose chunk ID is
+// below id_limit: the k best of each of the b columns go to nbr_ids /
+// nbr_cos rows c_base .. c_base+b-1.
 cudaError_t launch_select_signed(const SelectPlan &sp, const float *s, int64_t n, int bp, int b,
-                                 int k, unsigned long long *cand, int64_t c_base,
-                                 int32_t *nbr_ids, float *nbr_cos, int *status, cudaStream_t st,
-                                 int *launches);
+                                 int k, unsigned long long *cand, const int32_t *ext_of,
+                                 int64_t id_limit, int64_t c_base, int32_t *nbr_ids,
+                                 float *nbr_cos, int *status, cudaStream_t st, int *launches);
 
 }  // namespace ak

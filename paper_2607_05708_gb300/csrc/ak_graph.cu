@@ -1,5 +1,6 @@
 // Relation graph on the device: prefix sums, a stable LSD radix sort, the
-// in-edge transpose, relation weights, and the propagation hop (a2) that
+// in-edge transpose in store-row space, relation weights, the page-order
+// layout of appended chunks, and the propagation hop (a2) that
 // spreads scores along cross-chunk relations (arXiv 2607.05708, §4.1:
 // related chunks are recovered together).
 #include "ak_common.cuh"
@@ -296,18 +297,37 @@ cudaError_t launch_row_softmax(const int64_t *row_ptr, const float *aff, float *
     return cudaGetLastError();
 }
 
-__global__ void k_in_degree(const int32_t *__restrict__ col, int64_t nnz,
-                            unsigned long long *__restrict__ deg) {
+// In-degree of every store row (targets mapped from chunk IDs to rows).
+__global__ void k_in_degree(const int32_t *__restrict__ col, const int32_t *__restrict__ row_of,
+                            int64_t nnz, unsigned long long *__restrict__ deg) {
     for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < nnz;
          e += (int64_t)gridDim.x * blockDim.x)
-        atomicAdd(&deg[col[e]], 1ull);
+        atomicAdd(&deg[row_of[col[e]]], 1ull);
 }
 
-cudaError_t launch_in_degree(const int32_t *col, int64_t nnz, int64_t *deg, cudaStream_t st) {
+cudaError_t launch_in_degree(const int32_t *col, const int32_t *row_of, int64_t nnz, int64_t *deg,
+                             cudaStream_t st) {
     if (nnz <= 0) return cudaSuccess;
     int grid = (int)(nnz / 256 + 1 < (int64_t)device_sm_count() * 16 ? nnz / 256 + 1
                                                                      : device_sm_count() * 16);
-    k_in_degree<<<grid, 256, 0, st>>>(col, nnz, (unsigned long long *)deg);
+    k_in_degree<<<grid, 256, 0, st>>>(col, row_of, nnz, (unsigned long long *)deg);
+    return cudaGetLastError();
+}
+
+// keys[i] = row_of[ids[sel ? sel[i] : i]]: chunk IDs (of edge sources or
+// targets) mapped to store rows, optionally through a permutation.
+__global__ void k_map_keys(const uint32_t *__restrict__ sel, const int32_t *__restrict__ ids,
+                           const int32_t *__restrict__ row_of, uint32_t *__restrict__ keys,
+                           int64_t n) {
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n;
+         i += (int64_t)gridDim.x * blockDim.x)
+        keys[i] = (uint32_t)row_of[ids[sel ? sel[i] : (uint32_t)i]];
+}
+
+cudaError_t launch_map_keys(const uint32_t *sel, const int32_t *ids, const int32_t *row_of,
+                            uint32_t *keys, int64_t n, cudaStream_t st) {
+    if (n <= 0) return cudaSuccess;
+    k_map_keys<<<device_sm_count() * 8, 256, 0, st>>>(sel, ids, row_of, keys, n);
     return cudaGetLastError();
 }
 
@@ -324,72 +344,163 @@ cudaError_t launch_iota(uint32_t *v, int64_t n, cudaStream_t st) {
 }
 
 __global__ void k_gather_in(const uint32_t *__restrict__ order, const int32_t *__restrict__ src,
-                            const float *__restrict__ w, int32_t *__restrict__ in_src,
-                            float *__restrict__ in_w, int64_t nnz) {
+                            const int32_t *__restrict__ row_of, const float *__restrict__ w,
+                            int32_t *__restrict__ in_src, float *__restrict__ in_w, int64_t nnz) {
     for (int64_t p = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; p < nnz;
          p += (int64_t)gridDim.x * blockDim.x) {
         uint32_t e = order[p];
-        in_src[p] = src[e];
+        in_src[p] = row_of[src[e]];
         in_w[p] = w[e];
     }
 }
 
-cudaError_t launch_gather_in(const uint32_t *order, const int32_t *src, const float *w,
-                             int32_t *in_src, float *in_w, int64_t nnz, cudaStream_t st) {
+cudaError_t launch_gather_in(const uint32_t *order, const int32_t *src, const int32_t *row_of,
+                             const float *w, int32_t *in_src, float *in_w, int64_t nnz,
+                             cudaStream_t st) {
     if (nnz <= 0) return cudaSuccess;
-    k_gather_in<<<device_sm_count() * 8, 256, 0, st>>>(order, src, w, in_src, in_w, nnz);
+    k_gather_in<<<device_sm_count() * 8, 256, 0, st>>>(order, src, row_of, w, in_src, in_w, nnz);
     return cudaGetLastError();
 }
 
-// Rows whose in-degree exceeds seg_len are split into segments of seg_len
-// edges; nseg[j] = that count (0 for rows kept whole), flag[j] = nseg > 0.
-__global__ void k_split_count(const int64_t *__restrict__ in_ptr, int64_t n, int64_t seg_len,
+// Lay out one append batch in page order: row first+i of the store takes
+// chunk first+order[i] (embedding row, page, ID maps).  One warp per row.
+__global__ void k_batch_layout(const uint32_t *__restrict__ order, int64_t first, int64_t n,
+                               int dim, const uint16_t *__restrict__ emb_in,
+                               uint16_t *__restrict__ emb, const int32_t *__restrict__ page_in,
+                               int64_t first_page, int per_page, int32_t *__restrict__ page_row,
+                               int32_t *__restrict__ ext_of, int32_t *__restrict__ row_of) {
+    const int lane = threadIdx.x & 31;
+    int64_t i = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    const int64_t stride = ((int64_t)gridDim.x * blockDim.x) >> 5;
+    const int words = dim / 8;   // 16-byte words per row (dim is a multiple of 64)
+    for (; i < n; i += stride) {
+        const int64_t o = order ? (int64_t)order[i] : i;
+        const uint4 *src = (const uint4 *)(emb_in + o * dim);
+        uint4 *dst = (uint4 *)(emb + (first + i) * dim);
+        for (int t = lane; t < words; t += 32) dst[t] = src[t];
+        if (lane == 0) {
+            ext_of[first + i] = (int32_t)(first + o);
+            row_of[first + o] = (int32_t)(first + i);
+            page_row[first + i] = page_in ? page_in[o] : (int32_t)(first_page + o / per_page);
+        }
+    }
+}
+
+cudaError_t launch_batch_layout(const uint32_t *order, int64_t first, int64_t n, int dim,
+                                const uint16_t *emb_in, uint16_t *emb, const int32_t *page_in,
+                                int64_t first_page, int per_page, int32_t *page_row,
+                                int32_t *ext_of, int32_t *row_of, cudaStream_t st) {
+    if (n <= 0) return cudaSuccess;
+    k_batch_layout<<<device_sm_count() * 8, 256, 0, st>>>(order, first, n, dim, emb_in, emb,
+                                                          page_in, first_page, per_page, page_row,
+                                                          ext_of, row_of);
+    return cudaGetLastError();
+}
+
+// Split plan.  A row with more than SPLIT_T in-edges is cut at every source
+// window boundary (sources are sorted within a row, so the cut points are
+// found by binary search) and then every SEG_LEN edges.
+__device__ __forceinline__ int64_t lower_bound_src(const int32_t *__restrict__ src, int64_t lo,
+                                                   int64_t hi, int64_t key) {
+    while (lo < hi) {
+        const int64_t mid = (lo + hi) >> 1;
+        if ((int64_t)src[mid] < key) lo = mid + 1;
+        else hi = mid;
+    }
+    return lo;
+}
+
+template <bool FILL>
+__device__ __forceinline__ int64_t walk_segments(SplitParams sp, const int32_t *__restrict__ in_src,
+                                                 int64_t a, int64_t b, int64_t slot,
+                                                 int64_t *seg_e0, int64_t *seg_e1,
+                                                 uint32_t *seg_win) {
+    int64_t count = 0, lo = a;
+    while (lo < b) {
+        const int64_t w = (int64_t)in_src[lo] / sp.win_rows;
+        const int64_t hi = lower_bound_src(in_src, lo, b, (w + 1) * sp.win_rows);
+        for (int64_t e = lo; e < hi; e += sp.seg_len) {
+            if (FILL) {
+                seg_e0[slot + count] = e;
+                seg_e1[slot + count] = e + sp.seg_len < hi ? e + sp.seg_len : hi;
+                seg_win[slot + count] = (uint32_t)w;
+            }
+            ++count;
+        }
+        lo = hi;
+    }
+    return count;
+}
+
+__global__ void k_split_count(SplitParams sp, const int64_t *__restrict__ in_ptr,
+                              const int32_t *__restrict__ in_src, int64_t n,
                               int64_t *__restrict__ nseg, int64_t *__restrict__ flag) {
     for (int64_t j = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; j < n;
          j += (int64_t)gridDim.x * blockDim.x) {
-        int64_t d = in_ptr[j + 1] - in_ptr[j];
-        int64_t s = d > seg_len ? ceil_div<int64_t>(d, seg_len) : 0;
+        const int64_t a = in_ptr[j], b = in_ptr[j + 1];
+        const int64_t s = b - a > sp.split_t
+                              ? walk_segments<false>(sp, in_src, a, b, 0, nullptr, nullptr, nullptr)
+                              : 0;
         nseg[j] = s;
         flag[j] = s > 0;
     }
 }
 
-__global__ void k_split_fill(const int64_t *__restrict__ in_ptr, int64_t n, int64_t seg_len,
-                             const int64_t *__restrict__ nseg, const int64_t *__restrict__ slot_off,
+__global__ void k_split_fill(SplitParams sp, const int64_t *__restrict__ in_ptr,
+                             const int32_t *__restrict__ in_src, int64_t n,
+                             const int64_t *__restrict__ nseg,
+                             const int64_t *__restrict__ slot_off,
                              const int64_t *__restrict__ split_idx, int32_t *__restrict__ split_row,
                              int64_t *__restrict__ split_slot0, int64_t *__restrict__ seg_e0,
-                             int64_t *__restrict__ seg_e1) {
+                             int64_t *__restrict__ seg_e1, uint32_t *__restrict__ seg_win) {
     for (int64_t j = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; j < n;
          j += (int64_t)gridDim.x * blockDim.x) {
-        int64_t s = nseg[j];
-        if (s == 0) continue;
-        int64_t idx = split_idx[j];
+        if (nseg[j] == 0) continue;
+        const int64_t idx = split_idx[j];
         split_row[idx] = (int32_t)j;
         split_slot0[idx] = slot_off[j];
-        const int64_t a = in_ptr[j], b = in_ptr[j + 1];
-        for (int64_t t = 0; t < s; ++t) {
-            int64_t e0 = a + t * seg_len;
-            seg_e0[slot_off[j] + t] = e0;
-            seg_e1[slot_off[j] + t] = e0 + seg_len < b ? e0 + seg_len : b;
-        }
+        walk_segments<true>(sp, in_src, in_ptr[j], in_ptr[j + 1], slot_off[j], seg_e0, seg_e1,
+                            seg_win);
     }
 }
 
-cudaError_t launch_split_count(const int64_t *in_ptr, int64_t n, int64_t seg_len, int64_t *nseg,
-                               int64_t *flag, cudaStream_t st) {
+__global__ void k_seg_permute(const uint32_t *__restrict__ order, const int64_t *__restrict__ e0,
+                              const int64_t *__restrict__ e1, int64_t n_segs,
+                              int64_t *__restrict__ e0s, int64_t *__restrict__ e1s,
+                              int32_t *__restrict__ slot) {
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n_segs;
+         i += (int64_t)gridDim.x * blockDim.x) {
+        const uint32_t o = order[i];
+        e0s[i] = e0[o];
+        e1s[i] = e1[o];
+        slot[i] = (int32_t)o;
+    }
+}
+
+cudaError_t launch_split_count(const SplitParams &sp, const int64_t *in_ptr, const int32_t *in_src,
+                               int64_t n, int64_t *nseg, int64_t *flag, cudaStream_t st) {
     if (n <= 0) return cudaSuccess;
-    k_split_count<<<device_sm_count() * 4, 256, 0, st>>>(in_ptr, n, seg_len, nseg, flag);
+    k_split_count<<<device_sm_count() * 4, 256, 0, st>>>(sp, in_ptr, in_src, n, nseg, flag);
     return cudaGetLastError();
 }
 
-cudaError_t launch_split_fill(const int64_t *in_ptr, int64_t n, int64_t seg_len,
-                              const int64_t *nseg, const int64_t *slot_off,
+cudaError_t launch_split_fill(const SplitParams &sp, const int64_t *in_ptr, const int32_t *in_src,
+                              int64_t n, const int64_t *nseg, const int64_t *slot_off,
                               const int64_t *split_idx, int32_t *split_row, int64_t *split_slot0,
-                              int64_t *seg_e0, int64_t *seg_e1, cudaStream_t st) {
+                              int64_t *seg_e0, int64_t *seg_e1, uint32_t *seg_win,
+                              cudaStream_t st) {
     if (n <= 0) return cudaSuccess;
-    k_split_fill<<<device_sm_count() * 4, 256, 0, st>>>(in_ptr, n, seg_len, nseg, slot_off,
+    k_split_fill<<<device_sm_count() * 4, 256, 0, st>>>(sp, in_ptr, in_src, n, nseg, slot_off,
                                                         split_idx, split_row, split_slot0, seg_e0,
-                                                        seg_e1);
+                                                        seg_e1, seg_win);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_seg_permute(const uint32_t *order, const int64_t *e0, const int64_t *e1,
+                               int64_t n_segs, int64_t *e0s, int64_t *e1s, int32_t *slot,
+                               cudaStream_t st) {
+    if (n_segs <= 0) return cudaSuccess;
+    k_seg_permute<<<device_sm_count() * 2, 256, 0, st>>>(order, e0, e1, n_segs, e0s, e1s, slot);
     return cudaGetLastError();
 }
 
@@ -398,8 +509,8 @@ cudaError_t launch_split_fill(const int64_t *in_ptr, int64_t n, int64_t seg_len,
 // in-edge CSR, one warp per destination row.  A row holds BP fp32 values
 // (BP/4 float4).  For BP >= 128 each lane owns BP/128 float4 of the row; for
 // smaller BP the warp splits into 32/(BP/4) lane groups that take
-// alternate edges and are summed at the end.  Rows with more than
-// HOP_SEG in-edges are skipped here and handled by segments + fixup.
+// alternate edges and are summed at the end.  Rows with more than split_t
+// in-edges are skipped here and handled by window segments + fixup.
 template <int BP>
 struct HopShape {
     static constexpr int F = BP / 4;                       // float4 per row
@@ -414,54 +525,62 @@ __device__ __forceinline__ void hop_accumulate(const int32_t *__restrict__ in_sr
                                                int64_t e1, const float4 *__restrict__ in4,
                                                float4 (&acc)[HopShape<BP>::V]) {
     using S = HopShape<BP>;
+    constexpr int UN = 8 / S::V > 0 ? 8 / S::V : 1;   // gathers in flight: UN edges x V float4
     const int lane = threadIdx.x & 31;
     const int g = lane / S::LW, sub = lane % S::LW;
 #pragma unroll
     for (int v = 0; v < S::V; ++v) acc[v] = make_float4(0.f, 0.f, 0.f, 0.f);
+    // the next batch's (source, weight) pairs are loaded while this batch gathers
+    int32_t s_n = 0;
+    float w_n = 0.f;
+    if (e0 + lane < e1) {
+        s_n = in_src[e0 + lane];
+        w_n = in_w[e0 + lane];
+    }
     for (int64_t eb = e0; eb < e1; eb += 32) {
         const int cnt = (int)(e1 - eb < 32 ? e1 - eb : 32);
-        int32_t s_l = 0;
-        float w_l = 0.f;
-        if (lane < cnt) {
-            s_l = in_src[eb + lane];
-            w_l = in_w[eb + lane];
+        const int32_t s_l = s_n;
+        const float w_l = w_n;
+        if (eb + 32 + lane < e1) {
+            s_n = in_src[eb + 32 + lane];
+            w_n = in_w[eb + 32 + lane];
         }
         int t = 0;
-        for (; t + 4 * S::G <= cnt; t += 4 * S::G) {
-            int32_t s[4];
-            float w[4];
+        for (; t + UN * S::G <= cnt; t += UN * S::G) {
+            int32_t sq[UN];
+            float wq[UN];
 #pragma unroll
-            for (int q = 0; q < 4; ++q) {
-                s[q] = __shfl_sync(0xffffffffu, s_l, t + q * S::G + g);
-                w[q] = __shfl_sync(0xffffffffu, w_l, t + q * S::G + g);
+            for (int q = 0; q < UN; ++q) {
+                sq[q] = __shfl_sync(0xffffffffu, s_l, t + q * S::G + g);
+                wq[q] = __shfl_sync(0xffffffffu, w_l, t + q * S::G + g);
             }
-            float4 x[4][S::V];
+            float4 x[UN][S::V];
 #pragma unroll
-            for (int q = 0; q < 4; ++q)
+            for (int q = 0; q < UN; ++q)
 #pragma unroll
-                for (int v = 0; v < S::V; ++v) x[q][v] = in4[(int64_t)s[q] * S::F + sub + 32 * v];
+                for (int v = 0; v < S::V; ++v) x[q][v] = in4[(int64_t)sq[q] * S::F + sub + 32 * v];
 #pragma unroll
-            for (int q = 0; q < 4; ++q)
+            for (int q = 0; q < UN; ++q)
 #pragma unroll
                 for (int v = 0; v < S::V; ++v) {
-                    acc[v].x = fmaf(w[q], x[q][v].x, acc[v].x);
-                    acc[v].y = fmaf(w[q], x[q][v].y, acc[v].y);
-                    acc[v].z = fmaf(w[q], x[q][v].z, acc[v].z);
-                    acc[v].w = fmaf(w[q], x[q][v].w, acc[v].w);
+                    acc[v].x = fmaf(wq[q], x[q][v].x, acc[v].x);
+                    acc[v].y = fmaf(wq[q], x[q][v].y, acc[v].y);
+                    acc[v].z = fmaf(wq[q], x[q][v].z, acc[v].z);
+                    acc[v].w = fmaf(wq[q], x[q][v].w, acc[v].w);
                 }
         }
         for (; t < cnt; t += S::G) {
             const int idx = t + g;
-            int32_t s = __shfl_sync(0xffffffffu, s_l, idx < 32 ? idx : 31);
-            float w = __shfl_sync(0xffffffffu, w_l, idx < 32 ? idx : 31);
+            int32_t sv = __shfl_sync(0xffffffffu, s_l, idx < 32 ? idx : 31);
+            float wv = __shfl_sync(0xffffffffu, w_l, idx < 32 ? idx : 31);
             if (idx < cnt) {
 #pragma unroll
                 for (int v = 0; v < S::V; ++v) {
-                    float4 x = in4[(int64_t)s * S::F + sub + 32 * v];
-                    acc[v].x = fmaf(w, x.x, acc[v].x);
-                    acc[v].y = fmaf(w, x.y, acc[v].y);
-                    acc[v].z = fmaf(w, x.z, acc[v].z);
-                    acc[v].w = fmaf(w, x.w, acc[v].w);
+                    float4 x = in4[(int64_t)sv * S::F + sub + 32 * v];
+                    acc[v].x = fmaf(wv, x.x, acc[v].x);
+                    acc[v].y = fmaf(wv, x.y, acc[v].y);
+                    acc[v].z = fmaf(wv, x.z, acc[v].z);
+                    acc[v].w = fmaf(wv, x.w, acc[v].w);
                 }
             }
         }
@@ -480,57 +599,82 @@ __device__ __forceinline__ void hop_accumulate(const int32_t *__restrict__ in_sr
     }
 }
 
+// Rows kept whole: warps claim ROWS_PER_GRAB consecutive rows at a time from
+// a queue (load balance), read the row pointers of the whole group at once
+// and issue the row's u load before its gathers.
 template <int BP>
-__global__ __launch_bounds__(256) void k_hop_rows(const int64_t *__restrict__ in_ptr,
+__global__ __launch_bounds__(256, 3) void k_hop_rows(const int64_t *__restrict__ in_ptr,
                                                   const int32_t *__restrict__ in_src,
                                                   const float *__restrict__ in_w, int64_t n,
                                                   const float4 *__restrict__ u4,
                                                   const float4 *__restrict__ in4,
-                                                  float4 *__restrict__ out4, float alpha) {
+                                                  float4 *__restrict__ out4, float alpha,
+                                                  int64_t split_t, int *__restrict__ queue) {
     using S = HopShape<BP>;
     const int lane = threadIdx.x & 31;
     const int sub = lane % S::LW;
-    int64_t j = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
-    const int64_t stride = ((int64_t)gridDim.x * blockDim.x) >> 5;
-    for (; j < n; j += stride) {
-        const int64_t e0 = in_ptr[j], e1 = in_ptr[j + 1];
-        if (e1 - e0 > HOP_SEG) continue;
-        float4 acc[S::V];
-        hop_accumulate<BP>(in_src, in_w, e0, e1, in4, acc);
-        if (lane < S::LW) {
+    const int64_t groups = (n + ROWS_PER_GRAB - 1) / ROWS_PER_GRAB;
+    while (true) {
+        int64_t g = 0;
+        if (lane == 0) g = atomicAdd(queue, 1);
+        g = __shfl_sync(0xffffffffu, g, 0);
+        if (g >= groups) break;
+        const int64_t j0 = g * ROWS_PER_GRAB;
+        const int nr = (int)(n - j0 < ROWS_PER_GRAB ? n - j0 : ROWS_PER_GRAB);
+        int64_t p = 0;
+        if (lane <= nr) p = in_ptr[j0 + lane];
+#pragma unroll 1
+        for (int r = 0; r < nr; ++r) {
+            const int64_t e0 = __shfl_sync(0xffffffffu, p, r);
+            const int64_t e1 = __shfl_sync(0xffffffffu, p, r + 1);
+            if (e1 - e0 > split_t) continue;
+            const int64_t j = j0 + r;
+            float4 b[S::V];
+            if (lane < S::LW) {
 #pragma unroll
-            for (int v = 0; v < S::V; ++v) {
-                const int64_t o = j * S::F + sub + 32 * v;
-                float4 b = u4[o];
-                b.x = fmaf(alpha, acc[v].x, b.x);
-                b.y = fmaf(alpha, acc[v].y, b.y);
-                b.z = fmaf(alpha, acc[v].z, b.z);
-                b.w = fmaf(alpha, acc[v].w, b.w);
-                out4[o] = b;
+                for (int v = 0; v < S::V; ++v) b[v] = u4[j * S::F + sub + 32 * v];
+            }
+            float4 acc[S::V];
+            hop_accumulate<BP>(in_src, in_w, e0, e1, in4, acc);
+            if (lane < S::LW) {
+#pragma unroll
+                for (int v = 0; v < S::V; ++v) {
+                    b[v].x = fmaf(alpha, acc[v].x, b[v].x);
+                    b[v].y = fmaf(alpha, acc[v].y, b[v].y);
+                    b[v].z = fmaf(alpha, acc[v].z, b[v].z);
+                    b[v].w = fmaf(alpha, acc[v].w, b[v].w);
+                    out4[j * S::F + sub + 32 * v] = b[v];
+                }
             }
         }
     }
 }
 
+// Segments of split rows, claimed one at a time in window-major order.
 template <int BP>
-__global__ __launch_bounds__(256) void k_hop_segs(const int64_t *__restrict__ seg_e0,
+__global__ __launch_bounds__(256, 3) void k_hop_segs(const int64_t *__restrict__ seg_e0,
                                                   const int64_t *__restrict__ seg_e1,
+                                                  const int32_t *__restrict__ seg_slot,
                                                   int64_t n_segs,
                                                   const int32_t *__restrict__ in_src,
                                                   const float *__restrict__ in_w,
                                                   const float4 *__restrict__ in4,
-                                                  float4 *__restrict__ part4) {
+                                                  float4 *__restrict__ part4,
+                                                  int *__restrict__ queue) {
     using S = HopShape<BP>;
     const int lane = threadIdx.x & 31;
     const int sub = lane % S::LW;
-    int64_t s = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
-    const int64_t stride = ((int64_t)gridDim.x * blockDim.x) >> 5;
-    for (; s < n_segs; s += stride) {
+    while (true) {
+        int64_t s = 0;
+        if (lane == 0) s = atomicAdd(queue, 1);
+        s = __shfl_sync(0xffffffffu, s, 0);
+        if (s >= n_segs) break;
         float4 acc[S::V];
         hop_accumulate<BP>(in_src, in_w, seg_e0[s], seg_e1[s], in4, acc);
+        const int64_t slot = seg_slot[s];
         if (lane < S::LW) {
 #pragma unroll
-            for (int v = 0; v < S::V; ++v) part4[s * S::F + sub + 32 * v] = acc[v];
+            for (int v = 0; v < S::V; ++v) part4[slot * S::F + sub + 32 * v] = acc[v];
         }
     }
 }
@@ -567,39 +711,45 @@ __global__ __launch_bounds__(256) void k_hop_fixup(const int32_t *__restrict__ s
 
 template <int BP>
 static cudaError_t hop_bp(const HopPlan &p, const float *u, const float *in, float *out,
-                          float alpha, float *partial, cudaStream_t st, int *launches) {
+                          float alpha, float *partial, int *counters, cudaStream_t st,
+                          int *launches) {
     const int sms = device_sm_count();
-    const int64_t warps_rows = p.n;
-    int grid = (int)(ceil_div<int64_t>(warps_rows, 8) < (int64_t)sms * 8 ? ceil_div<int64_t>(warps_rows, 8)
-                                                                         : (int64_t)sms * 8);
-    if (grid < 1) grid = 1;
+    cudaError_t e = cudaMemsetAsync(counters, 0, 2 * sizeof(int), st);
+    if (e != cudaSuccess) return e;
+    if (p.n_segs > 0) {
+        const int64_t want = ceil_div<int64_t>(p.n_segs, 8);
+        const int g2 = (int)(want < (int64_t)sms * 3 ? want : (int64_t)sms * 3);
+        k_hop_segs<BP><<<g2, 256, 0, st>>>(p.seg_e0, p.seg_e1, p.seg_slot, p.n_segs, p.in_src,
+                                           p.in_w, (const float4 *)in, (float4 *)partial,
+                                           counters + 1);
+        e = cudaGetLastError();
+        if (e != cudaSuccess) return e;
+        if (launches) *launches += 1;
+    }
+    const int64_t want = ceil_div<int64_t>(ceil_div<int64_t>(p.n, ROWS_PER_GRAB), 8);
+    const int grid = (int)(want < (int64_t)sms * 3 ? (want < 1 ? 1 : want) : (int64_t)sms * 3);
     k_hop_rows<BP><<<grid, 256, 0, st>>>(p.in_ptr, p.in_src, p.in_w, p.n, (const float4 *)u,
-                                         (const float4 *)in, (float4 *)out, alpha);
-    cudaError_t e = cudaGetLastError();
+                                         (const float4 *)in, (float4 *)out, alpha,
+                                         p.split.split_t, counters);
+    e = cudaGetLastError();
     if (launches) *launches += 1;
     if (e != cudaSuccess || p.n_split_rows == 0) return e;
-    int g2 = (int)(ceil_div<int64_t>(p.n_segs, 8) < (int64_t)sms * 8 ? ceil_div<int64_t>(p.n_segs, 8)
-                                                                    : (int64_t)sms * 8);
-    k_hop_segs<BP><<<g2, 256, 0, st>>>(p.seg_e0, p.seg_e1, p.n_segs, p.in_src, p.in_w,
-                                       (const float4 *)in, (float4 *)partial);
-    e = cudaGetLastError();
-    if (e != cudaSuccess) return e;
-    int g3 = (int)ceil_div<int64_t>(p.n_split_rows, 8);
+    const int g3 = (int)ceil_div<int64_t>(p.n_split_rows, 8);
     k_hop_fixup<BP><<<g3, 256, 0, st>>>(p.split_row, p.split_slot0, p.n_split_rows,
                                         (const float4 *)partial, (const float4 *)u, (float4 *)out,
                                         alpha);
-    if (launches) *launches += 2;
+    if (launches) *launches += 1;
     return cudaGetLastError();
 }
 
 cudaError_t launch_hop(const HopPlan &p, const float *u, const float *in, float *out, int bp,
-                       float alpha, float *partial, cudaStream_t st, int *launches) {
+                       float alpha, float *partial, int *counters, cudaStream_t st,
+                       int *launches) {
     switch (bp) {
-    case 16: return hop_bp<16>(p, u, in, out, alpha, partial, st, launches);
-    case 32: return hop_bp<32>(p, u, in, out, alpha, partial, st, launches);
-    case 64: return hop_bp<64>(p, u, in, out, alpha, partial, st, launches);
-    case 128: return hop_bp<128>(p, u, in, out, alpha, partial, st, launches);
-    case 256: return hop_bp<256>(p, u, in, out, alpha, partial, st, launches);
+    case 32: return hop_bp<32>(p, u, in, out, alpha, partial, counters, st, launches);
+    case 64: return hop_bp<64>(p, u, in, out, alpha, partial, counters, st, launches);
+    case 128: return hop_bp<128>(p, u, in, out, alpha, partial, counters, st, launches);
+    case 256: return hop_bp<256>(p, u, in, out, alpha, partial, counters, st, launches);
     default: return cudaErrorInvalidValue;
     }
 }

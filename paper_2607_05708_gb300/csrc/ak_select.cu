@@ -29,7 +29,7 @@ __device__ __forceinline__ float sel_value(unsigned long long key) {
 template <bool SIGNED>
 __global__ __launch_bounds__(SEL_THREADS) void k_topk_candidates(
     const float *__restrict__ s, int64_t n, int bp, int lanes, int k, int64_t rows_per_cta,
-    unsigned long long *__restrict__ cand) {
+    const int32_t *__restrict__ ext_of, int64_t id_limit, unsigned long long *__restrict__ cand) {
     extern __shared__ unsigned long long lists[];   // [k][SEL_THREADS]
     const int tid = threadIdx.x;
     const int c = tid % bp, r = tid / bp;
@@ -39,17 +39,31 @@ __global__ __launch_bounds__(SEL_THREADS) void k_topk_candidates(
     if (active) {
         const int64_t r0 = (int64_t)blockIdx.x * rows_per_cta;
         const int64_t r1 = r0 + rows_per_cta < n ? r0 + rows_per_cta : n;
-        for (int64_t j = r0 + r; j < r1; j += lanes) {
-            const float v = s[j * bp + c];
-            const unsigned long long key = sel_key<SIGNED>(v, (uint32_t)j);
-            if (key > kth) {
-                int i = k - 1;
-                while (i > 0 && lists[(i - 1) * SEL_THREADS + tid] < key) {
-                    lists[i * SEL_THREADS + tid] = lists[(i - 1) * SEL_THREADS + tid];
-                    --i;
+        constexpr int U = 8;   // rows in flight per thread
+        for (int64_t j0 = r0 + r; j0 < r1; j0 += (int64_t)U * lanes) {
+            float v[U];
+            int32_t id[U];
+#pragma unroll
+            for (int q = 0; q < U; ++q) {
+                const int64_t j = j0 + (int64_t)q * lanes;
+                v[q] = j < r1 ? s[j * bp + c] : 0.f;
+                id[q] = j < r1 ? ext_of[j] : 0;
+            }
+#pragma unroll
+            for (int q = 0; q < U; ++q) {
+                const int64_t j = j0 + (int64_t)q * lanes;
+                if (j >= r1) break;
+                if ((int64_t)id[q] >= id_limit) continue;
+                const unsigned long long key = sel_key<SIGNED>(v[q], (uint32_t)id[q]);
+                if (key > kth) {
+                    int i = k - 1;
+                    while (i > 0 && lists[(i - 1) * SEL_THREADS + tid] < key) {
+                        lists[i * SEL_THREADS + tid] = lists[(i - 1) * SEL_THREADS + tid];
+                        --i;
+                    }
+                    lists[i * SEL_THREADS + tid] = key;
+                    kth = lists[(k - 1) * SEL_THREADS + tid];
                 }
-                lists[i * SEL_THREADS + tid] = key;
-                kth = lists[(k - 1) * SEL_THREADS + tid];
             }
         }
         const int64_t list = (int64_t)blockIdx.x * lanes + r;
@@ -117,9 +131,9 @@ __device__ void radix_select_column(const unsigned long long *__restrict__ cand,
 // partials, resolved to pages, and their distinct pages counted.
 __global__ __launch_bounds__(SEL_THREADS) void k_topk_merge(
     const unsigned long long *__restrict__ cand, int64_t lists, int bp, int k,
-    const float *__restrict__ zpart, int64_t n_ztiles, const int32_t *__restrict__ page_of,
-    int64_t *__restrict__ ids, float *__restrict__ scores, int32_t *__restrict__ page_ids,
-    int32_t *__restrict__ n_pages, int *status) {
+    const float *__restrict__ zpart, int64_t n_ztiles, const int32_t *__restrict__ row_of,
+    const int32_t *__restrict__ page_row, int64_t *__restrict__ ids, float *__restrict__ scores,
+    int32_t *__restrict__ page_ids, int32_t *__restrict__ n_pages, int *status) {
     __shared__ int hist[256];
     __shared__ unsigned long long s_prefix;
     __shared__ int s_remaining;
@@ -146,7 +160,7 @@ __global__ __launch_bounds__(SEL_THREADS) void k_topk_merge(
         const int64_t o = (int64_t)c * k + rank;
         ids[o] = (int64_t)id;
         scores[o] = (float)((double)sel_value<false>(key) / zsum);
-        const int32_t p = page_of ? page_of[id] : 0;
+        const int32_t p = page_row ? page_row[row_of[id]] : 0;
         pg[rank] = p;
         if (page_ids) page_ids[o] = p;
     }
@@ -201,9 +215,9 @@ SelectPlan select_plan(int64_t n, int bp, int k, int sm_count) {
 
 cudaError_t launch_select(const SelectPlan &sp, const float *s, int64_t n, int bp, int b, int k,
                           unsigned long long *cand, const float *zpart, int64_t n_ztiles,
-                          const int32_t *page_of, int64_t *ids, float *scores,
-                          int32_t *page_ids, int32_t *n_pages, int *status, cudaStream_t st,
-                          int *launches) {
+                          const int32_t *ext_of, const int32_t *row_of, const int32_t *page_row,
+                          int64_t *ids, float *scores, int32_t *page_ids, int32_t *n_pages,
+                          int *status, cudaStream_t st, int *launches) {
     const size_t smem = (size_t)k * SEL_THREADS * sizeof(unsigned long long);
     static bool attr_set[64] = {false};
     int dev = 0;
@@ -219,20 +233,20 @@ cudaError_t launch_select(const SelectPlan &sp, const float *s, int64_t n, int b
         attr_set[dev] = true;
     }
     const int64_t rows_per_cta = ceil_div<int64_t>(n, sp.grid);
-    k_topk_candidates<false><<<sp.grid, SEL_THREADS, smem, st>>>(s, n, bp, sp.lanes, k,
-                                                                 rows_per_cta, cand);
+    k_topk_candidates<false><<<sp.grid, SEL_THREADS, smem, st>>>(
+        s, n, bp, sp.lanes, k, rows_per_cta, ext_of, (int64_t)1 << 40, cand);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
-    k_topk_merge<<<b, SEL_THREADS, 0, st>>>(cand, sp.lists, bp, k, zpart, n_ztiles, page_of, ids,
-                                            scores, page_ids, n_pages, status);
+    k_topk_merge<<<b, SEL_THREADS, 0, st>>>(cand, sp.lists, bp, k, zpart, n_ztiles, row_of,
+                                            page_row, ids, scores, page_ids, n_pages, status);
     if (launches) *launches += 2;
     return cudaGetLastError();
 }
 
 cudaError_t launch_select_signed(const SelectPlan &sp, const float *s, int64_t n, int bp, int b,
-                                 int k, unsigned long long *cand, int64_t c_base,
-                                 int32_t *nbr_ids, float *nbr_cos, int *status, cudaStream_t st,
-                                 int *launches) {
+                                 int k, unsigned long long *cand, const int32_t *ext_of,
+                                 int64_t id_limit, int64_t c_base, int32_t *nbr_ids,
+                                 float *nbr_cos, int *status, cudaStream_t st, int *launches) {
     const size_t smem = (size_t)k * SEL_THREADS * sizeof(unsigned long long);
     cudaError_t e = cudaFuncSetAttribute(k_topk_candidates<true>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -240,7 +254,8 @@ cudaError_t launch_select_signed(const SelectPlan &sp, const float *s, int64_t n
     if (e != cudaSuccess) return e;
     const int64_t rows_per_cta = ceil_div<int64_t>(n, sp.grid);
     k_topk_candidates<true><<<sp.grid, SEL_THREADS, smem, st>>>(s, n, bp, sp.lanes, k,
-                                                                rows_per_cta, cand);
+                                                                rows_per_cta, ext_of, id_limit,
+                                                                cand);
     e = cudaGetLastError();
     if (e != cudaSuccess) return e;
     k_topm_merge<<<b, SEL_THREADS, 0, st>>>(cand, sp.lists, bp, k, c_base, nbr_ids, nbr_cos,

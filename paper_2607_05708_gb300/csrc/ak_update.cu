@@ -7,19 +7,22 @@
 
 namespace ak {
 
-// Copy rows [first+off, first+off+b) of emb into a zero-padded bp-row block.
-__global__ void k_pad_rows(const uint16_t *__restrict__ src, int b, int bp, int dim,
-                           uint16_t *__restrict__ dst) {
+// Gather the embeddings of chunks c0 .. c0+b-1 (rows row_of[c]) into a
+// zero-padded bp-row block.
+__global__ void k_gather_rows(const uint16_t *__restrict__ emb, const int32_t *__restrict__ row_of,
+                              int64_t c0, int b, int bp, int dim, uint16_t *__restrict__ dst) {
     const int64_t total = (int64_t)bp * dim;
     for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < total;
          i += (int64_t)gridDim.x * blockDim.x) {
-        const int64_t r = i / dim;
-        dst[i] = r < b ? src[i] : (uint16_t)0;
+        const int64_t r = i / dim, t = i % dim;
+        dst[i] = r < b ? emb[(int64_t)row_of[c0 + r] * dim + t] : (uint16_t)0;
     }
 }
 
 akashic_status_t relate_top_m(const UpdateArgs &a, cudaStream_t st, int *launches) {
-    const int64_t n_old = a.first;
+    // every row of the store is scored; rows holding chunks >= first are
+    // masked in the selection (rows are in page order, not ID order)
+    const int64_t n_old = a.n_rows;
     int bp_max = 32;
     while (bp_max < 256 && bp_max < a.n_new) bp_max <<= 1;
     uint16_t *qp = nullptr;
@@ -48,15 +51,15 @@ akashic_status_t relate_top_m(const UpdateArgs &a, cudaStream_t st, int *launche
         const int b = (int)(a.n_new - off < 256 ? a.n_new - off : 256);
         int bp = 32;
         while (bp < b) bp <<= 1;
-        k_pad_rows<<<device_sm_count(), 256, 0, st>>>(a.emb + (a.first + off) * a.dim, b, bp, a.dim,
-                                                       qp);
+        k_gather_rows<<<device_sm_count(), 256, 0, st>>>(a.emb, a.row_of, a.first + off, b, bp,
+                                                          a.dim, qp);
         e = cudaGetLastError();
         if (e == cudaSuccess)
             e = launch_dots(a.emb, n_old, a.dim, qp, bp, dots, a.status, st, launches);
         const SelectPlan sp = select_plan(n_old, bp, a.M, device_sm_count());
         if (e == cudaSuccess)
-            e = launch_select_signed(sp, dots, n_old, bp, b, a.M, cand, off, a.nbr_ids, a.nbr_cos,
-                                     a.status, st, launches);
+            e = launch_select_signed(sp, dots, n_old, bp, b, a.M, cand, a.ext_of, a.first, off,
+                                     a.nbr_ids, a.nbr_cos, a.status, st, launches);
         if (e != cudaSuccess) rc = AKASHIC_ECUDA;
         if (launches) *launches += 1;
     }

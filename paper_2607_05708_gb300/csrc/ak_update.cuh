@@ -6,7 +6,9 @@
 namespace ak {
 
 struct UpdateArgs {
-    const uint16_t *emb;   // store embeddings (n_rows x dim)
+    const uint16_t *emb;   // store embeddings (n_rows x dim), rows in page order
+    const int32_t *ext_of; // chunk ID of each row
+    const int32_t *row_of; // row of each chunk ID
     int dim;
     int64_t n_rows;        // chunks in the store
     int64_t first;         // first new chunk; prior chunks are [0, first)
