@@ -587,7 +587,7 @@ akashic_status_t akashic_mem_retrieve(akashic_mem_t *m, const uint16_t *q, int32
         AK_TRY(sc->shift.ensure((size_t)bp * 4));
         AK_TRY(sc->u.ensure((size_t)n * bp * 4));
         AK_TRY(sc->zpart.ensure((size_t)tiles * bp * 4));
-        AK_TRY(sc->cand.ensure((size_t)sp.lists * bp * k * 8));
+        AK_TRY(sc->cand.ensure((size_t)sp.words * 8));
         if (eff_hops >= 1) AK_TRY(sc->sa.ensure((size_t)n * bp * 4));
         if (eff_hops >= 2) AK_TRY(sc->sb.ensure((size_t)n * bp * 4));
         if (eff_hops >= 1 && m->n_segs > 0) AK_TRY(sc->partial.ensure((size_t)m->n_segs * bp * 4));
@@ -631,7 +631,7 @@ akashic_status_t akashic_mem_retrieve(akashic_mem_t *m, const uint16_t *q, int32
         }
         {
             PhaseScope ph(m, AKASHIC_PHASE_SELECT, st);
-            CUDA_TRY(launch_select(sp, fin, n, bp, b, k, sc->cand.as<unsigned long long>(),
+            CUDA_TRY(launch_select(sp, fin, b, sc->cand.as<unsigned long long>(),
                                    sc->zpart.as<float>(), zrows, m->ext_of.as<int32_t>(),
                                    m->row_of.as<int32_t>(), m->page_of.as<int32_t>(),
                                    ids + (int64_t)off * k, scores + (int64_t)off * k,

@@ -160,27 +160,35 @@ cudaError_t launch_hop(const HopPlan &p, const float *u, const float *in, float 
                        int *launches);
 
 // ------------------------------------------------------------------ selection
-// Per-CTA top-k candidate lists over the final slab (a3), then the merge
-// with normalisation by Z (a1), page resolve and distinct count (a4).
+// Top-k of every column of a slab (a3): bound from a row sample, filter
+// pass, merge (see ak_select.cu).  The workspace holds sp.words 64-bit words.
 struct SelectPlan {
-    int grid;        // CTAs of the candidate kernel
-    int lanes;       // row lanes per CTA (threads = lanes * bp)
-    int64_t lists;   // grid * lanes lists per column
+    int64_t n;          // rows
+    int bp, k;
+    int64_t stride;     // sample every stride-th row
+    int64_t n_sample;
+    int grid;           // CTAs of the sample pass
+    int lanes;          // row lanes per CTA (threads = lanes * bp)
+    int64_t lists;      // grid * lanes heaps per column
+    int64_t cap;        // buffer capacity per column
+    int64_t off_bound, off_cnt, off_buf, words;
 };
 SelectPlan select_plan(int64_t n, int bp, int k, int sm_count);
-// Rows are store rows; keys and outputs carry chunk IDs (ext_of), so ties
-// resolve to the lower chunk ID; page_row is indexed by row (row_of).
-cudaError_t launch_select(const SelectPlan &sp, const float *s, int64_t n, int bp, int b, int k,
-                          unsigned long long *cand, const float *zpart, int64_t n_ztiles,
-                          const int32_t *ext_of, const int32_t *row_of, const int32_t *page_row,
-                          int64_t *ids, float *scores, int32_t *page_ids, int32_t *n_pages,
-                          int *status, cudaStream_t st, int *launches);
+
+// Retrieval: rows are store rows; keys and outputs carry chunk IDs
+// (ext_of), so ties resolve to the lower chunk ID; page_row is indexed by
+// row (row_of).  Scores are divided by Z = sum of zpart's first n_ztiles rows.
+cudaError_t launch_select(const SelectPlan &sp, const float *s, int b, unsigned long long *ws,
+                          const float *zpart, int64_t n_ztiles, const int32_t *ext_of,
+                          const int32_t *row_of, const int32_t *page_row, int64_t *ids,
+                          float *scores, int32_t *page_ids, int32_t *n_pages, int *status,
+                          cudaStream_t st, int *launches);
 // Same selection over signed values (cosines) among rows whose chunk ID is
 // below id_limit: the k best of each of the b columns go to nbr_ids /
 // nbr_cos rows c_base .. c_base+b-1.
-cudaError_t launch_select_signed(const SelectPlan &sp, const float *s, int64_t n, int bp, int b,
-                                 int k, unsigned long long *cand, const int32_t *ext_of,
-                                 int64_t id_limit, int64_t c_base, int32_t *nbr_ids,
-                                 float *nbr_cos, int *status, cudaStream_t st, int *launches);
+cudaError_t launch_select_signed(const SelectPlan &sp, const float *s, int b,
+                                 unsigned long long *ws, const int32_t *ext_of, int64_t id_limit,
+                                 int64_t c_base, int32_t *nbr_ids, float *nbr_cos, int *status,
+                                 cudaStream_t st, int *launches);
 
 }  // namespace ak

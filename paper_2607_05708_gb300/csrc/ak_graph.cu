@@ -679,6 +679,9 @@ __global__ __launch_bounds__(256, 3) void k_hop_segs(const int64_t *__restrict__
     }
 }
 
+// Split rows: out = u + alpha * (sum of the row's segment partials, in slot
+// order).  One warp per row; each lane keeps 8 independent partial loads in
+// flight per float4 column it owns.
 template <int BP>
 __global__ __launch_bounds__(256) void k_hop_fixup(const int32_t *__restrict__ split_row,
                                                    const int64_t *__restrict__ split_slot0,
@@ -687,6 +690,7 @@ __global__ __launch_bounds__(256) void k_hop_fixup(const int32_t *__restrict__ s
                                                    const float4 *__restrict__ u4,
                                                    float4 *__restrict__ out4, float alpha) {
     constexpr int F = BP / 4;
+    constexpr int P = 8;
     int64_t r = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
     const int64_t stride = ((int64_t)gridDim.x * blockDim.x) >> 5;
     const int lane = threadIdx.x & 31;
@@ -695,8 +699,18 @@ __global__ __launch_bounds__(256) void k_hop_fixup(const int32_t *__restrict__ s
         const int64_t a = split_slot0[r], b = split_slot0[r + 1];
         for (int f = lane; f < F; f += 32) {
             float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-            for (int64_t s = a; s < b; ++s) {
-                float4 x = part4[s * F + f];
+            int64_t s = a;
+            for (; s + P <= b; s += P) {
+                float4 x[P];
+#pragma unroll
+                for (int q = 0; q < P; ++q) x[q] = part4[(s + q) * F + f];
+#pragma unroll
+                for (int q = 0; q < P; ++q) {
+                    acc.x += x[q].x; acc.y += x[q].y; acc.z += x[q].z; acc.w += x[q].w;
+                }
+            }
+            for (; s < b; ++s) {
+                const float4 x = part4[s * F + f];
                 acc.x += x.x; acc.y += x.y; acc.z += x.z; acc.w += x.w;
             }
             float4 o = u4[j * F + f];

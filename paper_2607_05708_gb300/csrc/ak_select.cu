@@ -1,12 +1,25 @@
 // Top-k selection (a3) with score normalisation by Z (a1) and the page
 // resolve + distinct-page count (a4): the top-p selection and FetchByID of
 // query-aware retrieval (arXiv 2607.05708, §4.1, Algorithm 1) and the
-// locality gap |P(R_t)| (§3.2).
+// locality gap |P(R_t)| (§3.2).  The same machinery, on signed keys, selects
+// the top-M prior chunks of the relation update.
+//
+// Three passes per batch of queries (columns of the score slab):
+//   bound   the k-th largest key of every column over a strided sample of
+//           the rows (per-thread heaps + radix-select merge).  A subset's
+//           k-th largest value never exceeds the whole column's, so it is a
+//           safe filter;
+//   filter  one streaming pass over the slab (warp per row, coalesced
+//           float4 loads) appending every key >= bound to a per-column
+//           buffer;
+//   merge   per column, an exact radix select of the k best buffered keys,
+//           or of the whole column if the buffer overflowed.
 #include "ak_common.cuh"
 
 namespace ak {
 
 constexpr int SEL_THREADS = 256;
+constexpr int SEL_STAGE = 4096;   // keys a merge CTA stages in shared memory
 
 // SIGNED=false: non-negative scores (retrieval); SIGNED=true: any finite
 // value (cosines of the relation update).  Either way a larger key is a
@@ -22,65 +35,41 @@ __device__ __forceinline__ float sel_value(unsigned long long key) {
     return SIGNED ? unordered_bits(hi) : __uint_as_float(hi);
 }
 
-// Candidate pass.  Thread (r, c) of CTA g scans rows g*rows_per_cta + r,
-// + lanes, ... for query column c and keeps its k best keys in a sorted
-// list in shared memory (slot-major, so a warp's accesses are contiguous).
-// Reads of a row by the CTA's threads are contiguous, hence coalesced.
-template <bool SIGNED>
-__global__ __launch_bounds__(SEL_THREADS) void k_topk_candidates(
-    const float *__restrict__ s, int64_t n, int bp, int lanes, int k, int64_t rows_per_cta,
-    const int32_t *__restrict__ ext_of, int64_t id_limit, unsigned long long *__restrict__ cand) {
-    extern __shared__ unsigned long long lists[];   // [k][SEL_THREADS]
-    const int tid = threadIdx.x;
-    const int c = tid % bp, r = tid / bp;
-    const bool active = r < lanes;
-    for (int i = 0; i < k; ++i) lists[i * SEL_THREADS + tid] = 0ull;
-    unsigned long long kth = 0ull;
-    if (active) {
-        const int64_t r0 = (int64_t)blockIdx.x * rows_per_cta;
-        const int64_t r1 = r0 + rows_per_cta < n ? r0 + rows_per_cta : n;
-        constexpr int U = 8;   // rows in flight per thread
-        for (int64_t j0 = r0 + r; j0 < r1; j0 += (int64_t)U * lanes) {
-            float v[U];
-            int32_t id[U];
-#pragma unroll
-            for (int q = 0; q < U; ++q) {
-                const int64_t j = j0 + (int64_t)q * lanes;
-                v[q] = j < r1 ? s[j * bp + c] : 0.f;
-                id[q] = j < r1 ? ext_of[j] : 0;
-            }
-#pragma unroll
-            for (int q = 0; q < U; ++q) {
-                const int64_t j = j0 + (int64_t)q * lanes;
-                if (j >= r1) break;
-                if ((int64_t)id[q] >= id_limit) continue;
-                const unsigned long long key = sel_key<SIGNED>(v[q], (uint32_t)id[q]);
-                if (key > kth) {
-                    int i = k - 1;
-                    while (i > 0 && lists[(i - 1) * SEL_THREADS + tid] < key) {
-                        lists[i * SEL_THREADS + tid] = lists[(i - 1) * SEL_THREADS + tid];
-                        --i;
-                    }
-                    lists[i * SEL_THREADS + tid] = key;
-                    kth = lists[(k - 1) * SEL_THREADS + tid];
-                }
-            }
-        }
-        const int64_t list = (int64_t)blockIdx.x * lanes + r;
-        unsigned long long *dst = cand + (list * bp + c) * k;
-        for (int i = 0; i < k; ++i) dst[i] = lists[i * SEL_THREADS + tid];
-    }
+// ------------------------------------------------------------------ plan
+SelectPlan select_plan(int64_t n, int bp, int k, int sm_count) {
+    SelectPlan sp;
+    sp.n = n;
+    sp.bp = bp;
+    sp.k = k;
+    // sample every stride-th row, at least 64 k rows (all rows of a small store)
+    int64_t stride = n / ((int64_t)64 * k);
+    stride = stride < 1 ? 1 : (stride > 32 ? 32 : stride);
+    sp.stride = stride;
+    sp.n_sample = ceil_div<int64_t>(n, stride);
+    sp.lanes = SEL_THREADS / bp > 0 ? SEL_THREADS / bp : 1;
+    int64_t want = ceil_div<int64_t>(sp.n_sample, (int64_t)sp.lanes * 4 * k);
+    int64_t capg = 4 * (int64_t)sm_count;
+    sp.grid = (int)(want < 1 ? 1 : (want > capg ? capg : want));
+    sp.lists = (int64_t)sp.grid * sp.lanes;
+    int64_t cap = 4 * (int64_t)k * stride;
+    sp.cap = cap < 8192 ? 8192 : cap;
+    sp.off_bound = sp.lists * bp * k;
+    sp.off_cnt = sp.off_bound + bp;
+    sp.off_buf = sp.off_cnt + bp;
+    sp.words = sp.off_buf + (int64_t)bp * sp.cap;
+    return sp;
 }
 
-// Exact k-th largest key of column c among all candidate lists by an
-// MSB-first radix select (8 bits a pass); the k winners are left in win[]
-// (unordered) and their count in *win_n.  Keys are unique (each row is seen
-// by one list only) and lists pad with key 0, below every real key.
-__device__ void radix_select_column(const unsigned long long *__restrict__ cand, int64_t lists,
-                                    int bp, int k, int c, unsigned long long *win, int *win_n,
-                                    int *hist, unsigned long long *s_prefix, int *s_remaining) {
-    const int tid = threadIdx.x;
-    const int64_t total = lists * (int64_t)k;
+// ------------------------------------------------------------------ radix select
+// Exact k-th largest of `total` keys given by key_at(i), MSB-first 8 bits a
+// pass with per-warp histograms; the (at most 64) keys >= it are left in
+// win[] (unordered) and their count in *win_n.  Keys are unique apart from
+// the padding key 0, which is below every real key and never selected.
+template <typename KeyAt>
+__device__ void radix_select(int64_t total, int k, KeyAt key_at, unsigned long long *win,
+                             int *win_n, int *hist, unsigned long long *s_prefix,
+                             int *s_remaining) {
+    const int tid = threadIdx.x, warp = tid >> 5;
     if (tid == 0) {
         *s_prefix = 0ull;
         *s_remaining = k;
@@ -90,13 +79,18 @@ __device__ void radix_select_column(const unsigned long long *__restrict__ cand,
     unsigned long long pmask = 0ull;
     for (int pass = 0; pass < 8; ++pass) {
         const int sh = 56 - 8 * pass;
-        hist[tid] = 0;
+        for (int w = 0; w < SEL_THREADS / 32; ++w) hist[w * 256 + tid] = 0;
         __syncthreads();
         const unsigned long long prefix = *s_prefix;
         for (int64_t i = tid; i < total; i += SEL_THREADS) {
-            const int64_t l = i / k, slot = i % k;
-            const unsigned long long key = cand[(l * bp + c) * k + slot];
-            if ((key & pmask) == prefix) atomicAdd(&hist[(key >> sh) & 0xff], 1);
+            const unsigned long long key = key_at(i);
+            if ((key & pmask) == prefix) atomicAdd(&hist[warp * 256 + ((key >> sh) & 0xff)], 1);
+        }
+        __syncthreads();
+        {
+            int sum = 0;
+            for (int w = 0; w < SEL_THREADS / 32; ++w) sum += hist[w * 256 + tid];
+            hist[tid] = sum;   // warp 0's row now holds the totals
         }
         __syncthreads();
         if (tid == 0) {
@@ -116,29 +110,202 @@ __device__ void radix_select_column(const unsigned long long *__restrict__ cand,
     }
     const unsigned long long kth = *s_prefix;
     for (int64_t i = tid; i < total; i += SEL_THREADS) {
-        const int64_t l = i / k, slot = i % k;
-        const unsigned long long key = cand[(l * bp + c) * k + slot];
+        const unsigned long long key = key_at(i);
         if (key >= kth && key != 0ull) {
-            int p = atomicAdd(win_n, 1);
+            const int p = atomicAdd(win_n, 1);
             if (p < 64) win[p] = key;
         }
     }
     __syncthreads();
 }
 
+// ------------------------------------------------------------------ bound pass
+// Thread (r, c) of CTA g scans sample rows of its CTA's range for column c
+// and keeps its k best keys in a binary min-heap in shared memory
+// (slot-major, so a warp's accesses are contiguous).
+template <bool SIGNED>
+__global__ __launch_bounds__(SEL_THREADS) void k_sample_heaps(
+    const float *__restrict__ s, int64_t n_sample, int64_t stride, int bp, int lanes, int k,
+    int64_t rows_per_cta, const int32_t *__restrict__ ext_of, int64_t id_limit,
+    unsigned long long *__restrict__ lists_g) {
+    extern __shared__ unsigned long long heap[];   // [k][SEL_THREADS]
+    const int tid = threadIdx.x;
+    const int c = tid % bp, r = tid / bp;
+    for (int i = 0; i < k; ++i) heap[i * SEL_THREADS + tid] = 0ull;
+    if (r >= lanes) return;
+    unsigned long long root = 0ull;
+    const int64_t v0 = (int64_t)blockIdx.x * rows_per_cta;
+    const int64_t v1 = v0 + rows_per_cta < n_sample ? v0 + rows_per_cta : n_sample;
+    for (int64_t v = v0 + r; v < v1; v += lanes) {
+        const int64_t j = v * stride;
+        const int32_t id = ext_of[j];
+        if ((int64_t)id >= id_limit) continue;
+        const unsigned long long key = sel_key<SIGNED>(s[j * bp + c], (uint32_t)id);
+        if (key <= root) continue;
+        int i = 0;   // replace the minimum, sift down
+        while (true) {
+            const int l = 2 * i + 1, rr = l + 1;
+            if (l >= k) break;
+            int m = l;
+            unsigned long long km = heap[l * SEL_THREADS + tid];
+            if (rr < k) {
+                const unsigned long long kr = heap[rr * SEL_THREADS + tid];
+                if (kr < km) {
+                    m = rr;
+                    km = kr;
+                }
+            }
+            if (km >= key) break;
+            heap[i * SEL_THREADS + tid] = km;
+            i = m;
+        }
+        heap[i * SEL_THREADS + tid] = key;
+        root = heap[tid];
+    }
+    const int64_t list = (int64_t)blockIdx.x * lanes + r;
+    unsigned long long *dst = lists_g + (list * bp + c) * k;
+    for (int i = 0; i < k; ++i) dst[i] = heap[i * SEL_THREADS + tid];
+}
+
+// bound[c] = k-th largest sampled key of column c (0 if fewer than k);
+// also clears the column's buffer count.
+__global__ __launch_bounds__(SEL_THREADS) void k_sample_bound(
+    const unsigned long long *__restrict__ lists_g, int64_t lists, int bp, int b, int k,
+    unsigned long long *__restrict__ bound, unsigned int *__restrict__ cnt) {
+    __shared__ int hist[256 * (SEL_THREADS / 32)];
+    __shared__ unsigned long long win[64];
+    __shared__ unsigned long long s_prefix;
+    __shared__ int s_remaining, win_n;
+    const int c = blockIdx.x;
+    if (c >= b) {   // padding column: nothing passes the filter
+        if (threadIdx.x == 0) {
+            bound[c] = ~0ull;
+            cnt[c] = 0u;
+        }
+        return;
+    }
+    auto key_at = [&](int64_t i) -> unsigned long long {
+        return lists_g[((i / k) * bp + c) * k + (i % k)];
+    };
+    radix_select(lists * (int64_t)k, k, key_at, win, &win_n, hist, &s_prefix, &s_remaining);
+    if (threadIdx.x == 0) {
+        bound[c] = win_n >= k ? s_prefix : 0ull;
+        cnt[c] = 0u;
+    }
+}
+
+// ------------------------------------------------------------------ filter pass
+template <int BP>
+struct SelShape {
+    static constexpr int F = BP / 4;                 // float4 per row
+    static constexpr int G = F >= 32 ? 1 : 32 / F;   // rows per warp step
+    static constexpr int V = F >= 32 ? F / 32 : 1;   // float4 per lane
+    static constexpr int LW = F >= 32 ? 32 : F;      // lanes per row
+};
+
+// Append key to column c's buffer if it clears the bound.
+__device__ __forceinline__ void sel_push(unsigned long long key, unsigned long long bound, int c,
+                                         unsigned int *__restrict__ cnt,
+                                         unsigned long long *__restrict__ buf, int64_t cap) {
+    if (key >= bound) {
+        const unsigned int p = atomicAdd(&cnt[c], 1u);
+        if ((int64_t)p < cap) buf[(int64_t)c * cap + p] = key;
+    }
+}
+
+template <int BP, bool SIGNED>
+__global__ __launch_bounds__(256) void k_filter(const float *__restrict__ s, int64_t n,
+                                                const int32_t *__restrict__ ext_of,
+                                                int64_t id_limit,
+                                                const unsigned long long *__restrict__ bound,
+                                                unsigned int *__restrict__ cnt,
+                                                unsigned long long *__restrict__ buf, int64_t cap) {
+    using S = SelShape<BP>;
+    constexpr int R = 4;   // row steps in flight per warp
+    const int lane = threadIdx.x & 31;
+    const int g = lane / S::LW, sub = lane % S::LW;
+    unsigned long long thr[S::V][4];
+#pragma unroll
+    for (int v = 0; v < S::V; ++v)
+#pragma unroll
+        for (int e = 0; e < 4; ++e) thr[v][e] = bound[(sub + 32 * v) * 4 + e];
+    const float4 *s4 = (const float4 *)s;
+    const int64_t steps = (n + S::G - 1) / S::G;
+    const int64_t warp = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
+    for (int64_t t0 = warp * R; t0 < steps; t0 += nwarps * R) {
+        float4 x[R][S::V];
+        int32_t id[R];
+#pragma unroll
+        for (int q = 0; q < R; ++q) {
+            const int64_t j = (t0 + q) * S::G + g;
+            const bool ok = t0 + q < steps && j < n;
+            id[q] = ok ? ext_of[j] : (int32_t)0x7fffffff;
+#pragma unroll
+            for (int v = 0; v < S::V; ++v)
+                x[q][v] = ok ? s4[j * S::F + sub + 32 * v] : make_float4(0.f, 0.f, 0.f, 0.f);
+        }
+#pragma unroll
+        for (int q = 0; q < R; ++q) {
+            if ((int64_t)id[q] >= id_limit) continue;
+            const uint32_t u = (uint32_t)id[q];
+#pragma unroll
+            for (int v = 0; v < S::V; ++v) {
+                const int c = (sub + 32 * v) * 4;
+                sel_push(sel_key<SIGNED>(x[q][v].x, u), thr[v][0], c, cnt, buf, cap);
+                sel_push(sel_key<SIGNED>(x[q][v].y, u), thr[v][1], c + 1, cnt, buf, cap);
+                sel_push(sel_key<SIGNED>(x[q][v].z, u), thr[v][2], c + 2, cnt, buf, cap);
+                sel_push(sel_key<SIGNED>(x[q][v].w, u), thr[v][3], c + 3, cnt, buf, cap);
+            }
+        }
+    }
+}
+
+// ------------------------------------------------------------------ merge pass
+// The k best keys of column c: from its buffer (staged in shared memory when
+// small), or from the whole column of the slab if the buffer overflowed.
+template <bool SIGNED>
+__device__ void column_top(const float *__restrict__ s, int64_t n, int bp, int k, int c,
+                           const int32_t *__restrict__ ext_of, int64_t id_limit,
+                           const unsigned int *__restrict__ cnt,
+                           const unsigned long long *__restrict__ buf, int64_t cap,
+                           unsigned long long *stage, unsigned long long *win, int *win_n,
+                           int *hist, unsigned long long *s_prefix, int *s_remaining) {
+    const int64_t m = cnt[c];
+    if (m <= cap) {
+        const unsigned long long *bc = buf + (int64_t)c * cap;
+        if (m <= SEL_STAGE) {
+            for (int64_t i = threadIdx.x; i < m; i += SEL_THREADS) stage[i] = bc[i];
+            __syncthreads();
+            auto key_at = [&](int64_t i) -> unsigned long long { return stage[i]; };
+            radix_select(m, k, key_at, win, win_n, hist, s_prefix, s_remaining);
+        } else {
+            auto key_at = [&](int64_t i) -> unsigned long long { return bc[i]; };
+            radix_select(m, k, key_at, win, win_n, hist, s_prefix, s_remaining);
+        }
+    } else {
+        auto key_at = [&](int64_t i) -> unsigned long long {
+            const int32_t id = ext_of[i];
+            return (int64_t)id >= id_limit ? 0ull : sel_key<SIGNED>(s[i * bp + c], (uint32_t)id);
+        };
+        radix_select(n, k, key_at, win, win_n, hist, s_prefix, s_remaining);
+    }
+}
+
 // Retrieval merge, one CTA per real query column: the k winners ordered by
-// key (score desc, id asc), normalised by Z = sum of the score pass's tile
+// key (score desc, id asc), normalised by Z = sum of the score pass's
 // partials, resolved to pages, and their distinct pages counted.
 __global__ __launch_bounds__(SEL_THREADS) void k_topk_merge(
-    const unsigned long long *__restrict__ cand, int64_t lists, int bp, int k,
+    const float *__restrict__ s, int64_t n, int bp, int k, const int32_t *__restrict__ ext_of,
+    const unsigned int *__restrict__ cnt, const unsigned long long *__restrict__ buf, int64_t cap,
     const float *__restrict__ zpart, int64_t n_ztiles, const int32_t *__restrict__ row_of,
     const int32_t *__restrict__ page_row, int64_t *__restrict__ ids, float *__restrict__ scores,
     int32_t *__restrict__ page_ids, int32_t *__restrict__ n_pages, int *status) {
-    __shared__ int hist[256];
-    __shared__ unsigned long long s_prefix;
-    __shared__ int s_remaining;
+    __shared__ int hist[256 * (SEL_THREADS / 32)];
+    __shared__ unsigned long long stage[SEL_STAGE];
     __shared__ unsigned long long win[64];
-    __shared__ int win_n;
+    __shared__ unsigned long long s_prefix;
+    __shared__ int s_remaining, win_n;
     __shared__ double zred[SEL_THREADS / 32];
     __shared__ int pg[64];
     const int c = blockIdx.x;
@@ -147,7 +314,8 @@ __global__ __launch_bounds__(SEL_THREADS) void k_topk_merge(
     for (int64_t t = tid; t < n_ztiles; t += SEL_THREADS) z += (double)zpart[t * bp + c];
     for (int o = 16; o > 0; o >>= 1) z += __shfl_xor_sync(0xffffffffu, z, o);
     if ((tid & 31) == 0) zred[tid >> 5] = z;
-    radix_select_column(cand, lists, bp, k, c, win, &win_n, hist, &s_prefix, &s_remaining);
+    column_top<false>(s, n, bp, k, c, ext_of, (int64_t)1 << 40, cnt, buf, cap, stage, win, &win_n,
+                      hist, &s_prefix, &s_remaining);
     if (tid == 0 && win_n != k) set_status(status, AKASHIC_EDEVICE);
     const int got = win_n < k ? win_n : k;
     if (tid < got) {
@@ -180,16 +348,19 @@ __global__ __launch_bounds__(SEL_THREADS) void k_topk_merge(
 // Relation-update merge: the M best prior chunks of new chunk c (ordered by
 // cosine desc, id asc) into nbr_ids / nbr_cos rows c_base + c.
 __global__ __launch_bounds__(SEL_THREADS) void k_topm_merge(
-    const unsigned long long *__restrict__ cand, int64_t lists, int bp, int k, int64_t c_base,
+    const float *__restrict__ s, int64_t n, int bp, int k, const int32_t *__restrict__ ext_of,
+    int64_t id_limit, const unsigned int *__restrict__ cnt,
+    const unsigned long long *__restrict__ buf, int64_t cap, int64_t c_base,
     int32_t *__restrict__ nbr_ids, float *__restrict__ nbr_cos, int *status) {
-    __shared__ int hist[256];
-    __shared__ unsigned long long s_prefix;
-    __shared__ int s_remaining;
+    __shared__ int hist[256 * (SEL_THREADS / 32)];
+    __shared__ unsigned long long stage[SEL_STAGE];
     __shared__ unsigned long long win[64];
-    __shared__ int win_n;
+    __shared__ unsigned long long s_prefix;
+    __shared__ int s_remaining, win_n;
     const int c = blockIdx.x;
     const int tid = threadIdx.x;
-    radix_select_column(cand, lists, bp, k, c, win, &win_n, hist, &s_prefix, &s_remaining);
+    column_top<true>(s, n, bp, k, c, ext_of, id_limit, cnt, buf, cap, stage, win, &win_n, hist,
+                     &s_prefix, &s_remaining);
     if (tid == 0 && win_n != k) set_status(status, AKASHIC_EDEVICE);
     const int got = win_n < k ? win_n : k;
     if (tid < got) {
@@ -202,65 +373,75 @@ __global__ __launch_bounds__(SEL_THREADS) void k_topm_merge(
     }
 }
 
-SelectPlan select_plan(int64_t n, int bp, int k, int sm_count) {
-    SelectPlan sp;
-    sp.lanes = SEL_THREADS / bp > 0 ? SEL_THREADS / bp : 1;
-    // at least ~4k rows per list, at most two CTAs per SM
-    int64_t want = ceil_div<int64_t>(n, (int64_t)sp.lanes * 4 * k);
-    int64_t cap = 2 * (int64_t)sm_count;
-    sp.grid = (int)(want < 1 ? 1 : (want > cap ? cap : want));
-    sp.lists = (int64_t)sp.grid * sp.lanes;
-    return sp;
-}
-
-cudaError_t launch_select(const SelectPlan &sp, const float *s, int64_t n, int bp, int b, int k,
-                          unsigned long long *cand, const float *zpart, int64_t n_ztiles,
-                          const int32_t *ext_of, const int32_t *row_of, const int32_t *page_row,
-                          int64_t *ids, float *scores, int32_t *page_ids, int32_t *n_pages,
-                          int *status, cudaStream_t st, int *launches) {
-    const size_t smem = (size_t)k * SEL_THREADS * sizeof(unsigned long long);
-    static bool attr_set[64] = {false};
+// ------------------------------------------------------------------ launchers
+template <bool SIGNED>
+static cudaError_t bound_and_filter(const SelectPlan &sp, const float *s, int b,
+                                    const int32_t *ext_of, int64_t id_limit,
+                                    unsigned long long *ws, cudaStream_t st, int *launches) {
+    static bool attr[2][64] = {{false}};
     int dev = 0;
     cudaGetDevice(&dev);
-    if (dev >= 0 && dev < 64 && !attr_set[dev]) {
-        const int mx = 64 * SEL_THREADS * (int)sizeof(unsigned long long);
-        cudaError_t e = cudaFuncSetAttribute(k_topk_candidates<false>,
-                                             cudaFuncAttributeMaxDynamicSharedMemorySize, mx);
-        if (e == cudaSuccess)
-            e = cudaFuncSetAttribute(k_topk_candidates<true>,
-                                     cudaFuncAttributeMaxDynamicSharedMemorySize, mx);
+    if (dev >= 0 && dev < 64 && !attr[SIGNED][dev]) {
+        cudaError_t e = cudaFuncSetAttribute(k_sample_heaps<SIGNED>,
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             64 * SEL_THREADS * (int)sizeof(unsigned long long));
         if (e != cudaSuccess) return e;
-        attr_set[dev] = true;
+        attr[SIGNED][dev] = true;
     }
-    const int64_t rows_per_cta = ceil_div<int64_t>(n, sp.grid);
-    k_topk_candidates<false><<<sp.grid, SEL_THREADS, smem, st>>>(
-        s, n, bp, sp.lanes, k, rows_per_cta, ext_of, (int64_t)1 << 40, cand);
+    const size_t smem = (size_t)sp.k * SEL_THREADS * sizeof(unsigned long long);
+    const int64_t rows_per_cta = ceil_div<int64_t>(sp.n_sample, sp.grid);
+    k_sample_heaps<SIGNED><<<sp.grid, SEL_THREADS, smem, st>>>(
+        s, sp.n_sample, sp.stride, sp.bp, sp.lanes, sp.k, rows_per_cta, ext_of, id_limit, ws);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
-    k_topk_merge<<<b, SEL_THREADS, 0, st>>>(cand, sp.lists, bp, k, zpart, n_ztiles, row_of,
-                                            page_row, ids, scores, page_ids, n_pages, status);
-    if (launches) *launches += 2;
+    unsigned long long *bound = ws + sp.off_bound;
+    unsigned int *cnt = (unsigned int *)(ws + sp.off_cnt);
+    unsigned long long *buf = ws + sp.off_buf;
+    k_sample_bound<<<sp.bp, SEL_THREADS, 0, st>>>(ws, sp.lists, sp.bp, b, sp.k, bound, cnt);
+    e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    const int64_t warps = ceil_div<int64_t>(sp.n, 4);
+    int grid = (int)(ceil_div<int64_t>(warps, 8) < (int64_t)device_sm_count() * 8
+                         ? ceil_div<int64_t>(warps, 8)
+                         : (int64_t)device_sm_count() * 8);
+    grid = grid < 1 ? 1 : grid;
+    switch (sp.bp) {
+    case 32: k_filter<32, SIGNED><<<grid, 256, 0, st>>>(s, sp.n, ext_of, id_limit, bound, cnt, buf, sp.cap); break;
+    case 64: k_filter<64, SIGNED><<<grid, 256, 0, st>>>(s, sp.n, ext_of, id_limit, bound, cnt, buf, sp.cap); break;
+    case 128: k_filter<128, SIGNED><<<grid, 256, 0, st>>>(s, sp.n, ext_of, id_limit, bound, cnt, buf, sp.cap); break;
+    case 256: k_filter<256, SIGNED><<<grid, 256, 0, st>>>(s, sp.n, ext_of, id_limit, bound, cnt, buf, sp.cap); break;
+    default: return cudaErrorInvalidValue;
+    }
+    if (launches) *launches += 3;
     return cudaGetLastError();
 }
 
-cudaError_t launch_select_signed(const SelectPlan &sp, const float *s, int64_t n, int bp, int b,
-                                 int k, unsigned long long *cand, const int32_t *ext_of,
-                                 int64_t id_limit, int64_t c_base, int32_t *nbr_ids,
-                                 float *nbr_cos, int *status, cudaStream_t st, int *launches) {
-    const size_t smem = (size_t)k * SEL_THREADS * sizeof(unsigned long long);
-    cudaError_t e = cudaFuncSetAttribute(k_topk_candidates<true>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         64 * SEL_THREADS * (int)sizeof(unsigned long long));
+cudaError_t launch_select(const SelectPlan &sp, const float *s, int b, unsigned long long *ws,
+                          const float *zpart, int64_t n_ztiles, const int32_t *ext_of,
+                          const int32_t *row_of, const int32_t *page_row, int64_t *ids,
+                          float *scores, int32_t *page_ids, int32_t *n_pages, int *status,
+                          cudaStream_t st, int *launches) {
+    cudaError_t e = bound_and_filter<false>(sp, s, b, ext_of, (int64_t)1 << 40, ws, st, launches);
     if (e != cudaSuccess) return e;
-    const int64_t rows_per_cta = ceil_div<int64_t>(n, sp.grid);
-    k_topk_candidates<true><<<sp.grid, SEL_THREADS, smem, st>>>(s, n, bp, sp.lanes, k,
-                                                                rows_per_cta, ext_of, id_limit,
-                                                                cand);
-    e = cudaGetLastError();
+    k_topk_merge<<<b, SEL_THREADS, 0, st>>>(s, sp.n, sp.bp, sp.k, ext_of,
+                                            (const unsigned int *)(ws + sp.off_cnt),
+                                            ws + sp.off_buf, sp.cap, zpart, n_ztiles, row_of,
+                                            page_row, ids, scores, page_ids, n_pages, status);
+    if (launches) *launches += 1;
+    return cudaGetLastError();
+}
+
+cudaError_t launch_select_signed(const SelectPlan &sp, const float *s, int b,
+                                 unsigned long long *ws, const int32_t *ext_of, int64_t id_limit,
+                                 int64_t c_base, int32_t *nbr_ids, float *nbr_cos, int *status,
+                                 cudaStream_t st, int *launches) {
+    cudaError_t e = bound_and_filter<true>(sp, s, b, ext_of, id_limit, ws, st, launches);
     if (e != cudaSuccess) return e;
-    k_topm_merge<<<b, SEL_THREADS, 0, st>>>(cand, sp.lists, bp, k, c_base, nbr_ids, nbr_cos,
+    k_topm_merge<<<b, SEL_THREADS, 0, st>>>(s, sp.n, sp.bp, sp.k, ext_of, id_limit,
+                                            (const unsigned int *)(ws + sp.off_cnt),
+                                            ws + sp.off_buf, sp.cap, c_base, nbr_ids, nbr_cos,
                                             status);
-    if (launches) *launches += 2;
+    if (launches) *launches += 1;
     return cudaGetLastError();
 }
 

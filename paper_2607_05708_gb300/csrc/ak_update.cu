@@ -36,11 +36,11 @@ akashic_status_t relate_top_m(const UpdateArgs &a, cudaStream_t st, int *launche
         int64_t lists = 0;
         for (int bp = 32; bp <= bp_max; bp <<= 1) {
             SelectPlan sp = select_plan(n_old, bp, a.M, device_sm_count());
-            int64_t need = sp.lists * bp;
+            int64_t need = sp.words;
             lists = need > lists ? need : lists;
         }
         (void)sp_max;
-        e = cudaMalloc(&cand, (size_t)lists * a.M * 8);
+        e = cudaMalloc(&cand, (size_t)lists * 8);
     }
     akashic_status_t rc = AKASHIC_OK;
     if (e != cudaSuccess) {
@@ -58,8 +58,8 @@ akashic_status_t relate_top_m(const UpdateArgs &a, cudaStream_t st, int *launche
             e = launch_dots(a.emb, n_old, a.dim, qp, bp, dots, a.status, st, launches);
         const SelectPlan sp = select_plan(n_old, bp, a.M, device_sm_count());
         if (e == cudaSuccess)
-            e = launch_select_signed(sp, dots, n_old, bp, b, a.M, cand, a.ext_of, a.first, off,
-                                     a.nbr_ids, a.nbr_cos, a.status, st, launches);
+            e = launch_select_signed(sp, dots, b, cand, a.ext_of, a.first, off, a.nbr_ids,
+                                     a.nbr_cos, a.status, st, launches);
         if (e != cudaSuccess) rc = AKASHIC_ECUDA;
         if (launches) *launches += 1;
     }
