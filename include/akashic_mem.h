@@ -171,6 +171,43 @@ enum {
 akashic_status_t akashic_mem_set_profiling(akashic_mem_t *m, int32_t on);
 akashic_status_t akashic_mem_phase_times(akashic_mem_t *m, float *ms, int32_t *launches);
 
+/* Softmax scores for callers that cannot allocate device memory.
+ *
+ * The paper has no counterpart: this is a library convenience.  Code that
+ * records work into a CUDA graph, runs inside a serving runtime's
+ * pre-reserved memory pool, or has no device allocator cannot call
+ * cudaMalloc when it needs scores, and akashic_mem_create allocates.  This
+ * call needs no store and allocates nothing: it computes, over caller-owned
+ * buffers, the score step of retrieval
+ *   u[j*B + b] = exp(tau <e_j, q_b> - c_b),   z[b] = sum_j u[j*B + b],
+ *   c_b = tau |q_b| max_j |e_j|,
+ * so that u[:, b] / z[b] is the softmax over the n chunks (the same kernel
+ * as the score step of akashic_mem_retrieve).
+ *   emb    device, n x dim bf16 bits (chunk j in row j), 16-byte aligned
+ *   q      device, B x dim bf16 bits, 16-byte aligned
+ *   B      32, 64, 128 or 256 (pad with zero queries); larger B is rejected
+ *          because the fixed scratch holds at most 256 queries
+ *   temperature  tau; 0 => 1/sqrt(dim)
+ *   u      device float[n*B] (output, chunk-major), 16-byte aligned
+ *   z      device float[B] (output)
+ *   shift  device float[B] (output c_b) or NULL
+ *   status device int32 (output) or NULL: 0, or ERANGE / ETIMEOUT found by
+ *          the kernels
+ * Its scratch is a fixed 320 KiB array in device memory, present on every
+ * GPU that runs this call until the process exits (no allocation ever
+ * happens).  The first call on a device looks up that array's address with
+ * cudaGetSymbolAddress while the device is current; make that first call
+ * before capturing a stream.  Every call shares the array, so calls whose
+ * work overlaps on the GPU (different streams without ordering) race and
+ * must not be issued.  Stream-ordered; does not synchronise.
+ * EINVAL for a NULL pointer, misalignment, n < 1, dim outside [64, 4096]
+ * or not a multiple of 64, B not in {32, 64, 128, 256}, or a device with
+ * more than 256 SMs; ECUDA if a launch fails. */
+akashic_status_t akashic_mem_softmax_scores_noalloc(const uint16_t *emb, int64_t n, int32_t dim,
+                                                    const uint16_t *q, int32_t B,
+                                                    float temperature, float *u, float *z,
+                                                    float *shift, int32_t *status, void *stream);
+
 /* Thread-local description of the last failure on this thread ("" if none). */
 const char *akashic_mem_last_error(void);
 

@@ -16,7 +16,8 @@ import os
 from ._build import LIB as LIB_PATH
 from ._build import build
 
-__all__ = ["MemStore", "AkashicError", "load_library", "build", "EXPORTS", "STATUS", "PHASES"]
+__all__ = ["MemStore", "AkashicError", "load_library", "build", "EXPORTS", "STATUS", "PHASES",
+           "softmax_scores_noalloc"]
 
 STATUS = {0: "OK", 1: "EINVAL", 2: "ENOMEM", 3: "ECAPACITY", 4: "ECUDA", 5: "ETIMEOUT",
           6: "EDEVICE", 7: "ERANGE"}
@@ -27,7 +28,7 @@ EXPORTS = (
     "akashic_mem_create", "akashic_mem_destroy", "akashic_mem_append_chunks",
     "akashic_mem_update_relations", "akashic_mem_retrieve", "akashic_mem_export_csr",
     "akashic_mem_size", "akashic_mem_sync", "akashic_mem_set_profiling",
-    "akashic_mem_phase_times", "akashic_mem_last_error",
+    "akashic_mem_phase_times", "akashic_mem_last_error", "akashic_mem_softmax_scores_noalloc",
 )
 
 
@@ -72,6 +73,8 @@ def load_library(path: str | None = None):
         "akashic_mem_phase_times": ([V, ctypes.POINTER(ctypes.c_float), ctypes.POINTER(I32)],
                                     ctypes.c_int),
         "akashic_mem_last_error": ([], ctypes.c_char_p),
+        "akashic_mem_softmax_scores_noalloc": ([V, I64, I32, V, I32, F, V, V, V, V, V],
+                                               ctypes.c_int),
     }
     for name, (args, res) in sig.items():
         fn = getattr(lib, name)
@@ -95,6 +98,22 @@ def _ptr(t):
 def _stream(torch, stream, device):
     s = stream if stream is not None else torch.cuda.current_stream(device)
     return ctypes.c_void_p(s.cuda_stream)
+
+
+def softmax_scores_noalloc(emb, q, u, z, temperature=0.0, shift=None, status=None, stream=None):
+    """Scores for callers that cannot allocate: fills the caller's u [n, B]
+    and z [B] (softmax = u[:, b] / z[b]) through
+    akashic_mem_softmax_scores_noalloc, which uses a fixed scratch array and
+    allocates nothing.  emb: int16 [n, dim], q: int16 [B, dim] with B in
+    {32, 64, 128, 256}, all CUDA tensors on the current device."""
+    import torch
+    for t, name in ((emb, "emb"), (q, "q"), (u, "u"), (z, "z")):
+        if not t.is_cuda or not t.is_contiguous():
+            raise ValueError(f"{name} must be a contiguous CUDA tensor")
+    s = stream if stream is not None else torch.cuda.current_stream(emb.device)
+    _check(load_library().akashic_mem_softmax_scores_noalloc(
+        _ptr(emb), emb.shape[0], emb.shape[1], _ptr(q), q.shape[0], float(temperature), _ptr(u),
+        _ptr(z), _ptr(shift), _ptr(status), ctypes.c_void_p(s.cuda_stream)))
 
 
 class MemStore:

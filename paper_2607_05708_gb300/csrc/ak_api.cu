@@ -20,6 +20,8 @@ using namespace ak;
 // ------------------------------------------------------------------ errors
 static thread_local std::string g_last_error;
 
+void ak::set_last_error(const char *msg) { g_last_error = msg ? msg : ""; }
+
 static akashic_status_t fail(akashic_status_t st, const char *fmt, ...) {
     char buf[512];
     va_list ap;

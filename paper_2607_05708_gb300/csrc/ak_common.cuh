@@ -48,6 +48,9 @@ __device__ __forceinline__ float unordered_bits(uint32_t o) {
     return __uint_as_float(u);
 }
 
+// Set the thread-local message returned by akashic_mem_last_error().
+void set_last_error(const char *msg);
+
 // ------------------------------------------------------------------ launchers
 // All launchers enqueue on `st` and report launch errors by return value.
 
