@@ -89,7 +89,7 @@ int device_sm_count();
 struct SplitParams {
     int64_t split_t = 256;      // in-degree above which a row is split
     int64_t seg_len = 512;      // edges per segment at most
-    int64_t win_rows = 16384;   // source window (rows); 16 MB of slab at 256 queries
+    int64_t win_rows = 32768;   // source window (rows); 32 MB of slab at 256 queries
 };
 constexpr int ROWS_PER_GRAB = 8;     // rows a warp claims at a time (dynamic scheduling)
 
