@@ -511,6 +511,28 @@ cudaError_t launch_seg_permute(const uint32_t *order, const int64_t *e0, const i
 // smaller BP the warp splits into 32/(BP/4) lane groups that take
 // alternate edges and are summed at the end.  Rows with more than split_t
 // in-edges are skipped here and handled by window segments + fixup.
+// L2 policy for the hop: gathered source rows are re-read ~32 times (once
+// per out-edge of the source), so they are loaded with an evict-last
+// policy; everything read or written once (graph arrays, u, the output
+// slab, partial sums) streams with evict-first (.cs) accesses so that it
+// does not push gathered rows out of L2.
+__device__ __forceinline__ uint64_t l2_keep_policy() {
+    uint64_t pol;
+    asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(pol));
+    return pol;
+}
+__device__ __forceinline__ float4 ld_keep(const float4 *p, uint64_t pol) {
+    float4 v;
+    asm volatile("ld.global.nc.L1::no_allocate.L2::cache_hint.v4.f32 {%0,%1,%2,%3}, [%4], %5;"
+                 : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
+                 : "l"(p), "l"(pol));
+    return v;
+}
+__device__ __forceinline__ float4 ld_stream(const float4 *p) { return __ldcs(p); }
+__device__ __forceinline__ void st_stream(float4 *p, float4 v) { __stcs(p, v); }
+__device__ __forceinline__ int32_t ld_stream(const int32_t *p) { return __ldcs(p); }
+__device__ __forceinline__ float ld_stream(const float *p) { return __ldcs(p); }
+
 template <int BP>
 struct HopShape {
     static constexpr int F = BP / 4;                       // float4 per row
@@ -528,22 +550,23 @@ __device__ __forceinline__ void hop_accumulate(const int32_t *__restrict__ in_sr
     constexpr int UN = 8 / S::V > 0 ? 8 / S::V : 1;   // gathers in flight: UN edges x V float4
     const int lane = threadIdx.x & 31;
     const int g = lane / S::LW, sub = lane % S::LW;
+    const uint64_t pol = l2_keep_policy();
 #pragma unroll
     for (int v = 0; v < S::V; ++v) acc[v] = make_float4(0.f, 0.f, 0.f, 0.f);
     // the next batch's (source, weight) pairs are loaded while this batch gathers
     int32_t s_n = 0;
     float w_n = 0.f;
     if (e0 + lane < e1) {
-        s_n = in_src[e0 + lane];
-        w_n = in_w[e0 + lane];
+        s_n = ld_stream(in_src + e0 + lane);
+        w_n = ld_stream(in_w + e0 + lane);
     }
     for (int64_t eb = e0; eb < e1; eb += 32) {
         const int cnt = (int)(e1 - eb < 32 ? e1 - eb : 32);
         const int32_t s_l = s_n;
         const float w_l = w_n;
         if (eb + 32 + lane < e1) {
-            s_n = in_src[eb + 32 + lane];
-            w_n = in_w[eb + 32 + lane];
+            s_n = ld_stream(in_src + eb + 32 + lane);
+            w_n = ld_stream(in_w + eb + 32 + lane);
         }
         int t = 0;
         for (; t + UN * S::G <= cnt; t += UN * S::G) {
@@ -558,7 +581,8 @@ __device__ __forceinline__ void hop_accumulate(const int32_t *__restrict__ in_sr
 #pragma unroll
             for (int q = 0; q < UN; ++q)
 #pragma unroll
-                for (int v = 0; v < S::V; ++v) x[q][v] = in4[(int64_t)sq[q] * S::F + sub + 32 * v];
+                for (int v = 0; v < S::V; ++v)
+                    x[q][v] = ld_keep(in4 + (int64_t)sq[q] * S::F + sub + 32 * v, pol);
 #pragma unroll
             for (int q = 0; q < UN; ++q)
 #pragma unroll
@@ -576,7 +600,7 @@ __device__ __forceinline__ void hop_accumulate(const int32_t *__restrict__ in_sr
             if (idx < cnt) {
 #pragma unroll
                 for (int v = 0; v < S::V; ++v) {
-                    float4 x = in4[(int64_t)sv * S::F + sub + 32 * v];
+                    float4 x = ld_keep(in4 + (int64_t)sv * S::F + sub + 32 * v, pol);
                     acc[v].x = fmaf(wv, x.x, acc[v].x);
                     acc[v].y = fmaf(wv, x.y, acc[v].y);
                     acc[v].z = fmaf(wv, x.z, acc[v].z);
@@ -632,7 +656,7 @@ __global__ __launch_bounds__(256, 3) void k_hop_rows(const int64_t *__restrict__
             float4 b[S::V];
             if (lane < S::LW) {
 #pragma unroll
-                for (int v = 0; v < S::V; ++v) b[v] = u4[j * S::F + sub + 32 * v];
+                for (int v = 0; v < S::V; ++v) b[v] = ld_stream(u4 + j * S::F + sub + 32 * v);
             }
             float4 acc[S::V];
             hop_accumulate<BP>(in_src, in_w, e0, e1, in4, acc);
@@ -643,7 +667,7 @@ __global__ __launch_bounds__(256, 3) void k_hop_rows(const int64_t *__restrict__
                     b[v].y = fmaf(alpha, acc[v].y, b[v].y);
                     b[v].z = fmaf(alpha, acc[v].z, b[v].z);
                     b[v].w = fmaf(alpha, acc[v].w, b[v].w);
-                    out4[j * S::F + sub + 32 * v] = b[v];
+                    st_stream(out4 + j * S::F + sub + 32 * v, b[v]);
                 }
             }
         }
@@ -674,7 +698,7 @@ __global__ __launch_bounds__(256, 3) void k_hop_segs(const int64_t *__restrict__
         const int64_t slot = seg_slot[s];
         if (lane < S::LW) {
 #pragma unroll
-            for (int v = 0; v < S::V; ++v) part4[slot * S::F + sub + 32 * v] = acc[v];
+            for (int v = 0; v < S::V; ++v) st_stream(part4 + slot * S::F + sub + 32 * v, acc[v]);
         }
     }
 }
@@ -703,7 +727,7 @@ __global__ __launch_bounds__(256) void k_hop_fixup(const int32_t *__restrict__ s
             for (; s + P <= b; s += P) {
                 float4 x[P];
 #pragma unroll
-                for (int q = 0; q < P; ++q) x[q] = part4[(s + q) * F + f];
+                for (int q = 0; q < P; ++q) x[q] = ld_stream(part4 + (s + q) * F + f);
 #pragma unroll
                 for (int q = 0; q < P; ++q) {
                     acc.x += x[q].x; acc.y += x[q].y; acc.z += x[q].z; acc.w += x[q].w;
