@@ -132,6 +132,24 @@ def cpu_baseline(wl, placement, n_queries, rng_seed=0):
                 seconds=dt)
 
 
+def max_over_ranks(values, device=None):
+    """Max of each value over all ranks of the default process group (the
+    slowest rank sets the job's time); identity when not distributed."""
+    import torch
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized()) or dist.get_world_size() == 1:
+        return [float(v) for v in values]
+    t = torch.tensor([float(v) for v in values], dtype=torch.float64,
+                     device=device if device is not None else "cpu")
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return t.tolist()
+
+
+def job_throughput(units_per_rank, world, ms):
+    """Whole-job throughput: the units every rank processed over the max time."""
+    return units_per_rank * world / (ms * 1e-3)
+
+
 def dist_env():
     ws = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
@@ -276,10 +294,7 @@ def main():
     d2h = sum(t.numel() * t.element_size() for t in outs_host)
 
     # max over ranks
-    if ws > 1:
-        t = torch.tensor([ms, ms_e2e], device=f"cuda:{dev}")
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        ms, ms_e2e = t.tolist()
+    ms, ms_e2e = max_over_ranks([ms, ms_e2e], device=f"cuda:{dev}" if ws > 1 else None)
 
     hbm, bf16, peak_kind = peaks()
     ab = algorithmic_bytes(wl.n, wl.dim, B, wl.nnz, wl.hops, k)
@@ -305,7 +320,7 @@ def main():
     achieved = per_launch_bytes / (dom_avg_ms * 1e-3) / 1e9
     line = {
         "metric": METRIC,
-        "value": B * args.steps * ws / (ms * 1e-3),
+        "value": job_throughput(B * args.steps, ws, ms),
         "unit": "queries/s",
         "n_gpus": ws,
         "steps": args.steps,
@@ -329,7 +344,7 @@ def main():
                           "flops": 2.0 * wl.n * B * wl.dim,
                           "peak_tflops_bf16": bf16},
         "phases_ms_per_step": {p: phases[p][0] / args.steps for p in ("score", "propagate", "select")},
-        "e2e": {"value": B * args.steps * ws / (ms_e2e * 1e-3), "unit": "queries/s",
+        "e2e": {"value": job_throughput(B * args.steps, ws, ms_e2e), "unit": "queries/s",
                 "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
         "gpu_launches": int(sum(v[1] for v in phases.values())),
         "pages_per_query": {args.placement: npg_clustered},

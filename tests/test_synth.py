@@ -1,0 +1,94 @@
+"""The seeded workload generator: determinism and the structure each
+workload promises (the inputs of every parity test and of the benchmark)."""
+import hashlib
+
+import numpy as np
+import pytest
+
+import synth
+
+
+def _digest(wl):
+    h = hashlib.sha256()
+    for a in (wl.emb, wl.queries, wl.row_ptr, wl.col, wl.aff, *wl.page_of.values()):
+        h.update(np.ascontiguousarray(a).tobytes())
+    return h.hexdigest()
+
+
+def test_deterministic():
+    assert _digest(synth.workload(0)) == _digest(synth.workload(0))
+    assert _digest(synth.workload(2, scale=1 / 256)) == _digest(synth.workload(2, scale=1 / 256))
+
+
+def test_bf16_rounding_ties_to_even():
+    v = np.array([1.0, 1.00390625, 1.005859375, -1.00390625, 3.0e-38, 0.0], np.float32)
+    assert list(synth.to_bf16(v)) == [0x3F80, 0x3F80, 0x3F81, 0xBF80, 0x0123, 0x0000]
+    x = np.random.default_rng(0).standard_normal(1000).astype(np.float32)
+    back = synth.bf16_to_f32(synth.to_bf16(x))
+    assert np.all(np.abs(back - x) <= np.abs(x) * 2.0 ** -8)
+
+
+def _check_csr(wl, deg):
+    n = wl.n
+    assert wl.row_ptr[0] == 0 and wl.row_ptr[-1] == wl.nnz
+    assert (np.diff(wl.row_ptr) == deg).all()
+    rows = np.repeat(np.arange(n), deg)
+    assert (wl.col != rows).all(), "self loops"
+    c = wl.col.reshape(n, deg)
+    assert (np.diff(c, axis=1) > 0).all(), "columns not strictly ascending"
+    assert (c >= 0).all() and (c < n).all()
+    assert np.isfinite(wl.aff).all()
+
+
+def test_tiny_store_shape():
+    wl = synth.workload(0)
+    assert (wl.n, wl.dim, wl.n_queries, wl.k, wl.hops, wl.alpha) == (4096, 256, 4, 8, 1, 0.5)
+    _check_csr(wl, 8)
+    assert (wl.aff <= 0).all()                         # ln U, U in (0, 1]
+    assert (wl.page_of["id"] == np.arange(wl.n) // 16).all()
+    norms = np.linalg.norm(synth.bf16_to_f32(wl.emb), axis=1)
+    assert np.allclose(norms, 1.0, atol=1e-2)
+
+
+def test_gmm65k_graph_is_exact_cosine_knn():
+    """Within-component top-16 equals the global top-16 (checked on a sample
+    against every chunk of the store)."""
+    wl = synth.workload(1, scale=1 / 16)
+    _check_csr(wl, 16)
+    E = synth.bf16_to_f32(wl.emb).astype(np.float64)
+    rng = np.random.default_rng(0)
+    for i in rng.choice(wl.n, size=40, replace=False):
+        dots = E @ E[i]
+        dots[i] = -np.inf
+        ref = np.lexsort((np.arange(wl.n), -dots))[:16]
+        assert sorted(ref) == sorted(wl.col[wl.row_ptr[i]:wl.row_ptr[i + 1]])
+        assert np.allclose(wl.aff[wl.row_ptr[i]:wl.row_ptr[i + 1]],
+                           10 * dots[np.sort(ref)], atol=1e-5)
+
+
+def test_gmm1m_recipe_power_law_and_placements():
+    wl = synth.workload(2, scale=1 / 64)
+    _check_csr(wl, 32)
+    indeg = np.bincount(wl.col, minlength=wl.n)
+    assert indeg.max() > 50 * np.median(indeg)        # heavy-tailed in-degree
+    sizes = np.bincount(wl.component)
+    assert sizes.sum() == wl.n and sizes.min() >= 1
+    assert sizes.max() > 20 * np.median(sizes)        # Zipf component sizes
+    for kind in ("clustered", "random"):
+        pages = wl.page_of[kind]
+        assert np.bincount(pages).max() <= wl.chunks_per_page
+    # clustered pages hold one component each except at component boundaries
+    cl = wl.page_of["clustered"]
+    mixed = sum(len(set(wl.component[cl == p])) > 1 for p in range(cl.max() + 1))
+    assert mixed <= wl.component.max() + 1
+
+
+def test_zipf_sizes():
+    s = synth.zipf_sizes(1000, 10, 1.1)
+    assert s.sum() == 1000 and (s >= 1).all() and (np.diff(s) <= 0).all()
+
+
+def test_update_workload():
+    wl = synth.workload(3, scale=1 / 256)
+    assert wl.new_emb.shape == (16, wl.dim) and wl.top_m == 32
+    assert wl.new_component.max() <= wl.component.max()
