@@ -703,9 +703,10 @@ __global__ __launch_bounds__(256, 3) void k_hop_segs(const int64_t *__restrict__
     }
 }
 
-// Split rows: out = u + alpha * (sum of the row's segment partials, in slot
-// order).  One warp per row; each lane keeps 8 independent partial loads in
-// flight per float4 column it owns.
+// Split rows: out = u + alpha * (sum of the row's segment partials).  One
+// CTA per row: warp w sums a fixed contiguous slice of the row's slots, the
+// eight slice sums are then added in warp order, so the result does not
+// depend on scheduling.  Lanes keep several partial loads in flight.
 template <int BP>
 __global__ __launch_bounds__(256) void k_hop_fixup(const int32_t *__restrict__ split_row,
                                                    const int64_t *__restrict__ split_slot0,
@@ -714,36 +715,67 @@ __global__ __launch_bounds__(256) void k_hop_fixup(const int32_t *__restrict__ s
                                                    const float4 *__restrict__ u4,
                                                    float4 *__restrict__ out4, float alpha) {
     constexpr int F = BP / 4;
-    constexpr int P = 8;
-    int64_t r = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
-    const int64_t stride = ((int64_t)gridDim.x * blockDim.x) >> 5;
-    const int lane = threadIdx.x & 31;
-    for (; r < n_split; r += stride) {
+    constexpr int PER_LANE = (F + 31) / 32;
+    constexpr int P = 4;
+    __shared__ float4 wsum[8][F];
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    for (int64_t r = blockIdx.x; r < n_split; r += gridDim.x) {
         const int64_t j = split_row[r];
         const int64_t a = split_slot0[r], b = split_slot0[r + 1];
-        for (int f = lane; f < F; f += 32) {
-            float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-            int64_t s = a;
-            for (; s + P <= b; s += P) {
-                float4 x[P];
+        const int64_t per = (b - a + 7) / 8;
+        const int64_t s0 = a + warp * per;
+        const int64_t s1 = s0 + per < b ? s0 + per : b;
+        float4 acc[PER_LANE];
 #pragma unroll
-                for (int q = 0; q < P; ++q) x[q] = ld_stream(part4 + (s + q) * F + f);
+        for (int t = 0; t < PER_LANE; ++t) acc[t] = make_float4(0.f, 0.f, 0.f, 0.f);
+        int64_t s = s0;
+        for (; s + P <= s1; s += P) {
+            float4 x[P][PER_LANE];
 #pragma unroll
-                for (int q = 0; q < P; ++q) {
-                    acc.x += x[q].x; acc.y += x[q].y; acc.z += x[q].z; acc.w += x[q].w;
+            for (int q = 0; q < P; ++q)
+#pragma unroll
+                for (int t = 0; t < PER_LANE; ++t) {
+                    const int f = lane + 32 * t;
+                    x[q][t] = f < F ? ld_stream(part4 + (s + q) * F + f) : make_float4(0.f, 0.f, 0.f, 0.f);
+                }
+#pragma unroll
+            for (int q = 0; q < P; ++q)
+#pragma unroll
+                for (int t = 0; t < PER_LANE; ++t) {
+                    acc[t].x += x[q][t].x; acc[t].y += x[q][t].y;
+                    acc[t].z += x[q][t].z; acc[t].w += x[q][t].w;
+                }
+        }
+        for (; s < s1; ++s)
+#pragma unroll
+            for (int t = 0; t < PER_LANE; ++t) {
+                const int f = lane + 32 * t;
+                if (f < F) {
+                    const float4 x = ld_stream(part4 + s * F + f);
+                    acc[t].x += x.x; acc[t].y += x.y; acc[t].z += x.z; acc[t].w += x.w;
                 }
             }
-            for (; s < b; ++s) {
-                const float4 x = part4[s * F + f];
-                acc.x += x.x; acc.y += x.y; acc.z += x.z; acc.w += x.w;
-            }
-            float4 o = u4[j * F + f];
-            o.x = fmaf(alpha, acc.x, o.x);
-            o.y = fmaf(alpha, acc.y, o.y);
-            o.z = fmaf(alpha, acc.z, o.z);
-            o.w = fmaf(alpha, acc.w, o.w);
-            out4[j * F + f] = o;
+#pragma unroll
+        for (int t = 0; t < PER_LANE; ++t) {
+            const int f = lane + 32 * t;
+            if (f < F) wsum[warp][f] = acc[t];
         }
+        __syncthreads();
+        for (int f = threadIdx.x; f < F; f += blockDim.x) {
+            float4 tot = wsum[0][f];
+#pragma unroll
+            for (int w = 1; w < 8; ++w) {
+                tot.x += wsum[w][f].x; tot.y += wsum[w][f].y;
+                tot.z += wsum[w][f].z; tot.w += wsum[w][f].w;
+            }
+            float4 o = ld_stream(u4 + j * F + f);
+            o.x = fmaf(alpha, tot.x, o.x);
+            o.y = fmaf(alpha, tot.y, o.y);
+            o.z = fmaf(alpha, tot.z, o.z);
+            o.w = fmaf(alpha, tot.w, o.w);
+            st_stream(out4 + j * F + f, o);
+        }
+        __syncthreads();
     }
 }
 
@@ -772,7 +804,7 @@ static cudaError_t hop_bp(const HopPlan &p, const float *u, const float *in, flo
     e = cudaGetLastError();
     if (launches) *launches += 1;
     if (e != cudaSuccess || p.n_split_rows == 0) return e;
-    const int g3 = (int)ceil_div<int64_t>(p.n_split_rows, 8);
+    const int g3 = (int)(p.n_split_rows < (int64_t)sms * 16 ? p.n_split_rows : (int64_t)sms * 16);
     k_hop_fixup<BP><<<g3, 256, 0, st>>>(p.split_row, p.split_slot0, p.n_split_rows,
                                         (const float4 *)partial, (const float4 *)u, (float4 *)out,
                                         alpha);
