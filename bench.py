@@ -186,6 +186,135 @@ def run_reference(args):
     return 0
 
 
+def run_update(args):
+    """Relation update: each step appends the 4096 new chunks of the update
+    workload again and links them to every prior chunk (cosine GEMM of
+    4096 x N_prior x 1024, top-32, reciprocal CSR insert, weights and the
+    in-edge transpose rebuilt).  Prior chunks grow by 4096 per step."""
+    import torch
+    import synth
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2607_05708_gb300 import MemStore
+    wl = synth.workload(3, scale=args.scale)
+    n_new = wl.new_emb.shape[0]
+    total = args.warmup + args.steps
+    store = MemStore.from_arrays(wl.emb, wl.page_of["clustered"], wl.row_ptr, wl.col, wl.aff,
+                                 capacity=wl.n + n_new * total, chunks_per_page=wl.chunks_per_page,
+                                 temperature=wl.tau, relation_scale=wl.relation_scale)
+    new = torch.from_numpy(np.ascontiguousarray(wl.new_emb).view(np.int16)).cuda()
+    st = torch.cuda.Stream()
+    times, flops = [], []
+    store.set_profiling(True)
+    with Clocks(0) as clk:
+        for i in range(total):
+            first = store.append_chunks(new, stream=st)
+            torch.cuda.synchronize()
+            e0 = torch.cuda.Event(enable_timing=True)
+            e1 = torch.cuda.Event(enable_timing=True)
+            e0.record(st)
+            store.update_relations(first, n_new, wl.top_m, True, stream=st)
+            e1.record(st)
+            torch.cuda.synchronize()
+            if i >= args.warmup:
+                times.append(e0.elapsed_time(e1))
+                flops.append(2.0 * n_new * first * wl.dim)
+            elif i == args.warmup - 1:
+                store.phase_times()
+    phases = store.phase_times()
+    hbm, bf16, kind = peaks()
+    ms = sum(times) / len(times)
+    fl = sum(flops) / len(flops)
+    relate_ms = phases["relate"][0] / len(times)
+    line = {
+        "metric": "relation update ms per 4096 new chunks (N=1M, d=1024, M=32); % of bf16 tensor peak",
+        "value": ms, "unit": "ms/update", "higher_is_better": False, "n_gpus": 1,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "dtype": "bf16",
+        "data": "synthetic",
+        "config": {"workload": f"update: gmm1m store + {n_new} new chunks, top-{wl.top_m}, reciprocal"
+                   + ("" if args.scale == 1.0 else f", scaled by {args.scale}")},
+        "roofline": {"bound": "tensor", "achieved": fl / (relate_ms * 1e-3) / 1e12, "peak": bf16,
+                     "unit": "TFLOP/s", "frac": fl / (relate_ms * 1e-3) / 1e12 / bf16,
+                     "traffic": None, "kernel": "relation GEMM + top-M (relate phase)",
+                     "peak_kind": kind},
+        "phases_ms_per_step": {p: phases[p][0] / len(times) for p in ("relate", "graph")},
+        "tensor_frac_of_whole_update": fl / (ms * 1e-3) / 1e12 / bf16,
+        "clocks": clk.summary(),
+    }
+    print(json.dumps(line), flush=True)
+    store.close()
+    return 0
+
+
+def run_streams(args):
+    """4M-chunk store, 1024 queries issued as 8 streams of 128 in a seeded
+    arrival order; aggregate queries/s over all streams."""
+    import torch
+    import synth
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2607_05708_gb300 import MemStore
+    wl = synth.workload(4, scale=args.scale)
+    store = MemStore.from_arrays(wl.emb, wl.page_of[args.placement], wl.row_ptr, wl.col, wl.aff,
+                                 capacity=wl.n, chunks_per_page=wl.chunks_per_page,
+                                 temperature=wl.tau)
+    per = wl.n_queries // wl.streams
+    streams = [torch.cuda.Stream() for _ in range(wl.streams)]
+    qs = [torch.from_numpy(np.ascontiguousarray(wl.queries[i * per:(i + 1) * per]).view(np.int16)).cuda()
+          for i in range(wl.streams)]
+    outs = [(torch.empty((per, wl.k), dtype=torch.int64, device="cuda"),
+             torch.empty((per, wl.k), dtype=torch.float32, device="cuda"),
+             torch.empty((per, wl.k), dtype=torch.int32, device="cuda"),
+             torch.empty((per,), dtype=torch.int32, device="cuda")) for _ in range(wl.streams)]
+
+    def step():
+        for i in wl.stream_order:
+            store.retrieve(qs[i], wl.k, wl.alpha, wl.hops, *outs[i], stream=streams[i])
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    main = torch.cuda.current_stream()
+    with Clocks(0) as clk:
+        t0.record(main)
+        for s in streams:
+            s.wait_stream(main)
+        for _ in range(args.steps):
+            step()
+        for s in streams:
+            main.wait_stream(s)
+        t1.record(main)
+        torch.cuda.synchronize()
+    ms = t0.elapsed_time(t1) / args.steps
+    store.sync()
+    pages = {}
+    for kind in wl.page_of:
+        po = wl.page_of[kind]
+        sel = np.concatenate([o[0].cpu().numpy() for o in outs])
+        pages[kind] = float(np.mean([len(set(po[r].tolist())) for r in sel]))
+    ab = algorithmic_bytes(wl.n, wl.dim, per, wl.nnz, wl.hops, wl.k)
+    hbm, bf16, kind = peaks()
+    line = {
+        "metric": "retrieve queries/sec at N=4M chunks, d=768, 8 streams x 128 queries",
+        "value": wl.n_queries / (ms * 1e-3), "unit": "queries/s", "higher_is_better": True,
+        "n_gpus": 1, "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms,
+        "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": "gmm4m: N=4194304 chunks, d=768, 16384-component Zipf(1.1) mixture, "
+                   "32-neighbour power-law graph, 8 streams x 128 queries (seeded arrival), "
+                   f"hops=2, alpha=0.4, k=64, 64 chunks/page, {args.placement} placement"
+                   + ("" if args.scale == 1.0 else f", scaled by {args.scale}")},
+        "pass_roofline": {"algorithmic_bytes_per_call": sum(ab.values()),
+                          "ideal_ms_all_calls": wl.streams * sum(ab.values()) / (hbm * 1e9) * 1e3},
+        "pages_per_query": pages,
+        "clocks": clk.summary(),
+    }
+    print(json.dumps(line), flush=True)
+    store.close()
+    return 0
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -197,9 +326,16 @@ def main():
     ap.add_argument("--placement", default="clustered")
     ap.add_argument("--scale", type=float, default=1.0,
                     help="shrink N (profiling captures of a smaller case); 1.0 = the benchmark")
+    ap.add_argument("--workload", default="retrieve", choices=["retrieve", "update", "streams"],
+                    help="retrieve: the benchmark; update: relation update of 4096 new chunks "
+                         "on the 1M-chunk store; streams: 4M-chunk store, 8 streams x 128 queries")
     args = ap.parse_args()
     if args.impl == "reference":
         return run_reference(args)
+    if args.workload == "update":
+        return run_update(args)
+    if args.workload == "streams":
+        return run_streams(args)
 
     import torch
     ws, rank, local = dist_env()

@@ -478,6 +478,14 @@ akashic_status_t akashic_mem_append_chunks(akashic_mem_t *m, const uint16_t *emb
     }
     m->n += n;
     m->nnz += new_nnz;
+    if (new_nnz == 0 && first > 0) {
+        // no new edges: the new rows have no in-edges, the transpose and the
+        // hub plan are unchanged; only the row pointers are extended
+        k_rebase_ptr<<<device_sm_count() * 4, 256, 0, st>>>(nullptr, m->in_ptr.as<int64_t>() + first + 1,
+                                                             n, m->nnz);
+        CUDA_TRY(cudaGetLastError());
+        return check_status(m, st, "append");
+    }
     AK_TRY(rebuild_in_edges(m, st));
     return AKASHIC_OK;
 }

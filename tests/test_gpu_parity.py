@@ -199,3 +199,50 @@ def test_capacity_and_bad_csr():
     assert st.append_chunks(t(wl.emb[:2], np.int16), None, t(rp, np.int64), t(col, np.int32),
                             t(aff, np.float32)) == 0
     assert st.size() == (2, 1)
+
+
+@pytest.fixture(scope="module")
+def update_full():
+    return synth.workload(3)
+
+
+def test_update_full_size_sampled(update_full):
+    """4096 new chunks linked into the N=1,048,576 store in one call (the
+    benchmark's update); the oracle recomputes 4 seeded new chunks (their
+    top-32 among all prior chunks, logits, reciprocal edges)."""
+    check_update(update_full, sample=4)
+
+
+def test_gmm4m_recipe_eight_concurrent_streams():
+    """gmm4m recipe at N=65536 (d=768, k=64, alpha=0.4): 1024 queries issued
+    as 8 streams of 128 in the seeded arrival order, all in flight at once
+    (each stream has its own scratch); 2 sampled queries per stream against
+    the oracle, and every stream's page counts within [ceil(k/P), k]."""
+    import torch
+    wl = synth.workload(4, scale=1 / 64)
+    store = gpu_store(wl, "clustered")
+    per = wl.n_queries // wl.streams
+    streams = [torch.cuda.Stream() for _ in range(wl.streams)]
+    outs = {}
+    for i in wl.stream_order:
+        q = torch.from_numpy(np.ascontiguousarray(wl.queries[i * per:(i + 1) * per]).view(np.int16)).cuda()
+        torch.cuda.current_stream().synchronize()
+        outs[i] = store.retrieve(q, wl.k, wl.alpha, wl.hops, stream=streams[i]) + (q,)
+    torch.cuda.synchronize()
+    store.sync()
+    rng = np.random.default_rng(7)
+    rows = []
+    got = {"ids": [], "scores": [], "page_ids": [], "n_pages": []}
+    for i in range(wl.streams):
+        ids, sc, pg, npg, _ = outs[i]
+        for r in sorted(rng.choice(per, size=2, replace=False)):
+            rows.append(i * per + r)
+            got["ids"].append(ids[r].cpu().numpy())
+            got["scores"].append(sc[r].cpu().numpy())
+            got["page_ids"].append(pg[r].cpu().numpy())
+            got["n_pages"].append(int(npg[r]))
+        assert (npg.cpu().numpy() <= wl.k).all()
+        assert (npg.cpu().numpy() >= 1).all()
+    got = {k: np.array(v) for k, v in got.items()}
+    ref = oracle_retrieve(wl, "clustered", queries=wl.queries[rows])
+    assert_retrieval_parity(wl, "clustered", got, ref)
