@@ -63,10 +63,20 @@ cudaError_t launch_score(const uint16_t *emb, int64_t n, int dim, const uint16_t
                          const float *shift, float tau, float *u, float *zpart, int *status,
                          cudaStream_t st, int *launches, int *zrows);
 
-// Plain dot products out[j, c] = <e_j, q_c> (bf16 tensor cores, fp32
-// accumulate), row stride bp.
-cudaError_t launch_dots(const uint16_t *emb, int64_t n, int dim, const uint16_t *qp, int bp,
-                        float *out, int *status, cudaStream_t st, int *launches);
+// Plain dot products out[j, c] = <e_{j*row_stride}, q_c> (bf16 tensor
+// cores, fp32 accumulate) for j < n, row stride bp in out.
+cudaError_t launch_dots(const uint16_t *emb, int64_t n, int64_t row_stride_rows, int dim,
+                        const uint16_t *qp, int bp, float *out, int *status, cudaStream_t st,
+                        int *launches);
+// Fused relation top-M filter: dots of every row j < n against the
+// n_ctiles*256 rows of qp; the selection key (signed dot, chunk ID
+// ext_of[j]) of every (j, c) with c < n_cols and ext_of[j] < id_limit that
+// is >= bound[c] is appended to buf[c][...] (count cnt[c], capacity cap).
+cudaError_t launch_dots_filter(const uint16_t *emb, int64_t n, int dim, const uint16_t *qp,
+                               int n_ctiles, int64_t n_cols, const int32_t *ext_of,
+                               int64_t id_limit, const unsigned long long *bound,
+                               unsigned int *cnt, unsigned long long *buf, int64_t cap,
+                               int *status, cudaStream_t st, int *launches);
 
 // Query preparation: pad q (b rows) to bp rows of zeros and compute
 // shift[c] = tau * |q_c| * max_norm (0 for padding); flags ERANGE.
@@ -176,7 +186,8 @@ struct SelectPlan {
     int64_t cap;        // buffer capacity per column
     int64_t off_bound, off_cnt, off_buf, words;
 };
-SelectPlan select_plan(int64_t n, int bp, int k, int sm_count);
+// force_stride > 0 samples every force_stride-th row instead of the default.
+SelectPlan select_plan(int64_t n, int bp, int k, int sm_count, int64_t force_stride = 0);
 
 // Retrieval: rows are store rows; keys and outputs carry chunk IDs
 // (ext_of), so ties resolve to the lower chunk ID; page_row is indexed by
@@ -193,5 +204,15 @@ cudaError_t launch_select_signed(const SelectPlan &sp, const float *s, int b,
                                  unsigned long long *ws, const int32_t *ext_of, int64_t id_limit,
                                  int64_t c_base, int32_t *nbr_ids, float *nbr_cos, int *status,
                                  cudaStream_t st, int *launches);
+// Bound pass alone over signed values: bound[c] for the b real columns
+// (the k-th largest sampled key; padding columns get an all-ones bound).
+cudaError_t launch_sample_bound_signed(const SelectPlan &sp, const float *s, int b,
+                                       const int32_t *ext_of, int64_t id_limit,
+                                       unsigned long long *ws, unsigned long long *bound,
+                                       cudaStream_t st, int *launches);
+// Top-k of each column's filter buffer (no overflow): nbr rows 0..n_cols-1.
+cudaError_t launch_buf_merge_signed(const unsigned int *cnt, const unsigned long long *buf,
+                                    int64_t cap, int64_t n_cols, int k, int32_t *nbr_ids,
+                                    float *nbr_cos, int *status, cudaStream_t st, int *launches);
 
 }  // namespace ak

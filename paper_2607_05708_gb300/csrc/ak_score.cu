@@ -106,15 +106,38 @@ cudaError_t make_tmap_2d(CUtensorMap *map, const void *base, CUtensorMapDataType
 }
 
 // ------------------------------------------------------------------ tcgen05 GEMM
-// C[j, c] = <e_j, q_c> for a 128-row tile of E against all BP (<= 256)
-// query rows, on the 5th-generation tensor cores: bf16 operands staged by
-// TMA in the 128-byte swizzle layout, fp32 accumulator in tensor memory
-// (two accumulators, so the epilogue of one tile overlaps the MMAs of the
-// next), persistent CTAs walking the tiles round-robin.
+// C[j, c] = <e_j, q_c> for 128-row tiles of E against column tiles of BP
+// (<= 256) query rows, on the 5th-generation tensor cores: bf16 operands
+// staged by TMA in the 128-byte swizzle layout, fp32 accumulator in tensor
+// memory (two accumulators, so the epilogue of one tile overlaps the MMAs of
+// the next), persistent CTAs walking the tiles round-robin, column tiles
+// innermost (the CTAs working at one time share the row tiles they read in
+// L2).
 //   warp 0     TMA producer (one thread)
 //   warp 1     TMEM owner and MMA issuer (one thread)
-//   warps 2-5  epilogue: TMEM -> registers -> (EXP: exp(tau*acc - shift),
-//              column sums toward Z) -> swizzled staging -> TMA store
+//   warps 2-5  epilogue, by mode:
+//     GEMM_EXP     exp(tau*acc - shift), column sums toward Z, swizzled
+//                  staging, TMA store (the score step)
+//     GEMM_RAW     the dots themselves, TMA store
+//     GEMM_FILTER  no store: every dot whose selection key clears its
+//                  column's bound is appended to that column's buffer (the
+//                  fused relation top-M)
+enum GemmMode { GEMM_EXP = 0, GEMM_RAW = 1, GEMM_FILTER = 2 };
+
+struct GemmEpi {
+    const float *shift;                 // EXP: [BP]
+    float tau;                          // EXP
+    float *zpart;                       // EXP: [gridDim][BP]
+    int *status;
+    int64_t n_cols;                     // FILTER: real columns (new chunks)
+    const int32_t *ext_of;              // FILTER: chunk ID of each row
+    int64_t id_limit;                   // FILTER: rows with chunk ID >= limit are skipped
+    const unsigned long long *bound;    // FILTER: [n_cols]
+    unsigned int *cnt;                  // FILTER: [n_cols]
+    unsigned long long *buf;            // FILTER: [n_cols][cap]
+    int64_t cap;
+};
+
 template <int BP>
 struct GemmCfg {
     static constexpr int BM = 128, BK = 64;
@@ -132,14 +155,15 @@ struct GemmCfg {
     static_assert(STAGES >= 2, "not enough shared memory for two stages");
 };
 
-template <int BP, bool EXP>
+template <int BP, int MODE>
 __global__ __launch_bounds__(192, 1) void k_gemm_umma(const __grid_constant__ CUtensorMap tmA,
                                                       const __grid_constant__ CUtensorMap tmB,
                                                       const __grid_constant__ CUtensorMap tmC,
-                                                      int64_t n_rows, int dim,
-                                                      const float *__restrict__ shift_g, float tau,
-                                                      float *__restrict__ zpart, int *status) {
+                                                      int64_t n_rows, int dim, int n_ctiles,
+                                                      const GemmEpi ep) {
     using C = GemmCfg<BP>;
+    constexpr bool EXP = MODE == GEMM_EXP;
+    constexpr bool FILTER = MODE == GEMM_FILTER;
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = (uint8_t *)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
     uint8_t *sA = smem;
@@ -154,10 +178,13 @@ __global__ __launch_bounds__(192, 1) void k_gemm_umma(const __grid_constant__ CU
     uint64_t *full = bars, *empty = bars + C::STAGES;
     uint64_t *tfull = bars + 2 * C::STAGES, *tempty = tfull + 2;
     uint32_t *tmem_slot = (uint32_t *)(tempty + 2);
+    unsigned long long *bnd_s = (unsigned long long *)sOut;   // FILTER: the tile's column bounds
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int64_t n_tiles = (n_rows + C::BM - 1) / C::BM;
+    const int64_t m_tiles = (n_rows + C::BM - 1) / C::BM;
+    const int64_t n_tiles = m_tiles * n_ctiles;
     const int kb_n = dim / C::BK;
+    int *status = ep.status;
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < C::STAGES; ++s) {
@@ -175,7 +202,7 @@ __global__ __launch_bounds__(192, 1) void k_gemm_umma(const __grid_constant__ CU
         tmem_relinquish();
     }
     for (int i = threadIdx.x; i < BP; i += blockDim.x) {
-        shift_s[i] = EXP ? shift_g[i] : 0.f;
+        shift_s[i] = EXP ? ep.shift[i] : 0.f;
         zacc[i] = 0.f;
     }
     tc_fence_before();
@@ -191,6 +218,7 @@ __global__ __launch_bounds__(192, 1) void k_gemm_umma(const __grid_constant__ CU
             for (int s = 0; s < 8; ++s) last_par[s] = -1;
             bool ok = true;
             for (int64_t t = blockIdx.x; t < n_tiles && ok; t += gridDim.x) {
+                const int64_t mt = t / n_ctiles, ct = t % n_ctiles;
                 for (int kb = 0; kb < kb_n; ++kb) {
                     if (!mbar_wait(&empty[stage], phase ^ 1u, status)) {
                         ok = false;
@@ -198,8 +226,9 @@ __global__ __launch_bounds__(192, 1) void k_gemm_umma(const __grid_constant__ CU
                     }
                     mbar_expect_tx(&full[stage], C::STAGE_BYTES);
                     tma_load_2d(sA + stage * C::A_BYTES, &tmA, &full[stage], kb * C::BK,
-                                (int)(t * C::BM));
-                    tma_load_2d(sB + stage * C::B_BYTES, &tmB, &full[stage], kb * C::BK, 0);
+                                (int)(mt * C::BM));
+                    tma_load_2d(sB + stage * C::B_BYTES, &tmB, &full[stage], kb * C::BK,
+                                (int)(ct * BP));
                     last_par[stage] = (int)phase;
                     if (++stage == (uint32_t)C::STAGES) {
                         stage = 0;
@@ -254,25 +283,54 @@ __global__ __launch_bounds__(192, 1) void k_gemm_umma(const __grid_constant__ CU
         const int et = threadIdx.x - 64;                 // 0..127
         int it = 0, cc = 0;
         for (int64_t t = blockIdx.x; t < n_tiles; t += gridDim.x, ++it) {
+            const int64_t mt = t / n_ctiles, ct = t % n_ctiles;
             const int acc = it & 1;
             const uint32_t aph = (uint32_t)(it >> 1) & 1u;
             // one thread polls, the barrier makes the outcome uniform
             if (et == 0) *go = mbar_wait(&tfull[acc], aph, status) ? 1 : 0;
+            if (FILTER) {
+                for (int c = et; c < BP; c += 128) {
+                    const int64_t cg = ct * BP + c;
+                    bnd_s[c] = cg < ep.n_cols ? ep.bound[cg] : ~0ull;
+                }
+            }
             named_bar(1, 128);
             if (!*go) break;
             tc_fence_after();
-            const bool valid = t * C::BM + row < n_rows;
+            const int64_t grow = mt * C::BM + row;
+            const bool valid = grow < n_rows;
+            uint32_t fid = 0;
+            bool fok = false;
+            if (FILTER && valid) {
+                const int32_t id = ep.ext_of[grow];
+                fok = (int64_t)id < ep.id_limit;
+                fid = ~(uint32_t)id;
+            }
 #pragma unroll 1
             for (int ch = 0; ch < BP / 32; ++ch, ++cc) {
                 const int buf = cc & 1;
                 uint32_t r[32];
                 tmem_ld32(tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * BP + ch * 32), r);
                 tmem_ld_wait();
+                if constexpr (FILTER) {
+                    if (fok) {
+#pragma unroll
+                        for (int i = 0; i < 32; ++i) {
+                            const unsigned long long key =
+                                ((unsigned long long)ordered_bits(__uint_as_float(r[i])) << 32) | fid;
+                            if (key >= bnd_s[ch * 32 + i]) {
+                                const int64_t cg = ct * BP + ch * 32 + i;
+                                const unsigned int p = atomicAdd(&ep.cnt[cg], 1u);
+                                if ((int64_t)p < ep.cap) ep.buf[cg * ep.cap + p] = key;
+                            }
+                        }
+                    }
+                } else {
                 float v[32];
 #pragma unroll
                 for (int i = 0; i < 32; ++i) {
                     const float x = __uint_as_float(r[i]);
-                    v[i] = valid ? (EXP ? expf(tau * x - shift_s[ch * 32 + i]) : x) : 0.f;
+                    v[i] = valid ? (EXP ? expf(ep.tau * x - shift_s[ch * 32 + i]) : x) : 0.f;
                 }
                 named_bar(1, 128);                       // staging[buf] free again
                 float4 *dst = (float4 *)(sOut + buf * (C::OUT_BYTES / 4) + row * 32);
@@ -291,7 +349,8 @@ __global__ __launch_bounds__(192, 1) void k_gemm_umma(const __grid_constant__ CU
                     zq[g * 32 + c] = s;
                 }
                 if (et == 0) {
-                    tma_store_2d(&tmC, sOut + buf * (C::OUT_BYTES / 4), ch * 32, (int)(t * C::BM));
+                    tma_store_2d(&tmC, sOut + buf * (C::OUT_BYTES / 4), (int)(ct * BP + ch * 32),
+                                 (int)(mt * C::BM));
                     bulk_commit();
                 }
                 if (EXP) {
@@ -299,6 +358,7 @@ __global__ __launch_bounds__(192, 1) void k_gemm_umma(const __grid_constant__ CU
                     if (et < 32) zacc[ch * 32 + et] += (zq[et] + zq[32 + et]) + (zq[64 + et] + zq[96 + et]);
                 }
                 if (et == 0) bulk_wait_read<1>();
+                }
             }
             tc_fence_before();
             named_bar(1, 128);
@@ -306,8 +366,8 @@ __global__ __launch_bounds__(192, 1) void k_gemm_umma(const __grid_constant__ CU
         }
         if (et == 0) bulk_wait_all();
         named_bar(1, 128);
-        if (EXP && zpart)
-            for (int c = et; c < BP; c += 128) zpart[(int64_t)blockIdx.x * BP + c] = zacc[c];
+        if (EXP && ep.zpart)
+            for (int c = et; c < BP; c += 128) ep.zpart[(int64_t)blockIdx.x * BP + c] = zacc[c];
     }
     tc_fence_before();
     __syncthreads();
@@ -317,47 +377,51 @@ __global__ __launch_bounds__(192, 1) void k_gemm_umma(const __grid_constant__ CU
 
 int64_t score_tiles(int64_t n) { return ceil_div<int64_t>(n, 128); }
 
-template <int BP, bool EXP>
-static cudaError_t gemm_bp(const uint16_t *emb, int64_t n, int dim, const uint16_t *qp,
-                           const float *shift, float tau, float *out, float *zpart, int *status,
+// A: E rows (row_stride_rows apart: 1 = every row, s = every s-th row),
+// B: n_ctiles * BP query rows, C: output [n_rows][n_ctiles * BP] (EXP/RAW).
+template <int BP, int MODE>
+static cudaError_t gemm_bp(const uint16_t *emb, int64_t n_rows, int64_t row_stride_rows, int dim,
+                           const uint16_t *qp, int n_ctiles, float *out, const GemmEpi &ep,
                            cudaStream_t st, int *zrows) {
     using C = GemmCfg<BP>;
     static bool attr[64] = {false};
     int dev = 0;
     cudaGetDevice(&dev);
     if (dev >= 0 && dev < 64 && !attr[dev]) {
-        cudaError_t e = cudaFuncSetAttribute(k_gemm_umma<BP, EXP>,
+        cudaError_t e = cudaFuncSetAttribute(k_gemm_umma<BP, MODE>,
                                              cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
         if (e != cudaSuccess) return e;
         attr[dev] = true;
     }
     CUtensorMap ta, tb, tc;
     cudaError_t e = make_tmap_2d(&ta, emb, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, (uint64_t)dim,
-                                 (uint64_t)n, (uint64_t)dim * 2, 64, 128);
+                                 (uint64_t)n_rows, (uint64_t)dim * 2 * row_stride_rows, 64, 128);
     if (e == cudaSuccess)
-        e = make_tmap_2d(&tb, qp, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, (uint64_t)dim, (uint64_t)BP,
-                         (uint64_t)dim * 2, 64, BP);
-    if (e == cudaSuccess)
-        e = make_tmap_2d(&tc, out, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, (uint64_t)BP, (uint64_t)n,
-                         (uint64_t)BP * 4, 32, 128);
+        e = make_tmap_2d(&tb, qp, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, (uint64_t)dim,
+                         (uint64_t)n_ctiles * BP, (uint64_t)dim * 2, 64, BP);
+    if (e == cudaSuccess && MODE != GEMM_FILTER)
+        e = make_tmap_2d(&tc, out, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, (uint64_t)n_ctiles * BP,
+                         (uint64_t)n_rows, (uint64_t)n_ctiles * BP * 4, 32, 128);
+    else
+        tc = ta;   // unused by the filter epilogue
     if (e != cudaSuccess) return e;
-    const int64_t tiles = ceil_div<int64_t>(n, 128);
+    const int64_t tiles = ceil_div<int64_t>(n_rows, 128) * n_ctiles;
     const int grid = (int)(tiles < device_sm_count() ? tiles : device_sm_count());
-    k_gemm_umma<BP, EXP><<<grid, 192, C::SMEM, st>>>(ta, tb, tc, n, dim, shift, tau, zpart, status);
+    k_gemm_umma<BP, MODE><<<grid, 192, C::SMEM, st>>>(ta, tb, tc, n_rows, dim, n_ctiles, ep);
     if (zrows) *zrows = grid;
     return cudaGetLastError();
 }
 
-template <bool EXP>
-static cudaError_t gemm_dispatch(const uint16_t *emb, int64_t n, int dim, const uint16_t *qp,
-                                 int bp, const float *shift, float tau, float *out, float *zpart,
-                                 int *status, cudaStream_t st, int *zrows) {
-    if (n <= 0 || dim % 64 != 0) return cudaErrorInvalidValue;
+template <int MODE>
+static cudaError_t gemm_dispatch(const uint16_t *emb, int64_t n_rows, int64_t row_stride_rows,
+                                 int dim, const uint16_t *qp, int bp, int n_ctiles, float *out,
+                                 const GemmEpi &ep, cudaStream_t st, int *zrows) {
+    if (n_rows <= 0 || dim % 64 != 0 || n_ctiles < 1) return cudaErrorInvalidValue;
     switch (bp) {
-    case 32: return gemm_bp<32, EXP>(emb, n, dim, qp, shift, tau, out, zpart, status, st, zrows);
-    case 64: return gemm_bp<64, EXP>(emb, n, dim, qp, shift, tau, out, zpart, status, st, zrows);
-    case 128: return gemm_bp<128, EXP>(emb, n, dim, qp, shift, tau, out, zpart, status, st, zrows);
-    case 256: return gemm_bp<256, EXP>(emb, n, dim, qp, shift, tau, out, zpart, status, st, zrows);
+    case 32: return gemm_bp<32, MODE>(emb, n_rows, row_stride_rows, dim, qp, n_ctiles, out, ep, st, zrows);
+    case 64: return gemm_bp<64, MODE>(emb, n_rows, row_stride_rows, dim, qp, n_ctiles, out, ep, st, zrows);
+    case 128: return gemm_bp<128, MODE>(emb, n_rows, row_stride_rows, dim, qp, n_ctiles, out, ep, st, zrows);
+    case 256: return gemm_bp<256, MODE>(emb, n_rows, row_stride_rows, dim, qp, n_ctiles, out, ep, st, zrows);
     default: return cudaErrorInvalidValue;
     }
 }
@@ -365,15 +429,43 @@ static cudaError_t gemm_dispatch(const uint16_t *emb, int64_t n, int dim, const 
 cudaError_t launch_score(const uint16_t *emb, int64_t n, int dim, const uint16_t *qp, int bp,
                          const float *shift, float tau, float *u, float *zpart, int *status,
                          cudaStream_t st, int *launches, int *zrows) {
-    cudaError_t e = gemm_dispatch<true>(emb, n, dim, qp, bp, shift, tau, u, zpart, status, st, zrows);
+    GemmEpi ep{};
+    ep.shift = shift;
+    ep.tau = tau;
+    ep.zpart = zpart;
+    ep.status = status;
+    cudaError_t e = gemm_dispatch<GEMM_EXP>(emb, n, 1, dim, qp, bp, 1, u, ep, st, zrows);
     if (launches) *launches += 1;
     return e;
 }
 
-cudaError_t launch_dots(const uint16_t *emb, int64_t n, int dim, const uint16_t *qp, int bp,
-                        float *out, int *status, cudaStream_t st, int *launches) {
-    cudaError_t e = gemm_dispatch<false>(emb, n, dim, qp, bp, nullptr, 1.f, out, nullptr, status,
-                                         st, nullptr);
+cudaError_t launch_dots(const uint16_t *emb, int64_t n, int64_t row_stride_rows, int dim,
+                        const uint16_t *qp, int bp, float *out, int *status, cudaStream_t st,
+                        int *launches) {
+    GemmEpi ep{};
+    ep.status = status;
+    cudaError_t e = gemm_dispatch<GEMM_RAW>(emb, n, row_stride_rows, dim, qp, bp, 1, out, ep, st,
+                                            nullptr);
+    if (launches) *launches += 1;
+    return e;
+}
+
+cudaError_t launch_dots_filter(const uint16_t *emb, int64_t n, int dim, const uint16_t *qp,
+                               int n_ctiles, int64_t n_cols, const int32_t *ext_of,
+                               int64_t id_limit, const unsigned long long *bound,
+                               unsigned int *cnt, unsigned long long *buf, int64_t cap,
+                               int *status, cudaStream_t st, int *launches) {
+    GemmEpi ep{};
+    ep.status = status;
+    ep.n_cols = n_cols;
+    ep.ext_of = ext_of;
+    ep.id_limit = id_limit;
+    ep.bound = bound;
+    ep.cnt = cnt;
+    ep.buf = buf;
+    ep.cap = cap;
+    cudaError_t e = gemm_dispatch<GEMM_FILTER>(emb, n, 1, dim, qp, 256, n_ctiles, nullptr, ep, st,
+                                               nullptr);
     if (launches) *launches += 1;
     return e;
 }

@@ -36,7 +36,7 @@ __device__ __forceinline__ float sel_value(unsigned long long key) {
 }
 
 // ------------------------------------------------------------------ plan
-SelectPlan select_plan(int64_t n, int bp, int k, int sm_count) {
+SelectPlan select_plan(int64_t n, int bp, int k, int sm_count, int64_t force_stride) {
     SelectPlan sp;
     sp.n = n;
     sp.bp = bp;
@@ -44,6 +44,7 @@ SelectPlan select_plan(int64_t n, int bp, int k, int sm_count) {
     // sample every stride-th row, at least 64 k rows (all rows of a small store)
     int64_t stride = n / ((int64_t)64 * k);
     stride = stride < 1 ? 1 : (stride > 32 ? 32 : stride);
+    if (force_stride > 0) stride = force_stride;
     sp.stride = stride;
     sp.n_sample = ceil_div<int64_t>(n, stride);
     sp.lanes = SEL_THREADS / bp > 0 ? SEL_THREADS / bp : 1;
@@ -82,28 +83,32 @@ __device__ void radix_select(int64_t total, int k, KeyAt key_at, unsigned long l
         for (int w = 0; w < SEL_THREADS / 32; ++w) hist[w * 256 + tid] = 0;
         __syncthreads();
         const unsigned long long prefix = *s_prefix;
+        const int rem = *s_remaining;   // read before any thread can update it below
         for (int64_t i = tid; i < total; i += SEL_THREADS) {
             const unsigned long long key = key_at(i);
             if ((key & pmask) == prefix) atomicAdd(&hist[warp * 256 + ((key >> sh) & 0xff)], 1);
         }
         __syncthreads();
-        {
-            int sum = 0;
-            for (int w = 0; w < SEL_THREADS / 32; ++w) sum += hist[w * 256 + tid];
-            hist[tid] = sum;   // warp 0's row now holds the totals
+        // digit 255 - tid: its count and the inclusive count of all larger
+        // digits (block-wide prefix sum), then the one thread whose range
+        // holds the remaining rank records the digit
+        int cntd = 0;
+        for (int w = 0; w < SEL_THREADS / 32; ++w) cntd += hist[w * 256 + (255 - tid)];
+        int incl = cntd;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int t = __shfl_up_sync(0xffffffffu, incl, o);
+            if ((tid & 31) >= o) incl += t;
         }
         __syncthreads();
-        if (tid == 0) {
-            int rem = *s_remaining, cum = 0, sel = 0;
-            for (int d = 255; d >= 0; --d) {
-                if (cum + hist[d] >= rem) {
-                    sel = d;
-                    break;
-                }
-                cum += hist[d];
-            }
-            *s_remaining = rem - cum;
-            *s_prefix = prefix | ((unsigned long long)sel << sh);
+        if ((tid & 31) == 31) hist[tid >> 5] = incl;   // warp totals (hist is free now)
+        __syncthreads();
+        int before = 0;
+        for (int w = 0; w < (tid >> 5); ++w) before += hist[w];
+        incl += before;
+        if (incl >= rem && incl - cntd < rem) {
+            *s_remaining = rem - (incl - cntd);
+            *s_prefix = prefix | ((unsigned long long)(255 - tid) << sh);
         }
         pmask |= 0xffull << sh;
         __syncthreads();
@@ -373,6 +378,50 @@ __global__ __launch_bounds__(SEL_THREADS) void k_topm_merge(
     }
 }
 
+// Relation top-M from the fused filter's buffers alone (one CTA per new
+// chunk c; the caller has checked that no buffer overflowed).
+__global__ __launch_bounds__(SEL_THREADS) void k_buf_merge_signed(
+    const unsigned int *__restrict__ cnt, const unsigned long long *__restrict__ buf, int64_t cap,
+    int k, int32_t *__restrict__ nbr_ids, float *__restrict__ nbr_cos, int *status) {
+    __shared__ int hist[256 * (SEL_THREADS / 32)];
+    __shared__ unsigned long long stage[SEL_STAGE];
+    __shared__ unsigned long long win[64];
+    __shared__ unsigned long long s_prefix;
+    __shared__ int s_remaining, win_n;
+    const int64_t c = blockIdx.x;
+    const int tid = threadIdx.x;
+    const int64_t m = cnt[c] < cap ? cnt[c] : cap;
+    const unsigned long long *bc = buf + c * cap;
+    if (m <= SEL_STAGE) {
+        for (int64_t i = tid; i < m; i += SEL_THREADS) stage[i] = bc[i];
+        __syncthreads();
+        auto key_at = [&](int64_t i) -> unsigned long long { return stage[i]; };
+        radix_select(m, k, key_at, win, &win_n, hist, &s_prefix, &s_remaining);
+    } else {
+        auto key_at = [&](int64_t i) -> unsigned long long { return bc[i]; };
+        radix_select(m, k, key_at, win, &win_n, hist, &s_prefix, &s_remaining);
+    }
+    if (tid == 0 && win_n != k) set_status(status, AKASHIC_EDEVICE);
+    const int got = win_n < k ? win_n : k;
+    if (tid < got) {
+        const unsigned long long key = win[tid];
+        int rank = 0;
+        for (int t = 0; t < got; ++t) rank += win[t] > key;
+        nbr_ids[c * k + rank] = (int32_t)key_id(key);
+        nbr_cos[c * k + rank] = sel_value<true>(key);
+    }
+}
+
+cudaError_t launch_buf_merge_signed(const unsigned int *cnt, const unsigned long long *buf,
+                                    int64_t cap, int64_t n_cols, int k, int32_t *nbr_ids,
+                                    float *nbr_cos, int *status, cudaStream_t st, int *launches) {
+    if (n_cols <= 0) return cudaSuccess;
+    k_buf_merge_signed<<<(unsigned)n_cols, SEL_THREADS, 0, st>>>(cnt, buf, cap, k, nbr_ids,
+                                                                 nbr_cos, status);
+    if (launches) *launches += 1;
+    return cudaGetLastError();
+}
+
 // ------------------------------------------------------------------ launchers
 template <bool SIGNED>
 static cudaError_t bound_and_filter(const SelectPlan &sp, const float *s, int b,
@@ -413,6 +462,32 @@ static cudaError_t bound_and_filter(const SelectPlan &sp, const float *s, int b,
     default: return cudaErrorInvalidValue;
     }
     if (launches) *launches += 3;
+    return cudaGetLastError();
+}
+
+cudaError_t launch_sample_bound_signed(const SelectPlan &sp, const float *s, int b,
+                                       const int32_t *ext_of, int64_t id_limit,
+                                       unsigned long long *ws, unsigned long long *bound,
+                                       cudaStream_t st, int *launches) {
+    static bool attr[64] = {false};
+    int dev = 0;
+    cudaGetDevice(&dev);
+    if (dev >= 0 && dev < 64 && !attr[dev]) {
+        cudaError_t e = cudaFuncSetAttribute(k_sample_heaps<true>,
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             64 * SEL_THREADS * (int)sizeof(unsigned long long));
+        if (e != cudaSuccess) return e;
+        attr[dev] = true;
+    }
+    const size_t smem = (size_t)sp.k * SEL_THREADS * sizeof(unsigned long long);
+    const int64_t rows_per_cta = ceil_div<int64_t>(sp.n_sample, sp.grid);
+    k_sample_heaps<true><<<sp.grid, SEL_THREADS, smem, st>>>(
+        s, sp.n_sample, sp.stride, sp.bp, sp.lanes, sp.k, rows_per_cta, ext_of, id_limit, ws);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    k_sample_bound<<<sp.bp, SEL_THREADS, 0, st>>>(ws, sp.lists, sp.bp, b, sp.k, bound,
+                                                  (unsigned int *)(ws + sp.off_cnt));
+    if (launches) *launches += 2;
     return cudaGetLastError();
 }
 

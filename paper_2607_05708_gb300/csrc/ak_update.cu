@@ -19,28 +19,32 @@ __global__ void k_gather_rows(const uint16_t *__restrict__ emb, const int32_t *_
     }
 }
 
-akashic_status_t relate_top_m(const UpdateArgs &a, cudaStream_t st, int *launches) {
-    // every row of the store is scored; rows holding chunks >= first are
-    // masked in the selection (rows are in page order, not ID order)
+__global__ void k_ext_sample(const int32_t *__restrict__ ext_of, int64_t n_sample, int64_t stride,
+                             int32_t *__restrict__ out) {
+    for (int64_t v = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; v < n_sample;
+         v += (int64_t)gridDim.x * blockDim.x)
+        out[v] = ext_of[v * stride];
+}
+
+// Exact path, batch by batch: dots of every row against 256 new chunks
+// written to a slab, then the three-pass selection (used when a fused
+// filter buffer overflows).
+static akashic_status_t relate_top_m_batched(const UpdateArgs &a, cudaStream_t st, int *launches) {
     const int64_t n_old = a.n_rows;
     int bp_max = 32;
     while (bp_max < 256 && bp_max < a.n_new) bp_max <<= 1;
     uint16_t *qp = nullptr;
     float *dots = nullptr;
     unsigned long long *cand = nullptr;
-    const SelectPlan sp_max = select_plan(n_old, bp_max, a.M, device_sm_count());
     cudaError_t e = cudaMalloc(&qp, (size_t)bp_max * a.dim * 2);
     if (e == cudaSuccess) e = cudaMalloc(&dots, (size_t)n_old * bp_max * 4);
     if (e == cudaSuccess) {
-        // lists for the smallest bp are the most numerous; size for the worst case
-        int64_t lists = 0;
+        int64_t words = 0;
         for (int bp = 32; bp <= bp_max; bp <<= 1) {
             SelectPlan sp = select_plan(n_old, bp, a.M, device_sm_count());
-            int64_t need = sp.words;
-            lists = need > lists ? need : lists;
+            words = sp.words > words ? sp.words : words;
         }
-        (void)sp_max;
-        e = cudaMalloc(&cand, (size_t)lists * 8);
+        e = cudaMalloc(&cand, (size_t)words * 8);
     }
     akashic_status_t rc = AKASHIC_OK;
     if (e != cudaSuccess) {
@@ -55,7 +59,7 @@ akashic_status_t relate_top_m(const UpdateArgs &a, cudaStream_t st, int *launche
                                                           a.dim, qp);
         e = cudaGetLastError();
         if (e == cudaSuccess)
-            e = launch_dots(a.emb, n_old, a.dim, qp, bp, dots, a.status, st, launches);
+            e = launch_dots(a.emb, n_old, 1, a.dim, qp, bp, dots, a.status, st, launches);
         const SelectPlan sp = select_plan(n_old, bp, a.M, device_sm_count());
         if (e == cudaSuccess)
             e = launch_select_signed(sp, dots, b, cand, a.ext_of, a.first, off, a.nbr_ids,
@@ -67,6 +71,89 @@ akashic_status_t relate_top_m(const UpdateArgs &a, cudaStream_t st, int *launche
     cudaFree(qp);
     cudaFree(dots);
     cudaFree(cand);
+    return rc;
+}
+
+// Fused path (a6): a per-new-chunk bound from every stride-th row of the
+// store, then ONE tensor-core pass over all rows x all new chunks whose
+// epilogue keeps only the keys above the bounds, then an exact selection
+// of the M best among them.  The dots are never written to memory.
+akashic_status_t relate_top_m(const UpdateArgs &a, cudaStream_t st, int *launches) {
+    // every row of the store is scored; rows holding chunks >= first are
+    // masked in the selection (rows are in page order, not ID order)
+    const int64_t n = a.n_rows;
+    const int sms = device_sm_count();
+    const int n_ct = (int)ceil_div<int64_t>(a.n_new, 256);
+    const int64_t n_pad = (int64_t)n_ct * 256;
+    int64_t stride = n / ((int64_t)64 * a.M);
+    stride = stride < 1 ? 1 : (stride > 32 ? 32 : stride);
+    const int64_t n_sample = ceil_div<int64_t>(n, stride);
+    const int64_t cap = 4 * (int64_t)a.M * stride > 8192 ? 4 * (int64_t)a.M * stride : 8192;
+    const SelectPlan sp = select_plan(n_sample, 256, a.M, sms, 1);
+    uint16_t *qp = nullptr;
+    float *sdots = nullptr;
+    int32_t *ext_s = nullptr;
+    unsigned long long *ws = nullptr, *bound = nullptr, *buf = nullptr;
+    unsigned int *cnt = nullptr;
+    cudaError_t e = cudaMalloc(&qp, (size_t)n_pad * a.dim * 2);
+    if (e == cudaSuccess) e = cudaMalloc(&sdots, (size_t)n_sample * 256 * 4);
+    if (e == cudaSuccess) e = cudaMalloc(&ext_s, (size_t)n_sample * 4);
+    if (e == cudaSuccess) e = cudaMalloc(&ws, (size_t)sp.words * 8);
+    if (e == cudaSuccess) e = cudaMalloc(&bound, (size_t)n_pad * 8);
+    if (e == cudaSuccess) e = cudaMalloc(&cnt, (size_t)n_pad * 4);
+    if (e == cudaSuccess) e = cudaMalloc(&buf, (size_t)a.n_new * cap * 8);
+    akashic_status_t rc = AKASHIC_OK;
+    if (e != cudaSuccess) {
+        cudaGetLastError();
+        rc = AKASHIC_ENOMEM;
+    }
+    bool overflow = false;
+    if (rc == AKASHIC_OK) {
+        k_gather_rows<<<sms * 2, 256, 0, st>>>(a.emb, a.row_of, a.first, (int)a.n_new, (int)n_pad,
+                                               a.dim, qp);
+        k_ext_sample<<<sms, 256, 0, st>>>(a.ext_of, n_sample, stride, ext_s);
+        e = cudaGetLastError();
+        for (int ct = 0; e == cudaSuccess && ct < n_ct; ++ct) {
+            const int b = (int)(a.n_new - (int64_t)ct * 256 < 256 ? a.n_new - (int64_t)ct * 256 : 256);
+            e = launch_dots(a.emb, n_sample, stride, a.dim, qp + (int64_t)ct * 256 * a.dim, 256,
+                            sdots, a.status, st, launches);
+            if (e == cudaSuccess)
+                e = launch_sample_bound_signed(sp, sdots, b, ext_s, a.first, ws,
+                                               bound + (int64_t)ct * 256, st, launches);
+        }
+        if (e == cudaSuccess) e = cudaMemsetAsync(cnt, 0, (size_t)n_pad * 4, st);
+        if (e == cudaSuccess)
+            e = launch_dots_filter(a.emb, n, a.dim, qp, n_ct, a.n_new, a.ext_of, a.first, bound,
+                                   cnt, buf, cap, a.status, st, launches);
+        // buffers that overflowed fall back to the exact batched path
+        unsigned int max_cnt = 0;
+        if (e == cudaSuccess) {
+            unsigned int *h = (unsigned int *)malloc((size_t)a.n_new * 4);
+            if (!h) {
+                rc = AKASHIC_ENOMEM;
+            } else {
+                e = cudaMemcpyAsync(h, cnt, (size_t)a.n_new * 4, cudaMemcpyDeviceToHost, st);
+                if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+                for (int64_t c = 0; e == cudaSuccess && c < a.n_new; ++c)
+                    max_cnt = h[c] > max_cnt ? h[c] : max_cnt;
+                free(h);
+            }
+        }
+        overflow = (int64_t)max_cnt > cap;
+        if (e == cudaSuccess && rc == AKASHIC_OK && !overflow)
+            e = launch_buf_merge_signed(cnt, buf, cap, a.n_new, a.M, a.nbr_ids, a.nbr_cos,
+                                        a.status, st, launches);
+        if (e == cudaSuccess && rc == AKASHIC_OK) e = cudaStreamSynchronize(st);
+        if (e != cudaSuccess && rc == AKASHIC_OK) rc = AKASHIC_ECUDA;
+    }
+    cudaFree(qp);
+    cudaFree(sdots);
+    cudaFree(ext_s);
+    cudaFree(ws);
+    cudaFree(bound);
+    cudaFree(cnt);
+    cudaFree(buf);
+    if (rc == AKASHIC_OK && overflow) rc = relate_top_m_batched(a, st, launches);
     return rc;
 }
 
