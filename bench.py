@@ -63,6 +63,14 @@ def hop_bytes(n, b, nnz):
     return (n + 1) * 8 + nnz * 8 + 2 * n * b * 4
 
 
+# DRAM bytes per propagation hop on this workload (sum over the hop's three
+# kernels: hub segments, rows kept whole, hub fixup), from an ncu capture of
+# `bench.py --steps 2 --warmup 1 --no-cpu-baseline` with the
+# dram__bytes_read/write counters (mean of the two hops).  Set to None when
+# the hop kernels change until they are captured again.
+HOP_DRAM_BYTES = 11.5e9
+
+
 def score_bytes(n, d, b):
     return n * d * 2 + n * b * 4 + b * d * 2
 
@@ -118,17 +126,20 @@ class Clocks:
                 "samples": len(sm)}
 
 
-def cpu_baseline(wl, placement, n_queries, rng_seed=0):
+def cpu_baseline(wl, placement, n_queries, rng_seed=0, weights=None):
+    """The oracle retrieving n_queries of the batch against the full store on
+    one host thread (the relation weights, which the GPU store computes at
+    append time, are computed once beforehand)."""
     import oracle
+    w = weights if weights is not None else oracle.row_softmax(wl.row_ptr, wl.aff)
     rows = np.random.default_rng(rng_seed).choice(wl.n_queries, size=n_queries, replace=False)
     t0 = time.perf_counter()
-    w = oracle.row_softmax(wl.row_ptr, wl.aff)
     oracle.retrieve(wl.emb, wl.queries[rows], wl.row_ptr, wl.col, w, tau=wl.tau, alpha=wl.alpha,
                     hops=wl.hops, k=wl.k, page_of=wl.page_of[placement])
     dt = time.perf_counter() - t0
     return dict(value=n_queries / dt, unit="queries/s", cores=1, kind="oracle",
-                sample=f"{n_queries} of the {wl.n_queries} queries against the full store "
-                       f"(relation weights included), one thread",
+                sample=f"{n_queries} of the {wl.n_queries} queries against the full store, "
+                       f"one thread",
                 seconds=dt)
 
 
@@ -161,12 +172,14 @@ def run_reference(args):
     ws, rank, _ = dist_env()
     if rank != 0:
         return 0
+    import oracle
     import synth
     wl = synth.workload(2, placements=("clustered",))
+    w = oracle.row_softmax(wl.row_ptr, wl.aff)
     per_step = 1
     times = []
     for i in range(args.warmup + args.steps):
-        r = cpu_baseline(wl, "clustered", per_step, rng_seed=i)
+        r = cpu_baseline(wl, "clustered", per_step, rng_seed=i, weights=w)
         if i >= args.warmup:
             times.append(r["seconds"])
     tot = sum(times)
@@ -318,7 +331,9 @@ def run_streams(args):
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--steps", type=int, default=None,
+                    help="timed steps (default: 100 for retrieve and the reference arm, "
+                         "5 for update, 20 for streams)")
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="native", choices=["native", "reference"])
     ap.add_argument("--cpu-queries", type=int, default=8)
@@ -330,6 +345,8 @@ def main():
                     help="retrieve: the benchmark; update: relation update of 4096 new chunks "
                          "on the 1M-chunk store; streams: 4M-chunk store, 8 streams x 128 queries")
     args = ap.parse_args()
+    if args.steps is None:
+        args.steps = {"retrieve": 100, "update": 5, "streams": 20}[args.workload]
     if args.impl == "reference":
         return run_reference(args)
     if args.workload == "update":
@@ -472,8 +489,10 @@ def main():
                    "each), no flush", "placement": args.placement,
                    "parallelism": "replicas" if ws > 1 else "single GPU"},
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": hbm, "unit": "GB/s",
-                     "frac": achieved / hbm, "traffic": None, "kernel": dom, "what": what,
-                     "peak_kind": peak_kind},
+                     "frac": achieved / hbm,
+                     "traffic": (HOP_DRAM_BYTES if dom == "propagate" and args.scale == 1.0
+                                 else None),
+                     "kernel": dom, "what": what, "peak_kind": peak_kind},
         "pass_roofline": {"algorithmic_bytes": total_ab,
                           "ideal_ms": total_ab / (hbm * 1e9) * 1e3,
                           "frac": (total_ab / (hbm * 1e9) * 1e3) / per_step_ms,
