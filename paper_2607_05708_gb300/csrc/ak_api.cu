@@ -120,7 +120,7 @@ struct akashic_mem {
     DevBuf in_ptr, in_src, in_w;
     SplitParams split;
     int64_t n_split = 0, n_segs = 0;
-    DevBuf split_row, split_slot0, seg_e0, seg_e1, seg_slot;
+    DevBuf split_row, split_slot0, seg_e0, seg_e1, seg_slot, split_order;
     std::mutex mu;
     std::unordered_map<void *, StreamScratch *> scratch;
     // profiling
@@ -300,6 +300,15 @@ static akashic_status_t rebuild_in_edges(akashic_mem *m, cudaStream_t st) {
                                     e0.as<int64_t>(), e1.as<int64_t>(), n_segs,
                                     m->seg_e0.as<int64_t>(), m->seg_e1.as<int64_t>(),
                                     m->seg_slot.as<int32_t>(), st));
+        // split rows heaviest first (the hop's fixup order)
+        AK_TRY(m->split_order.ensure((size_t)n_split * 4));
+        CUDA_TRY(launch_split_keys(m->split_slot0.as<int64_t>(), n_split, win.as<uint32_t>(),
+                                   order.as<uint32_t>(), st));
+        bool alt2 = false;
+        CUDA_TRY(radix_sort_pairs(win.as<uint32_t>(), order.as<uint32_t>(), win2.as<uint32_t>(),
+                                  order2.as<uint32_t>(), n_split, 32, rtmp.p, rtmp.cap, st, &alt2));
+        CUDA_TRY(cudaMemcpyAsync(m->split_order.p, alt2 ? order2.p : order.p, (size_t)n_split * 4,
+                                 cudaMemcpyDeviceToDevice, st));
         AK_TRY(check_status(m, st, "relation graph rebuild"));
     }
     return check_status(m, st, "relation graph rebuild");
@@ -630,6 +639,7 @@ akashic_status_t akashic_mem_retrieve(akashic_mem_t *m, const uint16_t *q, int32
             hp.seg_e0 = m->seg_e0.as<int64_t>();
             hp.seg_e1 = m->seg_e1.as<int64_t>();
             hp.seg_slot = m->seg_slot.as<int32_t>();
+            hp.split_order = m->split_order.as<int32_t>();
             float *bufs[2] = {sc->sa.as<float>(), sc->sb.as<float>()};
             for (int h = 0; h < eff_hops; ++h) {
                 float *out = bufs[h & 1];

@@ -151,6 +151,10 @@ cudaError_t launch_seg_permute(const uint32_t *order, const int64_t *e0, const i
                                int64_t n_segs, int64_t *e0s, int64_t *e1s, int32_t *slot,
                                cudaStream_t st);
 
+// keys[r] = ~(slot count of split row r), vals[r] = r (sorted: heaviest first).
+cudaError_t launch_split_keys(const int64_t *slot0, int64_t n_split, uint32_t *keys,
+                              uint32_t *vals, cudaStream_t st);
+
 // Propagation hop (a2): out[j,:] = u[j,:] + alpha * sum_{i->j} w_ij * in[i,:].
 struct HopPlan {
     SplitParams split;
@@ -166,6 +170,7 @@ struct HopPlan {
     const int64_t *seg_e0;      // [n_segs] first edge, window-major order
     const int64_t *seg_e1;      // [n_segs] end edge
     const int32_t *seg_slot;    // [n_segs] partial slot (segments of a row are contiguous)
+    const int32_t *split_order; // [n_split_rows] split rows by slot count, largest first
 };
 // `counters` = 2 device ints, zeroed by the launcher (work queues).
 cudaError_t launch_hop(const HopPlan &p, const float *u, const float *in, float *out, int bp,

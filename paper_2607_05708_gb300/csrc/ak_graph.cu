@@ -504,6 +504,26 @@ cudaError_t launch_seg_permute(const uint32_t *order, const int64_t *e0, const i
     return cudaGetLastError();
 }
 
+// Split rows ordered by their number of partial slots, largest first (the
+// hop sums each split row's slots in one warp and hands the heaviest out
+// first, so that they finish early).  keys = ~count, so an ascending stable
+// sort gives descending counts with ties in row order.
+__global__ void k_split_keys(const int64_t *__restrict__ slot0, int64_t n_split,
+                             uint32_t *__restrict__ keys, uint32_t *__restrict__ vals) {
+    for (int64_t r = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; r < n_split;
+         r += (int64_t)gridDim.x * blockDim.x) {
+        keys[r] = ~(uint32_t)(slot0[r + 1] - slot0[r]);
+        vals[r] = (uint32_t)r;
+    }
+}
+
+cudaError_t launch_split_keys(const int64_t *slot0, int64_t n_split, uint32_t *keys,
+                              uint32_t *vals, cudaStream_t st) {
+    if (n_split <= 0) return cudaSuccess;
+    k_split_keys<<<device_sm_count(), 256, 0, st>>>(slot0, n_split, keys, vals);
+    return cudaGetLastError();
+}
+
 // ================================================================== propagation hop
 // out[j,:] = u[j,:] + alpha * sum_{i->j} w_ij in[i,:], gathered over the
 // in-edge CSR, one warp per destination row.  A row holds BP fp32 values
@@ -623,9 +643,68 @@ __device__ __forceinline__ void hop_accumulate(const int32_t *__restrict__ in_sr
     }
 }
 
-// Rows kept whole: warps claim ROWS_PER_GRAB consecutive rows at a time from
-// a queue (load balance), read the row pointers of the whole group at once
-// and issue the row's u load before its gathers.
+// A split row: out = u + alpha * (sum of its partial slots a..b-1), summed
+// by one warp in slot order (lane groups take alternate slots and are
+// added in group order), so the result does not depend on scheduling.
+template <int BP>
+__device__ __forceinline__ void hop_fixup_row(int64_t j, int64_t a, int64_t b,
+                                              const float4 *__restrict__ part4,
+                                              const float4 *__restrict__ u4,
+                                              float4 *__restrict__ out4, float alpha) {
+    using S = HopShape<BP>;
+    constexpr int P = 8 / S::V > 0 ? 8 / S::V : 1;   // slots in flight per lane group
+    const int lane = threadIdx.x & 31;
+    const int g = lane / S::LW, sub = lane % S::LW;
+    float4 acc[S::V];
+#pragma unroll
+    for (int v = 0; v < S::V; ++v) acc[v] = make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int64_t t = a; t < b; t += P * S::G) {
+        float4 x[P][S::V];
+#pragma unroll
+        for (int q = 0; q < P; ++q) {
+            const int64_t sl = t + q * S::G + g;
+#pragma unroll
+            for (int v = 0; v < S::V; ++v)
+                x[q][v] = sl < b ? ld_stream(part4 + sl * S::F + sub + 32 * v)
+                                 : make_float4(0.f, 0.f, 0.f, 0.f);
+        }
+#pragma unroll
+        for (int q = 0; q < P; ++q)
+#pragma unroll
+            for (int v = 0; v < S::V; ++v) {
+                acc[v].x += x[q][v].x; acc[v].y += x[q][v].y;
+                acc[v].z += x[q][v].z; acc[v].w += x[q][v].w;
+            }
+    }
+    if (S::G > 1) {
+#pragma unroll
+        for (int o = S::LW; o < 32; o <<= 1)
+#pragma unroll
+            for (int v = 0; v < S::V; ++v) {
+                acc[v].x += __shfl_xor_sync(0xffffffffu, acc[v].x, o);
+                acc[v].y += __shfl_xor_sync(0xffffffffu, acc[v].y, o);
+                acc[v].z += __shfl_xor_sync(0xffffffffu, acc[v].z, o);
+                acc[v].w += __shfl_xor_sync(0xffffffffu, acc[v].w, o);
+            }
+    }
+    if (lane < S::LW) {
+#pragma unroll
+        for (int v = 0; v < S::V; ++v) {
+            float4 o = ld_stream(u4 + j * S::F + sub + 32 * v);
+            o.x = fmaf(alpha, acc[v].x, o.x);
+            o.y = fmaf(alpha, acc[v].y, o.y);
+            o.z = fmaf(alpha, acc[v].z, o.z);
+            o.w = fmaf(alpha, acc[v].w, o.w);
+            st_stream(out4 + j * S::F + sub + 32 * v, o);
+        }
+    }
+}
+
+// One queue: first the split rows (their segment partials are complete,
+// the segment kernel ran before), heaviest first, one warp each; then the
+// rows kept whole, ROWS_PER_GRAB consecutive rows per claim (load
+// balance), with the group's row pointers read at once and each row's u
+// load issued before its gathers.
 template <int BP>
 __global__ __launch_bounds__(256, 3) void k_hop_rows(const int64_t *__restrict__ in_ptr,
                                                   const int32_t *__restrict__ in_src,
@@ -633,17 +712,28 @@ __global__ __launch_bounds__(256, 3) void k_hop_rows(const int64_t *__restrict__
                                                   const float4 *__restrict__ u4,
                                                   const float4 *__restrict__ in4,
                                                   float4 *__restrict__ out4, float alpha,
-                                                  int64_t split_t, int *__restrict__ queue) {
+                                                  int64_t split_t, int64_t n_split,
+                                                  const int32_t *__restrict__ split_order,
+                                                  const int32_t *__restrict__ split_row,
+                                                  const int64_t *__restrict__ split_slot0,
+                                                  const float4 *__restrict__ part4,
+                                                  int *__restrict__ queue) {
     using S = HopShape<BP>;
     const int lane = threadIdx.x & 31;
     const int sub = lane % S::LW;
     const int64_t groups = (n + ROWS_PER_GRAB - 1) / ROWS_PER_GRAB;
     while (true) {
-        int64_t g = 0;
-        if (lane == 0) g = atomicAdd(queue, 1);
-        g = __shfl_sync(0xffffffffu, g, 0);
-        if (g >= groups) break;
-        const int64_t j0 = g * ROWS_PER_GRAB;
+        int64_t it = 0;
+        if (lane == 0) it = atomicAdd(queue, 1);
+        it = __shfl_sync(0xffffffffu, it, 0);
+        if (it >= n_split + groups) break;
+        if (it < n_split) {
+            const int32_t r = split_order[it];
+            hop_fixup_row<BP>(split_row[r], split_slot0[r], split_slot0[r + 1], part4, u4, out4,
+                              alpha);
+            continue;
+        }
+        const int64_t j0 = (it - n_split) * ROWS_PER_GRAB;
         const int nr = (int)(n - j0 < ROWS_PER_GRAB ? n - j0 : ROWS_PER_GRAB);
         int64_t p = 0;
         if (lane <= nr) p = in_ptr[j0 + lane];
@@ -703,82 +793,6 @@ __global__ __launch_bounds__(256, 3) void k_hop_segs(const int64_t *__restrict__
     }
 }
 
-// Split rows: out = u + alpha * (sum of the row's segment partials).  One
-// CTA per row: warp w sums a fixed contiguous slice of the row's slots, the
-// eight slice sums are then added in warp order, so the result does not
-// depend on scheduling.  Lanes keep several partial loads in flight.
-template <int BP>
-__global__ __launch_bounds__(256) void k_hop_fixup(const int32_t *__restrict__ split_row,
-                                                   const int64_t *__restrict__ split_slot0,
-                                                   int64_t n_split,
-                                                   const float4 *__restrict__ part4,
-                                                   const float4 *__restrict__ u4,
-                                                   float4 *__restrict__ out4, float alpha) {
-    constexpr int F = BP / 4;
-    constexpr int PER_LANE = (F + 31) / 32;
-    constexpr int P = 4;
-    __shared__ float4 wsum[8][F];
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    for (int64_t r = blockIdx.x; r < n_split; r += gridDim.x) {
-        const int64_t j = split_row[r];
-        const int64_t a = split_slot0[r], b = split_slot0[r + 1];
-        const int64_t per = (b - a + 7) / 8;
-        const int64_t s0 = a + warp * per;
-        const int64_t s1 = s0 + per < b ? s0 + per : b;
-        float4 acc[PER_LANE];
-#pragma unroll
-        for (int t = 0; t < PER_LANE; ++t) acc[t] = make_float4(0.f, 0.f, 0.f, 0.f);
-        int64_t s = s0;
-        for (; s + P <= s1; s += P) {
-            float4 x[P][PER_LANE];
-#pragma unroll
-            for (int q = 0; q < P; ++q)
-#pragma unroll
-                for (int t = 0; t < PER_LANE; ++t) {
-                    const int f = lane + 32 * t;
-                    x[q][t] = f < F ? ld_stream(part4 + (s + q) * F + f) : make_float4(0.f, 0.f, 0.f, 0.f);
-                }
-#pragma unroll
-            for (int q = 0; q < P; ++q)
-#pragma unroll
-                for (int t = 0; t < PER_LANE; ++t) {
-                    acc[t].x += x[q][t].x; acc[t].y += x[q][t].y;
-                    acc[t].z += x[q][t].z; acc[t].w += x[q][t].w;
-                }
-        }
-        for (; s < s1; ++s)
-#pragma unroll
-            for (int t = 0; t < PER_LANE; ++t) {
-                const int f = lane + 32 * t;
-                if (f < F) {
-                    const float4 x = ld_stream(part4 + s * F + f);
-                    acc[t].x += x.x; acc[t].y += x.y; acc[t].z += x.z; acc[t].w += x.w;
-                }
-            }
-#pragma unroll
-        for (int t = 0; t < PER_LANE; ++t) {
-            const int f = lane + 32 * t;
-            if (f < F) wsum[warp][f] = acc[t];
-        }
-        __syncthreads();
-        for (int f = threadIdx.x; f < F; f += blockDim.x) {
-            float4 tot = wsum[0][f];
-#pragma unroll
-            for (int w = 1; w < 8; ++w) {
-                tot.x += wsum[w][f].x; tot.y += wsum[w][f].y;
-                tot.z += wsum[w][f].z; tot.w += wsum[w][f].w;
-            }
-            float4 o = ld_stream(u4 + j * F + f);
-            o.x = fmaf(alpha, tot.x, o.x);
-            o.y = fmaf(alpha, tot.y, o.y);
-            o.z = fmaf(alpha, tot.z, o.z);
-            o.w = fmaf(alpha, tot.w, o.w);
-            st_stream(out4 + j * F + f, o);
-        }
-        __syncthreads();
-    }
-}
-
 template <int BP>
 static cudaError_t hop_bp(const HopPlan &p, const float *u, const float *in, float *out,
                           float alpha, float *partial, int *counters, cudaStream_t st,
@@ -796,18 +810,14 @@ static cudaError_t hop_bp(const HopPlan &p, const float *u, const float *in, flo
         if (e != cudaSuccess) return e;
         if (launches) *launches += 1;
     }
-    const int64_t want = ceil_div<int64_t>(ceil_div<int64_t>(p.n, ROWS_PER_GRAB), 8);
+    const int64_t items = ceil_div<int64_t>(p.n, ROWS_PER_GRAB) + p.n_split_rows;
+    const int64_t want = ceil_div<int64_t>(items, 8);
     const int grid = (int)(want < (int64_t)sms * 3 ? (want < 1 ? 1 : want) : (int64_t)sms * 3);
     k_hop_rows<BP><<<grid, 256, 0, st>>>(p.in_ptr, p.in_src, p.in_w, p.n, (const float4 *)u,
                                          (const float4 *)in, (float4 *)out, alpha,
-                                         p.split.split_t, counters);
-    e = cudaGetLastError();
-    if (launches) *launches += 1;
-    if (e != cudaSuccess || p.n_split_rows == 0) return e;
-    const int g3 = (int)(p.n_split_rows < (int64_t)sms * 16 ? p.n_split_rows : (int64_t)sms * 16);
-    k_hop_fixup<BP><<<g3, 256, 0, st>>>(p.split_row, p.split_slot0, p.n_split_rows,
-                                        (const float4 *)partial, (const float4 *)u, (float4 *)out,
-                                        alpha);
+                                         p.split.split_t, p.n_split_rows, p.split_order,
+                                         p.split_row, p.split_slot0, (const float4 *)partial,
+                                         counters);
     if (launches) *launches += 1;
     return cudaGetLastError();
 }
