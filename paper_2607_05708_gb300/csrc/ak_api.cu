@@ -119,6 +119,7 @@ struct akashic_mem {
     // in-edge transpose + split plan for the propagation hop
     DevBuf in_ptr, in_src, in_w;
     SplitParams split;
+    bool fuse_filter = true;     // top-k filter in the last hop's epilogue
     int64_t n_split = 0, n_segs = 0;
     DevBuf split_row, split_slot0, seg_e0, seg_e1, seg_slot, split_order;
     std::mutex mu;
@@ -349,6 +350,7 @@ akashic_status_t akashic_mem_create(const akashic_mem_config_t *cfg, akashic_mem
     // beyond fp32 summation order)
     if (const char *v = getenv("AKASHIC_SPLIT_T")) m->split.split_t = atoll(v) > 0 ? atoll(v) : m->split.split_t;
     if (const char *v = getenv("AKASHIC_SEG_LEN")) m->split.seg_len = atoll(v) > 0 ? atoll(v) : m->split.seg_len;
+    if (const char *v = getenv("AKASHIC_FUSE_FILTER")) m->fuse_filter = atoi(v) != 0;
     if (const char *v = getenv("AKASHIC_WIN_ROWS")) m->split.win_rows = atoll(v) > 0 ? atoll(v) : m->split.win_rows;
     akashic_status_t s;
     if ((s = m->emb.ensure((size_t)m->cap * m->dim * 2)) != AKASHIC_OK ||
@@ -625,7 +627,6 @@ akashic_status_t akashic_mem_retrieve(akashic_mem_t *m, const uint16_t *q, int32
         }
         const float *fin = sc->u.as<float>();
         if (eff_hops >= 1) {
-            PhaseScope ph(m, AKASHIC_PHASE_PROPAGATE, st);
             HopPlan hp;
             hp.split = m->split;
             hp.in_ptr = m->in_ptr.as<int64_t>();
@@ -641,23 +642,45 @@ akashic_status_t akashic_mem_retrieve(akashic_mem_t *m, const uint16_t *q, int32
             hp.seg_slot = m->seg_slot.as<int32_t>();
             hp.split_order = m->split_order.as<int32_t>();
             float *bufs[2] = {sc->sa.as<float>(), sc->sb.as<float>()};
+            unsigned long long *ws = sc->cand.as<unsigned long long>();
             for (int h = 0; h < eff_hops; ++h) {
                 float *out = bufs[h & 1];
+                const bool last = m->fuse_filter && h == eff_hops - 1;
+                if (last) {
+                    // Top-k filter fused into the last hop.  With w >= 0 and
+                    // alpha >= 0 every hop only adds to a score, and in fp32
+                    // too (same summation order, monotone rounding), so the
+                    // k-th largest key of s^(H-1) over the row sample is a
+                    // safe bound for s^(H).
+                    PhaseScope ps(m, AKASHIC_PHASE_SELECT, st);
+                    CUDA_TRY(launch_sample_bound(sp, fin, b, m->ext_of.as<int32_t>(), ws, st,
+                                                 &ps.launches));
+                }
+                const HopFilter flt{m->ext_of.as<int32_t>(), ws + sp.off_bound,
+                                    (unsigned int *)(ws + sp.off_cnt), ws + sp.off_buf, sp.cap};
+                PhaseScope ph(m, AKASHIC_PHASE_PROPAGATE, st);
                 CUDA_TRY(launch_hop(hp, sc->u.as<float>(), fin, out, bp, alpha,
-                                    sc->partial.as<float>(), sc->counters.as<int>(), st,
-                                    &ph.launches));
+                                    sc->partial.as<float>(), sc->counters.as<int>(),
+                                    last ? &flt : nullptr, st, &ph.launches));
                 fin = out;
             }
         }
         {
             PhaseScope ph(m, AKASHIC_PHASE_SELECT, st);
-            CUDA_TRY(launch_select(sp, fin, b, sc->cand.as<unsigned long long>(),
-                                   sc->zpart.as<float>(), zrows, m->ext_of.as<int32_t>(),
-                                   m->row_of.as<int32_t>(), m->page_of.as<int32_t>(),
-                                   ids + (int64_t)off * k, scores + (int64_t)off * k,
-                                   page_ids ? page_ids + (int64_t)off * k : nullptr,
-                                   n_pages ? n_pages + off : nullptr, m->status.as<int>(), st,
-                                   &ph.launches));
+            int32_t *pids = page_ids ? page_ids + (int64_t)off * k : nullptr;
+            int32_t *npg = n_pages ? n_pages + off : nullptr;
+            if (eff_hops >= 1 && m->fuse_filter)
+                CUDA_TRY(launch_topk_merge(sp, fin, b, sc->cand.as<unsigned long long>(),
+                                           sc->zpart.as<float>(), zrows, m->ext_of.as<int32_t>(),
+                                           m->row_of.as<int32_t>(), m->page_of.as<int32_t>(),
+                                           ids + (int64_t)off * k, scores + (int64_t)off * k,
+                                           pids, npg, m->status.as<int>(), st, &ph.launches));
+            else
+                CUDA_TRY(launch_select(sp, fin, b, sc->cand.as<unsigned long long>(),
+                                       sc->zpart.as<float>(), zrows, m->ext_of.as<int32_t>(),
+                                       m->row_of.as<int32_t>(), m->page_of.as<int32_t>(),
+                                       ids + (int64_t)off * k, scores + (int64_t)off * k, pids,
+                                       npg, m->status.as<int>(), st, &ph.launches));
         }
     }
     return AKASHIC_OK;

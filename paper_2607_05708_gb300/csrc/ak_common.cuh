@@ -172,10 +172,21 @@ struct HopPlan {
     const int32_t *seg_slot;    // [n_segs] partial slot (segments of a row are contiguous)
     const int32_t *split_order; // [n_split_rows] split rows by slot count, largest first
 };
+// Top-k filter fused into a hop's output: every written value whose key
+// (score bits, ~chunk ID) is >= bound[column] is appended to that column's
+// buffer, as the selection's filter pass would (see ak_select.cu).
+struct HopFilter {
+    const int32_t *ext_of;            // row -> chunk ID
+    const unsigned long long *bound;  // [bp]
+    unsigned int *cnt;                // [bp]
+    unsigned long long *buf;          // [bp][cap]
+    int64_t cap;
+};
 // `counters` = 2 device ints, zeroed by the launcher (work queues).
+// `flt` may be NULL (no filter).
 cudaError_t launch_hop(const HopPlan &p, const float *u, const float *in, float *out, int bp,
-                       float alpha, float *partial, int *counters, cudaStream_t st,
-                       int *launches);
+                       float alpha, float *partial, int *counters, const HopFilter *flt,
+                       cudaStream_t st, int *launches);
 
 // ------------------------------------------------------------------ selection
 // Top-k of every column of a slab (a3): bound from a row sample, filter
@@ -211,6 +222,19 @@ cudaError_t launch_select_signed(const SelectPlan &sp, const float *s, int b,
                                  cudaStream_t st, int *launches);
 // Bound pass alone over signed values: bound[c] for the b real columns
 // (the k-th largest sampled key; padding columns get an all-ones bound).
+// Bound only, unsigned keys (retrieval): ws + sp.off_bound gets the bound,
+// the column counts are cleared.  For a filter fused into the last hop.
+cudaError_t launch_sample_bound(const SelectPlan &sp, const float *s, int b,
+                                const int32_t *ext_of, unsigned long long *ws, cudaStream_t st,
+                                int *launches);
+// Merge only: the k winners per column from the buffers filled by a filter
+// pass (falls back to the column of `s` where a buffer overflowed).
+cudaError_t launch_topk_merge(const SelectPlan &sp, const float *s, int b,
+                              const unsigned long long *ws, const float *zpart, int64_t n_ztiles,
+                              const int32_t *ext_of, const int32_t *row_of,
+                              const int32_t *page_row, int64_t *ids, float *scores,
+                              int32_t *page_ids, int32_t *n_pages, int *status, cudaStream_t st,
+                              int *launches);
 cudaError_t launch_sample_bound_signed(const SelectPlan &sp, const float *s, int b,
                                        const int32_t *ext_of, int64_t id_limit,
                                        unsigned long long *ws, unsigned long long *bound,

@@ -646,15 +646,59 @@ __device__ __forceinline__ void hop_accumulate(const int32_t *__restrict__ in_sr
 // A split row: out = u + alpha * (sum of its partial slots a..b-1), summed
 // by one warp in slot order (lane groups take alternate slots and are
 // added in group order), so the result does not depend on scheduling.
+// Filter epilogue: lane `sub` holds columns (sub + 32 v) * 4 + 0..3 of row j.
+// thr[BP] holds the column bounds and thr_hi[BP/4] their upper words (the
+// score bits), four columns per uint4 so that a lane's test is one
+// conflict-free shared load and four 32-bit compares; only a value whose
+// bits reach the bound's (rare: ~ a few k per column) takes the 64-bit
+// compare and the append.
 template <int BP>
+__device__ __noinline__ void hop_filter_row(const HopFilter &f, const unsigned long long *thr,
+                                           const uint4 *thr_hi, int sub, uint32_t id,
+                                           const float4 (&o)[HopShape<BP>::V]) {
+#pragma unroll
+    for (int v = 0; v < HopShape<BP>::V; ++v) {
+        const uint4 h = thr_hi[sub + 32 * v];
+        const uint32_t x[4] = {__float_as_uint(o[v].x), __float_as_uint(o[v].y),
+                               __float_as_uint(o[v].z), __float_as_uint(o[v].w)};
+        const uint32_t hh[4] = {h.x, h.y, h.z, h.w};
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            if (x[e] >= hh[e]) {
+                const int c = (sub + 32 * v) * 4 + e;
+                const unsigned long long key =
+                    ((unsigned long long)x[e] << 32) | (unsigned long long)(~id);
+                if (key >= thr[c]) {
+                    const unsigned int p = atomicAdd(&f.cnt[c], 1u);
+                    if ((int64_t)p < f.cap) f.buf[(int64_t)c * f.cap + p] = key;
+                }
+            }
+        }
+    }
+}
+
+// Kept out of line: any inlined test here slowed the whole row loop of the
+// hop by ~5% (measured), while a call per row costs ~2%.
+template <int BP, bool FILTER>
+__device__ __forceinline__ void hop_emit(const HopFilter &f, const unsigned long long *thr,
+                                         const uint4 *thr_hi, int sub, uint32_t id,
+                                         const float4 (&o)[HopShape<BP>::V]) {
+    if constexpr (FILTER) hop_filter_row<BP>(f, thr, thr_hi, sub, id, o);
+}
+
+template <int BP, bool FILTER>
 __device__ __forceinline__ void hop_fixup_row(int64_t j, int64_t a, int64_t b,
                                               const float4 *__restrict__ part4,
                                               const float4 *__restrict__ u4,
-                                              float4 *__restrict__ out4, float alpha) {
+                                              float4 *__restrict__ out4, float alpha,
+                                              const HopFilter &f,
+                                              const unsigned long long *thr,
+                                              const uint4 *thr_hi) {
     using S = HopShape<BP>;
     constexpr int P = 8 / S::V > 0 ? 8 / S::V : 1;   // slots in flight per lane group
     const int lane = threadIdx.x & 31;
     const int g = lane / S::LW, sub = lane % S::LW;
+    const uint32_t id = FILTER ? (uint32_t)f.ext_of[j] : 0u;
     float4 acc[S::V];
 #pragma unroll
     for (int v = 0; v < S::V; ++v) acc[v] = make_float4(0.f, 0.f, 0.f, 0.f);
@@ -688,15 +732,17 @@ __device__ __forceinline__ void hop_fixup_row(int64_t j, int64_t a, int64_t b,
             }
     }
     if (lane < S::LW) {
+        float4 o[S::V];
 #pragma unroll
         for (int v = 0; v < S::V; ++v) {
-            float4 o = ld_stream(u4 + j * S::F + sub + 32 * v);
-            o.x = fmaf(alpha, acc[v].x, o.x);
-            o.y = fmaf(alpha, acc[v].y, o.y);
-            o.z = fmaf(alpha, acc[v].z, o.z);
-            o.w = fmaf(alpha, acc[v].w, o.w);
-            st_stream(out4 + j * S::F + sub + 32 * v, o);
+            o[v] = ld_stream(u4 + j * S::F + sub + 32 * v);
+            o[v].x = fmaf(alpha, acc[v].x, o[v].x);
+            o[v].y = fmaf(alpha, acc[v].y, o[v].y);
+            o[v].z = fmaf(alpha, acc[v].z, o[v].z);
+            o[v].w = fmaf(alpha, acc[v].w, o[v].w);
+            st_stream(out4 + j * S::F + sub + 32 * v, o[v]);
         }
+        hop_emit<BP, FILTER>(f, thr, thr_hi, sub, id, o);
     }
 }
 
@@ -705,7 +751,7 @@ __device__ __forceinline__ void hop_fixup_row(int64_t j, int64_t a, int64_t b,
 // rows kept whole, ROWS_PER_GRAB consecutive rows per claim (load
 // balance), with the group's row pointers read at once and each row's u
 // load issued before its gathers.
-template <int BP>
+template <int BP, bool FILTER>
 __global__ __launch_bounds__(256, 3) void k_hop_rows(const int64_t *__restrict__ in_ptr,
                                                   const int32_t *__restrict__ in_src,
                                                   const float *__restrict__ in_w, int64_t n,
@@ -717,11 +763,21 @@ __global__ __launch_bounds__(256, 3) void k_hop_rows(const int64_t *__restrict__
                                                   const int32_t *__restrict__ split_row,
                                                   const int64_t *__restrict__ split_slot0,
                                                   const float4 *__restrict__ part4,
-                                                  int *__restrict__ queue) {
+                                                  HopFilter f, int *__restrict__ queue) {
     using S = HopShape<BP>;
     const int lane = threadIdx.x & 31;
     const int sub = lane % S::LW;
     const int64_t groups = (n + ROWS_PER_GRAB - 1) / ROWS_PER_GRAB;
+    __shared__ unsigned long long thr[FILTER ? BP : 1];
+    __shared__ uint4 thr_hi[FILTER ? BP / 4 : 1];
+    if constexpr (FILTER) {
+        for (int c = threadIdx.x; c < BP; c += blockDim.x) {
+            const unsigned long long t = f.bound[c];
+            thr[c] = t;
+            reinterpret_cast<uint32_t *>(thr_hi)[c] = (uint32_t)(t >> 32);
+        }
+        __syncthreads();
+    }
     while (true) {
         int64_t it = 0;
         if (lane == 0) it = atomicAdd(queue, 1);
@@ -729,18 +785,21 @@ __global__ __launch_bounds__(256, 3) void k_hop_rows(const int64_t *__restrict__
         if (it >= n_split + groups) break;
         if (it < n_split) {
             const int32_t r = split_order[it];
-            hop_fixup_row<BP>(split_row[r], split_slot0[r], split_slot0[r + 1], part4, u4, out4,
-                              alpha);
+            hop_fixup_row<BP, FILTER>(split_row[r], split_slot0[r], split_slot0[r + 1], part4,
+                                      u4, out4, alpha, f, thr, thr_hi);
             continue;
         }
         const int64_t j0 = (it - n_split) * ROWS_PER_GRAB;
         const int nr = (int)(n - j0 < ROWS_PER_GRAB ? n - j0 : ROWS_PER_GRAB);
         int64_t p = 0;
         if (lane <= nr) p = in_ptr[j0 + lane];
+        int32_t ids = 0;
+        if (FILTER && lane < nr) ids = f.ext_of[j0 + lane];
 #pragma unroll 1
         for (int r = 0; r < nr; ++r) {
             const int64_t e0 = __shfl_sync(0xffffffffu, p, r);
             const int64_t e1 = __shfl_sync(0xffffffffu, p, r + 1);
+            const uint32_t id = FILTER ? (uint32_t)__shfl_sync(0xffffffffu, ids, r) : 0u;
             if (e1 - e0 > split_t) continue;
             const int64_t j = j0 + r;
             float4 b[S::V];
@@ -759,6 +818,7 @@ __global__ __launch_bounds__(256, 3) void k_hop_rows(const int64_t *__restrict__
                     b[v].w = fmaf(alpha, acc[v].w, b[v].w);
                     st_stream(out4 + j * S::F + sub + 32 * v, b[v]);
                 }
+                hop_emit<BP, FILTER>(f, thr, thr_hi, sub, id, b);
             }
         }
     }
@@ -795,8 +855,8 @@ __global__ __launch_bounds__(256, 3) void k_hop_segs(const int64_t *__restrict__
 
 template <int BP>
 static cudaError_t hop_bp(const HopPlan &p, const float *u, const float *in, float *out,
-                          float alpha, float *partial, int *counters, cudaStream_t st,
-                          int *launches) {
+                          float alpha, float *partial, int *counters, const HopFilter *flt,
+                          cudaStream_t st, int *launches) {
     const int sms = device_sm_count();
     cudaError_t e = cudaMemsetAsync(counters, 0, 2 * sizeof(int), st);
     if (e != cudaSuccess) return e;
@@ -813,23 +873,33 @@ static cudaError_t hop_bp(const HopPlan &p, const float *u, const float *in, flo
     const int64_t items = ceil_div<int64_t>(p.n, ROWS_PER_GRAB) + p.n_split_rows;
     const int64_t want = ceil_div<int64_t>(items, 8);
     const int grid = (int)(want < (int64_t)sms * 3 ? (want < 1 ? 1 : want) : (int64_t)sms * 3);
-    k_hop_rows<BP><<<grid, 256, 0, st>>>(p.in_ptr, p.in_src, p.in_w, p.n, (const float4 *)u,
-                                         (const float4 *)in, (float4 *)out, alpha,
-                                         p.split.split_t, p.n_split_rows, p.split_order,
-                                         p.split_row, p.split_slot0, (const float4 *)partial,
-                                         counters);
+    const HopFilter f = flt ? *flt : HopFilter{nullptr, nullptr, nullptr, nullptr, 0};
+    if (flt)
+        k_hop_rows<BP, true><<<grid, 256, 0, st>>>(p.in_ptr, p.in_src, p.in_w, p.n,
+                                                   (const float4 *)u, (const float4 *)in,
+                                                   (float4 *)out, alpha, p.split.split_t,
+                                                   p.n_split_rows, p.split_order, p.split_row,
+                                                   p.split_slot0, (const float4 *)partial, f,
+                                                   counters);
+    else
+        k_hop_rows<BP, false><<<grid, 256, 0, st>>>(p.in_ptr, p.in_src, p.in_w, p.n,
+                                                    (const float4 *)u, (const float4 *)in,
+                                                    (float4 *)out, alpha, p.split.split_t,
+                                                    p.n_split_rows, p.split_order, p.split_row,
+                                                    p.split_slot0, (const float4 *)partial, f,
+                                                    counters);
     if (launches) *launches += 1;
     return cudaGetLastError();
 }
 
 cudaError_t launch_hop(const HopPlan &p, const float *u, const float *in, float *out, int bp,
-                       float alpha, float *partial, int *counters, cudaStream_t st,
-                       int *launches) {
+                       float alpha, float *partial, int *counters, const HopFilter *flt,
+                       cudaStream_t st, int *launches) {
     switch (bp) {
-    case 32: return hop_bp<32>(p, u, in, out, alpha, partial, counters, st, launches);
-    case 64: return hop_bp<64>(p, u, in, out, alpha, partial, counters, st, launches);
-    case 128: return hop_bp<128>(p, u, in, out, alpha, partial, counters, st, launches);
-    case 256: return hop_bp<256>(p, u, in, out, alpha, partial, counters, st, launches);
+    case 32: return hop_bp<32>(p, u, in, out, alpha, partial, counters, flt, st, launches);
+    case 64: return hop_bp<64>(p, u, in, out, alpha, partial, counters, flt, st, launches);
+    case 128: return hop_bp<128>(p, u, in, out, alpha, partial, counters, flt, st, launches);
+    case 256: return hop_bp<256>(p, u, in, out, alpha, partial, counters, flt, st, launches);
     default: return cudaErrorInvalidValue;
     }
 }

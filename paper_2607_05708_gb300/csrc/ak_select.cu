@@ -465,23 +465,24 @@ static cudaError_t bound_and_filter(const SelectPlan &sp, const float *s, int b,
     return cudaGetLastError();
 }
 
-cudaError_t launch_sample_bound_signed(const SelectPlan &sp, const float *s, int b,
-                                       const int32_t *ext_of, int64_t id_limit,
-                                       unsigned long long *ws, unsigned long long *bound,
-                                       cudaStream_t st, int *launches) {
-    static bool attr[64] = {false};
+template <bool SIGNED>
+static cudaError_t sample_bound(const SelectPlan &sp, const float *s, int b,
+                                const int32_t *ext_of, int64_t id_limit,
+                                unsigned long long *ws, unsigned long long *bound,
+                                cudaStream_t st, int *launches) {
+    static bool attr[2][64] = {{false}};
     int dev = 0;
     cudaGetDevice(&dev);
-    if (dev >= 0 && dev < 64 && !attr[dev]) {
-        cudaError_t e = cudaFuncSetAttribute(k_sample_heaps<true>,
+    if (dev >= 0 && dev < 64 && !attr[SIGNED][dev]) {
+        cudaError_t e = cudaFuncSetAttribute(k_sample_heaps<SIGNED>,
                                              cudaFuncAttributeMaxDynamicSharedMemorySize,
                                              64 * SEL_THREADS * (int)sizeof(unsigned long long));
         if (e != cudaSuccess) return e;
-        attr[dev] = true;
+        attr[SIGNED][dev] = true;
     }
     const size_t smem = (size_t)sp.k * SEL_THREADS * sizeof(unsigned long long);
     const int64_t rows_per_cta = ceil_div<int64_t>(sp.n_sample, sp.grid);
-    k_sample_heaps<true><<<sp.grid, SEL_THREADS, smem, st>>>(
+    k_sample_heaps<SIGNED><<<sp.grid, SEL_THREADS, smem, st>>>(
         s, sp.n_sample, sp.stride, sp.bp, sp.lanes, sp.k, rows_per_cta, ext_of, id_limit, ws);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
@@ -491,6 +492,20 @@ cudaError_t launch_sample_bound_signed(const SelectPlan &sp, const float *s, int
     return cudaGetLastError();
 }
 
+cudaError_t launch_sample_bound_signed(const SelectPlan &sp, const float *s, int b,
+                                       const int32_t *ext_of, int64_t id_limit,
+                                       unsigned long long *ws, unsigned long long *bound,
+                                       cudaStream_t st, int *launches) {
+    return sample_bound<true>(sp, s, b, ext_of, id_limit, ws, bound, st, launches);
+}
+
+cudaError_t launch_sample_bound(const SelectPlan &sp, const float *s, int b,
+                                const int32_t *ext_of, unsigned long long *ws, cudaStream_t st,
+                                int *launches) {
+    return sample_bound<false>(sp, s, b, ext_of, (int64_t)1 << 40, ws, ws + sp.off_bound, st,
+                               launches);
+}
+
 cudaError_t launch_select(const SelectPlan &sp, const float *s, int b, unsigned long long *ws,
                           const float *zpart, int64_t n_ztiles, const int32_t *ext_of,
                           const int32_t *row_of, const int32_t *page_row, int64_t *ids,
@@ -498,6 +513,16 @@ cudaError_t launch_select(const SelectPlan &sp, const float *s, int b, unsigned 
                           cudaStream_t st, int *launches) {
     cudaError_t e = bound_and_filter<false>(sp, s, b, ext_of, (int64_t)1 << 40, ws, st, launches);
     if (e != cudaSuccess) return e;
+    return launch_topk_merge(sp, s, b, ws, zpart, n_ztiles, ext_of, row_of, page_row, ids, scores,
+                             page_ids, n_pages, status, st, launches);
+}
+
+cudaError_t launch_topk_merge(const SelectPlan &sp, const float *s, int b,
+                              const unsigned long long *ws, const float *zpart, int64_t n_ztiles,
+                              const int32_t *ext_of, const int32_t *row_of,
+                              const int32_t *page_row, int64_t *ids, float *scores,
+                              int32_t *page_ids, int32_t *n_pages, int *status, cudaStream_t st,
+                              int *launches) {
     k_topk_merge<<<b, SEL_THREADS, 0, st>>>(s, sp.n, sp.bp, sp.k, ext_of,
                                             (const unsigned int *)(ws + sp.off_cnt),
                                             ws + sp.off_buf, sp.cap, zpart, n_ztiles, row_of,

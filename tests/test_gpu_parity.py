@@ -70,6 +70,30 @@ def test_ragged_shapes(B, k, hops, alpha):
     assert_retrieval_parity(wl, "clustered", got, ref)
 
 
+def test_fused_filter_overflow_falls_back():
+    """Every row with out-edges to its 8 successors (uniform weights, no
+    hubs), alpha = 4, two hops, N = 16384: the last hop raises every score
+    about fourfold over the previous level, so all rows clear the bound
+    taken from that level's sample and the 8192-key buffer of every column
+    overflows; the merge then selects from the whole final column.  The
+    premise is checked on the oracle: even the k-th largest one-hop score (a
+    bound at least as high as any sample's) is reached by more than 8192 rows."""
+    import dataclasses
+    base = synth.workload(2, scale=1 / 64)
+    n = base.n
+    col = np.sort((np.arange(n)[:, None] + np.arange(1, 9)[None, :]) % n, axis=1)
+    wl = dataclasses.replace(base, row_ptr=np.arange(0, 8 * n + 1, 8, dtype=np.int64),
+                             col=col.astype(np.int32).ravel(), aff=np.zeros(8 * n, np.float32),
+                             alpha=4.0)
+    q = wl.queries[:8]
+    one = oracle_retrieve(wl, "clustered", queries=q, hops=1)["final"]
+    ref = oracle_retrieve(wl, "clustered", queries=q)
+    kth1 = -np.sort(-one, axis=1)[:, wl.k - 1]
+    assert ((ref["final"] >= kth1[:, None]).sum(axis=1) > 8192).all()
+    _, got = gpu_retrieve(wl, "clustered", queries=q)
+    assert_retrieval_parity(wl, "clustered", got, ref)
+
+
 def test_no_edges_and_single_chunk_pages():
     """A store without relations: propagation adds nothing."""
     wl0 = synth.workload(0)
