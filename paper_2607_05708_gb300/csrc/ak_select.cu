@@ -20,6 +20,7 @@ namespace ak {
 
 constexpr int SEL_THREADS = 256;
 constexpr int SEL_STAGE = 4096;   // keys a merge CTA stages in shared memory
+constexpr int BOUND_STAGE = 12288; // sampled keys a bound CTA stages (96 KiB, dynamic)
 
 // SIGNED=false: non-negative scores (retrieval); SIGNED=true: any finite
 // value (cosines of the relation update).  Either way a larger key is a
@@ -141,31 +142,43 @@ __global__ __launch_bounds__(SEL_THREADS) void k_sample_heaps(
     unsigned long long root = 0ull;
     const int64_t v0 = (int64_t)blockIdx.x * rows_per_cta;
     const int64_t v1 = v0 + rows_per_cta < n_sample ? v0 + rows_per_cta : n_sample;
-    for (int64_t v = v0 + r; v < v1; v += lanes) {
-        const int64_t j = v * stride;
-        const int32_t id = ext_of[j];
-        if ((int64_t)id >= id_limit) continue;
-        const unsigned long long key = sel_key<SIGNED>(s[j * bp + c], (uint32_t)id);
-        if (key <= root) continue;
-        int i = 0;   // replace the minimum, sift down
-        while (true) {
-            const int l = 2 * i + 1, rr = l + 1;
-            if (l >= k) break;
-            int m = l;
-            unsigned long long km = heap[l * SEL_THREADS + tid];
-            if (rr < k) {
-                const unsigned long long kr = heap[rr * SEL_THREADS + tid];
-                if (kr < km) {
-                    m = rr;
-                    km = kr;
-                }
+    constexpr int R = 8;   // sample rows loaded ahead (independent loads in flight)
+    for (int64_t vb = v0 + r; vb < v1; vb += (int64_t)R * lanes) {
+        unsigned long long kq[R];
+#pragma unroll
+        for (int q = 0; q < R; ++q) {
+            const int64_t v = vb + (int64_t)q * lanes;
+            kq[q] = 0ull;
+            if (v < v1) {
+                const int64_t j = v * stride;
+                const int32_t id = ext_of[j];
+                if ((int64_t)id < id_limit) kq[q] = sel_key<SIGNED>(s[j * bp + c], (uint32_t)id);
             }
-            if (km >= key) break;
-            heap[i * SEL_THREADS + tid] = km;
-            i = m;
         }
-        heap[i * SEL_THREADS + tid] = key;
-        root = heap[tid];
+#pragma unroll
+        for (int q = 0; q < R; ++q) {
+            const unsigned long long key = kq[q];
+            if (key <= root) continue;
+            int i = 0;   // replace the minimum, sift down
+            while (true) {
+                const int l = 2 * i + 1, rr = l + 1;
+                if (l >= k) break;
+                int m = l;
+                unsigned long long km = heap[l * SEL_THREADS + tid];
+                if (rr < k) {
+                    const unsigned long long kr = heap[rr * SEL_THREADS + tid];
+                    if (kr < km) {
+                        m = rr;
+                        km = kr;
+                    }
+                }
+                if (km >= key) break;
+                heap[i * SEL_THREADS + tid] = km;
+                i = m;
+            }
+            heap[i * SEL_THREADS + tid] = key;
+            root = heap[tid];
+        }
     }
     const int64_t list = (int64_t)blockIdx.x * lanes + r;
     unsigned long long *dst = lists_g + (list * bp + c) * k;
@@ -189,10 +202,21 @@ __global__ __launch_bounds__(SEL_THREADS) void k_sample_bound(
         }
         return;
     }
-    auto key_at = [&](int64_t i) -> unsigned long long {
-        return lists_g[((i / k) * bp + c) * k + (i % k)];
-    };
-    radix_select(lists * (int64_t)k, k, key_at, win, &win_n, hist, &s_prefix, &s_remaining);
+    const int64_t total = lists * (int64_t)k;
+    if (total <= BOUND_STAGE) {
+        // the column's keys, list by list (each list's k keys are contiguous)
+        extern __shared__ unsigned long long stage_b[];
+        for (int64_t i = threadIdx.x; i < total; i += SEL_THREADS)
+            stage_b[i] = lists_g[((i / k) * bp + c) * k + (i % k)];
+        __syncthreads();
+        auto key_at = [&](int64_t i) -> unsigned long long { return stage_b[i]; };
+        radix_select(total, k, key_at, win, &win_n, hist, &s_prefix, &s_remaining);
+    } else {
+        auto key_at = [&](int64_t i) -> unsigned long long {
+            return lists_g[((i / k) * bp + c) * k + (i % k)];
+        };
+        radix_select(total, k, key_at, win, &win_n, hist, &s_prefix, &s_remaining);
+    }
     if (threadIdx.x == 0) {
         bound[c] = win_n >= k ? s_prefix : 0ull;
         cnt[c] = 0u;
@@ -423,6 +447,24 @@ cudaError_t launch_buf_merge_signed(const unsigned int *cnt, const unsigned long
 }
 
 // ------------------------------------------------------------------ launchers
+static cudaError_t launch_bound(const SelectPlan &sp, int b, const unsigned long long *ws,
+                                unsigned long long *bound, unsigned int *cnt, cudaStream_t st) {
+    static bool attr[64] = {false};
+    int dev = 0;
+    cudaGetDevice(&dev);
+    if (dev >= 0 && dev < 64 && !attr[dev]) {
+        cudaError_t e = cudaFuncSetAttribute(k_sample_bound,
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             BOUND_STAGE * (int)sizeof(unsigned long long));
+        if (e != cudaSuccess) return e;
+        attr[dev] = true;
+    }
+    const int64_t total = sp.lists * (int64_t)sp.k;
+    const size_t smem = total <= BOUND_STAGE ? (size_t)total * sizeof(unsigned long long) : 0;
+    k_sample_bound<<<sp.bp, SEL_THREADS, smem, st>>>(ws, sp.lists, sp.bp, b, sp.k, bound, cnt);
+    return cudaGetLastError();
+}
+
 template <bool SIGNED>
 static cudaError_t bound_and_filter(const SelectPlan &sp, const float *s, int b,
                                     const int32_t *ext_of, int64_t id_limit,
@@ -446,8 +488,7 @@ static cudaError_t bound_and_filter(const SelectPlan &sp, const float *s, int b,
     unsigned long long *bound = ws + sp.off_bound;
     unsigned int *cnt = (unsigned int *)(ws + sp.off_cnt);
     unsigned long long *buf = ws + sp.off_buf;
-    k_sample_bound<<<sp.bp, SEL_THREADS, 0, st>>>(ws, sp.lists, sp.bp, b, sp.k, bound, cnt);
-    e = cudaGetLastError();
+    e = launch_bound(sp, b, ws, bound, cnt, st);
     if (e != cudaSuccess) return e;
     const int64_t warps = ceil_div<int64_t>(sp.n, 4);
     int grid = (int)(ceil_div<int64_t>(warps, 8) < (int64_t)device_sm_count() * 8
@@ -486,10 +527,9 @@ static cudaError_t sample_bound(const SelectPlan &sp, const float *s, int b,
         s, sp.n_sample, sp.stride, sp.bp, sp.lanes, sp.k, rows_per_cta, ext_of, id_limit, ws);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
-    k_sample_bound<<<sp.bp, SEL_THREADS, 0, st>>>(ws, sp.lists, sp.bp, b, sp.k, bound,
-                                                  (unsigned int *)(ws + sp.off_cnt));
+    e = launch_bound(sp, b, ws, bound, (unsigned int *)(ws + sp.off_cnt), st);
     if (launches) *launches += 2;
-    return cudaGetLastError();
+    return e;
 }
 
 cudaError_t launch_sample_bound_signed(const SelectPlan &sp, const float *s, int b,
