@@ -196,11 +196,10 @@ struct SelectPlan {
     int bp, k;
     int64_t stride;     // sample every stride-th row
     int64_t n_sample;
-    int grid;           // CTAs of the sample pass
-    int lanes;          // row lanes per CTA (threads = lanes * bp)
-    int64_t lists;      // grid * lanes heaps per column
     int64_t cap;        // buffer capacity per column
-    int64_t off_bound, off_cnt, off_buf, words;
+    // workspace offsets in 64-bit words: bounds, counts, buffers, the
+    // sample transposed to [bp][n_sample] 32-bit keys
+    int64_t off_bound, off_cnt, off_buf, off_tr, words;
 };
 // force_stride > 0 samples every force_stride-th row instead of the default.
 SelectPlan select_plan(int64_t n, int bp, int k, int sm_count, int64_t force_stride = 0);

@@ -138,30 +138,40 @@ struct GemmEpi {
     int64_t cap;
 };
 
-template <int BP>
+template <int BP, int MODE>
 struct GemmCfg {
     static constexpr int BM = 128, BK = 64;
     static constexpr int A_BYTES = BM * BK * 2;
     static constexpr int B_BYTES = BP * BK * 2;
     static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
     static constexpr int OUT_BYTES = BM * 32 * 4;
+    // the filter epilogue stores nothing: its region only holds the tile's
+    // column bounds, and the freed space goes to pipeline stages
+    static constexpr int OUT_REGION = MODE == GEMM_FILTER ? (BP * 12 < 1024 ? 1024 : BP * 12)
+                                                          : 2 * OUT_BYTES;
     static constexpr int MISC = 4096;   // shift, Z sums, flags, barriers
     static constexpr int BUDGET = 227 * 1024 - 1024;
-    static constexpr int S_FIT = (BUDGET - 2 * OUT_BYTES - MISC) / STAGE_BYTES;
+    static constexpr int S_FIT = (BUDGET - OUT_REGION - MISC) / STAGE_BYTES;
     static constexpr int STAGES = S_FIT > 8 ? 8 : S_FIT;
     static constexpr int TMEM_COLS = 2 * BP < 32 ? 32 : 2 * BP;
-    static constexpr int SMEM = 1024 + STAGES * STAGE_BYTES + 2 * OUT_BYTES + MISC;
+    // epilogue warps: the filter epilogue is issue-bound (one compare per
+    // dot), so it runs two warps per TMEM lane quarter, each on half the
+    // columns; the storing epilogues run one
+    static constexpr int EPI_W = (MODE == GEMM_FILTER && BP >= 64) ? 8 : 4;
+    static constexpr int EPI_T = 32 * EPI_W;
+    static constexpr int THREADS = 64 + EPI_T;
+    static constexpr int SMEM = 1024 + STAGES * STAGE_BYTES + OUT_REGION + MISC;
     static_assert(BP >= 32 && BP <= 256 && (BP & (BP - 1)) == 0, "BP must be 32..256, a power of 2");
     static_assert(STAGES >= 2, "not enough shared memory for two stages");
 };
 
 template <int BP, int MODE>
-__global__ __launch_bounds__(192, 1) void k_gemm_umma(const __grid_constant__ CUtensorMap tmA,
+__global__ __launch_bounds__(GemmCfg<BP, MODE>::THREADS, 1) void k_gemm_umma(const __grid_constant__ CUtensorMap tmA,
                                                       const __grid_constant__ CUtensorMap tmB,
                                                       const __grid_constant__ CUtensorMap tmC,
                                                       int64_t n_rows, int dim, int n_ctiles,
                                                       const GemmEpi ep) {
-    using C = GemmCfg<BP>;
+    using C = GemmCfg<BP, MODE>;
     constexpr bool EXP = MODE == GEMM_EXP;
     constexpr bool FILTER = MODE == GEMM_FILTER;
     extern __shared__ uint8_t smem_raw[];
@@ -169,7 +179,7 @@ __global__ __launch_bounds__(192, 1) void k_gemm_umma(const __grid_constant__ CU
     uint8_t *sA = smem;
     uint8_t *sB = smem + C::STAGES * C::A_BYTES;
     float *sOut = (float *)(smem + C::STAGES * C::STAGE_BYTES);     // 2 x [128][32], swizzled
-    uint8_t *misc = smem + C::STAGES * C::STAGE_BYTES + 2 * C::OUT_BYTES;
+    uint8_t *misc = smem + C::STAGES * C::STAGE_BYTES + C::OUT_REGION;
     float *shift_s = (float *)misc;                  // [BP]
     float *zacc = shift_s + BP;                      // [BP]
     float *zq = zacc + BP;                           // [4][32]  (ends below misc + 2560)
@@ -179,6 +189,7 @@ __global__ __launch_bounds__(192, 1) void k_gemm_umma(const __grid_constant__ CU
     uint64_t *tfull = bars + 2 * C::STAGES, *tempty = tfull + 2;
     uint32_t *tmem_slot = (uint32_t *)(tempty + 2);
     unsigned long long *bnd_s = (unsigned long long *)sOut;   // FILTER: the tile's column bounds
+    float *thr_s = (float *)(bnd_s + BP);   // FILTER: the bounds as float thresholds
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int64_t m_tiles = (n_rows + C::BM - 1) / C::BM;
@@ -277,10 +288,12 @@ __global__ __launch_bounds__(192, 1) void k_gemm_umma(const __grid_constant__ CU
             }
         }
     } else {
-        // ---------------- epilogue (128 threads; warp w reads TMEM lanes 32*(w%4)..)
+        // ---------------- epilogue (EPI_T threads; warp w reads TMEM lanes 32*(w%4)..)
         const int q = warp & 3;
         const int row = q * 32 + lane;                   // row inside the tile
-        const int et = threadIdx.x - 64;                 // 0..127
+        const int et = threadIdx.x - 64;                 // 0..EPI_T-1
+        constexpr int CH_PER = BP / 32 / (C::EPI_W / 4); // 32-column chunks per epilogue warp
+        const int hsel = (warp - 2) / 4;                 // which column share
         int it = 0, cc = 0;
         for (int64_t t = blockIdx.x; t < n_tiles; t += gridDim.x, ++it) {
             const int64_t mt = t / n_ctiles, ct = t % n_ctiles;
@@ -289,12 +302,18 @@ __global__ __launch_bounds__(192, 1) void k_gemm_umma(const __grid_constant__ CU
             // one thread polls, the barrier makes the outcome uniform
             if (et == 0) *go = mbar_wait(&tfull[acc], aph, status) ? 1 : 0;
             if (FILTER) {
-                for (int c = et; c < BP; c += 128) {
+                // threshold T with: v < T => key < bound; v > T => key > bound
+                // (keys order values like floats, -0 below +0); a bound of 0
+                // admits everything (-inf), the padding bound ~0 nothing (NaN)
+                for (int c = et; c < BP; c += C::EPI_T) {
                     const int64_t cg = ct * BP + c;
-                    bnd_s[c] = cg < ep.n_cols ? ep.bound[cg] : ~0ull;
+                    const unsigned long long bk = cg < ep.n_cols ? ep.bound[cg] : ~0ull;
+                    const uint32_t hi = (uint32_t)(bk >> 32);
+                    bnd_s[c] = bk;
+                    thr_s[c] = hi == 0u ? -INFINITY : unordered_bits(hi);
                 }
             }
-            named_bar(1, 128);
+            named_bar(1, C::EPI_T);
             if (!*go) break;
             tc_fence_after();
             const int64_t grow = mt * C::BM + row;
@@ -307,21 +326,33 @@ __global__ __launch_bounds__(192, 1) void k_gemm_umma(const __grid_constant__ CU
                 fid = ~(uint32_t)id;
             }
 #pragma unroll 1
-            for (int ch = 0; ch < BP / 32; ++ch, ++cc) {
+            for (int ch = hsel * CH_PER; ch < (hsel + 1) * CH_PER; ++ch, ++cc) {
                 const int buf = cc & 1;
                 uint32_t r[32];
                 tmem_ld32(tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * BP + ch * 32), r);
                 tmem_ld_wait();
                 if constexpr (FILTER) {
                     if (fok) {
+                        // one float compare per dot; the exact key test only
+                        // for the few at or above the threshold
+                        const float4 *t4 = (const float4 *)(thr_s + ch * 32);
 #pragma unroll
-                        for (int i = 0; i < 32; ++i) {
-                            const unsigned long long key =
-                                ((unsigned long long)ordered_bits(__uint_as_float(r[i])) << 32) | fid;
-                            if (key >= bnd_s[ch * 32 + i]) {
-                                const int64_t cg = ct * BP + ch * 32 + i;
-                                const unsigned int p = atomicAdd(&ep.cnt[cg], 1u);
-                                if ((int64_t)p < ep.cap) ep.buf[cg * ep.cap + p] = key;
+                        for (int i4 = 0; i4 < 8; ++i4) {
+                            const float4 t = t4[i4];
+                            const float tv[4] = {t.x, t.y, t.z, t.w};
+#pragma unroll
+                            for (int e = 0; e < 4; ++e) {
+                                const int i = i4 * 4 + e;
+                                const float v = __uint_as_float(r[i]);
+                                if (v >= tv[e]) {
+                                    const unsigned long long key =
+                                        ((unsigned long long)ordered_bits(v) << 32) | fid;
+                                    if (key >= bnd_s[ch * 32 + i]) {
+                                        const int64_t cg = ct * BP + ch * 32 + i;
+                                        const unsigned int p = atomicAdd(&ep.cnt[cg], 1u);
+                                        if ((int64_t)p < ep.cap) ep.buf[cg * ep.cap + p] = key;
+                                    }
+                                }
                             }
                         }
                     }
@@ -332,13 +363,13 @@ __global__ __launch_bounds__(192, 1) void k_gemm_umma(const __grid_constant__ CU
                     const float x = __uint_as_float(r[i]);
                     v[i] = valid ? (EXP ? expf(ep.tau * x - shift_s[ch * 32 + i]) : x) : 0.f;
                 }
-                named_bar(1, 128);                       // staging[buf] free again
+                named_bar(1, C::EPI_T);                       // staging[buf] free again
                 float4 *dst = (float4 *)(sOut + buf * (C::OUT_BYTES / 4) + row * 32);
 #pragma unroll
                 for (int j = 0; j < 8; ++j)
                     dst[j ^ (row & 7)] = make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
                 fence_async_smem();
-                named_bar(1, 128);                       // staging[buf] complete
+                named_bar(1, C::EPI_T);                       // staging[buf] complete
                 if (EXP) {
                     const int c = et & 31, g = et >> 5;
                     const float *so = sOut + buf * (C::OUT_BYTES / 4);
@@ -354,18 +385,18 @@ __global__ __launch_bounds__(192, 1) void k_gemm_umma(const __grid_constant__ CU
                     bulk_commit();
                 }
                 if (EXP) {
-                    named_bar(1, 128);
+                    named_bar(1, C::EPI_T);
                     if (et < 32) zacc[ch * 32 + et] += (zq[et] + zq[32 + et]) + (zq[64 + et] + zq[96 + et]);
                 }
                 if (et == 0) bulk_wait_read<1>();
                 }
             }
             tc_fence_before();
-            named_bar(1, 128);
+            named_bar(1, C::EPI_T);
             if (et == 0) mbar_arrive(&tempty[acc]);
         }
         if (et == 0) bulk_wait_all();
-        named_bar(1, 128);
+        named_bar(1, C::EPI_T);
         if (EXP && ep.zpart)
             for (int c = et; c < BP; c += 128) ep.zpart[(int64_t)blockIdx.x * BP + c] = zacc[c];
     }
@@ -383,7 +414,7 @@ template <int BP, int MODE>
 static cudaError_t gemm_bp(const uint16_t *emb, int64_t n_rows, int64_t row_stride_rows, int dim,
                            const uint16_t *qp, int n_ctiles, float *out, const GemmEpi &ep,
                            cudaStream_t st, int *zrows) {
-    using C = GemmCfg<BP>;
+    using C = GemmCfg<BP, MODE>;
     static bool attr[64] = {false};
     int dev = 0;
     cudaGetDevice(&dev);
@@ -407,7 +438,7 @@ static cudaError_t gemm_bp(const uint16_t *emb, int64_t n_rows, int64_t row_stri
     if (e != cudaSuccess) return e;
     const int64_t tiles = ceil_div<int64_t>(n_rows, 128) * n_ctiles;
     const int grid = (int)(tiles < device_sm_count() ? tiles : device_sm_count());
-    k_gemm_umma<BP, MODE><<<grid, 192, C::SMEM, st>>>(ta, tb, tc, n_rows, dim, n_ctiles, ep);
+    k_gemm_umma<BP, MODE><<<grid, C::THREADS, C::SMEM, st>>>(ta, tb, tc, n_rows, dim, n_ctiles, ep);
     if (zrows) *zrows = grid;
     return cudaGetLastError();
 }

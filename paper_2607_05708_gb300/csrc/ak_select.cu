@@ -5,10 +5,10 @@
 // the top-M prior chunks of the relation update.
 //
 // Three passes per batch of queries (columns of the score slab):
-//   bound   the k-th largest key of every column over a strided sample of
-//           the rows (per-thread heaps + radix-select merge).  A subset's
-//           k-th largest value never exceeds the whole column's, so it is a
-//           safe filter;
+//   bound   the k-th largest value of every column over a strided sample
+//           of the rows (a radix select per column).  A subset's k-th
+//           largest value never exceeds the whole column's, so it is a safe
+//           filter;
 //   filter  one streaming pass over the slab (warp per row, coalesced
 //           float4 loads) appending every key >= bound to a per-column
 //           buffer;
@@ -20,7 +20,6 @@ namespace ak {
 
 constexpr int SEL_THREADS = 256;
 constexpr int SEL_STAGE = 4096;   // keys a merge CTA stages in shared memory
-constexpr int BOUND_STAGE = 12288; // sampled keys a bound CTA stages (96 KiB, dynamic)
 
 // SIGNED=false: non-negative scores (retrieval); SIGNED=true: any finite
 // value (cosines of the relation update).  Either way a larger key is a
@@ -48,17 +47,14 @@ SelectPlan select_plan(int64_t n, int bp, int k, int sm_count, int64_t force_str
     if (force_stride > 0) stride = force_stride;
     sp.stride = stride;
     sp.n_sample = ceil_div<int64_t>(n, stride);
-    sp.lanes = SEL_THREADS / bp > 0 ? SEL_THREADS / bp : 1;
-    int64_t want = ceil_div<int64_t>(sp.n_sample, (int64_t)sp.lanes * 4 * k);
-    int64_t capg = 4 * (int64_t)sm_count;
-    sp.grid = (int)(want < 1 ? 1 : (want > capg ? capg : want));
-    sp.lists = (int64_t)sp.grid * sp.lanes;
+    (void)sm_count;
     int64_t cap = 4 * (int64_t)k * stride;
     sp.cap = cap < 8192 ? 8192 : cap;
-    sp.off_bound = sp.lists * bp * k;
+    sp.off_bound = 0;
     sp.off_cnt = sp.off_bound + bp;
     sp.off_buf = sp.off_cnt + bp;
-    sp.words = sp.off_buf + (int64_t)bp * sp.cap;
+    sp.off_tr = sp.off_buf + (int64_t)bp * sp.cap;
+    sp.words = sp.off_tr + ceil_div<int64_t>(sp.n_sample * bp, 2);
     return sp;
 }
 
@@ -126,99 +122,111 @@ __device__ void radix_select(int64_t total, int k, KeyAt key_at, unsigned long l
 }
 
 // ------------------------------------------------------------------ bound pass
-// Thread (r, c) of CTA g scans sample rows of its CTA's range for column c
-// and keeps its k best keys in a binary min-heap in shared memory
-// (slot-major, so a warp's accesses are contiguous).
+// bound[c] = the k-th largest sampled value of column c, as a key with the
+// chunk-ID half zero (every key of that value clears it); 0 (admit all) if
+// the sample holds fewer than k real values.  Sample rows are j = v*stride,
+// v < n_sample; rows whose chunk ID is >= id_limit count as value-key 0.
+constexpr int KTH_STAGE = 49152;   // sampled keys staged per CTA (192 KiB)
+
+// keysT[c][v] = key of sample row v in column c: 32 x 32 tiles through
+// shared memory, so both the row reads and the column writes are
+// coalesced.  Threads (tx, ty) = (tid % 32, tid / 32).
 template <bool SIGNED>
-__global__ __launch_bounds__(SEL_THREADS) void k_sample_heaps(
-    const float *__restrict__ s, int64_t n_sample, int64_t stride, int bp, int lanes, int k,
-    int64_t rows_per_cta, const int32_t *__restrict__ ext_of, int64_t id_limit,
-    unsigned long long *__restrict__ lists_g) {
-    extern __shared__ unsigned long long heap[];   // [k][SEL_THREADS]
-    const int tid = threadIdx.x;
-    const int c = tid % bp, r = tid / bp;
-    for (int i = 0; i < k; ++i) heap[i * SEL_THREADS + tid] = 0ull;
-    if (r >= lanes) return;
-    unsigned long long root = 0ull;
-    const int64_t v0 = (int64_t)blockIdx.x * rows_per_cta;
-    const int64_t v1 = v0 + rows_per_cta < n_sample ? v0 + rows_per_cta : n_sample;
-    constexpr int R = 8;   // sample rows loaded ahead (independent loads in flight)
-    for (int64_t vb = v0 + r; vb < v1; vb += (int64_t)R * lanes) {
-        unsigned long long kq[R];
+__global__ __launch_bounds__(256) void k_sample_transpose(
+    const float *__restrict__ s, int64_t n_sample, int64_t stride, int bp,
+    const int32_t *__restrict__ ext_of, int64_t id_limit, uint32_t *__restrict__ keysT) {
+    __shared__ uint32_t tile[32][33];
+    const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;
+    const int64_t v0 = (int64_t)blockIdx.x * 32;
+    const int c0 = blockIdx.y * 32;
 #pragma unroll
-        for (int q = 0; q < R; ++q) {
-            const int64_t v = vb + (int64_t)q * lanes;
-            kq[q] = 0ull;
-            if (v < v1) {
-                const int64_t j = v * stride;
-                const int32_t id = ext_of[j];
-                if ((int64_t)id < id_limit) kq[q] = sel_key<SIGNED>(s[j * bp + c], (uint32_t)id);
+    for (int i = 0; i < 4; ++i) {
+        const int r = ty + 8 * i;
+        const int64_t v = v0 + r;
+        uint32_t key = 0u;
+        if (v < n_sample) {
+            const int64_t j = v * stride;
+            if ((int64_t)ext_of[j] < id_limit) {
+                const float x = s[j * bp + c0 + tx];
+                key = SIGNED ? ordered_bits(x) : __float_as_uint(x);
             }
         }
-#pragma unroll
-        for (int q = 0; q < R; ++q) {
-            const unsigned long long key = kq[q];
-            if (key <= root) continue;
-            int i = 0;   // replace the minimum, sift down
-            while (true) {
-                const int l = 2 * i + 1, rr = l + 1;
-                if (l >= k) break;
-                int m = l;
-                unsigned long long km = heap[l * SEL_THREADS + tid];
-                if (rr < k) {
-                    const unsigned long long kr = heap[rr * SEL_THREADS + tid];
-                    if (kr < km) {
-                        m = rr;
-                        km = kr;
-                    }
-                }
-                if (km >= key) break;
-                heap[i * SEL_THREADS + tid] = km;
-                i = m;
-            }
-            heap[i * SEL_THREADS + tid] = key;
-            root = heap[tid];
-        }
+        tile[r][tx] = key;
     }
-    const int64_t list = (int64_t)blockIdx.x * lanes + r;
-    unsigned long long *dst = lists_g + (list * bp + c) * k;
-    for (int i = 0; i < k; ++i) dst[i] = heap[i * SEL_THREADS + tid];
+    __syncthreads();
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const int cc = ty + 8 * i;
+        const int64_t v = v0 + tx;
+        if (v < n_sample) keysT[(int64_t)(c0 + cc) * n_sample + v] = tile[tx][cc];
+    }
 }
 
-// bound[c] = k-th largest sampled key of column c (0 if fewer than k);
-// also clears the column's buffer count.
-__global__ __launch_bounds__(SEL_THREADS) void k_sample_bound(
-    const unsigned long long *__restrict__ lists_g, int64_t lists, int bp, int b, int k,
+// bound[c] from column c of keysT: staged in shared memory when it fits,
+// then an MSB-first 8-bit radix select with per-warp histograms, four
+// passes.  Every thread does the same work per key (no data-dependent
+// loops, unlike per-thread heaps whose sift loops diverge in a warp).
+__global__ __launch_bounds__(SEL_THREADS) void k_sample_kth(
+    const uint32_t *__restrict__ keysT, int64_t n_sample, int b, int k,
     unsigned long long *__restrict__ bound, unsigned int *__restrict__ cnt) {
-    __shared__ int hist[256 * (SEL_THREADS / 32)];
-    __shared__ unsigned long long win[64];
-    __shared__ unsigned long long s_prefix;
-    __shared__ int s_remaining, win_n;
-    const int c = blockIdx.x;
+    extern __shared__ uint32_t kst[];                 // [n_sample] when staged
+    __shared__ int hist[(SEL_THREADS / 32) * 256];
+    __shared__ int wsum[SEL_THREADS / 32];
+    __shared__ uint32_t s_prefix;
+    __shared__ int s_rem;
+    const int c = blockIdx.x, tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     if (c >= b) {   // padding column: nothing passes the filter
-        if (threadIdx.x == 0) {
+        if (tid == 0) {
             bound[c] = ~0ull;
             cnt[c] = 0u;
         }
         return;
     }
-    const int64_t total = lists * (int64_t)k;
-    if (total <= BOUND_STAGE) {
-        // the column's keys, list by list (each list's k keys are contiguous)
-        extern __shared__ unsigned long long stage_b[];
-        for (int64_t i = threadIdx.x; i < total; i += SEL_THREADS)
-            stage_b[i] = lists_g[((i / k) * bp + c) * k + (i % k)];
-        __syncthreads();
-        auto key_at = [&](int64_t i) -> unsigned long long { return stage_b[i]; };
-        radix_select(total, k, key_at, win, &win_n, hist, &s_prefix, &s_remaining);
-    } else {
-        auto key_at = [&](int64_t i) -> unsigned long long {
-            return lists_g[((i / k) * bp + c) * k + (i % k)];
-        };
-        radix_select(total, k, key_at, win, &win_n, hist, &s_prefix, &s_remaining);
+    const uint32_t *col = keysT + (int64_t)c * n_sample;
+    const bool staged = n_sample <= KTH_STAGE;
+    if (staged)
+        for (int64_t v = tid; v < n_sample; v += SEL_THREADS) kst[v] = col[v];
+    if (tid == 0) {
+        s_prefix = 0u;
+        s_rem = k;
     }
-    if (threadIdx.x == 0) {
-        bound[c] = win_n >= k ? s_prefix : 0ull;
+    __syncthreads();
+    uint32_t pmask = 0u;
+    for (int pass = 0; pass < 4; ++pass) {
+        const int sh = 24 - 8 * pass;
+        for (int w = 0; w < SEL_THREADS / 32; ++w) hist[w * 256 + tid] = 0;
+        __syncthreads();
+        const uint32_t prefix = s_prefix;
+        const int rem = s_rem;
+        for (int64_t v = tid; v < n_sample; v += SEL_THREADS) {
+            const uint32_t key = staged ? kst[v] : col[v];
+            if ((key & pmask) == prefix) atomicAdd(&hist[warp * 256 + ((key >> sh) & 0xff)], 1);
+        }
+        __syncthreads();
+        // thread t owns digit 255 - t: its count and the inclusive count of
+        // all larger digits; the thread whose range holds rank `rem` wins
+        int cntd = 0;
+        for (int w = 0; w < SEL_THREADS / 32; ++w) cntd += hist[w * 256 + (255 - tid)];
+        int incl = cntd;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int t = __shfl_up_sync(0xffffffffu, incl, o);
+            if (lane >= o) incl += t;
+        }
+        if (lane == 31) wsum[warp] = incl;
+        __syncthreads();
+        for (int w = 0; w < warp; ++w) incl += wsum[w];
+        if (incl >= rem && incl - cntd < rem) {
+            s_rem = rem - (incl - cntd);
+            s_prefix = prefix | ((uint32_t)(255 - tid) << sh);
+        }
+        pmask |= 0xffu << sh;
+        __syncthreads();
+    }
+    if (tid == 0) {
+        // fewer than k keys at all: no thread ever matched, s_prefix stays
+        // 0, which admits everything
+        bound[c] = (unsigned long long)s_prefix << 32;
         cnt[c] = 0u;
     }
 }
@@ -447,21 +455,28 @@ cudaError_t launch_buf_merge_signed(const unsigned int *cnt, const unsigned long
 }
 
 // ------------------------------------------------------------------ launchers
-static cudaError_t launch_bound(const SelectPlan &sp, int b, const unsigned long long *ws,
-                                unsigned long long *bound, unsigned int *cnt, cudaStream_t st) {
+template <bool SIGNED>
+static cudaError_t launch_kth(const SelectPlan &sp, const float *s, int b, const int32_t *ext_of,
+                              int64_t id_limit, unsigned long long *ws, unsigned long long *bound,
+                              unsigned int *cnt, cudaStream_t st) {
     static bool attr[64] = {false};
     int dev = 0;
     cudaGetDevice(&dev);
     if (dev >= 0 && dev < 64 && !attr[dev]) {
-        cudaError_t e = cudaFuncSetAttribute(k_sample_bound,
+        cudaError_t e = cudaFuncSetAttribute(k_sample_kth,
                                              cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             BOUND_STAGE * (int)sizeof(unsigned long long));
+                                             KTH_STAGE * (int)sizeof(uint32_t));
         if (e != cudaSuccess) return e;
         attr[dev] = true;
     }
-    const int64_t total = sp.lists * (int64_t)sp.k;
-    const size_t smem = total <= BOUND_STAGE ? (size_t)total * sizeof(unsigned long long) : 0;
-    k_sample_bound<<<sp.bp, SEL_THREADS, smem, st>>>(ws, sp.lists, sp.bp, b, sp.k, bound, cnt);
+    uint32_t *keysT = (uint32_t *)(ws + sp.off_tr);
+    const dim3 tgrid((unsigned)ceil_div<int64_t>(sp.n_sample, 32), (unsigned)(sp.bp / 32));
+    k_sample_transpose<SIGNED><<<tgrid, 256, 0, st>>>(s, sp.n_sample, sp.stride, sp.bp, ext_of,
+                                                      id_limit, keysT);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    const size_t smem = sp.n_sample <= KTH_STAGE ? (size_t)sp.n_sample * sizeof(uint32_t) : 0;
+    k_sample_kth<<<sp.bp, SEL_THREADS, smem, st>>>(keysT, sp.n_sample, b, sp.k, bound, cnt);
     return cudaGetLastError();
 }
 
@@ -469,26 +484,10 @@ template <bool SIGNED>
 static cudaError_t bound_and_filter(const SelectPlan &sp, const float *s, int b,
                                     const int32_t *ext_of, int64_t id_limit,
                                     unsigned long long *ws, cudaStream_t st, int *launches) {
-    static bool attr[2][64] = {{false}};
-    int dev = 0;
-    cudaGetDevice(&dev);
-    if (dev >= 0 && dev < 64 && !attr[SIGNED][dev]) {
-        cudaError_t e = cudaFuncSetAttribute(k_sample_heaps<SIGNED>,
-                                             cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             64 * SEL_THREADS * (int)sizeof(unsigned long long));
-        if (e != cudaSuccess) return e;
-        attr[SIGNED][dev] = true;
-    }
-    const size_t smem = (size_t)sp.k * SEL_THREADS * sizeof(unsigned long long);
-    const int64_t rows_per_cta = ceil_div<int64_t>(sp.n_sample, sp.grid);
-    k_sample_heaps<SIGNED><<<sp.grid, SEL_THREADS, smem, st>>>(
-        s, sp.n_sample, sp.stride, sp.bp, sp.lanes, sp.k, rows_per_cta, ext_of, id_limit, ws);
-    cudaError_t e = cudaGetLastError();
-    if (e != cudaSuccess) return e;
     unsigned long long *bound = ws + sp.off_bound;
     unsigned int *cnt = (unsigned int *)(ws + sp.off_cnt);
     unsigned long long *buf = ws + sp.off_buf;
-    e = launch_bound(sp, b, ws, bound, cnt, st);
+    cudaError_t e = launch_kth<SIGNED>(sp, s, b, ext_of, id_limit, ws, bound, cnt, st);
     if (e != cudaSuccess) return e;
     const int64_t warps = ceil_div<int64_t>(sp.n, 4);
     int grid = (int)(ceil_div<int64_t>(warps, 8) < (int64_t)device_sm_count() * 8
@@ -511,23 +510,8 @@ static cudaError_t sample_bound(const SelectPlan &sp, const float *s, int b,
                                 const int32_t *ext_of, int64_t id_limit,
                                 unsigned long long *ws, unsigned long long *bound,
                                 cudaStream_t st, int *launches) {
-    static bool attr[2][64] = {{false}};
-    int dev = 0;
-    cudaGetDevice(&dev);
-    if (dev >= 0 && dev < 64 && !attr[SIGNED][dev]) {
-        cudaError_t e = cudaFuncSetAttribute(k_sample_heaps<SIGNED>,
-                                             cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             64 * SEL_THREADS * (int)sizeof(unsigned long long));
-        if (e != cudaSuccess) return e;
-        attr[SIGNED][dev] = true;
-    }
-    const size_t smem = (size_t)sp.k * SEL_THREADS * sizeof(unsigned long long);
-    const int64_t rows_per_cta = ceil_div<int64_t>(sp.n_sample, sp.grid);
-    k_sample_heaps<SIGNED><<<sp.grid, SEL_THREADS, smem, st>>>(
-        s, sp.n_sample, sp.stride, sp.bp, sp.lanes, sp.k, rows_per_cta, ext_of, id_limit, ws);
-    cudaError_t e = cudaGetLastError();
-    if (e != cudaSuccess) return e;
-    e = launch_bound(sp, b, ws, bound, (unsigned int *)(ws + sp.off_cnt), st);
+    cudaError_t e = launch_kth<SIGNED>(sp, s, b, ext_of, id_limit, ws, bound,
+                                       (unsigned int *)(ws + sp.off_cnt), st);
     if (launches) *launches += 2;
     return e;
 }
