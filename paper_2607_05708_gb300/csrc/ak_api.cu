@@ -117,7 +117,13 @@ struct akashic_mem {
     int64_t nnz = 0;
     DevBuf row_ptr, col, aff, w;
     // in-edge transpose + split plan for the propagation hop
-    DevBuf in_ptr, in_src, in_w;
+    DevBuf in_ptr, in_src, in_w, in_aff;
+    DevBuf rstat;                // per chunk ID: (max, 1/sum) of its out-row softmax
+    // spares the relation update writes the next CSR / transpose into (then
+    // swapped with the live arrays), and grow-only scratch for its temporaries
+    DevBuf rp2, col2, aff2, in_ptr2, in_src2, in_aff2, in_w2;
+    DevBuf scr[SCR_COUNT];
+    bool inc_transpose = true;   // relation updates patch the transpose instead of re-sorting
     SplitParams split;
     bool fuse_filter = true;     // top-k filter in the last hop's epilogue
     int64_t n_split = 0, n_segs = 0;
@@ -211,11 +217,36 @@ static akashic_status_t check_status(akashic_mem *m, cudaStream_t st, const char
 
 // Rebuild the in-edge transpose (stable by source, hence sorted by source
 // within each destination), its weights, and the split plan of long rows.
+// Grow-only scratch of a store (UpdateArgs::scratch): 1/8 headroom when a
+// slot has to grow, so slowly growing sizes do not reallocate every call.
+static void *store_scratch(void *ctx, int slot, size_t bytes) {
+    akashic_mem *m = (akashic_mem *)ctx;
+    if (slot < 0 || slot >= SCR_COUNT) return nullptr;
+    DevBuf &b = m->scr[slot];
+    if (bytes > b.cap && b.ensure(bytes + bytes / 8) != AKASHIC_OK) return nullptr;
+    return b.p;
+}
+
+// A scratch buffer seen through the DevBuf-like accessors.
+struct Tmp {
+    void *p;
+    size_t cap;
+    template <typename T> T *as() const { return (T *)p; }
+};
+
+// Grow a spare buffer with 1/4 headroom (contents not kept).
+static akashic_status_t ensure_spare(DevBuf &b, size_t bytes) {
+    return bytes > b.cap ? b.ensure(bytes + bytes / 4) : AKASHIC_OK;
+}
+
+static akashic_status_t build_split_plan(akashic_mem *m, cudaStream_t st);
+
 static akashic_status_t rebuild_in_edges(akashic_mem *m, cudaStream_t st) {
     const int64_t n = m->n, nnz = m->nnz;
     AK_TRY(m->in_ptr.ensure((size_t)(m->cap + 1) * sizeof(int64_t)));
     AK_TRY(m->in_src.ensure((size_t)(nnz > 0 ? nnz : 1) * sizeof(int32_t)));
     AK_TRY(m->in_w.ensure((size_t)(nnz > 0 ? nnz : 1) * sizeof(float)));
+    AK_TRY(m->in_aff.ensure((size_t)(nnz > 0 ? nnz : 1) * sizeof(float)));
     DevBuf src, keys, vals, keys2, vals2, tmp, deg;
     const size_t tmp_bytes = (radix_tmp_bytes(nnz) > scan_tmp_bytes(n + 1) ? radix_tmp_bytes(nnz)
                                                                              : scan_tmp_bytes(n + 1)) +
@@ -248,18 +279,31 @@ static akashic_status_t rebuild_in_edges(akashic_mem *m, cudaStream_t st) {
         CUDA_TRY(radix_sort_pairs(k1, v1, k2, v2, nnz, bits_for(n - 1), tmp.p, tmp.cap, st, &alt2));
         const uint32_t *order = alt2 ? v2 : v1;
         CUDA_TRY(launch_gather_in(order, src.as<int32_t>(), row_of, m->w.as<float>(),
-                                  m->in_src.as<int32_t>(), m->in_w.as<float>(), nnz, st));
+                                  m->aff.as<float>(), m->in_src.as<int32_t>(), m->in_w.as<float>(),
+                                  m->in_aff.as<float>(), nnz, st));
     }
     int64_t *degp = deg.as<int64_t>();
     CUDA_TRY(cudaMemsetAsync(degp, 0, (size_t)(n + 1) * sizeof(int64_t), st));
     CUDA_TRY(launch_in_degree(m->col.as<int32_t>(), m->row_of.as<int32_t>(), nnz, degp, st));
     CUDA_TRY(scan_exclusive(degp, m->in_ptr.as<int64_t>(), n, tmp.p, tmp.cap, st));
-    // split plan: hub rows cut into window segments, segments in window-major order
-    DevBuf nseg, flag, slot_off, split_idx;
-    AK_TRY(nseg.ensure((size_t)(n + 1) * 8));
-    AK_TRY(flag.ensure((size_t)(n + 1) * 8));
-    AK_TRY(slot_off.ensure((size_t)(n + 1) * 8));
-    AK_TRY(split_idx.ensure((size_t)(n + 1) * 8));
+    return build_split_plan(m, st);
+}
+
+// Split plan: hub rows cut into window segments, segments in window-major
+// order, split rows heaviest first.
+static akashic_status_t build_split_plan(akashic_mem *m, cudaStream_t st) {
+    const int64_t n = m->n;
+    // temporaries from the store's scratch (slots SCR_SPLIT0..11)
+    akashic_status_t sc_rc = AKASHIC_OK;
+    auto get = [&](int i, size_t bytes) -> Tmp {
+        void *q = store_scratch(m, SCR_SPLIT0 + i, bytes);
+        if (!q) sc_rc = AKASHIC_ENOMEM;
+        return Tmp{q, bytes};
+    };
+    const Tmp tmp = get(0, scan_tmp_bytes(n + 1) + 4096);
+    const Tmp nseg = get(1, (size_t)(n + 1) * 8), flag = get(2, (size_t)(n + 1) * 8);
+    const Tmp slot_off = get(3, (size_t)(n + 1) * 8), split_idx = get(4, (size_t)(n + 1) * 8);
+    if (sc_rc != AKASHIC_OK) return fail(sc_rc, "relation graph rebuild: out of device memory");
     CUDA_TRY(launch_split_count(m->split, m->in_ptr.as<int64_t>(), m->in_src.as<int32_t>(), n,
                                 nseg.as<int64_t>(), flag.as<int64_t>(), st));
     CUDA_TRY(scan_exclusive(nseg.as<int64_t>(), slot_off.as<int64_t>(), n, tmp.p, tmp.cap, st));
@@ -272,19 +316,16 @@ static akashic_status_t rebuild_in_edges(akashic_mem *m, cudaStream_t st) {
     m->n_segs = n_segs;
     m->n_split = n_split;
     if (n_split > 0) {
-        DevBuf e0, e1, win, order, win2, order2, rtmp;
         AK_TRY(m->split_row.ensure((size_t)n_split * 4));
         AK_TRY(m->split_slot0.ensure((size_t)(n_split + 1) * 8));
         AK_TRY(m->seg_e0.ensure((size_t)n_segs * 8));
         AK_TRY(m->seg_e1.ensure((size_t)n_segs * 8));
         AK_TRY(m->seg_slot.ensure((size_t)n_segs * 4));
-        AK_TRY(e0.ensure((size_t)n_segs * 8));
-        AK_TRY(e1.ensure((size_t)n_segs * 8));
-        AK_TRY(win.ensure((size_t)n_segs * 4));
-        AK_TRY(order.ensure((size_t)n_segs * 4));
-        AK_TRY(win2.ensure((size_t)n_segs * 4));
-        AK_TRY(order2.ensure((size_t)n_segs * 4));
-        AK_TRY(rtmp.ensure(radix_tmp_bytes(n_segs) + 4096));
+        const Tmp e0 = get(5, (size_t)n_segs * 8), e1 = get(6, (size_t)n_segs * 8);
+        const Tmp win = get(7, (size_t)n_segs * 4), order = get(8, (size_t)n_segs * 4);
+        const Tmp win2 = get(9, (size_t)n_segs * 4), order2 = get(10, (size_t)n_segs * 4);
+        const Tmp rtmp = get(11, radix_tmp_bytes(n_segs) + 4096);
+        if (sc_rc != AKASHIC_OK) return fail(sc_rc, "relation graph rebuild: out of device memory");
         CUDA_TRY(launch_split_fill(m->split, m->in_ptr.as<int64_t>(), m->in_src.as<int32_t>(), n,
                                    nseg.as<int64_t>(), slot_off.as<int64_t>(),
                                    split_idx.as<int64_t>(), m->split_row.as<int32_t>(),
@@ -351,6 +392,7 @@ akashic_status_t akashic_mem_create(const akashic_mem_config_t *cfg, akashic_mem
     if (const char *v = getenv("AKASHIC_SPLIT_T")) m->split.split_t = atoll(v) > 0 ? atoll(v) : m->split.split_t;
     if (const char *v = getenv("AKASHIC_SEG_LEN")) m->split.seg_len = atoll(v) > 0 ? atoll(v) : m->split.seg_len;
     if (const char *v = getenv("AKASHIC_FUSE_FILTER")) m->fuse_filter = atoi(v) != 0;
+    if (const char *v = getenv("AKASHIC_FULL_TRANSPOSE")) m->inc_transpose = atoi(v) == 0;
     if (const char *v = getenv("AKASHIC_WIN_ROWS")) m->split.win_rows = atoll(v) > 0 ? atoll(v) : m->split.win_rows;
     akashic_status_t s;
     if ((s = m->emb.ensure((size_t)m->cap * m->dim * 2)) != AKASHIC_OK ||
@@ -358,6 +400,7 @@ akashic_status_t akashic_mem_create(const akashic_mem_config_t *cfg, akashic_mem
         (s = m->ext_of.ensure((size_t)m->cap * 4)) != AKASHIC_OK ||
         (s = m->row_of.ensure((size_t)m->cap * 4)) != AKASHIC_OK ||
         (s = m->max_norm.ensure(4)) != AKASHIC_OK || (s = m->status.ensure(4)) != AKASHIC_OK ||
+        (s = m->rstat.ensure((size_t)m->cap * 8)) != AKASHIC_OK ||
         (s = m->row_ptr.ensure((size_t)(m->cap + 1) * 8)) != AKASHIC_OK ||
         (s = m->in_ptr.ensure((size_t)(m->cap + 1) * 8)) != AKASHIC_OK) {
         delete m;
@@ -485,7 +528,8 @@ akashic_status_t akashic_mem_append_chunks(akashic_mem_t *m, const uint16_t *emb
                                  cudaMemcpyDeviceToDevice, st));
         CUDA_TRY(cudaMemcpyAsync(m->aff.as<float>() + m->nnz, aff + e_lo, (size_t)new_nnz * 4,
                                  cudaMemcpyDeviceToDevice, st));
-        CUDA_TRY(launch_row_softmax(rp, m->aff.as<float>(), m->w.as<float>(), n, st));
+        CUDA_TRY(launch_row_softmax(rp, m->aff.as<float>(), m->w.as<float>(), n,
+                                    m->rstat.as<float2>() + first, st));
     }
     m->n += n;
     m->nnz += new_nnz;
@@ -534,14 +578,15 @@ akashic_status_t akashic_mem_update_relations(akashic_mem_t *m, int64_t first, i
     int64_t nnz_new = m->nnz + n * M * (reciprocal ? 2 : 1);
     if (nnz_new > 0x7fffffffLL)
         return fail(AKASHIC_ECAPACITY, "update: more than 2^31-1 relation edges");
-    DevBuf ncol, naff, nrp, nbr_ids, nbr_cos;
-    AK_TRY(nbr_ids.ensure((size_t)n * M * 4));
-    AK_TRY(nbr_cos.ensure((size_t)n * M * 4));
-    ua.nbr_ids = nbr_ids.as<int32_t>();
-    ua.nbr_cos = nbr_cos.as<float>();
-    AK_TRY(ncol.ensure((size_t)(nnz_new + nnz_new / 4) * 4));
-    AK_TRY(naff.ensure((size_t)(nnz_new + nnz_new / 4) * 4));
-    AK_TRY(nrp.ensure((size_t)(m->cap + 1) * 8));
+    ua.scratch = store_scratch;
+    ua.scratch_ctx = m;
+    ua.nbr_ids = (int32_t *)store_scratch(m, SCR_NBR_IDS, (size_t)n * M * 4);
+    ua.nbr_cos = (float *)store_scratch(m, SCR_NBR_COS, (size_t)n * M * 4);
+    if (!ua.nbr_ids || !ua.nbr_cos) return fail(AKASHIC_ENOMEM, "update: out of device memory");
+    DevBuf &ncol = m->col2, &naff = m->aff2, &nrp = m->rp2;
+    AK_TRY(ensure_spare(ncol, (size_t)nnz_new * 4));
+    AK_TRY(ensure_spare(naff, (size_t)nnz_new * 4));
+    AK_TRY(ensure_spare(nrp, (size_t)(m->cap + 1) * 8));
     {
         PhaseScope ph(m, AKASHIC_PHASE_RELATE, st);
         akashic_status_t r = relate_top_m(ua, st, &ph.launches);
@@ -561,11 +606,69 @@ akashic_status_t akashic_mem_update_relations(akashic_mem_t *m, int64_t first, i
         std::swap(m->col.cap, ncol.cap);
         std::swap(m->aff.p, naff.p);
         std::swap(m->aff.cap, naff.cap);
+        const int64_t nnz_old = m->nnz;
         m->nnz = nnz_new;
         AK_TRY(m->w.ensure(m->col.cap, false));
         CUDA_TRY(launch_row_softmax(m->row_ptr.as<int64_t>(), m->aff.as<float>(), m->w.as<float>(),
-                                    m->n, st));
-        AK_TRY(rebuild_in_edges(m, st));
+                                    m->n, m->rstat.as<float2>(), st));
+        if (!m->inc_transpose || nnz_old == 0) {
+            AK_TRY(rebuild_in_edges(m, st));
+        } else {
+            // patch the transpose: old lists moved, new edges placed, weights
+            // recomputed from the logits (ak_inedges.cu)
+            DevBuf &ptr2 = m->in_ptr2, &src2 = m->in_src2, &aff2 = m->in_aff2, &w2 = m->in_w2;
+            const int64_t rows = m->n, pairs = n * (int64_t)M;
+            AK_TRY(ensure_spare(ptr2, (size_t)(m->cap + 1) * 8));
+            AK_TRY(ensure_spare(src2, (size_t)nnz_new * 4));
+            AK_TRY(ensure_spare(aff2, (size_t)nnz_new * 4));
+            AK_TRY(ensure_spare(w2, (size_t)nnz_new * 4));
+            const size_t tb = (radix_tmp_bytes(pairs) > scan_tmp_bytes(rows + 1)
+                                   ? radix_tmp_bytes(pairs) : scan_tmp_bytes(rows + 1)) + 4096;
+            void *p_inc = store_scratch(m, SCR_IN_INC, (size_t)(rows + 1) * 8);
+            void *p_deg = store_scratch(m, SCR_IN_DEG, (size_t)(rows + 1) * 8);
+            void *p_off = store_scratch(m, SCR_IN_OFF, (size_t)(rows + 1) * 8);
+            void *p_k = store_scratch(m, SCR_KEYS, (size_t)pairs * 4 + 16);
+            void *p_v = store_scratch(m, SCR_VALS, (size_t)pairs * 4 + 16);
+            void *p_k2 = store_scratch(m, SCR_KEYS2, (size_t)pairs * 4 + 16);
+            void *p_v2 = store_scratch(m, SCR_VALS2, (size_t)pairs * 4 + 16);
+            void *p_tmp = store_scratch(m, SCR_TMP, tb);
+            if (!p_inc || !p_deg || !p_off || !p_k || !p_v || !p_k2 || !p_v2 || !p_tmp)
+                return fail(AKASHIC_ENOMEM, "update: out of device memory");
+            InEdgeUpdate u;
+            u.n = rows;
+            u.nnz_new = nnz_new;
+            u.in_ptr_old = m->in_ptr.as<int64_t>();
+            u.in_src_old = m->in_src.as<int32_t>();
+            u.in_aff_old = m->in_aff.as<float>();
+            u.in_ptr_new = ptr2.as<int64_t>();
+            u.in_src_new = src2.as<int32_t>();
+            u.in_aff_new = aff2.as<float>();
+            u.in_w_new = w2.as<float>();
+            u.nbr_ids = ua.nbr_ids;
+            u.nbr_cos = ua.nbr_cos;
+            u.scale = m->rel_scale;
+            u.first = first;
+            u.n_new = n;
+            u.M = M;
+            u.reciprocal = reciprocal != 0;
+            u.row_bits = bits_for(rows - 1);
+            u.row_of = m->row_of.as<int32_t>();
+            u.ext_of = m->ext_of.as<int32_t>();
+            u.rstat = m->rstat.as<float2>();
+            InEdgeScratch sc{(int64_t *)p_inc, (int64_t *)p_deg, (int64_t *)p_off,
+                             (uint32_t *)p_k, (uint32_t *)p_v, (uint32_t *)p_k2, (uint32_t *)p_v2,
+                             p_tmp, tb};
+            CUDA_TRY(launch_in_edges_update(u, sc, st, &ph.launches));
+            std::swap(m->in_ptr.p, ptr2.p);
+            std::swap(m->in_ptr.cap, ptr2.cap);
+            std::swap(m->in_src.p, src2.p);
+            std::swap(m->in_src.cap, src2.cap);
+            std::swap(m->in_aff.p, aff2.p);
+            std::swap(m->in_aff.cap, aff2.cap);
+            std::swap(m->in_w.p, w2.p);
+            std::swap(m->in_w.cap, w2.cap);
+            AK_TRY(build_split_plan(m, st));
+        }
     }
     return AKASHIC_OK;
 }

@@ -119,8 +119,15 @@ cudaError_t radix_sort_pairs(uint32_t *keys, uint32_t *vals, uint32_t *keys_alt,
 cudaError_t launch_edge_src_check(const int64_t *row_ptr, const int32_t *col, int64_t n_rows,
                                   int64_t row_base, int64_t n_total, int32_t *src, int *status,
                                   cudaStream_t st);
+// w = row softmax of the logits, per row: w_e = exp(aff_e - max) * inv with
+// inv = 1 / sum exp(aff - max); (max, inv) of row r go to rstat[r] when
+// rstat is not NULL, so that any copy of a weight (the in-edge transpose)
+// can be recomputed bit for bit by row_softmax_weight.
+__device__ __forceinline__ float row_softmax_weight(float aff, float2 stat) {
+    return expf(aff - stat.x) * stat.y;
+}
 cudaError_t launch_row_softmax(const int64_t *row_ptr, const float *aff, float *w, int64_t n_rows,
-                               cudaStream_t st);
+                               float2 *rstat, cudaStream_t st);
 // The store keeps chunks in HBM in page order: row r holds chunk ext_of[r],
 // chunk c lives in row row_of[c].  The out-edge CSR stays in chunk IDs; the
 // in-edge transpose used by propagation is in rows.
@@ -130,8 +137,41 @@ cudaError_t launch_iota(uint32_t *v, int64_t n, cudaStream_t st);
 cudaError_t launch_map_keys(const uint32_t *sel, const int32_t *ids, const int32_t *row_of,
                             uint32_t *keys, int64_t n, cudaStream_t st);
 cudaError_t launch_gather_in(const uint32_t *order, const int32_t *src, const int32_t *row_of,
-                             const float *w, int32_t *in_src, float *in_w, int64_t nnz,
-                             cudaStream_t st);
+                             const float *w, const float *aff, int32_t *in_src, float *in_w,
+                             float *in_aff, int64_t nnz, cudaStream_t st);
+
+// Incremental in-edge transpose after a relation update (ak_inedges.cu).
+struct InEdgeUpdate {
+    int64_t n;                          // store rows (new chunks included)
+    int64_t nnz_new;                    // edges after the update
+    const int64_t *in_ptr_old;          // [n+1]
+    const int32_t *in_src_old;
+    const float *in_aff_old;
+    int64_t *in_ptr_new;                // [n+1]
+    int32_t *in_src_new;                // [nnz_new]
+    float *in_aff_new, *in_w_new;       // [nnz_new]
+    const int32_t *nbr_ids;             // [n_new][M] chosen prior chunk IDs
+    const float *nbr_cos;               // [n_new][M]
+    float scale;                        // logit = scale * cos
+    int64_t first, n_new;
+    int M;
+    bool reciprocal;
+    int row_bits;                       // key bits of a row index
+    const int32_t *row_of, *ext_of;
+    const float2 *rstat;                // per chunk ID: (max, inv) of its out-row
+};
+struct InEdgeScratch {
+    int64_t *inc, *deg, *fwd_off;       // [n+1] each
+    uint32_t *keys, *vals, *keys2, *vals2;   // [n_new * M] each
+    void *tmp;
+    size_t tmp_bytes;                   // >= radix and scan needs
+};
+cudaError_t launch_in_edges_update(const InEdgeUpdate &u, const InEdgeScratch &s, cudaStream_t st,
+                                   int *launches);
+// in_w[e] = row_softmax_weight(in_aff[e], rstat[ext_of[in_src[e]]])
+cudaError_t launch_in_weights(const int32_t *in_src, const float *in_aff, int64_t nnz,
+                              const int32_t *ext_of, const float2 *rstat, float *in_w,
+                              cudaStream_t st);
 cudaError_t launch_batch_layout(const uint32_t *order, int64_t first, int64_t n, int dim,
                                 const uint16_t *emb_in, uint16_t *emb, const int32_t *page_in,
                                 int64_t first_page, int per_page, int32_t *page_row,

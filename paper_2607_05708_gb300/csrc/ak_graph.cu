@@ -270,7 +270,7 @@ cudaError_t launch_edge_src_check(const int64_t *row_ptr, const int32_t *col, in
 
 // Relation weights: w = softmax of each row's edge logits (one warp per row).
 __global__ void k_row_softmax(const int64_t *__restrict__ row_ptr, const float *__restrict__ aff,
-                              float *__restrict__ w, int64_t n_rows) {
+                              float *__restrict__ w, int64_t n_rows, float2 *__restrict__ rstat) {
     const int lane = threadIdx.x & 31;
     int64_t r = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
     const int64_t stride = ((int64_t)gridDim.x * blockDim.x) >> 5;
@@ -283,17 +283,18 @@ __global__ void k_row_softmax(const int64_t *__restrict__ row_ptr, const float *
         float s = 0.f;
         for (int64_t e = a + lane; e < b; e += 32) s += expf(aff[e] - m);
         for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
-        const float inv = 1.f / s;
-        for (int64_t e = a + lane; e < b; e += 32) w[e] = expf(aff[e] - m) * inv;
+        const float2 stat = make_float2(m, 1.f / s);
+        if (rstat && lane == 0) rstat[r] = stat;
+        for (int64_t e = a + lane; e < b; e += 32) w[e] = row_softmax_weight(aff[e], stat);
     }
 }
 
 cudaError_t launch_row_softmax(const int64_t *row_ptr, const float *aff, float *w, int64_t n_rows,
-                               cudaStream_t st) {
+                               float2 *rstat, cudaStream_t st) {
     if (n_rows <= 0) return cudaSuccess;
     int64_t warps = n_rows < (int64_t)device_sm_count() * 64 ? n_rows : (int64_t)device_sm_count() * 64;
     k_row_softmax<<<(unsigned)ceil_div<int64_t>(warps * 32, 256), 256, 0, st>>>(row_ptr, aff, w,
-                                                                              n_rows);
+                                                                              n_rows, rstat);
     return cudaGetLastError();
 }
 
@@ -345,20 +346,23 @@ cudaError_t launch_iota(uint32_t *v, int64_t n, cudaStream_t st) {
 
 __global__ void k_gather_in(const uint32_t *__restrict__ order, const int32_t *__restrict__ src,
                             const int32_t *__restrict__ row_of, const float *__restrict__ w,
-                            int32_t *__restrict__ in_src, float *__restrict__ in_w, int64_t nnz) {
+                            const float *__restrict__ aff, int32_t *__restrict__ in_src,
+                            float *__restrict__ in_w, float *__restrict__ in_aff, int64_t nnz) {
     for (int64_t p = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; p < nnz;
          p += (int64_t)gridDim.x * blockDim.x) {
         uint32_t e = order[p];
         in_src[p] = row_of[src[e]];
         in_w[p] = w[e];
+        in_aff[p] = aff[e];
     }
 }
 
 cudaError_t launch_gather_in(const uint32_t *order, const int32_t *src, const int32_t *row_of,
-                             const float *w, int32_t *in_src, float *in_w, int64_t nnz,
-                             cudaStream_t st) {
+                             const float *w, const float *aff, int32_t *in_src, float *in_w,
+                             float *in_aff, int64_t nnz, cudaStream_t st) {
     if (nnz <= 0) return cudaSuccess;
-    k_gather_in<<<device_sm_count() * 8, 256, 0, st>>>(order, src, row_of, w, in_src, in_w, nnz);
+    k_gather_in<<<device_sm_count() * 8, 256, 0, st>>>(order, src, row_of, w, aff, in_src, in_w,
+                                                       in_aff, nnz);
     return cudaGetLastError();
 }
 

@@ -33,24 +33,16 @@ static akashic_status_t relate_top_m_batched(const UpdateArgs &a, cudaStream_t s
     const int64_t n_old = a.n_rows;
     int bp_max = 32;
     while (bp_max < 256 && bp_max < a.n_new) bp_max <<= 1;
-    uint16_t *qp = nullptr;
-    float *dots = nullptr;
-    unsigned long long *cand = nullptr;
-    cudaError_t e = cudaMalloc(&qp, (size_t)bp_max * a.dim * 2);
-    if (e == cudaSuccess) e = cudaMalloc(&dots, (size_t)n_old * bp_max * 4);
-    if (e == cudaSuccess) {
-        int64_t words = 0;
-        for (int bp = 32; bp <= bp_max; bp <<= 1) {
-            SelectPlan sp = select_plan(n_old, bp, a.M, device_sm_count());
-            words = sp.words > words ? sp.words : words;
-        }
-        e = cudaMalloc(&cand, (size_t)words * 8);
+    int64_t words = 0;
+    for (int bp = 32; bp <= bp_max; bp <<= 1) {
+        SelectPlan sp = select_plan(n_old, bp, a.M, device_sm_count());
+        words = sp.words > words ? sp.words : words;
     }
-    akashic_status_t rc = AKASHIC_OK;
-    if (e != cudaSuccess) {
-        cudaGetLastError();
-        rc = AKASHIC_ENOMEM;
-    }
+    uint16_t *qp = (uint16_t *)a.get(SCR_QP, (size_t)bp_max * a.dim * 2);
+    float *dots = (float *)a.get(SCR_DOTS, (size_t)n_old * bp_max * 4);
+    unsigned long long *cand = (unsigned long long *)a.get(SCR_CAND, (size_t)words * 8);
+    akashic_status_t rc = (qp && dots && cand) ? AKASHIC_OK : AKASHIC_ENOMEM;
+    cudaError_t e = cudaSuccess;
     for (int64_t off = 0; rc == AKASHIC_OK && off < a.n_new; off += 256) {
         const int b = (int)(a.n_new - off < 256 ? a.n_new - off : 256);
         int bp = 32;
@@ -68,9 +60,6 @@ static akashic_status_t relate_top_m_batched(const UpdateArgs &a, cudaStream_t s
         if (launches) *launches += 1;
     }
     if (rc == AKASHIC_OK && cudaStreamSynchronize(st) != cudaSuccess) rc = AKASHIC_ECUDA;
-    cudaFree(qp);
-    cudaFree(dots);
-    cudaFree(cand);
     return rc;
 }
 
@@ -90,23 +79,16 @@ akashic_status_t relate_top_m(const UpdateArgs &a, cudaStream_t st, int *launche
     const int64_t n_sample = ceil_div<int64_t>(n, stride);
     const int64_t cap = 4 * (int64_t)a.M * stride > 8192 ? 4 * (int64_t)a.M * stride : 8192;
     const SelectPlan sp = select_plan(n_sample, 256, a.M, sms, 1);
-    uint16_t *qp = nullptr;
-    float *sdots = nullptr;
-    int32_t *ext_s = nullptr;
-    unsigned long long *ws = nullptr, *bound = nullptr, *buf = nullptr;
-    unsigned int *cnt = nullptr;
-    cudaError_t e = cudaMalloc(&qp, (size_t)n_pad * a.dim * 2);
-    if (e == cudaSuccess) e = cudaMalloc(&sdots, (size_t)n_sample * 256 * 4);
-    if (e == cudaSuccess) e = cudaMalloc(&ext_s, (size_t)n_sample * 4);
-    if (e == cudaSuccess) e = cudaMalloc(&ws, (size_t)sp.words * 8);
-    if (e == cudaSuccess) e = cudaMalloc(&bound, (size_t)n_pad * 8);
-    if (e == cudaSuccess) e = cudaMalloc(&cnt, (size_t)n_pad * 4);
-    if (e == cudaSuccess) e = cudaMalloc(&buf, (size_t)a.n_new * cap * 8);
-    akashic_status_t rc = AKASHIC_OK;
-    if (e != cudaSuccess) {
-        cudaGetLastError();
-        rc = AKASHIC_ENOMEM;
-    }
+    uint16_t *qp = (uint16_t *)a.get(SCR_QP, (size_t)n_pad * a.dim * 2);
+    float *sdots = (float *)a.get(SCR_SDOTS, (size_t)n_sample * 256 * 4);
+    int32_t *ext_s = (int32_t *)a.get(SCR_EXTS, (size_t)n_sample * 4);
+    unsigned long long *ws = (unsigned long long *)a.get(SCR_WS, (size_t)sp.words * 8);
+    unsigned long long *bound = (unsigned long long *)a.get(SCR_BOUND, (size_t)n_pad * 8);
+    unsigned int *cnt = (unsigned int *)a.get(SCR_CNT, (size_t)n_pad * 4);
+    unsigned long long *buf = (unsigned long long *)a.get(SCR_BUF, (size_t)a.n_new * cap * 8);
+    akashic_status_t rc =
+        (qp && sdots && ext_s && ws && bound && cnt && buf) ? AKASHIC_OK : AKASHIC_ENOMEM;
+    cudaError_t e = cudaSuccess;
     bool overflow = false;
     if (rc == AKASHIC_OK) {
         k_gather_rows<<<sms * 2, 256, 0, st>>>(a.emb, a.row_of, a.first, (int)a.n_new, (int)n_pad,
@@ -146,13 +128,6 @@ akashic_status_t relate_top_m(const UpdateArgs &a, cudaStream_t st, int *launche
         if (e == cudaSuccess && rc == AKASHIC_OK) e = cudaStreamSynchronize(st);
         if (e != cudaSuccess && rc == AKASHIC_OK) rc = AKASHIC_ECUDA;
     }
-    cudaFree(qp);
-    cudaFree(sdots);
-    cudaFree(ext_s);
-    cudaFree(ws);
-    cudaFree(bound);
-    cudaFree(cnt);
-    cudaFree(buf);
     if (rc == AKASHIC_OK && overflow) rc = relate_top_m_batched(a, st, launches);
     return rc;
 }
@@ -253,25 +228,20 @@ akashic_status_t csr_insert(const UpdateArgs &a, const int64_t *rp, const int32_
                             float *new_aff, cudaStream_t st, int *launches) {
     const int64_t n_rows = a.n_rows, pairs = a.n_new * a.M;
     const int sms = device_sm_count();
-    int64_t *deg = nullptr, *recip = nullptr, *recip_off = nullptr;
-    uint32_t *keys = nullptr, *vals = nullptr, *keys2 = nullptr, *vals2 = nullptr;
-    void *tmp = nullptr;
     const size_t tmp_bytes = (radix_tmp_bytes(pairs) > scan_tmp_bytes(n_rows + 1)
                                   ? radix_tmp_bytes(pairs)
                                   : scan_tmp_bytes(n_rows + 1)) + 4096;
-    cudaError_t e = cudaMalloc(&deg, (size_t)(n_rows + 1) * 8);
-    if (e == cudaSuccess) e = cudaMalloc(&recip, (size_t)(n_rows + 1) * 8);
-    if (e == cudaSuccess) e = cudaMalloc(&recip_off, (size_t)(n_rows + 1) * 8);
-    if (e == cudaSuccess) e = cudaMalloc(&keys, (size_t)pairs * 4 + 16);
-    if (e == cudaSuccess) e = cudaMalloc(&vals, (size_t)pairs * 4 + 16);
-    if (e == cudaSuccess) e = cudaMalloc(&keys2, (size_t)pairs * 4 + 16);
-    if (e == cudaSuccess) e = cudaMalloc(&vals2, (size_t)pairs * 4 + 16);
-    if (e == cudaSuccess) e = cudaMalloc(&tmp, tmp_bytes);
-    akashic_status_t rc = AKASHIC_OK;
-    if (e != cudaSuccess) {
-        cudaGetLastError();
-        rc = AKASHIC_ENOMEM;
-    }
+    int64_t *deg = (int64_t *)a.get(SCR_DEG, (size_t)(n_rows + 1) * 8);
+    int64_t *recip = (int64_t *)a.get(SCR_RECIP, (size_t)(n_rows + 1) * 8);
+    int64_t *recip_off = (int64_t *)a.get(SCR_RECIP_OFF, (size_t)(n_rows + 1) * 8);
+    uint32_t *keys = (uint32_t *)a.get(SCR_KEYS, (size_t)pairs * 4 + 16);
+    uint32_t *vals = (uint32_t *)a.get(SCR_VALS, (size_t)pairs * 4 + 16);
+    uint32_t *keys2 = (uint32_t *)a.get(SCR_KEYS2, (size_t)pairs * 4 + 16);
+    uint32_t *vals2 = (uint32_t *)a.get(SCR_VALS2, (size_t)pairs * 4 + 16);
+    void *tmp = a.get(SCR_TMP, tmp_bytes);
+    akashic_status_t rc = (deg && recip && recip_off && keys && vals && keys2 && vals2 && tmp)
+                              ? AKASHIC_OK : AKASHIC_ENOMEM;
+    cudaError_t e = cudaSuccess;
     int L = 0;
     if (rc == AKASHIC_OK) {
         k_check_no_edge_into<<<sms * 4, 256, 0, st>>>(col, nnz, a.first, a.first + a.n_new, a.status);
@@ -312,14 +282,6 @@ akashic_status_t csr_insert(const UpdateArgs &a, const int64_t *rp, const int32_
         if (e != cudaSuccess) rc = AKASHIC_ECUDA;
     }
     if (launches) *launches += L;
-    cudaFree(deg);
-    cudaFree(recip);
-    cudaFree(recip_off);
-    cudaFree(keys);
-    cudaFree(vals);
-    cudaFree(keys2);
-    cudaFree(vals2);
-    cudaFree(tmp);
     return rc;
 }
 

@@ -5,6 +5,18 @@
 
 namespace ak {
 
+// Scratch slots of the store's grow-only update workspace.
+enum UpdateScratchSlot {
+    SCR_QP = 0, SCR_SDOTS, SCR_EXTS, SCR_WS, SCR_BOUND, SCR_CNT, SCR_BUF,   // relate (fused)
+    SCR_DOTS, SCR_CAND,                                                      // relate (batched)
+    SCR_DEG, SCR_RECIP, SCR_RECIP_OFF, SCR_KEYS, SCR_VALS, SCR_KEYS2, SCR_VALS2, SCR_TMP,
+    SCR_NBR_IDS, SCR_NBR_COS,                                                // update results
+    SCR_IN_INC, SCR_IN_DEG, SCR_IN_OFF,                                      // transpose patch
+    SCR_SPLIT0, SCR_SPLIT1, SCR_SPLIT2, SCR_SPLIT3, SCR_SPLIT4, SCR_SPLIT5,  // hub plan
+    SCR_SPLIT6, SCR_SPLIT7, SCR_SPLIT8, SCR_SPLIT9, SCR_SPLIT10, SCR_SPLIT11,
+    SCR_COUNT
+};
+
 struct UpdateArgs {
     const uint16_t *emb;   // store embeddings (n_rows x dim), rows in page order
     const int32_t *ext_of; // chunk ID of each row
@@ -19,6 +31,14 @@ struct UpdateArgs {
     int *status;
     int32_t *nbr_ids;      // [n_new * M] selected prior chunks, (cos desc, id asc)
     float *nbr_cos;        // [n_new * M]
+    // Grow-only scratch owned by the store: scratch(ctx, slot, bytes) returns
+    // a device buffer of at least `bytes` that stays allocated across calls
+    // (NULL if allocation fails), so the per-call temporaries cost no
+    // cudaMalloc / cudaFree once their sizes have been seen.  A call must
+    // not return before its work on these buffers has finished.
+    void *(*scratch)(void *ctx, int slot, size_t bytes);
+    void *scratch_ctx;
+    void *get(int slot, size_t bytes) const { return scratch(scratch_ctx, slot, bytes); }
 };
 
 // a6: top-M prior neighbours of every new chunk by <e_new, e_prior>.

@@ -225,6 +225,60 @@ def test_capacity_and_bad_csr():
     assert st.size() == (2, 1)
 
 
+def _pages_after_appends(wl, batches):
+    """Page table of a store holding wl (clustered placement) after appends
+    of the given sizes without a page table: each batch takes fresh pages
+    in ID order, starting after the last page in use."""
+    pages = [wl.page_of["clustered"].astype(np.int64)]
+    nxt = int(pages[0].max()) + 1
+    for n_b in batches:
+        pages.append(nxt + np.arange(n_b) // wl.chunks_per_page)
+        nxt += -(-n_b // wl.chunks_per_page)
+    return np.concatenate(pages).astype(np.int32)
+
+
+def _retrieval_on_store(wl, store, batches):
+    """Retrieval through the store after updates vs the oracle on the graph
+    the store exports (the transpose used by propagation is checked by it)."""
+    import dataclasses
+    n_new = sum(batches)
+    rp, col, aff, _ = (t.cpu().numpy() for t in store.export_csr())
+    wl2 = dataclasses.replace(wl, emb=np.concatenate([wl.emb, wl.new_emb[:n_new]]), row_ptr=rp,
+                              col=col, aff=aff,
+                              page_of={"clustered": _pages_after_appends(wl, batches)})
+    _, got = gpu_retrieve(wl2, "clustered", store=store)
+    ref = oracle_retrieve(wl2, "clustered")
+    assert_retrieval_parity(wl2, "clustered", got, ref)
+
+
+def test_retrieval_after_update():
+    """Retrieval on the store right after a relation update (the in-edge
+    transpose is patched, not rebuilt): 64 new chunks into 16384."""
+    wl = synth.workload(3, scale=1 / 64)
+    store = check_update(wl)
+    _retrieval_on_store(wl, store, [wl.new_emb.shape[0]])
+
+
+def test_retrieval_after_two_updates():
+    """Two appends + updates in a row (the second links new chunks to rows
+    that gained in-edges in the first), then retrieval parity."""
+    import torch
+    from paper_2607_05708_gb300 import MemStore
+    wl = synth.workload(3, scale=1 / 64)
+    n_new = wl.new_emb.shape[0]
+    store = MemStore.from_arrays(wl.emb, wl.page_of["clustered"], wl.row_ptr, wl.col, wl.aff,
+                                 capacity=wl.n + n_new, chunks_per_page=wl.chunks_per_page,
+                                 temperature=wl.tau, relation_scale=wl.relation_scale)
+    half = n_new // 2
+    for a, b in ((0, half), (half, n_new)):
+        new = torch.from_numpy(np.ascontiguousarray(wl.new_emb[a:b]).view(np.int16)).cuda()
+        first = store.append_chunks(new)
+        assert first == wl.n + a
+        store.update_relations(first, b - a, wl.top_m, reciprocal=True)
+    store.sync()
+    _retrieval_on_store(wl, store, [half, n_new - half])
+
+
 @pytest.fixture(scope="module")
 def update_full():
     return synth.workload(3)
