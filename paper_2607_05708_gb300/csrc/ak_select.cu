@@ -163,15 +163,21 @@ __global__ __launch_bounds__(256) void k_sample_transpose(
 }
 
 // bound[c] from column c of keysT: staged in shared memory when it fits,
-// then an MSB-first 8-bit radix select with per-warp histograms, four
-// passes.  Every thread does the same work per key (no data-dependent
-// loops, unlike per-thread heaps whose sift loops diverge in a warp).
+// then an MSB-first radix select over the bits below the column's common
+// prefix (the sampled values of one column mostly share sign, exponent and
+// leading mantissa bits, so starting below them both saves passes and
+// spreads the first digit).  Histograms are replicated per warp and per
+// lane quarter to cut shared-memory atomic contention on popular digits;
+// every thread does the same work per key (no data-dependent loops).
+constexpr int KTH_REP = (SEL_THREADS / 32) * 4;   // histogram replicas
+
 __global__ __launch_bounds__(SEL_THREADS) void k_sample_kth(
     const uint32_t *__restrict__ keysT, int64_t n_sample, int b, int k,
     unsigned long long *__restrict__ bound, unsigned int *__restrict__ cnt) {
     extern __shared__ uint32_t kst[];                 // [n_sample] when staged
-    __shared__ int hist[(SEL_THREADS / 32) * 256];
+    __shared__ int hist[KTH_REP * 256];
     __shared__ int wsum[SEL_THREADS / 32];
+    __shared__ uint32_t red_or[SEL_THREADS / 32], red_and[SEL_THREADS / 32];
     __shared__ uint32_t s_prefix;
     __shared__ int s_rem;
     const int c = blockIdx.x, tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -184,29 +190,57 @@ __global__ __launch_bounds__(SEL_THREADS) void k_sample_kth(
     }
     const uint32_t *col = keysT + (int64_t)c * n_sample;
     const bool staged = n_sample <= KTH_STAGE;
-    if (staged)
-        for (int64_t v = tid; v < n_sample; v += SEL_THREADS) kst[v] = col[v];
+    // stage, and find the bits on which the column's keys differ
+    uint32_t k_or = 0u, k_and = ~0u;
+    for (int64_t v = tid; v < n_sample; v += SEL_THREADS) {
+        const uint32_t x = col[v];
+        if (staged) kst[v] = x;
+        k_or |= x;
+        k_and &= x;
+    }
+    for (int o = 16; o > 0; o >>= 1) {
+        k_or |= __shfl_xor_sync(0xffffffffu, k_or, o);
+        k_and &= __shfl_xor_sync(0xffffffffu, k_and, o);
+    }
+    if (lane == 0) {
+        red_or[warp] = k_or;
+        red_and[warp] = k_and;
+    }
+    __syncthreads();
+    k_or = 0u;
+    k_and = ~0u;
+    for (int w = 0; w < SEL_THREADS / 32; ++w) {
+        k_or |= red_or[w];
+        k_and &= red_and[w];
+    }
+    const uint32_t diff = k_or & ~k_and;              // bits that vary
+    const int top0 = diff ? 31 - __clz(diff) : -1;    // highest varying bit
+    // bits above top0, identical in every key (all bits if no bit varies)
+    const uint32_t above = top0 < 0 ? ~0u : (top0 == 31 ? 0u : ~((2u << top0) - 1u));
+    const uint32_t common = k_and & above;
     if (tid == 0) {
-        s_prefix = 0u;
+        s_prefix = common;
         s_rem = k;
     }
     __syncthreads();
-    uint32_t pmask = 0u;
-    for (int pass = 0; pass < 4; ++pass) {
-        const int sh = 24 - 8 * pass;
-        for (int w = 0; w < SEL_THREADS / 32; ++w) hist[w * 256 + tid] = 0;
+    uint32_t pmask = above;                           // bits fixed so far
+    const int hrep = (warp * 4 + (lane & 3)) * 256;
+    for (int top = top0; top >= 0; top -= 8) {
+        const int sh = top >= 7 ? top - 7 : 0;
+        const uint32_t dmask = (2u << (top - sh)) - 1u;
+        for (int i = tid; i < KTH_REP * 256; i += SEL_THREADS) hist[i] = 0;
         __syncthreads();
         const uint32_t prefix = s_prefix;
         const int rem = s_rem;
         for (int64_t v = tid; v < n_sample; v += SEL_THREADS) {
             const uint32_t key = staged ? kst[v] : col[v];
-            if ((key & pmask) == prefix) atomicAdd(&hist[warp * 256 + ((key >> sh) & 0xff)], 1);
+            if ((key & pmask) == prefix) atomicAdd(&hist[hrep + ((key >> sh) & dmask)], 1);
         }
         __syncthreads();
         // thread t owns digit 255 - t: its count and the inclusive count of
         // all larger digits; the thread whose range holds rank `rem` wins
         int cntd = 0;
-        for (int w = 0; w < SEL_THREADS / 32; ++w) cntd += hist[w * 256 + (255 - tid)];
+        for (int r = 0; r < KTH_REP; ++r) cntd += hist[r * 256 + (255 - tid)];
         int incl = cntd;
 #pragma unroll
         for (int o = 1; o < 32; o <<= 1) {
@@ -220,13 +254,14 @@ __global__ __launch_bounds__(SEL_THREADS) void k_sample_kth(
             s_rem = rem - (incl - cntd);
             s_prefix = prefix | ((uint32_t)(255 - tid) << sh);
         }
-        pmask |= 0xffu << sh;
+        pmask |= dmask << sh;
         __syncthreads();
     }
     if (tid == 0) {
-        // fewer than k keys at all: no thread ever matched, s_prefix stays
-        // 0, which admits everything
-        bound[c] = (unsigned long long)s_prefix << 32;
+        // fewer than k keys: no thread ever matched and the prefix has not
+        // reached a key, so admit everything
+        const bool found = n_sample >= k;
+        bound[c] = found ? (unsigned long long)s_prefix << 32 : 0ull;
         cnt[c] = 0u;
     }
 }
