@@ -126,7 +126,7 @@ __device__ void radix_select(int64_t total, int k, KeyAt key_at, unsigned long l
 // chunk-ID half zero (every key of that value clears it); 0 (admit all) if
 // the sample holds fewer than k real values.  Sample rows are j = v*stride,
 // v < n_sample; rows whose chunk ID is >= id_limit count as value-key 0.
-constexpr int KTH_STAGE = 49152;   // sampled keys staged per CTA (192 KiB)
+constexpr int KTH_STAGE = 40960;   // sampled keys staged per CTA (160 KiB dynamic + ~49 KiB static)
 
 // keysT[c][v] = key of sample row v in column c: 32 x 32 tiles through
 // shared memory, so both the row reads and the column writes are
@@ -170,6 +170,7 @@ __global__ __launch_bounds__(256) void k_sample_transpose(
 // lane quarter to cut shared-memory atomic contention on popular digits;
 // every thread does the same work per key (no data-dependent loops).
 constexpr int KTH_REP = (SEL_THREADS / 32) * 4;   // histogram replicas
+constexpr int KTH_CBUF = 4096;                    // keys kept after the first digit
 
 __global__ __launch_bounds__(SEL_THREADS) void k_sample_kth(
     const uint32_t *__restrict__ keysT, int64_t n_sample, int b, int k,
@@ -178,8 +179,9 @@ __global__ __launch_bounds__(SEL_THREADS) void k_sample_kth(
     __shared__ int hist[KTH_REP * 256];
     __shared__ int wsum[SEL_THREADS / 32];
     __shared__ uint32_t red_or[SEL_THREADS / 32], red_and[SEL_THREADS / 32];
+    __shared__ uint32_t cbuf[KTH_CBUF];
     __shared__ uint32_t s_prefix;
-    __shared__ int s_rem;
+    __shared__ int s_rem, s_match, s_cn;
     const int c = blockIdx.x, tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     if (c >= b) {   // padding column: nothing passes the filter
         if (tid == 0) {
@@ -225,6 +227,10 @@ __global__ __launch_bounds__(SEL_THREADS) void k_sample_kth(
     __syncthreads();
     uint32_t pmask = above;                           // bits fixed so far
     const int hrep = (warp * 4 + (lane & 3)) * 256;
+    // keys still in play: the whole column, and after a digit that leaves
+    // at most KTH_CBUF candidates, just those (compacted into cbuf)
+    const uint32_t *keys = staged ? kst : col;
+    int64_t len = n_sample;
     for (int top = top0; top >= 0; top -= 8) {
         const int sh = top >= 7 ? top - 7 : 0;
         const uint32_t dmask = (2u << (top - sh)) - 1u;
@@ -232,8 +238,8 @@ __global__ __launch_bounds__(SEL_THREADS) void k_sample_kth(
         __syncthreads();
         const uint32_t prefix = s_prefix;
         const int rem = s_rem;
-        for (int64_t v = tid; v < n_sample; v += SEL_THREADS) {
-            const uint32_t key = staged ? kst[v] : col[v];
+        for (int64_t v = tid; v < len; v += SEL_THREADS) {
+            const uint32_t key = keys[v];
             if ((key & pmask) == prefix) atomicAdd(&hist[hrep + ((key >> sh) & dmask)], 1);
         }
         __syncthreads();
@@ -253,9 +259,21 @@ __global__ __launch_bounds__(SEL_THREADS) void k_sample_kth(
         if (incl >= rem && incl - cntd < rem) {
             s_rem = rem - (incl - cntd);
             s_prefix = prefix | ((uint32_t)(255 - tid) << sh);
+            s_match = cntd;
         }
         pmask |= dmask << sh;
+        if (tid == 0) s_cn = 0;
         __syncthreads();
+        if (sh > 0 && len > KTH_CBUF && n_sample >= k && s_match <= KTH_CBUF) {
+            const uint32_t pre = s_prefix;
+            for (int64_t v = tid; v < len; v += SEL_THREADS) {
+                const uint32_t key = keys[v];
+                if ((key & pmask) == pre) cbuf[atomicAdd(&s_cn, 1)] = key;
+            }
+            __syncthreads();
+            keys = cbuf;
+            len = s_match;
+        }
     }
     if (tid == 0) {
         // fewer than k keys: no thread ever matched and the prefix has not
