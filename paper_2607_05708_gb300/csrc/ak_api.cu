@@ -729,6 +729,7 @@ akashic_status_t akashic_mem_retrieve(akashic_mem_t *m, const uint16_t *q, int32
             ph.launches += 1;
         }
         const float *fin = sc->u.as<float>();
+        ColumnRecompute rc{};
         if (eff_hops >= 1) {
             HopPlan hp;
             hp.split = m->split;
@@ -746,6 +747,8 @@ akashic_status_t akashic_mem_retrieve(akashic_mem_t *m, const uint16_t *q, int32
             hp.split_order = m->split_order.as<int32_t>();
             float *bufs[2] = {sc->sa.as<float>(), sc->sb.as<float>()};
             unsigned long long *ws = sc->cand.as<unsigned long long>();
+            rc = ColumnRecompute{sc->u.as<float>(), nullptr, hp.in_ptr, hp.in_src, hp.in_w, alpha,
+                                 nullptr};
             for (int h = 0; h < eff_hops; ++h) {
                 float *out = bufs[h & 1];
                 const bool last = m->fuse_filter && h == eff_hops - 1;
@@ -765,6 +768,10 @@ akashic_status_t akashic_mem_retrieve(akashic_mem_t *m, const uint16_t *q, int32
                 CUDA_TRY(launch_hop(hp, sc->u.as<float>(), fin, out, bp, alpha,
                                     sc->partial.as<float>(), sc->counters.as<int>(),
                                     last ? &flt : nullptr, st, &ph.launches));
+                if (last) {
+                    rc.prev = fin;
+                    rc.dst = out;
+                }
                 fin = out;
             }
         }
@@ -777,7 +784,8 @@ akashic_status_t akashic_mem_retrieve(akashic_mem_t *m, const uint16_t *q, int32
                                            sc->zpart.as<float>(), zrows, m->ext_of.as<int32_t>(),
                                            m->row_of.as<int32_t>(), m->page_of.as<int32_t>(),
                                            ids + (int64_t)off * k, scores + (int64_t)off * k,
-                                           pids, npg, m->status.as<int>(), st, &ph.launches));
+                                           pids, npg, m->status.as<int>(), &rc, st,
+                                           &ph.launches));
             else
                 CUDA_TRY(launch_select(sp, fin, b, sc->cand.as<unsigned long long>(),
                                        sc->zpart.as<float>(), zrows, m->ext_of.as<int32_t>(),

@@ -266,14 +266,26 @@ cudaError_t launch_select_signed(const SelectPlan &sp, const float *s, int b,
 cudaError_t launch_sample_bound(const SelectPlan &sp, const float *s, int b,
                                 const int32_t *ext_of, unsigned long long *ws, cudaStream_t st,
                                 int *launches);
+// A column of the last hop recomputed by the merge when the filter fused
+// into that hop (which writes no output slab) overflowed its buffer:
+// dst[j,c] = u[j,c] + alpha * sum_{e in in(j)} in_w[e] * prev[in_src[e],c].
+struct ColumnRecompute {
+    const float *u, *prev;
+    const int64_t *in_ptr;
+    const int32_t *in_src;
+    const float *in_w;
+    float alpha;
+    float *dst;   // [n][bp]; the merge reads the overflowed column from here
+};
 // Merge only: the k winners per column from the buffers filled by a filter
-// pass (falls back to the column of `s` where a buffer overflowed).
+// pass (falls back to the column of `s` where a buffer overflowed, after
+// recomputing it into s when `rc` is given; then s must be rc->dst).
 cudaError_t launch_topk_merge(const SelectPlan &sp, const float *s, int b,
                               const unsigned long long *ws, const float *zpart, int64_t n_ztiles,
                               const int32_t *ext_of, const int32_t *row_of,
                               const int32_t *page_row, int64_t *ids, float *scores,
-                              int32_t *page_ids, int32_t *n_pages, int *status, cudaStream_t st,
-                              int *launches);
+                              int32_t *page_ids, int32_t *n_pages, int *status,
+                              const ColumnRecompute *rc, cudaStream_t st, int *launches);
 cudaError_t launch_sample_bound_signed(const SelectPlan &sp, const float *s, int b,
                                        const int32_t *ext_of, int64_t id_limit,
                                        unsigned long long *ws, unsigned long long *bound,

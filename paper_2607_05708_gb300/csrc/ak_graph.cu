@@ -744,12 +744,16 @@ __device__ __forceinline__ void hop_fixup_row(int64_t j, int64_t a, int64_t b,
             o[v].y = fmaf(alpha, acc[v].y, o[v].y);
             o[v].z = fmaf(alpha, acc[v].z, o[v].z);
             o[v].w = fmaf(alpha, acc[v].w, o[v].w);
-            st_stream(out4 + j * S::F + sub + 32 * v, o[v]);
+            if constexpr (!FILTER) st_stream(out4 + j * S::F + sub + 32 * v, o[v]);
         }
         hop_emit<BP, FILTER>(f, thr, thr_hi, sub, id, o);
     }
 }
 
+// With the filter (the last hop) the output slab is not written: the
+// selection needs only the keys the filter appends (a query whose buffer
+// overflows gets its column recomputed by the merge).
+//
 // One queue: first the split rows (their segment partials are complete,
 // the segment kernel ran before), heaviest first, one warp each; then the
 // rows kept whole, ROWS_PER_GRAB consecutive rows per claim (load
@@ -820,7 +824,7 @@ __global__ __launch_bounds__(256, 3) void k_hop_rows(const int64_t *__restrict__
                     b[v].y = fmaf(alpha, acc[v].y, b[v].y);
                     b[v].z = fmaf(alpha, acc[v].z, b[v].z);
                     b[v].w = fmaf(alpha, acc[v].w, b[v].w);
-                    st_stream(out4 + j * S::F + sub + 32 * v, b[v]);
+                    if constexpr (!FILTER) st_stream(out4 + j * S::F + sub + 32 * v, b[v]);
                 }
                 hop_emit<BP, FILTER>(f, thr, thr_hi, sub, id, b);
             }

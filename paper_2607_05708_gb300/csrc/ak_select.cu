@@ -390,7 +390,8 @@ __global__ __launch_bounds__(SEL_THREADS) void k_topk_merge(
     const unsigned int *__restrict__ cnt, const unsigned long long *__restrict__ buf, int64_t cap,
     const float *__restrict__ zpart, int64_t n_ztiles, const int32_t *__restrict__ row_of,
     const int32_t *__restrict__ page_row, int64_t *__restrict__ ids, float *__restrict__ scores,
-    int32_t *__restrict__ page_ids, int32_t *__restrict__ n_pages, int *status) {
+    int32_t *__restrict__ page_ids, int32_t *__restrict__ n_pages, int *status,
+    const ColumnRecompute rc) {
     __shared__ int hist[256 * (SEL_THREADS / 32)];
     __shared__ unsigned long long stage[SEL_STAGE];
     __shared__ unsigned long long win[64];
@@ -400,6 +401,20 @@ __global__ __launch_bounds__(SEL_THREADS) void k_topk_merge(
     __shared__ int pg[64];
     const int c = blockIdx.x;
     const int tid = threadIdx.x;
+    if (rc.dst && (int64_t)cnt[c] > cap) {
+        // the buffer overflowed and the last hop wrote no slab: recompute
+        // this column (warp per row, lanes over the row's in-edges)
+        const int lane = tid & 31;
+        for (int64_t j = tid >> 5; j < n; j += SEL_THREADS / 32) {
+            float acc = 0.f;
+            for (int64_t e = rc.in_ptr[j] + lane; e < rc.in_ptr[j + 1]; e += 32)
+                acc = fmaf(rc.in_w[e], rc.prev[(int64_t)rc.in_src[e] * bp + c], acc);
+            for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+            if (lane == 0) rc.dst[j * bp + c] = fmaf(rc.alpha, acc, rc.u[j * bp + c]);
+        }
+        __threadfence_block();
+        __syncthreads();
+    }
     double z = 0.0;
     for (int64_t t = tid; t < n_ztiles; t += SEL_THREADS) z += (double)zpart[t * bp + c];
     for (int o = 16; o > 0; o >>= 1) z += __shfl_xor_sync(0xffffffffu, z, o);
@@ -591,19 +606,21 @@ cudaError_t launch_select(const SelectPlan &sp, const float *s, int b, unsigned 
     cudaError_t e = bound_and_filter<false>(sp, s, b, ext_of, (int64_t)1 << 40, ws, st, launches);
     if (e != cudaSuccess) return e;
     return launch_topk_merge(sp, s, b, ws, zpart, n_ztiles, ext_of, row_of, page_row, ids, scores,
-                             page_ids, n_pages, status, st, launches);
+                             page_ids, n_pages, status, nullptr, st, launches);
 }
 
 cudaError_t launch_topk_merge(const SelectPlan &sp, const float *s, int b,
                               const unsigned long long *ws, const float *zpart, int64_t n_ztiles,
                               const int32_t *ext_of, const int32_t *row_of,
                               const int32_t *page_row, int64_t *ids, float *scores,
-                              int32_t *page_ids, int32_t *n_pages, int *status, cudaStream_t st,
-                              int *launches) {
+                              int32_t *page_ids, int32_t *n_pages, int *status,
+                              const ColumnRecompute *rc, cudaStream_t st, int *launches) {
+    const ColumnRecompute r = rc ? *rc : ColumnRecompute{nullptr, nullptr, nullptr, nullptr,
+                                                          nullptr, 0.f, nullptr};
     k_topk_merge<<<b, SEL_THREADS, 0, st>>>(s, sp.n, sp.bp, sp.k, ext_of,
                                             (const unsigned int *)(ws + sp.off_cnt),
                                             ws + sp.off_buf, sp.cap, zpart, n_ztiles, row_of,
-                                            page_row, ids, scores, page_ids, n_pages, status);
+                                            page_row, ids, scores, page_ids, n_pages, status, r);
     if (launches) *launches += 1;
     return cudaGetLastError();
 }
