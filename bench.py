@@ -59,16 +59,17 @@ def algorithmic_bytes(n, d, b, nnz, hops, k):
 
 
 def hop_bytes(n, b, nnz):
-    """One propagation hop: graph once + input slab read once + output slab written once."""
+    """One propagation hop: graph once + two slab passes (hop 1 reads u and
+    writes s1; the last hop reads s^(H-1) and u and writes nothing)."""
     return (n + 1) * 8 + nnz * 8 + 2 * n * b * 4
 
 
-# DRAM bytes per propagation hop on this workload (sum over the hop's three
-# kernels: hub segments, rows kept whole, hub fixup), from an ncu capture of
+# DRAM bytes per propagation hop on this workload (sum over the hop's two
+# kernels: hub segments, then hub sums + rows kept whole), from an ncu capture of
 # `bench.py --steps 2 --warmup 1 --no-cpu-baseline` with the
 # dram__bytes_read/write counters (mean of the two hops).  Set to None when
 # the hop kernels change until they are captured again.
-HOP_DRAM_BYTES = 11.5e9
+HOP_DRAM_BYTES = 10.85e9
 
 
 def score_bytes(n, d, b):
@@ -460,7 +461,7 @@ def main():
     if dom == "propagate":
         per_launch_bytes = hop_bytes(wl.n, 256, wl.nnz)
         units = args.steps * wl.hops
-        what = "propagation hop (graph once + input slab read once + output slab written once)"
+        what = "propagation hop (graph once + two slab passes)"
     elif dom == "score":
         per_launch_bytes = score_bytes(wl.n, wl.dim, 256)
         units = args.steps
