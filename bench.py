@@ -35,6 +35,9 @@ METRIC = "retrieve queries/sec at N=1M chunks, d=1024, B=256; % of roofline"
 WORKLOAD = ("gmm1m: N=1048576 chunks, d=1024 bf16, 4096-component Zipf(1.1) mixture, 32-neighbour "
             "power-law relation graph (nnz 33554432), B=256 queries, hops=2, alpha=0.5, k=32, "
             "64 chunks/page, clustered placement")
+DENSE_METRIC = "Dense-only retrieve queries/sec at N=1M chunks, d=1024, B=256, top-p 5, no hops"
+DENSE_WORKLOAD = ("gmm1m store (N=1048576, d=1024 bf16), B=256 queries, k=5, hops=0 "
+                  "(embedding similarity only), 64 chunks/page, clustered placement")
 
 
 def peaks():
@@ -127,16 +130,18 @@ class Clocks:
                 "samples": len(sm)}
 
 
-def cpu_baseline(wl, placement, n_queries, rng_seed=0, weights=None):
+def cpu_baseline(wl, placement, n_queries, rng_seed=0, weights=None, k=None, hops=None):
     """The oracle retrieving n_queries of the batch against the full store on
     one host thread (the relation weights, which the GPU store computes at
     append time, are computed once beforehand)."""
     import oracle
-    w = weights if weights is not None else oracle.row_softmax(wl.row_ptr, wl.aff)
+    hops = wl.hops if hops is None else hops
+    w = (weights if weights is not None else oracle.row_softmax(wl.row_ptr, wl.aff)) if hops else None
     rows = np.random.default_rng(rng_seed).choice(wl.n_queries, size=n_queries, replace=False)
     t0 = time.perf_counter()
-    oracle.retrieve(wl.emb, wl.queries[rows], wl.row_ptr, wl.col, w, tau=wl.tau, alpha=wl.alpha,
-                    hops=wl.hops, k=wl.k, page_of=wl.page_of[placement])
+    oracle.retrieve(wl.emb, wl.queries[rows], wl.row_ptr if hops else None,
+                    wl.col if hops else None, w, tau=wl.tau, alpha=wl.alpha, hops=hops,
+                    k=wl.k if k is None else k, page_of=wl.page_of[placement])
     dt = time.perf_counter() - t0
     return dict(value=n_queries / dt, unit="queries/s", cores=1, kind="oracle",
                 sample=f"{n_queries} of the {wl.n_queries} queries against the full store, "
@@ -342,19 +347,28 @@ def main():
     ap.add_argument("--placement", default="clustered")
     ap.add_argument("--scale", type=float, default=1.0,
                     help="shrink N (profiling captures of a smaller case); 1.0 = the benchmark")
-    ap.add_argument("--workload", default="retrieve", choices=["retrieve", "update", "streams"],
+    ap.add_argument("--workload", default="retrieve",
+                    choices=["retrieve", "update", "streams", "dense"],
                     help="retrieve: the benchmark; update: relation update of 4096 new chunks "
-                         "on the 1M-chunk store; streams: 4M-chunk store, 8 streams x 128 queries")
+                         "on the 1M-chunk store; streams: 4M-chunk store, 8 streams x 128 "
+                         "queries; dense: the Dense-only form (k=5, no hops) on the 1M store")
     args = ap.parse_args()
     if args.steps is None:
-        args.steps = {"retrieve": 100, "update": 5, "streams": 20}[args.workload]
+        args.steps = {"retrieve": 100, "update": 5, "streams": 20, "dense": 100}[args.workload]
     if args.impl == "reference":
         return run_reference(args)
     if args.workload == "update":
         return run_update(args)
     if args.workload == "streams":
         return run_streams(args)
+    if args.workload == "dense":
+        return run_retrieve(args, k=5, hops=0, metric=DENSE_METRIC, workload=DENSE_WORKLOAD)
+    return run_retrieve(args)
 
+
+def run_retrieve(args, k=None, hops=None, metric=METRIC, workload=WORKLOAD):
+    """The retrieval pass on the gmm1m store (k / hops override the
+    configuration: the Dense-only form uses k = 5, hops = 0)."""
     import torch
     ws, rank, local = dist_env()
     if ws > 1:
@@ -374,12 +388,14 @@ def main():
     t_gen = time.perf_counter() - t_gen
     cpu = None
     if rank == 0 and not args.no_cpu_baseline and ws == 1:
-        cpu = cpu_baseline(wl, args.placement, args.cpu_queries)
+        cpu = cpu_baseline(wl, args.placement, args.cpu_queries, k=k, hops=hops)
 
     store = MemStore.from_arrays(wl.emb, wl.page_of[args.placement], wl.row_ptr, wl.col, wl.aff,
                                  capacity=wl.n, chunks_per_page=wl.chunks_per_page,
                                  temperature=wl.tau, device=dev)
-    B, k = wl.n_queries, wl.k
+    B = wl.n_queries
+    k = wl.k if k is None else k
+    hops = wl.hops if hops is None else hops
     st = torch.cuda.Stream(device=dev)
     q_dev = torch.from_numpy(wl.queries.view(np.int16)).to(f"cuda:{dev}")
     ids = torch.empty((B, k), dtype=torch.int64, device=f"cuda:{dev}")
@@ -388,7 +404,7 @@ def main():
     npages = torch.empty((B,), dtype=torch.int32, device=f"cuda:{dev}")
 
     def step():
-        store.retrieve(q_dev, k, wl.alpha, wl.hops, ids, scores, pages, npages, stream=st)
+        store.retrieve(q_dev, k, wl.alpha, hops, ids, scores, pages, npages, stream=st)
 
     def barrier():
         torch.cuda.synchronize(dev)
@@ -451,7 +467,7 @@ def main():
     ms, ms_e2e = max_over_ranks([ms, ms_e2e], device=f"cuda:{dev}" if ws > 1 else None)
 
     hbm, bf16, peak_kind = peaks()
-    ab = algorithmic_bytes(wl.n, wl.dim, B, wl.nnz, wl.hops, k)
+    ab = algorithmic_bytes(wl.n, wl.dim, B, wl.nnz, hops, k)
     total_ab = sum(ab.values())
     per_step_ms = ms / args.steps
     # dominant phase
@@ -460,7 +476,7 @@ def main():
     dom_ms, dom_launches = phases[dom]
     if dom == "propagate":
         per_launch_bytes = hop_bytes(wl.n, 256, wl.nnz)
-        units = args.steps * wl.hops
+        units = args.steps * hops
         what = "propagation hop (graph once + two slab passes)"
     elif dom == "score":
         per_launch_bytes = score_bytes(wl.n, wl.dim, 256)
@@ -473,7 +489,7 @@ def main():
     dom_avg_ms = dom_ms / units
     achieved = per_launch_bytes / (dom_avg_ms * 1e-3) / 1e9
     line = {
-        "metric": METRIC,
+        "metric": metric,
         "value": job_throughput(B * args.steps, ws, ms),
         "unit": "queries/s",
         "n_gpus": ws,
@@ -485,7 +501,7 @@ def main():
         "vs_baseline": None,
         "dtype": "f32",
         "data": "synthetic",
-        "config": {"workload": WORKLOAD if args.scale == 1.0 else f"{WORKLOAD} scaled by {args.scale}",
+        "config": {"workload": workload if args.scale == 1.0 else f"{workload} scaled by {args.scale}",
                    "l2": "inputs larger than L2 (E 2.1 GB, score slabs 1.07 GB "
                    "each), no flush", "placement": args.placement,
                    "parallelism": "replicas" if ws > 1 else "single GPU"},

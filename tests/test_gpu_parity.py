@@ -237,7 +237,7 @@ def _pages_after_appends(wl, batches):
     return np.concatenate(pages).astype(np.int32)
 
 
-def _retrieval_on_store(wl, store, batches):
+def _retrieval_on_store(wl, store, batches, k=None, hops=None):
     """Retrieval through the store after updates vs the oracle on the graph
     the store exports (the transpose used by propagation is checked by it)."""
     import dataclasses
@@ -246,8 +246,8 @@ def _retrieval_on_store(wl, store, batches):
     wl2 = dataclasses.replace(wl, emb=np.concatenate([wl.emb, wl.new_emb[:n_new]]), row_ptr=rp,
                               col=col, aff=aff,
                               page_of={"clustered": _pages_after_appends(wl, batches)})
-    _, got = gpu_retrieve(wl2, "clustered", store=store)
-    ref = oracle_retrieve(wl2, "clustered")
+    _, got = gpu_retrieve(wl2, "clustered", store=store, k=k, hops=hops)
+    ref = oracle_retrieve(wl2, "clustered", k=k, hops=hops)
     assert_retrieval_parity(wl2, "clustered", got, ref)
 
 
@@ -257,6 +257,15 @@ def test_retrieval_after_update():
     wl = synth.workload(3, scale=1 / 64)
     store = check_update(wl)
     _retrieval_on_store(wl, store, [wl.new_emb.shape[0]])
+
+
+def test_dense_only_top5():
+    """The Dense-only form with the paper's top-p = 5: relation update with
+    M = 5 (whole CSR against the oracle), then retrieval with k = 5 and no
+    propagation on the updated store."""
+    wl = synth.workload(3, scale=1 / 64)
+    store = check_update(wl, M=5)
+    _retrieval_on_store(wl, store, [wl.new_emb.shape[0]], k=5, hops=0)
 
 
 def test_retrieval_after_two_updates():
