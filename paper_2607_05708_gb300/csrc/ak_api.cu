@@ -81,6 +81,7 @@ struct DevBuf {
 
 struct StreamScratch {
     DevBuf qp, shift, u, sa, sb, zpart, partial, cand, counters;
+    DevBuf samp, ext_s, zsamp;   // retrieval without hops: the score's row sample
 };
 
 struct ProfRec {
@@ -717,19 +718,58 @@ akashic_status_t akashic_mem_retrieve(akashic_mem_t *m, const uint16_t *q, int32
         if (eff_hops >= 1 && m->n_segs > 0) AK_TRY(sc->partial.ensure((size_t)m->n_segs * bp * 4));
         if (eff_hops >= 1) AK_TRY(sc->counters.ensure(64));
         const uint16_t *qb = q + (int64_t)off * m->dim;
+        // Without hops the top-k filter is fused into the score GEMM, which
+        // then writes no slab: the bound comes from the score of every
+        // stride-th row, computed first by the same kernel (same values).
+        const SelectPlan sp2 = select_plan(sp.n_sample, bp, k, sms, 1);
+        const bool dense_fused = eff_hops == 0 && m->fuse_filter && sp2.off_tr == sp.off_tr &&
+                                 sp2.words <= sp.words;
+        unsigned long long *ws = sc->cand.as<unsigned long long>();
+        ColumnRecompute rc{};
         {
             PhaseScope ph(m, AKASHIC_PHASE_SCORE, st);
             CUDA_TRY(launch_prep_queries(qb, b, bp, m->dim, m->tau, m->max_norm.as<float>(),
                                          sc->qp.as<uint16_t>(), sc->shift.as<float>(),
                                          m->status.as<int>(), st));
-            CUDA_TRY(launch_score(m->emb.as<uint16_t>(), n, m->dim, sc->qp.as<uint16_t>(), bp,
-                                  sc->shift.as<float>(), m->tau, sc->u.as<float>(),
-                                  sc->zpart.as<float>(), m->status.as<int>(), st, &ph.launches,
-                                  &zrows));
             ph.launches += 1;
+            if (!dense_fused)
+                CUDA_TRY(launch_score(m->emb.as<uint16_t>(), n, m->dim, sc->qp.as<uint16_t>(), bp,
+                                      sc->shift.as<float>(), m->tau, sc->u.as<float>(),
+                                      sc->zpart.as<float>(), m->status.as<int>(), st,
+                                      &ph.launches, &zrows));
+        }
+        if (dense_fused) {
+            {
+                PhaseScope ps(m, AKASHIC_PHASE_SELECT, st);
+                AK_TRY(sc->samp.ensure((size_t)sp.n_sample * bp * 4));
+                AK_TRY(sc->ext_s.ensure((size_t)sp.n_sample * 4));
+                AK_TRY(sc->zsamp.ensure((size_t)score_tiles(sp.n_sample) * bp * 4));
+                CUDA_TRY(launch_ext_sample(m->ext_of.as<int32_t>(), sp.n_sample, sp.stride,
+                                           sc->ext_s.as<int32_t>(), st));
+                CUDA_TRY(launch_score_sample(m->emb.as<uint16_t>(), sp.n_sample, sp.stride, m->dim,
+                                             sc->qp.as<uint16_t>(), bp, sc->shift.as<float>(),
+                                             m->tau, sc->samp.as<float>(), sc->zsamp.as<float>(),
+                                             m->status.as<int>(), st, &ps.launches));
+                CUDA_TRY(launch_sample_bound(sp2, sc->samp.as<float>(), b, sc->ext_s.as<int32_t>(),
+                                             ws, st, &ps.launches, 4u));
+                ps.launches += 1;
+            }
+            PhaseScope ph(m, AKASHIC_PHASE_SCORE, st);
+            CUDA_TRY(launch_score_filter(m->emb.as<uint16_t>(), n, m->dim, sc->qp.as<uint16_t>(),
+                                         bp, b, sc->shift.as<float>(), m->tau,
+                                         sc->zpart.as<float>(), m->ext_of.as<int32_t>(),
+                                         ws + sp.off_bound, (unsigned int *)(ws + sp.off_cnt),
+                                         ws + sp.off_buf, sp.cap, m->status.as<int>(), st,
+                                         &ph.launches, &zrows));
+            rc.kind = 2;
+            rc.emb = m->emb.as<uint16_t>();
+            rc.qp = sc->qp.as<uint16_t>();
+            rc.dim = m->dim;
+            rc.tau = m->tau;
+            rc.shift = sc->shift.as<float>();
+            rc.dst = sc->u.as<float>();
         }
         const float *fin = sc->u.as<float>();
-        ColumnRecompute rc{};
         if (eff_hops >= 1) {
             HopPlan hp;
             hp.split = m->split;
@@ -746,9 +786,11 @@ akashic_status_t akashic_mem_retrieve(akashic_mem_t *m, const uint16_t *q, int32
             hp.seg_slot = m->seg_slot.as<int32_t>();
             hp.split_order = m->split_order.as<int32_t>();
             float *bufs[2] = {sc->sa.as<float>(), sc->sb.as<float>()};
-            unsigned long long *ws = sc->cand.as<unsigned long long>();
-            rc = ColumnRecompute{sc->u.as<float>(), nullptr, hp.in_ptr, hp.in_src, hp.in_w, alpha,
-                                 nullptr};
+            rc.u = sc->u.as<float>();
+            rc.in_ptr = hp.in_ptr;
+            rc.in_src = hp.in_src;
+            rc.in_w = hp.in_w;
+            rc.alpha = alpha;
             for (int h = 0; h < eff_hops; ++h) {
                 float *out = bufs[h & 1];
                 const bool last = m->fuse_filter && h == eff_hops - 1;
@@ -769,6 +811,7 @@ akashic_status_t akashic_mem_retrieve(akashic_mem_t *m, const uint16_t *q, int32
                                     sc->partial.as<float>(), sc->counters.as<int>(),
                                     last ? &flt : nullptr, st, &ph.launches));
                 if (last) {
+                    rc.kind = 1;
                     rc.prev = fin;
                     rc.dst = out;
                 }
@@ -779,7 +822,7 @@ akashic_status_t akashic_mem_retrieve(akashic_mem_t *m, const uint16_t *q, int32
             PhaseScope ph(m, AKASHIC_PHASE_SELECT, st);
             int32_t *pids = page_ids ? page_ids + (int64_t)off * k : nullptr;
             int32_t *npg = n_pages ? n_pages + off : nullptr;
-            if (eff_hops >= 1 && m->fuse_filter)
+            if ((eff_hops >= 1 && m->fuse_filter) || dense_fused)
                 CUDA_TRY(launch_topk_merge(sp, fin, b, sc->cand.as<unsigned long long>(),
                                            sc->zpart.as<float>(), zrows, m->ext_of.as<int32_t>(),
                                            m->row_of.as<int32_t>(), m->page_of.as<int32_t>(),

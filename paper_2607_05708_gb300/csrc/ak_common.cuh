@@ -63,6 +63,25 @@ cudaError_t launch_score(const uint16_t *emb, int64_t n, int dim, const uint16_t
                          const float *shift, float tau, float *u, float *zpart, int *status,
                          cudaStream_t st, int *launches, int *zrows);
 
+// The score on every stride-th row only: out[v, c] = u[v*stride, c] for
+// v < n_sample (same kernel and arithmetic as launch_score, so the values
+// are those the full pass computes); zpart receives partial sums of the
+// sample (scratch, one row per CTA, at most score_tiles(n_sample) rows).
+cudaError_t launch_score_sample(const uint16_t *emb, int64_t n_sample, int64_t stride, int dim,
+                                const uint16_t *qp, int bp, const float *shift, float tau,
+                                float *out, float *zpart, int *status, cudaStream_t st,
+                                int *launches);
+// Score with the top-k filter fused and no slab written: zpart as in
+// launch_score; the key (u bits, chunk ID ext_of[j]) of every (j, c) with
+// c < n_cols that is >= bound[c] is appended to buf[c][...] (count cnt[c],
+// capacity cap).
+cudaError_t launch_score_filter(const uint16_t *emb, int64_t n, int dim, const uint16_t *qp,
+                                int bp, int64_t n_cols, const float *shift, float tau,
+                                float *zpart, const int32_t *ext_of,
+                                const unsigned long long *bound, unsigned int *cnt,
+                                unsigned long long *buf, int64_t cap, int *status,
+                                cudaStream_t st, int *launches, int *zrows);
+
 // Plain dot products out[j, c] = <e_{j*row_stride}, q_c> (bf16 tensor
 // cores, fp32 accumulate) for j < n, row stride bp in out.
 cudaError_t launch_dots(const uint16_t *emb, int64_t n, int64_t row_stride_rows, int dim,
@@ -262,21 +281,33 @@ cudaError_t launch_select_signed(const SelectPlan &sp, const float *s, int b,
 // Bound pass alone over signed values: bound[c] for the b real columns
 // (the k-th largest sampled key; padding columns get an all-ones bound).
 // Bound only, unsigned keys (retrieval): ws + sp.off_bound gets the bound,
-// the column counts are cleared.  For a filter fused into the last hop.
+// the column counts are cleared.  For a filter fused into the last hop or
+// into the score.  `slack` lowers each bound by that many units of the
+// score's last place (margin for a sample computed by another launch).
 cudaError_t launch_sample_bound(const SelectPlan &sp, const float *s, int b,
                                 const int32_t *ext_of, unsigned long long *ws, cudaStream_t st,
-                                int *launches);
+                                int *launches, uint32_t slack = 0);
 // A column of the last hop recomputed by the merge when the filter fused
 // into that hop (which writes no output slab) overflowed its buffer:
 // dst[j,c] = u[j,c] + alpha * sum_{e in in(j)} in_w[e] * prev[in_src[e],c].
+// Without hops (the score itself, fused with the filter, wrote no slab):
+// dst[j,c] = exp(tau <e_j, q_c> - shift[c]) from the stored bf16 values.
 struct ColumnRecompute {
+    int kind;     // 0 none, 1 last hop, 2 score
     const float *u, *prev;
     const int64_t *in_ptr;
     const int32_t *in_src;
     const float *in_w;
     float alpha;
+    const uint16_t *emb, *qp;   // kind 2: E [n][dim], padded queries [bp][dim]
+    int dim;
+    float tau;
+    const float *shift;
     float *dst;   // [n][bp]; the merge reads the overflowed column from here
 };
+// Row j -> chunk ID of a strided sample: out[v] = ext_of[v * stride].
+cudaError_t launch_ext_sample(const int32_t *ext_of, int64_t n_sample, int64_t stride,
+                              int32_t *out, cudaStream_t st);
 // Merge only: the k winners per column from the buffers filled by a filter
 // pass (falls back to the column of `s` where a buffer overflowed, after
 // recomputing it into s when `rc` is given; then s must be rc->dst).

@@ -122,7 +122,11 @@ cudaError_t make_tmap_2d(CUtensorMap *map, const void *base, CUtensorMapDataType
 //     GEMM_FILTER  no store: every dot whose selection key clears its
 //                  column's bound is appended to that column's buffer (the
 //                  fused relation top-M)
-enum GemmMode { GEMM_EXP = 0, GEMM_RAW = 1, GEMM_FILTER = 2 };
+//     GEMM_EXP_FILTER  the score step with the top-k filter fused and no
+//                  store: exp, column sums toward Z, and every value whose
+//                  key clears its query's bound appended to that query's
+//                  buffer (retrieval without hops)
+enum GemmMode { GEMM_EXP = 0, GEMM_RAW = 1, GEMM_FILTER = 2, GEMM_EXP_FILTER = 3 };
 
 struct GemmEpi {
     const float *shift;                 // EXP: [BP]
@@ -148,7 +152,8 @@ struct GemmCfg {
     // the filter epilogue stores nothing: its region only holds the tile's
     // column bounds, and the freed space goes to pipeline stages
     static constexpr int OUT_REGION = MODE == GEMM_FILTER ? (BP * 12 < 1024 ? 1024 : BP * 12)
-                                                          : 2 * OUT_BYTES;
+                                      : MODE == GEMM_EXP_FILTER ? 2 * OUT_BYTES + BP * 12
+                                                                : 2 * OUT_BYTES;
     static constexpr int MISC = 4096;   // shift, Z sums, flags, barriers
     static constexpr int BUDGET = 227 * 1024 - 1024;
     static constexpr int S_FIT = (BUDGET - OUT_REGION - MISC) / STAGE_BYTES;
@@ -172,7 +177,8 @@ __global__ __launch_bounds__(GemmCfg<BP, MODE>::THREADS, 1) void k_gemm_umma(con
                                                       int64_t n_rows, int dim, int n_ctiles,
                                                       const GemmEpi ep) {
     using C = GemmCfg<BP, MODE>;
-    constexpr bool EXP = MODE == GEMM_EXP;
+    constexpr bool EXPF = MODE == GEMM_EXP_FILTER;
+    constexpr bool EXP = MODE == GEMM_EXP || EXPF;
     constexpr bool FILTER = MODE == GEMM_FILTER;
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = (uint8_t *)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
@@ -188,8 +194,9 @@ __global__ __launch_bounds__(GemmCfg<BP, MODE>::THREADS, 1) void k_gemm_umma(con
     uint64_t *full = bars, *empty = bars + C::STAGES;
     uint64_t *tfull = bars + 2 * C::STAGES, *tempty = tfull + 2;
     uint32_t *tmem_slot = (uint32_t *)(tempty + 2);
-    unsigned long long *bnd_s = (unsigned long long *)sOut;   // FILTER: the tile's column bounds
-    float *thr_s = (float *)(bnd_s + BP);   // FILTER: the bounds as float thresholds
+    // filters: the tile's column bounds and the same as float thresholds
+    unsigned long long *bnd_s = (unsigned long long *)(sOut + (EXPF ? 2 * C::OUT_BYTES / 4 : 0));
+    float *thr_s = (float *)(bnd_s + BP);
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int64_t m_tiles = (n_rows + C::BM - 1) / C::BM;
@@ -301,16 +308,19 @@ __global__ __launch_bounds__(GemmCfg<BP, MODE>::THREADS, 1) void k_gemm_umma(con
             const uint32_t aph = (uint32_t)(it >> 1) & 1u;
             // one thread polls, the barrier makes the outcome uniform
             if (et == 0) *go = mbar_wait(&tfull[acc], aph, status) ? 1 : 0;
-            if (FILTER) {
+            if (FILTER || EXPF) {
                 // threshold T with: v < T => key < bound; v > T => key > bound
-                // (keys order values like floats, -0 below +0); a bound of 0
-                // admits everything (-inf), the padding bound ~0 nothing (NaN)
+                // (signed keys order values like floats, -0 below +0; the
+                // exp values are >= 0 and their keys are the plain bits); a
+                // bound of 0 admits everything, the padding bound ~0 nothing
+                // (a NaN threshold)
                 for (int c = et; c < BP; c += C::EPI_T) {
                     const int64_t cg = ct * BP + c;
                     const unsigned long long bk = cg < ep.n_cols ? ep.bound[cg] : ~0ull;
                     const uint32_t hi = (uint32_t)(bk >> 32);
                     bnd_s[c] = bk;
-                    thr_s[c] = hi == 0u ? -INFINITY : unordered_bits(hi);
+                    if (FILTER) thr_s[c] = hi == 0u ? -INFINITY : unordered_bits(hi);
+                    else thr_s[c] = __uint_as_float(hi);
                 }
             }
             named_bar(1, C::EPI_T);
@@ -320,7 +330,7 @@ __global__ __launch_bounds__(GemmCfg<BP, MODE>::THREADS, 1) void k_gemm_umma(con
             const bool valid = grow < n_rows;
             uint32_t fid = 0;
             bool fok = false;
-            if (FILTER && valid) {
+            if ((FILTER || EXPF) && valid) {
                 const int32_t id = ep.ext_of[grow];
                 fok = (int64_t)id < ep.id_limit;
                 fid = ~(uint32_t)id;
@@ -333,25 +343,28 @@ __global__ __launch_bounds__(GemmCfg<BP, MODE>::THREADS, 1) void k_gemm_umma(con
                 tmem_ld_wait();
                 if constexpr (FILTER) {
                     if (fok) {
-                        // one float compare per dot; the exact key test only
-                        // for the few at or above the threshold
+                        // one float compare per dot, branch-free, into a mask;
+                        // the exact key test only for the few flagged
                         const float4 *t4 = (const float4 *)(thr_s + ch * 32);
+                        uint32_t pass = 0u;
 #pragma unroll
                         for (int i4 = 0; i4 < 8; ++i4) {
                             const float4 t = t4[i4];
-                            const float tv[4] = {t.x, t.y, t.z, t.w};
+                            pass |= (__uint_as_float(r[4 * i4]) >= t.x ? 1u : 0u) << (4 * i4);
+                            pass |= (__uint_as_float(r[4 * i4 + 1]) >= t.y ? 1u : 0u) << (4 * i4 + 1);
+                            pass |= (__uint_as_float(r[4 * i4 + 2]) >= t.z ? 1u : 0u) << (4 * i4 + 2);
+                            pass |= (__uint_as_float(r[4 * i4 + 3]) >= t.w ? 1u : 0u) << (4 * i4 + 3);
+                        }
+                        if (pass) {
 #pragma unroll
-                            for (int e = 0; e < 4; ++e) {
-                                const int i = i4 * 4 + e;
-                                const float v = __uint_as_float(r[i]);
-                                if (v >= tv[e]) {
-                                    const unsigned long long key =
-                                        ((unsigned long long)ordered_bits(v) << 32) | fid;
-                                    if (key >= bnd_s[ch * 32 + i]) {
-                                        const int64_t cg = ct * BP + ch * 32 + i;
-                                        const unsigned int p = atomicAdd(&ep.cnt[cg], 1u);
-                                        if ((int64_t)p < ep.cap) ep.buf[cg * ep.cap + p] = key;
-                                    }
+                            for (int i = 0; i < 32; ++i) {
+                                if (!((pass >> i) & 1u)) continue;
+                                const unsigned long long key =
+                                    ((unsigned long long)ordered_bits(__uint_as_float(r[i])) << 32) | fid;
+                                if (key >= bnd_s[ch * 32 + i]) {
+                                    const int64_t cg = ct * BP + ch * 32 + i;
+                                    const unsigned int p = atomicAdd(&ep.cnt[cg], 1u);
+                                    if ((int64_t)p < ep.cap) ep.buf[cg * ep.cap + p] = key;
                                 }
                             }
                         }
@@ -362,6 +375,22 @@ __global__ __launch_bounds__(GemmCfg<BP, MODE>::THREADS, 1) void k_gemm_umma(con
                 for (int i = 0; i < 32; ++i) {
                     const float x = __uint_as_float(r[i]);
                     v[i] = valid ? (EXP ? expf(ep.tau * x - shift_s[ch * 32 + i]) : x) : 0.f;
+                }
+                // filter, first half: which of this row's 32 values reach
+                // their query's threshold (branch-free; rarely any)
+                uint32_t pass = 0u;
+                if constexpr (EXPF) {
+                    if (fok) {
+                        const float4 *t4 = (const float4 *)(thr_s + ch * 32);
+#pragma unroll
+                        for (int i4 = 0; i4 < 8; ++i4) {
+                            const float4 t = t4[i4];
+                            pass |= (v[4 * i4] >= t.x ? 1u : 0u) << (4 * i4);
+                            pass |= (v[4 * i4 + 1] >= t.y ? 1u : 0u) << (4 * i4 + 1);
+                            pass |= (v[4 * i4 + 2] >= t.z ? 1u : 0u) << (4 * i4 + 2);
+                            pass |= (v[4 * i4 + 3] >= t.w ? 1u : 0u) << (4 * i4 + 3);
+                        }
+                    }
                 }
                 named_bar(1, C::EPI_T);                       // staging[buf] free again
                 float4 *dst = (float4 *)(sOut + buf * (C::OUT_BYTES / 4) + row * 32);
@@ -379,7 +408,24 @@ __global__ __launch_bounds__(GemmCfg<BP, MODE>::THREADS, 1) void k_gemm_umma(con
                         s += so[rr * 32 + ((((c >> 2) ^ (rr & 7))) << 2) + (c & 3)];
                     zq[g * 32 + c] = s;
                 }
-                if (et == 0) {
+                if constexpr (EXPF) {
+                    // second half: the exact key test and append for the
+                    // flagged values, read back from the staged row
+                    const float *so = sOut + buf * (C::OUT_BYTES / 4) + row * 32;
+                    while (pass) {
+                        const int i = __ffs(pass) - 1;
+                        pass &= pass - 1u;
+                        const float x = so[(((i >> 2) ^ (row & 7)) << 2) + (i & 3)];
+                        const unsigned long long key =
+                            ((unsigned long long)__float_as_uint(x) << 32) | fid;
+                        if (key >= bnd_s[ch * 32 + i]) {
+                            const int64_t cg = ct * BP + ch * 32 + i;
+                            const unsigned int p = atomicAdd(&ep.cnt[cg], 1u);
+                            if ((int64_t)p < ep.cap) ep.buf[cg * ep.cap + p] = key;
+                        }
+                    }
+                }
+                if (!EXPF && et == 0) {
                     tma_store_2d(&tmC, sOut + buf * (C::OUT_BYTES / 4), (int)(ct * BP + ch * 32),
                                  (int)(mt * C::BM));
                     bulk_commit();
@@ -388,14 +434,14 @@ __global__ __launch_bounds__(GemmCfg<BP, MODE>::THREADS, 1) void k_gemm_umma(con
                     named_bar(1, C::EPI_T);
                     if (et < 32) zacc[ch * 32 + et] += (zq[et] + zq[32 + et]) + (zq[64 + et] + zq[96 + et]);
                 }
-                if (et == 0) bulk_wait_read<1>();
+                if (!EXPF && et == 0) bulk_wait_read<1>();
                 }
             }
             tc_fence_before();
             named_bar(1, C::EPI_T);
             if (et == 0) mbar_arrive(&tempty[acc]);
         }
-        if (et == 0) bulk_wait_all();
+        if (!EXPF && et == 0) bulk_wait_all();
         named_bar(1, C::EPI_T);
         if (EXP && ep.zpart)
             for (int c = et; c < BP; c += 128) ep.zpart[(int64_t)blockIdx.x * BP + c] = zacc[c];
@@ -430,7 +476,7 @@ static cudaError_t gemm_bp(const uint16_t *emb, int64_t n_rows, int64_t row_stri
     if (e == cudaSuccess)
         e = make_tmap_2d(&tb, qp, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, (uint64_t)dim,
                          (uint64_t)n_ctiles * BP, (uint64_t)dim * 2, 64, BP);
-    if (e == cudaSuccess && MODE != GEMM_FILTER)
+    if (e == cudaSuccess && MODE != GEMM_FILTER && MODE != GEMM_EXP_FILTER)
         e = make_tmap_2d(&tc, out, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, (uint64_t)n_ctiles * BP,
                          (uint64_t)n_rows, (uint64_t)n_ctiles * BP * 4, 32, 128);
     else
@@ -466,6 +512,45 @@ cudaError_t launch_score(const uint16_t *emb, int64_t n, int dim, const uint16_t
     ep.zpart = zpart;
     ep.status = status;
     cudaError_t e = gemm_dispatch<GEMM_EXP>(emb, n, 1, dim, qp, bp, 1, u, ep, st, zrows);
+    if (launches) *launches += 1;
+    return e;
+}
+
+cudaError_t launch_score_sample(const uint16_t *emb, int64_t n_sample, int64_t stride, int dim,
+                                const uint16_t *qp, int bp, const float *shift, float tau,
+                                float *out, float *zpart, int *status, cudaStream_t st,
+                                int *launches) {
+    GemmEpi ep{};
+    ep.shift = shift;
+    ep.tau = tau;
+    ep.zpart = zpart;
+    ep.status = status;
+    cudaError_t e = gemm_dispatch<GEMM_EXP>(emb, n_sample, stride, dim, qp, bp, 1, out, ep, st,
+                                            nullptr);
+    if (launches) *launches += 1;
+    return e;
+}
+
+cudaError_t launch_score_filter(const uint16_t *emb, int64_t n, int dim, const uint16_t *qp,
+                                int bp, int64_t n_cols, const float *shift, float tau,
+                                float *zpart, const int32_t *ext_of,
+                                const unsigned long long *bound, unsigned int *cnt,
+                                unsigned long long *buf, int64_t cap, int *status,
+                                cudaStream_t st, int *launches, int *zrows) {
+    GemmEpi ep{};
+    ep.shift = shift;
+    ep.tau = tau;
+    ep.zpart = zpart;
+    ep.status = status;
+    ep.n_cols = n_cols;
+    ep.ext_of = ext_of;
+    ep.id_limit = (int64_t)1 << 40;
+    ep.bound = bound;
+    ep.cnt = cnt;
+    ep.buf = buf;
+    ep.cap = cap;
+    cudaError_t e = gemm_dispatch<GEMM_EXP_FILTER>(emb, n, 1, dim, qp, bp, 1, nullptr, ep, st,
+                                                   zrows);
     if (launches) *launches += 1;
     return e;
 }

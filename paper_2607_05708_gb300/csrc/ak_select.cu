@@ -173,7 +173,7 @@ constexpr int KTH_REP = (SEL_THREADS / 32) * 4;   // histogram replicas
 constexpr int KTH_CBUF = 4096;                    // keys kept after the first digit
 
 __global__ __launch_bounds__(SEL_THREADS) void k_sample_kth(
-    const uint32_t *__restrict__ keysT, int64_t n_sample, int b, int k,
+    const uint32_t *__restrict__ keysT, int64_t n_sample, int b, int k, uint32_t slack,
     unsigned long long *__restrict__ bound, unsigned int *__restrict__ cnt) {
     extern __shared__ uint32_t kst[];                 // [n_sample] when staged
     __shared__ int hist[KTH_REP * 256];
@@ -279,7 +279,8 @@ __global__ __launch_bounds__(SEL_THREADS) void k_sample_kth(
         // fewer than k keys: no thread ever matched and the prefix has not
         // reached a key, so admit everything
         const bool found = n_sample >= k;
-        bound[c] = found ? (unsigned long long)s_prefix << 32 : 0ull;
+        const uint32_t kth = s_prefix > slack ? s_prefix - slack : 0u;
+        bound[c] = found ? (unsigned long long)kth << 32 : 0ull;
         cnt[c] = 0u;
     }
 }
@@ -401,16 +402,25 @@ __global__ __launch_bounds__(SEL_THREADS) void k_topk_merge(
     __shared__ int pg[64];
     const int c = blockIdx.x;
     const int tid = threadIdx.x;
-    if (rc.dst && (int64_t)cnt[c] > cap) {
-        // the buffer overflowed and the last hop wrote no slab: recompute
-        // this column (warp per row, lanes over the row's in-edges)
+    if (rc.kind != 0 && (int64_t)cnt[c] > cap) {
+        // the buffer overflowed and no slab holds the final column:
+        // recompute it (warp per row; lanes over the row's in-edges for the
+        // last hop, over the embedding for the score)
         const int lane = tid & 31;
         for (int64_t j = tid >> 5; j < n; j += SEL_THREADS / 32) {
             float acc = 0.f;
-            for (int64_t e = rc.in_ptr[j] + lane; e < rc.in_ptr[j + 1]; e += 32)
-                acc = fmaf(rc.in_w[e], rc.prev[(int64_t)rc.in_src[e] * bp + c], acc);
+            if (rc.kind == 1) {
+                for (int64_t e = rc.in_ptr[j] + lane; e < rc.in_ptr[j + 1]; e += 32)
+                    acc = fmaf(rc.in_w[e], rc.prev[(int64_t)rc.in_src[e] * bp + c], acc);
+            } else {
+                const uint16_t *ej = rc.emb + j * rc.dim, *qc = rc.qp + (int64_t)c * rc.dim;
+                for (int t = lane; t < rc.dim; t += 32)
+                    acc = fmaf(bf16_to_f32(ej[t]), bf16_to_f32(qc[t]), acc);
+            }
             for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
-            if (lane == 0) rc.dst[j * bp + c] = fmaf(rc.alpha, acc, rc.u[j * bp + c]);
+            if (lane == 0)
+                rc.dst[j * bp + c] = rc.kind == 1 ? fmaf(rc.alpha, acc, rc.u[j * bp + c])
+                                                  : expf(rc.tau * acc - rc.shift[c]);
         }
         __threadfence_block();
         __syncthreads();
@@ -526,7 +536,7 @@ cudaError_t launch_buf_merge_signed(const unsigned int *cnt, const unsigned long
 template <bool SIGNED>
 static cudaError_t launch_kth(const SelectPlan &sp, const float *s, int b, const int32_t *ext_of,
                               int64_t id_limit, unsigned long long *ws, unsigned long long *bound,
-                              unsigned int *cnt, cudaStream_t st) {
+                              unsigned int *cnt, cudaStream_t st, uint32_t slack = 0) {
     static bool attr[64] = {false};
     int dev = 0;
     cudaGetDevice(&dev);
@@ -544,7 +554,8 @@ static cudaError_t launch_kth(const SelectPlan &sp, const float *s, int b, const
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
     const size_t smem = sp.n_sample <= KTH_STAGE ? (size_t)sp.n_sample * sizeof(uint32_t) : 0;
-    k_sample_kth<<<sp.bp, SEL_THREADS, smem, st>>>(keysT, sp.n_sample, b, sp.k, bound, cnt);
+    k_sample_kth<<<sp.bp, SEL_THREADS, smem, st>>>(keysT, sp.n_sample, b, sp.k, slack, bound,
+                                                   cnt);
     return cudaGetLastError();
 }
 
@@ -577,9 +588,9 @@ template <bool SIGNED>
 static cudaError_t sample_bound(const SelectPlan &sp, const float *s, int b,
                                 const int32_t *ext_of, int64_t id_limit,
                                 unsigned long long *ws, unsigned long long *bound,
-                                cudaStream_t st, int *launches) {
+                                cudaStream_t st, int *launches, uint32_t slack = 0) {
     cudaError_t e = launch_kth<SIGNED>(sp, s, b, ext_of, id_limit, ws, bound,
-                                       (unsigned int *)(ws + sp.off_cnt), st);
+                                       (unsigned int *)(ws + sp.off_cnt), st, slack);
     if (launches) *launches += 2;
     return e;
 }
@@ -593,9 +604,9 @@ cudaError_t launch_sample_bound_signed(const SelectPlan &sp, const float *s, int
 
 cudaError_t launch_sample_bound(const SelectPlan &sp, const float *s, int b,
                                 const int32_t *ext_of, unsigned long long *ws, cudaStream_t st,
-                                int *launches) {
+                                int *launches, uint32_t slack) {
     return sample_bound<false>(sp, s, b, ext_of, (int64_t)1 << 40, ws, ws + sp.off_bound, st,
-                               launches);
+                               launches, slack);
 }
 
 cudaError_t launch_select(const SelectPlan &sp, const float *s, int b, unsigned long long *ws,
@@ -615,8 +626,8 @@ cudaError_t launch_topk_merge(const SelectPlan &sp, const float *s, int b,
                               const int32_t *page_row, int64_t *ids, float *scores,
                               int32_t *page_ids, int32_t *n_pages, int *status,
                               const ColumnRecompute *rc, cudaStream_t st, int *launches) {
-    const ColumnRecompute r = rc ? *rc : ColumnRecompute{nullptr, nullptr, nullptr, nullptr,
-                                                          nullptr, 0.f, nullptr};
+    ColumnRecompute r{};
+    if (rc) r = *rc;
     k_topk_merge<<<b, SEL_THREADS, 0, st>>>(s, sp.n, sp.bp, sp.k, ext_of,
                                             (const unsigned int *)(ws + sp.off_cnt),
                                             ws + sp.off_buf, sp.cap, zpart, n_ztiles, row_of,

@@ -26,6 +26,13 @@ __global__ void k_ext_sample(const int32_t *__restrict__ ext_of, int64_t n_sampl
         out[v] = ext_of[v * stride];
 }
 
+cudaError_t launch_ext_sample(const int32_t *ext_of, int64_t n_sample, int64_t stride,
+                              int32_t *out, cudaStream_t st) {
+    if (n_sample <= 0) return cudaSuccess;
+    k_ext_sample<<<device_sm_count(), 256, 0, st>>>(ext_of, n_sample, stride, out);
+    return cudaGetLastError();
+}
+
 // Exact path, batch by batch: dots of every row against 256 new chunks
 // written to a slab, then the three-pass selection (used when a fused
 // filter buffer overflows).

@@ -94,6 +94,23 @@ def test_fused_filter_overflow_falls_back():
     assert_retrieval_parity(wl, "clustered", got, ref)
 
 
+def test_score_filter_overflow_falls_back():
+    """No hops, N = 16384 chunks sharing one embedding: every score is equal,
+    all rows clear the bound taken from the score's row sample and the
+    8192-key buffer of every query overflows; the merge recomputes the
+    query's scores and selects the k lowest IDs among the ties."""
+    import dataclasses
+    base = synth.workload(2, scale=1 / 64)
+    emb = np.repeat(base.emb[:1], base.n, axis=0)
+    wl = dataclasses.replace(base, emb=emb, row_ptr=np.zeros(base.n + 1, np.int64),
+                             col=np.zeros(0, np.int32), aff=np.zeros(0, np.float32), hops=0)
+    q = wl.queries[:4]
+    _, got = gpu_retrieve(wl, "clustered", queries=q, k=8)
+    ref = oracle_retrieve(wl, "clustered", queries=q, k=8)
+    assert_retrieval_parity(wl, "clustered", got, ref)
+    assert (np.sort(got["ids"], axis=1) == np.arange(8)).all()
+
+
 def test_no_edges_and_single_chunk_pages():
     """A store without relations: propagation adds nothing."""
     wl0 = synth.workload(0)
