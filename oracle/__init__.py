@@ -58,6 +58,9 @@ def _load():
             lib.ora_retrieve.argtypes = [P, i64, i32, P, i32, P, P, P, f64, f64, i32, i32, P,
                                          P, P, P, P, P, P, P]
             lib.ora_retrieve.restype = ctypes.c_int
+            lib.ora_retrieve_scoped.argtypes = [P, i64, i32, P, i32, P, P, P, f64, f64, i32, i32,
+                                                P, P, P, i32, P, P, P, P, P]
+            lib.ora_retrieve_scoped.restype = ctypes.c_int
             lib.ora_update_relations.argtypes = [P, i32, i64, i64, i32, f64, i32, P, P, P, P, P, P,
                                                  P, P]
             lib.ora_update_relations.restype = ctypes.c_int
@@ -89,12 +92,20 @@ def row_softmax(row_ptr: np.ndarray, aff: np.ndarray) -> np.ndarray:
 
 
 def retrieve(emb, queries, row_ptr, col, w, *, tau, alpha, hops, k, page_of=None,
-             want_final=False):
+             want_final=False, ns_of=None, q_ns=None, sort_by_time=False):
     """Score -> propagate -> top-k -> page resolve for every query (fp64).
 
     Returns dict(ids int64[B,k], scores float64[B,k], page_ids int32[B,k],
     n_pages int32[B], z float64[B], shift float64[B], final float64[B,N] if
-    want_final)."""
+    want_final).  With ns_of (int32[N], a namespace tag per chunk) and q_ns
+    (int32[B]) query b selects only among chunks tagged q_ns[b] (padding:
+    ID -1, score 0, page -1; z and shift are then not reported); with
+    sort_by_time the selected IDs come in ascending ID order (§4.1,
+    Algorithm 1: namespace-scoped candidates, SortByTime)."""
+    if ns_of is not None or q_ns is not None or sort_by_time:
+        return _retrieve_scoped(emb, queries, row_ptr, col, w, tau=tau, alpha=alpha, hops=hops,
+                                k=k, page_of=page_of, want_final=want_final, ns_of=ns_of,
+                                q_ns=q_ns, sort_by_time=sort_by_time)
     emb = np.ascontiguousarray(emb, dtype=np.uint16)
     queries = np.ascontiguousarray(queries, dtype=np.uint16)
     n, d = emb.shape
@@ -117,6 +128,34 @@ def retrieve(emb, queries, row_ptr, col, w, *, tau, alpha, hops, k, page_of=None
         _ptr(out["scores"]), _ptr(out["page_ids"]), _ptr(out["n_pages"]), _ptr(final),
         _ptr(out["z"]), _ptr(out["shift"]))
     _check(rc, "retrieve")
+    if final is not None:
+        out["final"] = final
+    return out
+
+
+def _retrieve_scoped(emb, queries, row_ptr, col, w, *, tau, alpha, hops, k, page_of, want_final,
+                     ns_of, q_ns, sort_by_time):
+    emb = np.ascontiguousarray(emb, dtype=np.uint16)
+    queries = np.ascontiguousarray(queries, dtype=np.uint16)
+    n, d = emb.shape
+    b = queries.shape[0]
+    if row_ptr is not None:
+        row_ptr = np.ascontiguousarray(row_ptr, dtype=np.int64)
+        col = np.ascontiguousarray(col, dtype=np.int32)
+        w = np.ascontiguousarray(w, dtype=np.float64)
+    if page_of is not None:
+        page_of = np.ascontiguousarray(page_of, dtype=np.int32)
+    ns_of = np.ascontiguousarray(np.zeros(n, np.int32) if ns_of is None else ns_of, dtype=np.int32)
+    q_ns = np.ascontiguousarray(np.zeros(b, np.int32) if q_ns is None else q_ns, dtype=np.int32)
+    out = dict(ids=np.zeros((b, k), np.int64), scores=np.zeros((b, k), np.float64),
+               page_ids=np.zeros((b, k), np.int32), n_pages=np.zeros(b, np.int32))
+    final = np.zeros((b, n), np.float64) if want_final else None
+    rc = _load().ora_retrieve_scoped(
+        _ptr(emb), n, d, _ptr(queries), b, _ptr(row_ptr), _ptr(col), _ptr(w), float(tau),
+        float(alpha), int(hops), int(k), _ptr(page_of), _ptr(ns_of), _ptr(q_ns),
+        int(bool(sort_by_time)), _ptr(out["ids"]), _ptr(out["scores"]), _ptr(out["page_ids"]),
+        _ptr(out["n_pages"]), _ptr(final))
+    _check(rc, "retrieve_scoped")
     if final is not None:
         out["final"] = final
     return out

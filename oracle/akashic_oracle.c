@@ -39,6 +39,17 @@
  *      j also gets the edge j -> n with the same logit.  Rows stay sorted by
  *      column; the weights of every row are the row softmax of its logits.
  *
+ *  Namespace-scoped retrieval (the candidate set is the chunk table T[u][s]
+ *      of the caller's (user_id, session_id), §4.1 and Algorithm 1 retrieval
+ *      half) and SortByTime (Algorithm 1: the selected chunks are returned in
+ *      chronological order):  every chunk carries a namespace tag ns_of[i];
+ *      query b selects only among chunks with ns_of[i] == q_ns[b] (scores,
+ *      Z and propagation are those of the whole store; the scope applies to
+ *      the candidates); with fewer than k such chunks the list is padded
+ *      with ID -1, score 0, page -1.  With sort_by_time the selected IDs
+ *      are reordered by ascending chunk ID (IDs are assigned in append
+ *      order), padding last.
+ *
  * Readings where the paper is silent (also recorded in the design notes):
  *   - temperature tau defaults to 1/sqrt(dim) for every store;
  *   - multi-hop form s^(h) = u + alpha * s^(h-1) R (truncated personalised
@@ -128,11 +139,57 @@ static int cmp_i64(const void *pa, const void *pb)
  * optional final_out[n_q*n] (every final score), z_out[n_q] (Z_b),
  *          shift_out[n_q] (c_b)
  */
+static int retrieve_impl(const uint16_t *emb, int64_t n, int32_t dim, const uint16_t *q,
+                         int32_t n_q, const int64_t *row_ptr, const int32_t *col, const double *w,
+                         double tau, double alpha, int32_t hops, int32_t k,
+                         const int32_t *page_of, const int32_t *ns_of, const int32_t *q_ns,
+                         int32_t sort_by_time, int64_t *ids, double *scores, int32_t *page_ids,
+                         int32_t *n_pages, double *final_out, double *z_out, double *shift_out);
+
 int ora_retrieve(const uint16_t *emb, int64_t n, int32_t dim, const uint16_t *q, int32_t n_q,
                  const int64_t *row_ptr, const int32_t *col, const double *w, double tau,
                  double alpha, int32_t hops, int32_t k, const int32_t *page_of, int64_t *ids,
                  double *scores, int32_t *page_ids, int32_t *n_pages, double *final_out,
                  double *z_out, double *shift_out)
+{
+    return retrieve_impl(emb, n, dim, q, n_q, row_ptr, col, w, tau, alpha, hops, k, page_of,
+                         NULL, NULL, 0, ids, scores, page_ids, n_pages, final_out, z_out,
+                         shift_out);
+}
+
+/*
+ * As ora_retrieve, with query b selecting only among the chunks whose
+ * ns_of[i] equals q_ns[b] (ns_of[n], q_ns[n_q]), padded with ID -1 when
+ * fewer than k exist, and with sort_by_time != 0 returning the selected IDs
+ * in ascending ID order.
+ */
+int ora_retrieve_scoped(const uint16_t *emb, int64_t n, int32_t dim, const uint16_t *q,
+                        int32_t n_q, const int64_t *row_ptr, const int32_t *col, const double *w,
+                        double tau, double alpha, int32_t hops, int32_t k,
+                        const int32_t *page_of, const int32_t *ns_of, const int32_t *q_ns,
+                        int32_t sort_by_time, int64_t *ids, double *scores, int32_t *page_ids,
+                        int32_t *n_pages, double *final_out)
+{
+    if (!ns_of || !q_ns)
+        return ORA_EINVAL;
+    return retrieve_impl(emb, n, dim, q, n_q, row_ptr, col, w, tau, alpha, hops, k, page_of,
+                         ns_of, q_ns, sort_by_time, ids, scores, page_ids, n_pages, final_out,
+                         NULL, NULL);
+}
+
+/* selected entries of one query by ascending ID (padding -1 stays last) */
+static int cmp_id_time(const void *pa, const void *pb)
+{
+    const ora_pair *a = (const ora_pair *)pa, *b = (const ora_pair *)pb;
+    return (a->id < b->id) ? -1 : (a->id > b->id);
+}
+
+static int retrieve_impl(const uint16_t *emb, int64_t n, int32_t dim, const uint16_t *q,
+                         int32_t n_q, const int64_t *row_ptr, const int32_t *col, const double *w,
+                         double tau, double alpha, int32_t hops, int32_t k,
+                         const int32_t *page_of, const int32_t *ns_of, const int32_t *q_ns,
+                         int32_t sort_by_time, int64_t *ids, double *scores, int32_t *page_ids,
+                         int32_t *n_pages, double *final_out, double *z_out, double *shift_out)
 {
     if (n < 1 || dim < 1 || n_q < 0 || k < 1 || k > n || hops < 0 || alpha < 0.0)
         return ORA_EINVAL;
@@ -180,10 +237,14 @@ int ora_retrieve(const uint16_t *emb, int64_t n, int32_t dim, const uint16_t *q,
             for (int64_t j = 0; j < n; ++j)
                 s[j] = u[j] + alpha * t[j];
         }
+        int64_t n_cand = 0;
         for (int64_t i = 0; i < n; ++i) {
             s[i] /= zsum;
-            order[i].key = s[i];
-            order[i].id = i;
+            if (ns_of && ns_of[i] != q_ns[b])
+                continue;   /* outside the query's namespace: not a candidate */
+            order[n_cand].key = s[i];
+            order[n_cand].id = i;
+            ++n_cand;
         }
         if (final_out)
             memcpy(final_out + (int64_t)b * n, s, sizeof(double) * n);
@@ -191,22 +252,26 @@ int ora_retrieve(const uint16_t *emb, int64_t n, int32_t dim, const uint16_t *q,
             z_out[b] = zsum;
         if (shift_out)
             shift_out[b] = cmax;
-        /* top-k by full sort */
-        qsort(order, (size_t)n, sizeof(ora_pair), cmp_desc_id);
+        /* top-k by full sort of the candidates */
+        qsort(order, (size_t)n_cand, sizeof(ora_pair), cmp_desc_id);
+        const int32_t got = n_cand < k ? (int32_t)n_cand : k;
+        if (sort_by_time)
+            qsort(order, (size_t)got, sizeof(ora_pair), cmp_id_time);
         for (int32_t r = 0; r < k; ++r) {
-            ids[(int64_t)b * k + r] = order[r].id;
-            scores[(int64_t)b * k + r] = order[r].key;
+            ids[(int64_t)b * k + r] = r < got ? order[r].id : -1;
+            scores[(int64_t)b * k + r] = r < got ? order[r].key : 0.0;
         }
         /* page resolve */
         if (page_of) {
             for (int32_t r = 0; r < k; ++r) {
-                int32_t p = page_of[order[r].id];
+                int32_t p = r < got ? page_of[order[r].id] : -1;
                 page_ids[(int64_t)b * k + r] = p;
-                pg[r] = p;
+                if (r < got)
+                    pg[r] = p;
             }
-            qsort(pg, (size_t)k, sizeof(int64_t), cmp_i64);
+            qsort(pg, (size_t)got, sizeof(int64_t), cmp_i64);
             int32_t distinct = 0;
-            for (int32_t r = 0; r < k; ++r)
+            for (int32_t r = 0; r < got; ++r)
                 if (r == 0 || pg[r] != pg[r - 1])
                     ++distinct;
             n_pages[b] = distinct;

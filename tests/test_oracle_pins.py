@@ -419,3 +419,61 @@ def test_update_rejects_nonempty_new_rows():
     rp[first + 1:] += 1                                   # row `first` gains an edge
     with pytest.raises(ValueError):
         oracle.update_relations(emb, first, n_new, m, rp, col2, aff2)
+
+
+# --------------------------------------------------------------------------- namespaces, SortByTime
+def _dense_final(emb, q, row_ptr, col, w, tau, alpha, hops):
+    """Final scores from the dense power series (numpy, gather form)."""
+    n = emb.shape[0]
+    S = sum(np.linalg.matrix_power(alpha * dense_R(n, row_ptr, col, w), h) for h in range(hops + 1))
+    z = tau * widen(q) @ widen(emb).T
+    return np.stack([softmax_lib(z[b]) @ S for b in range(q.shape[0])])
+
+
+@pytest.mark.parametrize("hops", [0, 2])
+def test_scoped_selection_is_restricted_sort(hops):
+    """Namespace scope (§4.1: candidates are the caller's (user, session)
+    chunks): the selected IDs are the top-k of the whole store's final
+    scores restricted to the query's namespace, from the dense closed form.
+    Catches masking applied to the wrong side (query vs chunk), masks that
+    leak into propagation, and the padding when a namespace is smaller than k."""
+    n, k = 150, 9
+    emb, q, row_ptr, col, aff = tiny_store(21, n, 16, 6, n_q=4)
+    w = oracle.row_softmax(row_ptr, aff)
+    rng = np.random.default_rng(5)
+    ns_of = rng.integers(0, 5, n).astype(np.int32)
+    ns_of[ns_of == 4] = 3
+    ns_of[:4] = 4                      # namespace 4 holds only chunks 0..3 (< k)
+    q_ns = np.array([0, 2, 3, 4], np.int32)
+    page_of = (np.arange(n) // 10).astype(np.int32)
+    out = oracle.retrieve(emb, q, row_ptr, col, w, tau=0.3, alpha=0.5, hops=hops, k=k,
+                          page_of=page_of, ns_of=ns_of, q_ns=q_ns, want_final=True)
+    ref = _dense_final(emb, q, row_ptr, col, w, 0.3, 0.5, hops)
+    for b in range(4):
+        cand = np.nonzero(ns_of == q_ns[b])[0]
+        top = cand[np.lexsort((cand, -ref[b][cand]))][:k]
+        got = out["ids"][b]
+        assert list(got[:len(top)]) == list(top)
+        assert (got[len(top):] == -1).all() and (out["page_ids"][b][len(top):] == -1).all()
+        assert np.allclose(out["scores"][b][:len(top)], ref[b][top], rtol=1e-12)
+        assert out["n_pages"][b] == len(set(page_of[top].tolist()))
+        assert np.allclose(out["final"][b], ref[b], rtol=1e-12)   # scores of the whole store
+
+
+def test_sort_by_time_reorders_only():
+    """SortByTime (Algorithm 1): the same chunks as the score order, returned
+    in ascending chunk ID (append order), padding last; with one namespace
+    holding every chunk the scoped result equals the unscoped one."""
+    n, k = 120, 7
+    emb, q, row_ptr, col, aff = tiny_store(22, n, 16, 5, n_q=3)
+    w = oracle.row_softmax(row_ptr, aff)
+    base = oracle.retrieve(emb, q, row_ptr, col, w, tau=0.3, alpha=0.5, hops=1, k=k)
+    one = oracle.retrieve(emb, q, row_ptr, col, w, tau=0.3, alpha=0.5, hops=1, k=k,
+                          ns_of=np.zeros(n, np.int32), q_ns=np.zeros(3, np.int32))
+    assert (one["ids"] == base["ids"]).all()
+    tm = oracle.retrieve(emb, q, row_ptr, col, w, tau=0.3, alpha=0.5, hops=1, k=k,
+                         sort_by_time=True)
+    for b in range(3):
+        assert list(tm["ids"][b]) == sorted(base["ids"][b].tolist())
+        sc = dict(zip(base["ids"][b].tolist(), base["scores"][b].tolist()))
+        assert [sc[i] for i in tm["ids"][b]] == tm["scores"][b].tolist()
