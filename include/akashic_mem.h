@@ -139,6 +139,34 @@ akashic_status_t akashic_mem_retrieve(akashic_mem_t *m, const uint16_t *q, int32
                                       float alpha, int32_t hops, int64_t *ids, float *scores,
                                       int32_t *page_ids, int32_t *n_pages, void *stream);
 
+/* Namespace tags (§4.1: memory chunks are keyed by (user_id, session_id),
+ * which isolate tenants and sessions).  The caller maps each (user_id,
+ * session_id) pair to one int32 tag; ns (device int32[n]) sets the tags of
+ * chunk IDs [first, first+n).  Every chunk starts with tag 0.
+ * EINVAL if the range leaves the store or ns is NULL with n > 0.
+ * Stream-ordered, does not synchronise. */
+akashic_status_t akashic_mem_set_namespace(akashic_mem_t *m, int64_t first, int64_t n,
+                                           const int32_t *ns, void *stream);
+
+/* Retrieval scoped to the caller's namespace, with optional chronological
+ * order (§4.1: candidates are the chunks of the current user_id/session_id;
+ * Algorithm 1 lines SortByTime: the selected chunks are returned in time
+ * order).  As akashic_mem_retrieve, except:
+ *   q_ns          device int32[B] or NULL: query b selects only among chunks
+ *                 whose tag equals q_ns[b] (scores, Z and propagation are
+ *                 those of the whole store; the scope applies to the
+ *                 candidates).  A namespace with fewer than k chunks pads
+ *                 the query's list with ID -1, score 0, page -1, and
+ *                 n_pages counts the real entries only.
+ *   sort_by_time  != 0: the k selected chunks are written in ascending chunk
+ *                 ID (IDs are assigned in append order) instead of by score.
+ * Errors as akashic_mem_retrieve.  Does not synchronise. */
+akashic_status_t akashic_mem_retrieve_scoped(akashic_mem_t *m, const uint16_t *q, int32_t B,
+                                             int32_t k, float alpha, int32_t hops,
+                                             const int32_t *q_ns, int32_t sort_by_time,
+                                             int64_t *ids, float *scores, int32_t *page_ids,
+                                             int32_t *n_pages, void *stream);
+
 /* Read back the canonical out-edge CSR.  With all array pointers NULL only
  * the sizes are returned (host n_rows, host nnz).  Otherwise row_ptr device
  * int64[n_rows+1], col device int32[nnz], and optionally aff / w device

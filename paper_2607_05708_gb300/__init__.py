@@ -29,6 +29,7 @@ EXPORTS = (
     "akashic_mem_update_relations", "akashic_mem_retrieve", "akashic_mem_export_csr",
     "akashic_mem_size", "akashic_mem_sync", "akashic_mem_set_profiling",
     "akashic_mem_phase_times", "akashic_mem_last_error", "akashic_mem_softmax_scores_noalloc",
+    "akashic_mem_set_namespace", "akashic_mem_retrieve_scoped",
 )
 
 
@@ -66,6 +67,9 @@ def load_library(path: str | None = None):
         "akashic_mem_append_chunks": ([V, V, I64, V, V, V, V, P64, V], ctypes.c_int),
         "akashic_mem_update_relations": ([V, I64, I64, I32, I32, V], ctypes.c_int),
         "akashic_mem_retrieve": ([V, V, I32, I32, F, I32, V, V, V, V, V], ctypes.c_int),
+        "akashic_mem_retrieve_scoped": ([V, V, I32, I32, F, I32, V, I32, V, V, V, V, V],
+                                        ctypes.c_int),
+        "akashic_mem_set_namespace": ([V, I64, I64, V, V], ctypes.c_int),
         "akashic_mem_export_csr": ([V, P64, P64, V, V, V, V, V], ctypes.c_int),
         "akashic_mem_size": ([V, P64, P64], ctypes.c_int),
         "akashic_mem_sync": ([V, V], ctypes.c_int),
@@ -200,10 +204,19 @@ class MemStore:
         _check(load_library().akashic_mem_update_relations(
             self._h, first, n, M, int(bool(reciprocal)), _stream(self._torch, stream, self.device)))
 
+    def set_namespace(self, first: int, ns, stream=None):
+        """Tags of chunk IDs [first, first+len(ns)) (int32 device tensor)."""
+        torch = self._torch
+        self._dev(ns, torch.int32, "ns")
+        _check(load_library().akashic_mem_set_namespace(
+            self._h, first, ns.numel(), _ptr(ns), _stream(torch, stream, self.device)))
+
     def retrieve(self, q, k: int, alpha: float, hops: int, ids=None, scores=None, page_ids=None,
-                 n_pages=None, stream=None):
+                 n_pages=None, stream=None, q_ns=None, sort_by_time: bool = False):
         """q: int16 [B, dim] bf16 bits.  Returns (ids int64 [B,k], scores f32 [B,k],
-        page_ids int32 [B,k], n_pages int32 [B]); outputs are allocated unless given."""
+        page_ids int32 [B,k], n_pages int32 [B]); outputs are allocated unless given.
+        q_ns (int32 [B] device tensor) scopes each query to its namespace;
+        sort_by_time returns the winners in ascending chunk ID."""
         torch = self._torch
         self._dev(q, torch.int16, "q")
         B = q.shape[0]
@@ -220,9 +233,17 @@ class MemStore:
         self._dev(scores, torch.float32, "scores", B * k)
         self._dev(page_ids, torch.int32, "page_ids", B * k)
         self._dev(n_pages, torch.int32, "n_pages", B)
-        _check(load_library().akashic_mem_retrieve(
-            self._h, _ptr(q), B, k, float(alpha), hops, _ptr(ids), _ptr(scores), _ptr(page_ids),
-            _ptr(n_pages), _stream(torch, stream, self.device)))
+        if q_ns is None and not sort_by_time:
+            _check(load_library().akashic_mem_retrieve(
+                self._h, _ptr(q), B, k, float(alpha), hops, _ptr(ids), _ptr(scores),
+                _ptr(page_ids), _ptr(n_pages), _stream(torch, stream, self.device)))
+        else:
+            if q_ns is not None:
+                self._dev(q_ns, torch.int32, "q_ns", B)
+            _check(load_library().akashic_mem_retrieve_scoped(
+                self._h, _ptr(q), B, k, float(alpha), hops,
+                None if q_ns is None else _ptr(q_ns), int(bool(sort_by_time)), _ptr(ids),
+                _ptr(scores), _ptr(page_ids), _ptr(n_pages), _stream(torch, stream, self.device)))
         return ids, scores, page_ids, n_pages
 
     def size(self):

@@ -82,6 +82,7 @@ struct DevBuf {
 struct StreamScratch {
     DevBuf qp, shift, u, sa, sb, zpart, partial, cand, counters;
     DevBuf samp, ext_s, zsamp;   // retrieval without hops: the score's row sample
+    DevBuf qns, ns_s;            // namespace scope: per query column, per sample row
 };
 
 struct ProfRec {
@@ -114,6 +115,7 @@ struct akashic_mem {
     // chunks live in HBM in page order: row r holds chunk ext_of[r], chunk c
     // is in row row_of[c]; page_of is indexed by row
     DevBuf emb, page_of, ext_of, row_of, max_norm, status;
+    DevBuf ns_row;               // namespace tag of the chunk in each row (0 by default)
     // canonical out-edge CSR
     int64_t nnz = 0;
     DevBuf row_ptr, col, aff, w;
@@ -402,6 +404,7 @@ akashic_status_t akashic_mem_create(const akashic_mem_config_t *cfg, akashic_mem
         (s = m->row_of.ensure((size_t)m->cap * 4)) != AKASHIC_OK ||
         (s = m->max_norm.ensure(4)) != AKASHIC_OK || (s = m->status.ensure(4)) != AKASHIC_OK ||
         (s = m->rstat.ensure((size_t)m->cap * 8)) != AKASHIC_OK ||
+        (s = m->ns_row.ensure((size_t)m->cap * 4)) != AKASHIC_OK ||
         (s = m->row_ptr.ensure((size_t)(m->cap + 1) * 8)) != AKASHIC_OK ||
         (s = m->in_ptr.ensure((size_t)(m->cap + 1) * 8)) != AKASHIC_OK) {
         delete m;
@@ -409,6 +412,7 @@ akashic_status_t akashic_mem_create(const akashic_mem_config_t *cfg, akashic_mem
     }
     if (cudaMemset(m->max_norm.p, 0, 4) != cudaSuccess || cudaMemset(m->status.p, 0, 4) != cudaSuccess ||
         cudaMemset(m->row_ptr.p, 0, 8) != cudaSuccess || cudaMemset(m->in_ptr.p, 0, 8) != cudaSuccess ||
+        cudaMemset(m->ns_row.p, 0, (size_t)m->cap * 4) != cudaSuccess ||
         cudaDeviceSynchronize() != cudaSuccess) {
         delete m;
         return fail(AKASHIC_ECUDA, "create: initialisation failed");
@@ -683,10 +687,49 @@ static StreamScratch *scratch_for(akashic_mem *m, void *stream) {
     return s;
 }
 
+static akashic_status_t retrieve_impl(akashic_mem *m, const uint16_t *q, int32_t B, int32_t k,
+                                      float alpha, int32_t hops, const int32_t *q_ns,
+                                      int32_t sort_by_time, int64_t *ids, float *scores,
+                                      int32_t *page_ids, int32_t *n_pages, void *stream);
+
 akashic_status_t akashic_mem_retrieve(akashic_mem_t *m, const uint16_t *q, int32_t B, int32_t k,
                                       float alpha, int32_t hops, int64_t *ids, float *scores,
                                       int32_t *page_ids, int32_t *n_pages, void *stream) {
     g_last_error.clear();
+    return retrieve_impl(m, q, B, k, alpha, hops, nullptr, 0, ids, scores, page_ids, n_pages,
+                         stream);
+}
+
+akashic_status_t akashic_mem_retrieve_scoped(akashic_mem_t *m, const uint16_t *q, int32_t B,
+                                             int32_t k, float alpha, int32_t hops,
+                                             const int32_t *q_ns, int32_t sort_by_time,
+                                             int64_t *ids, float *scores, int32_t *page_ids,
+                                             int32_t *n_pages, void *stream) {
+    g_last_error.clear();
+    return retrieve_impl(m, q, B, k, alpha, hops, q_ns, sort_by_time, ids, scores, page_ids,
+                         n_pages, stream);
+}
+
+akashic_status_t akashic_mem_set_namespace(akashic_mem_t *m, int64_t first, int64_t n,
+                                           const int32_t *ns, void *stream) {
+    g_last_error.clear();
+    if (!m) return fail(AKASHIC_EINVAL, "set_namespace: NULL store");
+    if (first < 0 || n < 0 || first + n > m->n)
+        return fail(AKASHIC_EINVAL, "set_namespace: range [%lld, %lld) outside the store of %lld",
+                    (long long)first, (long long)(first + n), (long long)m->n);
+    if (n == 0) return AKASHIC_OK;
+    if (!ns) return fail(AKASHIC_EINVAL, "set_namespace: NULL ns");
+    DeviceGuard g(m->device);
+    CUDA_TRY(launch_scatter_by_row(ns, m->row_of.as<int32_t>(), first, n, m->ns_row.as<int32_t>(),
+                                   (cudaStream_t)stream));
+    return AKASHIC_OK;
+}
+}  // extern "C"
+
+static akashic_status_t retrieve_impl(akashic_mem *m, const uint16_t *q, int32_t B, int32_t k,
+                                      float alpha, int32_t hops, const int32_t *q_ns,
+                                      int32_t sort_by_time, int64_t *ids, float *scores,
+                                      int32_t *page_ids, int32_t *n_pages, void *stream) {
     if (!m) return fail(AKASHIC_EINVAL, "retrieve: NULL store");
     if (!q || !ids || !scores) return fail(AKASHIC_EINVAL, "retrieve: NULL q/ids/scores");
     if (B < 1) return fail(AKASHIC_EINVAL, "retrieve: B < 1");
@@ -718,6 +761,15 @@ akashic_status_t akashic_mem_retrieve(akashic_mem_t *m, const uint16_t *q, int32
         if (eff_hops >= 1 && m->n_segs > 0) AK_TRY(sc->partial.ensure((size_t)m->n_segs * bp * 4));
         if (eff_hops >= 1) AK_TRY(sc->counters.ensure(64));
         const uint16_t *qb = q + (int64_t)off * m->dim;
+        // namespace scope of this batch's queries (padding columns get -1)
+        NsScope ns{};
+        if (q_ns) {
+            AK_TRY(sc->qns.ensure((size_t)bp * 4));
+            CUDA_TRY(cudaMemsetAsync(sc->qns.p, 0xff, (size_t)bp * 4, st));
+            CUDA_TRY(cudaMemcpyAsync(sc->qns.p, q_ns + off, (size_t)b * 4,
+                                     cudaMemcpyDeviceToDevice, st));
+            ns = NsScope{m->ns_row.as<int32_t>(), sc->qns.as<int32_t>()};
+        }
         // Without hops the top-k filter is fused into the score GEMM, which
         // then writes no slab: the bound comes from the score of every
         // stride-th row, computed first by the same kernel (same values).
@@ -746,12 +798,19 @@ akashic_status_t akashic_mem_retrieve(akashic_mem_t *m, const uint16_t *q, int32
                 AK_TRY(sc->zsamp.ensure((size_t)score_tiles(sp.n_sample) * bp * 4));
                 CUDA_TRY(launch_ext_sample(m->ext_of.as<int32_t>(), sp.n_sample, sp.stride,
                                            sc->ext_s.as<int32_t>(), st));
+                NsScope ns_samp{};
+                if (q_ns) {
+                    AK_TRY(sc->ns_s.ensure((size_t)sp.n_sample * 4));
+                    CUDA_TRY(launch_ext_sample(m->ns_row.as<int32_t>(), sp.n_sample, sp.stride,
+                                               sc->ns_s.as<int32_t>(), st));
+                    ns_samp = NsScope{sc->ns_s.as<int32_t>(), sc->qns.as<int32_t>()};
+                }
                 CUDA_TRY(launch_score_sample(m->emb.as<uint16_t>(), sp.n_sample, sp.stride, m->dim,
                                              sc->qp.as<uint16_t>(), bp, sc->shift.as<float>(),
                                              m->tau, sc->samp.as<float>(), sc->zsamp.as<float>(),
                                              m->status.as<int>(), st, &ps.launches));
                 CUDA_TRY(launch_sample_bound(sp2, sc->samp.as<float>(), b, sc->ext_s.as<int32_t>(),
-                                             ws, st, &ps.launches, 4u));
+                                             ws, st, &ps.launches, 4u, ns_samp));
                 ps.launches += 1;
             }
             PhaseScope ph(m, AKASHIC_PHASE_SCORE, st);
@@ -759,7 +818,7 @@ akashic_status_t akashic_mem_retrieve(akashic_mem_t *m, const uint16_t *q, int32
                                          bp, b, sc->shift.as<float>(), m->tau,
                                          sc->zpart.as<float>(), m->ext_of.as<int32_t>(),
                                          ws + sp.off_bound, (unsigned int *)(ws + sp.off_cnt),
-                                         ws + sp.off_buf, sp.cap, m->status.as<int>(), st,
+                                         ws + sp.off_buf, sp.cap, ns, m->status.as<int>(), st,
                                          &ph.launches, &zrows));
             rc.kind = 2;
             rc.emb = m->emb.as<uint16_t>();
@@ -802,10 +861,11 @@ akashic_status_t akashic_mem_retrieve(akashic_mem_t *m, const uint16_t *q, int32
                     // safe bound for s^(H).
                     PhaseScope ps(m, AKASHIC_PHASE_SELECT, st);
                     CUDA_TRY(launch_sample_bound(sp, fin, b, m->ext_of.as<int32_t>(), ws, st,
-                                                 &ps.launches));
+                                                 &ps.launches, 0u, ns));
                 }
                 const HopFilter flt{m->ext_of.as<int32_t>(), ws + sp.off_bound,
-                                    (unsigned int *)(ws + sp.off_cnt), ws + sp.off_buf, sp.cap};
+                                    (unsigned int *)(ws + sp.off_cnt), ws + sp.off_buf, sp.cap,
+                                    ns};
                 PhaseScope ph(m, AKASHIC_PHASE_PROPAGATE, st);
                 CUDA_TRY(launch_hop(hp, sc->u.as<float>(), fin, out, bp, alpha,
                                     sc->partial.as<float>(), sc->counters.as<int>(),
@@ -827,18 +887,21 @@ akashic_status_t akashic_mem_retrieve(akashic_mem_t *m, const uint16_t *q, int32
                                            sc->zpart.as<float>(), zrows, m->ext_of.as<int32_t>(),
                                            m->row_of.as<int32_t>(), m->page_of.as<int32_t>(),
                                            ids + (int64_t)off * k, scores + (int64_t)off * k,
-                                           pids, npg, m->status.as<int>(), &rc, st,
-                                           &ph.launches));
+                                           pids, npg, m->status.as<int>(), &rc, ns,
+                                           sort_by_time, st, &ph.launches));
             else
                 CUDA_TRY(launch_select(sp, fin, b, sc->cand.as<unsigned long long>(),
                                        sc->zpart.as<float>(), zrows, m->ext_of.as<int32_t>(),
                                        m->row_of.as<int32_t>(), m->page_of.as<int32_t>(),
                                        ids + (int64_t)off * k, scores + (int64_t)off * k, pids,
-                                       npg, m->status.as<int>(), st, &ph.launches));
+                                       npg, m->status.as<int>(), ns, sort_by_time, st,
+                                       &ph.launches));
         }
     }
     return AKASHIC_OK;
 }
+
+extern "C" {
 
 akashic_status_t akashic_mem_export_csr(akashic_mem_t *m, int64_t *n_rows, int64_t *nnz,
                                         int64_t *row_ptr, int32_t *col, float *aff, float *w,

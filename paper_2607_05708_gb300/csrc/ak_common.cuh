@@ -37,6 +37,17 @@ __device__ __forceinline__ uint32_t key_id(unsigned long long key) {
     return ~(uint32_t)(key & 0xffffffffull);
 }
 
+// Namespace scope of a retrieval (§4.1: the candidates of a query are the
+// chunks of the caller's (user_id, session_id) table): row j is a candidate
+// for query column c iff ns_row[j] == q_ns[c].  q_ns == NULL: no scope.
+struct NsScope {
+    const int32_t *ns_row;   // [rows] tag of the chunk in each row (or sample row)
+    const int32_t *q_ns;     // [bp] tag of each query column
+};
+__device__ __forceinline__ bool in_scope(const NsScope &s, int64_t row, int col) {
+    return !s.q_ns || s.ns_row[row] == s.q_ns[col];
+}
+
 // Keys for signed cosine values: order-preserving map of any finite fp32 to
 // uint32 (flip all bits of negatives, set the sign bit of non-negatives).
 __device__ __forceinline__ uint32_t ordered_bits(float v) {
@@ -79,7 +90,7 @@ cudaError_t launch_score_filter(const uint16_t *emb, int64_t n, int dim, const u
                                 int bp, int64_t n_cols, const float *shift, float tau,
                                 float *zpart, const int32_t *ext_of,
                                 const unsigned long long *bound, unsigned int *cnt,
-                                unsigned long long *buf, int64_t cap, int *status,
+                                unsigned long long *buf, int64_t cap, NsScope ns, int *status,
                                 cudaStream_t st, int *launches, int *zrows);
 
 // Plain dot products out[j, c] = <e_{j*row_stride}, q_c> (bf16 tensor
@@ -153,6 +164,9 @@ cudaError_t launch_row_softmax(const int64_t *row_ptr, const float *aff, float *
 cudaError_t launch_in_degree(const int32_t *col, const int32_t *row_of, int64_t nnz, int64_t *deg,
                              cudaStream_t st);
 cudaError_t launch_iota(uint32_t *v, int64_t n, cudaStream_t st);
+// out[row_of[first + i]] = in[i], i < n.
+cudaError_t launch_scatter_by_row(const int32_t *in, const int32_t *row_of, int64_t first,
+                                  int64_t n, int32_t *out, cudaStream_t st);
 cudaError_t launch_map_keys(const uint32_t *sel, const int32_t *ids, const int32_t *row_of,
                             uint32_t *keys, int64_t n, cudaStream_t st);
 cudaError_t launch_gather_in(const uint32_t *order, const int32_t *src, const int32_t *row_of,
@@ -240,6 +254,7 @@ struct HopFilter {
     unsigned int *cnt;                // [bp]
     unsigned long long *buf;          // [bp][cap]
     int64_t cap;
+    NsScope ns;                       // candidates only within the query's namespace
 };
 // `counters` = 2 device ints, zeroed by the launcher (work queues).
 // `flt` may be NULL (no filter).
@@ -266,11 +281,15 @@ SelectPlan select_plan(int64_t n, int bp, int k, int sm_count, int64_t force_str
 // Retrieval: rows are store rows; keys and outputs carry chunk IDs
 // (ext_of), so ties resolve to the lower chunk ID; page_row is indexed by
 // row (row_of).  Scores are divided by Z = sum of zpart's first n_ztiles rows.
+// With a scope (ns.q_ns != NULL) a query whose namespace holds fewer than k
+// chunks gets its list padded with ID -1, score 0, page -1; with
+// sort_by_time the k winners are written in ascending chunk ID order
+// (Algorithm 1, SortByTime) instead of by score.
 cudaError_t launch_select(const SelectPlan &sp, const float *s, int b, unsigned long long *ws,
                           const float *zpart, int64_t n_ztiles, const int32_t *ext_of,
                           const int32_t *row_of, const int32_t *page_row, int64_t *ids,
                           float *scores, int32_t *page_ids, int32_t *n_pages, int *status,
-                          cudaStream_t st, int *launches);
+                          NsScope ns, int sort_by_time, cudaStream_t st, int *launches);
 // Same selection over signed values (cosines) among rows whose chunk ID is
 // below id_limit: the k best of each of the b columns go to nbr_ids /
 // nbr_cos rows c_base .. c_base+b-1.
@@ -286,7 +305,7 @@ cudaError_t launch_select_signed(const SelectPlan &sp, const float *s, int b,
 // score's last place (margin for a sample computed by another launch).
 cudaError_t launch_sample_bound(const SelectPlan &sp, const float *s, int b,
                                 const int32_t *ext_of, unsigned long long *ws, cudaStream_t st,
-                                int *launches, uint32_t slack = 0);
+                                int *launches, uint32_t slack = 0, NsScope ns = NsScope{});
 // A column of the last hop recomputed by the merge when the filter fused
 // into that hop (which writes no output slab) overflowed its buffer:
 // dst[j,c] = u[j,c] + alpha * sum_{e in in(j)} in_w[e] * prev[in_src[e],c].
@@ -316,7 +335,8 @@ cudaError_t launch_topk_merge(const SelectPlan &sp, const float *s, int b,
                               const int32_t *ext_of, const int32_t *row_of,
                               const int32_t *page_row, int64_t *ids, float *scores,
                               int32_t *page_ids, int32_t *n_pages, int *status,
-                              const ColumnRecompute *rc, cudaStream_t st, int *launches);
+                              const ColumnRecompute *rc, NsScope ns, int sort_by_time,
+                              cudaStream_t st, int *launches);
 cudaError_t launch_sample_bound_signed(const SelectPlan &sp, const float *s, int b,
                                        const int32_t *ext_of, int64_t id_limit,
                                        unsigned long long *ws, unsigned long long *bound,

@@ -401,6 +401,21 @@ cudaError_t launch_batch_layout(const uint32_t *order, int64_t first, int64_t n,
     return cudaGetLastError();
 }
 
+// out[row_of[first + i]] = in[i] for i < n (per-chunk values into row order).
+__global__ void k_scatter_by_row(const int32_t *__restrict__ in, const int32_t *__restrict__ row_of,
+                                 int64_t first, int64_t n, int32_t *__restrict__ out) {
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n;
+         i += (int64_t)gridDim.x * blockDim.x)
+        out[row_of[first + i]] = in[i];
+}
+
+cudaError_t launch_scatter_by_row(const int32_t *in, const int32_t *row_of, int64_t first,
+                                  int64_t n, int32_t *out, cudaStream_t st) {
+    if (n <= 0) return cudaSuccess;
+    k_scatter_by_row<<<device_sm_count() * 2, 256, 0, st>>>(in, row_of, first, n, out);
+    return cudaGetLastError();
+}
+
 // Split plan.  A row with more than SPLIT_T in-edges is cut at every source
 // window boundary (sources are sorted within a row, so the cut points are
 // found by binary search) and then every SEG_LEN edges.
@@ -658,7 +673,7 @@ __device__ __forceinline__ void hop_accumulate(const int32_t *__restrict__ in_sr
 // compare and the append.
 template <int BP>
 __device__ __noinline__ void hop_filter_row(const HopFilter &f, const unsigned long long *thr,
-                                           const uint4 *thr_hi, int sub, uint32_t id,
+                                           const uint4 *thr_hi, int sub, int64_t j, uint32_t id,
                                            const float4 (&o)[HopShape<BP>::V]) {
 #pragma unroll
     for (int v = 0; v < HopShape<BP>::V; ++v) {
@@ -672,7 +687,7 @@ __device__ __noinline__ void hop_filter_row(const HopFilter &f, const unsigned l
                 const int c = (sub + 32 * v) * 4 + e;
                 const unsigned long long key =
                     ((unsigned long long)x[e] << 32) | (unsigned long long)(~id);
-                if (key >= thr[c]) {
+                if (key >= thr[c] && in_scope(f.ns, j, c)) {
                     const unsigned int p = atomicAdd(&f.cnt[c], 1u);
                     if ((int64_t)p < f.cap) f.buf[(int64_t)c * f.cap + p] = key;
                 }
@@ -685,9 +700,9 @@ __device__ __noinline__ void hop_filter_row(const HopFilter &f, const unsigned l
 // hop by ~5% (measured), while a call per row costs ~2%.
 template <int BP, bool FILTER>
 __device__ __forceinline__ void hop_emit(const HopFilter &f, const unsigned long long *thr,
-                                         const uint4 *thr_hi, int sub, uint32_t id,
+                                         const uint4 *thr_hi, int sub, int64_t j, uint32_t id,
                                          const float4 (&o)[HopShape<BP>::V]) {
-    if constexpr (FILTER) hop_filter_row<BP>(f, thr, thr_hi, sub, id, o);
+    if constexpr (FILTER) hop_filter_row<BP>(f, thr, thr_hi, sub, j, id, o);
 }
 
 template <int BP, bool FILTER>
@@ -746,7 +761,7 @@ __device__ __forceinline__ void hop_fixup_row(int64_t j, int64_t a, int64_t b,
             o[v].w = fmaf(alpha, acc[v].w, o[v].w);
             if constexpr (!FILTER) st_stream(out4 + j * S::F + sub + 32 * v, o[v]);
         }
-        hop_emit<BP, FILTER>(f, thr, thr_hi, sub, id, o);
+        hop_emit<BP, FILTER>(f, thr, thr_hi, sub, j, id, o);
     }
 }
 
@@ -826,7 +841,7 @@ __global__ __launch_bounds__(256, 3) void k_hop_rows(const int64_t *__restrict__
                     b[v].w = fmaf(alpha, acc[v].w, b[v].w);
                     if constexpr (!FILTER) st_stream(out4 + j * S::F + sub + 32 * v, b[v]);
                 }
-                hop_emit<BP, FILTER>(f, thr, thr_hi, sub, id, b);
+                hop_emit<BP, FILTER>(f, thr, thr_hi, sub, j, id, b);
             }
         }
     }
@@ -881,7 +896,7 @@ static cudaError_t hop_bp(const HopPlan &p, const float *u, const float *in, flo
     const int64_t items = ceil_div<int64_t>(p.n, ROWS_PER_GRAB) + p.n_split_rows;
     const int64_t want = ceil_div<int64_t>(items, 8);
     const int grid = (int)(want < (int64_t)sms * 3 ? (want < 1 ? 1 : want) : (int64_t)sms * 3);
-    const HopFilter f = flt ? *flt : HopFilter{nullptr, nullptr, nullptr, nullptr, 0};
+    const HopFilter f = flt ? *flt : HopFilter{nullptr, nullptr, nullptr, nullptr, 0, NsScope{}};
     if (flt)
         k_hop_rows<BP, true><<<grid, 256, 0, st>>>(p.in_ptr, p.in_src, p.in_w, p.n,
                                                    (const float4 *)u, (const float4 *)in,

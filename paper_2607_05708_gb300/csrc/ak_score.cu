@@ -140,6 +140,7 @@ struct GemmEpi {
     unsigned int *cnt;                  // FILTER: [n_cols]
     unsigned long long *buf;            // FILTER: [n_cols][cap]
     int64_t cap;
+    NsScope ns;                         // EXP_FILTER: namespace scope of the queries
 };
 
 template <int BP, int MODE>
@@ -418,7 +419,8 @@ __global__ __launch_bounds__(GemmCfg<BP, MODE>::THREADS, 1) void k_gemm_umma(con
                         const float x = so[(((i >> 2) ^ (row & 7)) << 2) + (i & 3)];
                         const unsigned long long key =
                             ((unsigned long long)__float_as_uint(x) << 32) | fid;
-                        if (key >= bnd_s[ch * 32 + i]) {
+                        if (key >= bnd_s[ch * 32 + i] &&
+                            in_scope(ep.ns, grow, (int)(ct * BP + ch * 32 + i))) {
                             const int64_t cg = ct * BP + ch * 32 + i;
                             const unsigned int p = atomicAdd(&ep.cnt[cg], 1u);
                             if ((int64_t)p < ep.cap) ep.buf[cg * ep.cap + p] = key;
@@ -535,9 +537,10 @@ cudaError_t launch_score_filter(const uint16_t *emb, int64_t n, int dim, const u
                                 int bp, int64_t n_cols, const float *shift, float tau,
                                 float *zpart, const int32_t *ext_of,
                                 const unsigned long long *bound, unsigned int *cnt,
-                                unsigned long long *buf, int64_t cap, int *status,
+                                unsigned long long *buf, int64_t cap, NsScope ns, int *status,
                                 cudaStream_t st, int *launches, int *zrows) {
     GemmEpi ep{};
+    ep.ns = ns;
     ep.shift = shift;
     ep.tau = tau;
     ep.zpart = zpart;

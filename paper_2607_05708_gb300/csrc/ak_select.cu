@@ -134,7 +134,8 @@ constexpr int KTH_STAGE = 40960;   // sampled keys staged per CTA (160 KiB dynam
 template <bool SIGNED>
 __global__ __launch_bounds__(256) void k_sample_transpose(
     const float *__restrict__ s, int64_t n_sample, int64_t stride, int bp,
-    const int32_t *__restrict__ ext_of, int64_t id_limit, uint32_t *__restrict__ keysT) {
+    const int32_t *__restrict__ ext_of, int64_t id_limit, NsScope ns,
+    uint32_t *__restrict__ keysT) {
     __shared__ uint32_t tile[32][33];
     const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;
     const int64_t v0 = (int64_t)blockIdx.x * 32;
@@ -146,7 +147,7 @@ __global__ __launch_bounds__(256) void k_sample_transpose(
         uint32_t key = 0u;
         if (v < n_sample) {
             const int64_t j = v * stride;
-            if ((int64_t)ext_of[j] < id_limit) {
+            if ((int64_t)ext_of[j] < id_limit && in_scope(ns, j, c0 + tx)) {
                 const float x = s[j * bp + c0 + tx];
                 key = SIGNED ? ordered_bits(x) : __float_as_uint(x);
             }
@@ -297,8 +298,9 @@ struct SelShape {
 // Append key to column c's buffer if it clears the bound.
 __device__ __forceinline__ void sel_push(unsigned long long key, unsigned long long bound, int c,
                                          unsigned int *__restrict__ cnt,
-                                         unsigned long long *__restrict__ buf, int64_t cap) {
-    if (key >= bound) {
+                                         unsigned long long *__restrict__ buf, int64_t cap,
+                                         const NsScope &ns, int64_t j) {
+    if (key >= bound && in_scope(ns, j, c)) {
         const unsigned int p = atomicAdd(&cnt[c], 1u);
         if ((int64_t)p < cap) buf[(int64_t)c * cap + p] = key;
     }
@@ -307,7 +309,7 @@ __device__ __forceinline__ void sel_push(unsigned long long key, unsigned long l
 template <int BP, bool SIGNED>
 __global__ __launch_bounds__(256) void k_filter(const float *__restrict__ s, int64_t n,
                                                 const int32_t *__restrict__ ext_of,
-                                                int64_t id_limit,
+                                                int64_t id_limit, NsScope ns,
                                                 const unsigned long long *__restrict__ bound,
                                                 unsigned int *__restrict__ cnt,
                                                 unsigned long long *__restrict__ buf, int64_t cap) {
@@ -340,13 +342,14 @@ __global__ __launch_bounds__(256) void k_filter(const float *__restrict__ s, int
         for (int q = 0; q < R; ++q) {
             if ((int64_t)id[q] >= id_limit) continue;
             const uint32_t u = (uint32_t)id[q];
+            const int64_t j = (t0 + q) * S::G + g;
 #pragma unroll
             for (int v = 0; v < S::V; ++v) {
                 const int c = (sub + 32 * v) * 4;
-                sel_push(sel_key<SIGNED>(x[q][v].x, u), thr[v][0], c, cnt, buf, cap);
-                sel_push(sel_key<SIGNED>(x[q][v].y, u), thr[v][1], c + 1, cnt, buf, cap);
-                sel_push(sel_key<SIGNED>(x[q][v].z, u), thr[v][2], c + 2, cnt, buf, cap);
-                sel_push(sel_key<SIGNED>(x[q][v].w, u), thr[v][3], c + 3, cnt, buf, cap);
+                sel_push(sel_key<SIGNED>(x[q][v].x, u), thr[v][0], c, cnt, buf, cap, ns, j);
+                sel_push(sel_key<SIGNED>(x[q][v].y, u), thr[v][1], c + 1, cnt, buf, cap, ns, j);
+                sel_push(sel_key<SIGNED>(x[q][v].z, u), thr[v][2], c + 2, cnt, buf, cap, ns, j);
+                sel_push(sel_key<SIGNED>(x[q][v].w, u), thr[v][3], c + 3, cnt, buf, cap, ns, j);
             }
         }
     }
@@ -361,7 +364,8 @@ __device__ void column_top(const float *__restrict__ s, int64_t n, int bp, int k
                            const unsigned int *__restrict__ cnt,
                            const unsigned long long *__restrict__ buf, int64_t cap,
                            unsigned long long *stage, unsigned long long *win, int *win_n,
-                           int *hist, unsigned long long *s_prefix, int *s_remaining) {
+                           int *hist, unsigned long long *s_prefix, int *s_remaining,
+                           NsScope ns = NsScope{}) {
     const int64_t m = cnt[c];
     if (m <= cap) {
         const unsigned long long *bc = buf + (int64_t)c * cap;
@@ -377,7 +381,8 @@ __device__ void column_top(const float *__restrict__ s, int64_t n, int bp, int k
     } else {
         auto key_at = [&](int64_t i) -> unsigned long long {
             const int32_t id = ext_of[i];
-            return (int64_t)id >= id_limit ? 0ull : sel_key<SIGNED>(s[i * bp + c], (uint32_t)id);
+            return ((int64_t)id >= id_limit || !in_scope(ns, i, c))
+                       ? 0ull : sel_key<SIGNED>(s[i * bp + c], (uint32_t)id);
         };
         radix_select(n, k, key_at, win, win_n, hist, s_prefix, s_remaining);
     }
@@ -392,7 +397,7 @@ __global__ __launch_bounds__(SEL_THREADS) void k_topk_merge(
     const float *__restrict__ zpart, int64_t n_ztiles, const int32_t *__restrict__ row_of,
     const int32_t *__restrict__ page_row, int64_t *__restrict__ ids, float *__restrict__ scores,
     int32_t *__restrict__ page_ids, int32_t *__restrict__ n_pages, int *status,
-    const ColumnRecompute rc) {
+    const ColumnRecompute rc, const NsScope ns, const int sort_by_time) {
     __shared__ int hist[256 * (SEL_THREADS / 32)];
     __shared__ unsigned long long stage[SEL_STAGE];
     __shared__ unsigned long long win[64];
@@ -430,22 +435,31 @@ __global__ __launch_bounds__(SEL_THREADS) void k_topk_merge(
     for (int o = 16; o > 0; o >>= 1) z += __shfl_xor_sync(0xffffffffu, z, o);
     if ((tid & 31) == 0) zred[tid >> 5] = z;
     column_top<false>(s, n, bp, k, c, ext_of, (int64_t)1 << 40, cnt, buf, cap, stage, win, &win_n,
-                      hist, &s_prefix, &s_remaining);
-    if (tid == 0 && win_n != k) set_status(status, AKASHIC_EDEVICE);
+                      hist, &s_prefix, &s_remaining, ns);
+    // without a scope every query has k winners; with one, a namespace
+    // holding fewer than k chunks pads its list
+    if (tid == 0 && (win_n > k || (!ns.q_ns && win_n != k))) set_status(status, AKASHIC_EDEVICE);
     const int got = win_n < k ? win_n : k;
     if (tid < got) {
         const unsigned long long key = win[tid];
+        const uint32_t id = key_id(key);
+        // rank by score (key desc) or, with SortByTime, by chunk ID
         int rank = 0;
-        for (int t = 0; t < got; ++t) rank += win[t] > key;
+        for (int t = 0; t < got; ++t)
+            rank += sort_by_time ? (key_id(win[t]) < id) : (win[t] > key);
         double zsum = 0.0;
         for (int w = 0; w < SEL_THREADS / 32; ++w) zsum += zred[w];
-        const uint32_t id = key_id(key);
         const int64_t o = (int64_t)c * k + rank;
         ids[o] = (int64_t)id;
         scores[o] = (float)((double)sel_value<false>(key) / zsum);
         const int32_t p = page_row ? page_row[row_of[id]] : 0;
         pg[rank] = p;
         if (page_ids) page_ids[o] = p;
+    } else if (tid < k) {
+        const int64_t o = (int64_t)c * k + tid;
+        ids[o] = -1;
+        scores[o] = 0.f;
+        if (page_ids) page_ids[o] = -1;
     }
     __syncthreads();
     if (n_pages && tid < 32) {
@@ -536,7 +550,8 @@ cudaError_t launch_buf_merge_signed(const unsigned int *cnt, const unsigned long
 template <bool SIGNED>
 static cudaError_t launch_kth(const SelectPlan &sp, const float *s, int b, const int32_t *ext_of,
                               int64_t id_limit, unsigned long long *ws, unsigned long long *bound,
-                              unsigned int *cnt, cudaStream_t st, uint32_t slack = 0) {
+                              unsigned int *cnt, cudaStream_t st, uint32_t slack = 0,
+                              NsScope ns = NsScope{}) {
     static bool attr[64] = {false};
     int dev = 0;
     cudaGetDevice(&dev);
@@ -550,7 +565,7 @@ static cudaError_t launch_kth(const SelectPlan &sp, const float *s, int b, const
     uint32_t *keysT = (uint32_t *)(ws + sp.off_tr);
     const dim3 tgrid((unsigned)ceil_div<int64_t>(sp.n_sample, 32), (unsigned)(sp.bp / 32));
     k_sample_transpose<SIGNED><<<tgrid, 256, 0, st>>>(s, sp.n_sample, sp.stride, sp.bp, ext_of,
-                                                      id_limit, keysT);
+                                                      id_limit, ns, keysT);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
     const size_t smem = sp.n_sample <= KTH_STAGE ? (size_t)sp.n_sample * sizeof(uint32_t) : 0;
@@ -562,11 +577,12 @@ static cudaError_t launch_kth(const SelectPlan &sp, const float *s, int b, const
 template <bool SIGNED>
 static cudaError_t bound_and_filter(const SelectPlan &sp, const float *s, int b,
                                     const int32_t *ext_of, int64_t id_limit,
-                                    unsigned long long *ws, cudaStream_t st, int *launches) {
+                                    unsigned long long *ws, cudaStream_t st, int *launches,
+                                    NsScope ns = NsScope{}) {
     unsigned long long *bound = ws + sp.off_bound;
     unsigned int *cnt = (unsigned int *)(ws + sp.off_cnt);
     unsigned long long *buf = ws + sp.off_buf;
-    cudaError_t e = launch_kth<SIGNED>(sp, s, b, ext_of, id_limit, ws, bound, cnt, st);
+    cudaError_t e = launch_kth<SIGNED>(sp, s, b, ext_of, id_limit, ws, bound, cnt, st, 0, ns);
     if (e != cudaSuccess) return e;
     const int64_t warps = ceil_div<int64_t>(sp.n, 4);
     int grid = (int)(ceil_div<int64_t>(warps, 8) < (int64_t)device_sm_count() * 8
@@ -574,10 +590,10 @@ static cudaError_t bound_and_filter(const SelectPlan &sp, const float *s, int b,
                          : (int64_t)device_sm_count() * 8);
     grid = grid < 1 ? 1 : grid;
     switch (sp.bp) {
-    case 32: k_filter<32, SIGNED><<<grid, 256, 0, st>>>(s, sp.n, ext_of, id_limit, bound, cnt, buf, sp.cap); break;
-    case 64: k_filter<64, SIGNED><<<grid, 256, 0, st>>>(s, sp.n, ext_of, id_limit, bound, cnt, buf, sp.cap); break;
-    case 128: k_filter<128, SIGNED><<<grid, 256, 0, st>>>(s, sp.n, ext_of, id_limit, bound, cnt, buf, sp.cap); break;
-    case 256: k_filter<256, SIGNED><<<grid, 256, 0, st>>>(s, sp.n, ext_of, id_limit, bound, cnt, buf, sp.cap); break;
+    case 32: k_filter<32, SIGNED><<<grid, 256, 0, st>>>(s, sp.n, ext_of, id_limit, ns, bound, cnt, buf, sp.cap); break;
+    case 64: k_filter<64, SIGNED><<<grid, 256, 0, st>>>(s, sp.n, ext_of, id_limit, ns, bound, cnt, buf, sp.cap); break;
+    case 128: k_filter<128, SIGNED><<<grid, 256, 0, st>>>(s, sp.n, ext_of, id_limit, ns, bound, cnt, buf, sp.cap); break;
+    case 256: k_filter<256, SIGNED><<<grid, 256, 0, st>>>(s, sp.n, ext_of, id_limit, ns, bound, cnt, buf, sp.cap); break;
     default: return cudaErrorInvalidValue;
     }
     if (launches) *launches += 3;
@@ -588,9 +604,10 @@ template <bool SIGNED>
 static cudaError_t sample_bound(const SelectPlan &sp, const float *s, int b,
                                 const int32_t *ext_of, int64_t id_limit,
                                 unsigned long long *ws, unsigned long long *bound,
-                                cudaStream_t st, int *launches, uint32_t slack = 0) {
+                                cudaStream_t st, int *launches, uint32_t slack = 0,
+                                NsScope ns = NsScope{}) {
     cudaError_t e = launch_kth<SIGNED>(sp, s, b, ext_of, id_limit, ws, bound,
-                                       (unsigned int *)(ws + sp.off_cnt), st, slack);
+                                       (unsigned int *)(ws + sp.off_cnt), st, slack, ns);
     if (launches) *launches += 2;
     return e;
 }
@@ -604,20 +621,21 @@ cudaError_t launch_sample_bound_signed(const SelectPlan &sp, const float *s, int
 
 cudaError_t launch_sample_bound(const SelectPlan &sp, const float *s, int b,
                                 const int32_t *ext_of, unsigned long long *ws, cudaStream_t st,
-                                int *launches, uint32_t slack) {
+                                int *launches, uint32_t slack, NsScope ns) {
     return sample_bound<false>(sp, s, b, ext_of, (int64_t)1 << 40, ws, ws + sp.off_bound, st,
-                               launches, slack);
+                               launches, slack, ns);
 }
 
 cudaError_t launch_select(const SelectPlan &sp, const float *s, int b, unsigned long long *ws,
                           const float *zpart, int64_t n_ztiles, const int32_t *ext_of,
                           const int32_t *row_of, const int32_t *page_row, int64_t *ids,
                           float *scores, int32_t *page_ids, int32_t *n_pages, int *status,
-                          cudaStream_t st, int *launches) {
-    cudaError_t e = bound_and_filter<false>(sp, s, b, ext_of, (int64_t)1 << 40, ws, st, launches);
+                          NsScope ns, int sort_by_time, cudaStream_t st, int *launches) {
+    cudaError_t e = bound_and_filter<false>(sp, s, b, ext_of, (int64_t)1 << 40, ws, st, launches,
+                                            ns);
     if (e != cudaSuccess) return e;
     return launch_topk_merge(sp, s, b, ws, zpart, n_ztiles, ext_of, row_of, page_row, ids, scores,
-                             page_ids, n_pages, status, nullptr, st, launches);
+                             page_ids, n_pages, status, nullptr, ns, sort_by_time, st, launches);
 }
 
 cudaError_t launch_topk_merge(const SelectPlan &sp, const float *s, int b,
@@ -625,13 +643,15 @@ cudaError_t launch_topk_merge(const SelectPlan &sp, const float *s, int b,
                               const int32_t *ext_of, const int32_t *row_of,
                               const int32_t *page_row, int64_t *ids, float *scores,
                               int32_t *page_ids, int32_t *n_pages, int *status,
-                              const ColumnRecompute *rc, cudaStream_t st, int *launches) {
+                              const ColumnRecompute *rc, NsScope ns, int sort_by_time,
+                              cudaStream_t st, int *launches) {
     ColumnRecompute r{};
     if (rc) r = *rc;
     k_topk_merge<<<b, SEL_THREADS, 0, st>>>(s, sp.n, sp.bp, sp.k, ext_of,
                                             (const unsigned int *)(ws + sp.off_cnt),
                                             ws + sp.off_buf, sp.cap, zpart, n_ztiles, row_of,
-                                            page_row, ids, scores, page_ids, n_pages, status, r);
+                                            page_row, ids, scores, page_ids, n_pages, status, r,
+                                            ns, sort_by_time);
     if (launches) *launches += 1;
     return cudaGetLastError();
 }

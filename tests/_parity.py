@@ -97,6 +97,43 @@ def assert_retrieval_parity(wl, placement, got, ref, rows=None):
         assert got["n_pages"][r] == ref["n_pages"][b] or set(gi.tolist()) != set(oi.tolist())
 
 
+def assert_scoped_parity(wl, placement, got, ref, ns_of, q_ns, sort_by_time):
+    """Namespace-scoped retrieval: every real ID lies in the query's
+    namespace, the real IDs equal the oracle's up to near-tie swaps at the
+    k-th in-namespace score, padding (-1) exactly where the oracle pads, the
+    order is by score (up to near-ties) or, with SortByTime, by ascending ID;
+    scores, page IDs and page counts as in assert_retrieval_parity."""
+    page_of = wl.page_of[placement]
+    k = ref["ids"].shape[1]
+    for b in range(got["ids"].shape[0]):
+        gi = got["ids"][b].astype(np.int64)
+        oi = ref["ids"][b]
+        fin = ref["final"][b]
+        nv = int((oi >= 0).sum())
+        assert (gi[nv:] == -1).all() and (gi[:nv] >= 0).all(), f"query {b}: padding {gi}"
+        assert (got["page_ids"][b][nv:] == -1).all(), f"query {b}: padding pages"
+        g, o = gi[:nv], oi[:nv]
+        assert len(set(g.tolist())) == nv, f"query {b}: repeated IDs"
+        assert (ns_of[g] == q_ns[b]).all(), f"query {b}: ID outside namespace {q_ns[b]}"
+        if nv:
+            sk = ref["scores"][b][:nv].min()
+            for x in set(g.tolist()) ^ set(o.tolist()):
+                assert abs(fin[x] - sk) <= SWAP_REL * max(abs(fin[x]), abs(sk)), (
+                    f"query {b}: chunk {x} swapped outside the near-tie band")
+        if sort_by_time:
+            assert (np.diff(g) > 0).all(), f"query {b}: not in ascending ID order {g}"
+        else:
+            sg = fin[g]
+            for a in range(nv - 1):
+                assert sg[a] >= sg[a + 1] - SWAP_REL * max(abs(sg[a]), abs(sg[a + 1])), (
+                    f"query {b}: score order differs at {a}")
+        if nv:
+            rel = np.abs(got["scores"][b][:nv].astype(np.float64) - fin[g]) / np.abs(fin[g])
+            assert rel.max() <= SCORE_REL, f"query {b}: score error {rel.max():.3g}"
+        assert (got["page_ids"][b][:nv] == page_of[g]).all(), f"query {b}: page IDs differ"
+        assert got["n_pages"][b] == len(set(page_of[g].tolist())), f"query {b}: page count"
+
+
 # --------------------------------------------------------------------------- relation update
 def check_update(wl, sample=None, M=None, seed=0):
     """Append wl.new_emb to a store holding wl, run the update on the GPU and

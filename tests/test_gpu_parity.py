@@ -4,8 +4,8 @@ import numpy as np
 import pytest
 
 import synth
-from _parity import (assert_retrieval_parity, check_update, gpu_retrieve, gpu_store,
-                     oracle_retrieve)
+from _parity import (assert_retrieval_parity, assert_scoped_parity, check_update, gpu_retrieve,
+                     gpu_store, oracle_retrieve, oracle_weights)
 
 pytestmark = pytest.mark.gpu
 
@@ -109,6 +109,37 @@ def test_score_filter_overflow_falls_back():
     ref = oracle_retrieve(wl, "clustered", queries=q, k=8)
     assert_retrieval_parity(wl, "clustered", got, ref)
     assert (np.sort(got["ids"], axis=1) == np.arange(8)).all()
+
+
+@pytest.mark.parametrize("hops,sort_by_time", [(0, False), (2, False), (2, True), (1, True)])
+def test_namespace_scoped_retrieval(hops, sort_by_time):
+    """Chunks tagged by component mod 5, plus a namespace of only 3 chunks;
+    each of the 256 queries scoped to a seeded namespace (every 17th to the
+    small one, which pads its list); scores and propagation over the whole
+    store, candidates from the namespace only; score order or SortByTime.
+    N = 16384 from the gmm1m recipe."""
+    import oracle
+    import torch
+    wl = synth.workload(2, scale=1 / 64)
+    rng = np.random.default_rng(11)
+    ns_of = (wl.component % 5).astype(np.int32)
+    ns_of[rng.choice(wl.n, 3, replace=False)] = 7
+    q_ns = rng.integers(0, 5, wl.n_queries).astype(np.int32)
+    q_ns[::17] = 7
+    store = gpu_store(wl, "clustered")
+    store.set_namespace(0, torch.from_numpy(ns_of).cuda())
+    q = torch.from_numpy(np.ascontiguousarray(wl.queries).view(np.int16)).cuda()
+    ids, sc, pg, npg = store.retrieve(q, wl.k, wl.alpha, hops,
+                                      q_ns=torch.from_numpy(q_ns).cuda(),
+                                      sort_by_time=sort_by_time)
+    store.sync()
+    got = dict(ids=ids.cpu().numpy(), scores=sc.cpu().numpy(), page_ids=pg.cpu().numpy(),
+               n_pages=npg.cpu().numpy())
+    ref = oracle.retrieve(wl.emb, wl.queries, wl.row_ptr, wl.col, oracle_weights(wl), tau=wl.tau,
+                          alpha=wl.alpha, hops=hops, k=wl.k, page_of=wl.page_of["clustered"],
+                          want_final=True, ns_of=ns_of, q_ns=q_ns, sort_by_time=sort_by_time)
+    assert_scoped_parity(wl, "clustered", got, ref, ns_of, q_ns, sort_by_time)
+    assert (got["ids"][::17][:, 3:] == -1).all()
 
 
 def test_no_edges_and_single_chunk_pages():
