@@ -35,6 +35,11 @@ METRIC = "retrieve queries/sec at N=1M chunks, d=1024, B=256; % of roofline"
 WORKLOAD = ("gmm1m: N=1048576 chunks, d=1024 bf16, 4096-component Zipf(1.1) mixture, 32-neighbour "
             "power-law relation graph (nnz 33554432), B=256 queries, hops=2, alpha=0.5, k=32, "
             "64 chunks/page, clustered placement")
+SCOPED_METRIC = ("namespace-scoped retrieve queries/sec at N=1M chunks, d=1024, B=256, "
+                 "SortByTime")
+SCOPED_WORKLOAD = ("gmm1m store with 64 namespaces (chunk tag = mixture component mod 64), each "
+                   "query scoped to a seeded namespace, hops=2, alpha=0.5, k=32, results in "
+                   "chronological (chunk ID) order, clustered placement")
 DENSE_METRIC = "Dense-only retrieve queries/sec at N=1M chunks, d=1024, B=256, top-p 5, no hops"
 DENSE_WORKLOAD = ("gmm1m store (N=1048576, d=1024 bf16), B=256 queries, k=5, hops=0 "
                   "(embedding similarity only), 64 chunks/page, clustered placement")
@@ -130,7 +135,8 @@ class Clocks:
                 "samples": len(sm)}
 
 
-def cpu_baseline(wl, placement, n_queries, rng_seed=0, weights=None, k=None, hops=None):
+def cpu_baseline(wl, placement, n_queries, rng_seed=0, weights=None, k=None, hops=None,
+                 ns_of=None, q_ns=None, sort_by_time=False):
     """The oracle retrieving n_queries of the batch against the full store on
     one host thread (the relation weights, which the GPU store computes at
     append time, are computed once beforehand)."""
@@ -141,7 +147,8 @@ def cpu_baseline(wl, placement, n_queries, rng_seed=0, weights=None, k=None, hop
     t0 = time.perf_counter()
     oracle.retrieve(wl.emb, wl.queries[rows], wl.row_ptr if hops else None,
                     wl.col if hops else None, w, tau=wl.tau, alpha=wl.alpha, hops=hops,
-                    k=wl.k if k is None else k, page_of=wl.page_of[placement])
+                    k=wl.k if k is None else k, page_of=wl.page_of[placement], ns_of=ns_of,
+                    q_ns=None if q_ns is None else q_ns[rows], sort_by_time=sort_by_time)
     dt = time.perf_counter() - t0
     return dict(value=n_queries / dt, unit="queries/s", cores=1, kind="oracle",
                 sample=f"{n_queries} of the {wl.n_queries} queries against the full store, "
@@ -348,13 +355,15 @@ def main():
     ap.add_argument("--scale", type=float, default=1.0,
                     help="shrink N (profiling captures of a smaller case); 1.0 = the benchmark")
     ap.add_argument("--workload", default="retrieve",
-                    choices=["retrieve", "update", "streams", "dense"],
+                    choices=["retrieve", "update", "streams", "dense", "scoped"],
                     help="retrieve: the benchmark; update: relation update of 4096 new chunks "
                          "on the 1M-chunk store; streams: 4M-chunk store, 8 streams x 128 "
-                         "queries; dense: the Dense-only form (k=5, no hops) on the 1M store")
+                         "queries; dense: the Dense-only form (k=5, no hops) on the 1M store; "
+                         "scoped: namespace-scoped retrieval with SortByTime on the 1M store")
     args = ap.parse_args()
     if args.steps is None:
-        args.steps = {"retrieve": 100, "update": 5, "streams": 20, "dense": 100}[args.workload]
+        args.steps = {"retrieve": 100, "update": 5, "streams": 20, "dense": 100,
+                      "scoped": 100}[args.workload]
     if args.impl == "reference":
         return run_reference(args)
     if args.workload == "update":
@@ -363,12 +372,16 @@ def main():
         return run_streams(args)
     if args.workload == "dense":
         return run_retrieve(args, k=5, hops=0, metric=DENSE_METRIC, workload=DENSE_WORKLOAD)
+    if args.workload == "scoped":
+        return run_retrieve(args, metric=SCOPED_METRIC, workload=SCOPED_WORKLOAD, scoped=True)
     return run_retrieve(args)
 
 
-def run_retrieve(args, k=None, hops=None, metric=METRIC, workload=WORKLOAD):
+def run_retrieve(args, k=None, hops=None, metric=METRIC, workload=WORKLOAD, scoped=False):
     """The retrieval pass on the gmm1m store (k / hops override the
-    configuration: the Dense-only form uses k = 5, hops = 0)."""
+    configuration: the Dense-only form uses k = 5, hops = 0; `scoped` tags
+    chunks by component mod 64 and scopes each query to a namespace, with
+    results in chronological order)."""
     import torch
     ws, rank, local = dist_env()
     if ws > 1:
@@ -386,9 +399,14 @@ def run_retrieve(args, k=None, hops=None, metric=METRIC, workload=WORKLOAD):
     t_gen = time.perf_counter()
     wl = synth.workload(2, scale=args.scale)
     t_gen = time.perf_counter() - t_gen
+    ns_of = q_ns_host = None
+    if scoped:
+        ns_of = (wl.component % 64).astype(np.int32)
+        q_ns_host = np.random.default_rng(64).integers(0, 64, wl.n_queries).astype(np.int32)
     cpu = None
     if rank == 0 and not args.no_cpu_baseline and ws == 1:
-        cpu = cpu_baseline(wl, args.placement, args.cpu_queries, k=k, hops=hops)
+        cpu = cpu_baseline(wl, args.placement, args.cpu_queries, k=k, hops=hops, ns_of=ns_of,
+                           q_ns=q_ns_host, sort_by_time=scoped)
 
     store = MemStore.from_arrays(wl.emb, wl.page_of[args.placement], wl.row_ptr, wl.col, wl.aff,
                                  capacity=wl.n, chunks_per_page=wl.chunks_per_page,
@@ -403,8 +421,14 @@ def run_retrieve(args, k=None, hops=None, metric=METRIC, workload=WORKLOAD):
     pages = torch.empty((B, k), dtype=torch.int32, device=f"cuda:{dev}")
     npages = torch.empty((B,), dtype=torch.int32, device=f"cuda:{dev}")
 
+    q_ns = None
+    if scoped:
+        store.set_namespace(0, torch.from_numpy(ns_of).to(f"cuda:{dev}"))
+        q_ns = torch.from_numpy(q_ns_host).to(f"cuda:{dev}")
+
     def step():
-        store.retrieve(q_dev, k, wl.alpha, hops, ids, scores, pages, npages, stream=st)
+        store.retrieve(q_dev, k, wl.alpha, hops, ids, scores, pages, npages, stream=st,
+                       q_ns=q_ns, sort_by_time=scoped)
 
     def barrier():
         torch.cuda.synchronize(dev)
