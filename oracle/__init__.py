@@ -59,8 +59,10 @@ def _load():
                                          P, P, P, P, P, P, P]
             lib.ora_retrieve.restype = ctypes.c_int
             lib.ora_retrieve_scoped.argtypes = [P, i64, i32, P, i32, P, P, P, f64, f64, i32, i32,
-                                                P, P, P, i32, P, P, P, P, P]
+                                                P, P, P, P, i32, P, P, P, P, P]
             lib.ora_retrieve_scoped.restype = ctypes.c_int
+            lib.ora_drop_dead.argtypes = [i64, P, P, P, P, P, P, P]
+            lib.ora_drop_dead.restype = ctypes.c_int
             lib.ora_update_relations.argtypes = [P, i32, i64, i64, i32, f64, i32, P, P, P, P, P, P,
                                                  P, P]
             lib.ora_update_relations.restype = ctypes.c_int
@@ -92,7 +94,7 @@ def row_softmax(row_ptr: np.ndarray, aff: np.ndarray) -> np.ndarray:
 
 
 def retrieve(emb, queries, row_ptr, col, w, *, tau, alpha, hops, k, page_of=None,
-             want_final=False, ns_of=None, q_ns=None, sort_by_time=False):
+             want_final=False, ns_of=None, q_ns=None, sort_by_time=False, dead=None):
     """Score -> propagate -> top-k -> page resolve for every query (fp64).
 
     Returns dict(ids int64[B,k], scores float64[B,k], page_ids int32[B,k],
@@ -101,11 +103,12 @@ def retrieve(emb, queries, row_ptr, col, w, *, tau, alpha, hops, k, page_of=None
     (int32[B]) query b selects only among chunks tagged q_ns[b] (padding:
     ID -1, score 0, page -1; z and shift are then not reported); with
     sort_by_time the selected IDs come in ascending ID order (§4.1,
-    Algorithm 1: namespace-scoped candidates, SortByTime)."""
-    if ns_of is not None or q_ns is not None or sort_by_time:
+    Algorithm 1: namespace-scoped candidates, SortByTime).  With dead
+    (bool[N]) deleted chunks get no score and are never selected."""
+    if ns_of is not None or q_ns is not None or sort_by_time or dead is not None:
         return _retrieve_scoped(emb, queries, row_ptr, col, w, tau=tau, alpha=alpha, hops=hops,
                                 k=k, page_of=page_of, want_final=want_final, ns_of=ns_of,
-                                q_ns=q_ns, sort_by_time=sort_by_time)
+                                q_ns=q_ns, sort_by_time=sort_by_time, dead=dead)
     emb = np.ascontiguousarray(emb, dtype=np.uint16)
     queries = np.ascontiguousarray(queries, dtype=np.uint16)
     n, d = emb.shape
@@ -134,7 +137,7 @@ def retrieve(emb, queries, row_ptr, col, w, *, tau, alpha, hops, k, page_of=None
 
 
 def _retrieve_scoped(emb, queries, row_ptr, col, w, *, tau, alpha, hops, k, page_of, want_final,
-                     ns_of, q_ns, sort_by_time):
+                     ns_of, q_ns, sort_by_time, dead):
     emb = np.ascontiguousarray(emb, dtype=np.uint16)
     queries = np.ascontiguousarray(queries, dtype=np.uint16)
     n, d = emb.shape
@@ -145,20 +148,40 @@ def _retrieve_scoped(emb, queries, row_ptr, col, w, *, tau, alpha, hops, k, page
         w = np.ascontiguousarray(w, dtype=np.float64)
     if page_of is not None:
         page_of = np.ascontiguousarray(page_of, dtype=np.int32)
-    ns_of = np.ascontiguousarray(np.zeros(n, np.int32) if ns_of is None else ns_of, dtype=np.int32)
-    q_ns = np.ascontiguousarray(np.zeros(b, np.int32) if q_ns is None else q_ns, dtype=np.int32)
+    if (ns_of is None) != (q_ns is None):
+        raise ValueError("ns_of and q_ns go together")
+    if ns_of is not None:
+        ns_of = np.ascontiguousarray(ns_of, dtype=np.int32)
+        q_ns = np.ascontiguousarray(q_ns, dtype=np.int32)
+    if dead is not None:
+        dead = np.ascontiguousarray(dead, dtype=np.uint8)
     out = dict(ids=np.zeros((b, k), np.int64), scores=np.zeros((b, k), np.float64),
                page_ids=np.zeros((b, k), np.int32), n_pages=np.zeros(b, np.int32))
     final = np.zeros((b, n), np.float64) if want_final else None
     rc = _load().ora_retrieve_scoped(
         _ptr(emb), n, d, _ptr(queries), b, _ptr(row_ptr), _ptr(col), _ptr(w), float(tau),
-        float(alpha), int(hops), int(k), _ptr(page_of), _ptr(ns_of), _ptr(q_ns),
+        float(alpha), int(hops), int(k), _ptr(page_of), _ptr(ns_of), _ptr(q_ns), _ptr(dead),
         int(bool(sort_by_time)), _ptr(out["ids"]), _ptr(out["scores"]), _ptr(out["page_ids"]),
         _ptr(out["n_pages"]), _ptr(final))
     _check(rc, "retrieve_scoped")
     if final is not None:
         out["final"] = final
     return out
+
+
+def drop_dead(row_ptr, col, aff, dead):
+    """The CSR without every edge into or out of a deleted chunk (dead bool[N])."""
+    row_ptr = np.ascontiguousarray(row_ptr, dtype=np.int64)
+    col = np.ascontiguousarray(col, dtype=np.int32)
+    aff = np.ascontiguousarray(aff, dtype=np.float32)
+    dead = np.ascontiguousarray(dead, dtype=np.uint8)
+    n = row_ptr.shape[0] - 1
+    rp = np.zeros(n + 1, np.int64)
+    c = np.zeros(max(col.shape[0], 1), np.int32)
+    a = np.zeros(max(col.shape[0], 1), np.float32)
+    _check(_load().ora_drop_dead(n, _ptr(row_ptr), _ptr(col), _ptr(aff), _ptr(dead), _ptr(rp),
+                                 _ptr(c), _ptr(a)), "drop_dead")
+    return rp, c[:rp[-1]], a[:rp[-1]]
 
 
 def update_relations(emb, first, n_new, m, row_ptr, col, aff, *, scale=10.0, reciprocal=True):

@@ -50,6 +50,14 @@
  *      are reordered by ascending chunk ID (IDs are assigned in append
  *      order), padding last.
  *
+ *  Deletion (JointCompact's deletions D applied to the chunk table,
+ *      Algorithm 1; invalidated copies are logically tombstoned, §4.2): a
+ *      deleted chunk is no longer part of the store's memory: it gets no
+ *      score (u = 0, so it adds nothing to Z or to propagation) and is never
+ *      selected; every relation edge into or out of it is dropped and the
+ *      weights of the rows that lost edges are the row softmax of what
+ *      remains.
+ *
  * Readings where the paper is silent (also recorded in the design notes):
  *   - temperature tau defaults to 1/sqrt(dim) for every store;
  *   - multi-hop form s^(h) = u + alpha * s^(h-1) R (truncated personalised
@@ -143,8 +151,9 @@ static int retrieve_impl(const uint16_t *emb, int64_t n, int32_t dim, const uint
                          int32_t n_q, const int64_t *row_ptr, const int32_t *col, const double *w,
                          double tau, double alpha, int32_t hops, int32_t k,
                          const int32_t *page_of, const int32_t *ns_of, const int32_t *q_ns,
-                         int32_t sort_by_time, int64_t *ids, double *scores, int32_t *page_ids,
-                         int32_t *n_pages, double *final_out, double *z_out, double *shift_out);
+                         const uint8_t *dead, int32_t sort_by_time, int64_t *ids, double *scores,
+                         int32_t *page_ids, int32_t *n_pages, double *final_out, double *z_out,
+                         double *shift_out);
 
 int ora_retrieve(const uint16_t *emb, int64_t n, int32_t dim, const uint16_t *q, int32_t n_q,
                  const int64_t *row_ptr, const int32_t *col, const double *w, double tau,
@@ -153,28 +162,55 @@ int ora_retrieve(const uint16_t *emb, int64_t n, int32_t dim, const uint16_t *q,
                  double *z_out, double *shift_out)
 {
     return retrieve_impl(emb, n, dim, q, n_q, row_ptr, col, w, tau, alpha, hops, k, page_of,
-                         NULL, NULL, 0, ids, scores, page_ids, n_pages, final_out, z_out,
+                         NULL, NULL, NULL, 0, ids, scores, page_ids, n_pages, final_out, z_out,
                          shift_out);
 }
 
 /*
  * As ora_retrieve, with query b selecting only among the chunks whose
- * ns_of[i] equals q_ns[b] (ns_of[n], q_ns[n_q]), padded with ID -1 when
- * fewer than k exist, and with sort_by_time != 0 returning the selected IDs
- * in ascending ID order.
+ * ns_of[i] equals q_ns[b] (ns_of[n], q_ns[n_q]; both NULL: no scope), and
+ * none of the chunks with dead[i] != 0 (dead[n] or NULL), padded with ID -1
+ * when fewer than k remain, and with sort_by_time != 0 returning the
+ * selected IDs in ascending ID order.
  */
 int ora_retrieve_scoped(const uint16_t *emb, int64_t n, int32_t dim, const uint16_t *q,
                         int32_t n_q, const int64_t *row_ptr, const int32_t *col, const double *w,
                         double tau, double alpha, int32_t hops, int32_t k,
                         const int32_t *page_of, const int32_t *ns_of, const int32_t *q_ns,
-                        int32_t sort_by_time, int64_t *ids, double *scores, int32_t *page_ids,
-                        int32_t *n_pages, double *final_out)
+                        const uint8_t *dead, int32_t sort_by_time, int64_t *ids, double *scores,
+                        int32_t *page_ids, int32_t *n_pages, double *final_out)
 {
-    if (!ns_of || !q_ns)
+    if ((ns_of == NULL) != (q_ns == NULL))
         return ORA_EINVAL;
     return retrieve_impl(emb, n, dim, q, n_q, row_ptr, col, w, tau, alpha, hops, k, page_of,
-                         ns_of, q_ns, sort_by_time, ids, scores, page_ids, n_pages, final_out,
-                         NULL, NULL);
+                         ns_of, q_ns, dead, sort_by_time, ids, scores, page_ids, n_pages,
+                         final_out, NULL, NULL);
+}
+
+/*
+ * Deletion of chunks from the relation graph: the CSR without every edge
+ * i -> j where dead[i] or dead[j].  new_row_ptr[n+1]; new_col / new_aff with
+ * room for nnz entries.  (The weights are then ora_row_softmax of the new
+ * logits.)
+ */
+int ora_drop_dead(int64_t n, const int64_t *row_ptr, const int32_t *col, const float *aff,
+                  const uint8_t *dead, int64_t *new_row_ptr, int32_t *new_col, float *new_aff)
+{
+    if (n < 0 || !row_ptr || !dead || !new_row_ptr)
+        return ORA_EINVAL;
+    int64_t o = 0;
+    new_row_ptr[0] = 0;
+    for (int64_t i = 0; i < n; ++i) {
+        for (int64_t e = row_ptr[i]; e < row_ptr[i + 1]; ++e) {
+            if (dead[i] || dead[col[e]])
+                continue;
+            new_col[o] = col[e];
+            new_aff[o] = aff[e];
+            ++o;
+        }
+        new_row_ptr[i + 1] = o;
+    }
+    return ORA_OK;
 }
 
 /* selected entries of one query by ascending ID (padding -1 stays last) */
@@ -188,8 +224,9 @@ static int retrieve_impl(const uint16_t *emb, int64_t n, int32_t dim, const uint
                          int32_t n_q, const int64_t *row_ptr, const int32_t *col, const double *w,
                          double tau, double alpha, int32_t hops, int32_t k,
                          const int32_t *page_of, const int32_t *ns_of, const int32_t *q_ns,
-                         int32_t sort_by_time, int64_t *ids, double *scores, int32_t *page_ids,
-                         int32_t *n_pages, double *final_out, double *z_out, double *shift_out)
+                         const uint8_t *dead, int32_t sort_by_time, int64_t *ids, double *scores,
+                         int32_t *page_ids, int32_t *n_pages, double *final_out, double *z_out,
+                         double *shift_out)
 {
     if (n < 1 || dim < 1 || n_q < 0 || k < 1 || k > n || hops < 0 || alpha < 0.0)
         return ORA_EINVAL;
@@ -222,7 +259,7 @@ static int retrieve_impl(const uint16_t *emb, int64_t n, int32_t dim, const uint
         }
         double zsum = 0.0;
         for (int64_t i = 0; i < n; ++i) {
-            u[i] = exp(z[i] - cmax);
+            u[i] = (dead && dead[i]) ? 0.0 : exp(z[i] - cmax);   /* deleted: no score */
             zsum += u[i];
         }
         /* propagate: scatter over out-edges */
@@ -242,6 +279,8 @@ static int retrieve_impl(const uint16_t *emb, int64_t n, int32_t dim, const uint
             s[i] /= zsum;
             if (ns_of && ns_of[i] != q_ns[b])
                 continue;   /* outside the query's namespace: not a candidate */
+            if (dead && dead[i])
+                continue;   /* deleted: not a candidate */
             order[n_cand].key = s[i];
             order[n_cand].id = i;
             ++n_cand;

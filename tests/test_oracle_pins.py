@@ -477,3 +477,43 @@ def test_sort_by_time_reorders_only():
         assert list(tm["ids"][b]) == sorted(base["ids"][b].tolist())
         sc = dict(zip(base["ids"][b].tolist(), base["scores"][b].tolist()))
         assert [sc[i] for i in tm["ids"][b]] == tm["scores"][b].tolist()
+
+
+# --------------------------------------------------------------------------- deletion
+def test_drop_dead_is_edge_filter():
+    """Deleting chunks drops exactly the edges into or out of them (numpy
+    filter over the edge list), rows keep their column order."""
+    emb, q, row_ptr, col, aff = tiny_store(31, 90, 8, 6)
+    dead = np.zeros(90, bool)
+    dead[[3, 17, 40, 41, 89]] = True
+    rp, c, a = oracle.drop_dead(row_ptr, col, aff, dead)
+    src = np.repeat(np.arange(90), np.diff(row_ptr))
+    keep = ~dead[src] & ~dead[col]
+    assert (np.diff(rp) == np.bincount(src[keep], minlength=90)).all()
+    assert (c == col[keep]).all() and (a == aff[keep]).all()
+
+
+@pytest.mark.parametrize("hops", [0, 2])
+def test_deleted_chunks_equal_removed_store(hops):
+    """A store with tombstoned chunks retrieves exactly like the store
+    rebuilt without them (rows removed, graph re-indexed, weights re-softmaxed):
+    same IDs (mapped back), same scores.  Catches a deleted chunk still
+    counted in Z, still propagating mass, or still selectable."""
+    n, k = 140, 8
+    emb, q, row_ptr, col, aff = tiny_store(32, n, 16, 6, n_q=3)
+    rng = np.random.default_rng(9)
+    dead = np.zeros(n, bool)
+    dead[rng.choice(n, 25, replace=False)] = True
+    rp, c, a = oracle.drop_dead(row_ptr, col, aff, dead)
+    w = oracle.row_softmax(rp, a)
+    out = oracle.retrieve(emb, q, rp, c, w, tau=0.3, alpha=0.5, hops=hops, k=k, dead=dead)
+    live = np.nonzero(~dead)[0]
+    new_id = -np.ones(n, np.int64)
+    new_id[live] = np.arange(live.size)
+    src = np.repeat(np.arange(n), np.diff(rp))
+    rp2 = np.concatenate([[0], np.cumsum(np.bincount(new_id[src], minlength=live.size))])
+    c2 = new_id[c].astype(np.int32)
+    w2 = oracle.row_softmax(rp2, a)
+    ref = oracle.retrieve(emb[live], q, rp2, c2, w2, tau=0.3, alpha=0.5, hops=hops, k=k)
+    assert (out["ids"] == live[ref["ids"]]).all()
+    assert np.allclose(out["scores"], ref["scores"], rtol=1e-12)
