@@ -148,6 +148,20 @@ akashic_status_t akashic_mem_retrieve(akashic_mem_t *m, const uint16_t *q, int32
 akashic_status_t akashic_mem_set_namespace(akashic_mem_t *m, int64_t first, int64_t n,
                                            const int32_t *ns, void *stream);
 
+/* Delete chunks (the deletions of cross-chunk compaction, Algorithm 1
+ * JointCompact / "Apply updates U and deletions D"; stale copies are
+ * logically tombstoned, §4.2).  ids: device int64[n] chunk IDs.  A deleted
+ * chunk keeps its ID and row but gets no score (it adds nothing to Z or to
+ * propagation), is never selected by retrieval and never chosen by a
+ * relation update; every relation edge into or out of it is dropped and the
+ * rows that lost edges are re-softmaxed; the in-edge transpose and the hub
+ * plan are compacted to match.  Deleting a chunk twice is harmless.  A later
+ * append may not pass edges that point at a deleted chunk (EDEVICE).
+ * EINVAL if n < 0, ids is NULL with n > 0, or any ID lies outside
+ * [0, size) (then nothing changes).  Synchronises `stream`. */
+akashic_status_t akashic_mem_delete(akashic_mem_t *m, const int64_t *ids, int64_t n,
+                                    void *stream);
+
 /* Retrieval scoped to the caller's namespace, with optional chronological
  * order (§4.1: candidates are the chunks of the current user_id/session_id;
  * Algorithm 1 lines SortByTime: the selected chunks are returned in time

@@ -29,7 +29,7 @@ EXPORTS = (
     "akashic_mem_update_relations", "akashic_mem_retrieve", "akashic_mem_export_csr",
     "akashic_mem_size", "akashic_mem_sync", "akashic_mem_set_profiling",
     "akashic_mem_phase_times", "akashic_mem_last_error", "akashic_mem_softmax_scores_noalloc",
-    "akashic_mem_set_namespace", "akashic_mem_retrieve_scoped",
+    "akashic_mem_set_namespace", "akashic_mem_retrieve_scoped", "akashic_mem_delete",
 )
 
 
@@ -70,6 +70,7 @@ def load_library(path: str | None = None):
         "akashic_mem_retrieve_scoped": ([V, V, I32, I32, F, I32, V, I32, V, V, V, V, V],
                                         ctypes.c_int),
         "akashic_mem_set_namespace": ([V, I64, I64, V, V], ctypes.c_int),
+        "akashic_mem_delete": ([V, V, I64, V], ctypes.c_int),
         "akashic_mem_export_csr": ([V, P64, P64, V, V, V, V, V], ctypes.c_int),
         "akashic_mem_size": ([V, P64, P64], ctypes.c_int),
         "akashic_mem_sync": ([V, V], ctypes.c_int),
@@ -203,6 +204,13 @@ class MemStore:
     def update_relations(self, first: int, n: int, M: int, reciprocal: bool = True, stream=None):
         _check(load_library().akashic_mem_update_relations(
             self._h, first, n, M, int(bool(reciprocal)), _stream(self._torch, stream, self.device)))
+
+    def delete(self, ids, stream=None):
+        """Delete chunks (int64 device tensor of chunk IDs)."""
+        torch = self._torch
+        self._dev(ids, torch.int64, "ids")
+        _check(load_library().akashic_mem_delete(self._h, _ptr(ids), ids.numel(),
+                                                 _stream(torch, stream, self.device)))
 
     def set_namespace(self, first: int, ns, stream=None):
         """Tags of chunk IDs [first, first+len(ns)) (int32 device tensor)."""

@@ -82,7 +82,7 @@ struct DevBuf {
 struct StreamScratch {
     DevBuf qp, shift, u, sa, sb, zpart, partial, cand, counters;
     DevBuf samp, ext_s, zsamp;   // retrieval without hops: the score's row sample
-    DevBuf qns, ns_s;            // namespace scope: per query column, per sample row
+    DevBuf qns, ns_s, dead_s;    // scope: per query column, per sample row
 };
 
 struct ProfRec {
@@ -116,6 +116,8 @@ struct akashic_mem {
     // is in row row_of[c]; page_of is indexed by row
     DevBuf emb, page_of, ext_of, row_of, max_norm, status;
     DevBuf ns_row;               // namespace tag of the chunk in each row (0 by default)
+    DevBuf dead_row;             // 1 in the rows of deleted chunks
+    bool has_dead = false;       // any chunk deleted (enables the masks)
     // canonical out-edge CSR
     int64_t nnz = 0;
     DevBuf row_ptr, col, aff, w;
@@ -218,8 +220,6 @@ static akashic_status_t check_status(akashic_mem *m, cudaStream_t st, const char
     return AKASHIC_OK;
 }
 
-// Rebuild the in-edge transpose (stable by source, hence sorted by source
-// within each destination), its weights, and the split plan of long rows.
 // Grow-only scratch of a store (UpdateArgs::scratch): 1/8 headroom when a
 // slot has to grow, so slowly growing sizes do not reallocate every call.
 static void *store_scratch(void *ctx, int slot, size_t bytes) {
@@ -244,6 +244,8 @@ static akashic_status_t ensure_spare(DevBuf &b, size_t bytes) {
 
 static akashic_status_t build_split_plan(akashic_mem *m, cudaStream_t st);
 
+// Rebuild the in-edge transpose (stable by source, hence sorted by source
+// within each destination), its weights, and the split plan of long rows.
 static akashic_status_t rebuild_in_edges(akashic_mem *m, cudaStream_t st) {
     const int64_t n = m->n, nnz = m->nnz;
     AK_TRY(m->in_ptr.ensure((size_t)(m->cap + 1) * sizeof(int64_t)));
@@ -405,6 +407,7 @@ akashic_status_t akashic_mem_create(const akashic_mem_config_t *cfg, akashic_mem
         (s = m->max_norm.ensure(4)) != AKASHIC_OK || (s = m->status.ensure(4)) != AKASHIC_OK ||
         (s = m->rstat.ensure((size_t)m->cap * 8)) != AKASHIC_OK ||
         (s = m->ns_row.ensure((size_t)m->cap * 4)) != AKASHIC_OK ||
+        (s = m->dead_row.ensure((size_t)m->cap * 4)) != AKASHIC_OK ||
         (s = m->row_ptr.ensure((size_t)(m->cap + 1) * 8)) != AKASHIC_OK ||
         (s = m->in_ptr.ensure((size_t)(m->cap + 1) * 8)) != AKASHIC_OK) {
         delete m;
@@ -413,6 +416,7 @@ akashic_status_t akashic_mem_create(const akashic_mem_config_t *cfg, akashic_mem
     if (cudaMemset(m->max_norm.p, 0, 4) != cudaSuccess || cudaMemset(m->status.p, 0, 4) != cudaSuccess ||
         cudaMemset(m->row_ptr.p, 0, 8) != cudaSuccess || cudaMemset(m->in_ptr.p, 0, 8) != cudaSuccess ||
         cudaMemset(m->ns_row.p, 0, (size_t)m->cap * 4) != cudaSuccess ||
+        cudaMemset(m->dead_row.p, 0, (size_t)m->cap * 4) != cudaSuccess ||
         cudaDeviceSynchronize() != cudaSuccess) {
         delete m;
         return fail(AKASHIC_ECUDA, "create: initialisation failed");
@@ -470,6 +474,12 @@ akashic_status_t akashic_mem_append_chunks(akashic_mem_t *m, const uint16_t *emb
                                        m->status.as<int>(), st));
         AK_TRY(check_status(m, st, "append: edge check"));
         if (e_hi < e_lo) return fail(AKASHIC_EINVAL, "append: row_ptr decreases");
+        if (m->has_dead && e_hi > e_lo && col) {
+            CUDA_TRY(launch_check_dead_targets(col + e_lo, e_hi - e_lo, first,
+                                               m->row_of.as<int32_t>(), m->dead_row.as<int32_t>(),
+                                               m->status.as<int>(), st));
+            AK_TRY(check_status(m, st, "append: an edge points at a deleted chunk"));
+        }
         if (e_hi > e_lo && !(col && aff))
             return fail(AKASHIC_EINVAL, "append: edges given without col or aff");
         if (m->nnz + (e_hi - e_lo) > 0x7fffffffLL)
@@ -585,6 +595,7 @@ akashic_status_t akashic_mem_update_relations(akashic_mem_t *m, int64_t first, i
         return fail(AKASHIC_ECAPACITY, "update: more than 2^31-1 relation edges");
     ua.scratch = store_scratch;
     ua.scratch_ctx = m;
+    ua.dead_row = m->has_dead ? m->dead_row.as<int32_t>() : nullptr;
     ua.nbr_ids = (int32_t *)store_scratch(m, SCR_NBR_IDS, (size_t)n * M * 4);
     ua.nbr_cos = (float *)store_scratch(m, SCR_NBR_COS, (size_t)n * M * 4);
     if (!ua.nbr_ids || !ua.nbr_cos) return fail(AKASHIC_ENOMEM, "update: out of device memory");
@@ -724,6 +735,75 @@ akashic_status_t akashic_mem_set_namespace(akashic_mem_t *m, int64_t first, int6
                                    (cudaStream_t)stream));
     return AKASHIC_OK;
 }
+akashic_status_t akashic_mem_delete(akashic_mem_t *m, const int64_t *ids, int64_t n,
+                                    void *stream) {
+    g_last_error.clear();
+    if (!m) return fail(AKASHIC_EINVAL, "delete: NULL store");
+    if (n < 0) return fail(AKASHIC_EINVAL, "delete: n < 0");
+    if (n == 0) return AKASHIC_OK;
+    if (!ids) return fail(AKASHIC_EINVAL, "delete: NULL ids");
+    DeviceGuard g(m->device);
+    cudaStream_t st = (cudaStream_t)stream;
+    // check every ID first, so that a bad list changes nothing
+    CUDA_TRY(launch_mark_dead(ids, n, m->n, m->row_of.as<int32_t>(), nullptr,
+                              m->status.as<int>(), st));
+    AK_TRY(check_status(m, st, "delete: chunk IDs must lie in [0, size)"));
+    CUDA_TRY(launch_mark_dead(ids, n, m->n, m->row_of.as<int32_t>(), m->dead_row.as<int32_t>(),
+                              m->status.as<int>(), st));
+    m->has_dead = true;
+    const int64_t rows = m->n, nnz = m->nnz;
+    if (nnz == 0) return AKASHIC_OK;
+    const size_t tb = scan_tmp_bytes(nnz + 1) + 4096;
+    int64_t *keep = (int64_t *)store_scratch(m, SCR_DEL_KEEP, (size_t)(nnz + 1) * 8);
+    int64_t *pos = (int64_t *)store_scratch(m, SCR_DEL_POS, (size_t)(nnz + 1) * 8);
+    void *tmp = store_scratch(m, SCR_DEL_TMP, tb);
+    if (!keep || !pos || !tmp) return fail(AKASHIC_ENOMEM, "delete: out of device memory");
+    // out-edge CSR (rows are chunk IDs, targets chunk IDs)
+    AK_TRY(ensure_spare(m->rp2, (size_t)(m->cap + 1) * 8));
+    AK_TRY(ensure_spare(m->col2, (size_t)nnz * 4));
+    AK_TRY(ensure_spare(m->aff2, (size_t)nnz * 4));
+    DropDead d{rows, nnz, m->row_ptr.as<int64_t>(), m->col.as<int32_t>(), m->aff.as<float>(),
+               m->row_of.as<int32_t>(), m->dead_row.as<int32_t>(), ids, n, rows, nullptr,
+               keep, pos, tmp, tb, m->rp2.as<int64_t>(), m->col2.as<int32_t>(),
+               m->aff2.as<float>()};
+    CUDA_TRY(launch_drop_dead_edges(d, st));
+    int64_t nnz_new = 0;
+    CUDA_TRY(cudaMemcpyAsync(&nnz_new, pos + nnz, 8, cudaMemcpyDeviceToHost, st));
+    CUDA_TRY(cudaStreamSynchronize(st));
+    std::swap(m->row_ptr.p, m->rp2.p);
+    std::swap(m->row_ptr.cap, m->rp2.cap);
+    std::swap(m->col.p, m->col2.p);
+    std::swap(m->col.cap, m->col2.cap);
+    std::swap(m->aff.p, m->aff2.p);
+    std::swap(m->aff.cap, m->aff2.cap);
+    m->nnz = nnz_new;
+    AK_TRY(m->w.ensure(m->col.cap > 4 ? m->col.cap : 4, false));
+    CUDA_TRY(launch_row_softmax(m->row_ptr.as<int64_t>(), m->aff.as<float>(), m->w.as<float>(),
+                                rows, m->rstat.as<float2>(), st));
+    // in-edge transpose (rows are store rows, sources rows); the same edges go
+    AK_TRY(ensure_spare(m->in_ptr2, (size_t)(m->cap + 1) * 8));
+    AK_TRY(ensure_spare(m->in_src2, (size_t)nnz * 4));
+    AK_TRY(ensure_spare(m->in_aff2, (size_t)nnz * 4));
+    AK_TRY(ensure_spare(m->in_w2, (size_t)nnz * 4));
+    DropDead di{rows, nnz, m->in_ptr.as<int64_t>(), m->in_src.as<int32_t>(), m->in_aff.as<float>(),
+                nullptr, m->dead_row.as<int32_t>(), ids, n, rows, m->row_of.as<int32_t>(),
+                keep, pos, tmp, tb, m->in_ptr2.as<int64_t>(), m->in_src2.as<int32_t>(),
+                m->in_aff2.as<float>()};
+    CUDA_TRY(launch_drop_dead_edges(di, st));
+    CUDA_TRY(launch_in_weights(m->in_src2.as<int32_t>(), m->in_aff2.as<float>(), nnz_new,
+                               m->ext_of.as<int32_t>(), m->rstat.as<float2>(),
+                               m->in_w2.as<float>(), st));
+    std::swap(m->in_ptr.p, m->in_ptr2.p);
+    std::swap(m->in_ptr.cap, m->in_ptr2.cap);
+    std::swap(m->in_src.p, m->in_src2.p);
+    std::swap(m->in_src.cap, m->in_src2.cap);
+    std::swap(m->in_aff.p, m->in_aff2.p);
+    std::swap(m->in_aff.cap, m->in_aff2.cap);
+    std::swap(m->in_w.p, m->in_w2.p);
+    std::swap(m->in_w.cap, m->in_w2.cap);
+    AK_TRY(build_split_plan(m, st));
+    return check_status(m, st, "delete");
+}
 }  // extern "C"
 
 static akashic_status_t retrieve_impl(akashic_mem *m, const uint16_t *q, int32_t B, int32_t k,
@@ -768,8 +848,9 @@ static akashic_status_t retrieve_impl(akashic_mem *m, const uint16_t *q, int32_t
             CUDA_TRY(cudaMemsetAsync(sc->qns.p, 0xff, (size_t)bp * 4, st));
             CUDA_TRY(cudaMemcpyAsync(sc->qns.p, q_ns + off, (size_t)b * 4,
                                      cudaMemcpyDeviceToDevice, st));
-            ns = NsScope{m->ns_row.as<int32_t>(), sc->qns.as<int32_t>()};
+            ns = NsScope{m->ns_row.as<int32_t>(), sc->qns.as<int32_t>(), nullptr};
         }
+        if (m->has_dead) ns.dead = m->dead_row.as<int32_t>();
         // Without hops the top-k filter is fused into the score GEMM, which
         // then writes no slab: the bound comes from the score of every
         // stride-th row, computed first by the same kernel (same values).
@@ -788,7 +869,7 @@ static akashic_status_t retrieve_impl(akashic_mem *m, const uint16_t *q, int32_t
                 CUDA_TRY(launch_score(m->emb.as<uint16_t>(), n, m->dim, sc->qp.as<uint16_t>(), bp,
                                       sc->shift.as<float>(), m->tau, sc->u.as<float>(),
                                       sc->zpart.as<float>(), m->status.as<int>(), st,
-                                      &ph.launches, &zrows));
+                                      &ph.launches, &zrows, ns.dead));
         }
         if (dense_fused) {
             {
@@ -803,7 +884,13 @@ static akashic_status_t retrieve_impl(akashic_mem *m, const uint16_t *q, int32_t
                     AK_TRY(sc->ns_s.ensure((size_t)sp.n_sample * 4));
                     CUDA_TRY(launch_ext_sample(m->ns_row.as<int32_t>(), sp.n_sample, sp.stride,
                                                sc->ns_s.as<int32_t>(), st));
-                    ns_samp = NsScope{sc->ns_s.as<int32_t>(), sc->qns.as<int32_t>()};
+                    ns_samp = NsScope{sc->ns_s.as<int32_t>(), sc->qns.as<int32_t>(), nullptr};
+                }
+                if (m->has_dead) {
+                    AK_TRY(sc->dead_s.ensure((size_t)sp.n_sample * 4));
+                    CUDA_TRY(launch_ext_sample(m->dead_row.as<int32_t>(), sp.n_sample, sp.stride,
+                                               sc->dead_s.as<int32_t>(), st));
+                    ns_samp.dead = sc->dead_s.as<int32_t>();
                 }
                 CUDA_TRY(launch_score_sample(m->emb.as<uint16_t>(), sp.n_sample, sp.stride, m->dim,
                                              sc->qp.as<uint16_t>(), bp, sc->shift.as<float>(),

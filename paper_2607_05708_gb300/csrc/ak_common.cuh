@@ -37,15 +37,21 @@ __device__ __forceinline__ uint32_t key_id(unsigned long long key) {
     return ~(uint32_t)(key & 0xffffffffull);
 }
 
-// Namespace scope of a retrieval (§4.1: the candidates of a query are the
-// chunks of the caller's (user_id, session_id) table): row j is a candidate
-// for query column c iff ns_row[j] == q_ns[c].  q_ns == NULL: no scope.
+// Candidate scope of a selection.  Namespaces (§4.1: the candidates of a
+// query are the chunks of the caller's (user_id, session_id) table): row j
+// is a candidate for query column c only if ns_row[j] == q_ns[c]
+// (q_ns == NULL: no namespace scope).  Deletions (tombstones): a row with
+// dead[j] != 0 is never a candidate (dead == NULL: none deleted).
 struct NsScope {
     const int32_t *ns_row;   // [rows] tag of the chunk in each row (or sample row)
     const int32_t *q_ns;     // [bp] tag of each query column
+    const int32_t *dead;     // [rows] 1 where the chunk was deleted
 };
 __device__ __forceinline__ bool in_scope(const NsScope &s, int64_t row, int col) {
-    return !s.q_ns || s.ns_row[row] == s.q_ns[col];
+    return (!s.dead || !s.dead[row]) && (!s.q_ns || s.ns_row[row] == s.q_ns[col]);
+}
+__host__ __device__ __forceinline__ bool scope_active(const NsScope &s) {
+    return s.q_ns != nullptr || s.dead != nullptr;
 }
 
 // Keys for signed cosine values: order-preserving map of any finite fp32 to
@@ -70,9 +76,11 @@ void set_last_error(const char *msg);
 // stride bp; zpart[r, c] = sum of u over the rows handled by score CTA r,
 // for r < *zrows.  score_tiles(n) bounds *zrows.
 int64_t score_tiles(int64_t n);
+// dead_row (or NULL): rows of deleted chunks score u = 0 (no part in Z).
 cudaError_t launch_score(const uint16_t *emb, int64_t n, int dim, const uint16_t *qp, int bp,
                          const float *shift, float tau, float *u, float *zpart, int *status,
-                         cudaStream_t st, int *launches, int *zrows);
+                         cudaStream_t st, int *launches, int *zrows,
+                         const int32_t *dead_row = nullptr);
 
 // The score on every stride-th row only: out[v, c] = u[v*stride, c] for
 // v < n_sample (same kernel and arithmetic as launch_score, so the values
@@ -106,7 +114,8 @@ cudaError_t launch_dots_filter(const uint16_t *emb, int64_t n, int dim, const ui
                                int n_ctiles, int64_t n_cols, const int32_t *ext_of,
                                int64_t id_limit, const unsigned long long *bound,
                                unsigned int *cnt, unsigned long long *buf, int64_t cap,
-                               int *status, cudaStream_t st, int *launches);
+                               int *status, cudaStream_t st, int *launches,
+                               const int32_t *dead_row = nullptr);
 
 // Query preparation: pad q (b rows) to bp rows of zeros and compute
 // shift[c] = tau * |q_c| * max_norm (0 for padding); flags ERANGE.
@@ -228,6 +237,38 @@ cudaError_t launch_seg_permute(const uint32_t *order, const int64_t *e0, const i
 cudaError_t launch_split_keys(const int64_t *slot0, int64_t n_split, uint32_t *keys,
                               uint32_t *vals, cudaStream_t st);
 
+// Chunk deletion (ak_delete.cu).  dead_row[row_of[id]] = 1 for the listed
+// IDs (out-of-range IDs set EINVAL in *status and are skipped; dead_row
+// NULL: check only).
+cudaError_t launch_mark_dead(const int64_t *ids, int64_t n, int64_t n_total, const int32_t *row_of,
+                             int32_t *dead_row, int *status, cudaStream_t st);
+// EDEVICE in *status if any col[e] < first names a deleted chunk.
+cudaError_t launch_check_dead_targets(const int32_t *col, int64_t nnz, int64_t first,
+                                      const int32_t *row_of, const int32_t *dead_row, int *status,
+                                      cudaStream_t st);
+// One CSR without the edges that touch a dead row: an edge survives if its
+// target (tgt[e], mapped through tgt_row_of unless NULL) is not dead and it
+// is not in the row of a listed ID (rows found through own_row_of unless
+// NULL).  Survivors keep their order; ptr_out[r] = new start of row r.
+struct DropDead {
+    int64_t n_rows, nnz;
+    const int64_t *ptr;                 // [n_rows+1]
+    const int32_t *tgt;                 // [nnz]
+    const float *val;                   // [nnz] carried along (logits)
+    const int32_t *tgt_row_of;          // chunk ID -> row for targets, or NULL (targets are rows)
+    const int32_t *dead_row;            // [rows]
+    const int64_t *ids;                 // [n_ids] deleted chunk IDs
+    int64_t n_ids, n_total;
+    const int32_t *own_row_of;          // chunk ID -> row of the CSR, or NULL (CSR rows are IDs)
+    int64_t *keep, *pos;                // scratch [nnz+1] each
+    void *tmp;                          // scan scratch
+    size_t tmp_bytes;
+    int64_t *ptr_out;                   // [n_rows+1]
+    int32_t *tgt_out;                   // [nnz]
+    float *val_out;                     // [nnz]
+};
+cudaError_t launch_drop_dead_edges(const DropDead &d, cudaStream_t st);
+
 // Propagation hop (a2): out[j,:] = u[j,:] + alpha * sum_{i->j} w_ij * in[i,:].
 struct HopPlan {
     SplitParams split;
@@ -296,7 +337,7 @@ cudaError_t launch_select(const SelectPlan &sp, const float *s, int b, unsigned 
 cudaError_t launch_select_signed(const SelectPlan &sp, const float *s, int b,
                                  unsigned long long *ws, const int32_t *ext_of, int64_t id_limit,
                                  int64_t c_base, int32_t *nbr_ids, float *nbr_cos, int *status,
-                                 cudaStream_t st, int *launches);
+                                 cudaStream_t st, int *launches, NsScope ns = NsScope{});
 // Bound pass alone over signed values: bound[c] for the b real columns
 // (the k-th largest sampled key; padding columns get an all-ones bound).
 // Bound only, unsigned keys (retrieval): ws + sp.off_bound gets the bound,
@@ -340,7 +381,7 @@ cudaError_t launch_topk_merge(const SelectPlan &sp, const float *s, int b,
 cudaError_t launch_sample_bound_signed(const SelectPlan &sp, const float *s, int b,
                                        const int32_t *ext_of, int64_t id_limit,
                                        unsigned long long *ws, unsigned long long *bound,
-                                       cudaStream_t st, int *launches);
+                                       cudaStream_t st, int *launches, NsScope ns = NsScope{});
 // Top-k of each column's filter buffer (no overflow): nbr rows 0..n_cols-1.
 cudaError_t launch_buf_merge_signed(const unsigned int *cnt, const unsigned long long *buf,
                                     int64_t cap, int64_t n_cols, int k, int32_t *nbr_ids,

@@ -141,6 +141,8 @@ struct GemmEpi {
     unsigned long long *buf;            // FILTER: [n_cols][cap]
     int64_t cap;
     NsScope ns;                         // EXP_FILTER: namespace scope of the queries
+    const int32_t *dead_row;            // EXP, EXP_FILTER, FILTER: deleted rows (or NULL):
+                                        // no score (u = 0) / never a filter candidate
 };
 
 template <int BP, int MODE>
@@ -328,7 +330,9 @@ __global__ __launch_bounds__(GemmCfg<BP, MODE>::THREADS, 1) void k_gemm_umma(con
             if (!*go) break;
             tc_fence_after();
             const int64_t grow = mt * C::BM + row;
-            const bool valid = grow < n_rows;
+            const bool in_rows = grow < n_rows;
+            const bool valid =
+                in_rows && (MODE == GEMM_RAW || !ep.dead_row || !ep.dead_row[grow]);
             uint32_t fid = 0;
             bool fok = false;
             if ((FILTER || EXPF) && valid) {
@@ -507,8 +511,9 @@ static cudaError_t gemm_dispatch(const uint16_t *emb, int64_t n_rows, int64_t ro
 
 cudaError_t launch_score(const uint16_t *emb, int64_t n, int dim, const uint16_t *qp, int bp,
                          const float *shift, float tau, float *u, float *zpart, int *status,
-                         cudaStream_t st, int *launches, int *zrows) {
+                         cudaStream_t st, int *launches, int *zrows, const int32_t *dead_row) {
     GemmEpi ep{};
+    ep.dead_row = dead_row;
     ep.shift = shift;
     ep.tau = tau;
     ep.zpart = zpart;
@@ -541,6 +546,7 @@ cudaError_t launch_score_filter(const uint16_t *emb, int64_t n, int dim, const u
                                 cudaStream_t st, int *launches, int *zrows) {
     GemmEpi ep{};
     ep.ns = ns;
+    ep.dead_row = ns.dead;
     ep.shift = shift;
     ep.tau = tau;
     ep.zpart = zpart;
@@ -573,8 +579,10 @@ cudaError_t launch_dots_filter(const uint16_t *emb, int64_t n, int dim, const ui
                                int n_ctiles, int64_t n_cols, const int32_t *ext_of,
                                int64_t id_limit, const unsigned long long *bound,
                                unsigned int *cnt, unsigned long long *buf, int64_t cap,
-                               int *status, cudaStream_t st, int *launches) {
+                               int *status, cudaStream_t st, int *launches,
+                               const int32_t *dead_row) {
     GemmEpi ep{};
+    ep.dead_row = dead_row;
     ep.status = status;
     ep.n_cols = n_cols;
     ep.ext_of = ext_of;

@@ -438,7 +438,8 @@ __global__ __launch_bounds__(SEL_THREADS) void k_topk_merge(
                       hist, &s_prefix, &s_remaining, ns);
     // without a scope every query has k winners; with one, a namespace
     // holding fewer than k chunks pads its list
-    if (tid == 0 && (win_n > k || (!ns.q_ns && win_n != k))) set_status(status, AKASHIC_EDEVICE);
+    if (tid == 0 && (win_n > k || (!scope_active(ns) && win_n != k)))
+        set_status(status, AKASHIC_EDEVICE);
     const int got = win_n < k ? win_n : k;
     if (tid < got) {
         const unsigned long long key = win[tid];
@@ -480,7 +481,7 @@ __global__ __launch_bounds__(SEL_THREADS) void k_topm_merge(
     const float *__restrict__ s, int64_t n, int bp, int k, const int32_t *__restrict__ ext_of,
     int64_t id_limit, const unsigned int *__restrict__ cnt,
     const unsigned long long *__restrict__ buf, int64_t cap, int64_t c_base,
-    int32_t *__restrict__ nbr_ids, float *__restrict__ nbr_cos, int *status) {
+    int32_t *__restrict__ nbr_ids, float *__restrict__ nbr_cos, int *status, const NsScope ns) {
     __shared__ int hist[256 * (SEL_THREADS / 32)];
     __shared__ unsigned long long stage[SEL_STAGE];
     __shared__ unsigned long long win[64];
@@ -489,7 +490,7 @@ __global__ __launch_bounds__(SEL_THREADS) void k_topm_merge(
     const int c = blockIdx.x;
     const int tid = threadIdx.x;
     column_top<true>(s, n, bp, k, c, ext_of, id_limit, cnt, buf, cap, stage, win, &win_n, hist,
-                     &s_prefix, &s_remaining);
+                     &s_prefix, &s_remaining, ns);
     if (tid == 0 && win_n != k) set_status(status, AKASHIC_EDEVICE);
     const int got = win_n < k ? win_n : k;
     if (tid < got) {
@@ -615,8 +616,8 @@ static cudaError_t sample_bound(const SelectPlan &sp, const float *s, int b,
 cudaError_t launch_sample_bound_signed(const SelectPlan &sp, const float *s, int b,
                                        const int32_t *ext_of, int64_t id_limit,
                                        unsigned long long *ws, unsigned long long *bound,
-                                       cudaStream_t st, int *launches) {
-    return sample_bound<true>(sp, s, b, ext_of, id_limit, ws, bound, st, launches);
+                                       cudaStream_t st, int *launches, NsScope ns) {
+    return sample_bound<true>(sp, s, b, ext_of, id_limit, ws, bound, st, launches, 0, ns);
 }
 
 cudaError_t launch_sample_bound(const SelectPlan &sp, const float *s, int b,
@@ -659,13 +660,13 @@ cudaError_t launch_topk_merge(const SelectPlan &sp, const float *s, int b,
 cudaError_t launch_select_signed(const SelectPlan &sp, const float *s, int b,
                                  unsigned long long *ws, const int32_t *ext_of, int64_t id_limit,
                                  int64_t c_base, int32_t *nbr_ids, float *nbr_cos, int *status,
-                                 cudaStream_t st, int *launches) {
-    cudaError_t e = bound_and_filter<true>(sp, s, b, ext_of, id_limit, ws, st, launches);
+                                 cudaStream_t st, int *launches, NsScope ns) {
+    cudaError_t e = bound_and_filter<true>(sp, s, b, ext_of, id_limit, ws, st, launches, ns);
     if (e != cudaSuccess) return e;
     k_topm_merge<<<b, SEL_THREADS, 0, st>>>(s, sp.n, sp.bp, sp.k, ext_of, id_limit,
                                             (const unsigned int *)(ws + sp.off_cnt),
                                             ws + sp.off_buf, sp.cap, c_base, nbr_ids, nbr_cos,
-                                            status);
+                                            status, ns);
     if (launches) *launches += 1;
     return cudaGetLastError();
 }

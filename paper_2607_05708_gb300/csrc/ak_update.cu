@@ -62,7 +62,8 @@ static akashic_status_t relate_top_m_batched(const UpdateArgs &a, cudaStream_t s
         const SelectPlan sp = select_plan(n_old, bp, a.M, device_sm_count());
         if (e == cudaSuccess)
             e = launch_select_signed(sp, dots, b, cand, a.ext_of, a.first, off, a.nbr_ids,
-                                     a.nbr_cos, a.status, st, launches);
+                                     a.nbr_cos, a.status, st, launches,
+                                     NsScope{nullptr, nullptr, a.dead_row});
         if (e != cudaSuccess) rc = AKASHIC_ECUDA;
         if (launches) *launches += 1;
     }
@@ -102,21 +103,33 @@ akashic_status_t relate_top_m(const UpdateArgs &a, cudaStream_t st, int *launche
                                                a.dim, qp);
         k_ext_sample<<<sms, 256, 0, st>>>(a.ext_of, n_sample, stride, ext_s);
         e = cudaGetLastError();
-        for (int ct = 0; e == cudaSuccess && ct < n_ct; ++ct) {
+        // deleted chunks are never neighbours: their sample rows carry no key
+        NsScope dscope{};
+        if (e == cudaSuccess && a.dead_row) {
+            int32_t *dead_s = (int32_t *)a.get(SCR_DEAD_S, (size_t)n_sample * 4);
+            if (!dead_s) {
+                rc = AKASHIC_ENOMEM;
+            } else {
+                k_ext_sample<<<sms, 256, 0, st>>>(a.dead_row, n_sample, stride, dead_s);
+                e = cudaGetLastError();
+                dscope = NsScope{nullptr, nullptr, dead_s};
+            }
+        }
+        for (int ct = 0; rc == AKASHIC_OK && e == cudaSuccess && ct < n_ct; ++ct) {
             const int b = (int)(a.n_new - (int64_t)ct * 256 < 256 ? a.n_new - (int64_t)ct * 256 : 256);
             e = launch_dots(a.emb, n_sample, stride, a.dim, qp + (int64_t)ct * 256 * a.dim, 256,
                             sdots, a.status, st, launches);
             if (e == cudaSuccess)
                 e = launch_sample_bound_signed(sp, sdots, b, ext_s, a.first, ws,
-                                               bound + (int64_t)ct * 256, st, launches);
+                                               bound + (int64_t)ct * 256, st, launches, dscope);
         }
-        if (e == cudaSuccess) e = cudaMemsetAsync(cnt, 0, (size_t)n_pad * 4, st);
-        if (e == cudaSuccess)
+        if (rc == AKASHIC_OK && e == cudaSuccess) e = cudaMemsetAsync(cnt, 0, (size_t)n_pad * 4, st);
+        if (rc == AKASHIC_OK && e == cudaSuccess)
             e = launch_dots_filter(a.emb, n, a.dim, qp, n_ct, a.n_new, a.ext_of, a.first, bound,
-                                   cnt, buf, cap, a.status, st, launches);
+                                   cnt, buf, cap, a.status, st, launches, a.dead_row);
         // buffers that overflowed fall back to the exact batched path
         unsigned int max_cnt = 0;
-        if (e == cudaSuccess) {
+        if (rc == AKASHIC_OK && e == cudaSuccess) {
             unsigned int *h = (unsigned int *)malloc((size_t)a.n_new * 4);
             if (!h) {
                 rc = AKASHIC_ENOMEM;

@@ -12,6 +12,8 @@ enum UpdateScratchSlot {
     SCR_DEG, SCR_RECIP, SCR_RECIP_OFF, SCR_KEYS, SCR_VALS, SCR_KEYS2, SCR_VALS2, SCR_TMP,
     SCR_NBR_IDS, SCR_NBR_COS,                                                // update results
     SCR_IN_INC, SCR_IN_DEG, SCR_IN_OFF,                                      // transpose patch
+    SCR_DEAD_S,                                                              // relate sample
+    SCR_DEL_KEEP, SCR_DEL_POS, SCR_DEL_TMP,                                  // deletion
     SCR_SPLIT0, SCR_SPLIT1, SCR_SPLIT2, SCR_SPLIT3, SCR_SPLIT4, SCR_SPLIT5,  // hub plan
     SCR_SPLIT6, SCR_SPLIT7, SCR_SPLIT8, SCR_SPLIT9, SCR_SPLIT10, SCR_SPLIT11,
     SCR_COUNT
@@ -29,6 +31,7 @@ struct UpdateArgs {
     bool reciprocal;
     float scale;           // edge logit = scale * cos
     int *status;
+    const int32_t *dead_row;   // [n_rows] 1 for deleted chunks (never neighbours), or NULL
     int32_t *nbr_ids;      // [n_new * M] selected prior chunks, (cos desc, id asc)
     float *nbr_cos;        // [n_new * M]
     // Grow-only scratch owned by the store: scratch(ctx, slot, bytes) returns

@@ -142,6 +142,119 @@ def test_namespace_scoped_retrieval(hops, sort_by_time):
     assert (got["ids"][::17][:, 3:] == -1).all()
 
 
+@pytest.mark.parametrize("hops", [0, 2])
+def test_delete_then_retrieve(hops):
+    """Delete 600 chunks (the 20 most-pointed-at hubs among them) from the
+    16384-chunk gmm1m-recipe store: the exported CSR equals the oracle's edge
+    drop exactly and its weights are the row softmax of what remains, and
+    retrieval (deleted chunks score nothing and are never selected) matches
+    the oracle with the same tombstones."""
+    import oracle
+    import torch
+    wl = synth.workload(2, scale=1 / 64)
+    rng = np.random.default_rng(17)
+    indeg = np.bincount(wl.col, minlength=wl.n)
+    victims = np.unique(np.concatenate([np.argsort(-indeg)[:20],
+                                        rng.choice(wl.n, 580, replace=False)]))
+    dead = np.zeros(wl.n, bool)
+    dead[victims] = True
+    store = gpu_store(wl, "clustered")
+    store.delete(torch.from_numpy(victims.astype(np.int64)).cuda())
+    store.sync()
+    rp, col, aff, w = (t.cpu().numpy() for t in store.export_csr())
+    orp, ocol, oaff = oracle.drop_dead(wl.row_ptr, wl.col, wl.aff, dead)
+    assert (rp == orp).all() and (col == ocol).all() and (aff == oaff).all()
+    assert np.allclose(w, oracle.row_softmax(rp, aff), rtol=2e-3, atol=0)
+    q = torch.from_numpy(np.ascontiguousarray(wl.queries).view(np.int16)).cuda()
+    ids, sc, pg, npg = store.retrieve(q, wl.k, wl.alpha, hops)
+    store.sync()
+    got = dict(ids=ids.cpu().numpy(), scores=sc.cpu().numpy(), page_ids=pg.cpu().numpy(),
+               n_pages=npg.cpu().numpy())
+    assert not dead[got["ids"]].any()
+    ref = oracle.retrieve(wl.emb, wl.queries, rp, col, oracle.row_softmax(rp, aff), tau=wl.tau,
+                          alpha=wl.alpha, hops=hops, k=wl.k, page_of=wl.page_of["clustered"],
+                          want_final=True, dead=dead)
+    assert_retrieval_parity(wl, "clustered", got, ref)
+
+
+def test_delete_then_update_skips_deleted():
+    """After deletions a relation update links each new chunk to its top-M
+    among the live prior chunks only: its neighbour set equals the oracle's
+    on the store rebuilt without the deleted chunks (IDs mapped back), and
+    retrieval on the result matches the oracle."""
+    import dataclasses
+    import oracle
+    import torch
+    from paper_2607_05708_gb300 import MemStore
+    wl = synth.workload(3, scale=1 / 64)
+    n_old, n_new, M = wl.n, wl.new_emb.shape[0], wl.top_m
+    store = MemStore.from_arrays(wl.emb, wl.page_of["clustered"], wl.row_ptr, wl.col, wl.aff,
+                                 capacity=n_old + n_new, chunks_per_page=wl.chunks_per_page,
+                                 temperature=wl.tau, relation_scale=wl.relation_scale)
+    # delete, for each new chunk, its best prior neighbour (and more at random)
+    all_emb = np.concatenate([wl.emb, wl.new_emb])
+    E = synth.bf16_to_f32(all_emb).astype(np.float64)
+    best = np.argmax(E[n_old:] @ E[:n_old].T, axis=1)
+    victims = np.unique(np.concatenate([best, np.random.default_rng(3).choice(n_old, 200, replace=False)]))
+    dead = np.zeros(n_old + n_new, bool)
+    dead[victims] = True
+    store.delete(torch.from_numpy(victims.astype(np.int64)).cuda())
+    first = store.append_chunks(torch.from_numpy(np.ascontiguousarray(wl.new_emb).view(np.int16)).cuda())
+    store.update_relations(first, n_new, M, reciprocal=True)
+    store.sync()
+    rp, col, aff, _ = (t.cpu().numpy() for t in store.export_csr())
+    live = np.nonzero(~dead[:n_old])[0]
+    for a in range(n_new):
+        nbrs = col[rp[n_old + a]:rp[n_old + a + 1]]
+        assert len(nbrs) == M and not dead[nbrs].any()
+    # oracle on the live-only prior store (edges among live chunks, re-indexed)
+    orp, ocol, oaff = oracle.drop_dead(wl.row_ptr, wl.col, wl.aff, dead[:n_old])
+    new_id = -np.ones(n_old, np.int64)
+    new_id[live] = np.arange(live.size)
+    src = np.repeat(np.arange(n_old), np.diff(orp))
+    rp_l = np.concatenate([[0], np.cumsum(np.bincount(new_id[src], minlength=live.size)),
+                           np.full(n_new, len(ocol))])
+    ref = oracle.update_relations(np.concatenate([wl.emb[live], wl.new_emb]), live.size, n_new, M,
+                                  rp_l, new_id[ocol].astype(np.int32), oaff,
+                                  scale=wl.relation_scale, reciprocal=True)
+    for a in range(n_new):
+        g = set(col[rp[n_old + a]:rp[n_old + a + 1]].tolist())
+        o = set(live[ref["nbr_ids"][a]].tolist())
+        kth = ref["nbr_cos"][a][M - 1]
+        for x in g ^ o:
+            assert abs(float(E[x] @ E[n_old + a]) - kth) < 1e-4, f"new chunk {a}: {x} swapped"
+    wl2 = dataclasses.replace(wl, emb=all_emb, row_ptr=rp, col=col, aff=aff,
+                              page_of={"clustered": _pages_after_appends(wl, [n_new])})
+    _, got = gpu_retrieve(wl2, "clustered", store=store)
+    ref2 = oracle.retrieve(all_emb, wl.queries, rp, col, oracle.row_softmax(rp, aff), tau=wl.tau,
+                           alpha=wl.alpha, hops=wl.hops, k=wl.k,
+                           page_of=wl2.page_of["clustered"], want_final=True, dead=dead)
+    assert_retrieval_parity(wl2, "clustered", got, ref2)
+
+
+def test_delete_errors():
+    """An out-of-range ID deletes nothing (EINVAL); an appended edge that
+    points at a deleted chunk is rejected (EDEVICE) and nothing is appended."""
+    import torch
+    from paper_2607_05708_gb300 import AkashicError, MemStore
+    wl = synth.workload(0)
+    st = MemStore.from_arrays(wl.emb, wl.page_of["id"], wl.row_ptr, wl.col, wl.aff,
+                              capacity=wl.n + 8, chunks_per_page=wl.chunks_per_page)
+    before = [t.cpu().numpy() for t in st.export_csr()]
+    with pytest.raises(AkashicError) as e:
+        st.delete(torch.tensor([3, wl.n + 5], dtype=torch.int64, device="cuda"))
+    assert e.value.code == "EINVAL"
+    after = [t.cpu().numpy() for t in st.export_csr()]
+    assert all((x == y).all() for x, y in zip(before, after))
+    st.delete(torch.tensor([3], dtype=torch.int64, device="cuda"))
+    t = lambda x, dt: torch.from_numpy(np.ascontiguousarray(x).view(dt)).cuda()
+    with pytest.raises(AkashicError) as e:
+        st.append_chunks(t(wl.emb[:1], np.int16), None, t(np.array([0, 1], np.int64), np.int64),
+                         t(np.array([3], np.int32), np.int32), t(np.array([1.0], np.float32), np.float32))
+    assert e.value.code == "EDEVICE"
+    assert st.size()[0] == wl.n
+
+
 def test_no_edges_and_single_chunk_pages():
     """A store without relations: propagation adds nothing."""
     wl0 = synth.workload(0)
