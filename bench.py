@@ -272,6 +272,59 @@ def run_update(args):
     return 0
 
 
+def run_delete(args):
+    """Chunk deletion: each step deletes 1024 fresh random chunks of the
+    gmm1m store (tombstones, edges into and out of them dropped from the CSR
+    and the transpose, rows re-softmaxed, hub plan rebuilt).  Bytes moved per
+    call: both edge lists read, flagged and compacted once."""
+    import torch
+    import synth
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2607_05708_gb300 import MemStore
+    wl = synth.workload(2, scale=args.scale)
+    store = MemStore.from_arrays(wl.emb, wl.page_of["clustered"], wl.row_ptr, wl.col, wl.aff,
+                                 capacity=wl.n, chunks_per_page=wl.chunks_per_page,
+                                 temperature=wl.tau)
+    total = args.warmup + args.steps
+    order = np.random.default_rng(5).permutation(wl.n)[:1024 * total]
+    st = torch.cuda.Stream()
+    times = []
+    with Clocks(0) as clk:
+        for i in range(total):
+            ids = torch.from_numpy(order[i * 1024:(i + 1) * 1024].astype(np.int64)).cuda()
+            torch.cuda.synchronize()
+            e0 = torch.cuda.Event(enable_timing=True)
+            e1 = torch.cuda.Event(enable_timing=True)
+            e0.record(st)
+            store.delete(ids, stream=st)
+            e1.record(st)
+            torch.cuda.synchronize()
+            if i >= args.warmup:
+                times.append(e0.elapsed_time(e1))
+    ms = sum(times) / len(times)
+    n_rows, nnz = store.size()
+    hbm, _, kind = peaks()
+    # per call: out CSR (col+aff read, flags, scan, compacted write) and the
+    # same for the transpose, plus the row softmax over the CSR
+    moved = nnz * (4 + 4 + 8 + 8 + 8 + 4 + 4) * 2 + nnz * 12
+    line = {
+        "metric": "delete ms per 1024 chunks (N=1M, nnz 33.5M)", "value": ms, "unit": "ms/delete",
+        "higher_is_better": False, "n_gpus": 1, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": ms, "dtype": "f32", "data": "synthetic",
+        "config": {"workload": "gmm1m store, 1024 random chunks deleted per step"
+                   + ("" if args.scale == 1.0 else f", scaled by {args.scale}")},
+        "roofline": {"bound": "hbm", "achieved": moved / (ms * 1e-3) / 1e9, "peak": hbm,
+                     "unit": "GB/s", "frac": moved / (ms * 1e-3) / 1e9 / hbm, "traffic": None,
+                     "kernel": "whole delete call", "peak_kind": kind},
+        "edges_left": nnz,
+        "clocks": clk.summary(),
+    }
+    print(json.dumps(line), flush=True)
+    store.close()
+    return 0
+
+
 def run_streams(args):
     """4M-chunk store, 1024 queries issued as 8 streams of 128 in a seeded
     arrival order; aggregate queries/s over all streams."""
@@ -355,21 +408,24 @@ def main():
     ap.add_argument("--scale", type=float, default=1.0,
                     help="shrink N (profiling captures of a smaller case); 1.0 = the benchmark")
     ap.add_argument("--workload", default="retrieve",
-                    choices=["retrieve", "update", "streams", "dense", "scoped"],
+                    choices=["retrieve", "update", "streams", "dense", "scoped", "delete"],
                     help="retrieve: the benchmark; update: relation update of 4096 new chunks "
                          "on the 1M-chunk store; streams: 4M-chunk store, 8 streams x 128 "
                          "queries; dense: the Dense-only form (k=5, no hops) on the 1M store; "
-                         "scoped: namespace-scoped retrieval with SortByTime on the 1M store")
+                         "scoped: namespace-scoped retrieval with SortByTime on the 1M store; "
+                         "delete: 1024 chunks deleted per step from the 1M store")
     args = ap.parse_args()
     if args.steps is None:
         args.steps = {"retrieve": 100, "update": 5, "streams": 20, "dense": 100,
-                      "scoped": 100}[args.workload]
+                      "scoped": 100, "delete": 10}[args.workload]
     if args.impl == "reference":
         return run_reference(args)
     if args.workload == "update":
         return run_update(args)
     if args.workload == "streams":
         return run_streams(args)
+    if args.workload == "delete":
+        return run_delete(args)
     if args.workload == "dense":
         return run_retrieve(args, k=5, hops=0, metric=DENSE_METRIC, workload=DENSE_WORKLOAD)
     if args.workload == "scoped":
