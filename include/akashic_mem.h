@@ -162,6 +162,47 @@ akashic_status_t akashic_mem_set_namespace(akashic_mem_t *m, int64_t first, int6
 akashic_status_t akashic_mem_delete(akashic_mem_t *m, const int64_t *ids, int64_t n,
                                     void *stream);
 
+/* Memory Manager (§4.2, Algorithm 2), on the page directory (page_of).
+ * The model calls have dense stand-ins: co-retrieval statistics over the
+ * requests passed in (sel(c) = requests that retrieved c, co(a, b) = those
+ * that retrieved both); affinity(a, b) = co / (sel(a) + sel(b) - co), "high
+ * association" when co >= tau_assoc * (sel(a) + sel(b) - co) (fp64, tau
+ * rounded to fp32; the paper's tau_assoc is 0.7, §5.5).
+ *
+ * Relocation (Algorithm 2, lines 3-8).  S: device int64[n_req][s_len]
+ * retrieved chunk IDs per request (-1, IDs outside the store, deleted
+ * chunks and repeats are skipped), 1 <= s_len <= 64.  The batch's statistics
+ * are added first; then, request by request, the chunks of the request that
+ * are highly associated with another of its chunks (LLMCoLocate), if two or
+ * more and not all on one page, are written out of place in chunk-ID order
+ * (SortByTime) into fresh pages of chunks_per_page slots; each old copy
+ * becomes an invalid slot of its page.  Synchronises `stream`.
+ * EINVAL on bad sizes or tau outside [0, 1]. */
+akashic_status_t akashic_mem_relocate(akashic_mem_t *m, const int64_t *S, int32_t n_req,
+                                      int32_t s_len, float tau_assoc, void *stream);
+
+/* Block compaction (Algorithm 2, lines 11-24; phi(B) of §4.2): every page
+ * whose invalid ratio phi = (slots - live) / slots is >= theta (0.75 in the
+ * paper) is compacted: its live chunks are partitioned by namespace
+ * (akashic_mem_set_namespace), grouped within a partition by the connected
+ * components of highly associated pairs (LLMGroup), and repacked into fresh
+ * pages partition by partition, group by group (groups by earliest chunk
+ * ID), chunk ID order within a group; the page is released.  *released
+ * (may be NULL) = pages released.  Synchronises `stream`.
+ * EINVAL if theta is outside (0, 1] or tau outside [0, 1]. */
+akashic_status_t akashic_mem_compact_pages(akashic_mem_t *m, float theta, float tau_assoc,
+                                           int64_t *released, void *stream);
+
+/* Page accounting, host int64 out[5]: pages in use, slots in use (live and
+ * invalid), live slots, chunk writes (appends + relocations + compaction
+ * moves), chunks appended.  Space amplification = out[1] / out[2]; write
+ * amplification = out[3] / out[4].  Synchronises the device. */
+akashic_status_t akashic_mem_page_stats(akashic_mem_t *m, int64_t *out);
+
+/* page_of: device int32[size]: the page of every chunk ID (the directory
+ * retrieval resolves through).  Stream-ordered. */
+akashic_status_t akashic_mem_export_pages(akashic_mem_t *m, int32_t *page_of, void *stream);
+
 /* Retrieval scoped to the caller's namespace, with optional chronological
  * order (§4.1: candidates are the chunks of the current user_id/session_id;
  * Algorithm 1 lines SortByTime: the selected chunks are returned in time

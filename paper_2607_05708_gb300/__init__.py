@@ -30,6 +30,8 @@ EXPORTS = (
     "akashic_mem_size", "akashic_mem_sync", "akashic_mem_set_profiling",
     "akashic_mem_phase_times", "akashic_mem_last_error", "akashic_mem_softmax_scores_noalloc",
     "akashic_mem_set_namespace", "akashic_mem_retrieve_scoped", "akashic_mem_delete",
+    "akashic_mem_relocate", "akashic_mem_compact_pages", "akashic_mem_page_stats",
+    "akashic_mem_export_pages",
 )
 
 
@@ -71,6 +73,10 @@ def load_library(path: str | None = None):
                                         ctypes.c_int),
         "akashic_mem_set_namespace": ([V, I64, I64, V, V], ctypes.c_int),
         "akashic_mem_delete": ([V, V, I64, V], ctypes.c_int),
+        "akashic_mem_relocate": ([V, V, I32, I32, F, V], ctypes.c_int),
+        "akashic_mem_compact_pages": ([V, F, F, P64, V], ctypes.c_int),
+        "akashic_mem_page_stats": ([V, P64], ctypes.c_int),
+        "akashic_mem_export_pages": ([V, V, V], ctypes.c_int),
         "akashic_mem_export_csr": ([V, P64, P64, V, V, V, V, V], ctypes.c_int),
         "akashic_mem_size": ([V, P64, P64], ctypes.c_int),
         "akashic_mem_sync": ([V, V], ctypes.c_int),
@@ -204,6 +210,36 @@ class MemStore:
     def update_relations(self, first: int, n: int, M: int, reciprocal: bool = True, stream=None):
         _check(load_library().akashic_mem_update_relations(
             self._h, first, n, M, int(bool(reciprocal)), _stream(self._torch, stream, self.device)))
+
+    def relocate(self, S, tau_assoc: float = 0.7, stream=None):
+        """Relocation of co-retrieved chunks (S: int64 [n_req, s_len] device tensor)."""
+        torch = self._torch
+        self._dev(S, torch.int64, "S")
+        n_req, s_len = (S.shape[0], S.shape[1]) if S.dim() == 2 else (1, S.shape[0])
+        _check(load_library().akashic_mem_relocate(self._h, _ptr(S), n_req, s_len,
+                                                   float(tau_assoc),
+                                                   _stream(torch, stream, self.device)))
+
+    def compact_pages(self, theta: float = 0.75, tau_assoc: float = 0.7, stream=None) -> int:
+        rel = ctypes.c_int64()
+        _check(load_library().akashic_mem_compact_pages(
+            self._h, float(theta), float(tau_assoc), ctypes.byref(rel),
+            _stream(self._torch, stream, self.device)))
+        return rel.value
+
+    def page_stats(self) -> dict:
+        out = (ctypes.c_int64 * 5)()
+        _check(load_library().akashic_mem_page_stats(self._h, out))
+        keys = ("pages_in_use", "slots_total", "slots_live", "chunk_writes", "appended")
+        return dict(zip(keys, list(out)))
+
+    def export_pages(self, stream=None):
+        torch = self._torch
+        n, _ = self.size()
+        out = torch.empty(max(n, 1), dtype=torch.int32, device=torch.device("cuda", self.device))
+        _check(load_library().akashic_mem_export_pages(self._h, _ptr(out),
+                                                       _stream(torch, stream, self.device)))
+        return out[:n]
 
     def delete(self, ids, stream=None):
         """Delete chunks (int64 device tensor of chunk IDs)."""

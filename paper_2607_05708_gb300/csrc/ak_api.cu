@@ -118,6 +118,10 @@ struct akashic_mem {
     DevBuf ns_row;               // namespace tag of the chunk in each row (0 by default)
     DevBuf dead_row;             // 1 in the rows of deleted chunks
     bool has_dead = false;       // any chunk deleted (enables the masks)
+    // memory manager: per-page slot counters, co-retrieval statistics
+    DevBuf page_total, page_live, sel, co_key, co_val, mm_ctr;
+    int64_t page_cap = 0, co_cap = 0, co_upper = 0;
+    int64_t appended = 0, moves = 0;
     // canonical out-edge CSR
     int64_t nnz = 0;
     DevBuf row_ptr, col, aff, w;
@@ -228,6 +232,54 @@ static void *store_scratch(void *ctx, int slot, size_t bytes) {
     DevBuf &b = m->scr[slot];
     if (bytes > b.cap && b.ensure(bytes + bytes / 8) != AKASHIC_OK) return nullptr;
     return b.p;
+}
+
+static MmTables mm_tables(akashic_mem *m) {
+    MmTables t;
+    t.page_total = m->page_total.as<int32_t>();
+    t.page_live = m->page_live.as<int32_t>();
+    t.sel = m->sel.as<int32_t>();
+    t.co_key = m->co_key.as<unsigned long long>();
+    t.co_val = m->co_val.as<uint32_t>();
+    t.co_cap = m->co_cap;
+    t.next_page = m->mm_ctr.as<int64_t>();
+    t.writes = m->mm_ctr.as<int64_t>() + 1;
+    return t;
+}
+
+// Page counters for page IDs below `need` (grown by doubling, new tail zeroed).
+static akashic_status_t mm_ensure_pages(akashic_mem *m, int64_t need, cudaStream_t st) {
+    if (need <= m->page_cap) return AKASHIC_OK;
+    int64_t cap = m->page_cap > 0 ? m->page_cap : 1024;
+    while (cap < need) cap *= 2;
+    AK_TRY(m->page_total.ensure((size_t)cap * 4, true, st));
+    AK_TRY(m->page_live.ensure((size_t)cap * 4, true, st));
+    CUDA_TRY(cudaMemsetAsync(m->page_total.as<int32_t>() + m->page_cap, 0,
+                             (size_t)(cap - m->page_cap) * 4, st));
+    CUDA_TRY(cudaMemsetAsync(m->page_live.as<int32_t>() + m->page_cap, 0,
+                             (size_t)(cap - m->page_cap) * 4, st));
+    m->page_cap = cap;
+    return AKASHIC_OK;
+}
+
+// Co-retrieval table able to take `more` new pairs at load <= 1/2.
+static akashic_status_t mm_ensure_pairs(akashic_mem *m, int64_t more, cudaStream_t st) {
+    if (m->co_cap > 0 && m->co_upper + more <= m->co_cap / 2) return AKASHIC_OK;
+    int64_t cap = m->co_cap > 0 ? m->co_cap : ((int64_t)1 << 20);
+    while (m->co_upper + more > cap / 2) cap *= 2;
+    DevBuf nk, nv;
+    AK_TRY(nk.ensure((size_t)cap * 8));
+    AK_TRY(nv.ensure((size_t)cap * 4));
+    std::swap(m->co_key.p, nk.p);
+    std::swap(m->co_key.cap, nk.cap);
+    std::swap(m->co_val.p, nv.p);
+    std::swap(m->co_val.cap, nv.cap);
+    const int64_t old_cap = m->co_cap;
+    m->co_cap = cap;
+    CUDA_TRY(launch_mm_rehash(nk.as<unsigned long long>(), nv.as<uint32_t>(), old_cap,
+                              mm_tables(m), m->status.as<int>(), st));
+    CUDA_TRY(cudaStreamSynchronize(st));   // the old table is freed on return
+    return AKASHIC_OK;
 }
 
 // A scratch buffer seen through the DevBuf-like accessors.
@@ -417,6 +469,10 @@ akashic_status_t akashic_mem_create(const akashic_mem_config_t *cfg, akashic_mem
         cudaMemset(m->row_ptr.p, 0, 8) != cudaSuccess || cudaMemset(m->in_ptr.p, 0, 8) != cudaSuccess ||
         cudaMemset(m->ns_row.p, 0, (size_t)m->cap * 4) != cudaSuccess ||
         cudaMemset(m->dead_row.p, 0, (size_t)m->cap * 4) != cudaSuccess ||
+        m->sel.ensure((size_t)m->cap * 4) != AKASHIC_OK ||
+        cudaMemset(m->sel.p, 0, (size_t)m->cap * 4) != cudaSuccess ||
+        m->mm_ctr.ensure(16) != AKASHIC_OK || cudaMemset(m->mm_ctr.p, 0, 16) != cudaSuccess ||
+        mm_ensure_pages(m, 1024, 0) != AKASHIC_OK || mm_ensure_pairs(m, 0, 0) != AKASHIC_OK ||
         cudaDeviceSynchronize() != cudaSuccess) {
         delete m;
         return fail(AKASHIC_ECUDA, "create: initialisation failed");
@@ -532,6 +588,10 @@ akashic_status_t akashic_mem_append_chunks(akashic_mem_t *m, const uint16_t *emb
     } else {
         m->next_page += ceil_div<int64_t>(n, m->per_page);
     }
+    // the new chunks occupy a slot of their pages
+    AK_TRY(mm_ensure_pages(m, m->next_page + 1, st));
+    CUDA_TRY(launch_mm_count_pages(m->page_of.as<int32_t>(), first, n, mm_tables(m), st));
+    m->appended += n;
     CUDA_TRY(launch_row_norm_max(m->emb.as<uint16_t>() + first * m->dim, n, m->dim,
                                  m->max_norm.as<float>(), st));
     int64_t *rp = m->row_ptr.as<int64_t>() + first;   // rp[0] is already m->nnz
@@ -749,7 +809,8 @@ akashic_status_t akashic_mem_delete(akashic_mem_t *m, const int64_t *ids, int64_
                               m->status.as<int>(), st));
     AK_TRY(check_status(m, st, "delete: chunk IDs must lie in [0, size)"));
     CUDA_TRY(launch_mark_dead(ids, n, m->n, m->row_of.as<int32_t>(), m->dead_row.as<int32_t>(),
-                              m->status.as<int>(), st));
+                              m->status.as<int>(), st, m->page_of.as<int32_t>(),
+                              m->page_live.as<int32_t>()));
     m->has_dead = true;
     const int64_t rows = m->n, nnz = m->nnz;
     if (nnz == 0) return AKASHIC_OK;
@@ -803,6 +864,141 @@ akashic_status_t akashic_mem_delete(akashic_mem_t *m, const int64_t *ids, int64_
     std::swap(m->in_w.cap, m->in_w2.cap);
     AK_TRY(build_split_plan(m, st));
     return check_status(m, st, "delete");
+}
+akashic_status_t akashic_mem_relocate(akashic_mem_t *m, const int64_t *S, int32_t n_req,
+                                      int32_t s_len, float tau_assoc, void *stream) {
+    g_last_error.clear();
+    if (!m) return fail(AKASHIC_EINVAL, "relocate: NULL store");
+    if (n_req < 0 || s_len < 1 || s_len > 64)
+        return fail(AKASHIC_EINVAL, "relocate: need n_req >= 0 and 1 <= s_len <= 64");
+    if (!(tau_assoc >= 0.f && tau_assoc <= 1.f))
+        return fail(AKASHIC_EINVAL, "relocate: tau_assoc must lie in [0, 1]");
+    if (n_req == 0) return AKASHIC_OK;
+    if (!S) return fail(AKASHIC_EINVAL, "relocate: NULL S");
+    DeviceGuard g(m->device);
+    cudaStream_t st = (cudaStream_t)stream;
+    const int64_t pairs = (int64_t)n_req * s_len * (s_len - 1) / 2;
+    AK_TRY(mm_ensure_pairs(m, pairs, st));
+    AK_TRY(mm_ensure_pages(m, m->next_page + (int64_t)n_req * ceil_div<int64_t>(64, m->per_page) + 1,
+                           st));
+    int32_t *gb = (int32_t *)store_scratch(m, SCR_MM_G, (size_t)n_req * 64 * 4);
+    int32_t *gn = (int32_t *)store_scratch(m, SCR_MM_GN, (size_t)n_req * 4);
+    if (!gb || !gn) return fail(AKASHIC_ENOMEM, "relocate: out of device memory");
+    int64_t ctr[2] = {m->next_page, 0};
+    CUDA_TRY(cudaMemcpyAsync(m->mm_ctr.p, ctr, 16, cudaMemcpyHostToDevice, st));
+    const int32_t *dead = m->has_dead ? m->dead_row.as<int32_t>() : nullptr;
+    const MmTables t = mm_tables(m);
+    CUDA_TRY(launch_mm_count(S, n_req, s_len, m->n, m->row_of.as<int32_t>(), dead, t,
+                             m->status.as<int>(), st));
+    CUDA_TRY(launch_mm_relocate(S, n_req, s_len, m->n, m->row_of.as<int32_t>(), dead,
+                                m->page_of.as<int32_t>(), t, tau_assoc, m->per_page, gb, gn, st));
+    CUDA_TRY(cudaMemcpyAsync(ctr, m->mm_ctr.p, 16, cudaMemcpyDeviceToHost, st));
+    AK_TRY(check_status(m, st, "relocate"));
+    m->next_page = ctr[0];
+    m->moves += ctr[1];
+    m->co_upper += pairs;
+    return AKASHIC_OK;
+}
+
+akashic_status_t akashic_mem_compact_pages(akashic_mem_t *m, float theta, float tau_assoc,
+                                           int64_t *released, void *stream) {
+    g_last_error.clear();
+    if (!m) return fail(AKASHIC_EINVAL, "compact: NULL store");
+    if (!(theta > 0.f && theta <= 1.f))
+        return fail(AKASHIC_EINVAL, "compact: theta must lie in (0, 1]");
+    if (!(tau_assoc >= 0.f && tau_assoc <= 1.f))
+        return fail(AKASHIC_EINVAL, "compact: tau_assoc must lie in [0, 1]");
+    DeviceGuard g(m->device);
+    cudaStream_t st = (cudaStream_t)stream;
+    const int64_t n = m->n, pages = m->next_page;
+    if (released) *released = 0;
+    if (n == 0) return AKASHIC_OK;
+    const size_t tb = (scan_tmp_bytes(n + 1) > radix_tmp_bytes(n) ? scan_tmp_bytes(n + 1)
+                                                                   : radix_tmp_bytes(n)) + 4096;
+    int32_t *cand = (int32_t *)store_scratch(m, SCR_MM_CAND, (size_t)(pages + 1) * 4);
+    int64_t *moving = (int64_t *)store_scratch(m, SCR_MM_MOVING, (size_t)(n + 1) * 8);
+    int64_t *pos = (int64_t *)store_scratch(m, SCR_MM_POS, (size_t)(n + 1) * 8);
+    int32_t *parent = (int32_t *)store_scratch(m, SCR_MM_PARENT, (size_t)n * 4);
+    int32_t *ns_id = (int32_t *)store_scratch(m, SCR_MM_NS, (size_t)n * 4);
+    uint32_t *ids = (uint32_t *)store_scratch(m, SCR_MM_IDS, (size_t)n * 4 + 16);
+    uint32_t *root = (uint32_t *)store_scratch(m, SCR_MM_ROOT, (size_t)n * 4 + 16);
+    uint32_t *nsk = (uint32_t *)store_scratch(m, SCR_MM_NSK, (size_t)n * 4 + 16);
+    uint32_t *k2 = (uint32_t *)store_scratch(m, SCR_MM_K2, (size_t)n * 4 + 16);
+    uint32_t *v2 = (uint32_t *)store_scratch(m, SCR_MM_V2, (size_t)n * 4 + 16);
+    void *tmp = store_scratch(m, SCR_MM_TMP, tb);
+    if (!cand || !moving || !pos || !parent || !ns_id || !ids || !root || !nsk || !k2 || !v2 || !tmp)
+        return fail(AKASHIC_ENOMEM, "compact: out of device memory");
+    const MmTables t = mm_tables(m);
+    const int32_t *dead = m->has_dead ? m->dead_row.as<int32_t>() : nullptr;
+    const int32_t *row_of = m->row_of.as<int32_t>();
+    CUDA_TRY(launch_mm_compact_prepare(t, pages, theta, n, row_of, dead, m->page_of.as<int32_t>(),
+                                       cand, moving, parent, st));
+    CUDA_TRY(cudaMemsetAsync(moving + n, 0, 8, st));
+    CUDA_TRY(launch_by_id(m->ns_row.as<int32_t>(), row_of, n, ns_id, st));
+    CUDA_TRY(launch_mm_union(t, moving, ns_id, tau_assoc, parent, m->status.as<int>(), st));
+    CUDA_TRY(scan_exclusive(moving, pos, n + 1, tmp, tb, st));
+    int64_t count = 0;
+    CUDA_TRY(cudaMemcpyAsync(&count, pos + n, 8, cudaMemcpyDeviceToHost, st));
+    AK_TRY(check_status(m, st, "compact"));
+    int64_t n_rel = 0;
+    {
+        // pages released: the candidates (counted on the host from the flags)
+        std::vector<int32_t> h((size_t)pages);
+        if (pages > 0)
+            CUDA_TRY(cudaMemcpy(h.data(), cand, (size_t)pages * 4, cudaMemcpyDeviceToHost));
+        for (int32_t v : h) n_rel += v != 0;
+    }
+    if (count > 0) {
+        CUDA_TRY(launch_mm_keys(moving, pos, n, parent, ns_id, ids, root, nsk, st));
+        // order (namespace, group root, chunk ID): the list is in ID order;
+        // stable sorts by root, then by namespace
+        bool alt = false;
+        CUDA_TRY(radix_sort_pairs(root, ids, k2, v2, count, 32, tmp, tb, st, &alt));
+        uint32_t *sid = alt ? v2 : ids, *spare_v = alt ? ids : v2;
+        uint32_t *nk = alt ? root : k2;
+        CUDA_TRY(launch_mm_ns_keys(sid, count, ns_id, nsk, st));
+        bool alt2 = false;
+        CUDA_TRY(radix_sort_pairs(nsk, sid, nk, spare_v, count, 32, tmp, tb, st, &alt2));
+        const uint32_t *order = alt2 ? spare_v : sid;
+        AK_TRY(mm_ensure_pages(m, m->next_page + ceil_div<int64_t>(count, m->per_page) + 1, st));
+        CUDA_TRY(launch_mm_release_repack(mm_tables(m), pages, cand, order, count, row_of,
+                                          m->page_of.as<int32_t>(), m->next_page, m->per_page,
+                                          st));
+        m->next_page += ceil_div<int64_t>(count, m->per_page);
+        m->moves += count;
+    } else if (n_rel > 0) {
+        CUDA_TRY(launch_mm_release_repack(t, pages, cand, nullptr, 0, row_of,
+                                          m->page_of.as<int32_t>(), m->next_page, m->per_page,
+                                          st));
+    }
+    if (released) *released = n_rel;
+    return check_status(m, st, "compact");
+}
+
+akashic_status_t akashic_mem_page_stats(akashic_mem_t *m, int64_t *out) {
+    g_last_error.clear();
+    if (!m || !out) return fail(AKASHIC_EINVAL, "page_stats: NULL argument");
+    DeviceGuard g(m->device);
+    unsigned long long *d = (unsigned long long *)store_scratch(m, SCR_MM_TMP, 64);
+    if (!d) return fail(AKASHIC_ENOMEM, "page_stats: out of device memory");
+    CUDA_TRY(launch_mm_stats(mm_tables(m), m->next_page, d, 0));
+    unsigned long long h[3] = {0, 0, 0};
+    CUDA_TRY(cudaMemcpy(h, d, sizeof h, cudaMemcpyDeviceToHost));
+    out[0] = (int64_t)h[0];
+    out[1] = (int64_t)h[1];
+    out[2] = (int64_t)h[2];
+    out[3] = m->appended + m->moves;
+    out[4] = m->appended;
+    return AKASHIC_OK;
+}
+
+akashic_status_t akashic_mem_export_pages(akashic_mem_t *m, int32_t *page_of, void *stream) {
+    g_last_error.clear();
+    if (!m || !page_of) return fail(AKASHIC_EINVAL, "export_pages: NULL argument");
+    DeviceGuard g(m->device);
+    CUDA_TRY(launch_by_id(m->page_of.as<int32_t>(), m->row_of.as<int32_t>(), m->n, page_of,
+                          (cudaStream_t)stream));
+    return AKASHIC_OK;
 }
 }  // extern "C"
 

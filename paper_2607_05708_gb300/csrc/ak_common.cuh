@@ -237,11 +237,60 @@ cudaError_t launch_seg_permute(const uint32_t *order, const int64_t *e0, const i
 cudaError_t launch_split_keys(const int64_t *slot0, int64_t n_split, uint32_t *keys,
                               uint32_t *vals, cudaStream_t st);
 
+// Memory Manager tables (ak_mm.cu): the page directory's slot counters,
+// the co-retrieval statistics and the running counters.
+struct MmTables {
+    int32_t *page_total, *page_live;   // [page capacity] slots used / live chunks per page
+    int32_t *sel;                      // [chunk capacity] requests that retrieved the chunk
+    unsigned long long *co_key;        // [co_cap] chunk pair (lo << 32 | hi), ~0 = empty
+    uint32_t *co_val;                  // [co_cap] requests that retrieved both
+    int64_t co_cap;                    // power of two
+    int64_t *next_page;                // device copy of the next fresh page ID
+    int64_t *writes;                   // chunks written (appends, relocations, compaction)
+};
+cudaError_t launch_mm_count(const int64_t *S, int n_req, int s_len, int64_t n,
+                            const int32_t *row_of, const int32_t *dead_row, const MmTables &t,
+                            int *status, cudaStream_t st);
+// g_buf [n_req][64], g_n [n_req] scratch.
+cudaError_t launch_mm_relocate(const int64_t *S, int n_req, int s_len, int64_t n,
+                               const int32_t *row_of, const int32_t *dead_row, int32_t *page_row,
+                               const MmTables &t, float tau, int per_page, int32_t *g_buf,
+                               int32_t *g_n, cudaStream_t st);
+cudaError_t launch_mm_compact_prepare(const MmTables &t, int64_t n_pages, float theta, int64_t n,
+                                      const int32_t *row_of, const int32_t *dead_row,
+                                      const int32_t *page_row, int32_t *cand, int64_t *moving,
+                                      int32_t *parent, cudaStream_t st);
+cudaError_t launch_mm_union(const MmTables &t, const int64_t *moving, const int32_t *ns_by_id,
+                            float tau, int32_t *parent, int *status, cudaStream_t st);
+cudaError_t launch_mm_keys(const int64_t *moving, const int64_t *pos, int64_t n,
+                           const int32_t *parent, const int32_t *ns_by_id, uint32_t *ids,
+                           uint32_t *root_key, uint32_t *ns_key, cudaStream_t st);
+cudaError_t launch_mm_release_repack(const MmTables &t, int64_t n_pages, const int32_t *cand,
+                                     const uint32_t *order_ids, int64_t count,
+                                     const int32_t *row_of, int32_t *page_row, int64_t first_page,
+                                     int per_page, cudaStream_t st);
+cudaError_t launch_mm_count_pages(const int32_t *page_row, int64_t first, int64_t n,
+                                  const MmTables &t, cudaStream_t st);
+// out[0..2] = pages in use, slots in use, live slots
+cudaError_t launch_mm_stats(const MmTables &t, int64_t n_pages, unsigned long long *out,
+                            cudaStream_t st);
+cudaError_t launch_mm_rehash(const unsigned long long *old_key, const uint32_t *old_val,
+                             int64_t old_cap, const MmTables &t, int *status, cudaStream_t st);
+// out[i] = ns_by_id[ids[i]] as an order-preserving unsigned key
+cudaError_t launch_mm_ns_keys(const uint32_t *ids, int64_t count, const int32_t *ns_by_id,
+                              uint32_t *out, cudaStream_t st);
+// out[c] = by_row[row_of[c]], c < n
+cudaError_t launch_by_id(const int32_t *by_row, const int32_t *row_of, int64_t n, int32_t *out,
+                         cudaStream_t st);
+
 // Chunk deletion (ak_delete.cu).  dead_row[row_of[id]] = 1 for the listed
 // IDs (out-of-range IDs set EINVAL in *status and are skipped; dead_row
 // NULL: check only).
+// A newly deleted chunk's slot becomes invalid: page_live[page_row[row]]
+// drops by one (page_row / page_live may be NULL).
 cudaError_t launch_mark_dead(const int64_t *ids, int64_t n, int64_t n_total, const int32_t *row_of,
-                             int32_t *dead_row, int *status, cudaStream_t st);
+                             int32_t *dead_row, int *status, cudaStream_t st,
+                             const int32_t *page_row = nullptr, int32_t *page_live = nullptr);
 // EDEVICE in *status if any col[e] < first names a deleted chunk.
 cudaError_t launch_check_dead_targets(const int32_t *col, int64_t nnz, int64_t first,
                                       const int32_t *row_of, const int32_t *dead_row, int *status,

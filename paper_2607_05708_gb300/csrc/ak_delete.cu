@@ -13,7 +13,8 @@ namespace ak {
 // IDs outside [0, n_total) set EINVAL in the status word and are skipped.
 __global__ void k_mark_dead(const int64_t *__restrict__ ids, int64_t n, int64_t n_total,
                             const int32_t *__restrict__ row_of, int32_t *__restrict__ dead_row,
-                            int *status) {
+                            int *status, const int32_t *__restrict__ page_row,
+                            int32_t *__restrict__ page_live) {
     for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n;
          i += (int64_t)gridDim.x * blockDim.x) {
         const int64_t id = ids[i];
@@ -21,7 +22,9 @@ __global__ void k_mark_dead(const int64_t *__restrict__ ids, int64_t n, int64_t 
             set_status(status, AKASHIC_EINVAL);
             continue;
         }
-        if (dead_row) dead_row[row_of[id]] = 1;
+        if (!dead_row) continue;
+        const int64_t r = row_of[id];
+        if (atomicExch(&dead_row[r], 1) == 0 && page_live) atomicSub(&page_live[page_row[r]], 1);
     }
 }
 
@@ -95,9 +98,11 @@ cudaError_t launch_check_dead_targets(const int32_t *col, int64_t nnz, int64_t f
 }
 
 cudaError_t launch_mark_dead(const int64_t *ids, int64_t n, int64_t n_total, const int32_t *row_of,
-                             int32_t *dead_row, int *status, cudaStream_t st) {
+                             int32_t *dead_row, int *status, cudaStream_t st,
+                             const int32_t *page_row, int32_t *page_live) {
     if (n <= 0) return cudaSuccess;
-    k_mark_dead<<<device_sm_count(), 256, 0, st>>>(ids, n, n_total, row_of, dead_row, status);
+    k_mark_dead<<<device_sm_count(), 256, 0, st>>>(ids, n, n_total, row_of, dead_row, status,
+                                                   page_row, page_live);
     return cudaGetLastError();
 }
 

@@ -14,6 +14,9 @@ enum UpdateScratchSlot {
     SCR_IN_INC, SCR_IN_DEG, SCR_IN_OFF,                                      // transpose patch
     SCR_DEAD_S,                                                              // relate sample
     SCR_DEL_KEEP, SCR_DEL_POS, SCR_DEL_TMP,                                  // deletion
+    SCR_MM_G, SCR_MM_GN, SCR_MM_CAND, SCR_MM_MOVING, SCR_MM_POS, SCR_MM_PARENT,  // memory
+    SCR_MM_NS, SCR_MM_IDS, SCR_MM_ROOT, SCR_MM_NSK, SCR_MM_K2, SCR_MM_V2,          // manager
+    SCR_MM_TMP,
     SCR_SPLIT0, SCR_SPLIT1, SCR_SPLIT2, SCR_SPLIT3, SCR_SPLIT4, SCR_SPLIT5,  // hub plan
     SCR_SPLIT6, SCR_SPLIT7, SCR_SPLIT8, SCR_SPLIT9, SCR_SPLIT10, SCR_SPLIT11,
     SCR_COUNT
