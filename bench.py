@@ -43,6 +43,12 @@ SCOPED_WORKLOAD = ("gmm1m store with 64 namespaces (chunk tag = mixture componen
 DENSE_METRIC = "Dense-only retrieve queries/sec at N=1M chunks, d=1024, B=256, top-p 5, no hops"
 DENSE_WORKLOAD = ("gmm1m store (N=1048576, d=1024 bf16), B=256 queries, k=5, hops=0 "
                   "(embedding similarity only), 64 chunks/page, clustered placement")
+MEMORY_METRIC = ("Memory Manager requests/sec (co-retrieval counts, relocation, block compaction) "
+                 "at N=1M chunks, batches of 256 top-5 requests")
+MEMORY_WORKLOAD = ("gmm1m store (N=1048576, d=1024 bf16, 64 chunks/page) in random placement (the "
+                   "append-only log); trace of Dense-only top-5 retrievals, queries = one of 4096 "
+                   "anchor chunks drawn with Zipf(1.1) popularity + N(0,(0.05/sqrt d)^2) noise; per "
+                   "step relocate(S, tau_assoc=0.7) then compact(theta=0.75, tau_assoc=0.7)")
 
 
 def peaks():
@@ -325,6 +331,146 @@ def run_delete(args):
     return 0
 
 
+def _numpy_top5(wl, q_bf16, block=65536):
+    """Top-5 chunk IDs by dot product, plain numpy fp32 (input preparation of
+    the CPU sample; ties broken arbitrarily, which timing does not mind)."""
+    import synth
+    q = synth.bf16_to_f32(q_bf16)
+    best_v = np.full((q.shape[0], 5), -np.inf, np.float32)
+    best_i = np.zeros((q.shape[0], 5), np.int64)
+    for r0 in range(0, wl.n, block):
+        e = synth.bf16_to_f32(wl.emb[r0:r0 + block])
+        d = q @ e.T
+        part = np.argpartition(-d, 5, axis=1)[:, :5]
+        v = np.take_along_axis(d, part, axis=1)
+        cv = np.concatenate([best_v, v], axis=1)
+        ci = np.concatenate([best_i, part + r0], axis=1)
+        top = np.argpartition(-cv, 5, axis=1)[:, :5]
+        best_v = np.take_along_axis(cv, top, axis=1)
+        best_i = np.take_along_axis(ci, top, axis=1)
+    return best_i
+
+
+def run_memory(args):
+    """The Memory Manager (co-retrieval statistics, relocation of associated
+    chunks, block compaction) fed by the retrieval it serves: every step
+    takes one batch of 256 Dense-only top-5 request sets of a replayed trace
+    and runs relocate + compact on the gmm1m directory.  Reports pages per
+    request over the trace before and after, and space / write
+    amplification."""
+    import torch
+    import synth
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2607_05708_gb300 import MemStore
+    wl = synth.workload(2, scale=args.scale)
+    B, K, W = 256, args.steps, args.warmup
+    T = W + 2 * K
+    Q = synth.request_trace(wl, T * B, n_topics=max(64, wl.n // 256))
+    cpu = None
+    if not args.no_cpu_baseline:
+        from oracle.memory_manager import MemoryManager
+        n_b = 4
+        S_cpu = _numpy_top5(wl, Q[:n_b * B])
+        mm = MemoryManager(wl.page_of["random"], wl.chunks_per_page)
+        t0 = time.perf_counter()
+        for b in range(n_b):
+            mm.relocate(S_cpu[b * B:(b + 1) * B], 0.7)
+            mm.compact(0.75, 0.7)
+        t = time.perf_counter() - t0
+        cpu = {"value": n_b * B / t, "unit": "requests/s", "cores": 1, "kind": "oracle",
+               "sample": f"first {n_b} batches of 256 requests on the fresh 1M-chunk directory "
+                         "(request sets from a numpy fp32 top-5, untimed)"}
+    store = MemStore.from_arrays(wl.emb, wl.page_of["random"], wl.row_ptr, wl.col, wl.aff,
+                                 capacity=wl.n, chunks_per_page=wl.chunks_per_page,
+                                 temperature=wl.tau)
+    st = torch.cuda.Stream()
+    q_dev = torch.from_numpy(Q.view(np.int16)).cuda()
+    S = torch.empty((T, B, 5), dtype=torch.int64, device="cuda")
+    sc = torch.empty((B, 5), dtype=torch.float32, device="cuda")
+    pg = torch.empty((B, 5), dtype=torch.int32, device="cuda")
+    npg = torch.empty((T, B), dtype=torch.int32, device="cuda")
+
+    def replay():
+        for b in range(T):
+            store.retrieve(q_dev[b * B:(b + 1) * B], 5, wl.alpha, 0, S[b], sc, pg, npg[b],
+                           stream=st)
+        torch.cuda.synchronize()
+        return npg.float().mean().item()
+
+    before = replay()
+
+    def step(b):
+        store.relocate(S[b], 0.7, stream=st)
+        store.compact_pages(0.75, 0.7, stream=st)
+
+    for b in range(W):
+        step(b)
+    torch.cuda.synchronize()
+    store.set_profiling(True)
+    store.phase_times()
+    ev0 = torch.cuda.Event(enable_timing=True)
+    ev1 = torch.cuda.Event(enable_timing=True)
+    with Clocks(0) as clk:
+        ev0.record(st)
+        for b in range(W, W + K):
+            step(b)
+        ev1.record(st)
+        torch.cuda.synchronize()
+    ms = ev0.elapsed_time(ev1) / K
+    phases = store.phase_times()
+    store.set_profiling(False)
+    # end to end: request sets from pinned host memory, page accounting read back
+    S_host = S[W + K:].cpu().pin_memory()
+    s_dev = torch.empty((B, 5), dtype=torch.int64, device="cuda")
+    torch.cuda.synchronize()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(st)
+    for i in range(K):
+        with torch.cuda.stream(st):
+            s_dev.copy_(S_host[i], non_blocking=True)
+        store.relocate(s_dev, 0.7, stream=st)
+        store.compact_pages(0.75, 0.7, stream=st)
+        stats = store.page_stats()
+    e1.record(st)
+    torch.cuda.synchronize()
+    e2e_ms = e0.elapsed_time(e1) / K
+    after = replay()
+    stats = store.page_stats()
+    n_pages = stats["pages_in_use"]
+    hbm, _, kind = peaks()
+    rel_ms, rel_l = phases["relocate"]
+    cmp_ms, cmp_l = phases["compact"]
+    # compaction: every page's two counters and every chunk's page and
+    # tombstone read once (the directory scan that finds what moves)
+    cmp_bytes = n_pages * 8 + wl.n * 8
+    achieved = cmp_bytes / (cmp_ms / K * 1e-3) / 1e9
+    line = {
+        "metric": MEMORY_METRIC, "value": B * 1000.0 / ms, "unit": "requests/s",
+        "n_gpus": 1, "steps": K, "warmup": W, "ms_per_step": ms, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "int32", "data": "synthetic",
+        "config": {"workload": MEMORY_WORKLOAD
+                   + ("" if args.scale == 1.0 else f", scaled by {args.scale}"),
+                   "l2": "directory and tables stay resident; the step's work is latency-bound"},
+        "roofline": {"bound": "hbm", "achieved": achieved, "peak": hbm, "unit": "GB/s",
+                     "frac": achieved / hbm, "traffic": None,
+                     "kernel": "whole compaction call", "peak_kind": kind},
+        "phases_ms_per_step": {"relocate": rel_ms / K, "compact": cmp_ms / K},
+        "pages_per_request": {"before": before, "after": after},
+        "space_amplification": stats["slots_total"] / max(1, stats["slots_live"]),
+        "write_amplification": stats["chunk_writes"] / max(1, stats["appended"]),
+        "e2e": {"value": B * 1000.0 / e2e_ms, "unit": "requests/s",
+                "h2d_bytes_per_step": B * 5 * 8, "d2h_bytes_per_step": 5 * 8},
+        "gpu_launches": int(rel_l + cmp_l),
+        "cpu_baseline": cpu,
+        "clocks": clk.summary(),
+    }
+    print(json.dumps(line), flush=True)
+    store.close()
+    return 0
+
+
 def run_streams(args):
     """4M-chunk store, 1024 queries issued as 8 streams of 128 in a seeded
     arrival order; aggregate queries/s over all streams."""
@@ -408,16 +554,18 @@ def main():
     ap.add_argument("--scale", type=float, default=1.0,
                     help="shrink N (profiling captures of a smaller case); 1.0 = the benchmark")
     ap.add_argument("--workload", default="retrieve",
-                    choices=["retrieve", "update", "streams", "dense", "scoped", "delete"],
+                    choices=["retrieve", "update", "streams", "dense", "scoped", "delete",
+                             "memory"],
                     help="retrieve: the benchmark; update: relation update of 4096 new chunks "
                          "on the 1M-chunk store; streams: 4M-chunk store, 8 streams x 128 "
                          "queries; dense: the Dense-only form (k=5, no hops) on the 1M store; "
                          "scoped: namespace-scoped retrieval with SortByTime on the 1M store; "
-                         "delete: 1024 chunks deleted per step from the 1M store")
+                         "delete: 1024 chunks deleted per step from the 1M store; memory: "
+                         "relocation + block compaction of 256 top-5 requests per step")
     args = ap.parse_args()
     if args.steps is None:
         args.steps = {"retrieve": 100, "update": 5, "streams": 20, "dense": 100,
-                      "scoped": 100, "delete": 10}[args.workload]
+                      "scoped": 100, "delete": 10, "memory": 20}[args.workload]
     if args.impl == "reference":
         return run_reference(args)
     if args.workload == "update":
@@ -426,6 +574,8 @@ def main():
         return run_streams(args)
     if args.workload == "delete":
         return run_delete(args)
+    if args.workload == "memory":
+        return run_memory(args)
     if args.workload == "dense":
         return run_retrieve(args, k=5, hops=0, metric=DENSE_METRIC, workload=DENSE_WORKLOAD)
     if args.workload == "scoped":

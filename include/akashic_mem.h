@@ -249,7 +249,9 @@ enum {
     AKASHIC_PHASE_SELECT = 2,    /* top-k candidates, merge, page resolve       */
     AKASHIC_PHASE_RELATE = 3,    /* new x store cosine GEMM + top-M             */
     AKASHIC_PHASE_GRAPH = 4,     /* CSR insert, weights, transpose rebuild      */
-    AKASHIC_PHASE_COUNT = 5
+    AKASHIC_PHASE_RELOCATE = 5,  /* co-retrieval counts + relocation            */
+    AKASHIC_PHASE_COMPACT = 6,   /* block compaction                            */
+    AKASHIC_PHASE_COUNT = 7
 };
 akashic_status_t akashic_mem_set_profiling(akashic_mem_t *m, int32_t on);
 akashic_status_t akashic_mem_phase_times(akashic_mem_t *m, float *ms, int32_t *launches);

@@ -244,6 +244,7 @@ static MmTables mm_tables(akashic_mem *m) {
     t.co_cap = m->co_cap;
     t.next_page = m->mm_ctr.as<int64_t>();
     t.writes = m->mm_ctr.as<int64_t>() + 1;
+    t.released = m->mm_ctr.as<unsigned long long>() + 2;
     return t;
 }
 
@@ -263,7 +264,8 @@ static akashic_status_t mm_ensure_pages(akashic_mem *m, int64_t need, cudaStream
 }
 
 // Co-retrieval table able to take `more` new pairs at load <= 1/2.
-static akashic_status_t mm_ensure_pairs(akashic_mem *m, int64_t more, cudaStream_t st) {
+static akashic_status_t mm_ensure_pairs(akashic_mem *m, int64_t more, cudaStream_t st,
+                                        int *launches = nullptr) {
     if (m->co_cap > 0 && m->co_upper + more <= m->co_cap / 2) return AKASHIC_OK;
     int64_t cap = m->co_cap > 0 ? m->co_cap : ((int64_t)1 << 20);
     while (m->co_upper + more > cap / 2) cap *= 2;
@@ -278,6 +280,7 @@ static akashic_status_t mm_ensure_pairs(akashic_mem *m, int64_t more, cudaStream
     m->co_cap = cap;
     CUDA_TRY(launch_mm_rehash(nk.as<unsigned long long>(), nv.as<uint32_t>(), old_cap,
                               mm_tables(m), m->status.as<int>(), st));
+    if (launches && old_cap > 0) *launches += 1;
     CUDA_TRY(cudaStreamSynchronize(st));   // the old table is freed on return
     return AKASHIC_OK;
 }
@@ -471,7 +474,7 @@ akashic_status_t akashic_mem_create(const akashic_mem_config_t *cfg, akashic_mem
         cudaMemset(m->dead_row.p, 0, (size_t)m->cap * 4) != cudaSuccess ||
         m->sel.ensure((size_t)m->cap * 4) != AKASHIC_OK ||
         cudaMemset(m->sel.p, 0, (size_t)m->cap * 4) != cudaSuccess ||
-        m->mm_ctr.ensure(16) != AKASHIC_OK || cudaMemset(m->mm_ctr.p, 0, 16) != cudaSuccess ||
+        m->mm_ctr.ensure(32) != AKASHIC_OK || cudaMemset(m->mm_ctr.p, 0, 32) != cudaSuccess ||
         mm_ensure_pages(m, 1024, 0) != AKASHIC_OK || mm_ensure_pairs(m, 0, 0) != AKASHIC_OK ||
         cudaDeviceSynchronize() != cudaSuccess) {
         delete m;
@@ -877,8 +880,9 @@ akashic_status_t akashic_mem_relocate(akashic_mem_t *m, const int64_t *S, int32_
     if (!S) return fail(AKASHIC_EINVAL, "relocate: NULL S");
     DeviceGuard g(m->device);
     cudaStream_t st = (cudaStream_t)stream;
+    PhaseScope ph(m, AKASHIC_PHASE_RELOCATE, st);
     const int64_t pairs = (int64_t)n_req * s_len * (s_len - 1) / 2;
-    AK_TRY(mm_ensure_pairs(m, pairs, st));
+    AK_TRY(mm_ensure_pairs(m, pairs, st, &ph.launches));
     AK_TRY(mm_ensure_pages(m, m->next_page + (int64_t)n_req * ceil_div<int64_t>(64, m->per_page) + 1,
                            st));
     int32_t *gb = (int32_t *)store_scratch(m, SCR_MM_G, (size_t)n_req * 64 * 4);
@@ -892,6 +896,7 @@ akashic_status_t akashic_mem_relocate(akashic_mem_t *m, const int64_t *S, int32_
                              m->status.as<int>(), st));
     CUDA_TRY(launch_mm_relocate(S, n_req, s_len, m->n, m->row_of.as<int32_t>(), dead,
                                 m->page_of.as<int32_t>(), t, tau_assoc, m->per_page, gb, gn, st));
+    ph.launches += 3;
     CUDA_TRY(cudaMemcpyAsync(ctr, m->mm_ctr.p, 16, cudaMemcpyDeviceToHost, st));
     AK_TRY(check_status(m, st, "relocate"));
     m->next_page = ctr[0];
@@ -928,48 +933,49 @@ akashic_status_t akashic_mem_compact_pages(akashic_mem_t *m, float theta, float 
     void *tmp = store_scratch(m, SCR_MM_TMP, tb);
     if (!cand || !moving || !pos || !parent || !ns_id || !ids || !root || !nsk || !k2 || !v2 || !tmp)
         return fail(AKASHIC_ENOMEM, "compact: out of device memory");
+    PhaseScope ph(m, AKASHIC_PHASE_COMPACT, st);
     const MmTables t = mm_tables(m);
     const int32_t *dead = m->has_dead ? m->dead_row.as<int32_t>() : nullptr;
     const int32_t *row_of = m->row_of.as<int32_t>();
+    CUDA_TRY(cudaMemsetAsync(t.released, 0, 8, st));
     CUDA_TRY(launch_mm_compact_prepare(t, pages, theta, n, row_of, dead, m->page_of.as<int32_t>(),
                                        cand, moving, parent, st));
     CUDA_TRY(cudaMemsetAsync(moving + n, 0, 8, st));
     CUDA_TRY(launch_by_id(m->ns_row.as<int32_t>(), row_of, n, ns_id, st));
     CUDA_TRY(launch_mm_union(t, moving, ns_id, tau_assoc, parent, m->status.as<int>(), st));
-    CUDA_TRY(scan_exclusive(moving, pos, n + 1, tmp, tb, st));
-    int64_t count = 0;
-    CUDA_TRY(cudaMemcpyAsync(&count, pos + n, 8, cudaMemcpyDeviceToHost, st));
+    ph.launches += (pages > 0) + 3;
+    CUDA_TRY(scan_exclusive(moving, pos, n + 1, tmp, tb, st, &ph.launches));
+    // released pages and moving chunks, read back together
+    CUDA_TRY(cudaMemcpyAsync(t.released + 1, pos + n, 8, cudaMemcpyDeviceToDevice, st));
+    int64_t rc[2] = {0, 0};
+    CUDA_TRY(cudaMemcpyAsync(rc, t.released, 16, cudaMemcpyDeviceToHost, st));
     AK_TRY(check_status(m, st, "compact"));
-    int64_t n_rel = 0;
-    {
-        // pages released: the candidates (counted on the host from the flags)
-        std::vector<int32_t> h((size_t)pages);
-        if (pages > 0)
-            CUDA_TRY(cudaMemcpy(h.data(), cand, (size_t)pages * 4, cudaMemcpyDeviceToHost));
-        for (int32_t v : h) n_rel += v != 0;
-    }
+    const int64_t n_rel = rc[0], count = rc[1];
     if (count > 0) {
         CUDA_TRY(launch_mm_keys(moving, pos, n, parent, ns_id, ids, root, nsk, st));
         // order (namespace, group root, chunk ID): the list is in ID order;
         // stable sorts by root, then by namespace
         bool alt = false;
-        CUDA_TRY(radix_sort_pairs(root, ids, k2, v2, count, 32, tmp, tb, st, &alt));
+        CUDA_TRY(radix_sort_pairs(root, ids, k2, v2, count, 32, tmp, tb, st, &alt, &ph.launches));
         uint32_t *sid = alt ? v2 : ids, *spare_v = alt ? ids : v2;
         uint32_t *nk = alt ? root : k2;
         CUDA_TRY(launch_mm_ns_keys(sid, count, ns_id, nsk, st));
         bool alt2 = false;
-        CUDA_TRY(radix_sort_pairs(nsk, sid, nk, spare_v, count, 32, tmp, tb, st, &alt2));
+        CUDA_TRY(radix_sort_pairs(nsk, sid, nk, spare_v, count, 32, tmp, tb, st, &alt2,
+                                  &ph.launches));
         const uint32_t *order = alt2 ? spare_v : sid;
         AK_TRY(mm_ensure_pages(m, m->next_page + ceil_div<int64_t>(count, m->per_page) + 1, st));
         CUDA_TRY(launch_mm_release_repack(mm_tables(m), pages, cand, order, count, row_of,
                                           m->page_of.as<int32_t>(), m->next_page, m->per_page,
                                           st));
+        ph.launches += 2 + (pages > 0) + 1;
         m->next_page += ceil_div<int64_t>(count, m->per_page);
         m->moves += count;
     } else if (n_rel > 0) {
         CUDA_TRY(launch_mm_release_repack(t, pages, cand, nullptr, 0, row_of,
                                           m->page_of.as<int32_t>(), m->next_page, m->per_page,
                                           st));
+        ph.launches += 1;
     }
     if (released) *released = n_rel;
     return check_status(m, st, "compact");

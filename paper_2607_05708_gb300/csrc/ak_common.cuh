@@ -143,8 +143,9 @@ struct SplitParams {
 constexpr int ROWS_PER_GRAB = 8;     // rows a warp claims at a time (dynamic scheduling)
 
 // Exclusive prefix sum of `in` (n values) into out (n+1 values; out[n] = total).
+// `launches`, if given, is incremented by the kernels launched.
 cudaError_t scan_exclusive(const int64_t *in, int64_t *out, int64_t n, void *tmp,
-                           size_t tmp_bytes, cudaStream_t st);
+                           size_t tmp_bytes, cudaStream_t st, int *launches = nullptr);
 size_t scan_tmp_bytes(int64_t n);
 
 // Stable LSD radix sort of (key, value) pairs on the low `bits` key bits;
@@ -152,7 +153,8 @@ size_t scan_tmp_bytes(int64_t n);
 size_t radix_tmp_bytes(int64_t n);
 cudaError_t radix_sort_pairs(uint32_t *keys, uint32_t *vals, uint32_t *keys_alt,
                              uint32_t *vals_alt, int64_t n, int bits, void *tmp,
-                             size_t tmp_bytes, cudaStream_t st, bool *result_in_alt);
+                             size_t tmp_bytes, cudaStream_t st, bool *result_in_alt,
+                             int *launches = nullptr);
 
 // CSR helpers (see ak_graph.cu).
 cudaError_t launch_edge_src_check(const int64_t *row_ptr, const int32_t *col, int64_t n_rows,
@@ -247,6 +249,7 @@ struct MmTables {
     int64_t co_cap;                    // power of two
     int64_t *next_page;                // device copy of the next fresh page ID
     int64_t *writes;                   // chunks written (appends, relocations, compaction)
+    unsigned long long *released;      // pages released by the last compaction
 };
 cudaError_t launch_mm_count(const int64_t *S, int n_req, int s_len, int64_t n,
                             const int32_t *row_of, const int32_t *dead_row, const MmTables &t,

@@ -93,25 +93,28 @@ size_t scan_tmp_bytes(int64_t n) {
 }
 
 static cudaError_t scan_rec(const int64_t *in, int64_t *out, int64_t n, int64_t *tmp,
-                            cudaStream_t st) {
+                            cudaStream_t st, int *launches) {
     if (n <= 0) return cudaSuccess;
     int64_t tiles = ceil_div<int64_t>(n, SCAN_TILE);
     int64_t *sums = tmp, *offs = tmp + tiles;
     k_scan_tile<<<(unsigned)tiles, SCAN_THREADS, 0, st>>>(in, out, n, sums);
+    if (launches) *launches += 1;
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess || tiles == 1) return e;
-    e = scan_rec(sums, offs, tiles, tmp + 2 * tiles + 2, st);
+    e = scan_rec(sums, offs, tiles, tmp + 2 * tiles + 2, st, launches);
     if (e != cudaSuccess) return e;
     k_scan_add<<<(unsigned)ceil_div<int64_t>(n, 256), 256, 0, st>>>(out, n, offs);
+    if (launches) *launches += 1;
     return cudaGetLastError();
 }
 
 cudaError_t scan_exclusive(const int64_t *in, int64_t *out, int64_t n, void *tmp,
-                           size_t tmp_bytes, cudaStream_t st) {
+                           size_t tmp_bytes, cudaStream_t st, int *launches) {
     if (tmp_bytes < scan_tmp_bytes(n)) return cudaErrorInvalidValue;
-    cudaError_t e = scan_rec(in, out, n, (int64_t *)tmp, st);
+    cudaError_t e = scan_rec(in, out, n, (int64_t *)tmp, st, launches);
     if (e != cudaSuccess) return e;
     k_scan_total<<<1, 1, 0, st>>>(in, out, n);
+    if (launches) *launches += 1;
     return cudaGetLastError();
 }
 
@@ -198,7 +201,8 @@ size_t radix_tmp_bytes(int64_t n) {
 
 cudaError_t radix_sort_pairs(uint32_t *keys, uint32_t *vals, uint32_t *keys_alt,
                              uint32_t *vals_alt, int64_t n, int bits, void *tmp,
-                             size_t tmp_bytes, cudaStream_t st, bool *result_in_alt) {
+                             size_t tmp_bytes, cudaStream_t st, bool *result_in_alt,
+                             int *launches) {
     *result_in_alt = false;
     if (n <= 1 || bits <= 0) return cudaSuccess;
     if (tmp_bytes < radix_tmp_bytes(n)) return cudaErrorInvalidValue;
@@ -215,10 +219,11 @@ cudaError_t radix_sort_pairs(uint32_t *keys, uint32_t *vals, uint32_t *keys_alt,
         k_rs_hist<<<(unsigned)n_tiles, RS_THREADS, 0, st>>>(ki, n, sh, mask, n_tiles, hist);
         cudaError_t e = cudaGetLastError();
         if (e != cudaSuccess) return e;
-        e = scan_exclusive(hist, offs, m, stmp, stmp_bytes, st);
+        e = scan_exclusive(hist, offs, m, stmp, stmp_bytes, st, launches);
         if (e != cudaSuccess) return e;
         k_rs_scatter<<<(unsigned)n_tiles, RS_THREADS, 0, st>>>(ki, vi, n, sh, mask, n_tiles, offs,
                                                                 ko, vo);
+        if (launches) *launches += 2;
         e = cudaGetLastError();
         if (e != cudaSuccess) return e;
         uint32_t *t;

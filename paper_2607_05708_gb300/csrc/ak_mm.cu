@@ -191,10 +191,19 @@ __global__ void k_mm_relocate(const int32_t *__restrict__ g_in, const int32_t *_
 
 // ------------------------------------------------------------------ compaction
 __global__ void k_mm_candidates(MmTables t, int64_t n_pages, float theta, int32_t *__restrict__ cand) {
-    for (int64_t p = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; p < n_pages;
-         p += (int64_t)gridDim.x * blockDim.x) {
-        const int32_t tot = t.page_total[p], live = t.page_live[p];
-        cand[p] = tot > 0 && (double)(tot - live) >= (double)theta * (double)tot;
+    // warp-uniform trip count, so the whole warp takes part in every ballot
+    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    for (int64_t base = (int64_t)blockIdx.x * blockDim.x + (threadIdx.x & ~31); base < n_pages;
+         base += stride) {
+        const int64_t p = base + (threadIdx.x & 31);
+        bool c = false;
+        if (p < n_pages) {
+            const int32_t tot = t.page_total[p], live = t.page_live[p];
+            c = tot > 0 && (double)(tot - live) >= (double)theta * (double)tot;
+            cand[p] = c;
+        }
+        const unsigned ballot = __ballot_sync(0xffffffffu, c);
+        if ((threadIdx.x & 31) == 0 && ballot) atomicAdd(t.released, (unsigned long long)__popc(ballot));
     }
 }
 

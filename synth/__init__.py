@@ -453,3 +453,23 @@ def workload(index: int, scale: float = 1.0, placements=None) -> Workload:
                       "to its size), "
                       "top-32 cosine neighbours among the old store, reciprocal edges")
     return wl
+
+
+def request_trace(wl: Workload, n_queries: int, n_topics: int = 4096, s: float = 1.1,
+                  seed: int = 2607, noise: float = 0.05) -> np.ndarray:
+    """A replayable query trace for the Memory Manager workload: `n_topics`
+    anchor chunks drawn uniformly from the store, each query an anchor drawn
+    with Zipf(s) popularity by rank plus N(0, (noise/sqrt(d))^2 I), unit
+    length, bf16.  Popular anchors recur, as the memory a long-running agent
+    keeps re-reading does, so the same top-p sets are retrieved again and
+    again.  Returns uint16 [n_queries, dim]."""
+    ss = np.random.SeedSequence(seed)
+    s_anchor, s_pick, s_noise = ss.spawn(3)
+    anchors = np.random.default_rng(s_anchor).choice(wl.n, size=n_topics, replace=False)
+    w = 1.0 / np.arange(1, n_topics + 1, dtype=np.float64) ** s
+    pick = np.random.default_rng(s_pick).choice(n_topics, size=n_queries, p=w / w.sum())
+    rows = bf16_to_f32(wl.emb[anchors[pick]])
+    x = np.random.default_rng(s_noise).standard_normal(rows.shape, dtype=np.float32)
+    x *= np.float32(noise / math.sqrt(wl.dim))
+    x += rows
+    return to_bf16(_unit_rows(x))
