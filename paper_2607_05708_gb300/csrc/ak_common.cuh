@@ -102,10 +102,11 @@ cudaError_t launch_score_filter(const uint16_t *emb, int64_t n, int dim, const u
                                 cudaStream_t st, int *launches, int *zrows);
 
 // Plain dot products out[j, c] = <e_{j*row_stride}, q_c> (bf16 tensor
-// cores, fp32 accumulate) for j < n, row stride bp in out.
+// cores, fp32 accumulate) for j < n and the n_ctiles * bp columns of qp;
+// row stride n_ctiles * bp in out.
 cudaError_t launch_dots(const uint16_t *emb, int64_t n, int64_t row_stride_rows, int dim,
-                        const uint16_t *qp, int bp, float *out, int *status, cudaStream_t st,
-                        int *launches);
+                        const uint16_t *qp, int bp, int n_ctiles, float *out, int *status,
+                        cudaStream_t st, int *launches);
 // Fused relation top-M filter: dots of every row j < n against the
 // n_ctiles*256 rows of qp; the selection key (signed dot, chunk ID
 // ext_of[j]) of every (j, c) with c < n_cols and ext_of[j] < id_limit that

@@ -565,12 +565,12 @@ cudaError_t launch_score_filter(const uint16_t *emb, int64_t n, int dim, const u
 }
 
 cudaError_t launch_dots(const uint16_t *emb, int64_t n, int64_t row_stride_rows, int dim,
-                        const uint16_t *qp, int bp, float *out, int *status, cudaStream_t st,
-                        int *launches) {
+                        const uint16_t *qp, int bp, int n_ctiles, float *out, int *status,
+                        cudaStream_t st, int *launches) {
     GemmEpi ep{};
     ep.status = status;
-    cudaError_t e = gemm_dispatch<GEMM_RAW>(emb, n, row_stride_rows, dim, qp, bp, 1, out, ep, st,
-                                            nullptr);
+    cudaError_t e = gemm_dispatch<GEMM_RAW>(emb, n, row_stride_rows, dim, qp, bp, n_ctiles, out,
+                                            ep, st, nullptr);
     if (launches) *launches += 1;
     return e;
 }

@@ -58,7 +58,7 @@ static akashic_status_t relate_top_m_batched(const UpdateArgs &a, cudaStream_t s
                                                           a.dim, qp);
         e = cudaGetLastError();
         if (e == cudaSuccess)
-            e = launch_dots(a.emb, n_old, 1, a.dim, qp, bp, dots, a.status, st, launches);
+            e = launch_dots(a.emb, n_old, 1, a.dim, qp, bp, 1, dots, a.status, st, launches);
         const SelectPlan sp = select_plan(n_old, bp, a.M, device_sm_count());
         if (e == cudaSuccess)
             e = launch_select_signed(sp, dots, b, cand, a.ext_of, a.first, off, a.nbr_ids,
@@ -82,13 +82,24 @@ akashic_status_t relate_top_m(const UpdateArgs &a, cudaStream_t st, int *launche
     const int sms = device_sm_count();
     const int n_ct = (int)ceil_div<int64_t>(a.n_new, 256);
     const int64_t n_pad = (int64_t)n_ct * 256;
-    int64_t stride = n / ((int64_t)64 * a.M);
-    stride = stride < 1 ? 1 : (stride > 32 ? 32 : stride);
+    // every stride-th row is sampled: about 512 M rows, so the bound (the
+    // M-th largest sampled value) lets through about M * stride rows per
+    // new chunk, which the merge stages in shared memory
+    int64_t stride = n / ((int64_t)512 * a.M);
+    stride = stride < 1 ? 1 : (stride > 64 ? 64 : stride);
     const int64_t n_sample = ceil_div<int64_t>(n, stride);
     const int64_t cap = 4 * (int64_t)a.M * stride > 8192 ? 4 * (int64_t)a.M * stride : 8192;
-    const SelectPlan sp = select_plan(n_sample, 256, a.M, sms, 1);
+    // the sample bounds of G column tiles come from one dots GEMM, one
+    // transpose and one k-th launch (G tiles of sampled dots: <= 256 MB)
+    const int64_t tile_bytes = n_sample * 256 * 4;
+    int64_t G = ((int64_t)256 << 20) / tile_bytes;
+    G = G < 1 ? 1 : (G > n_ct ? n_ct : G);
+    SelectPlan sp = select_plan(n_sample, (int)G * 256, a.M, sms, 1);
+    sp.cap = 0;                      // no candidate buffers: bounds only
+    sp.off_tr = sp.off_buf;
+    sp.words = sp.off_tr + ceil_div<int64_t>(sp.n_sample * sp.bp, 2);
     uint16_t *qp = (uint16_t *)a.get(SCR_QP, (size_t)n_pad * a.dim * 2);
-    float *sdots = (float *)a.get(SCR_SDOTS, (size_t)n_sample * 256 * 4);
+    float *sdots = (float *)a.get(SCR_SDOTS, (size_t)G * tile_bytes);
     int32_t *ext_s = (int32_t *)a.get(SCR_EXTS, (size_t)n_sample * 4);
     unsigned long long *ws = (unsigned long long *)a.get(SCR_WS, (size_t)sp.words * 8);
     unsigned long long *bound = (unsigned long long *)a.get(SCR_BOUND, (size_t)n_pad * 8);
@@ -115,13 +126,17 @@ akashic_status_t relate_top_m(const UpdateArgs &a, cudaStream_t st, int *launche
                 dscope = NsScope{nullptr, nullptr, dead_s};
             }
         }
-        for (int ct = 0; rc == AKASHIC_OK && e == cudaSuccess && ct < n_ct; ++ct) {
-            const int b = (int)(a.n_new - (int64_t)ct * 256 < 256 ? a.n_new - (int64_t)ct * 256 : 256);
-            e = launch_dots(a.emb, n_sample, stride, a.dim, qp + (int64_t)ct * 256 * a.dim, 256,
-                            sdots, a.status, st, launches);
+        for (int64_t g0 = 0; rc == AKASHIC_OK && e == cudaSuccess && g0 < n_ct; g0 += G) {
+            const int gt = (int)(n_ct - g0 < G ? n_ct - g0 : G);
+            const int64_t left = a.n_new - g0 * 256;
+            const int b = (int)(left < (int64_t)gt * 256 ? left : (int64_t)gt * 256);
+            SelectPlan spg = sp;
+            spg.bp = gt * 256;
+            e = launch_dots(a.emb, n_sample, stride, a.dim, qp + g0 * 256 * a.dim, 256, gt, sdots,
+                            a.status, st, launches);
             if (e == cudaSuccess)
-                e = launch_sample_bound_signed(sp, sdots, b, ext_s, a.first, ws,
-                                               bound + (int64_t)ct * 256, st, launches, dscope);
+                e = launch_sample_bound_signed(spg, sdots, b, ext_s, a.first, ws, bound + g0 * 256,
+                                               st, launches, dscope);
         }
         if (rc == AKASHIC_OK && e == cudaSuccess) e = cudaMemsetAsync(cnt, 0, (size_t)n_pad * 4, st);
         if (rc == AKASHIC_OK && e == cudaSuccess)
