@@ -273,31 +273,61 @@ cudaError_t launch_edge_src_check(const int64_t *row_ptr, const int32_t *col, in
     return cudaGetLastError();
 }
 
-// Relation weights: w = softmax of each row's edge logits (one warp per row).
+// Relation weights: w = softmax of each row's edge logits.  Eight lanes per
+// row and four rows per warp step (rows are short: 32 edges plus the
+// reciprocal ones), so a warp keeps four rows' loads in flight; a row of up
+// to 64 edges is read once and kept in registers.
+constexpr int RSM_LANES = 8, RSM_KEEP = 8;
 __global__ void k_row_softmax(const int64_t *__restrict__ row_ptr, const float *__restrict__ aff,
                               float *__restrict__ w, int64_t n_rows, float2 *__restrict__ rstat) {
-    const int lane = threadIdx.x & 31;
-    int64_t r = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
-    const int64_t stride = ((int64_t)gridDim.x * blockDim.x) >> 5;
-    for (; r < n_rows; r += stride) {
-        int64_t a = row_ptr[r], b = row_ptr[r + 1];
-        if (b <= a) continue;
+    constexpr int L = RSM_LANES, R = 32 / RSM_LANES;
+    const int lane = threadIdx.x & 31, sub = lane % L, grp = lane / L;
+    const int64_t nw = ((int64_t)gridDim.x * blockDim.x) >> 5;
+    for (int64_t r0 = (((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5) * R; r0 < n_rows;
+         r0 += nw * R) {
+        const int64_t r = r0 + grp;
+        int64_t a = 0, b = 0;
+        if (r < n_rows) {
+            a = row_ptr[r];
+            b = row_ptr[r + 1];
+        }
+        float v[RSM_KEEP];
         float m = -INFINITY;
-        for (int64_t e = a + lane; e < b; e += 32) m = fmaxf(m, aff[e]);
-        for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
+#pragma unroll
+        for (int t = 0; t < RSM_KEEP; ++t) {
+            const int64_t e = a + sub + t * L;
+            v[t] = e < b ? aff[e] : -INFINITY;
+            m = fmaxf(m, v[t]);
+        }
+        for (int64_t e = a + sub + RSM_KEEP * L; e < b; e += L) m = fmaxf(m, aff[e]);
+#pragma unroll
+        for (int o = L / 2; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
         float s = 0.f;
-        for (int64_t e = a + lane; e < b; e += 32) s += expf(aff[e] - m);
-        for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
-        const float2 stat = make_float2(m, 1.f / s);
-        if (rstat && lane == 0) rstat[r] = stat;
-        for (int64_t e = a + lane; e < b; e += 32) w[e] = row_softmax_weight(aff[e], stat);
+#pragma unroll
+        for (int t = 0; t < RSM_KEEP; ++t)
+            if (a + sub + t * L < b) s += expf(v[t] - m);
+        for (int64_t e = a + sub + RSM_KEEP * L; e < b; e += L) s += expf(aff[e] - m);
+#pragma unroll
+        for (int o = L / 2; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+        if (b > a) {
+            const float2 stat = make_float2(m, 1.f / s);
+            if (rstat && sub == 0) rstat[r] = stat;
+#pragma unroll
+            for (int t = 0; t < RSM_KEEP; ++t) {
+                const int64_t e = a + sub + t * L;
+                if (e < b) w[e] = row_softmax_weight(v[t], stat);
+            }
+            for (int64_t e = a + sub + RSM_KEEP * L; e < b; e += L)
+                w[e] = row_softmax_weight(aff[e], stat);
+        }
     }
 }
 
 cudaError_t launch_row_softmax(const int64_t *row_ptr, const float *aff, float *w, int64_t n_rows,
                                float2 *rstat, cudaStream_t st) {
     if (n_rows <= 0) return cudaSuccess;
-    int64_t warps = n_rows < (int64_t)device_sm_count() * 64 ? n_rows : (int64_t)device_sm_count() * 64;
+    const int64_t want = ceil_div<int64_t>(n_rows, 32 / RSM_LANES);
+    const int64_t warps = want < (int64_t)device_sm_count() * 64 ? want : (int64_t)device_sm_count() * 64;
     k_row_softmax<<<(unsigned)ceil_div<int64_t>(warps * 32, 256), 256, 0, st>>>(row_ptr, aff, w,
                                                                               n_rows, rstat);
     return cudaGetLastError();
@@ -434,39 +464,76 @@ __device__ __forceinline__ int64_t lower_bound_src(const int32_t *__restrict__ s
     return lo;
 }
 
+// A hub row (more than split_t in-edges, sorted by source row) cut by one
+// warp: lane l takes source windows w0 + l, w0 + l + 32, ...; the edge range
+// of each window comes from two binary searches, and its segments (at most
+// seg_len edges each) are numbered by a scan across the lanes in window
+// order.  Returns the row's segment count (on every lane).
 template <bool FILL>
-__device__ __forceinline__ int64_t walk_segments(SplitParams sp, const int32_t *__restrict__ in_src,
-                                                 int64_t a, int64_t b, int64_t slot,
-                                                 int64_t *seg_e0, int64_t *seg_e1,
-                                                 uint32_t *seg_win) {
-    int64_t count = 0, lo = a;
-    while (lo < b) {
-        const int64_t w = (int64_t)in_src[lo] / sp.win_rows;
-        const int64_t hi = lower_bound_src(in_src, lo, b, (w + 1) * sp.win_rows);
-        for (int64_t e = lo; e < hi; e += sp.seg_len) {
-            if (FILL) {
-                seg_e0[slot + count] = e;
-                seg_e1[slot + count] = e + sp.seg_len < hi ? e + sp.seg_len : hi;
-                seg_win[slot + count] = (uint32_t)w;
-            }
-            ++count;
+__device__ int64_t warp_segments(const SplitParams &sp, const int32_t *__restrict__ in_src,
+                                 int64_t a, int64_t b, int64_t slot, int64_t *seg_e0,
+                                 int64_t *seg_e1, uint32_t *seg_win) {
+    const int lane = threadIdx.x & 31;
+    const int64_t w0 = (int64_t)in_src[a] / sp.win_rows, w1 = (int64_t)in_src[b - 1] / sp.win_rows;
+    int64_t base = 0;
+    for (int64_t wb = w0; wb <= w1; wb += 32) {
+        const int64_t w = wb + lane;
+        int64_t lo = 0, cnt = 0, hi = 0;
+        if (w <= w1) {
+            lo = w == w0 ? a : lower_bound_src(in_src, a, b, w * sp.win_rows);
+            hi = w == w1 ? b : lower_bound_src(in_src, lo, b, (w + 1) * sp.win_rows);
+            cnt = (hi - lo + sp.seg_len - 1) / sp.seg_len;
         }
-        lo = hi;
+        int64_t incl = cnt;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int64_t t = __shfl_up_sync(0xffffffffu, incl, o);
+            if (lane >= o) incl += t;
+        }
+        if (FILL) {
+            const int64_t at = slot + base + incl - cnt;
+            for (int64_t t = 0; t < cnt; ++t) {
+                const int64_t e = lo + t * sp.seg_len;
+                seg_e0[at + t] = e;
+                seg_e1[at + t] = e + sp.seg_len < hi ? e + sp.seg_len : hi;
+                seg_win[at + t] = (uint32_t)w;
+            }
+        }
+        base += __shfl_sync(0xffffffffu, incl, 31);
     }
-    return count;
+    return base;
 }
 
+// Segment count of every row (0 below split_t).  A warp takes 32 rows; its
+// hub rows are then cut one after another by the whole warp.
 __global__ void k_split_count(SplitParams sp, const int64_t *__restrict__ in_ptr,
                               const int32_t *__restrict__ in_src, int64_t n,
                               int64_t *__restrict__ nseg, int64_t *__restrict__ flag) {
-    for (int64_t j = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; j < n;
-         j += (int64_t)gridDim.x * blockDim.x) {
-        const int64_t a = in_ptr[j], b = in_ptr[j + 1];
-        const int64_t s = b - a > sp.split_t
-                              ? walk_segments<false>(sp, in_src, a, b, 0, nullptr, nullptr, nullptr)
-                              : 0;
-        nseg[j] = s;
-        flag[j] = s > 0;
+    const int lane = threadIdx.x & 31;
+    const int64_t nw = ((int64_t)gridDim.x * blockDim.x) >> 5;
+    for (int64_t r0 = (((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5) * 32; r0 < n;
+         r0 += nw * 32) {
+        const int64_t j = r0 + lane;
+        bool heavy = false;
+        if (j < n) {
+            heavy = in_ptr[j + 1] - in_ptr[j] > sp.split_t;
+            if (!heavy) {
+                nseg[j] = 0;
+                flag[j] = 0;
+            }
+        }
+        unsigned hv = __ballot_sync(0xffffffffu, heavy);
+        while (hv) {
+            const int l = __ffs(hv) - 1;
+            hv &= hv - 1;
+            const int64_t h = r0 + l;
+            const int64_t s = warp_segments<false>(sp, in_src, in_ptr[h], in_ptr[h + 1], 0, nullptr,
+                                                   nullptr, nullptr);
+            if (lane == 0) {
+                nseg[h] = s;
+                flag[h] = s > 0;
+            }
+        }
     }
 }
 
@@ -477,14 +544,24 @@ __global__ void k_split_fill(SplitParams sp, const int64_t *__restrict__ in_ptr,
                              const int64_t *__restrict__ split_idx, int32_t *__restrict__ split_row,
                              int64_t *__restrict__ split_slot0, int64_t *__restrict__ seg_e0,
                              int64_t *__restrict__ seg_e1, uint32_t *__restrict__ seg_win) {
-    for (int64_t j = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; j < n;
-         j += (int64_t)gridDim.x * blockDim.x) {
-        if (nseg[j] == 0) continue;
-        const int64_t idx = split_idx[j];
-        split_row[idx] = (int32_t)j;
-        split_slot0[idx] = slot_off[j];
-        walk_segments<true>(sp, in_src, in_ptr[j], in_ptr[j + 1], slot_off[j], seg_e0, seg_e1,
-                            seg_win);
+    const int lane = threadIdx.x & 31;
+    const int64_t nw = ((int64_t)gridDim.x * blockDim.x) >> 5;
+    for (int64_t r0 = (((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5) * 32; r0 < n;
+         r0 += nw * 32) {
+        const int64_t j = r0 + lane;
+        unsigned hv = __ballot_sync(0xffffffffu, j < n && nseg[j] > 0);
+        while (hv) {
+            const int l = __ffs(hv) - 1;
+            hv &= hv - 1;
+            const int64_t h = r0 + l;
+            if (lane == 0) {
+                const int64_t idx = split_idx[h];
+                split_row[idx] = (int32_t)h;
+                split_slot0[idx] = slot_off[h];
+            }
+            warp_segments<true>(sp, in_src, in_ptr[h], in_ptr[h + 1], slot_off[h], seg_e0, seg_e1,
+                                seg_win);
+        }
     }
 }
 
