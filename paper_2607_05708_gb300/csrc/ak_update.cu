@@ -90,9 +90,9 @@ akashic_status_t relate_top_m(const UpdateArgs &a, cudaStream_t st, int *launche
     const int64_t n_sample = ceil_div<int64_t>(n, stride);
     const int64_t cap = 4 * (int64_t)a.M * stride > 8192 ? 4 * (int64_t)a.M * stride : 8192;
     // the sample bounds of G column tiles come from one dots GEMM, one
-    // transpose and one k-th launch (G tiles of sampled dots: <= 256 MB)
+    // transpose and one k-th launch (G tiles of sampled dots: <= 512 MB)
     const int64_t tile_bytes = n_sample * 256 * 4;
-    int64_t G = ((int64_t)256 << 20) / tile_bytes;
+    int64_t G = ((int64_t)512 << 20) / tile_bytes;
     G = G < 1 ? 1 : (G > n_ct ? n_ct : G);
     SelectPlan sp = select_plan(n_sample, (int)G * 256, a.M, sms, 1);
     sp.cap = 0;                      // no candidate buffers: bounds only
