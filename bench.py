@@ -78,12 +78,13 @@ def hop_bytes(n, b, nnz):
     return (n + 1) * 8 + nnz * 8 + 2 * n * b * 4
 
 
-# DRAM bytes per propagation hop on this workload (sum over the hop's two
-# kernels: hub segments, then hub sums + rows kept whole), from an ncu capture of
+# DRAM bytes of one full propagation hop on this workload (the first hop:
+# hub segments 3.795 GB read + 0.361 GB written, then hub sums + rows kept
+# whole 5.948 + 1.060 GB), from an ncu capture of
 # `bench.py --steps 2 --warmup 1 --no-cpu-baseline` with the
-# dram__bytes_read/write counters (mean of the two hops).  Set to None when
-# the hop kernels change until they are captured again.
-HOP_DRAM_BYTES = 10.85e9
+# dram__bytes_read/write counters.  Set to None when the hop kernels change
+# until they are captured again.
+HOP_DRAM_BYTES = 11.16e9
 
 
 def score_bytes(n, d, b):
@@ -700,14 +701,17 @@ def run_retrieve(args, k=None, hops=None, metric=METRIC, workload=WORKLOAD, scop
     ab = algorithmic_bytes(wl.n, wl.dim, B, wl.nnz, hops, k)
     total_ab = sum(ab.values())
     per_step_ms = ms / args.steps
-    # dominant phase
-    names = {"score": None, "propagate": None, "select": None}
+    # dominant phase.  "propagate" holds the hops before the last (full
+    # hops); the last hop ("last_hop") skips the rows whose bound stays
+    # below the top-k floor, so its bytes are not a full hop's.
+    retr = ("score", "propagate", "last_hop", "bound", "select")
+    full_hops = hops - 1 if phases["last_hop"][0] > 0 else hops
     dom = max(("score", "propagate", "select"), key=lambda p: phases[p][0])
     dom_ms, dom_launches = phases[dom]
     if dom == "propagate":
         per_launch_bytes = hop_bytes(wl.n, 256, wl.nnz)
-        units = args.steps * hops
-        what = "propagation hop (graph once + two slab passes)"
+        units = args.steps * max(1, full_hops)
+        what = "full propagation hop (graph once + two slab passes)"
     elif dom == "score":
         per_launch_bytes = score_bytes(wl.n, wl.dim, 256)
         units = args.steps
@@ -745,7 +749,7 @@ def run_retrieve(args, k=None, hops=None, metric=METRIC, workload=WORKLOAD, scop
                           "frac": (total_ab / (hbm * 1e9) * 1e3) / per_step_ms,
                           "flops": 2.0 * wl.n * B * wl.dim,
                           "peak_tflops_bf16": bf16},
-        "phases_ms_per_step": {p: phases[p][0] / args.steps for p in ("score", "propagate", "select")},
+        "phases_ms_per_step": {p: phases[p][0] / args.steps for p in retr},
         "e2e": {"value": job_throughput(B * args.steps, ws, ms_e2e), "unit": "queries/s",
                 "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
         "gpu_launches": int(sum(v[1] for v in phases.values())),

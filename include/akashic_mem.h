@@ -251,7 +251,9 @@ enum {
     AKASHIC_PHASE_GRAPH = 4,     /* CSR insert, weights, transpose rebuild      */
     AKASHIC_PHASE_RELOCATE = 5,  /* co-retrieval counts + relocation            */
     AKASHIC_PHASE_COMPACT = 6,   /* block compaction                            */
-    AKASHIC_PHASE_COUNT = 7
+    AKASHIC_PHASE_BOUND = 7,     /* last hop's row bounds, floor and skip flags */
+    AKASHIC_PHASE_LAST_HOP = 8,  /* last hop with the top-k filter fused        */
+    AKASHIC_PHASE_COUNT = 9
 };
 akashic_status_t akashic_mem_set_profiling(akashic_mem_t *m, int32_t on);
 akashic_status_t akashic_mem_phase_times(akashic_mem_t *m, float *ms, int32_t *launches);

@@ -21,7 +21,8 @@ __all__ = ["MemStore", "AkashicError", "load_library", "build", "EXPORTS", "STAT
 
 STATUS = {0: "OK", 1: "EINVAL", 2: "ENOMEM", 3: "ECAPACITY", 4: "ECUDA", 5: "ETIMEOUT",
           6: "EDEVICE", 7: "ERANGE"}
-PHASES = ("score", "propagate", "select", "relate", "graph", "relocate", "compact")
+PHASES = ("score", "propagate", "select", "relate", "graph", "relocate", "compact", "bound",
+          "last_hop")
 
 # Every function declared in include/akashic_mem.h.
 EXPORTS = (

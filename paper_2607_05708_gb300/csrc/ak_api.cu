@@ -83,6 +83,9 @@ struct StreamScratch {
     DevBuf qp, shift, u, sa, sb, zpart, partial, cand, counters;
     DevBuf samp, ext_s, zsamp;   // retrieval without hops: the score's row sample
     DevBuf qns, ns_s, dead_s;    // scope: per query column, per sample row
+    DevBuf rmax_u, rmin_u;       // u's row maxima / minima over the real queries
+    DevBuf ub, lb, ext, pfloor;  // the last hop's row bounds, extremes, floor
+    DevBuf skip_split, skip_slot;
 };
 
 struct ProfRec {
@@ -135,8 +138,14 @@ struct akashic_mem {
     bool inc_transpose = true;   // relation updates patch the transpose instead of re-sorting
     SplitParams split;
     bool fuse_filter = true;     // top-k filter in the last hop's epilogue
+    bool hop_prune = true;       // last hop skips rows bounded below every filter threshold
     int64_t n_split = 0, n_segs = 0;
-    DevBuf split_row, split_slot0, seg_e0, seg_e1, seg_slot, split_order;
+    DevBuf split_row, split_slot0, seg_e0, seg_e1, seg_slot, split_order, slot_split;
+    // graph-only mass vectors of the last hop's row bounds, levels 0..mass_levels
+    // (recomputed lazily after the graph changes)
+    DevBuf mass_up, mass_dn, mass_zero, mass_vu, mass_vl;
+    int mass_levels = -1;
+    int64_t mass_n = -1;      // rows they were computed for
     std::mutex mu;
     std::unordered_map<void *, StreamScratch *> scratch;
     // profiling
@@ -353,6 +362,7 @@ static akashic_status_t rebuild_in_edges(akashic_mem *m, cudaStream_t st) {
 // order, split rows heaviest first.
 static akashic_status_t build_split_plan(akashic_mem *m, cudaStream_t st) {
     const int64_t n = m->n;
+    m->mass_levels = -1;   // the graph changed
     // temporaries from the store's scratch (slots SCR_SPLIT0..11)
     akashic_status_t sc_rc = AKASHIC_OK;
     auto get = [&](int i, size_t bytes) -> Tmp {
@@ -411,6 +421,9 @@ static akashic_status_t build_split_plan(akashic_mem *m, cudaStream_t st) {
                                   order2.as<uint32_t>(), n_split, 32, rtmp.p, rtmp.cap, st, &alt2));
         CUDA_TRY(cudaMemcpyAsync(m->split_order.p, alt2 ? order2.p : order.p, (size_t)n_split * 4,
                                  cudaMemcpyDeviceToDevice, st));
+        AK_TRY(m->slot_split.ensure((size_t)n_segs * 4));
+        CUDA_TRY(launch_slot_owner(m->split_slot0.as<int64_t>(), n_split,
+                                   m->slot_split.as<int32_t>(), st));
         AK_TRY(check_status(m, st, "relation graph rebuild"));
     }
     return check_status(m, st, "relation graph rebuild");
@@ -452,6 +465,7 @@ akashic_status_t akashic_mem_create(const akashic_mem_config_t *cfg, akashic_mem
     if (const char *v = getenv("AKASHIC_SPLIT_T")) m->split.split_t = atoll(v) > 0 ? atoll(v) : m->split.split_t;
     if (const char *v = getenv("AKASHIC_SEG_LEN")) m->split.seg_len = atoll(v) > 0 ? atoll(v) : m->split.seg_len;
     if (const char *v = getenv("AKASHIC_FUSE_FILTER")) m->fuse_filter = atoi(v) != 0;
+    if (const char *v = getenv("AKASHIC_HOP_PRUNE")) m->hop_prune = atoi(v) != 0;
     if (const char *v = getenv("AKASHIC_FULL_TRANSPOSE")) m->inc_transpose = atoi(v) == 0;
     if (const char *v = getenv("AKASHIC_WIN_ROWS")) m->split.win_rows = atoll(v) > 0 ? atoll(v) : m->split.win_rows;
     akashic_status_t s;
@@ -1008,6 +1022,31 @@ akashic_status_t akashic_mem_export_pages(akashic_mem_t *m, int32_t *page_of, vo
 }
 }  // extern "C"
 
+// Mass levels 0..H of the row bounds (level 0 all ones), extended as needed.
+static akashic_status_t ensure_mass(akashic_mem *m, const HopPlan &hp, int H, cudaStream_t st) {
+    const int64_t n = m->n;
+    if (m->mass_n != n) m->mass_levels = -1;
+    if (m->mass_levels >= H) return AKASHIC_OK;
+    const size_t lv = (size_t)(H + 1) * n * 4;
+    if (m->mass_levels < 0 || m->mass_up.cap < lv) {
+        AK_TRY(m->mass_up.ensure(lv));
+        AK_TRY(m->mass_dn.ensure(lv));
+        AK_TRY(m->mass_zero.ensure((size_t)n * 4));
+        AK_TRY(m->mass_vu.ensure((size_t)(m->n_split + 1) * 4));
+        AK_TRY(m->mass_vl.ensure((size_t)(m->n_split + 1) * 4));
+        CUDA_TRY(cudaMemsetAsync(m->mass_zero.p, 0, (size_t)n * 4, st));
+        CUDA_TRY(launch_fill_f32(m->mass_up.as<float>(), n, 1.f, st));
+        CUDA_TRY(launch_fill_f32(m->mass_dn.as<float>(), n, 1.f, st));
+        m->mass_levels = 0;
+        m->mass_n = n;
+    }
+    CUDA_TRY(launch_mass_levels(hp, m->mass_levels + 1, H, m->mass_up.as<float>(),
+                                m->mass_dn.as<float>(), m->mass_zero.as<float>(),
+                                m->mass_vu.as<float>(), m->mass_vl.as<float>(), st));
+    m->mass_levels = H;
+    return AKASHIC_OK;
+}
+
 static akashic_status_t retrieve_impl(akashic_mem *m, const uint16_t *q, int32_t B, int32_t k,
                                       float alpha, int32_t hops, const int32_t *q_ns,
                                       int32_t sort_by_time, int64_t *ids, float *scores,
@@ -1042,6 +1081,18 @@ static akashic_status_t retrieve_impl(akashic_mem *m, const uint16_t *q, int32_t
         if (eff_hops >= 2) AK_TRY(sc->sb.ensure((size_t)n * bp * 4));
         if (eff_hops >= 1 && m->n_segs > 0) AK_TRY(sc->partial.ensure((size_t)m->n_segs * bp * 4));
         if (eff_hops >= 1) AK_TRY(sc->counters.ensure(64));
+        // row bounds for the last hop (fused filter only)
+        const bool prune = eff_hops >= 1 && m->fuse_filter && m->hop_prune;
+        if (prune) {
+            AK_TRY(sc->rmax_u.ensure((size_t)n * 4));
+            AK_TRY(sc->rmin_u.ensure((size_t)n * 4));
+            AK_TRY(sc->ub.ensure((size_t)n * 4));
+            AK_TRY(sc->lb.ensure((size_t)n * 4));
+            AK_TRY(sc->ext.ensure(16));
+            AK_TRY(sc->skip_split.ensure((size_t)(m->n_split + 1) * 4));
+            AK_TRY(sc->skip_slot.ensure((size_t)(m->n_segs + 1) * 4));
+            AK_TRY(sc->pfloor.ensure(16));
+        }
         const uint16_t *qb = q + (int64_t)off * m->dim;
         // namespace scope of this batch's queries (padding columns get -1)
         NsScope ns{};
@@ -1071,7 +1122,9 @@ static akashic_status_t retrieve_impl(akashic_mem *m, const uint16_t *q, int32_t
                 CUDA_TRY(launch_score(m->emb.as<uint16_t>(), n, m->dim, sc->qp.as<uint16_t>(), bp,
                                       sc->shift.as<float>(), m->tau, sc->u.as<float>(),
                                       sc->zpart.as<float>(), m->status.as<int>(), st,
-                                      &ph.launches, &zrows, ns.dead));
+                                      &ph.launches, &zrows, ns.dead,
+                                      prune ? sc->rmax_u.as<float>() : nullptr,
+                                      prune ? sc->rmin_u.as<float>() : nullptr, b));
         }
         if (dense_fused) {
             {
@@ -1133,12 +1186,26 @@ static akashic_status_t retrieve_impl(akashic_mem *m, const uint16_t *q, int32_t
             hp.seg_e1 = m->seg_e1.as<int64_t>();
             hp.seg_slot = m->seg_slot.as<int32_t>();
             hp.split_order = m->split_order.as<int32_t>();
+            hp.slot_split = m->slot_split.as<int32_t>();
             float *bufs[2] = {sc->sa.as<float>(), sc->sb.as<float>()};
             rc.u = sc->u.as<float>();
             rc.in_ptr = hp.in_ptr;
             rc.in_src = hp.in_src;
             rc.in_w = hp.in_w;
             rc.alpha = alpha;
+            // scalar row bounds of the last hop's output, from u's row extremes
+            const float *row_ub = nullptr, *row_lb = nullptr;
+            if (prune) {
+                PhaseScope ph(m, AKASHIC_PHASE_BOUND, st);
+                AK_TRY(ensure_mass(m, hp, eff_hops, st));
+                CUDA_TRY(launch_final_bounds(sc->rmax_u.as<float>(), sc->rmin_u.as<float>(),
+                                             m->mass_up.as<float>(), m->mass_dn.as<float>(), n,
+                                             eff_hops, alpha, sc->ext.as<unsigned int>(),
+                                             sc->ub.as<float>(), sc->lb.as<float>(), st,
+                                             &ph.launches));
+                row_ub = sc->ub.as<float>();
+                row_lb = sc->lb.as<float>();
+            }
             for (int h = 0; h < eff_hops; ++h) {
                 float *out = bufs[h & 1];
                 const bool last = m->fuse_filter && h == eff_hops - 1;
@@ -1148,17 +1215,37 @@ static akashic_status_t retrieve_impl(akashic_mem *m, const uint16_t *q, int32_t
                     // too (same summation order, monotone rounding), so the
                     // k-th largest key of s^(H-1) over the row sample is a
                     // safe bound for s^(H).
-                    PhaseScope ps(m, AKASHIC_PHASE_SELECT, st);
-                    CUDA_TRY(launch_sample_bound(sp, fin, b, m->ext_of.as<int32_t>(), ws, st,
-                                                 &ps.launches, 0u, ns));
+                    {
+                        PhaseScope ps(m, AKASHIC_PHASE_SELECT, st);
+                        CUDA_TRY(launch_sample_bound(sp, fin, b, m->ext_of.as<int32_t>(), ws, st,
+                                                     &ps.launches, 0u, ns));
+                    }
+                    if (prune) {
+                        PhaseScope ps(m, AKASHIC_PHASE_BOUND, st);
+                        // floor: the filter bounds', raised without a namespace
+                        // scope to the k-th largest lower bound of the heaviest
+                        // split rows (where the top scores lie)
+                        const int64_t n_lb = m->n_split < 1024 ? m->n_split : 1024;
+                        CUDA_TRY(launch_prune_floor(ws + sp.off_bound, b, row_lb,
+                                                    q_ns ? nullptr : hp.split_row,
+                                                    hp.split_order, n_lb, k,
+                                                    sc->pfloor.as<float>(), st));
+                        CUDA_TRY(launch_split_flags(hp, row_ub, sc->pfloor.as<float>(),
+                                                    sc->skip_split.as<int32_t>(),
+                                                    sc->skip_slot.as<int32_t>(), st));
+                        ps.launches += 1 + (m->n_split > 0);
+                    }
                 }
                 const HopFilter flt{m->ext_of.as<int32_t>(), ws + sp.off_bound,
                                     (unsigned int *)(ws + sp.off_cnt), ws + sp.off_buf, sp.cap,
                                     ns};
-                PhaseScope ph(m, AKASHIC_PHASE_PROPAGATE, st);
+                const HopBound hb{row_ub, sc->pfloor.as<float>(), sc->skip_split.as<int32_t>(),
+                                  sc->skip_slot.as<int32_t>()};
+                PhaseScope ph(m, last ? AKASHIC_PHASE_LAST_HOP : AKASHIC_PHASE_PROPAGATE, st);
                 CUDA_TRY(launch_hop(hp, sc->u.as<float>(), fin, out, bp, alpha,
                                     sc->partial.as<float>(), sc->counters.as<int>(),
-                                    last ? &flt : nullptr, st, &ph.launches));
+                                    last ? &flt : nullptr, st, &ph.launches,
+                                    (last && prune) ? &hb : nullptr));
                 if (last) {
                     rc.kind = 1;
                     rc.prev = fin;

@@ -77,10 +77,14 @@ void set_last_error(const char *msg);
 // for r < *zrows.  score_tiles(n) bounds *zrows.
 int64_t score_tiles(int64_t n);
 // dead_row (or NULL): rows of deleted chunks score u = 0 (no part in Z).
+// row_max / row_min (optional, together): [n] the largest and smallest u of
+// each row over the first n_real columns (the real queries), for the
+// propagation's row bounds.
 cudaError_t launch_score(const uint16_t *emb, int64_t n, int dim, const uint16_t *qp, int bp,
                          const float *shift, float tau, float *u, float *zpart, int *status,
                          cudaStream_t st, int *launches, int *zrows,
-                         const int32_t *dead_row = nullptr);
+                         const int32_t *dead_row = nullptr, float *row_max = nullptr,
+                         float *row_min = nullptr, int n_real = 0);
 
 // The score on every stride-th row only: out[v, c] = u[v*stride, c] for
 // v < n_sample (same kernel and arithmetic as launch_score, so the values
@@ -338,6 +342,7 @@ struct HopPlan {
     const int64_t *seg_e1;      // [n_segs] end edge
     const int32_t *seg_slot;    // [n_segs] partial slot (segments of a row are contiguous)
     const int32_t *split_order; // [n_split_rows] split rows by slot count, largest first
+    const int32_t *slot_split;  // [n_segs] split row owning each partial slot
 };
 // Top-k filter fused into a hop's output: every written value whose key
 // (score bits, ~chunk ID) is >= bound[column] is appended to that column's
@@ -350,11 +355,57 @@ struct HopFilter {
     int64_t cap;
     NsScope ns;                       // candidates only within the query's namespace
 };
+// Row bounds for the last hop, whose output only feeds the fused top-k
+// filter: row_ub[j] bounds every real query column's fp32 value of the
+// hop's output s_j from above (launch_row_bounds), `floor` is at most every
+// real query's k-th largest final value (launch_prune_floor); a row with
+// row_ub < floor appends nothing in any column and is skipped, so the
+// filter's output is unchanged.
+struct HopBound {
+    const float *row_ub;       // [n]
+    const float *floor;        // device scalar
+    const int32_t *split_skip; // [n_split_rows] split rows to skip (launch_split_flags)
+    const int32_t *slot_skip;  // [n_segs] their partial slots
+};
+// Graph-only mass vectors for the row bounds, levels t0..t1 (level 0, all
+// ones, already in place): mup[t] >= g (1 + eps) sum_i w_ij mup[t-1]_i and
+// mdn[t] <= g' (1 - eps) sum_i w_ij mdn[t-1]_i, g / g' the rounding growth of
+// a hop's sum over the row's edges.  mup / mdn are [levels + 1][n];
+// `zeros` is [n]; split_vu/vl [n_split_rows] scratch.  With them, for every
+// real query column (U0 / L0 u's row maxima / minima, Umax / Lmin their
+// extremes over the live rows):
+//   s^(H)_j <= (U0_j + Umax sum_{t<=H} alpha^t mup[t]_j) (1 + eps),
+//   s^(H)_j >= (L0_j + Lmin sum_{t<=H} alpha^t mdn[t]_j) (1 - eps)
+// (by induction over the hops: every source's value lies in
+// [Lmin (1 + ...), Umax (1 + ...)]).
+cudaError_t launch_mass_levels(const HopPlan &p, int t0, int t1, float *mup, float *mdn,
+                               const float *zeros, float *split_vu, float *split_vl,
+                               cudaStream_t st);
+// Per call: ub / lb [n] from u's row extremes u0 / l0 and the mass levels
+// 1..H; ext is [2] device scratch.
+cudaError_t launch_final_bounds(const float *u0, const float *l0, const float *mup,
+                                const float *mdn, int64_t n, int H, float alpha,
+                                unsigned int *ext, float *ub, float *lb, cudaStream_t st,
+                                int *launches);
+cudaError_t launch_split_flags(const HopPlan &p, const float *row_ub, const float *floor_p,
+                               int32_t *split_skip, int32_t *slot_skip, cudaStream_t st);
+// floor = max(the smallest score any real column's filter bound admits,
+// and, if lb_rows != NULL, the k-th largest lb over the rows
+// lb_rows[order[i]], i < n_lb_rows), written to floor_out.  The second term
+// is only valid when every row may be selected by every query (no namespace
+// scope).
+cudaError_t launch_prune_floor(const unsigned long long *bound, int n_real, const float *lb,
+                               const int32_t *lb_rows, const int32_t *order, int64_t n_lb_rows,
+                               int k, float *floor_out, cudaStream_t st);
+cudaError_t launch_fill_f32(float *v, int64_t n, float x, cudaStream_t st);
+// slot_split[s] = r for every partial slot s of split row r.
+cudaError_t launch_slot_owner(const int64_t *split_slot0, int64_t n_split, int32_t *slot_split,
+                              cudaStream_t st);
 // `counters` = 2 device ints, zeroed by the launcher (work queues).
-// `flt` may be NULL (no filter).
+// `flt` may be NULL (no filter), `hb` NULL (no row bounds).
 cudaError_t launch_hop(const HopPlan &p, const float *u, const float *in, float *out, int bp,
                        float alpha, float *partial, int *counters, const HopFilter *flt,
-                       cudaStream_t st, int *launches);
+                       cudaStream_t st, int *launches, const HopBound *hb = nullptr);
 
 // ------------------------------------------------------------------ selection
 // Top-k of every column of a slab (a3): bound from a row sample, filter

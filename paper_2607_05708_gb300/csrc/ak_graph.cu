@@ -744,6 +744,289 @@ __device__ __forceinline__ void hop_accumulate(const int32_t *__restrict__ in_sr
     }
 }
 
+// ------------------------------------------------------------------ row bounds
+// Scalar bounds on the hops' fp32 values, one pair per row: U[j] is at least
+// and L[j] at most every real query column's value of s^(h)_j.  Level 0 is
+// u's row maximum / minimum (from the score step); level h follows the hop
+// s^(h)_j = fma(alpha, sum_{i->j} w_ij s^(h-1)_i, u_j) with the sums of
+// w * U and w * L over the row's in-edges (w, s >= 0), widened for rounding:
+// the hop's sum takes at most 2n + 10 roundings on any term's path
+// (segments and partial slots included) and the bound's own sum at most
+// n + 5, so exp(+-x), x = 3.25 (n + 8) 2^-24, covers both (with 1 + x + x^2
+// >= exp(x) and 1 - x <= exp(-x) for 0 <= x <= 1), and a factor 1 -+ 4e-6
+// (~67 ulp) covers the final rounding of the hop and of evaluating the
+// bound in fp32.
+__device__ __forceinline__ float bound_x(int64_t n) {
+    return 3.25f * (float)(n + 8) * 5.9604645e-8f;
+}
+__device__ __forceinline__ float bound_up(float u0, float v, int64_t n, float alpha) {
+    const float x = bound_x(n);
+    if (!(x <= 1.f)) return INFINITY;
+    return fmaf(alpha * v, 1.f + x + x * x, u0) * (1.f + 4e-6f);
+}
+__device__ __forceinline__ float bound_dn(float l0, float v, int64_t n, float alpha) {
+    const float x = bound_x(n);
+    const float g = x < 1.f ? 1.f - x : 0.f;
+    return fmaf(alpha * v, g, l0) * (1.f - 4e-6f);
+}
+
+// The sums of w * U[source] and w * L[source] over in-edges e0..e1, by a
+// group of LN lanes (lane `sl` of the group), four edges in flight per lane;
+// every lane of the group returns them.
+template <int LN>
+__device__ __forceinline__ void bound_sums(const int32_t *__restrict__ in_src,
+                                           const float *__restrict__ in_w, int64_t e0, int64_t e1,
+                                           const float *__restrict__ U, const float *__restrict__ L,
+                                           int sl, float &vu, float &vl) {
+    vu = 0.f;
+    vl = 0.f;
+    for (int64_t eb = e0 + sl; eb < e1; eb += 4 * LN) {
+        int32_t s[4];
+        float w[4];
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            const int64_t e = eb + LN * q;
+            s[q] = e < e1 ? __ldcs(in_src + e) : 0;
+            w[q] = e < e1 ? __ldcs(in_w + e) : 0.f;
+        }
+        float a[4], c[4];
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            const bool in = eb + LN * q < e1;
+            a[q] = in ? __ldg(U + s[q]) : 0.f;
+            c[q] = in ? __ldg(L + s[q]) : 0.f;
+        }
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            vu = fmaf(w[q], a[q], vu);
+            vl = fmaf(w[q], c[q], vl);
+        }
+    }
+#pragma unroll
+    for (int off = LN / 2; off > 0; off >>= 1) {
+        vu += __shfl_xor_sync(0xffffffffu, vu, off);
+        vl += __shfl_xor_sync(0xffffffffu, vl, off);
+    }
+}
+
+// One level for the rows kept whole: four lanes per row, eight rows per warp.
+constexpr int BND_LANES = 4;
+__global__ void k_bound_rows(const int64_t *__restrict__ in_ptr, const int32_t *__restrict__ in_src,
+                             const float *__restrict__ in_w, int64_t n, int64_t split_t,
+                             const float *__restrict__ u0, const float *__restrict__ l0,
+                             const float *__restrict__ Up, const float *__restrict__ Lp,
+                             float alpha, float *__restrict__ Un, float *__restrict__ Ln) {
+    constexpr int R = 32 / BND_LANES;
+    const int lane = threadIdx.x & 31, sl = lane % BND_LANES, grp = lane / BND_LANES;
+    const int64_t nw = ((int64_t)gridDim.x * blockDim.x) >> 5;
+    for (int64_t r0 = (((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5) * R; r0 < n;
+         r0 += nw * R) {
+        const int64_t j = r0 + grp;
+        int64_t e0 = 0, e1 = 0;
+        if (j < n) {
+            e0 = in_ptr[j];
+            e1 = in_ptr[j + 1];
+        }
+        const bool whole = j < n && e1 - e0 <= split_t;
+        float vu, vl;
+        bound_sums<BND_LANES>(in_src, in_w, e0, whole ? e1 : e0, Up, Lp, sl, vu, vl);
+        if (whole && sl == 0) {
+            Un[j] = bound_up(u0[j], vu, e1 - e0, alpha);
+            Ln[j] = bound_dn(l0[j], vl, e1 - e0, alpha);
+        }
+    }
+}
+
+// Split rows: one warp per segment, its sums added into the owning row's
+// totals (the order of the additions does not change the bound: every
+// term is >= 0 and a term's path stays within the row's edge count + 5
+// roundings) ...
+__global__ void k_seg_bound(const int64_t *__restrict__ seg_e0, const int64_t *__restrict__ seg_e1,
+                            const int32_t *__restrict__ seg_slot, int64_t n_segs,
+                            const int32_t *__restrict__ slot_split,
+                            const int32_t *__restrict__ in_src, const float *__restrict__ in_w,
+                            const float *__restrict__ Up, const float *__restrict__ Lp,
+                            float *__restrict__ split_vu, float *__restrict__ split_vl) {
+    const int lane = threadIdx.x & 31;
+    const int64_t nw = ((int64_t)gridDim.x * blockDim.x) >> 5;
+    for (int64_t s = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5; s < n_segs; s += nw) {
+        float vu, vl;
+        bound_sums<32>(in_src, in_w, seg_e0[s], seg_e1[s], Up, Lp, lane, vu, vl);
+        if (lane == 0) {
+            const int32_t r = slot_split[seg_slot[s]];
+            atomicAdd(split_vu + r, vu);
+            atomicAdd(split_vl + r, vl);
+        }
+    }
+}
+
+// ... then each split row's bounds.
+__global__ void k_split_bound(const int64_t *__restrict__ in_ptr, int64_t n_split,
+                              const int32_t *__restrict__ split_row,
+                              const float *__restrict__ u0, const float *__restrict__ l0,
+                              const float *__restrict__ split_vu, const float *__restrict__ split_vl,
+                              float alpha, float *__restrict__ Un, float *__restrict__ Ln) {
+    for (int64_t r = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; r < n_split;
+         r += (int64_t)gridDim.x * blockDim.x) {
+        const int64_t j = split_row[r];
+        const int64_t n = in_ptr[j + 1] - in_ptr[j];
+        Un[j] = bound_up(u0[j], split_vu[r], n, alpha);
+        Ln[j] = bound_dn(l0[j], split_vl[r], n, alpha);
+    }
+}
+
+// Last hop: split rows whose bound stays below the floor, and their partial
+// slots (the segment kernel skips those).  One warp per row.
+__global__ void k_split_flags(int64_t n_split, const int32_t *__restrict__ split_row,
+                              const int64_t *__restrict__ split_slot0,
+                              const float *__restrict__ row_ub, const float *__restrict__ floor_p,
+                              int32_t *__restrict__ split_skip, int32_t *__restrict__ slot_skip) {
+    const float floor_ = *floor_p;
+    const int lane = threadIdx.x & 31;
+    const int64_t nw = ((int64_t)gridDim.x * blockDim.x) >> 5;
+    for (int64_t r = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5; r < n_split; r += nw) {
+        const int32_t skip = row_ub[split_row[r]] < floor_ ? 1 : 0;
+        if (lane == 0) split_skip[r] = skip;
+        for (int64_t s = split_slot0[r] + lane; s < split_slot0[r + 1]; s += 32) slot_skip[s] = skip;
+    }
+}
+
+__global__ void k_slot_owner(const int64_t *__restrict__ split_slot0, int64_t n_split,
+                             int32_t *__restrict__ slot_split) {
+    const int lane = threadIdx.x & 31;
+    const int64_t nw = ((int64_t)gridDim.x * blockDim.x) >> 5;
+    for (int64_t r = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5; r < n_split; r += nw)
+        for (int64_t s = split_slot0[r] + lane; s < split_slot0[r + 1]; s += 32)
+            slot_split[s] = (int32_t)r;
+}
+
+__global__ void k_fill_f32(float *__restrict__ v, int64_t n, float x) {
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n;
+         i += (int64_t)gridDim.x * blockDim.x)
+        v[i] = x;
+}
+
+cudaError_t launch_fill_f32(float *v, int64_t n, float x, cudaStream_t st) {
+    if (n <= 0) return cudaSuccess;
+    k_fill_f32<<<device_sm_count() * 2, 256, 0, st>>>(v, n, x);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_slot_owner(const int64_t *split_slot0, int64_t n_split, int32_t *slot_split,
+                              cudaStream_t st) {
+    if (n_split <= 0) return cudaSuccess;
+    k_slot_owner<<<device_sm_count() * 4, 256, 0, st>>>(split_slot0, n_split, slot_split);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_mass_levels(const HopPlan &p, int t0, int t1, float *mup, float *mdn,
+                               const float *zeros, float *split_vu, float *split_vl,
+                               cudaStream_t st) {
+    const int sms = device_sm_count();
+    const int64_t n = p.n;
+    for (int t = t0; t <= t1; ++t) {
+        const float *Up = mup + (int64_t)(t - 1) * n, *Lp = mdn + (int64_t)(t - 1) * n;
+        float *Un = mup + (int64_t)t * n, *Ln = mdn + (int64_t)t * n;
+        const int64_t want = ceil_div<int64_t>(n, 32);
+        const int g = (int)(want < (int64_t)sms * 8 ? (want < 1 ? 1 : want) : (int64_t)sms * 8);
+        k_bound_rows<<<g, 256, 0, st>>>(p.in_ptr, p.in_src, p.in_w, n, p.split.split_t, zeros,
+                                         zeros, Up, Lp, 1.f, Un, Ln);
+        cudaError_t e = cudaGetLastError();
+        if (e != cudaSuccess) return e;
+        if (p.n_split_rows > 0) {
+            e = cudaMemsetAsync(split_vu, 0, (size_t)p.n_split_rows * 4, st);
+            if (e == cudaSuccess) e = cudaMemsetAsync(split_vl, 0, (size_t)p.n_split_rows * 4, st);
+            if (e != cudaSuccess) return e;
+            const int64_t ws = ceil_div<int64_t>(p.n_segs, 8);
+            const int gs = (int)(ws < (int64_t)sms * 8 ? (ws < 1 ? 1 : ws) : (int64_t)sms * 8);
+            k_seg_bound<<<gs, 256, 0, st>>>(p.seg_e0, p.seg_e1, p.seg_slot, p.n_segs,
+                                            p.slot_split, p.in_src, p.in_w, Up, Lp, split_vu,
+                                            split_vl);
+            const int64_t wr = ceil_div<int64_t>(p.n_split_rows, 256);
+            const int gr = (int)(wr < (int64_t)sms * 2 ? wr : (int64_t)sms * 2);
+            k_split_bound<<<gr, 256, 0, st>>>(p.in_ptr, p.n_split_rows, p.split_row, zeros, zeros,
+                                              split_vu, split_vl, 1.f, Un, Ln);
+            e = cudaGetLastError();
+            if (e != cudaSuccess) return e;
+        }
+    }
+    return cudaSuccess;
+}
+
+// The store-wide extremes of u's row maxima and (over rows with u > 0, i.e.
+// live rows, the only possible edge sources) row minima: ext[0] = Umax,
+// ext[1] = Lmin, as float bits (values >= 0 order like their bits).
+__global__ void k_ext_init(unsigned int *ext) {
+    ext[0] = 0u;
+    ext[1] = 0x7f800000u;
+}
+__global__ void k_row_extremes(const float *__restrict__ u0, const float *__restrict__ l0,
+                               int64_t n, unsigned int *__restrict__ ext) {
+    unsigned int mx = 0u, mn = 0x7f800000u;
+    for (int64_t j = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; j < n;
+         j += (int64_t)gridDim.x * blockDim.x) {
+        const unsigned int a = __float_as_uint(u0[j]);
+        mx = a > mx ? a : mx;
+        if (a > 0u) {
+            const unsigned int b = __float_as_uint(l0[j]);
+            mn = b < mn ? b : mn;
+        }
+    }
+    for (int off = 16; off > 0; off >>= 1) {
+        const unsigned int x = __shfl_xor_sync(0xffffffffu, mx, off);
+        const unsigned int y = __shfl_xor_sync(0xffffffffu, mn, off);
+        mx = x > mx ? x : mx;
+        mn = y < mn ? y : mn;
+    }
+    if ((threadIdx.x & 31) == 0) {
+        atomicMax(ext, mx);
+        atomicMin(ext + 1, mn);
+    }
+}
+
+// ub_j = (U0_j + Umax * sum_t alpha^t Mup[t]_j) (1 + 1e-5) and
+// lb_j = (L0_j + Lmin * sum_t alpha^t Mdn[t]_j) (1 - 1e-5): the (1 +- eps) of
+// the hop's last rounding and the at most ~3H roundings of this evaluation
+// (Horner, alpha^t) stay far below the 1e-5 (~168 eps) for H <= 16.
+__global__ void k_final_bounds(const float *__restrict__ u0, const float *__restrict__ l0,
+                               const float *__restrict__ mup, const float *__restrict__ mdn,
+                               int64_t n, int H, float alpha, const unsigned int *__restrict__ ext,
+                               float *__restrict__ ub, float *__restrict__ lb) {
+    const float umax = __uint_as_float(ext[0]), lmin = __uint_as_float(ext[1]);
+    for (int64_t j = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; j < n;
+         j += (int64_t)gridDim.x * blockDim.x) {
+        float cu = 0.f, cl = 0.f;
+        for (int t = H; t >= 1; --t) {
+            cu = alpha * (cu + __ldg(mup + (int64_t)t * n + j));
+            cl = alpha * (cl + __ldg(mdn + (int64_t)t * n + j));
+        }
+        ub[j] = fmaf(umax, cu, u0[j]) * (1.f + 1e-5f);
+        lb[j] = lmin < INFINITY ? fmaf(lmin, cl, l0[j]) * (1.f - 1e-5f) : 0.f;
+    }
+}
+
+cudaError_t launch_final_bounds(const float *u0, const float *l0, const float *mup,
+                                const float *mdn, int64_t n, int H, float alpha,
+                                unsigned int *ext, float *ub, float *lb, cudaStream_t st,
+                                int *launches) {
+    const int sms = device_sm_count();
+    k_ext_init<<<1, 1, 0, st>>>(ext);
+    k_row_extremes<<<sms * 4, 256, 0, st>>>(u0, l0, n, ext);
+    k_final_bounds<<<sms * 4, 256, 0, st>>>(u0, l0, mup, mdn, n, H, alpha, ext, ub, lb);
+    if (launches) *launches += 3;
+    return cudaGetLastError();
+}
+
+cudaError_t launch_split_flags(const HopPlan &p, const float *row_ub, const float *floor_p,
+                               int32_t *split_skip, int32_t *slot_skip, cudaStream_t st) {
+    if (p.n_split_rows <= 0) return cudaSuccess;
+    const int64_t want = ceil_div<int64_t>(p.n_split_rows, 8);
+    const int g = (int)(want < (int64_t)device_sm_count() * 4 ? want : (int64_t)device_sm_count() * 4);
+    k_split_flags<<<g, 256, 0, st>>>(p.n_split_rows, p.split_row, p.split_slot0, row_ub, floor_p,
+                                     split_skip, slot_skip);
+    return cudaGetLastError();
+}
+
 // A split row: out = u + alpha * (sum of its partial slots a..b-1), summed
 // by one warp in slot order (lane groups take alternate slots and are
 // added in group order), so the result does not depend on scheduling.
@@ -868,13 +1151,20 @@ __global__ __launch_bounds__(256, 3) void k_hop_rows(const int64_t *__restrict__
                                                   const int32_t *__restrict__ split_row,
                                                   const int64_t *__restrict__ split_slot0,
                                                   const float4 *__restrict__ part4,
-                                                  HopFilter f, int *__restrict__ queue) {
+                                                  HopFilter f,
+                                                  const float *__restrict__ row_ub,
+                                                  const float *__restrict__ floor_p,
+                                                  const int32_t *__restrict__ split_skip,
+                                                  int *__restrict__ queue) {
     using S = HopShape<BP>;
     const int lane = threadIdx.x & 31;
     const int sub = lane % S::LW;
     const int64_t groups = (n + ROWS_PER_GRAB - 1) / ROWS_PER_GRAB;
     __shared__ unsigned long long thr[FILTER ? BP : 1];
     __shared__ uint4 thr_hi[FILTER ? BP / 4 : 1];
+    // last hop: rows whose bound stays below the floor append nothing
+    const bool prune = FILTER && row_ub != nullptr;
+    const float floor_ = prune ? *floor_p : 0.f;
     if constexpr (FILTER) {
         for (int c = threadIdx.x; c < BP; c += blockDim.x) {
             const unsigned long long t = f.bound[c];
@@ -890,6 +1180,7 @@ __global__ __launch_bounds__(256, 3) void k_hop_rows(const int64_t *__restrict__
         if (it >= n_split + groups) break;
         if (it < n_split) {
             const int32_t r = split_order[it];
+            if (prune && split_skip[r]) continue;
             hop_fixup_row<BP, FILTER>(split_row[r], split_slot0[r], split_slot0[r + 1], part4,
                                       u4, out4, alpha, f, thr, thr_hi);
             continue;
@@ -907,6 +1198,7 @@ __global__ __launch_bounds__(256, 3) void k_hop_rows(const int64_t *__restrict__
             const uint32_t id = FILTER ? (uint32_t)__shfl_sync(0xffffffffu, ids, r) : 0u;
             if (e1 - e0 > split_t) continue;
             const int64_t j = j0 + r;
+            if (prune && __ldg(row_ub + j) < floor_) continue;
             float4 b[S::V];
             if (lane < S::LW) {
 #pragma unroll
@@ -939,6 +1231,7 @@ __global__ __launch_bounds__(256, 3) void k_hop_segs(const int64_t *__restrict__
                                                   const float *__restrict__ in_w,
                                                   const float4 *__restrict__ in4,
                                                   float4 *__restrict__ part4,
+                                                  const int32_t *__restrict__ slot_skip,
                                                   int *__restrict__ queue) {
     using S = HopShape<BP>;
     const int lane = threadIdx.x & 31;
@@ -948,9 +1241,10 @@ __global__ __launch_bounds__(256, 3) void k_hop_segs(const int64_t *__restrict__
         if (lane == 0) s = atomicAdd(queue, 1);
         s = __shfl_sync(0xffffffffu, s, 0);
         if (s >= n_segs) break;
+        const int64_t slot = seg_slot[s];
+        if (slot_skip && slot_skip[slot]) continue;   // its row is pruned
         float4 acc[S::V];
         hop_accumulate<BP>(in_src, in_w, seg_e0[s], seg_e1[s], in4, acc);
-        const int64_t slot = seg_slot[s];
         if (lane < S::LW) {
 #pragma unroll
             for (int v = 0; v < S::V; ++v) st_stream(part4 + slot * S::F + sub + 32 * v, acc[v]);
@@ -961,8 +1255,11 @@ __global__ __launch_bounds__(256, 3) void k_hop_segs(const int64_t *__restrict__
 template <int BP>
 static cudaError_t hop_bp(const HopPlan &p, const float *u, const float *in, float *out,
                           float alpha, float *partial, int *counters, const HopFilter *flt,
-                          cudaStream_t st, int *launches) {
+                          cudaStream_t st, int *launches, const HopBound *hbp) {
     const int sms = device_sm_count();
+    // the last hop skips rows whose bound stays below the filter floor
+    const bool prune = flt && hbp && hbp->row_ub && hbp->floor &&
+                       (p.n_split_rows == 0 || (hbp->split_skip && hbp->slot_skip));
     cudaError_t e = cudaMemsetAsync(counters, 0, 2 * sizeof(int), st);
     if (e != cudaSuccess) return e;
     if (p.n_segs > 0) {
@@ -970,7 +1267,7 @@ static cudaError_t hop_bp(const HopPlan &p, const float *u, const float *in, flo
         const int g2 = (int)(want < (int64_t)sms * 3 ? want : (int64_t)sms * 3);
         k_hop_segs<BP><<<g2, 256, 0, st>>>(p.seg_e0, p.seg_e1, p.seg_slot, p.n_segs, p.in_src,
                                            p.in_w, (const float4 *)in, (float4 *)partial,
-                                           counters + 1);
+                                           prune ? hbp->slot_skip : nullptr, counters + 1);
         e = cudaGetLastError();
         if (e != cudaSuccess) return e;
         if (launches) *launches += 1;
@@ -985,26 +1282,28 @@ static cudaError_t hop_bp(const HopPlan &p, const float *u, const float *in, flo
                                                    (float4 *)out, alpha, p.split.split_t,
                                                    p.n_split_rows, p.split_order, p.split_row,
                                                    p.split_slot0, (const float4 *)partial, f,
-                                                   counters);
+                                                   prune ? hbp->row_ub : nullptr,
+                                                   prune ? hbp->floor : nullptr,
+                                                   prune ? hbp->split_skip : nullptr, counters);
     else
         k_hop_rows<BP, false><<<grid, 256, 0, st>>>(p.in_ptr, p.in_src, p.in_w, p.n,
                                                     (const float4 *)u, (const float4 *)in,
                                                     (float4 *)out, alpha, p.split.split_t,
                                                     p.n_split_rows, p.split_order, p.split_row,
                                                     p.split_slot0, (const float4 *)partial, f,
-                                                    counters);
+                                                    nullptr, nullptr, nullptr, counters);
     if (launches) *launches += 1;
     return cudaGetLastError();
 }
 
 cudaError_t launch_hop(const HopPlan &p, const float *u, const float *in, float *out, int bp,
                        float alpha, float *partial, int *counters, const HopFilter *flt,
-                       cudaStream_t st, int *launches) {
+                       cudaStream_t st, int *launches, const HopBound *hb) {
     switch (bp) {
-    case 32: return hop_bp<32>(p, u, in, out, alpha, partial, counters, flt, st, launches);
-    case 64: return hop_bp<64>(p, u, in, out, alpha, partial, counters, flt, st, launches);
-    case 128: return hop_bp<128>(p, u, in, out, alpha, partial, counters, flt, st, launches);
-    case 256: return hop_bp<256>(p, u, in, out, alpha, partial, counters, flt, st, launches);
+    case 32: return hop_bp<32>(p, u, in, out, alpha, partial, counters, flt, st, launches, hb);
+    case 64: return hop_bp<64>(p, u, in, out, alpha, partial, counters, flt, st, launches, hb);
+    case 128: return hop_bp<128>(p, u, in, out, alpha, partial, counters, flt, st, launches, hb);
+    case 256: return hop_bp<256>(p, u, in, out, alpha, partial, counters, flt, st, launches, hb);
     default: return cudaErrorInvalidValue;
     }
 }

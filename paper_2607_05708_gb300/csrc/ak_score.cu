@@ -143,6 +143,8 @@ struct GemmEpi {
     NsScope ns;                         // EXP_FILTER: namespace scope of the queries
     const int32_t *dead_row;            // EXP, EXP_FILTER, FILTER: deleted rows (or NULL):
                                         // no score (u = 0) / never a filter candidate
+    float *row_max, *row_min;           // EXP (or NULL): [n_rows] largest / smallest u of
+    int n_real;                         // the row over the first n_real columns
 };
 
 template <int BP, int MODE>
@@ -367,6 +369,7 @@ __global__ __launch_bounds__(GemmCfg<BP, MODE>::THREADS, 1) void k_gemm_umma(con
                 in_rows && (MODE == GEMM_RAW || !ep.dead_row || !ep.dead_row[grow]);
             uint32_t fid = 0;
             bool fok = false;
+            float rmax = 0.f, rmin = INFINITY;           // u >= 0
             if ((FILTER || EXPF) && valid) {
                 const int32_t id = ep.ext_of[grow];
                 fok = (int64_t)id < ep.id_limit;
@@ -412,6 +415,14 @@ __global__ __launch_bounds__(GemmCfg<BP, MODE>::THREADS, 1) void k_gemm_umma(con
                 for (int i = 0; i < 32; ++i) {
                     const float x = __uint_as_float(r[i]);
                     v[i] = valid ? (EXP ? expf(ep.tau * x - shift_s[ch * 32 + i]) : x) : 0.f;
+                }
+                if (MODE == GEMM_EXP && ep.row_max) {
+#pragma unroll
+                    for (int i = 0; i < 32; ++i)
+                        if (ch * 32 + i < ep.n_real) {
+                            rmax = fmaxf(rmax, v[i]);
+                            rmin = fminf(rmin, v[i]);
+                        }
                 }
                 // filter, first half: which of this row's 32 values reach
                 // their query's threshold (branch-free; rarely any)
@@ -474,6 +485,10 @@ __global__ __launch_bounds__(GemmCfg<BP, MODE>::THREADS, 1) void k_gemm_umma(con
                 }
                 if (!EXPF && et == 0) bulk_wait_read<1>();
                 }
+            }
+            if (MODE == GEMM_EXP && ep.row_max && in_rows) {
+                ep.row_max[grow] = rmax;
+                ep.row_min[grow] = rmin;
             }
             tc_fence_before();
             named_bar(1, C::EPI_T);
@@ -604,9 +619,13 @@ static cudaError_t gemm_dispatch(const uint16_t *emb, int64_t n_rows, int64_t ro
 
 cudaError_t launch_score(const uint16_t *emb, int64_t n, int dim, const uint16_t *qp, int bp,
                          const float *shift, float tau, float *u, float *zpart, int *status,
-                         cudaStream_t st, int *launches, int *zrows, const int32_t *dead_row) {
+                         cudaStream_t st, int *launches, int *zrows, const int32_t *dead_row,
+                         float *row_max, float *row_min, int n_real) {
     GemmEpi ep{};
     ep.dead_row = dead_row;
+    ep.row_max = row_max;
+    ep.row_min = row_min;
+    ep.n_real = n_real;
     ep.shift = shift;
     ep.tau = tau;
     ep.zpart = zpart;

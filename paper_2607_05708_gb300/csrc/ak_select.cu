@@ -547,6 +547,59 @@ cudaError_t launch_buf_merge_signed(const unsigned int *cnt, const unsigned long
     return cudaGetLastError();
 }
 
+// ------------------------------------------------------------------ last-hop floor
+// The smallest final score any real query could still select: the largest of
+// (a) the smallest score bits that any real column's filter bound admits
+// (keys of non-negative scores order like their values; padding bounds,
+// above +inf's bits, admit nothing) and (b), without a namespace scope, the
+// k-th largest lower bound lb over the rows lb_rows[order[i]], i < n_rows:
+// every query's k-th largest final score is at least that, as each of
+// those k rows scores at least its lb for every query (any subset of the
+// rows gives a valid floor).  One CTA.
+__global__ __launch_bounds__(SEL_THREADS) void k_prune_floor(
+    const unsigned long long *__restrict__ bound, int n_real, const float *__restrict__ lb,
+    const int32_t *__restrict__ lb_rows, const int32_t *__restrict__ order, int64_t n_rows,
+    int k, float *__restrict__ floor_out) {
+    __shared__ int hist[256 * (SEL_THREADS / 32)];
+    __shared__ unsigned long long win[64];
+    __shared__ unsigned long long s_prefix;
+    __shared__ int s_remaining, win_n;
+    __shared__ unsigned int s_min;
+    const int tid = threadIdx.x;
+    if (tid == 0) s_min = 0x7f800000u;
+    __syncthreads();
+    unsigned int m = 0x7f800000u;
+    for (int c = tid; c < n_real; c += SEL_THREADS) {
+        const unsigned int hi = (unsigned int)(bound[c] >> 32);
+        m = hi < m ? hi : m;
+    }
+    atomicMin(&s_min, m);
+    __syncthreads();
+    float fl = __uint_as_float(s_min);
+    if (lb_rows && n_rows >= k) {
+        // keys (lb bits, position): unique, and ordered like lb (lb >= 0)
+        auto key_at = [&](int64_t i) -> unsigned long long {
+            return ((unsigned long long)__float_as_uint(lb[lb_rows[order[i]]]) << 32) |
+                   (unsigned long long)(uint32_t)i;
+        };
+        radix_select(n_rows, k, key_at, win, &win_n, hist, &s_prefix, &s_remaining);
+        if (tid == 0 && win_n >= k) {
+            unsigned long long mn = ~0ull;
+            for (int t = 0; t < win_n; ++t) mn = win[t] < mn ? win[t] : mn;
+            fl = fmaxf(fl, __uint_as_float((uint32_t)(mn >> 32)));
+        }
+    }
+    if (tid == 0) *floor_out = fl;
+}
+
+cudaError_t launch_prune_floor(const unsigned long long *bound, int n_real, const float *lb,
+                               const int32_t *lb_rows, const int32_t *order, int64_t n_lb_rows,
+                               int k, float *floor_out, cudaStream_t st) {
+    k_prune_floor<<<1, SEL_THREADS, 0, st>>>(bound, n_real, lb, lb_rows, order, n_lb_rows, k,
+                                             floor_out);
+    return cudaGetLastError();
+}
+
 // ------------------------------------------------------------------ launchers
 template <bool SIGNED>
 static cudaError_t launch_kth(const SelectPlan &sp, const float *s, int b, const int32_t *ext_of,

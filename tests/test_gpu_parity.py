@@ -94,6 +94,28 @@ def test_fused_filter_overflow_falls_back():
     assert_retrieval_parity(wl, "clustered", got, ref)
 
 
+@pytest.mark.parametrize("hops,k", [(1, 32), (2, 32), (2, 1), (3, 8), (2, 64)])
+def test_last_hop_row_bounds_change_nothing(hops, k, monkeypatch):
+    """The last hop skips every row whose upper bound (propagated from u's
+    row extremes, widened by the fp32 rounding of each level) stays below a
+    floor that every query's k-th largest final score reaches.  The selected
+    IDs, pages and page counts must equal those computed without the skip,
+    and the oracle's (gmm1m recipe at N = 16384, hub rows split).  Scores may
+    differ in the last bits only: without the skip more rows clear the
+    filter's sample bound, a query's buffer can overflow, and its column is
+    then recomputed by the merge with another summation order."""
+    import dataclasses
+    wl = dataclasses.replace(synth.workload(2, scale=1 / 64), hops=hops, k=k)
+    monkeypatch.setenv("AKASHIC_HOP_PRUNE", "0")
+    _, full = gpu_retrieve(wl, "clustered")
+    monkeypatch.setenv("AKASHIC_HOP_PRUNE", "1")
+    _, pruned = gpu_retrieve(wl, "clustered")
+    for key in ("ids", "page_ids", "n_pages"):
+        assert np.array_equal(full[key], pruned[key]), key
+    np.testing.assert_allclose(pruned["scores"], full["scores"], rtol=1e-5, atol=0)
+    assert_retrieval_parity(wl, "clustered", pruned, oracle_retrieve(wl, "clustered"))
+
+
 def test_score_filter_overflow_falls_back():
     """No hops, N = 16384 chunks sharing one embedding: every score is equal,
     all rows clear the bound taken from the score's row sample and the
