@@ -1159,7 +1159,9 @@ __global__ __launch_bounds__(256, 3) void k_hop_rows(const int64_t *__restrict__
     using S = HopShape<BP>;
     const int lane = threadIdx.x & 31;
     const int sub = lane % S::LW;
-    const int64_t groups = (n + ROWS_PER_GRAB - 1) / ROWS_PER_GRAB;
+    // with the skip, a claim takes 32 rows, tested at once (one ballot)
+    const int64_t grab = (FILTER && row_ub) ? 32 : ROWS_PER_GRAB;
+    const int64_t groups = (n + grab - 1) / grab;
     __shared__ unsigned long long thr[FILTER ? BP : 1];
     __shared__ uint4 thr_hi[FILTER ? BP / 4 : 1];
     // last hop: rows whose bound stays below the floor append nothing
@@ -1185,20 +1187,28 @@ __global__ __launch_bounds__(256, 3) void k_hop_rows(const int64_t *__restrict__
                                       u4, out4, alpha, f, thr, thr_hi);
             continue;
         }
-        const int64_t j0 = (it - n_split) * ROWS_PER_GRAB;
-        const int nr = (int)(n - j0 < ROWS_PER_GRAB ? n - j0 : ROWS_PER_GRAB);
-        int64_t p = 0;
-        if (lane <= nr) p = in_ptr[j0 + lane];
+        const int64_t j0 = (it - n_split) * grab;
+        const int nr = (int)(n - j0 < grab ? n - j0 : grab);
+        // lane r: row j0 + r's edge range; `todo`: rows kept whole (and,
+        // in the pruned last hop, not below the floor)
+        int64_t p0 = 0, p1 = 0;
+        if (lane < nr) {
+            p0 = in_ptr[j0 + lane];
+            p1 = in_ptr[j0 + lane + 1];
+        }
+        bool want = lane < nr && p1 - p0 <= split_t;
+        if (prune && want) want = __ldg(row_ub + j0 + lane) >= floor_;
+        unsigned todo = __ballot_sync(0xffffffffu, want);
         int32_t ids = 0;
-        if (FILTER && lane < nr) ids = f.ext_of[j0 + lane];
+        if (FILTER && want) ids = f.ext_of[j0 + lane];
 #pragma unroll 1
-        for (int r = 0; r < nr; ++r) {
-            const int64_t e0 = __shfl_sync(0xffffffffu, p, r);
-            const int64_t e1 = __shfl_sync(0xffffffffu, p, r + 1);
+        while (todo) {
+            const int r = __ffs(todo) - 1;
+            todo &= todo - 1;
+            const int64_t e0 = __shfl_sync(0xffffffffu, p0, r);
+            const int64_t e1 = __shfl_sync(0xffffffffu, p1, r);
             const uint32_t id = FILTER ? (uint32_t)__shfl_sync(0xffffffffu, ids, r) : 0u;
-            if (e1 - e0 > split_t) continue;
             const int64_t j = j0 + r;
-            if (prune && __ldg(row_ub + j) < floor_) continue;
             float4 b[S::V];
             if (lane < S::LW) {
 #pragma unroll
@@ -1272,7 +1282,7 @@ static cudaError_t hop_bp(const HopPlan &p, const float *u, const float *in, flo
         if (e != cudaSuccess) return e;
         if (launches) *launches += 1;
     }
-    const int64_t items = ceil_div<int64_t>(p.n, ROWS_PER_GRAB) + p.n_split_rows;
+    const int64_t items = ceil_div<int64_t>(p.n, prune ? 32 : ROWS_PER_GRAB) + p.n_split_rows;
     const int64_t want = ceil_div<int64_t>(items, 8);
     const int grid = (int)(want < (int64_t)sms * 3 ? (want < 1 ? 1 : want) : (int64_t)sms * 3);
     const HopFilter f = flt ? *flt : HopFilter{nullptr, nullptr, nullptr, nullptr, 0, NsScope{}};
