@@ -199,6 +199,52 @@ def test_delete_then_retrieve(hops):
     assert_retrieval_parity(wl, "clustered", got, ref)
 
 
+def test_row_bounds_follow_graph_changes():
+    """The last hop's graph-only mass levels are cached on the store and
+    must be recomputed after the graph changes: retrieve (fills the cache),
+    delete 300 chunks including 10 hubs, retrieve, then append 64 chunks
+    without edges and retrieve again (N changes, the graph does not) - each
+    retrieval against the oracle on the store's current graph."""
+    import oracle
+    import torch
+    wl = synth.workload(2, scale=1 / 64)
+    store = gpu_store(wl, "clustered", capacity=wl.n + 64)
+    _, got = gpu_retrieve(wl, "clustered", store=store)
+    assert_retrieval_parity(wl, "clustered", got, oracle_retrieve(wl, "clustered"))
+    rng = np.random.default_rng(23)
+    indeg = np.bincount(wl.col, minlength=wl.n)
+    victims = np.unique(np.concatenate([np.argsort(-indeg)[:10],
+                                        rng.choice(wl.n, 290, replace=False)]))
+    dead = np.zeros(wl.n, bool)
+    dead[victims] = True
+    store.delete(torch.from_numpy(victims.astype(np.int64)).cuda())
+    rp, col, aff, _ = (t.cpu().numpy() for t in store.export_csr())
+    w = oracle.row_softmax(rp, aff)
+
+    def check(n_extra):
+        emb = wl.emb if n_extra == 0 else np.concatenate([wl.emb, wl.emb[:n_extra]])
+        d = np.concatenate([dead, np.zeros(n_extra, bool)])
+        rp2 = np.concatenate([rp, np.full(n_extra, rp[-1], np.int64)])
+        pages = np.concatenate([wl.page_of["clustered"],
+                                wl.page_of["clustered"].max() + 1 + np.arange(n_extra) // 64])
+        q = torch.from_numpy(np.ascontiguousarray(wl.queries).view(np.int16)).cuda()
+        ids, sc, pg, npg = store.retrieve(q, wl.k, wl.alpha, wl.hops)
+        store.sync()
+        got = dict(ids=ids.cpu().numpy(), scores=sc.cpu().numpy(), page_ids=pg.cpu().numpy(),
+                   n_pages=npg.cpu().numpy())
+        assert not d[got["ids"]].any()
+        ref = oracle.retrieve(emb, wl.queries, rp2, col, w, tau=wl.tau, alpha=wl.alpha,
+                              hops=wl.hops, k=wl.k, page_of=pages.astype(np.int32),
+                              want_final=True, dead=d)
+        import dataclasses
+        wl2 = dataclasses.replace(wl, emb=emb, page_of={"clustered": pages.astype(np.int32)})
+        assert_retrieval_parity(wl2, "clustered", got, ref)
+
+    check(0)
+    store.append_chunks(torch.from_numpy(np.ascontiguousarray(wl.emb[:64]).view(np.int16)).cuda())
+    check(64)
+
+
 def test_delete_then_update_skips_deleted():
     """After deletions a relation update links each new chunk to its top-M
     among the live prior chunks only: its neighbour set equals the oracle's
