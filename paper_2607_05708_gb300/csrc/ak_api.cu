@@ -85,7 +85,7 @@ struct StreamScratch {
     DevBuf qns, ns_s, dead_s;    // scope: per query column, per sample row
     DevBuf rmax_u, rmin_u;       // u's row maxima / minima over the real queries
     DevBuf ub, lb, ext, pfloor;  // the last hop's row bounds, extremes, floor
-    DevBuf skip_split, skip_slot;
+    DevBuf skip_split, skip_slot, kept_rows, kept_count, kept_segs, kflag, kpos, ktmp;
 };
 
 struct ProfRec {
@@ -1090,6 +1090,13 @@ static akashic_status_t retrieve_impl(akashic_mem *m, const uint16_t *q, int32_t
             AK_TRY(sc->lb.ensure((size_t)n * 4));
             AK_TRY(sc->ext.ensure(16));
             AK_TRY(sc->skip_split.ensure((size_t)(m->n_split + 1) * 4));
+            AK_TRY(sc->kept_rows.ensure((size_t)n * 4));
+            AK_TRY(sc->kept_count.ensure(16));
+            AK_TRY(sc->kept_segs.ensure((size_t)(m->n_segs + 1) * 4));
+            const int64_t nk = n > m->n_segs ? n : m->n_segs;
+            AK_TRY(sc->kflag.ensure((size_t)(nk + 1) * 8));
+            AK_TRY(sc->kpos.ensure((size_t)(nk + 1) * 8));
+            AK_TRY(sc->ktmp.ensure(scan_tmp_bytes(nk + 1) + 4096));
             AK_TRY(sc->skip_slot.ensure((size_t)(m->n_segs + 1) * 4));
             AK_TRY(sc->pfloor.ensure(16));
         }
@@ -1230,17 +1237,24 @@ static akashic_status_t retrieve_impl(akashic_mem *m, const uint16_t *q, int32_t
                                                     q_ns ? nullptr : hp.split_row,
                                                     hp.split_order, n_lb, k,
                                                     sc->pfloor.as<float>(), st));
+                        KeptScratch ks{sc->kflag.as<int64_t>(), sc->kpos.as<int64_t>(),
+                                       sc->ktmp.p, sc->ktmp.cap};
                         CUDA_TRY(launch_split_flags(hp, row_ub, sc->pfloor.as<float>(),
                                                     sc->skip_split.as<int32_t>(),
-                                                    sc->skip_slot.as<int32_t>(), st));
-                        ps.launches += 1 + (m->n_split > 0);
+                                                    sc->skip_slot.as<int32_t>(),
+                                                    sc->kept_rows.as<int32_t>(),
+                                                    sc->kept_count.as<int64_t>(),
+                                                    sc->kept_segs.as<int32_t>(), ks, st,
+                                                    &ps.launches));
+                        ps.launches += 1;
                     }
                 }
                 const HopFilter flt{m->ext_of.as<int32_t>(), ws + sp.off_bound,
                                     (unsigned int *)(ws + sp.off_cnt), ws + sp.off_buf, sp.cap,
                                     ns};
                 const HopBound hb{row_ub, sc->pfloor.as<float>(), sc->skip_split.as<int32_t>(),
-                                  sc->skip_slot.as<int32_t>()};
+                                  sc->skip_slot.as<int32_t>(), sc->kept_rows.as<int32_t>(),
+                                  sc->kept_count.as<int64_t>(), sc->kept_segs.as<int32_t>()};
                 PhaseScope ph(m, last ? AKASHIC_PHASE_LAST_HOP : AKASHIC_PHASE_PROPAGATE, st);
                 CUDA_TRY(launch_hop(hp, sc->u.as<float>(), fin, out, bp, alpha,
                                     sc->partial.as<float>(), sc->counters.as<int>(),

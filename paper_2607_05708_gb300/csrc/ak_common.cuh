@@ -366,6 +366,16 @@ struct HopBound {
     const float *floor;        // device scalar
     const int32_t *split_skip; // [n_split_rows] split rows to skip (launch_split_flags)
     const int32_t *slot_skip;  // [n_segs] their partial slots
+    const int32_t *kept_rows;  // [n] rows kept whole that reach the floor ...
+    const int64_t *kept_count; // ... [0] their number, [1] that of kept_segs (device)
+    const int32_t *kept_segs;  // [n_segs] segments of the unpruned split rows
+};
+// Scratch of the kept lists' compaction: flag / pos [max(n, n_segs) + 1]
+// int64, tmp of scan_tmp_bytes(max(n, n_segs)) bytes.
+struct KeptScratch {
+    int64_t *flag, *pos;
+    void *tmp;
+    size_t tmp_bytes;
 };
 // Graph-only mass vectors for the row bounds, levels t0..t1 (level 0, all
 // ones, already in place): mup[t] >= g (1 + eps) sum_i w_ij mup[t-1]_i and
@@ -388,7 +398,9 @@ cudaError_t launch_final_bounds(const float *u0, const float *l0, const float *m
                                 unsigned int *ext, float *ub, float *lb, cudaStream_t st,
                                 int *launches);
 cudaError_t launch_split_flags(const HopPlan &p, const float *row_ub, const float *floor_p,
-                               int32_t *split_skip, int32_t *slot_skip, cudaStream_t st);
+                               int32_t *split_skip, int32_t *slot_skip, int32_t *kept_rows,
+                               int64_t *kept_count, int32_t *kept_segs, KeptScratch &ks,
+                               cudaStream_t st, int *launches);
 // floor = max(the smallest score any real column's filter bound admits,
 // and, if lb_rows != NULL, the k-th largest lb over the rows
 // lb_rows[order[i]], i < n_lb_rows), written to floor_out.  The second term

@@ -662,13 +662,15 @@ struct HopShape {
     static constexpr int LW = F >= 32 ? 32 : F;            // lanes per group
 };
 
-template <int BP>
+template <int BP, int WIDTH = 1>
 __device__ __forceinline__ void hop_accumulate(const int32_t *__restrict__ in_src,
                                                const float *__restrict__ in_w, int64_t e0,
                                                int64_t e1, const float4 *__restrict__ in4,
                                                float4 (&acc)[HopShape<BP>::V]) {
     using S = HopShape<BP>;
-    constexpr int UN = 8 / S::V > 0 ? 8 / S::V : 1;   // gathers in flight: UN edges x V float4
+    // gathers in flight: UN edges x V float4 (WIDTH times more in the wide
+    // variant, which runs fewer warps)
+    constexpr int UN = WIDTH * (8 / S::V > 0 ? 8 / S::V : 1);
     const int lane = threadIdx.x & 31;
     const int g = lane / S::LW, sub = lane % S::LW;
     const uint64_t pol = l2_keep_policy();
@@ -1017,13 +1019,62 @@ cudaError_t launch_final_bounds(const float *u0, const float *l0, const float *m
     return cudaGetLastError();
 }
 
+// Last hop: keep flags of the rows kept whole whose bound reaches the floor,
+// and of the segments of unpruned split rows; the lists are compacted by an
+// exclusive scan, so they keep row order and window-major order (the order
+// that keeps gathered source rows in L2).
+__global__ void k_keep_rows(const int64_t *__restrict__ in_ptr, int64_t n, int64_t split_t,
+                            const float *__restrict__ row_ub, const float *__restrict__ floor_p,
+                            int64_t *__restrict__ flag) {
+    const float floor_ = *floor_p;
+    for (int64_t j = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; j < n;
+         j += (int64_t)gridDim.x * blockDim.x)
+        flag[j] = in_ptr[j + 1] - in_ptr[j] <= split_t && row_ub[j] >= floor_;
+}
+__global__ void k_keep_segs(const int32_t *__restrict__ seg_slot, int64_t n_segs,
+                            const int32_t *__restrict__ slot_skip, int64_t *__restrict__ flag) {
+    for (int64_t s = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; s < n_segs;
+         s += (int64_t)gridDim.x * blockDim.x)
+        flag[s] = slot_skip[seg_slot[s]] == 0;
+}
+__global__ void k_compact_kept(const int64_t *__restrict__ flag, const int64_t *__restrict__ pos,
+                               int64_t n, int32_t *__restrict__ out, int64_t *__restrict__ count) {
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n;
+         i += (int64_t)gridDim.x * blockDim.x)
+        if (flag[i]) out[pos[i]] = (int32_t)i;
+    if (blockIdx.x == 0 && threadIdx.x == 0) *count = pos[n];
+}
+
 cudaError_t launch_split_flags(const HopPlan &p, const float *row_ub, const float *floor_p,
-                               int32_t *split_skip, int32_t *slot_skip, cudaStream_t st) {
-    if (p.n_split_rows <= 0) return cudaSuccess;
-    const int64_t want = ceil_div<int64_t>(p.n_split_rows, 8);
-    const int g = (int)(want < (int64_t)device_sm_count() * 4 ? want : (int64_t)device_sm_count() * 4);
-    k_split_flags<<<g, 256, 0, st>>>(p.n_split_rows, p.split_row, p.split_slot0, row_ub, floor_p,
-                                     split_skip, slot_skip);
+                               int32_t *split_skip, int32_t *slot_skip, int32_t *kept_rows,
+                               int64_t *kept_count, int32_t *kept_segs, KeptScratch &ks,
+                               cudaStream_t st, int *launches) {
+    const int sms = device_sm_count();
+    if (p.n_split_rows > 0) {
+        const int64_t want = ceil_div<int64_t>(p.n_split_rows, 8);
+        const int g = (int)(want < (int64_t)sms * 4 ? want : (int64_t)sms * 4);
+        k_split_flags<<<g, 256, 0, st>>>(p.n_split_rows, p.split_row, p.split_slot0, row_ub,
+                                         floor_p, split_skip, slot_skip);
+    }
+    if (launches && p.n_split_rows > 0) *launches += 1;
+    // kept_count[0]: rows, kept_count[1]: segments
+    k_keep_rows<<<sms * 4, 256, 0, st>>>(p.in_ptr, p.n, p.split.split_t, row_ub, floor_p,
+                                         ks.flag);
+    cudaError_t e = scan_exclusive(ks.flag, ks.pos, p.n, ks.tmp, ks.tmp_bytes, st, launches);
+    if (e != cudaSuccess) return e;
+    k_compact_kept<<<sms * 4, 256, 0, st>>>(ks.flag, ks.pos, p.n, kept_rows, kept_count);
+    if (launches) *launches += 2;
+    if (p.n_segs > 0) {
+        k_keep_segs<<<sms * 4, 256, 0, st>>>(p.seg_slot, p.n_segs, slot_skip, ks.flag);
+        e = scan_exclusive(ks.flag, ks.pos, p.n_segs, ks.tmp, ks.tmp_bytes, st, launches);
+        if (e != cudaSuccess) return e;
+        k_compact_kept<<<sms * 4, 256, 0, st>>>(ks.flag, ks.pos, p.n_segs, kept_segs,
+                                                kept_count + 1);
+        if (launches) *launches += 2;
+    } else {
+        e = cudaMemsetAsync(kept_count + 1, 0, sizeof(int64_t), st);
+        if (e != cudaSuccess) return e;
+    }
     return cudaGetLastError();
 }
 
@@ -1070,7 +1121,7 @@ __device__ __forceinline__ void hop_emit(const HopFilter &f, const unsigned long
     if constexpr (FILTER) hop_filter_row<BP>(f, thr, thr_hi, sub, j, id, o);
 }
 
-template <int BP, bool FILTER>
+template <int BP, bool FILTER, int WIDTH = 1>
 __device__ __forceinline__ void hop_fixup_row(int64_t j, int64_t a, int64_t b,
                                               const float4 *__restrict__ part4,
                                               const float4 *__restrict__ u4,
@@ -1079,7 +1130,7 @@ __device__ __forceinline__ void hop_fixup_row(int64_t j, int64_t a, int64_t b,
                                               const unsigned long long *thr,
                                               const uint4 *thr_hi) {
     using S = HopShape<BP>;
-    constexpr int P = 8 / S::V > 0 ? 8 / S::V : 1;   // slots in flight per lane group
+    constexpr int P = WIDTH * (8 / S::V > 0 ? 8 / S::V : 1);   // slots in flight per lane group
     const int lane = threadIdx.x & 31;
     const int g = lane / S::LW, sub = lane % S::LW;
     const uint32_t id = FILTER ? (uint32_t)f.ext_of[j] : 0u;
@@ -1139,8 +1190,10 @@ __device__ __forceinline__ void hop_fixup_row(int64_t j, int64_t a, int64_t b,
 // rows kept whole, ROWS_PER_GRAB consecutive rows per claim (load
 // balance), with the group's row pointers read at once and each row's u
 // load issued before its gathers.
-template <int BP, bool FILTER>
-__global__ __launch_bounds__(256, 3) void k_hop_rows(const int64_t *__restrict__ in_ptr,
+// WIDTH 2 (the pruned last hop, few work items): twice the loads in flight
+// per warp, two CTAs per SM.
+template <int BP, bool FILTER, int WIDTH = 1>
+__global__ __launch_bounds__(256, WIDTH > 1 ? 2 : 3) void k_hop_rows(const int64_t *__restrict__ in_ptr,
                                                   const int32_t *__restrict__ in_src,
                                                   const float *__restrict__ in_w, int64_t n,
                                                   const float4 *__restrict__ u4,
@@ -1155,18 +1208,22 @@ __global__ __launch_bounds__(256, 3) void k_hop_rows(const int64_t *__restrict__
                                                   const float *__restrict__ row_ub,
                                                   const float *__restrict__ floor_p,
                                                   const int32_t *__restrict__ split_skip,
+                                                  const int32_t *__restrict__ kept_rows,
+                                                  const int64_t *__restrict__ kept_count,
                                                   int *__restrict__ queue) {
     using S = HopShape<BP>;
     const int lane = threadIdx.x & 31;
     const int sub = lane % S::LW;
-    // with the skip, a claim takes 32 rows, tested at once (one ballot)
-    const int64_t grab = (FILTER && row_ub) ? 32 : ROWS_PER_GRAB;
-    const int64_t groups = (n + grab - 1) / grab;
+    // with the skip (last hop), the rows kept whole that reach the floor
+    // come as a compact list; a claim takes ROWS_PER_GRAB rows either way
+    const bool listed = FILTER && kept_rows != nullptr;
+    const int64_t grab = ROWS_PER_GRAB;
+    const int64_t n_items = listed ? *kept_count : n;
+    const int64_t groups = (n_items + grab - 1) / grab;
     __shared__ unsigned long long thr[FILTER ? BP : 1];
     __shared__ uint4 thr_hi[FILTER ? BP / 4 : 1];
     // last hop: rows whose bound stays below the floor append nothing
     const bool prune = FILTER && row_ub != nullptr;
-    const float floor_ = prune ? *floor_p : 0.f;
     if constexpr (FILTER) {
         for (int c = threadIdx.x; c < BP; c += blockDim.x) {
             const unsigned long long t = f.bound[c];
@@ -1183,24 +1240,24 @@ __global__ __launch_bounds__(256, 3) void k_hop_rows(const int64_t *__restrict__
         if (it < n_split) {
             const int32_t r = split_order[it];
             if (prune && split_skip[r]) continue;
-            hop_fixup_row<BP, FILTER>(split_row[r], split_slot0[r], split_slot0[r + 1], part4,
+            hop_fixup_row<BP, FILTER, WIDTH>(split_row[r], split_slot0[r], split_slot0[r + 1], part4,
                                       u4, out4, alpha, f, thr, thr_hi);
             continue;
         }
-        const int64_t j0 = (it - n_split) * grab;
-        const int nr = (int)(n - j0 < grab ? n - j0 : grab);
-        // lane r: row j0 + r's edge range; `todo`: rows kept whole (and,
-        // in the pruned last hop, not below the floor)
-        int64_t p0 = 0, p1 = 0;
+        // lane r: the claim's r-th row (consecutive rows, or listed ones),
+        // its edge range; `todo`: the rows kept whole
+        const int64_t i0 = (it - n_split) * grab;
+        const int nr = (int)(n_items - i0 < grab ? n_items - i0 : grab);
+        int64_t myrow = 0, p0 = 0, p1 = 0;
         if (lane < nr) {
-            p0 = in_ptr[j0 + lane];
-            p1 = in_ptr[j0 + lane + 1];
+            myrow = listed ? (int64_t)kept_rows[i0 + lane] : i0 + lane;
+            p0 = in_ptr[myrow];
+            p1 = in_ptr[myrow + 1];
         }
-        bool want = lane < nr && p1 - p0 <= split_t;
-        if (prune && want) want = __ldg(row_ub + j0 + lane) >= floor_;
+        const bool want = lane < nr && p1 - p0 <= split_t;
         unsigned todo = __ballot_sync(0xffffffffu, want);
         int32_t ids = 0;
-        if (FILTER && want) ids = f.ext_of[j0 + lane];
+        if (FILTER && want) ids = f.ext_of[myrow];
 #pragma unroll 1
         while (todo) {
             const int r = __ffs(todo) - 1;
@@ -1208,14 +1265,14 @@ __global__ __launch_bounds__(256, 3) void k_hop_rows(const int64_t *__restrict__
             const int64_t e0 = __shfl_sync(0xffffffffu, p0, r);
             const int64_t e1 = __shfl_sync(0xffffffffu, p1, r);
             const uint32_t id = FILTER ? (uint32_t)__shfl_sync(0xffffffffu, ids, r) : 0u;
-            const int64_t j = j0 + r;
+            const int64_t j = __shfl_sync(0xffffffffu, myrow, r);
             float4 b[S::V];
             if (lane < S::LW) {
 #pragma unroll
                 for (int v = 0; v < S::V; ++v) b[v] = ld_stream(u4 + j * S::F + sub + 32 * v);
             }
             float4 acc[S::V];
-            hop_accumulate<BP>(in_src, in_w, e0, e1, in4, acc);
+            hop_accumulate<BP, WIDTH>(in_src, in_w, e0, e1, in4, acc);
             if (lane < S::LW) {
 #pragma unroll
                 for (int v = 0; v < S::V; ++v) {
@@ -1232,8 +1289,8 @@ __global__ __launch_bounds__(256, 3) void k_hop_rows(const int64_t *__restrict__
 }
 
 // Segments of split rows, claimed one at a time in window-major order.
-template <int BP>
-__global__ __launch_bounds__(256, 3) void k_hop_segs(const int64_t *__restrict__ seg_e0,
+template <int BP, int WIDTH = 1>
+__global__ __launch_bounds__(256, WIDTH > 1 ? 2 : 3) void k_hop_segs(const int64_t *__restrict__ seg_e0,
                                                   const int64_t *__restrict__ seg_e1,
                                                   const int32_t *__restrict__ seg_slot,
                                                   int64_t n_segs,
@@ -1241,20 +1298,23 @@ __global__ __launch_bounds__(256, 3) void k_hop_segs(const int64_t *__restrict__
                                                   const float *__restrict__ in_w,
                                                   const float4 *__restrict__ in4,
                                                   float4 *__restrict__ part4,
-                                                  const int32_t *__restrict__ slot_skip,
+                                                  const int32_t *__restrict__ kept_segs,
+                                                  const int64_t *__restrict__ kept_count,
                                                   int *__restrict__ queue) {
     using S = HopShape<BP>;
     const int lane = threadIdx.x & 31;
     const int sub = lane % S::LW;
+    // last hop: only the listed segments (those of unpruned split rows)
+    const int64_t total = kept_segs ? *kept_count : n_segs;
     while (true) {
-        int64_t s = 0;
-        if (lane == 0) s = atomicAdd(queue, 1);
-        s = __shfl_sync(0xffffffffu, s, 0);
-        if (s >= n_segs) break;
-        const int64_t slot = seg_slot[s];
-        if (slot_skip && slot_skip[slot]) continue;   // its row is pruned
+        int64_t i = 0;
+        if (lane == 0) i = atomicAdd(queue, 1);
+        i = __shfl_sync(0xffffffffu, i, 0);
+        if (i >= total) break;
+        const int64_t s = kept_segs ? (int64_t)kept_segs[i] : i;
         float4 acc[S::V];
-        hop_accumulate<BP>(in_src, in_w, seg_e0[s], seg_e1[s], in4, acc);
+        hop_accumulate<BP, WIDTH>(in_src, in_w, seg_e0[s], seg_e1[s], in4, acc);
+        const int64_t slot = seg_slot[s];
         if (lane < S::LW) {
 #pragma unroll
             for (int v = 0; v < S::V; ++v) st_stream(part4 + slot * S::F + sub + 32 * v, acc[v]);
@@ -1268,40 +1328,60 @@ static cudaError_t hop_bp(const HopPlan &p, const float *u, const float *in, flo
                           cudaStream_t st, int *launches, const HopBound *hbp) {
     const int sms = device_sm_count();
     // the last hop skips rows whose bound stays below the filter floor
-    const bool prune = flt && hbp && hbp->row_ub && hbp->floor &&
-                       (p.n_split_rows == 0 || (hbp->split_skip && hbp->slot_skip));
+    const bool prune = flt && hbp && hbp->row_ub && hbp->floor && hbp->kept_rows &&
+                       hbp->kept_count &&
+                       (p.n_split_rows == 0 ||
+                        (hbp->split_skip && hbp->slot_skip && hbp->kept_segs));
     cudaError_t e = cudaMemsetAsync(counters, 0, 2 * sizeof(int), st);
     if (e != cudaSuccess) return e;
     if (p.n_segs > 0) {
         const int64_t want = ceil_div<int64_t>(p.n_segs, 8);
-        const int g2 = (int)(want < (int64_t)sms * 3 ? want : (int64_t)sms * 3);
-        k_hop_segs<BP><<<g2, 256, 0, st>>>(p.seg_e0, p.seg_e1, p.seg_slot, p.n_segs, p.in_src,
-                                           p.in_w, (const float4 *)in, (float4 *)partial,
-                                           prune ? hbp->slot_skip : nullptr, counters + 1);
+        const int cps = prune ? 2 : 3;
+        const int g2 = (int)(want < (int64_t)sms * cps ? want : (int64_t)sms * cps);
+        if (prune)
+            k_hop_segs<BP, 2><<<g2, 256, 0, st>>>(p.seg_e0, p.seg_e1, p.seg_slot, p.n_segs,
+                                                  p.in_src, p.in_w, (const float4 *)in,
+                                                  (float4 *)partial, hbp->kept_segs,
+                                                  hbp->kept_count + 1, counters + 1);
+        else
+            k_hop_segs<BP><<<g2, 256, 0, st>>>(p.seg_e0, p.seg_e1, p.seg_slot, p.n_segs, p.in_src,
+                                               p.in_w, (const float4 *)in, (float4 *)partial,
+                                               nullptr, nullptr, counters + 1);
         e = cudaGetLastError();
         if (e != cudaSuccess) return e;
         if (launches) *launches += 1;
     }
-    const int64_t items = ceil_div<int64_t>(p.n, prune ? 32 : ROWS_PER_GRAB) + p.n_split_rows;
+    // (pruned: split rows + the kept list, its length known on the device only)
+    const int64_t items = prune ? p.n_split_rows + 4096
+                                : ceil_div<int64_t>(p.n, ROWS_PER_GRAB) + p.n_split_rows;
     const int64_t want = ceil_div<int64_t>(items, 8);
-    const int grid = (int)(want < (int64_t)sms * 3 ? (want < 1 ? 1 : want) : (int64_t)sms * 3);
+    const int cpr = prune ? 2 : 3;
+    const int grid = (int)(want < (int64_t)sms * cpr ? (want < 1 ? 1 : want) : (int64_t)sms * cpr);
     const HopFilter f = flt ? *flt : HopFilter{nullptr, nullptr, nullptr, nullptr, 0, NsScope{}};
-    if (flt)
+    if (prune)
+        k_hop_rows<BP, true, 2><<<grid, 256, 0, st>>>(p.in_ptr, p.in_src, p.in_w, p.n,
+                                                      (const float4 *)u, (const float4 *)in,
+                                                      (float4 *)out, alpha, p.split.split_t,
+                                                      p.n_split_rows, p.split_order, p.split_row,
+                                                      p.split_slot0, (const float4 *)partial, f,
+                                                      hbp->row_ub, hbp->floor, hbp->split_skip,
+                                                      hbp->kept_rows, hbp->kept_count, counters);
+    else if (flt)
         k_hop_rows<BP, true><<<grid, 256, 0, st>>>(p.in_ptr, p.in_src, p.in_w, p.n,
                                                    (const float4 *)u, (const float4 *)in,
                                                    (float4 *)out, alpha, p.split.split_t,
                                                    p.n_split_rows, p.split_order, p.split_row,
                                                    p.split_slot0, (const float4 *)partial, f,
-                                                   prune ? hbp->row_ub : nullptr,
-                                                   prune ? hbp->floor : nullptr,
-                                                   prune ? hbp->split_skip : nullptr, counters);
+                                                   nullptr, nullptr, nullptr, nullptr, nullptr,
+                                                   counters);
     else
         k_hop_rows<BP, false><<<grid, 256, 0, st>>>(p.in_ptr, p.in_src, p.in_w, p.n,
                                                     (const float4 *)u, (const float4 *)in,
                                                     (float4 *)out, alpha, p.split.split_t,
                                                     p.n_split_rows, p.split_order, p.split_row,
                                                     p.split_slot0, (const float4 *)partial, f,
-                                                    nullptr, nullptr, nullptr, counters);
+                                                    nullptr, nullptr, nullptr, nullptr, nullptr,
+                                                    counters);
     if (launches) *launches += 1;
     return cudaGetLastError();
 }

@@ -49,15 +49,15 @@ def gpu_retrieve(wl, placement, store=None, queries=None, k=None, alpha=None, ho
                        n_pages=npg.cpu().numpy())
 
 
-_W_CACHE = {}
-
-
 def oracle_weights(wl):
-    key = id(wl)
-    if key not in _W_CACHE:
-        _W_CACHE.clear()
-        _W_CACHE[key] = oracle.row_softmax(wl.row_ptr, wl.aff)
-    return _W_CACHE[key]
+    # cached on the workload object itself (a dataclasses.replace copy starts
+    # without it); an id()-keyed cache could hand a new object the weights of
+    # a freed one whose id it reuses
+    w = wl.__dict__.get("_oracle_w")
+    if w is None:
+        w = oracle.row_softmax(wl.row_ptr, wl.aff)
+        wl.__dict__["_oracle_w"] = w
+    return w
 
 
 def oracle_retrieve(wl, placement, queries=None, k=None, alpha=None, hops=None):
