@@ -16,7 +16,7 @@ CSRC = os.path.join(HERE, "csrc")
 OBJ = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libakashic_mem.so")
 SOURCES = ["ak_api.cu", "ak_score.cu", "ak_graph.cu", "ak_select.cu", "ak_update.cu",
-           "ak_inedges.cu", "ak_delete.cu", "ak_mm.cu", "ak_noalloc.cu"]
+           "ak_inedges.cu", "ak_delete.cu", "ak_mm.cu", "ak_noalloc.cu", "ak_reach.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "--expt-relaxed-constexpr"]
 

@@ -86,6 +86,7 @@ struct StreamScratch {
     DevBuf rmax_u, rmin_u;       // u's row maxima / minima over the real queries
     DevBuf ub, lb, ext, pfloor;  // the last hop's row bounds, extremes, floor
     DevBuf skip_split, skip_slot, kept_rows, kept_count, kept_segs, kflag, kpos, ktmp;
+    DevBuf reach_keep, reach_bad, reach_part;
 };
 
 struct ProfRec {
@@ -146,6 +147,12 @@ struct akashic_mem {
     DevBuf mass_up, mass_dn, mass_zero, mass_vu, mass_vl;
     int mass_levels = -1;
     int64_t mass_n = -1;      // rows they were computed for
+    // reach coefficients of the candidate rows (ak_reach.cu), same lifetime
+    DevBuf reach_rows, reach_t, reach_map, reach_c;
+    int reach_levels = -1;
+    int reach_T = 0;          // candidate rows (host copy)
+    int64_t reach_n = -1;     // rows they were computed for
+    bool reach_on = true;     // AKASHIC_REACH=0: always run the hops
     std::mutex mu;
     std::unordered_map<void *, StreamScratch *> scratch;
     // profiling
@@ -363,6 +370,7 @@ static akashic_status_t rebuild_in_edges(akashic_mem *m, cudaStream_t st) {
 static akashic_status_t build_split_plan(akashic_mem *m, cudaStream_t st) {
     const int64_t n = m->n;
     m->mass_levels = -1;   // the graph changed
+    m->reach_levels = -1;
     // temporaries from the store's scratch (slots SCR_SPLIT0..11)
     akashic_status_t sc_rc = AKASHIC_OK;
     auto get = [&](int i, size_t bytes) -> Tmp {
@@ -466,6 +474,7 @@ akashic_status_t akashic_mem_create(const akashic_mem_config_t *cfg, akashic_mem
     if (const char *v = getenv("AKASHIC_SEG_LEN")) m->split.seg_len = atoll(v) > 0 ? atoll(v) : m->split.seg_len;
     if (const char *v = getenv("AKASHIC_FUSE_FILTER")) m->fuse_filter = atoi(v) != 0;
     if (const char *v = getenv("AKASHIC_HOP_PRUNE")) m->hop_prune = atoi(v) != 0;
+    if (const char *v = getenv("AKASHIC_REACH")) m->reach_on = atoi(v) != 0;
     if (const char *v = getenv("AKASHIC_FULL_TRANSPOSE")) m->inc_transpose = atoi(v) == 0;
     if (const char *v = getenv("AKASHIC_WIN_ROWS")) m->split.win_rows = atoll(v) > 0 ? atoll(v) : m->split.win_rows;
     akashic_status_t s;
@@ -1047,6 +1056,42 @@ static akashic_status_t ensure_mass(akashic_mem *m, const HopPlan &hp, int H, cu
     return AKASHIC_OK;
 }
 
+// Reach coefficients of the candidate rows for H hops (after the mass levels).
+static akashic_status_t ensure_reach(akashic_mem *m, const HopPlan &hp, int H, cudaStream_t st) {
+    const int64_t n = m->n;
+    if (m->reach_levels == H && m->reach_n == n) return AKASHIC_OK;
+    AK_TRY(m->reach_rows.ensure(REACH_T * 4));
+    AK_TRY(m->reach_t.ensure(16));
+    AK_TRY(m->reach_map.ensure((size_t)n * 4));
+    AK_TRY(m->reach_c.ensure((size_t)H * n * REACH_T * 4));
+    ReachBuild rb{};
+    rb.n = n;
+    rb.n_split = m->n_split;
+    rb.H = H;
+    rb.split_row = hp.split_row;
+    rb.split_order = hp.split_order;
+    rb.mup = m->mass_up.as<float>();
+    rb.in_ptr = hp.in_ptr;
+    rb.in_src = hp.in_src;
+    rb.in_w = hp.in_w;
+    rb.row_ptr = m->row_ptr.as<int64_t>();
+    rb.col = m->col.as<int32_t>();
+    rb.row_of = m->row_of.as<int32_t>();
+    rb.w = m->w.as<float>();
+    rb.rows = m->reach_rows.as<int32_t>();
+    rb.t_cnt = m->reach_t.as<int>();
+    rb.map = m->reach_map.as<int32_t>();
+    rb.C = m->reach_c.as<float>();
+    CUDA_TRY(launch_reach_build(rb, st));
+    int t = 0;
+    CUDA_TRY(cudaMemcpyAsync(&t, m->reach_t.p, 4, cudaMemcpyDeviceToHost, st));
+    CUDA_TRY(cudaStreamSynchronize(st));
+    m->reach_T = t;
+    m->reach_levels = H;
+    m->reach_n = n;
+    return AKASHIC_OK;
+}
+
 static akashic_status_t retrieve_impl(akashic_mem *m, const uint16_t *q, int32_t B, int32_t k,
                                       float alpha, int32_t hops, const int32_t *q_ns,
                                       int32_t sort_by_time, int64_t *ids, float *scores,
@@ -1213,7 +1258,49 @@ static akashic_status_t retrieve_impl(akashic_mem *m, const uint16_t *q, int32_t
                 row_ub = sc->ub.as<float>();
                 row_lb = sc->lb.as<float>();
             }
-            for (int h = 0; h < eff_hops; ++h) {
+            // Two hops without running them: when every row whose upper bound
+            // reaches the floor (here the k-th largest lower bound) is a
+            // candidate with reach coefficients, their final scores come from
+            // one pass over u and they alone are the selection's candidates.
+            bool reach_done = false;
+            if (prune && eff_hops == 2 && !q_ns && m->reach_on && m->n_split > 0) {
+                int bad = -1;
+                int32_t keep[REACH_T] = {0};
+                {
+                    PhaseScope ph(m, AKASHIC_PHASE_BOUND, st);
+                    AK_TRY(ensure_reach(m, hp, eff_hops, st));
+                    AK_TRY(sc->reach_keep.ensure(REACH_T * 4));
+                    AK_TRY(sc->reach_bad.ensure(16));
+                    const int64_t n_lb = m->n_split < 1024 ? m->n_split : 1024;
+                    CUDA_TRY(launch_prune_floor(nullptr, 0, row_lb, hp.split_row, hp.split_order,
+                                                n_lb, k, sc->pfloor.as<float>(), st));
+                    CUDA_TRY(launch_reach_check(row_ub, sc->pfloor.as<float>(),
+                                                m->reach_map.as<int32_t>(), n,
+                                                sc->reach_keep.as<int32_t>(),
+                                                sc->reach_bad.as<int>(), st));
+                    CUDA_TRY(cudaMemcpyAsync(&bad, sc->reach_bad.p, 4, cudaMemcpyDeviceToHost, st));
+                    CUDA_TRY(cudaMemcpyAsync(keep, sc->reach_keep.p, sizeof keep,
+                                             cudaMemcpyDeviceToHost, st));
+                    CUDA_TRY(cudaStreamSynchronize(st));
+                    ph.launches += 2;
+                }
+                ReachSlots rs{};
+                for (int t = 0; t < REACH_T; ++t)
+                    if (keep[t]) rs.slot[rs.nk++] = t;
+                if (bad == 0 && m->reach_T >= k && rs.nk >= k) {
+                    PhaseScope ph(m, AKASHIC_PHASE_LAST_HOP, st);
+                    AK_TRY(sc->reach_part.ensure((size_t)reach_parts() * REACH_T * bp * 4));
+                    CUDA_TRY(launch_reach_scores(sc->u.as<float>(), bp, b, n, m->reach_c.as<float>(),
+                                                 eff_hops, alpha, rs, m->reach_rows.as<int32_t>(),
+                                                 m->ext_of.as<int32_t>(),
+                                                 sc->reach_part.as<float>(),
+                                                 (unsigned int *)(ws + sp.off_cnt), ws + sp.off_buf,
+                                                 sp.cap, st, &ph.launches));
+                    rc = ColumnRecompute{};   // the buffers hold every candidate
+                    reach_done = true;
+                }
+            }
+            for (int h = 0; h < eff_hops && !reach_done; ++h) {
                 float *out = bufs[h & 1];
                 const bool last = m->fuse_filter && h == eff_hops - 1;
                 if (last) {

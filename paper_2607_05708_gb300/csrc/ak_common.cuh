@@ -410,6 +410,46 @@ cudaError_t launch_prune_floor(const unsigned long long *bound, int n_real, cons
                                const int32_t *lb_rows, const int32_t *order, int64_t n_lb_rows,
                                int k, float *floor_out, cudaStream_t st);
 cudaError_t launch_fill_f32(float *v, int64_t n, float x, cudaStream_t st);
+
+// ------------------------------------------------------------------ reach (ak_reach.cu)
+// Final scores of a few candidate rows straight from u: s^(H)_j = u_j +
+// sum_t alpha^t sum_k C_t[k][j] u_k with graph-only reach coefficients.
+constexpr int REACH_T = 64;          // candidate rows kept
+struct ReachBuild {
+    int64_t n, n_split;
+    int H;
+    const int32_t *split_row, *split_order;
+    const float *mup;                // mass levels [H + 1][n] (candidate choice)
+    const int64_t *in_ptr;           // in-edge CSR (row space)
+    const int32_t *in_src;
+    const float *in_w;
+    const int64_t *row_ptr;          // out-edge CSR (chunk IDs)
+    const int32_t *col, *row_of;
+    const float *w;
+    int32_t *rows;                   // [REACH_T] candidate rows
+    int *t_cnt;                      // their number (device)
+    int32_t *map;                    // [n] row -> candidate slot or -1
+    float *C;                        // [H][n][REACH_T]
+};
+cudaError_t launch_reach_build(const ReachBuild &rb, cudaStream_t st);
+// keep[REACH_T] flags the candidates whose upper bound reaches the floor;
+// *bad counts the other rows that do (the candidates then do not suffice).
+cudaError_t launch_reach_check(const float *ub, const float *floor_p, const int32_t *map,
+                               int64_t n, int32_t *keep, int *bad, cudaStream_t st);
+int reach_parts();                   // CTAs of the score pass (partial rows)
+// The flagged candidates (slots in ascending order), built on the host from
+// the check's flags.
+struct ReachSlots {
+    int32_t slot[REACH_T];
+    int nk;
+};
+// partial: [reach_parts()][REACH_T][bp] scratch; the flagged candidates'
+// keys are written to each real column's buffer (cnt[b] = their number).
+cudaError_t launch_reach_scores(const float *u, int bp, int B, int64_t n, const float *C, int H,
+                                float alpha, const ReachSlots &rs, const int32_t *rows,
+                                const int32_t *ext_of, float *partial, unsigned int *cnt,
+                                unsigned long long *buf, int64_t cap, cudaStream_t st,
+                                int *launches);
 // slot_split[s] = r for every partial slot s of split row r.
 cudaError_t launch_slot_owner(const int64_t *split_slot0, int64_t n_split, int32_t *slot_split,
                               cudaStream_t st);

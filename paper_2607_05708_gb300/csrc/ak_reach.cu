@@ -1,0 +1,249 @@
+// Two-hop scores of the top-k candidates without the hops.
+//
+// Unrolling the hop recursion s^(h) = u + alpha R^T s^(h-1) (the relation
+// propagation of §3, R_ki = w(k -> i)) gives, for a row j,
+//   s^(H)_j = u_j + sum_{t=1..H} alpha^t sum_k C_t[k][j] u_k,
+//   C_1[k][j] = w(k -> j),   C_t = R C_{t-1},
+// with reach coefficients C_t that depend on the graph alone.  The row
+// bounds of the last hop (ak_graph.cu) prove that only the rows whose
+// upper bound reaches the top-k floor can be selected; when all of them lie
+// in a small set of heavy candidate rows whose coefficients are kept, their
+// final scores for every query come from one pass over the score slab u,
+// and the hops are not run.  The selection is the same as the hops' (the
+// values differ only by fp32 summation order).
+#include "ak_common.cuh"
+
+namespace ak {
+
+// ------------------------------------------------------------------ graph-only
+// Candidates: the REACH_T rows of largest upper mass sum_{t<=H} mup[t]
+// among the (up to 1024) heaviest split rows; ties to the lower row.  One
+// CTA of 1024 threads, bitonic sort of the keys in shared memory.
+__global__ __launch_bounds__(1024) void k_reach_pick(const int32_t *__restrict__ split_row,
+                                                      const int32_t *__restrict__ split_order,
+                                                      int64_t n_split,
+                                                      const float *__restrict__ mup, int64_t n,
+                                                      int H, int32_t *__restrict__ rows,
+                                                      int *__restrict__ t_out) {
+    __shared__ unsigned long long key[1024];
+    const int tid = threadIdx.x;
+    const int nc = (int)(n_split < 1024 ? n_split : 1024);
+    unsigned long long k = 0ull;
+    if (tid < nc) {
+        const int32_t r = split_row[split_order[tid]];
+        float m = 0.f;
+        for (int t = 1; t <= H; ++t) m += mup[(int64_t)t * n + r];
+        k = ((unsigned long long)__float_as_uint(m) << 32) | (unsigned long long)(~(uint32_t)r);
+    }
+    key[tid] = k;
+    __syncthreads();
+    // descending bitonic sort
+    for (int size = 2; size <= 1024; size <<= 1) {
+        for (int stride = size >> 1; stride > 0; stride >>= 1) {
+            const int other = tid ^ stride;
+            if (other > tid) {
+                const unsigned long long a = key[tid], b = key[other];
+                const bool desc = (tid & size) == 0;
+                if (desc ? a < b : a > b) {
+                    key[tid] = b;
+                    key[other] = a;
+                }
+            }
+            __syncthreads();
+        }
+    }
+    const int T = nc < REACH_T ? nc : REACH_T;
+    if (tid < T) rows[tid] = (int32_t)~(uint32_t)(key[tid] & 0xffffffffull);
+    if (tid == 0) *t_out = T;
+}
+
+__global__ void k_reach_map(const int32_t *__restrict__ rows, const int *__restrict__ t_cnt,
+                            int32_t *__restrict__ map) {
+    if ((int)threadIdx.x < *t_cnt) map[rows[threadIdx.x]] = (int32_t)threadIdx.x;
+}
+
+// C_1[k][t] = w(k -> rows[t]): the candidate's in-edges (one CTA each).
+__global__ void k_reach_c1(const int32_t *__restrict__ rows, const int *__restrict__ t_cnt,
+                           const int64_t *__restrict__ in_ptr, const int32_t *__restrict__ in_src,
+                           const float *__restrict__ in_w, float *__restrict__ C1) {
+    const int t = blockIdx.x;
+    if (t >= *t_cnt) return;
+    const int64_t j = rows[t];
+    for (int64_t e = in_ptr[j] + threadIdx.x; e < in_ptr[j + 1]; e += blockDim.x)
+        C1[(int64_t)in_src[e] * REACH_T + t] = in_w[e];
+}
+
+// Cn[row(k)][:] = sum over k's out-edges (k -> i) of w * Cp[row(i)][:]: one
+// warp per chunk ID k, two columns per lane, edges in CSR order.
+__global__ void k_reach_spmm(const int64_t *__restrict__ row_ptr, const int32_t *__restrict__ col,
+                             const float *__restrict__ w, const int32_t *__restrict__ row_of,
+                             int64_t n, const float *__restrict__ Cp, float *__restrict__ Cn) {
+    static_assert(REACH_T == 64, "two columns per lane");
+    const int lane = threadIdx.x & 31;
+    const int64_t nw = ((int64_t)gridDim.x * blockDim.x) >> 5;
+    for (int64_t k = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5; k < n; k += nw) {
+        float a0 = 0.f, a1 = 0.f;
+        for (int64_t e = row_ptr[k]; e < row_ptr[k + 1]; ++e) {
+            const float we = w[e];
+            const float *ci = Cp + (int64_t)row_of[col[e]] * REACH_T;
+            a0 = fmaf(we, ci[lane], a0);
+            a1 = fmaf(we, ci[lane + 32], a1);
+        }
+        float *cn = Cn + (int64_t)row_of[k] * REACH_T;
+        cn[lane] = a0;
+        cn[lane + 32] = a1;
+    }
+}
+
+cudaError_t launch_reach_build(const ReachBuild &rb, cudaStream_t st) {
+    const int sms = device_sm_count();
+    cudaError_t e = cudaMemsetAsync(rb.map, 0xff, (size_t)rb.n * 4, st);
+    if (e == cudaSuccess)
+        e = cudaMemsetAsync(rb.C, 0, (size_t)rb.H * rb.n * REACH_T * 4, st);
+    if (e != cudaSuccess) return e;
+    k_reach_pick<<<1, 1024, 0, st>>>(rb.split_row, rb.split_order, rb.n_split, rb.mup, rb.n, rb.H,
+                                     rb.rows, rb.t_cnt);
+    k_reach_map<<<1, REACH_T, 0, st>>>(rb.rows, rb.t_cnt, rb.map);
+    k_reach_c1<<<REACH_T, 256, 0, st>>>(rb.rows, rb.t_cnt, rb.in_ptr, rb.in_src, rb.in_w, rb.C);
+    for (int t = 2; t <= rb.H; ++t)
+        k_reach_spmm<<<sms * 8, 256, 0, st>>>(rb.row_ptr, rb.col, rb.w, rb.row_of, rb.n,
+                                              rb.C + (int64_t)(t - 2) * rb.n * REACH_T,
+                                              rb.C + (int64_t)(t - 1) * rb.n * REACH_T);
+    return cudaGetLastError();
+}
+
+// ------------------------------------------------------------------ per call
+// Rows whose upper bound reaches the floor: a candidate's slot is flagged,
+// any other row counted in *bad (then the hops run instead).
+__global__ void k_reach_check(const float *__restrict__ ub, const float *__restrict__ floor_p,
+                              const int32_t *__restrict__ map, int64_t n,
+                              int32_t *__restrict__ keep, int *__restrict__ bad) {
+    const float floor_ = *floor_p;
+    int nb = 0;
+    for (int64_t j = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; j < n;
+         j += (int64_t)gridDim.x * blockDim.x) {
+        if (ub[j] >= floor_) {
+            const int32_t t = map[j];
+            if (t >= 0) keep[t] = 1;
+            else ++nb;
+        }
+    }
+    if (nb) atomicAdd(bad, nb);
+}
+
+// partial[cta][i][b] = sum over this CTA's rows k of
+// (sum_t alpha^t C_t[k][slot_i]) u[k][b], for the flagged slots (their
+// number NK rounded up to 8; the host chose the instance).  One thread per
+// query column.  REACH_ROWS rows at a time are staged in shared memory
+// (their u rows, every load in flight at once, and their coefficients, the
+// slots past the flagged ones zero), then summed in row order, four
+// coefficients per shared load.
+constexpr int REACH_ROWS = 32;
+
+template <int NK>
+__global__ __launch_bounds__(256, NK <= 24 ? 4 : (NK <= 32 ? 3 : 2)) void k_reach_terms(
+    const float *__restrict__ u, int bp, int64_t n, const float *__restrict__ C, int H,
+    float alpha, const ReachSlots rs, float *__restrict__ partial) {
+    __shared__ __align__(16) float coef[REACH_ROWS][NK];
+    __shared__ float us[REACH_ROWS][256];
+    const int b = threadIdx.x;
+    const int64_t per = (n + gridDim.x - 1) / gridDim.x;
+    const int64_t k0 = (int64_t)blockIdx.x * per;
+    const int64_t k1 = k0 + per < n ? k0 + per : n;
+    float acc[NK];
+#pragma unroll
+    for (int i = 0; i < NK; ++i) acc[i] = 0.f;
+    for (int64_t kb = k0; kb < k1; kb += REACH_ROWS) {
+        const int rows = (int)(k1 - kb < REACH_ROWS ? k1 - kb : REACH_ROWS);
+        if (b < bp) {
+#pragma unroll 8
+            for (int r = 0; r < rows; ++r) us[r][b] = __ldcs(u + (kb + r) * bp + b);
+        }
+        for (int x = threadIdx.x; x < REACH_ROWS * NK; x += blockDim.x) {
+            const int r = x / NK, i = x % NK;
+            float c = 0.f;
+            if (r < rows && i < rs.nk) {
+                const int64_t at = (kb + r) * REACH_T + rs.slot[i];
+                for (int t = H; t >= 1; --t)
+                    c = alpha * (c + C[(int64_t)(t - 1) * n * REACH_T + at]);
+            }
+            coef[r][i] = c;
+        }
+        __syncthreads();
+        if (b < bp) {
+            for (int r = 0; r < rows; ++r) {
+                const float xu = us[r][b];
+                const float4 *c4 = reinterpret_cast<const float4 *>(coef[r]);
+#pragma unroll
+                for (int q = 0; q < NK / 4; ++q) {
+                    const float4 c = c4[q];
+                    acc[4 * q] = fmaf(c.x, xu, acc[4 * q]);
+                    acc[4 * q + 1] = fmaf(c.y, xu, acc[4 * q + 1]);
+                    acc[4 * q + 2] = fmaf(c.z, xu, acc[4 * q + 2]);
+                    acc[4 * q + 3] = fmaf(c.w, xu, acc[4 * q + 3]);
+                }
+            }
+        }
+        __syncthreads();
+    }
+    if (b < bp) {
+#pragma unroll
+        for (int i = 0; i < NK; ++i)
+            if (i < rs.nk) partial[((int64_t)blockIdx.x * REACH_T + i) * bp + b] = acc[i];
+    }
+}
+
+// Final score of each flagged candidate for each real query column: its u
+// plus the partials in CTA order, appended as a filter key (score bits,
+// ~chunk ID) to the column's buffer; the buffer then holds exactly them.
+__global__ void k_reach_emit(const float *__restrict__ u, int bp,
+                             const float *__restrict__ partial, int n_parts, const ReachSlots rs,
+                             const int32_t *__restrict__ rows, const int32_t *__restrict__ ext_of,
+                             unsigned int *__restrict__ cnt, unsigned long long *__restrict__ buf,
+                             int64_t cap) {
+    const int b = blockIdx.x;
+    for (int i = threadIdx.x; i < rs.nk; i += blockDim.x) {
+        const int64_t j = rows[rs.slot[i]];
+        float acc = 0.f;
+        for (int p = 0; p < n_parts; ++p) acc += partial[((int64_t)p * REACH_T + i) * bp + b];
+        const float s = u[j * bp + b] + acc;
+        buf[(int64_t)b * cap + i] =
+            ((unsigned long long)__float_as_uint(s) << 32) | (unsigned long long)(~(uint32_t)ext_of[j]);
+    }
+    if (threadIdx.x == 0) cnt[b] = (unsigned int)rs.nk;
+}
+
+cudaError_t launch_reach_check(const float *ub, const float *floor_p, const int32_t *map,
+                               int64_t n, int32_t *keep, int *bad, cudaStream_t st) {
+    cudaError_t e = cudaMemsetAsync(keep, 0, REACH_T * 4, st);
+    if (e == cudaSuccess) e = cudaMemsetAsync(bad, 0, 4, st);
+    if (e != cudaSuccess) return e;
+    k_reach_check<<<device_sm_count() * 4, 256, 0, st>>>(ub, floor_p, map, n, keep, bad);
+    return cudaGetLastError();
+}
+
+int reach_parts() { return device_sm_count() * 2; }
+
+cudaError_t launch_reach_scores(const float *u, int bp, int B, int64_t n, const float *C, int H,
+                                float alpha, const ReachSlots &rs, const int32_t *rows,
+                                const int32_t *ext_of, float *partial, unsigned int *cnt,
+                                unsigned long long *buf, int64_t cap, cudaStream_t st,
+                                int *launches) {
+    const int parts = reach_parts();
+    switch ((rs.nk + 7) & ~7) {
+    case 8: k_reach_terms<8><<<parts, 256, 0, st>>>(u, bp, n, C, H, alpha, rs, partial); break;
+    case 16: k_reach_terms<16><<<parts, 256, 0, st>>>(u, bp, n, C, H, alpha, rs, partial); break;
+    case 24: k_reach_terms<24><<<parts, 256, 0, st>>>(u, bp, n, C, H, alpha, rs, partial); break;
+    case 32: k_reach_terms<32><<<parts, 256, 0, st>>>(u, bp, n, C, H, alpha, rs, partial); break;
+    case 40: k_reach_terms<40><<<parts, 256, 0, st>>>(u, bp, n, C, H, alpha, rs, partial); break;
+    case 48: k_reach_terms<48><<<parts, 256, 0, st>>>(u, bp, n, C, H, alpha, rs, partial); break;
+    case 56: k_reach_terms<56><<<parts, 256, 0, st>>>(u, bp, n, C, H, alpha, rs, partial); break;
+    case 64: k_reach_terms<64><<<parts, 256, 0, st>>>(u, bp, n, C, H, alpha, rs, partial); break;
+    default: return cudaErrorInvalidValue;
+    }
+    k_reach_emit<<<B, 64, 0, st>>>(u, bp, partial, parts, rs, rows, ext_of, cnt, buf, cap);
+    if (launches) *launches += 2;
+    return cudaGetLastError();
+}
+
+}  // namespace ak

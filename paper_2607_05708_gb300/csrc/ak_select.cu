@@ -569,13 +569,14 @@ __global__ __launch_bounds__(SEL_THREADS) void k_prune_floor(
     if (tid == 0) s_min = 0x7f800000u;
     __syncthreads();
     unsigned int m = 0x7f800000u;
-    for (int c = tid; c < n_real; c += SEL_THREADS) {
+    for (int c = tid; bound && c < n_real; c += SEL_THREADS) {
         const unsigned int hi = (unsigned int)(bound[c] >> 32);
         m = hi < m ? hi : m;
     }
     atomicMin(&s_min, m);
     __syncthreads();
-    float fl = __uint_as_float(s_min);
+    // without filter bounds (no first term) the floor starts at 0
+    float fl = bound ? __uint_as_float(s_min) : 0.f;
     if (lb_rows && n_rows >= k) {
         // keys (lb bits, position): unique, and ordered like lb (lb >= 0)
         auto key_at = [&](int64_t i) -> unsigned long long {

@@ -199,6 +199,33 @@ def test_delete_then_retrieve(hops):
     assert_retrieval_parity(wl, "clustered", got, ref)
 
 
+@pytest.mark.parametrize("placement", ["clustered", "random"])
+def test_two_hop_scores_from_reach_coefficients(placement, monkeypatch):
+    """Two hops without running them: when every row that can reach the
+    top-k floor is one of the candidate rows with graph-only reach
+    coefficients, s^(2) of those rows comes from one pass over u.  On the
+    gmm1m recipe (N = 16384) that path must be taken (no propagation hop is
+    launched) and select what the hops select: equal IDs, pages and counts,
+    scores within fp32 reordering, and the oracle's selection."""
+    monkeypatch.setenv("AKASHIC_REACH", "0")
+    wl = synth.workload(2, scale=1 / 64)
+    _, hops_out = gpu_retrieve(wl, placement)
+    monkeypatch.setenv("AKASHIC_REACH", "1")
+    store = gpu_store(wl, placement)
+    gpu_retrieve(wl, placement, store=store)          # builds the reach coefficients
+    store.set_profiling(True)
+    store.phase_times()
+    _, reach_out = gpu_retrieve(wl, placement, store=store)
+    ph = store.phase_times()
+    store.set_profiling(False)
+    assert ph["propagate"][1] == 0, ph                # no hop launched
+    assert ph["last_hop"][1] > 0, ph                  # the reach scores were
+    for key in ("ids", "page_ids", "n_pages"):
+        assert np.array_equal(hops_out[key], reach_out[key]), key
+    np.testing.assert_allclose(reach_out["scores"], hops_out["scores"], rtol=1e-5, atol=0)
+    assert_retrieval_parity(wl, placement, reach_out, oracle_retrieve(wl, placement))
+
+
 def test_row_bounds_follow_graph_changes():
     """The last hop's graph-only mass levels are cached on the store and
     must be recomputed after the graph changes: retrieve (fills the cache),
