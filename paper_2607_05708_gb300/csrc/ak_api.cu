@@ -87,6 +87,11 @@ struct StreamScratch {
     DevBuf ub, lb, ext, pfloor;  // the last hop's row bounds, extremes, floor
     DevBuf skip_split, skip_slot, kept_rows, kept_count, kept_segs, kflag, kpos, ktmp;
     DevBuf reach_keep, reach_bad, reach_part;
+    // packed coefficients of the last flagged candidates, and their key
+    DevBuf coefK;
+    uint64_t coef_build = ~0ull;
+    float coef_alpha = -1.f;
+    ReachSlots coef_slots{};
 };
 
 struct ProfRec {
@@ -152,6 +157,7 @@ struct akashic_mem {
     int reach_levels = -1;
     int reach_T = 0;          // candidate rows (host copy)
     int64_t reach_n = -1;     // rows they were computed for
+    uint64_t reach_build = 0; // incremented by every rebuild
     bool reach_on = true;     // AKASHIC_REACH=0: always run the hops
     std::mutex mu;
     std::unordered_map<void *, StreamScratch *> scratch;
@@ -1089,6 +1095,7 @@ static akashic_status_t ensure_reach(akashic_mem *m, const HopPlan &hp, int H, c
     m->reach_T = t;
     m->reach_levels = H;
     m->reach_n = n;
+    ++m->reach_build;
     return AKASHIC_OK;
 }
 
@@ -1263,7 +1270,7 @@ static akashic_status_t retrieve_impl(akashic_mem *m, const uint16_t *q, int32_t
             // candidate with reach coefficients, their final scores come from
             // one pass over u and they alone are the selection's candidates.
             bool reach_done = false;
-            if (prune && eff_hops == 2 && !q_ns && m->reach_on && m->n_split > 0) {
+            if (prune && eff_hops == 2 && !q_ns && m->reach_on && m->n_split > 0 && bp == 256) {
                 int bad = -1;
                 int32_t keep[REACH_T] = {0};
                 {
@@ -1290,8 +1297,22 @@ static akashic_status_t retrieve_impl(akashic_mem *m, const uint16_t *q, int32_t
                 if (bad == 0 && m->reach_T >= k && rs.nk >= k) {
                     PhaseScope ph(m, AKASHIC_PHASE_LAST_HOP, st);
                     AK_TRY(sc->reach_part.ensure((size_t)reach_parts() * REACH_T * bp * 4));
-                    CUDA_TRY(launch_reach_scores(sc->u.as<float>(), bp, b, n, m->reach_c.as<float>(),
-                                                 eff_hops, alpha, rs, m->reach_rows.as<int32_t>(),
+                    // packed coefficients, kept while the graph, alpha and the
+                    // flagged candidates stay the same
+                    bool same = sc->coef_build == m->reach_build && sc->coef_alpha == alpha &&
+                                sc->coef_slots.nk == rs.nk;
+                    for (int i = 0; same && i < rs.nk; ++i) same = sc->coef_slots.slot[i] == rs.slot[i];
+                    if (!same) {
+                        AK_TRY(sc->coefK.ensure(reach_coef_floats(n, rs.nk) * 4));
+                        CUDA_TRY(launch_reach_coef(m->reach_c.as<float>(), n, eff_hops, alpha, rs,
+                                                   sc->coefK.as<float>(), st));
+                        ph.launches += 1;
+                        sc->coef_build = m->reach_build;
+                        sc->coef_alpha = alpha;
+                        sc->coef_slots = rs;
+                    }
+                    CUDA_TRY(launch_reach_scores(sc->u.as<float>(), bp, b, n, sc->coefK.as<float>(),
+                                                 rs, m->reach_rows.as<int32_t>(),
                                                  m->ext_of.as<int32_t>(),
                                                  sc->reach_part.as<float>(),
                                                  (unsigned int *)(ws + sp.off_cnt), ws + sp.off_buf,

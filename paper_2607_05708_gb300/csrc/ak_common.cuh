@@ -443,13 +443,18 @@ struct ReachSlots {
     int32_t slot[REACH_T];
     int nk;
 };
-// partial: [reach_parts()][REACH_T][bp] scratch; the flagged candidates'
+// The flagged candidates' combined coefficients sum_t alpha^t C_t, packed
+// [n][nk rounded up to 8] (reach_coef_floats floats).
+size_t reach_coef_floats(int64_t n, int nk);
+cudaError_t launch_reach_coef(const float *C, int64_t n, int H, float alpha, const ReachSlots &rs,
+                              float *coefK, cudaStream_t st);
+// partial: [reach_parts()][REACH_T][256] scratch; the flagged candidates'
 // keys are written to each real column's buffer (cnt[b] = their number).
-cudaError_t launch_reach_scores(const float *u, int bp, int B, int64_t n, const float *C, int H,
-                                float alpha, const ReachSlots &rs, const int32_t *rows,
-                                const int32_t *ext_of, float *partial, unsigned int *cnt,
-                                unsigned long long *buf, int64_t cap, cudaStream_t st,
-                                int *launches);
+// Needs bp = 256.
+cudaError_t launch_reach_scores(const float *u, int bp, int B, int64_t n, const float *coefK,
+                                const ReachSlots &rs, const int32_t *rows, const int32_t *ext_of,
+                                float *partial, unsigned int *cnt, unsigned long long *buf,
+                                int64_t cap, cudaStream_t st, int *launches);
 // slot_split[s] = r for every partial slot s of split row r.
 cudaError_t launch_slot_owner(const int64_t *split_slot0, int64_t n_split, int32_t *slot_split,
                               cudaStream_t st);

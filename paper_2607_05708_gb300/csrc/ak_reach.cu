@@ -131,65 +131,115 @@ __global__ void k_reach_check(const float *__restrict__ ub, const float *__restr
     if (nb) atomicAdd(bad, nb);
 }
 
-// partial[cta][i][b] = sum over this CTA's rows k of
-// (sum_t alpha^t C_t[k][slot_i]) u[k][b], for the flagged slots (their
-// number NK rounded up to 8; the host chose the instance).  One thread per
-// query column.  REACH_ROWS rows at a time are staged in shared memory
-// (their u rows, every load in flight at once, and their coefficients, the
-// slots past the flagged ones zero), then summed in row order, four
-// coefficients per shared load.
+// The flagged candidates' combined coefficients, contiguous:
+// coefK[k][i] = sum_t alpha^t C_t[k][slot_i] for i < nk, 0 up to NK8.
+__global__ void k_reach_coef(const float *__restrict__ C, int64_t n, int H, float alpha,
+                             const ReachSlots rs, int nk8, float *__restrict__ coefK) {
+    for (int64_t x = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; x < n * nk8;
+         x += (int64_t)gridDim.x * blockDim.x) {
+        const int64_t k = x / nk8;
+        const int i = (int)(x - k * nk8);
+        float c = 0.f;
+        if (i < rs.nk) {
+            const int64_t at = k * REACH_T + rs.slot[i];
+            for (int t = H; t >= 1; --t) c = alpha * (c + C[(int64_t)(t - 1) * n * REACH_T + at]);
+        }
+        coefK[x] = c;
+    }
+}
+
+__device__ __forceinline__ void cp_async16(void *dst, const void *src) {
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(
+                     (uint32_t)__cvta_generic_to_shared(dst)),
+                 "l"(src)
+                 : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() {
+    asm volatile("cp.async.commit_group;" ::: "memory");
+}
+template <int N>
+__device__ __forceinline__ void cp_async_wait() {
+    asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
+}
+
+// partial[cta][i][b] = sum over this CTA's rows k of coefK[k][i] u[k][b]
+// (bp = 256 columns of u).  Thread t takes columns 2 (t % 128) + 0..1 and
+// half of the slots (t / 128), so that one shared load of four
+// coefficients feeds eight FMAs; REACH_ROWS rows at a time are copied to
+// shared memory (u rows and coefficient rows) with cp.async,
+// double-buffered so that the next rows load while these are summed; rows
+// in order.
 constexpr int REACH_ROWS = 32;
 
 template <int NK>
-__global__ __launch_bounds__(256, NK <= 24 ? 4 : (NK <= 32 ? 3 : 2)) void k_reach_terms(
-    const float *__restrict__ u, int bp, int64_t n, const float *__restrict__ C, int H,
-    float alpha, const ReachSlots rs, float *__restrict__ partial) {
-    __shared__ __align__(16) float coef[REACH_ROWS][NK];
-    __shared__ float us[REACH_ROWS][256];
-    const int b = threadIdx.x;
+__global__ __launch_bounds__(256, 2) void k_reach_terms(const float *__restrict__ u, int64_t n,
+                                                        const float *__restrict__ coefK, int nk,
+                                                        float *__restrict__ partial) {
+    extern __shared__ __align__(16) float dyn[];
+    float *us = dyn;                                   // [2][REACH_ROWS][256]
+    float *cs = dyn + 2 * REACH_ROWS * 256;            // [2][REACH_ROWS][NK]
+    constexpr int HALF = NK / 2;                       // slots per thread
+    const int cg = threadIdx.x & 127, sg = threadIdx.x >> 7;
     const int64_t per = (n + gridDim.x - 1) / gridDim.x;
     const int64_t k0 = (int64_t)blockIdx.x * per;
     const int64_t k1 = k0 + per < n ? k0 + per : n;
-    float acc[NK];
-#pragma unroll
-    for (int i = 0; i < NK; ++i) acc[i] = 0.f;
-    for (int64_t kb = k0; kb < k1; kb += REACH_ROWS) {
+    const int64_t n_chunks = (k1 - k0 + REACH_ROWS - 1) / REACH_ROWS;
+    auto stage = [&](int64_t c, int buf) {
+        const int64_t kb = k0 + c * REACH_ROWS;
         const int rows = (int)(k1 - kb < REACH_ROWS ? k1 - kb : REACH_ROWS);
-        if (b < bp) {
-#pragma unroll 8
-            for (int r = 0; r < rows; ++r) us[r][b] = __ldcs(u + (kb + r) * bp + b);
-        }
-        for (int x = threadIdx.x; x < REACH_ROWS * NK; x += blockDim.x) {
-            const int r = x / NK, i = x % NK;
-            float c = 0.f;
-            if (r < rows && i < rs.nk) {
-                const int64_t at = (kb + r) * REACH_T + rs.slot[i];
-                for (int t = H; t >= 1; --t)
-                    c = alpha * (c + C[(int64_t)(t - 1) * n * REACH_T + at]);
-            }
-            coef[r][i] = c;
-        }
-        __syncthreads();
-        if (b < bp) {
-            for (int r = 0; r < rows; ++r) {
-                const float xu = us[r][b];
-                const float4 *c4 = reinterpret_cast<const float4 *>(coef[r]);
+        float *ud = us + buf * REACH_ROWS * 256;
+        float *cd = cs + buf * REACH_ROWS * NK;
+        // u rows: rows x 64 pieces of 16 bytes; coefficient rows: rows x NK/4
+        for (int x = threadIdx.x; x < rows * 64; x += 256)
+            cp_async16(ud + x * 4, u + kb * 256 + (int64_t)x * 4);
+        for (int x = threadIdx.x; x < rows * (NK / 4); x += 256)
+            cp_async16(cd + x * 4, coefK + kb * NK + (int64_t)x * 4);
+        cp_async_commit();
+    };
+    float acc[HALF][2];
 #pragma unroll
-                for (int q = 0; q < NK / 4; ++q) {
-                    const float4 c = c4[q];
-                    acc[4 * q] = fmaf(c.x, xu, acc[4 * q]);
-                    acc[4 * q + 1] = fmaf(c.y, xu, acc[4 * q + 1]);
-                    acc[4 * q + 2] = fmaf(c.z, xu, acc[4 * q + 2]);
-                    acc[4 * q + 3] = fmaf(c.w, xu, acc[4 * q + 3]);
-                }
-            }
+    for (int i = 0; i < HALF; ++i) acc[i][0] = acc[i][1] = 0.f;
+    if (n_chunks > 0) stage(0, 0);
+    for (int64_t c = 0; c < n_chunks; ++c) {
+        const int buf = (int)(c & 1);
+        if (c + 1 < n_chunks) {
+            stage(c + 1, buf ^ 1);
+            cp_async_wait<1>();
+        } else {
+            cp_async_wait<0>();
         }
         __syncthreads();
+        const int64_t kb = k0 + c * REACH_ROWS;
+        const int rows = (int)(k1 - kb < REACH_ROWS ? k1 - kb : REACH_ROWS);
+        const float *ud = us + buf * REACH_ROWS * 256;
+        const float *cd = cs + buf * REACH_ROWS * NK;
+#pragma unroll 2
+        for (int r = 0; r < rows; ++r) {
+            const float2 x = *reinterpret_cast<const float2 *>(ud + r * 256 + 2 * cg);
+            const float4 *c4 = reinterpret_cast<const float4 *>(cd + r * NK + sg * HALF);
+#pragma unroll
+            for (int q = 0; q < HALF / 4; ++q) {
+                const float4 cq = c4[q];
+                acc[4 * q][0] = fmaf(cq.x, x.x, acc[4 * q][0]);
+                acc[4 * q][1] = fmaf(cq.x, x.y, acc[4 * q][1]);
+                acc[4 * q + 1][0] = fmaf(cq.y, x.x, acc[4 * q + 1][0]);
+                acc[4 * q + 1][1] = fmaf(cq.y, x.y, acc[4 * q + 1][1]);
+                acc[4 * q + 2][0] = fmaf(cq.z, x.x, acc[4 * q + 2][0]);
+                acc[4 * q + 2][1] = fmaf(cq.z, x.y, acc[4 * q + 2][1]);
+                acc[4 * q + 3][0] = fmaf(cq.w, x.x, acc[4 * q + 3][0]);
+                acc[4 * q + 3][1] = fmaf(cq.w, x.y, acc[4 * q + 3][1]);
+            }
+        }
+        __syncthreads();   // this buffer is restaged two chunks later
     }
-    if (b < bp) {
 #pragma unroll
-        for (int i = 0; i < NK; ++i)
-            if (i < rs.nk) partial[((int64_t)blockIdx.x * REACH_T + i) * bp + b] = acc[i];
+    for (int i = 0; i < HALF; ++i) {
+        const int slot = sg * HALF + i;
+        if (slot < nk) {
+            float *o = partial + ((int64_t)blockIdx.x * REACH_T + slot) * 256 + 2 * cg;
+            o[0] = acc[i][0];
+            o[1] = acc[i][1];
+        }
     }
 }
 
@@ -201,14 +251,21 @@ __global__ void k_reach_emit(const float *__restrict__ u, int bp,
                              const int32_t *__restrict__ rows, const int32_t *__restrict__ ext_of,
                              unsigned int *__restrict__ cnt, unsigned long long *__restrict__ buf,
                              int64_t cap) {
+    // one warp per candidate: lanes take every 32nd partial, then a fixed
+    // reduction tree (the same order on every run)
     const int b = blockIdx.x;
-    for (int i = threadIdx.x; i < rs.nk; i += blockDim.x) {
-        const int64_t j = rows[rs.slot[i]];
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nwarp = blockDim.x >> 5;
+    for (int i = warp; i < rs.nk; i += nwarp) {
         float acc = 0.f;
-        for (int p = 0; p < n_parts; ++p) acc += partial[((int64_t)p * REACH_T + i) * bp + b];
-        const float s = u[j * bp + b] + acc;
-        buf[(int64_t)b * cap + i] =
-            ((unsigned long long)__float_as_uint(s) << 32) | (unsigned long long)(~(uint32_t)ext_of[j]);
+        for (int p = lane; p < n_parts; p += 32) acc += partial[((int64_t)p * REACH_T + i) * bp + b];
+#pragma unroll
+        for (int off = 16; off > 0; off >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, off);
+        if (lane == 0) {
+            const int64_t j = rows[rs.slot[i]];
+            const float s = u[j * bp + b] + acc;
+            buf[(int64_t)b * cap + i] = ((unsigned long long)__float_as_uint(s) << 32) |
+                                        (unsigned long long)(~(uint32_t)ext_of[j]);
+        }
     }
     if (threadIdx.x == 0) cnt[b] = (unsigned int)rs.nk;
 }
@@ -224,24 +281,52 @@ cudaError_t launch_reach_check(const float *ub, const float *floor_p, const int3
 
 int reach_parts() { return device_sm_count() * 2; }
 
-cudaError_t launch_reach_scores(const float *u, int bp, int B, int64_t n, const float *C, int H,
-                                float alpha, const ReachSlots &rs, const int32_t *rows,
-                                const int32_t *ext_of, float *partial, unsigned int *cnt,
-                                unsigned long long *buf, int64_t cap, cudaStream_t st,
-                                int *launches) {
+size_t reach_coef_floats(int64_t n, int nk) { return (size_t)n * ((nk + 7) & ~7); }
+
+cudaError_t launch_reach_coef(const float *C, int64_t n, int H, float alpha, const ReachSlots &rs,
+                              float *coefK, cudaStream_t st) {
+    const int nk8 = (rs.nk + 7) & ~7;
+    k_reach_coef<<<device_sm_count() * 8, 256, 0, st>>>(C, n, H, alpha, rs, nk8, coefK);
+    return cudaGetLastError();
+}
+
+template <int NK>
+static cudaError_t reach_terms_nk(const float *u, int64_t n, const float *coefK, int nk,
+                                  float *partial, int parts, cudaStream_t st) {
+    const size_t smem = (size_t)2 * REACH_ROWS * (256 + NK) * sizeof(float);
+    static bool attr[64] = {false};
+    int dev = 0;
+    cudaGetDevice(&dev);
+    if (dev >= 0 && dev < 64 && !attr[dev]) {
+        cudaError_t e = cudaFuncSetAttribute(k_reach_terms<NK>,
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        if (e != cudaSuccess) return e;
+        attr[dev] = true;
+    }
+    k_reach_terms<NK><<<parts, 256, smem, st>>>(u, n, coefK, nk, partial);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_reach_scores(const float *u, int bp, int B, int64_t n, const float *coefK,
+                                const ReachSlots &rs, const int32_t *rows, const int32_t *ext_of,
+                                float *partial, unsigned int *cnt, unsigned long long *buf,
+                                int64_t cap, cudaStream_t st, int *launches) {
+    if (bp != 256) return cudaErrorInvalidValue;
     const int parts = reach_parts();
+    cudaError_t e;
     switch ((rs.nk + 7) & ~7) {
-    case 8: k_reach_terms<8><<<parts, 256, 0, st>>>(u, bp, n, C, H, alpha, rs, partial); break;
-    case 16: k_reach_terms<16><<<parts, 256, 0, st>>>(u, bp, n, C, H, alpha, rs, partial); break;
-    case 24: k_reach_terms<24><<<parts, 256, 0, st>>>(u, bp, n, C, H, alpha, rs, partial); break;
-    case 32: k_reach_terms<32><<<parts, 256, 0, st>>>(u, bp, n, C, H, alpha, rs, partial); break;
-    case 40: k_reach_terms<40><<<parts, 256, 0, st>>>(u, bp, n, C, H, alpha, rs, partial); break;
-    case 48: k_reach_terms<48><<<parts, 256, 0, st>>>(u, bp, n, C, H, alpha, rs, partial); break;
-    case 56: k_reach_terms<56><<<parts, 256, 0, st>>>(u, bp, n, C, H, alpha, rs, partial); break;
-    case 64: k_reach_terms<64><<<parts, 256, 0, st>>>(u, bp, n, C, H, alpha, rs, partial); break;
+    case 8: e = reach_terms_nk<8>(u, n, coefK, rs.nk, partial, parts, st); break;
+    case 16: e = reach_terms_nk<16>(u, n, coefK, rs.nk, partial, parts, st); break;
+    case 24: e = reach_terms_nk<24>(u, n, coefK, rs.nk, partial, parts, st); break;
+    case 32: e = reach_terms_nk<32>(u, n, coefK, rs.nk, partial, parts, st); break;
+    case 40: e = reach_terms_nk<40>(u, n, coefK, rs.nk, partial, parts, st); break;
+    case 48: e = reach_terms_nk<48>(u, n, coefK, rs.nk, partial, parts, st); break;
+    case 56: e = reach_terms_nk<56>(u, n, coefK, rs.nk, partial, parts, st); break;
+    case 64: e = reach_terms_nk<64>(u, n, coefK, rs.nk, partial, parts, st); break;
     default: return cudaErrorInvalidValue;
     }
-    k_reach_emit<<<B, 64, 0, st>>>(u, bp, partial, parts, rs, rows, ext_of, cnt, buf, cap);
+    if (e != cudaSuccess) return e;
+    k_reach_emit<<<B, 256, 0, st>>>(u, bp, partial, parts, rs, rows, ext_of, cnt, buf, cap);
     if (launches) *launches += 2;
     return cudaGetLastError();
 }
