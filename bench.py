@@ -722,6 +722,17 @@ def run_retrieve(args, k=None, hops=None, metric=METRIC, workload=WORKLOAD, scop
         what = "selection pass (final slab read once)"
     dom_avg_ms = dom_ms / units
     achieved = per_launch_bytes / (dom_avg_ms * 1e-3) / 1e9
+    # which propagation ran: the hops, or (two hops, every row that can reach
+    # the top-k among the reach candidates) the candidates' scores from u
+    if hops >= 1 and phases["propagate"][1] == 0 and phases["last_hop"][1] > 0:
+        path_note = {"propagation": "two-hop scores of the top-k candidates from graph-only "
+                                    "reach coefficients, one pass over u (no hop run)",
+                     "bytes_moved_per_step": wl.n * wl.dim * 2 + 2 * wl.n * 256 * 4
+                                             + wl.n * 40 * 4,
+                     "note": "pass_roofline counts full hops (five slab passes); this path "
+                             "reads E, writes u and reads u and the candidates' coefficients"}
+    else:
+        path_note = {"propagation": "hops (the last one skips rows below the top-k floor)"}
     line = {
         "metric": metric,
         "value": job_throughput(B * args.steps, ws, ms),
@@ -750,6 +761,7 @@ def run_retrieve(args, k=None, hops=None, metric=METRIC, workload=WORKLOAD, scop
                           "flops": 2.0 * wl.n * B * wl.dim,
                           "peak_tflops_bf16": bf16},
         "phases_ms_per_step": {p: phases[p][0] / args.steps for p in retr},
+        "path": path_note,
         "e2e": {"value": job_throughput(B * args.steps, ws, ms_e2e), "unit": "queries/s",
                 "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
         "gpu_launches": int(sum(v[1] for v in phases.values())),
