@@ -85,6 +85,9 @@ def hop_bytes(n, b, nnz):
 # dram__bytes_read/write counters.  Set to None when the hop kernels change
 # until they are captured again.
 HOP_DRAM_BYTES = 11.16e9
+# DRAM bytes of the score GEMM (E read once, the u slab written once; 2.148 +
+# 1.034 GB) from the same kind of capture.
+SCORE_DRAM_BYTES = 3.182e9
 
 
 def score_bytes(n, d, b):
@@ -752,8 +755,9 @@ def run_retrieve(args, k=None, hops=None, metric=METRIC, workload=WORKLOAD, scop
                    "parallelism": "replicas" if ws > 1 else "single GPU"},
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": hbm, "unit": "GB/s",
                      "frac": achieved / hbm,
-                     "traffic": (HOP_DRAM_BYTES if dom == "propagate" and args.scale == 1.0
-                                 else None),
+                     "traffic": (None if args.scale != 1.0 else
+                                 HOP_DRAM_BYTES if dom == "propagate" else
+                                 SCORE_DRAM_BYTES if dom == "score" else None),
                      "kernel": dom, "what": what, "peak_kind": peak_kind},
         "pass_roofline": {"algorithmic_bytes": total_ab,
                           "ideal_ms": total_ab / (hbm * 1e9) * 1e3,
