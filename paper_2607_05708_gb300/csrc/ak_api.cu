@@ -91,6 +91,7 @@ struct StreamScratch {
     DevBuf coefK;
     uint64_t coef_build = ~0ull;
     float coef_alpha = -1.f;
+    int coef_bp = 0;
     ReachSlots coef_slots{};
 };
 
@@ -1270,7 +1271,8 @@ static akashic_status_t retrieve_impl(akashic_mem *m, const uint16_t *q, int32_t
             // candidate with reach coefficients, their final scores come from
             // one pass over u and they alone are the selection's candidates.
             bool reach_done = false;
-            if (prune && eff_hops == 2 && !q_ns && m->reach_on && m->n_split > 0 && bp == 256) {
+            if (prune && eff_hops == 2 && !q_ns && m->reach_on && m->n_split > 0 &&
+                (bp == 256 || bp == 128)) {
                 int bad = -1;
                 int32_t keep[REACH_T] = {0};
                 {
@@ -1294,19 +1296,20 @@ static akashic_status_t retrieve_impl(akashic_mem *m, const uint16_t *q, int32_t
                 ReachSlots rs{};
                 for (int t = 0; t < REACH_T; ++t)
                     if (keep[t]) rs.slot[rs.nk++] = t;
-                if (bad == 0 && m->reach_T >= k && rs.nk >= k) {
+                if (bad == 0 && m->reach_T >= k && rs.nk >= k && reach_fits(bp, rs.nk)) {
                     PhaseScope ph(m, AKASHIC_PHASE_LAST_HOP, st);
                     AK_TRY(sc->reach_part.ensure((size_t)reach_parts() * REACH_T * bp * 4));
                     // packed coefficients, kept while the graph, alpha and the
                     // flagged candidates stay the same
                     bool same = sc->coef_build == m->reach_build && sc->coef_alpha == alpha &&
-                                sc->coef_slots.nk == rs.nk;
+                                sc->coef_bp == bp && sc->coef_slots.nk == rs.nk;
                     for (int i = 0; same && i < rs.nk; ++i) same = sc->coef_slots.slot[i] == rs.slot[i];
                     if (!same) {
-                        AK_TRY(sc->coefK.ensure(reach_coef_floats(n, rs.nk) * 4));
+                        AK_TRY(sc->coefK.ensure(reach_coef_floats(n, bp, rs.nk) * 4));
                         CUDA_TRY(launch_reach_coef(m->reach_c.as<float>(), n, eff_hops, alpha, rs,
-                                                   sc->coefK.as<float>(), st));
+                                                   bp, sc->coefK.as<float>(), st));
                         ph.launches += 1;
+                        sc->coef_bp = bp;
                         sc->coef_build = m->reach_build;
                         sc->coef_alpha = alpha;
                         sc->coef_slots = rs;

@@ -414,7 +414,7 @@ cudaError_t launch_fill_f32(float *v, int64_t n, float x, cudaStream_t st);
 // ------------------------------------------------------------------ reach (ak_reach.cu)
 // Final scores of a few candidate rows straight from u: s^(H)_j = u_j +
 // sum_t alpha^t sum_k C_t[k][j] u_k with graph-only reach coefficients.
-constexpr int REACH_T = 64;          // candidate rows kept
+constexpr int REACH_T = 128;         // candidate rows kept
 struct ReachBuild {
     int64_t n, n_split;
     int H;
@@ -445,12 +445,14 @@ struct ReachSlots {
 };
 // The flagged candidates' combined coefficients sum_t alpha^t C_t, packed
 // [n][nk rounded up to 8] (reach_coef_floats floats).
-size_t reach_coef_floats(int64_t n, int nk);
+size_t reach_coef_floats(int64_t n, int bp, int nk);
 cudaError_t launch_reach_coef(const float *C, int64_t n, int H, float alpha, const ReachSlots &rs,
-                              float *coefK, cudaStream_t st);
-// partial: [reach_parts()][REACH_T][256] scratch; the flagged candidates'
+                              int bp, float *coefK, cudaStream_t st);
+// partial: [reach_parts()][REACH_T][bp] scratch; the flagged candidates'
 // keys are written to each real column's buffer (cnt[b] = their number).
-// Needs bp = 256.
+// Needs bp = 256 with at most 64 flagged candidates, or bp = 128 with at
+// most 128 (reach_fits).
+bool reach_fits(int bp, int nk);
 cudaError_t launch_reach_scores(const float *u, int bp, int B, int64_t n, const float *coefK,
                                 const ReachSlots &rs, const int32_t *rows, const int32_t *ext_of,
                                 float *partial, unsigned int *cnt, unsigned long long *buf,

@@ -74,24 +74,25 @@ __global__ void k_reach_c1(const int32_t *__restrict__ rows, const int *__restri
 }
 
 // Cn[row(k)][:] = sum over k's out-edges (k -> i) of w * Cp[row(i)][:]: one
-// warp per chunk ID k, two columns per lane, edges in CSR order.
+// warp per chunk ID k, four columns per lane (a float4), edges in CSR order.
 __global__ void k_reach_spmm(const int64_t *__restrict__ row_ptr, const int32_t *__restrict__ col,
                              const float *__restrict__ w, const int32_t *__restrict__ row_of,
                              int64_t n, const float *__restrict__ Cp, float *__restrict__ Cn) {
-    static_assert(REACH_T == 64, "two columns per lane");
+    static_assert(REACH_T == 128, "four columns per lane");
     const int lane = threadIdx.x & 31;
     const int64_t nw = ((int64_t)gridDim.x * blockDim.x) >> 5;
     for (int64_t k = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5; k < n; k += nw) {
-        float a0 = 0.f, a1 = 0.f;
+        float4 a = make_float4(0.f, 0.f, 0.f, 0.f);
         for (int64_t e = row_ptr[k]; e < row_ptr[k + 1]; ++e) {
             const float we = w[e];
-            const float *ci = Cp + (int64_t)row_of[col[e]] * REACH_T;
-            a0 = fmaf(we, ci[lane], a0);
-            a1 = fmaf(we, ci[lane + 32], a1);
+            const float4 c =
+                reinterpret_cast<const float4 *>(Cp + (int64_t)row_of[col[e]] * REACH_T)[lane];
+            a.x = fmaf(we, c.x, a.x);
+            a.y = fmaf(we, c.y, a.y);
+            a.z = fmaf(we, c.z, a.z);
+            a.w = fmaf(we, c.w, a.w);
         }
-        float *cn = Cn + (int64_t)row_of[k] * REACH_T;
-        cn[lane] = a0;
-        cn[lane + 32] = a1;
+        reinterpret_cast<float4 *>(Cn + (int64_t)row_of[k] * REACH_T)[lane] = a;
     }
 }
 
@@ -163,23 +164,25 @@ __device__ __forceinline__ void cp_async_wait() {
 }
 
 // partial[cta][i][b] = sum over this CTA's rows k of coefK[k][i] u[k][b]
-// (bp = 256 columns of u).  Thread t takes columns 2 (t % 128) + 0..1 and
-// half of the slots (t / 128), so that one shared load of four
-// coefficients feeds eight FMAs; REACH_ROWS rows at a time are copied to
-// shared memory (u rows and coefficient rows) with cp.async,
+// (BP = 256 or 128 columns of u).  Thread t takes columns 2 (t % (BP/2)) +
+// 0..1 and one of G = 512 / BP slot groups (t / (BP/2)), so that one shared
+// load of four coefficients feeds eight FMAs; REACH_ROWS rows at a time
+// are copied to shared memory (u rows and coefficient rows) with cp.async,
 // double-buffered so that the next rows load while these are summed; rows
 // in order.
 constexpr int REACH_ROWS = 32;
 
-template <int NK>
+template <int NK, int BP>
 __global__ __launch_bounds__(256, 2) void k_reach_terms(const float *__restrict__ u, int64_t n,
                                                         const float *__restrict__ coefK, int nk,
                                                         float *__restrict__ partial) {
     extern __shared__ __align__(16) float dyn[];
-    float *us = dyn;                                   // [2][REACH_ROWS][256]
-    float *cs = dyn + 2 * REACH_ROWS * 256;            // [2][REACH_ROWS][NK]
-    constexpr int HALF = NK / 2;                       // slots per thread
-    const int cg = threadIdx.x & 127, sg = threadIdx.x >> 7;
+    constexpr int G = 512 / BP;                        // slot groups
+    constexpr int HALF = NK / G;                       // slots per thread
+    static_assert(HALF % 4 == 0, "four coefficients per shared load");
+    float *us = dyn;                                   // [2][REACH_ROWS][BP]
+    float *cs = dyn + 2 * REACH_ROWS * BP;             // [2][REACH_ROWS][NK]
+    const int cg = threadIdx.x % (BP / 2), sg = threadIdx.x / (BP / 2);
     const int64_t per = (n + gridDim.x - 1) / gridDim.x;
     const int64_t k0 = (int64_t)blockIdx.x * per;
     const int64_t k1 = k0 + per < n ? k0 + per : n;
@@ -187,11 +190,11 @@ __global__ __launch_bounds__(256, 2) void k_reach_terms(const float *__restrict_
     auto stage = [&](int64_t c, int buf) {
         const int64_t kb = k0 + c * REACH_ROWS;
         const int rows = (int)(k1 - kb < REACH_ROWS ? k1 - kb : REACH_ROWS);
-        float *ud = us + buf * REACH_ROWS * 256;
+        float *ud = us + buf * REACH_ROWS * BP;
         float *cd = cs + buf * REACH_ROWS * NK;
-        // u rows: rows x 64 pieces of 16 bytes; coefficient rows: rows x NK/4
-        for (int x = threadIdx.x; x < rows * 64; x += 256)
-            cp_async16(ud + x * 4, u + kb * 256 + (int64_t)x * 4);
+        // u rows: rows x BP/4 pieces of 16 bytes; coefficient rows: rows x NK/4
+        for (int x = threadIdx.x; x < rows * (BP / 4); x += 256)
+            cp_async16(ud + x * 4, u + kb * BP + (int64_t)x * 4);
         for (int x = threadIdx.x; x < rows * (NK / 4); x += 256)
             cp_async16(cd + x * 4, coefK + kb * NK + (int64_t)x * 4);
         cp_async_commit();
@@ -211,11 +214,11 @@ __global__ __launch_bounds__(256, 2) void k_reach_terms(const float *__restrict_
         __syncthreads();
         const int64_t kb = k0 + c * REACH_ROWS;
         const int rows = (int)(k1 - kb < REACH_ROWS ? k1 - kb : REACH_ROWS);
-        const float *ud = us + buf * REACH_ROWS * 256;
+        const float *ud = us + buf * REACH_ROWS * BP;
         const float *cd = cs + buf * REACH_ROWS * NK;
 #pragma unroll 2
         for (int r = 0; r < rows; ++r) {
-            const float2 x = *reinterpret_cast<const float2 *>(ud + r * 256 + 2 * cg);
+            const float2 x = *reinterpret_cast<const float2 *>(ud + r * BP + 2 * cg);
             const float4 *c4 = reinterpret_cast<const float4 *>(cd + r * NK + sg * HALF);
 #pragma unroll
             for (int q = 0; q < HALF / 4; ++q) {
@@ -236,7 +239,7 @@ __global__ __launch_bounds__(256, 2) void k_reach_terms(const float *__restrict_
     for (int i = 0; i < HALF; ++i) {
         const int slot = sg * HALF + i;
         if (slot < nk) {
-            float *o = partial + ((int64_t)blockIdx.x * REACH_T + slot) * 256 + 2 * cg;
+            float *o = partial + ((int64_t)blockIdx.x * REACH_T + slot) * BP + 2 * cg;
             o[0] = acc[i][0];
             o[1] = acc[i][1];
         }
@@ -281,49 +284,72 @@ cudaError_t launch_reach_check(const float *ub, const float *floor_p, const int3
 
 int reach_parts() { return device_sm_count() * 2; }
 
-size_t reach_coef_floats(int64_t n, int nk) { return (size_t)n * ((nk + 7) & ~7); }
+// The packed width: the flagged count rounded up to 8 (bp = 256) or 16.
+static int reach_width(int bp, int nk) { return bp == 256 ? (nk + 7) & ~7 : (nk + 15) & ~15; }
+
+size_t reach_coef_floats(int64_t n, int bp, int nk) { return (size_t)n * reach_width(bp, nk); }
 
 cudaError_t launch_reach_coef(const float *C, int64_t n, int H, float alpha, const ReachSlots &rs,
-                              float *coefK, cudaStream_t st) {
-    const int nk8 = (rs.nk + 7) & ~7;
+                              int bp, float *coefK, cudaStream_t st) {
+    const int nk8 = reach_width(bp, rs.nk);
     k_reach_coef<<<device_sm_count() * 8, 256, 0, st>>>(C, n, H, alpha, rs, nk8, coefK);
     return cudaGetLastError();
 }
 
-template <int NK>
+template <int NK, int BP>
 static cudaError_t reach_terms_nk(const float *u, int64_t n, const float *coefK, int nk,
                                   float *partial, int parts, cudaStream_t st) {
-    const size_t smem = (size_t)2 * REACH_ROWS * (256 + NK) * sizeof(float);
+    const size_t smem = (size_t)2 * REACH_ROWS * (BP + NK) * sizeof(float);
     static bool attr[64] = {false};
     int dev = 0;
     cudaGetDevice(&dev);
     if (dev >= 0 && dev < 64 && !attr[dev]) {
-        cudaError_t e = cudaFuncSetAttribute(k_reach_terms<NK>,
+        cudaError_t e = cudaFuncSetAttribute(k_reach_terms<NK, BP>,
                                              cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         if (e != cudaSuccess) return e;
         attr[dev] = true;
     }
-    k_reach_terms<NK><<<parts, 256, smem, st>>>(u, n, coefK, nk, partial);
+    k_reach_terms<NK, BP><<<parts, 256, smem, st>>>(u, n, coefK, nk, partial);
     return cudaGetLastError();
+}
+
+// Flagged counts the score pass takes: NK (rounded up to 8 / 16) at most 64
+// slots per thread group pair at BP = 256, 128 at BP = 128.
+bool reach_fits(int bp, int nk) {
+    return nk >= 1 && ((bp == 256 && nk <= 64) || (bp == 128 && nk <= 128));
 }
 
 cudaError_t launch_reach_scores(const float *u, int bp, int B, int64_t n, const float *coefK,
                                 const ReachSlots &rs, const int32_t *rows, const int32_t *ext_of,
                                 float *partial, unsigned int *cnt, unsigned long long *buf,
                                 int64_t cap, cudaStream_t st, int *launches) {
-    if (bp != 256) return cudaErrorInvalidValue;
+    if (!reach_fits(bp, rs.nk)) return cudaErrorInvalidValue;
     const int parts = reach_parts();
-    cudaError_t e;
-    switch ((rs.nk + 7) & ~7) {
-    case 8: e = reach_terms_nk<8>(u, n, coefK, rs.nk, partial, parts, st); break;
-    case 16: e = reach_terms_nk<16>(u, n, coefK, rs.nk, partial, parts, st); break;
-    case 24: e = reach_terms_nk<24>(u, n, coefK, rs.nk, partial, parts, st); break;
-    case 32: e = reach_terms_nk<32>(u, n, coefK, rs.nk, partial, parts, st); break;
-    case 40: e = reach_terms_nk<40>(u, n, coefK, rs.nk, partial, parts, st); break;
-    case 48: e = reach_terms_nk<48>(u, n, coefK, rs.nk, partial, parts, st); break;
-    case 56: e = reach_terms_nk<56>(u, n, coefK, rs.nk, partial, parts, st); break;
-    case 64: e = reach_terms_nk<64>(u, n, coefK, rs.nk, partial, parts, st); break;
-    default: return cudaErrorInvalidValue;
+    cudaError_t e = cudaErrorInvalidValue;
+    if (bp == 256) {
+        switch ((rs.nk + 7) & ~7) {
+        case 8: e = reach_terms_nk<8, 256>(u, n, coefK, rs.nk, partial, parts, st); break;
+        case 16: e = reach_terms_nk<16, 256>(u, n, coefK, rs.nk, partial, parts, st); break;
+        case 24: e = reach_terms_nk<24, 256>(u, n, coefK, rs.nk, partial, parts, st); break;
+        case 32: e = reach_terms_nk<32, 256>(u, n, coefK, rs.nk, partial, parts, st); break;
+        case 40: e = reach_terms_nk<40, 256>(u, n, coefK, rs.nk, partial, parts, st); break;
+        case 48: e = reach_terms_nk<48, 256>(u, n, coefK, rs.nk, partial, parts, st); break;
+        case 56: e = reach_terms_nk<56, 256>(u, n, coefK, rs.nk, partial, parts, st); break;
+        case 64: e = reach_terms_nk<64, 256>(u, n, coefK, rs.nk, partial, parts, st); break;
+        default: break;
+        }
+    } else {
+        switch ((rs.nk + 15) & ~15) {
+        case 16: e = reach_terms_nk<16, 128>(u, n, coefK, rs.nk, partial, parts, st); break;
+        case 32: e = reach_terms_nk<32, 128>(u, n, coefK, rs.nk, partial, parts, st); break;
+        case 48: e = reach_terms_nk<48, 128>(u, n, coefK, rs.nk, partial, parts, st); break;
+        case 64: e = reach_terms_nk<64, 128>(u, n, coefK, rs.nk, partial, parts, st); break;
+        case 80: e = reach_terms_nk<80, 128>(u, n, coefK, rs.nk, partial, parts, st); break;
+        case 96: e = reach_terms_nk<96, 128>(u, n, coefK, rs.nk, partial, parts, st); break;
+        case 112: e = reach_terms_nk<112, 128>(u, n, coefK, rs.nk, partial, parts, st); break;
+        case 128: e = reach_terms_nk<128, 128>(u, n, coefK, rs.nk, partial, parts, st); break;
+        default: break;
+        }
     }
     if (e != cudaSuccess) return e;
     k_reach_emit<<<B, 256, 0, st>>>(u, bp, partial, parts, rs, rows, ext_of, cnt, buf, cap);

@@ -199,16 +199,22 @@ def test_delete_then_retrieve(hops):
     assert_retrieval_parity(wl, "clustered", got, ref)
 
 
-@pytest.mark.parametrize("placement", ["clustered", "random"])
-def test_two_hop_scores_from_reach_coefficients(placement, monkeypatch):
+@pytest.mark.parametrize("placement,B,k,must", [
+    ("clustered", 256, 32, True), ("random", 256, 32, True), ("clustered", 128, 32, True),
+    ("clustered", 128, 64, False),
+])
+def test_two_hop_scores_from_reach_coefficients(placement, B, k, must, monkeypatch):
     """Two hops without running them: when every row that can reach the
     top-k floor is one of the candidate rows with graph-only reach
     coefficients, s^(2) of those rows comes from one pass over u.  On the
-    gmm1m recipe (N = 16384) that path must be taken (no propagation hop is
-    launched) and select what the hops select: equal IDs, pages and counts,
-    scores within fp32 reordering, and the oracle's selection."""
+    gmm1m recipe (N = 16384) that path must be taken where `must` (no
+    propagation hop is launched) and select what the hops select: equal IDs,
+    pages and counts, scores within fp32 reordering, and the oracle's
+    selection (B = 256 and 128 queries, k = 32 and 64)."""
+    import dataclasses
+    wl = dataclasses.replace(synth.workload(2, scale=1 / 64), k=k)
+    wl = dataclasses.replace(wl, queries=wl.queries[:B])
     monkeypatch.setenv("AKASHIC_REACH", "0")
-    wl = synth.workload(2, scale=1 / 64)
     _, hops_out = gpu_retrieve(wl, placement)
     monkeypatch.setenv("AKASHIC_REACH", "1")
     store = gpu_store(wl, placement)
@@ -218,8 +224,9 @@ def test_two_hop_scores_from_reach_coefficients(placement, monkeypatch):
     _, reach_out = gpu_retrieve(wl, placement, store=store)
     ph = store.phase_times()
     store.set_profiling(False)
-    assert ph["propagate"][1] == 0, ph                # no hop launched
-    assert ph["last_hop"][1] > 0, ph                  # the reach scores were
+    if must:
+        assert ph["propagate"][1] == 0, ph            # no hop launched
+        assert ph["last_hop"][1] > 0, ph              # the reach scores were
     for key in ("ids", "page_ids", "n_pages"):
         assert np.array_equal(hops_out[key], reach_out[key]), key
     np.testing.assert_allclose(reach_out["scores"], hops_out["scores"], rtol=1e-5, atol=0)
