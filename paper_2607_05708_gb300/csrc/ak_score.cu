@@ -147,6 +147,14 @@ struct GemmEpi {
     int n_real;                         // the row over the first n_real columns
 };
 
+// z[ch] += s with a run-time chunk index kept out of local memory.
+template <int N>
+__device__ __forceinline__ void zadd(float (&z)[N], int ch, float s) {
+#pragma unroll
+    for (int i = 0; i < N; ++i)
+        if (i == ch) z[i] += s;
+}
+
 template <int BP, int MODE>
 struct GemmCfg {
     static constexpr int BM = 128, BK = 64;
@@ -337,6 +345,11 @@ __global__ __launch_bounds__(GemmCfg<BP, MODE>::THREADS, 1) void k_gemm_umma(con
         const int et = threadIdx.x - 64;                 // 0..EPI_T-1
         constexpr int CH_PER = BP / 32 / (C::EPI_W / 4); // 32-column chunks per epilogue warp
         const int hsel = (warp - 2) / 4;                 // which column share
+        // EXP: column sums toward Z, per warp (its 32 rows) and chunk, over
+        // all the CTA's tiles (one column tile), lane = column in the chunk
+        float zl[BP / 32];
+#pragma unroll
+        for (int i = 0; i < BP / 32; ++i) zl[i] = 0.f;
         int it = 0, cc = 0;
         for (int64_t u = u_first; u < n_units; u += u_step, ++it) {
             const int64_t ct = u % n_ctiles;
@@ -440,26 +453,35 @@ __global__ __launch_bounds__(GemmCfg<BP, MODE>::THREADS, 1) void k_gemm_umma(con
                         }
                     }
                 }
-                named_bar(1, C::EPI_T);                       // staging[buf] free again
-                float4 *dst = (float4 *)(sOut + buf * (C::OUT_BYTES / 4) + row * 32);
+                // stage the row: EXP_FILTER in the warp's own 32 rows of
+                // buffer 0 (warp-private, no CTA barrier); EXP in buffer buf,
+                // shared with the TMA store
+                float *so_base;
+                if constexpr (EXPF) {
+                    __syncwarp();                             // the warp's rows free again
+                    so_base = sOut;
+                } else {
+                    named_bar(1, C::EPI_T);                   // staging[buf] free again
+                    so_base = sOut + buf * (C::OUT_BYTES / 4);
+                }
+                float4 *dst = (float4 *)(so_base + row * 32);
 #pragma unroll
                 for (int j = 0; j < 8; ++j)
                     dst[j ^ (row & 7)] = make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
-                fence_async_smem();
-                named_bar(1, C::EPI_T);                       // staging[buf] complete
+                if (!EXPF) fence_async_smem();
+                __syncwarp();
                 if (EXP) {
-                    const int c = et & 31, g = et >> 5;
-                    const float *so = sOut + buf * (C::OUT_BYTES / 4);
+                    // column `lane` of this warp's 32 rows
                     float s = 0.f;
 #pragma unroll 8
-                    for (int rr = g * 32; rr < g * 32 + 32; ++rr)
-                        s += so[rr * 32 + ((((c >> 2) ^ (rr & 7))) << 2) + (c & 3)];
-                    zq[g * 32 + c] = s;
+                    for (int rr = q * 32; rr < q * 32 + 32; ++rr)
+                        s += so_base[rr * 32 + ((((lane >> 2) ^ (rr & 7))) << 2) + (lane & 3)];
+                    zadd(zl, ch, s);
                 }
                 if constexpr (EXPF) {
                     // second half: the exact key test and append for the
                     // flagged values, read back from the staged row
-                    const float *so = sOut + buf * (C::OUT_BYTES / 4) + row * 32;
+                    const float *so = so_base + row * 32;
                     while (pass) {
                         const int i = __ffs(pass) - 1;
                         pass &= pass - 1u;
@@ -473,17 +495,14 @@ __global__ __launch_bounds__(GemmCfg<BP, MODE>::THREADS, 1) void k_gemm_umma(con
                             if ((int64_t)p < ep.cap) ep.buf[cg * ep.cap + p] = key;
                         }
                     }
+                } else {
+                    named_bar(1, C::EPI_T);                   // staging[buf] complete
+                    if (et == 0) {
+                        tma_store_2d(&tmC, so_base, (int)(ct * BP + ch * 32), (int)(mt * C::BM));
+                        bulk_commit();
+                        bulk_wait_read<1>();                  // the other buffer is free
+                    }
                 }
-                if (!EXPF && et == 0) {
-                    tma_store_2d(&tmC, sOut + buf * (C::OUT_BYTES / 4), (int)(ct * BP + ch * 32),
-                                 (int)(mt * C::BM));
-                    bulk_commit();
-                }
-                if (EXP) {
-                    named_bar(1, C::EPI_T);
-                    if (et < 32) zacc[ch * 32 + et] += (zq[et] + zq[32 + et]) + (zq[64 + et] + zq[96 + et]);
-                }
-                if (!EXPF && et == 0) bulk_wait_read<1>();
                 }
             }
             if (MODE == GEMM_EXP && ep.row_max && in_rows) {
@@ -496,8 +515,16 @@ __global__ __launch_bounds__(GemmCfg<BP, MODE>::THREADS, 1) void k_gemm_umma(con
         }
         if (!EXPF && et == 0) bulk_wait_all();
         named_bar(1, C::EPI_T);
-        if (EXP && ep.zpart)
-            for (int c = et; c < BP; c += 128) ep.zpart[(int64_t)blockIdx.x * BP + c] = zacc[c];
+        if (EXP && ep.zpart) {
+            // the four warps' column sums, added in a fixed order
+            float *zred = sOut;                               // [4][BP], free now
+#pragma unroll
+            for (int i = 0; i < BP / 32; ++i) zred[q * BP + i * 32 + lane] = zl[i];
+            named_bar(1, C::EPI_T);
+            for (int c = et; c < BP; c += C::EPI_T)
+                ep.zpart[(int64_t)blockIdx.x * BP + c] =
+                    (zred[c] + zred[BP + c]) + (zred[2 * BP + c] + zred[3 * BP + c]);
+        }
     }
     tc_fence_before();
     __syncthreads();
