@@ -548,8 +548,9 @@ def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=None,
-                    help="timed steps (default: 100 for retrieve and the reference arm, "
-                         "5 for update, 20 for streams)")
+                    help="timed steps (default: 400 for retrieve and dense, 100 for scoped and "
+                         "the reference arm, 5 for update, 20 for streams and memory, 10 for "
+                         "delete)")
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="native", choices=["native", "reference"])
     ap.add_argument("--cpu-queries", type=int, default=8)
@@ -567,8 +568,10 @@ def main():
                          "delete: 1024 chunks deleted per step from the 1M store; memory: "
                          "relocation + block compaction of 256 top-5 requests per step")
     args = ap.parse_args()
+    if args.steps is None and args.impl == "reference":
+        args.steps = 100          # one oracle query per step, ~1 s each
     if args.steps is None:
-        args.steps = {"retrieve": 100, "update": 5, "streams": 20, "dense": 100,
+        args.steps = {"retrieve": 400, "update": 5, "streams": 20, "dense": 400,
                       "scoped": 100, "delete": 10, "memory": 20}[args.workload]
     if args.impl == "reference":
         return run_reference(args)
