@@ -1,0 +1,78 @@
+"""The row bounds behind the last hop's skip and the two-hop reach path,
+checked in exact (fp64) arithmetic against the oracle's propagated scores.
+
+With u >= 0 and w >= 0, s^(H) = u * sum_{h=0..H} (alpha R)^h (the hop
+recursion s^(h) = u + alpha s^(h-1) R of §3), and the mass levels
+M^(0) = 1, M^(t) = M^(t-1) R (in-weight sums of the previous level):
+
+  L0_j + Lmin sum_{t=1..H} alpha^t M^(t)_j  <=  s^(H)_{j,b}
+                                              <=  U0_j + Umax sum_t alpha^t M^(t)_j
+
+for every row j and query b, where U0 / L0 are the row's largest / smallest
+u over the queries and Umax / Lmin their extremes over the rows that have
+out-edges (the only sources).  The device evaluates the same sums in fp32
+and widens them by the rounding bound of each sum; here the inequalities are
+checked without that margin.  A dropped term, a transposed R (out- instead
+of in-weights) or a wrong extreme makes one of them fail.
+"""
+import numpy as np
+import pytest
+
+import oracle
+from test_oracle_pins import dense_R, softmax_lib, tiny_store, widen
+
+
+def _case(seed, n, deg, alpha, hops, empty_rows):
+    emb, q, row_ptr, col, aff = tiny_store(seed, n, 16, deg, n_q=9, empty_rows=empty_rows)
+    w = oracle.row_softmax(row_ptr, aff)
+    out = oracle.retrieve(emb, q, row_ptr, col, w, tau=0.5, alpha=alpha, hops=hops, k=8,
+                          want_final=True)
+    R = dense_R(n, row_ptr, col, w)
+    # the normalised first-level scores u/Z (the bounds are per-query scale free)
+    z = 0.5 * widen(q) @ widen(emb).T
+    u = np.stack([softmax_lib(z[b]) for b in range(z.shape[0])])
+    return out, R, u, row_ptr
+
+
+@pytest.mark.parametrize("hops,alpha", [(1, 0.5), (2, 0.5), (3, 0.4), (2, 1.0)])
+@pytest.mark.parametrize("empty_rows", [False, True])
+def test_row_bounds_bracket_propagated_scores(hops, alpha, empty_rows):
+    out, R, u, row_ptr = _case(11, 90, 6, alpha, hops, empty_rows)
+    n = R.shape[0]
+    s = out["final"]                                   # [B][n], s^(H) / Z
+    u0, l0 = u.max(axis=0), u.min(axis=0)
+    sources = np.diff(row_ptr) > 0
+    umax, lmin = u0.max(), l0[sources].min()
+    M = [np.ones(n)]
+    for _ in range(hops):
+        M.append(M[-1] @ R)
+    c = sum(alpha ** t * M[t] for t in range(1, hops + 1))
+    ub, lb = u0 + umax * c, l0 + lmin * c
+    tol = 1e-12
+    assert (s <= ub[None, :] * (1 + tol)).all()
+    assert (s >= lb[None, :] * (1 - tol)).all()
+
+
+@pytest.mark.parametrize("hops", [1, 2])
+def test_floor_is_below_every_kth_score(hops):
+    """The skip's floor, the k-th largest lower bound over any subset of the
+    rows, never exceeds a query's k-th largest final score; every row whose
+    upper bound is below it is outside every query's top-k."""
+    alpha, k = 0.5, 8
+    out, R, u, row_ptr = _case(12, 120, 7, alpha, hops, False)
+    n = R.shape[0]
+    s = out["final"]
+    u0, l0 = u.max(axis=0), u.min(axis=0)
+    umax, lmin = u0.max(), l0.min()
+    M = [np.ones(n)]
+    for _ in range(hops):
+        M.append(M[-1] @ R)
+    c = sum(alpha ** t * M[t] for t in range(1, hops + 1))
+    ub, lb = u0 + umax * c, l0 + lmin * c
+    heavy = np.argsort(-np.array(M[1]))[:40]           # a subset: the heaviest rows
+    floor = np.sort(lb[heavy])[::-1][k - 1]
+    kth = np.sort(s, axis=1)[:, ::-1][:, k - 1]
+    assert (floor <= kth * (1 + 1e-12)).all()
+    pruned = np.nonzero(ub < floor)[0]
+    for b in range(s.shape[0]):
+        assert not set(pruned.tolist()) & set(out["ids"][b].tolist())
