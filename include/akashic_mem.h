@@ -59,6 +59,9 @@ typedef enum {
     AKASHIC_ERANGE = 7     /* scores would leave fp32 range (see retrieve)       */
 } akashic_status_t;
 
+/* Largest hop count retrieve accepts. */
+#define AKASHIC_MAX_HOPS 16
+
 typedef struct {
     int32_t dim;             /* embedding width; multiple of 64, 64..4096          */
     int64_t capacity;        /* maximum number of chunks, 1..2^31-1                */
@@ -134,7 +137,14 @@ akashic_status_t akashic_mem_update_relations(akashic_mem_t *m, int64_t first, i
  * bound tau |q_b| max_i |e_i|, so no extra pass is needed; ERANGE (via
  * akashic_mem_sync) if 2 c_b > 80, where exp would leave fp32 range.
  * EINVAL if B < 1, k < 1, k > 64, k > size, hops < 0, hops > 16, alpha < 0
- * or not finite.  Does not synchronise. */
+ * or not finite.
+ * Does not synchronise, with one exception: with hops = 2, alpha > 0 and
+ * 65 to 256 queries in a batch of 256, the call waits on `stream` once per
+ * such batch to read which candidate rows the bounds flag (the two-hop
+ * path from reach coefficients); the first such call after the graph
+ * changed also waits while it builds their graph-only tables.
+ * Graph-only tables built by a call on one stream are waited for (an event,
+ * not a host wait) by calls on every other stream. */
 akashic_status_t akashic_mem_retrieve(akashic_mem_t *m, const uint16_t *q, int32_t B, int32_t k,
                                       float alpha, int32_t hops, int64_t *ids, float *scores,
                                       int32_t *page_ids, int32_t *n_pages, void *stream);

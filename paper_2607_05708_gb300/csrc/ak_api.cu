@@ -160,6 +160,12 @@ struct akashic_mem {
     int64_t reach_n = -1;     // rows they were computed for
     uint64_t reach_build = 0; // incremented by every rebuild
     bool reach_on = true;     // AKASHIC_REACH=0: always run the hops
+    // the mass levels and reach tables are built by whichever retrieve needs
+    // them first, on its own stream: table_mu serialises the builders and
+    // every retrieve that reads them waits on table_ev, recorded after the
+    // last build (retrieves on other streams may run concurrently)
+    std::mutex table_mu;
+    cudaEvent_t table_ev = nullptr;
     std::mutex mu;
     std::unordered_map<void *, StreamScratch *> scratch;
     // profiling
@@ -173,6 +179,7 @@ struct akashic_mem {
             cudaEventDestroy(r.b);
         }
         for (auto e : ev_pool) cudaEventDestroy(e);
+        if (table_ev) cudaEventDestroy(table_ev);
     }
 };
 
@@ -1038,12 +1045,30 @@ akashic_status_t akashic_mem_export_pages(akashic_mem_t *m, int32_t *page_of, vo
 }
 }  // extern "C"
 
+// Orders `st` after every earlier table build (any stream); called with
+// table_mu held, before the tables are read or extended.
+static akashic_status_t wait_tables(akashic_mem *m, cudaStream_t st) {
+    if (m->table_ev) CUDA_TRY(cudaStreamWaitEvent(st, m->table_ev, 0));
+    return AKASHIC_OK;
+}
+
+// Records the end of a table build on `st` (table_mu held).
+static akashic_status_t tables_built(akashic_mem *m, cudaStream_t st) {
+    if (!m->table_ev) CUDA_TRY(cudaEventCreateWithFlags(&m->table_ev, cudaEventDisableTiming));
+    CUDA_TRY(cudaEventRecord(m->table_ev, st));
+    return AKASHIC_OK;
+}
+
 // Mass levels 0..H of the row bounds (level 0 all ones), extended as needed.
+// Room for the largest hop count is taken at once, so extending the levels
+// never moves a buffer that a retrieve on another stream may be reading.
+// table_mu held.
 static akashic_status_t ensure_mass(akashic_mem *m, const HopPlan &hp, int H, cudaStream_t st) {
     const int64_t n = m->n;
+    AK_TRY(wait_tables(m, st));
     if (m->mass_n != n) m->mass_levels = -1;
     if (m->mass_levels >= H) return AKASHIC_OK;
-    const size_t lv = (size_t)(H + 1) * n * 4;
+    const size_t lv = (size_t)(AKASHIC_MAX_HOPS + 1) * n * 4;
     if (m->mass_levels < 0 || m->mass_up.cap < lv) {
         AK_TRY(m->mass_up.ensure(lv));
         AK_TRY(m->mass_dn.ensure(lv));
@@ -1060,12 +1085,14 @@ static akashic_status_t ensure_mass(akashic_mem *m, const HopPlan &hp, int H, cu
                                 m->mass_dn.as<float>(), m->mass_zero.as<float>(),
                                 m->mass_vu.as<float>(), m->mass_vl.as<float>(), st));
     m->mass_levels = H;
-    return AKASHIC_OK;
+    return tables_built(m, st);
 }
 
-// Reach coefficients of the candidate rows for H hops (after the mass levels).
+// Reach coefficients of the candidate rows for H hops (after the mass
+// levels).  table_mu held.
 static akashic_status_t ensure_reach(akashic_mem *m, const HopPlan &hp, int H, cudaStream_t st) {
     const int64_t n = m->n;
+    AK_TRY(wait_tables(m, st));
     if (m->reach_levels == H && m->reach_n == n) return AKASHIC_OK;
     AK_TRY(m->reach_rows.ensure(REACH_T * 4));
     AK_TRY(m->reach_t.ensure(16));
@@ -1097,7 +1124,7 @@ static akashic_status_t ensure_reach(akashic_mem *m, const HopPlan &hp, int H, c
     m->reach_levels = H;
     m->reach_n = n;
     ++m->reach_build;
-    return AKASHIC_OK;
+    return tables_built(m, st);
 }
 
 static akashic_status_t retrieve_impl(akashic_mem *m, const uint16_t *q, int32_t B, int32_t k,
@@ -1109,7 +1136,7 @@ static akashic_status_t retrieve_impl(akashic_mem *m, const uint16_t *q, int32_t
     if (B < 1) return fail(AKASHIC_EINVAL, "retrieve: B < 1");
     if (k < 1 || k > 64) return fail(AKASHIC_EINVAL, "retrieve: k must be in [1, 64]");
     if (k > m->n) return fail(AKASHIC_EINVAL, "retrieve: k=%d exceeds the %lld chunks", k, (long long)m->n);
-    if (hops < 0 || hops > 16) return fail(AKASHIC_EINVAL, "retrieve: hops must be in [0, 16]");
+    if (hops < 0 || hops > AKASHIC_MAX_HOPS) return fail(AKASHIC_EINVAL, "retrieve: hops must be in [0, 16]");
     if (!(alpha >= 0.f) || !isfinite(alpha)) return fail(AKASHIC_EINVAL, "retrieve: alpha must be finite and >= 0");
     DeviceGuard g(m->device);
     cudaStream_t st = (cudaStream_t)stream;
@@ -1257,7 +1284,10 @@ static akashic_status_t retrieve_impl(akashic_mem *m, const uint16_t *q, int32_t
             const float *row_ub = nullptr, *row_lb = nullptr;
             if (prune) {
                 PhaseScope ph(m, AKASHIC_PHASE_BOUND, st);
-                AK_TRY(ensure_mass(m, hp, eff_hops, st));
+                {
+                    std::lock_guard<std::mutex> lk(m->table_mu);
+                    AK_TRY(ensure_mass(m, hp, eff_hops, st));
+                }
                 CUDA_TRY(launch_final_bounds(sc->rmax_u.as<float>(), sc->rmin_u.as<float>(),
                                              m->mass_up.as<float>(), m->mass_dn.as<float>(), n,
                                              eff_hops, alpha, sc->ext.as<unsigned int>(),
@@ -1277,7 +1307,10 @@ static akashic_status_t retrieve_impl(akashic_mem *m, const uint16_t *q, int32_t
                 int32_t keep[REACH_T] = {0};
                 {
                     PhaseScope ph(m, AKASHIC_PHASE_BOUND, st);
-                    AK_TRY(ensure_reach(m, hp, eff_hops, st));
+                    {
+                        std::lock_guard<std::mutex> lk(m->table_mu);
+                        AK_TRY(ensure_reach(m, hp, eff_hops, st));
+                    }
                     AK_TRY(sc->reach_keep.ensure(REACH_T * 4));
                     AK_TRY(sc->reach_bad.ensure(16));
                     const int64_t n_lb = m->n_split < 1024 ? m->n_split : 1024;

@@ -596,3 +596,45 @@ def test_gmm4m_recipe_eight_concurrent_streams():
     got = {k: np.array(v) for k, v in got.items()}
     ref = oracle_retrieve(wl, "clustered", queries=wl.queries[rows])
     assert_retrieval_parity(wl, "clustered", got, ref)
+
+
+@pytest.mark.parametrize("hops", [3, 2])
+def test_first_retrieves_from_two_threads(hops):
+    """Two host threads, each with its own stream, make the first retrieves
+    of a fresh store at the same moment (gmm1m recipe at N = 16384, 128
+    queries each).  The graph-only tables of the last hop's row bounds (and,
+    for two hops, the reach coefficients) are built by whichever call comes
+    first; the other call's stream is ordered after that build.  Both
+    threads' results must match the oracle."""
+    import dataclasses
+    import threading
+    import torch
+    wl = dataclasses.replace(synth.workload(2, scale=1 / 64), hops=hops)
+    store = gpu_store(wl, "clustered")
+    half = wl.n_queries // 2
+    streams = [torch.cuda.Stream() for _ in range(2)]
+    qs = [torch.from_numpy(np.ascontiguousarray(wl.queries[i * half:(i + 1) * half])
+                           .view(np.int16)).cuda() for i in range(2)]
+    torch.cuda.synchronize()
+    outs, errs = [None, None], []
+    gate = threading.Barrier(2)
+
+    def run(i):
+        try:
+            with torch.cuda.stream(streams[i]):
+                gate.wait()
+                outs[i] = store.retrieve(qs[i], wl.k, wl.alpha, wl.hops, stream=streams[i])
+        except Exception as e:      # re-raised on the main thread below
+            errs.append(e)
+
+    threads = [threading.Thread(target=run, args=(i,)) for i in range(2)]
+    for t in threads:
+        t.start()
+    for t in threads:
+        t.join()
+    torch.cuda.synchronize()
+    store.sync()
+    assert not errs, errs
+    got = {key: np.concatenate([o[j].cpu().numpy() for o in outs])
+           for j, key in enumerate(("ids", "scores", "page_ids", "n_pages"))}
+    assert_retrieval_parity(wl, "clustered", got, oracle_retrieve(wl, "clustered"))
