@@ -1201,9 +1201,13 @@ static akashic_status_t retrieve_impl(akashic_mem *m, const uint16_t *q, int32_t
         ColumnRecompute rc{};
         {
             PhaseScope ph(m, AKASHIC_PHASE_SCORE, st);
+            // with the row bounds (never with the dense fused filter) the
+            // score GEMM's epilogue reduces u's row extremes into sc->ext,
+            // zeroed here
             CUDA_TRY(launch_prep_queries(qb, b, bp, m->dim, m->tau, m->max_norm.as<float>(),
                                          sc->qp.as<uint16_t>(), sc->shift.as<float>(),
-                                         m->status.as<int>(), st));
+                                         m->status.as<int>(), st,
+                                         prune ? sc->ext.as<unsigned int>() : nullptr));
             ph.launches += 1;
             if (!dense_fused)
                 CUDA_TRY(launch_score(m->emb.as<uint16_t>(), n, m->dim, sc->qp.as<uint16_t>(), bp,
@@ -1211,7 +1215,8 @@ static akashic_status_t retrieve_impl(akashic_mem *m, const uint16_t *q, int32_t
                                       sc->zpart.as<float>(), m->status.as<int>(), st,
                                       &ph.launches, &zrows, ns.dead,
                                       prune ? sc->rmax_u.as<float>() : nullptr,
-                                      prune ? sc->rmin_u.as<float>() : nullptr, b));
+                                      prune ? sc->rmin_u.as<float>() : nullptr, b,
+                                      prune ? sc->ext.as<unsigned int>() : nullptr));
         }
         if (dense_fused) {
             {
@@ -1292,7 +1297,7 @@ static akashic_status_t retrieve_impl(akashic_mem *m, const uint16_t *q, int32_t
                                              m->mass_up.as<float>(), m->mass_dn.as<float>(), n,
                                              eff_hops, alpha, sc->ext.as<unsigned int>(),
                                              sc->ub.as<float>(), sc->lb.as<float>(), st,
-                                             &ph.launches));
+                                             &ph.launches, true));
                 row_ub = sc->ub.as<float>();
                 row_lb = sc->lb.as<float>();
             }

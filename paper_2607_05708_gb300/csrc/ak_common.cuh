@@ -79,12 +79,13 @@ int64_t score_tiles(int64_t n);
 // dead_row (or NULL): rows of deleted chunks score u = 0 (no part in Z).
 // row_max / row_min (optional, together): [n] the largest and smallest u of
 // each row over the first n_real columns (the real queries), for the
-// propagation's row bounds.
+// propagation's row bounds; with them, ext (optional, [2], zeroed before)
+// gets their extremes in launch_final_bounds' encoding.
 cudaError_t launch_score(const uint16_t *emb, int64_t n, int dim, const uint16_t *qp, int bp,
                          const float *shift, float tau, float *u, float *zpart, int *status,
                          cudaStream_t st, int *launches, int *zrows,
                          const int32_t *dead_row = nullptr, float *row_max = nullptr,
-                         float *row_min = nullptr, int n_real = 0);
+                         float *row_min = nullptr, int n_real = 0, unsigned int *ext = nullptr);
 
 // The score on every stride-th row only: out[v, c] = u[v*stride, c] for
 // v < n_sample (same kernel and arithmetic as launch_score, so the values
@@ -124,9 +125,10 @@ cudaError_t launch_dots_filter(const uint16_t *emb, int64_t n, int dim, const ui
 
 // Query preparation: pad q (b rows) to bp rows of zeros and compute
 // shift[c] = tau * |q_c| * max_norm (0 for padding); flags ERANGE.
+// ext_zero (or NULL): two words set to 0 (the row extremes' initial value).
 cudaError_t launch_prep_queries(const uint16_t *q, int b, int bp, int dim, float tau,
                                 const float *max_norm, uint16_t *qp, float *shift, int *status,
-                                cudaStream_t st);
+                                cudaStream_t st, unsigned int *ext_zero = nullptr);
 
 // Running maximum of row norms of emb[0..n) into *max_norm (monotone).
 cudaError_t launch_row_norm_max(const uint16_t *emb, int64_t n, int dim, float *max_norm,
@@ -392,11 +394,14 @@ cudaError_t launch_mass_levels(const HopPlan &p, int t0, int t1, float *mup, flo
                                const float *zeros, float *split_vu, float *split_vl,
                                cudaStream_t st);
 // Per call: ub / lb [n] from u's row extremes u0 / l0 and the mass levels
-// 1..H; ext is [2] device scratch.
+// 1..H.  ext [2]: ext[0] the bits of Umax = max_j u0_j, ext[1] 0x7f800000
+// minus the bits of Lmin = min over u0_j > 0 of l0_j (both maxima, so zero
+// is the empty value); computed here unless ext_ready (the score GEMM's
+// epilogue already reduced them).
 cudaError_t launch_final_bounds(const float *u0, const float *l0, const float *mup,
                                 const float *mdn, int64_t n, int H, float alpha,
                                 unsigned int *ext, float *ub, float *lb, cudaStream_t st,
-                                int *launches);
+                                int *launches, bool ext_ready = false);
 cudaError_t launch_split_flags(const HopPlan &p, const float *row_ub, const float *floor_p,
                                int32_t *split_skip, int32_t *slot_skip, int32_t *kept_rows,
                                int64_t *kept_count, int32_t *kept_segs, KeptScratch &ks,

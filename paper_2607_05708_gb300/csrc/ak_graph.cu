@@ -958,10 +958,6 @@ cudaError_t launch_mass_levels(const HopPlan &p, int t0, int t1, float *mup, flo
 // The store-wide extremes of u's row maxima and (over rows with u > 0, i.e.
 // live rows, the only possible edge sources) row minima: ext[0] = Umax,
 // ext[1] = Lmin, as float bits (values >= 0 order like their bits).
-__global__ void k_ext_init(unsigned int *ext) {
-    ext[0] = 0u;
-    ext[1] = 0x7f800000u;
-}
 __global__ void k_row_extremes(const float *__restrict__ u0, const float *__restrict__ l0,
                                int64_t n, unsigned int *__restrict__ ext) {
     unsigned int mx = 0u, mn = 0x7f800000u;
@@ -982,7 +978,7 @@ __global__ void k_row_extremes(const float *__restrict__ u0, const float *__rest
     }
     if ((threadIdx.x & 31) == 0) {
         atomicMax(ext, mx);
-        atomicMin(ext + 1, mn);
+        atomicMax(ext + 1, 0x7f800000u - mn);
     }
 }
 
@@ -994,7 +990,7 @@ __global__ void k_final_bounds(const float *__restrict__ u0, const float *__rest
                                const float *__restrict__ mup, const float *__restrict__ mdn,
                                int64_t n, int H, float alpha, const unsigned int *__restrict__ ext,
                                float *__restrict__ ub, float *__restrict__ lb) {
-    const float umax = __uint_as_float(ext[0]), lmin = __uint_as_float(ext[1]);
+    const float umax = __uint_as_float(ext[0]), lmin = __uint_as_float(0x7f800000u - ext[1]);
     for (int64_t j = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; j < n;
          j += (int64_t)gridDim.x * blockDim.x) {
         float cu = 0.f, cl = 0.f;
@@ -1010,12 +1006,20 @@ __global__ void k_final_bounds(const float *__restrict__ u0, const float *__rest
 cudaError_t launch_final_bounds(const float *u0, const float *l0, const float *mup,
                                 const float *mdn, int64_t n, int H, float alpha,
                                 unsigned int *ext, float *ub, float *lb, cudaStream_t st,
-                                int *launches) {
+                                int *launches, bool ext_ready) {
     const int sms = device_sm_count();
-    k_ext_init<<<1, 1, 0, st>>>(ext);
-    k_row_extremes<<<sms * 4, 256, 0, st>>>(u0, l0, n, ext);
-    k_final_bounds<<<sms * 4, 256, 0, st>>>(u0, l0, mup, mdn, n, H, alpha, ext, ub, lb);
-    if (launches) *launches += 3;
+    if (!ext_ready) {
+        cudaError_t e = cudaMemsetAsync(ext, 0, 2 * sizeof(unsigned int), st);
+        if (e != cudaSuccess) return e;
+        k_row_extremes<<<sms * 4, 256, 0, st>>>(u0, l0, n, ext);
+        if (launches) *launches += 1;
+    }
+    // one row per thread up to 32 CTAs per SM: a few loads per row, so the
+    // rows in flight set the rate
+    const int64_t fb = ceil_div<int64_t>(n, 256);
+    k_final_bounds<<<(unsigned)(fb < (int64_t)sms * 32 ? (fb > 0 ? fb : 1) : (int64_t)sms * 32), 256, 0,
+                     st>>>(u0, l0, mup, mdn, n, H, alpha, ext, ub, lb);
+    if (launches) *launches += 1;
     return cudaGetLastError();
 }
 

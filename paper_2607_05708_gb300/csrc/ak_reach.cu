@@ -247,30 +247,36 @@ __global__ __launch_bounds__(256, 2) void k_reach_terms(const float *__restrict_
 }
 
 // Final score of each flagged candidate for each real query column: its u
-// plus the partials in CTA order, appended as a filter key (score bits,
-// ~chunk ID) to the column's buffer; the buffer then holds exactly them.
-__global__ void k_reach_emit(const float *__restrict__ u, int bp,
-                             const float *__restrict__ partial, int n_parts, const ReachSlots rs,
-                             const int32_t *__restrict__ rows, const int32_t *__restrict__ ext_of,
-                             unsigned int *__restrict__ cnt, unsigned long long *__restrict__ buf,
-                             int64_t cap) {
-    // one warp per candidate: lanes take every 32nd partial, then a fixed
-    // reduction tree (the same order on every run)
-    const int b = blockIdx.x;
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nwarp = blockDim.x >> 5;
-    for (int i = warp; i < rs.nk; i += nwarp) {
-        float acc = 0.f;
-        for (int p = lane; p < n_parts; p += 32) acc += partial[((int64_t)p * REACH_T + i) * bp + b];
-#pragma unroll
-        for (int off = 16; off > 0; off >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, off);
-        if (lane == 0) {
-            const int64_t j = rows[rs.slot[i]];
-            const float s = u[j * bp + b] + acc;
-            buf[(int64_t)b * cap + i] = ((unsigned long long)__float_as_uint(s) << 32) |
-                                        (unsigned long long)(~(uint32_t)ext_of[j]);
-        }
+// plus the CTAs' partials, appended as a filter key (score bits, ~chunk ID)
+// to the column's buffer; the buffer then holds exactly them.  One block per
+// candidate: thread t takes column t % bp and every (1024 / bp)-th partial
+// from t / bp on (coalesced rows of the partials), and the groups are added
+// in group order (the same order on every run).
+__global__ __launch_bounds__(1024) void k_reach_emit(const float *__restrict__ u, int bp, int B,
+                                                     const float *__restrict__ partial,
+                                                     int n_parts, const ReachSlots rs,
+                                                     const int32_t *__restrict__ rows,
+                                                     const int32_t *__restrict__ ext_of,
+                                                     unsigned int *__restrict__ cnt,
+                                                     unsigned long long *__restrict__ buf,
+                                                     int64_t cap) {
+    __shared__ float red[1024];
+    const int i = blockIdx.x;
+    const int b = threadIdx.x % bp, g = threadIdx.x / bp, ng = blockDim.x / bp;
+    float acc = 0.f;
+#pragma unroll 16
+    for (int p = g; p < n_parts; p += ng) acc += partial[((int64_t)p * REACH_T + i) * bp + b];
+    red[threadIdx.x] = acc;
+    __syncthreads();
+    if (g == 0 && b < B) {
+        float sum = red[b];
+        for (int h = 1; h < ng; ++h) sum += red[h * bp + b];
+        const int64_t j = rows[rs.slot[i]];
+        const float s = u[j * bp + b] + sum;
+        buf[(int64_t)b * cap + i] = ((unsigned long long)__float_as_uint(s) << 32) |
+                                    (unsigned long long)(~(uint32_t)ext_of[j]);
+        if (i == 0) cnt[b] = (unsigned int)rs.nk;
     }
-    if (threadIdx.x == 0) cnt[b] = (unsigned int)rs.nk;
 }
 
 cudaError_t launch_reach_check(const float *ub, const float *floor_p, const int32_t *map,
@@ -352,7 +358,7 @@ cudaError_t launch_reach_scores(const float *u, int bp, int B, int64_t n, const 
         }
     }
     if (e != cudaSuccess) return e;
-    k_reach_emit<<<B, 256, 0, st>>>(u, bp, partial, parts, rs, rows, ext_of, cnt, buf, cap);
+    k_reach_emit<<<rs.nk, 1024, 0, st>>>(u, bp, B, partial, parts, rs, rows, ext_of, cnt, buf, cap);
     if (launches) *launches += 2;
     return cudaGetLastError();
 }

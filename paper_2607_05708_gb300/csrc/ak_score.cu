@@ -12,17 +12,37 @@ namespace ak {
 // One CTA per padded query row.  shift[c] = tau * |q_c| * max_i |e_i| bounds
 // z from above, so u = exp(z - shift) <= 1 never overflows; padding rows are
 // zero with shift 0.
+// VEC: q 16-byte aligned (dim is a multiple of 64), eight values per load.
+template <bool VEC>
 __global__ void k_prep_queries(const uint16_t *__restrict__ q, int b, int dim, float tau,
                                const float *__restrict__ max_norm, uint16_t *__restrict__ qp,
-                               float *__restrict__ shift, int *status) {
+                               float *__restrict__ shift, int *status,
+                               unsigned int *__restrict__ ext_zero) {
     const int c = blockIdx.x;
+    if (ext_zero && c == 0 && threadIdx.x < 2) ext_zero[threadIdx.x] = 0u;
     __shared__ float red[32];
     float ss = 0.f;
-    for (int t = threadIdx.x; t < dim; t += blockDim.x) {
-        uint16_t h = (c < b) ? q[(int64_t)c * dim + t] : (uint16_t)0;
-        qp[(int64_t)c * dim + t] = h;
-        float v = bf16_to_f32(h);
-        ss = fmaf(v, v, ss);
+    if constexpr (VEC) {
+        for (int t = threadIdx.x * 8; t < dim; t += blockDim.x * 8) {
+            const uint4 h = (c < b) ? *reinterpret_cast<const uint4 *>(q + (int64_t)c * dim + t)
+                                    : make_uint4(0u, 0u, 0u, 0u);
+            *reinterpret_cast<uint4 *>(qp + (int64_t)c * dim + t) = h;
+            const uint32_t w[4] = {h.x, h.y, h.z, h.w};
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                const float lo = bf16_to_f32((uint16_t)(w[i] & 0xffffu));
+                const float hi = bf16_to_f32((uint16_t)(w[i] >> 16));
+                ss = fmaf(lo, lo, ss);
+                ss = fmaf(hi, hi, ss);
+            }
+        }
+    } else {
+        for (int t = threadIdx.x; t < dim; t += blockDim.x) {
+            uint16_t h = (c < b) ? q[(int64_t)c * dim + t] : (uint16_t)0;
+            qp[(int64_t)c * dim + t] = h;
+            float v = bf16_to_f32(h);
+            ss = fmaf(v, v, ss);
+        }
     }
     for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
     if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = ss;
@@ -38,8 +58,13 @@ __global__ void k_prep_queries(const uint16_t *__restrict__ q, int b, int dim, f
 
 cudaError_t launch_prep_queries(const uint16_t *q, int b, int bp, int dim, float tau,
                                 const float *max_norm, uint16_t *qp, float *shift, int *status,
-                                cudaStream_t st) {
-    k_prep_queries<<<bp, 128, 0, st>>>(q, b, dim, tau, max_norm, qp, shift, status);
+                                cudaStream_t st, unsigned int *ext_zero) {
+    if (((uintptr_t)q & 15) == 0 && dim % 8 == 0)
+        k_prep_queries<true><<<bp, 128, 0, st>>>(q, b, dim, tau, max_norm, qp, shift, status,
+                                                 ext_zero);
+    else
+        k_prep_queries<false><<<bp, 128, 0, st>>>(q, b, dim, tau, max_norm, qp, shift, status,
+                                                  ext_zero);
     return cudaGetLastError();
 }
 
@@ -145,6 +170,10 @@ struct GemmEpi {
                                         // no score (u = 0) / never a filter candidate
     float *row_max, *row_min;           // EXP (or NULL): [n_rows] largest / smallest u of
     int n_real;                         // the row over the first n_real columns
+    unsigned int *ext;                  // with row_max (or NULL), atomically maxed, zeroed
+                                        // before: [0] bits of the largest row_max, [1]
+                                        // 0x7f800000 - bits of the smallest row_min over
+                                        // the rows whose row_max > 0
 };
 
 // z[ch] += s with a run-time chunk index kept out of local memory.
@@ -350,6 +379,7 @@ __global__ __launch_bounds__(GemmCfg<BP, MODE>::THREADS, 1) void k_gemm_umma(con
         float zl[BP / 32];
 #pragma unroll
         for (int i = 0; i < BP / 32; ++i) zl[i] = 0.f;
+        float emx = 0.f, emn = INFINITY;                 // this thread's rows' extremes
         int it = 0, cc = 0;
         for (int64_t u = u_first; u < n_units; u += u_step, ++it) {
             const int64_t ct = u % n_ctiles;
@@ -508,10 +538,25 @@ __global__ __launch_bounds__(GemmCfg<BP, MODE>::THREADS, 1) void k_gemm_umma(con
             if (MODE == GEMM_EXP && ep.row_max && in_rows) {
                 ep.row_max[grow] = rmax;
                 ep.row_min[grow] = rmin;
+                emx = fmaxf(emx, rmax);
+                if (rmax > 0.f) emn = fminf(emn, rmin);
             }
             tc_fence_before();
             named_bar(1, C::EPI_T);
             if (et == 0) mbar_arrive(&tempty[acc]);
+        }
+        if (MODE == GEMM_EXP && ep.ext) {
+            // u >= 0: float bits order like the values
+            unsigned int mx = __float_as_uint(emx), mn = 0x7f800000u - __float_as_uint(emn);
+#pragma unroll
+            for (int off = 16; off > 0; off >>= 1) {
+                mx = max(mx, __shfl_xor_sync(0xffffffffu, mx, off));
+                mn = max(mn, __shfl_xor_sync(0xffffffffu, mn, off));
+            }
+            if (lane == 0) {
+                atomicMax(ep.ext, mx);
+                atomicMax(ep.ext + 1, mn);
+            }
         }
         if (!EXPF && et == 0) bulk_wait_all();
         named_bar(1, C::EPI_T);
@@ -647,12 +692,13 @@ static cudaError_t gemm_dispatch(const uint16_t *emb, int64_t n_rows, int64_t ro
 cudaError_t launch_score(const uint16_t *emb, int64_t n, int dim, const uint16_t *qp, int bp,
                          const float *shift, float tau, float *u, float *zpart, int *status,
                          cudaStream_t st, int *launches, int *zrows, const int32_t *dead_row,
-                         float *row_max, float *row_min, int n_real) {
+                         float *row_max, float *row_min, int n_real, unsigned int *ext) {
     GemmEpi ep{};
     ep.dead_row = dead_row;
     ep.row_max = row_max;
     ep.row_min = row_min;
     ep.n_real = n_real;
+    ep.ext = row_max ? ext : nullptr;
     ep.shift = shift;
     ep.tau = tau;
     ep.zpart = zpart;

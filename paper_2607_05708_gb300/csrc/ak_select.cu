@@ -552,52 +552,69 @@ cudaError_t launch_buf_merge_signed(const unsigned int *cnt, const unsigned long
 // (a) the smallest score bits that any real column's filter bound admits
 // (keys of non-negative scores order like their values; padding bounds,
 // above +inf's bits, admit nothing) and (b), without a namespace scope, the
-// k-th largest lower bound lb over the rows lb_rows[order[i]], i < n_rows:
-// every query's k-th largest final score is at least that, as each of
-// those k rows scores at least its lb for every query (any subset of the
-// rows gives a valid floor).  One CTA.
-__global__ __launch_bounds__(SEL_THREADS) void k_prune_floor(
+// k-th largest lower bound lb over the rows lb_rows[order[i]], i < n_rows
+// (at most PF_ROWS): every query's k-th largest final score is at least
+// that, as each of those k rows scores at least its lb for every query (any
+// subset of the rows gives a valid floor).  One CTA, one key per thread:
+// (b) sorts the unique keys (lb bits, position) descending with a bitonic
+// network (partners within a warp by shuffles, farther ones through a
+// ping-pong pair of shared arrays) and reads the k-th.
+constexpr int PF_ROWS = 1024;
+
+__global__ __launch_bounds__(PF_ROWS) void k_prune_floor(
     const unsigned long long *__restrict__ bound, int n_real, const float *__restrict__ lb,
     const int32_t *__restrict__ lb_rows, const int32_t *__restrict__ order, int64_t n_rows,
     int k, float *__restrict__ floor_out) {
-    __shared__ int hist[256 * (SEL_THREADS / 32)];
-    __shared__ unsigned long long win[64];
-    __shared__ unsigned long long s_prefix;
-    __shared__ int s_remaining, win_n;
+    __shared__ unsigned long long xk[2][PF_ROWS];
     __shared__ unsigned int s_min;
-    const int tid = threadIdx.x;
-    if (tid == 0) s_min = 0x7f800000u;
+    const int t = threadIdx.x;
+    if (t == 0) s_min = 0x7f800000u;
     __syncthreads();
-    unsigned int m = 0x7f800000u;
-    for (int c = tid; bound && c < n_real; c += SEL_THREADS) {
-        const unsigned int hi = (unsigned int)(bound[c] >> 32);
-        m = hi < m ? hi : m;
-    }
-    atomicMin(&s_min, m);
-    __syncthreads();
-    // without filter bounds (no first term) the floor starts at 0
-    float fl = bound ? __uint_as_float(s_min) : 0.f;
-    if (lb_rows && n_rows >= k) {
-        // keys (lb bits, position): unique, and ordered like lb (lb >= 0)
-        auto key_at = [&](int64_t i) -> unsigned long long {
-            return ((unsigned long long)__float_as_uint(lb[lb_rows[order[i]]]) << 32) |
-                   (unsigned long long)(uint32_t)i;
-        };
-        radix_select(n_rows, k, key_at, win, &win_n, hist, &s_prefix, &s_remaining);
-        if (tid == 0 && win_n >= k) {
-            unsigned long long mn = ~0ull;
-            for (int t = 0; t < win_n; ++t) mn = win[t] < mn ? win[t] : mn;
-            fl = fmaxf(fl, __uint_as_float((uint32_t)(mn >> 32)));
+    if (bound && t < n_real) atomicMin(&s_min, (unsigned int)(bound[t] >> 32));
+    const bool want_lb = lb_rows && n_rows >= k;
+    // absent keys are 0, below every real key but (lb = 0, position 0),
+    // which they equal
+    unsigned long long key =
+        want_lb && t < n_rows
+            ? ((unsigned long long)__float_as_uint(lb[lb_rows[order[t]]]) << 32) |
+                  (unsigned long long)(uint32_t)t
+            : 0ull;
+    int cur = 0;
+    if (want_lb) {
+        for (int size = 2; size <= PF_ROWS; size <<= 1) {
+            for (int stride = size >> 1; stride > 0; stride >>= 1) {
+                unsigned long long other;
+                if (stride >= 32) {
+                    xk[cur][t] = key;
+                    __syncthreads();
+                    other = xk[cur][t ^ stride];
+                    cur ^= 1;          // the next write goes to the other array
+                } else {
+                    other = __shfl_xor_sync(0xffffffffu, key, stride);
+                }
+                // segments with (t & size) == 0 run descending: there the
+                // lower position of each pair keeps the larger key
+                const bool keep_max = ((t & size) == 0) == ((t & stride) == 0);
+                key = keep_max ? (key > other ? key : other) : (key < other ? key : other);
+            }
         }
+        if (t == k - 1) xk[cur][0] = key;
     }
-    if (tid == 0) *floor_out = fl;
+    __syncthreads();
+    if (t == 0) {
+        // without filter bounds (no first term) the floor starts at 0
+        float fl = bound ? __uint_as_float(s_min) : 0.f;
+        if (want_lb) fl = fmaxf(fl, __uint_as_float((uint32_t)(xk[cur][0] >> 32)));
+        *floor_out = fl;
+    }
 }
 
 cudaError_t launch_prune_floor(const unsigned long long *bound, int n_real, const float *lb,
                                const int32_t *lb_rows, const int32_t *order, int64_t n_lb_rows,
                                int k, float *floor_out, cudaStream_t st) {
-    k_prune_floor<<<1, SEL_THREADS, 0, st>>>(bound, n_real, lb, lb_rows, order, n_lb_rows, k,
-                                             floor_out);
+    if (n_lb_rows > PF_ROWS || n_real > PF_ROWS || k < 1) return cudaErrorInvalidValue;
+    k_prune_floor<<<1, PF_ROWS, 0, st>>>(bound, n_real, lb, lb_rows, order, n_lb_rows, k,
+                                         floor_out);
     return cudaGetLastError();
 }
 
