@@ -164,25 +164,28 @@ __device__ __forceinline__ void cp_async_wait() {
 }
 
 // partial[cta][i][b] = sum over this CTA's rows k of coefK[k][i] u[k][b]
-// (BP = 256 or 128 columns of u).  Thread t takes columns 2 (t % (BP/2)) +
-// 0..1 and one of G = 512 / BP slot groups (t / (BP/2)), so that one shared
-// load of four coefficients feeds eight FMAs; REACH_ROWS rows at a time
-// are copied to shared memory (u rows and coefficient rows) with cp.async,
-// double-buffered so that the next rows load while these are summed; rows
-// in order.
+// (BP = 256 or 128 columns of u).  REACH_T_THREADS threads: thread t takes
+// columns 4 (t % (BP/4)) + 0..3 and one of G = 512 / BP slot groups
+// (t / (BP/4)), so that one shared load of four coefficients feeds sixteen
+// FMAs; REACH_ROWS rows at a time are copied to shared memory (u rows and
+// coefficient rows) with cp.async, double-buffered so that the next rows
+// load while these are summed; rows in order.
 constexpr int REACH_ROWS = 32;
+constexpr int REACH_T_THREADS = 128;
 
 template <int NK, int BP>
-__global__ __launch_bounds__(256, 2) void k_reach_terms(const float *__restrict__ u, int64_t n,
-                                                        const float *__restrict__ coefK, int nk,
-                                                        float *__restrict__ partial) {
+__global__ __launch_bounds__(REACH_T_THREADS, 2) void k_reach_terms(
+    const float *__restrict__ u, int64_t n, const float *__restrict__ coefK, int nk,
+    float *__restrict__ partial) {
     extern __shared__ __align__(16) float dyn[];
-    constexpr int G = 512 / BP;                        // slot groups
+    constexpr int TT = REACH_T_THREADS;
+    constexpr int G = TT / (BP / 4);                   // slot groups (= 512 / BP)
     constexpr int HALF = NK / G;                       // slots per thread
+    static_assert(G * (BP / 4) == TT, "every thread one column quad and one slot group");
     static_assert(HALF % 4 == 0, "four coefficients per shared load");
     float *us = dyn;                                   // [2][REACH_ROWS][BP]
     float *cs = dyn + 2 * REACH_ROWS * BP;             // [2][REACH_ROWS][NK]
-    const int cg = threadIdx.x % (BP / 2), sg = threadIdx.x / (BP / 2);
+    const int cg = threadIdx.x % (BP / 4), sg = threadIdx.x / (BP / 4);
     const int64_t per = (n + gridDim.x - 1) / gridDim.x;
     const int64_t k0 = (int64_t)blockIdx.x * per;
     const int64_t k1 = k0 + per < n ? k0 + per : n;
@@ -193,15 +196,15 @@ __global__ __launch_bounds__(256, 2) void k_reach_terms(const float *__restrict_
         float *ud = us + buf * REACH_ROWS * BP;
         float *cd = cs + buf * REACH_ROWS * NK;
         // u rows: rows x BP/4 pieces of 16 bytes; coefficient rows: rows x NK/4
-        for (int x = threadIdx.x; x < rows * (BP / 4); x += 256)
+        for (int x = threadIdx.x; x < rows * (BP / 4); x += TT)
             cp_async16(ud + x * 4, u + kb * BP + (int64_t)x * 4);
-        for (int x = threadIdx.x; x < rows * (NK / 4); x += 256)
+        for (int x = threadIdx.x; x < rows * (NK / 4); x += TT)
             cp_async16(cd + x * 4, coefK + kb * NK + (int64_t)x * 4);
         cp_async_commit();
     };
-    float acc[HALF][2];
+    float acc[HALF][4];
 #pragma unroll
-    for (int i = 0; i < HALF; ++i) acc[i][0] = acc[i][1] = 0.f;
+    for (int i = 0; i < HALF; ++i) acc[i][0] = acc[i][1] = acc[i][2] = acc[i][3] = 0.f;
     if (n_chunks > 0) stage(0, 0);
     for (int64_t c = 0; c < n_chunks; ++c) {
         const int buf = (int)(c & 1);
@@ -218,19 +221,19 @@ __global__ __launch_bounds__(256, 2) void k_reach_terms(const float *__restrict_
         const float *cd = cs + buf * REACH_ROWS * NK;
 #pragma unroll 2
         for (int r = 0; r < rows; ++r) {
-            const float2 x = *reinterpret_cast<const float2 *>(ud + r * BP + 2 * cg);
+            const float4 x = *reinterpret_cast<const float4 *>(ud + r * BP + 4 * cg);
             const float4 *c4 = reinterpret_cast<const float4 *>(cd + r * NK + sg * HALF);
 #pragma unroll
             for (int q = 0; q < HALF / 4; ++q) {
                 const float4 cq = c4[q];
-                acc[4 * q][0] = fmaf(cq.x, x.x, acc[4 * q][0]);
-                acc[4 * q][1] = fmaf(cq.x, x.y, acc[4 * q][1]);
-                acc[4 * q + 1][0] = fmaf(cq.y, x.x, acc[4 * q + 1][0]);
-                acc[4 * q + 1][1] = fmaf(cq.y, x.y, acc[4 * q + 1][1]);
-                acc[4 * q + 2][0] = fmaf(cq.z, x.x, acc[4 * q + 2][0]);
-                acc[4 * q + 2][1] = fmaf(cq.z, x.y, acc[4 * q + 2][1]);
-                acc[4 * q + 3][0] = fmaf(cq.w, x.x, acc[4 * q + 3][0]);
-                acc[4 * q + 3][1] = fmaf(cq.w, x.y, acc[4 * q + 3][1]);
+                const float cv[4] = {cq.x, cq.y, cq.z, cq.w};
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    acc[4 * q + i][0] = fmaf(cv[i], x.x, acc[4 * q + i][0]);
+                    acc[4 * q + i][1] = fmaf(cv[i], x.y, acc[4 * q + i][1]);
+                    acc[4 * q + i][2] = fmaf(cv[i], x.z, acc[4 * q + i][2]);
+                    acc[4 * q + i][3] = fmaf(cv[i], x.w, acc[4 * q + i][3]);
+                }
             }
         }
         __syncthreads();   // this buffer is restaged two chunks later
@@ -238,11 +241,10 @@ __global__ __launch_bounds__(256, 2) void k_reach_terms(const float *__restrict_
 #pragma unroll
     for (int i = 0; i < HALF; ++i) {
         const int slot = sg * HALF + i;
-        if (slot < nk) {
-            float *o = partial + ((int64_t)blockIdx.x * REACH_T + slot) * BP + 2 * cg;
-            o[0] = acc[i][0];
-            o[1] = acc[i][1];
-        }
+        if (slot < nk)
+            *reinterpret_cast<float4 *>(partial + ((int64_t)blockIdx.x * REACH_T + slot) * BP +
+                                        4 * cg) =
+                make_float4(acc[i][0], acc[i][1], acc[i][2], acc[i][3]);
     }
 }
 
@@ -315,7 +317,7 @@ static cudaError_t reach_terms_nk(const float *u, int64_t n, const float *coefK,
         if (e != cudaSuccess) return e;
         attr[dev] = true;
     }
-    k_reach_terms<NK, BP><<<parts, 256, smem, st>>>(u, n, coefK, nk, partial);
+    k_reach_terms<NK, BP><<<parts, REACH_T_THREADS, smem, st>>>(u, n, coefK, nk, partial);
     return cudaGetLastError();
 }
 
