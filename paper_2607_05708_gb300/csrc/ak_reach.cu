@@ -1,7 +1,7 @@
 // Two-hop scores of the top-k candidates without the hops.
 //
 // Unrolling the hop recursion s^(h) = u + alpha R^T s^(h-1) (the relation
-// propagation of §3, R_ki = w(k -> i)) gives, for a row j,
+// propagation of §4.1, R_ki = w(k -> i)) gives, for a row j,
 //   s^(H)_j = u_j + sum_{t=1..H} alpha^t sum_k C_t[k][j] u_k,
 //   C_1[k][j] = w(k -> j),   C_t = R C_{t-1},
 // with reach coefficients C_t that depend on the graph alone.  The row

@@ -2,7 +2,7 @@
 checked in exact (fp64) arithmetic against the oracle's propagated scores.
 
 With u >= 0 and w >= 0, s^(H) = u * sum_{h=0..H} (alpha R)^h (the hop
-recursion s^(h) = u + alpha s^(h-1) R of §3), and the mass levels
+recursion s^(h) = u + alpha s^(h-1) R of §4.1), and the mass levels
 M^(0) = 1, M^(t) = M^(t-1) R (in-weight sums of the previous level):
 
   L0_j + Lmin sum_{t=1..H} alpha^t M^(t)_j  <=  s^(H)_{j,b}
