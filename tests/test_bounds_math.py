@@ -76,3 +76,31 @@ def test_floor_is_below_every_kth_score(hops):
     pruned = np.nonzero(ub < floor)[0]
     for b in range(s.shape[0]):
         assert not set(pruned.tolist()) & set(out["ids"][b].tolist())
+
+
+@pytest.mark.parametrize("hops,alpha", [(1, 0.5), (2, 0.5), (2, 1.0), (3, 0.4)])
+def test_reach_coefficients_reproduce_propagated_scores(hops, alpha):
+    """The unrolled recursion behind the two-hop path.  With the graph-only
+    reach coefficients C_1[k][j] = w(k -> j) (column j: row j's in-weights)
+    and C_t = R C_{t-1} (row k: k's out-edges applied to the previous
+    level), s^(H)_j = u_j + sum_t alpha^t sum_k C_t[k][j] u_k for every row
+    and query: the oracle's propagated scores.  Only the candidates' columns
+    are ever needed, and each column follows the recursion on its own.  A
+    transposed C_1 (out- instead of in-weights) fails."""
+    out, R, u, _ = _case(13, 80, 5, alpha, hops, True)
+    s = out["final"]
+    C = [R.copy()]
+    for _ in range(2, hops + 1):
+        C.append(R @ C[-1])
+    got = u + sum(alpha ** (t + 1) * (u @ C[t]) for t in range(hops))
+    np.testing.assert_allclose(got, s, rtol=1e-12, atol=0)
+    # the same for a subset of columns, computed column by column
+    cols = [3, 17, 41]
+    Csub = [R[:, cols]]
+    for _ in range(2, hops + 1):
+        Csub.append(R @ Csub[-1])
+    sub = u[:, cols] + sum(alpha ** (t + 1) * (u @ Csub[t]) for t in range(hops))
+    np.testing.assert_allclose(sub, s[:, cols], rtol=1e-12, atol=0)
+    # planted: out-weights in place of in-weights
+    bad = u + sum(alpha ** (t + 1) * (u @ np.linalg.matrix_power(R.T, t + 1)) for t in range(hops))
+    assert not np.allclose(bad, s, rtol=1e-6, atol=0)
