@@ -198,8 +198,9 @@ def run_reference(args):
         return 0
     import oracle
     import synth
-    wl = synth.workload(2, placements=("clustered",))
+    wl = synth.workload(2, scale=args.scale, placements=("clustered",))
     w = oracle.row_softmax(wl.row_ptr, wl.aff)
+    workload = WORKLOAD if args.scale == 1.0 else f"{WORKLOAD} scaled by {args.scale}"
     per_step = 1
     times = []
     for i in range(args.warmup + args.steps):
@@ -213,9 +214,9 @@ def run_reference(args):
         "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
         "ms_per_step": 1e3 * tot / len(times), "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-        "config": {"workload": WORKLOAD, "sample": f"{per_step} query per step"},
+        "config": {"workload": workload, "sample": f"{per_step} query per step"},
         "cpu_baseline": {"value": value, "unit": "queries/s", "cores": 1, "kind": "oracle",
-                         "sample": f"{per_step} query of 256 per step, full store, one thread"},
+                         "sample": f"{per_step} query of 256 per step, whole store, one thread"},
         "e2e": {"value": value, "unit": "queries/s", "h2d_bytes_per_step": 0,
                 "d2h_bytes_per_step": 0},
     }
