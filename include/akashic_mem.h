@@ -225,7 +225,8 @@ akashic_status_t akashic_mem_export_pages(akashic_mem_t *m, int32_t *page_of, vo
  *                 n_pages counts the real entries only.
  *   sort_by_time  != 0: the k selected chunks are written in ascending chunk
  *                 ID (IDs are assigned in append order) instead of by score.
- * Errors as akashic_mem_retrieve.  Does not synchronise. */
+ * Errors as akashic_mem_retrieve.  With q_ns given it does not synchronise;
+ * with q_ns NULL it may wait on `stream` as akashic_mem_retrieve does. */
 akashic_status_t akashic_mem_retrieve_scoped(akashic_mem_t *m, const uint16_t *q, int32_t B,
                                              int32_t k, float alpha, int32_t hops,
                                              const int32_t *q_ns, int32_t sort_by_time,
