@@ -10,13 +10,15 @@
  *             chunks), spread the scores along the cross-chunk relation
  *             graph, keep the top-k chunks per query and resolve them to the
  *             pages that hold them (query-aware retrieval, §4.1 and
- *             Algorithm 1, lines 14-18; the locality gap |P(R_t)|, §3.2);
+ *             Algorithm 1's retrieval steps; the locality gap |P(R_t)|,
+ *             §3.2);
  *   append    add immutable chunk records, each with a logical ID and a
  *             physical page (§4.2: logical identity is separate from
  *             physical placement);
  *   update    for new chunks, select the top-M related prior chunks by
  *             cosine similarity and link them both ways in the relation
- *             graph (cross-chunk selection, §4.1 and Algorithm 1, line 7).
+ *             graph (cross-chunk selection, §4.1 and Algorithm 1's
+ *             LLMSelect of related prior chunks).
  *
  * Conventions
  *   - Every entry point returns an akashic_status_t and never throws.
@@ -107,7 +109,8 @@ akashic_status_t akashic_mem_append_chunks(akashic_mem_t *m, const uint16_t *emb
                                            int64_t *first_id_out, void *stream);
 
 /* Relation update for the chunks [first, first+n) (cross-chunk selection,
- * Algorithm 1 line 7, in its dense form): for each such chunk c, its top-M
+ * Algorithm 1's LLMSelect of related prior chunks, in its dense form): for
+ * each such chunk c, its top-M
  * prior chunks j < first by cosine <e_c, e_j> of the stored bf16 values
  * (no further normalisation), ordered by cosine descending then lower ID,
  * become its out-edges with logit relation_scale * cos; with reciprocal != 0
@@ -120,7 +123,7 @@ akashic_status_t akashic_mem_append_chunks(akashic_mem_t *m, const uint16_t *emb
 akashic_status_t akashic_mem_update_relations(akashic_mem_t *m, int64_t first, int64_t n,
                                               int32_t M, int32_t reciprocal, void *stream);
 
-/* Query-aware retrieval (§4.1, Algorithm 1 lines 14-18, Dense-only form):
+/* Query-aware retrieval (§4.1, Algorithm 1's retrieval steps, Dense-only form):
  *   z[b,i] = tau <q_b, e_i>;  s0[b,:] = softmax over chunks of z[b,:];
  *   s^(0) = u = exp(z - c_b);  s^(h)_j = u_j + alpha sum_{i->j} w_ij s^(h-1)_i
  *   for h = 1..hops (mass flows along out-edges i -> j);
@@ -179,19 +182,22 @@ akashic_status_t akashic_mem_delete(akashic_mem_t *m, const int64_t *ids, int64_
  * association" when co >= tau_assoc * (sel(a) + sel(b) - co) (fp64, tau
  * rounded to fp32; the paper's tau_assoc is 0.7, §5.5).
  *
- * Relocation (Algorithm 2, lines 3-8).  S: device int64[n_req][s_len]
- * retrieved chunk IDs per request (-1, IDs outside the store, deleted
- * chunks and repeats are skipped), 1 <= s_len <= 64.  The batch's statistics
- * are added first; then, request by request, the chunks of the request that
- * are highly associated with another of its chunks (LLMCoLocate), if two or
- * more and not all on one page, are written out of place in chunk-ID order
- * (SortByTime) into fresh pages of chunks_per_page slots; each old copy
- * becomes an invalid slot of its page.  Synchronises `stream`.
+ * Relocation (Algorithm 2: LLMCoLocate, then PackIntoNewBlocks of the
+ * time-sorted group and MarkInvalid of the old copies).
+ *   S  device int64[n_req][s_len], the retrieved chunk IDs per request
+ *      (-1, IDs outside the store, deleted chunks and repeats are
+ *      skipped), 1 <= s_len <= 64.
+ * The batch's statistics are added first; then, request by request, the
+ * chunks of the request that are highly associated with another of its
+ * chunks (LLMCoLocate), if two or more and not all on one page, are written
+ * out of place in chunk-ID order (SortByTime) into fresh pages of
+ * chunks_per_page slots; each old copy becomes an invalid slot of its page.  Synchronises `stream`.
  * EINVAL on bad sizes or tau outside [0, 1]. */
 akashic_status_t akashic_mem_relocate(akashic_mem_t *m, const int64_t *S, int32_t n_req,
                                       int32_t s_len, float tau_assoc, void *stream);
 
-/* Block compaction (Algorithm 2, lines 11-24; phi(B) of §4.2): every page
+/* Block compaction (Algorithm 2: LiveChunks, PartitionByUserSession,
+ * LLMGroup, PackIntoNewBlocks, Release; phi(B) of §4.2): every page
  * whose invalid ratio phi = (slots - live) / slots is >= theta (0.75 in the
  * paper) is compacted: its live chunks are partitioned by namespace
  * (akashic_mem_set_namespace), grouped within a partition by the connected
@@ -215,7 +221,7 @@ akashic_status_t akashic_mem_export_pages(akashic_mem_t *m, int32_t *page_of, vo
 
 /* Retrieval scoped to the caller's namespace, with optional chronological
  * order (§4.1: candidates are the chunks of the current user_id/session_id;
- * Algorithm 1 lines SortByTime: the selected chunks are returned in time
+ * Algorithm 1's SortByTime: the selected chunks are returned in time
  * order).  As akashic_mem_retrieve, except:
  *   q_ns          device int32[B] or NULL: query b selects only among chunks
  *                 whose tag equals q_ns[b] (scores, Z and propagation are

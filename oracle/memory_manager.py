@@ -96,7 +96,7 @@ class MemoryManager:
         self.next_page += -(-len(chunks) // self.P)
         self.writes += len(chunks)
 
-    # ------------------------------------------------------------------ Algorithm 2, lines 3-8
+    # ------------------------------------------------------------------ Algorithm 2, relocation
     def relocate(self, requests, tau):
         """requests: int array [R, s] of retrieved chunk IDs (-1 padding)."""
         sets = []
@@ -115,7 +115,7 @@ class MemoryManager:
                 continue
             self._new_pages(sorted(g))
 
-    # ------------------------------------------------------------------ Algorithm 2, lines 11-24
+    # ------------------------------------------------------------------ Algorithm 2, block compaction
     def compact(self, theta, tau):
         t = float(np.float32(theta))
         cand = sorted(p for p, tot in self.total.items()

@@ -1,8 +1,8 @@
 // Relation update (a6, a7): for new chunks, the top-M related prior chunks
 // by cosine of the stored embeddings, then the reciprocal insertion of those
 // edges into the relation graph's CSR (arXiv 2607.05708, §4.1: cross-chunk
-// inference selects the related prior chunks of each new chunk; Algorithm 1,
-// line 7, in its Dense-only form of §5.5).
+// inference selects the related prior chunks of each new chunk; Algorithm 1's
+// LLMSelect of related prior chunks, in its Dense-only form of §5.5).
 #include "ak_update.cuh"
 
 namespace ak {
