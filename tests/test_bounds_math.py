@@ -34,7 +34,7 @@ def _case(seed, n, deg, alpha, hops, empty_rows):
     return out, R, u, row_ptr
 
 
-@pytest.mark.parametrize("hops,alpha", [(1, 0.5), (2, 0.5), (3, 0.4), (2, 1.0)])
+@pytest.mark.parametrize("hops,alpha", [(1, 0.5), (2, 0.5), (3, 0.4), (2, 1.0), (16, 0.6)])
 @pytest.mark.parametrize("empty_rows", [False, True])
 def test_row_bounds_bracket_propagated_scores(hops, alpha, empty_rows):
     out, R, u, row_ptr = _case(11, 90, 6, alpha, hops, empty_rows)

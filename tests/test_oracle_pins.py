@@ -164,7 +164,7 @@ def test_alpha_zero_is_argsort():
 
 
 # --------------------------------------------------------------------------- propagation
-@pytest.mark.parametrize("hops,alpha", [(1, 0.5), (2, 0.5), (3, 0.4), (2, 1.0)])
+@pytest.mark.parametrize("hops,alpha", [(1, 0.5), (2, 0.5), (3, 0.4), (2, 1.0), (16, 0.6)])
 def test_propagation_matrix_power_closed_form(hops, alpha):
     """s^(H) = u * sum_{h=0..H} (alpha R)^h, evaluated with numpy
     matrix_power on the dense R: a different formula (power series, dense,
@@ -187,9 +187,10 @@ def test_propagation_matrix_power_closed_form(hops, alpha):
         assert np.allclose(out["scores"][b], ref[top], rtol=1e-12)
 
 
-@pytest.mark.parametrize("hops,alpha", [(1, 0.5), (2, 0.5), (2, 0.4), (4, 0.3)])
+@pytest.mark.parametrize("hops,alpha", [(1, 0.5), (2, 0.5), (2, 0.4), (4, 0.3), (16, 0.9)])
 def test_mass_conservation(hops, alpha):
-    """With no empty rows each hop preserves mass: sum_j s_j = sum_h alpha^h."""
+    """With no empty rows each hop preserves mass: sum_j s_j = sum_h alpha^h
+    (up to the largest hop count the library accepts, 16)."""
     emb, q, row_ptr, col, aff = tiny_store(4, 200, 16, 9)
     w = oracle.row_softmax(row_ptr, aff)
     out = oracle.retrieve(emb, q, row_ptr, col, w, tau=0.3, alpha=alpha, hops=hops, k=5,
