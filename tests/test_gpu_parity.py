@@ -665,3 +665,15 @@ def test_first_retrieves_from_two_threads(hops):
     got = {key: np.concatenate([o[j].cpu().numpy() for o in outs])
            for j, key in enumerate(("ids", "scores", "page_ids", "n_pages"))}
     assert_retrieval_parity(wl, "clustered", got, oracle_retrieve(wl, "clustered"))
+
+
+@pytest.mark.parametrize("B", [64, 256])
+def test_sixteen_hops(B):
+    """The largest hop count retrieve accepts: H = 16 on the gmm1m recipe at
+    N = 16384 (alpha = 0.5, k = 32), the last hop's row bounds over 16 mass
+    levels; oracle parity."""
+    import dataclasses
+    wl = synth.workload(2, scale=1 / 64)
+    wl = dataclasses.replace(wl, hops=16, queries=wl.queries[:B])
+    _, got = gpu_retrieve(wl, "clustered")
+    assert_retrieval_parity(wl, "clustered", got, oracle_retrieve(wl, "clustered"))
