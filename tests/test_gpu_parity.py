@@ -677,3 +677,22 @@ def test_sixteen_hops(B):
     wl = dataclasses.replace(wl, hops=16, queries=wl.queries[:B])
     _, got = gpu_retrieve(wl, "clustered")
     assert_retrieval_parity(wl, "clustered", got, oracle_retrieve(wl, "clustered"))
+
+
+@pytest.mark.parametrize("dim", [64, 4096])
+def test_embedding_width_limits(dim):
+    """The narrowest and widest embeddings a store accepts, d = 64 and 4096
+    (the score GEMM's K loop runs over 1 and 64 blocks of 64): the tiny
+    store's graph and pages with fresh unit-length bf16 rows of that width,
+    37 queries, two hops, k = 16; oracle parity."""
+    import dataclasses
+    base = synth.workload(0)
+    rng = np.random.default_rng(dim)
+
+    def unit(m):
+        x = rng.standard_normal((m, dim)).astype(np.float32)
+        return synth.to_bf16(x / np.linalg.norm(x, axis=1, keepdims=True))
+
+    wl = dataclasses.replace(base, dim=dim, emb=unit(base.n), queries=unit(37), hops=2, k=16)
+    _, got = gpu_retrieve(wl, "id")
+    assert_retrieval_parity(wl, "id", got, oracle_retrieve(wl, "id"))
