@@ -74,8 +74,10 @@ def test_affinity_is_jaccard_of_request_sets():
                 continue
             inter = len(sets[a] & sets[b])
             union = len(sets[a] | sets[b])
-            for tau in (0.3, 0.5, 0.7):
-                want = inter > 0 and inter / union >= np.float32(tau) - 1e-12
+            for tau in (0.2, 0.3, 0.5, 0.7):
+                # the decision in fp64 with tau rounded to fp32 (exact here:
+                # small integers times a 24-bit fraction)
+                want = inter > 0 and inter >= float(np.float32(tau)) * union
                 assert mm.affinity_at_least(a, b, tau) == want
 
 
@@ -108,3 +110,52 @@ def test_directory_invariants(seed):
         st = mm.stats()
         assert st["slots_live"] == int(live.sum())
         assert st["slots_total"] >= st["slots_live"]
+
+
+@pytest.mark.parametrize("seed", [5, 6, 7])
+def test_compaction_packs_connected_components(seed):
+    """Block compaction against an independent construction: the live
+    chunks of the pages whose invalid ratio reaches theta, the graph of
+    their associated pairs (same namespace, Jaccard index of the two chunks'
+    request sets >= tau, computed here from the trace), its connected
+    components (networkx), and the packing by (namespace, earliest chunk of
+    the component, chunk ID), P chunks per fresh page from the next free
+    page on."""
+    nx = pytest.importorskip("networkx")
+    # relocation at 0.5 leaves tombstones; compaction groups at 0.2, so that
+    # associated pairs remain among the chunks it moves
+    tau_r, tau, theta, P = 0.5, 0.2, 0.75, 8
+    page_of, reqs, comp = _random_trace(seed)
+    ns = comp % 3
+    mm = MemoryManager(page_of, P, ns_of=ns)
+    mm.relocate(reqs, tau_r)
+    rng = np.random.default_rng(seed)
+    mm.delete(rng.choice(mm.n, 60, replace=False))
+    cand = sorted(p for p, tot in mm.total.items()
+                  if tot > 0 and (tot - mm.live[p]) >= np.float32(theta) * tot)
+    moving = [c for c in range(mm.n) if not mm.dead[c] and int(mm.page[c]) in set(cand)]
+    sets = {}
+    for r, row in enumerate(reqs):
+        for c in set(int(x) for x in row if x >= 0):
+            sets.setdefault(c, set()).add(r)
+    g = nx.Graph()
+    g.add_nodes_from(moving)
+    for i, a in enumerate(moving):
+        for b in moving[i + 1:]:
+            if ns[a] != ns[b] or a not in sets or b not in sets:
+                continue
+            inter = len(sets[a] & sets[b])
+            if inter and inter >= float(np.float32(tau)) * len(sets[a] | sets[b]):
+                g.add_edge(a, b)
+    comps = sorted((sorted(cc) for cc in nx.connected_components(g)),
+                   key=lambda cc: (int(ns[cc[0]]), cc[0]))
+    order = [c for cc in comps for c in cc]
+    assert cand and max(len(cc) for cc in comps) >= 2          # not vacuous
+    first = mm.next_page
+    released = mm.compact(theta, tau)
+    assert released == cand
+    for i, c in enumerate(order):
+        assert mm.page[c] == first + i // P, (c, i)
+    assert mm.next_page == first + -(-len(order) // P)
+    for p in cand:
+        assert mm.total[p] == 0 and mm.live[p] == 0
