@@ -38,8 +38,10 @@ compaction moves); space amplification = slots_total / slots_live, write
 amplification = chunk_writes / appended chunks.
 
 Pins: tests/test_memory_manager_oracle.py (a hand-worked trace in
-tests/golden, invariants of the directory and of the counters, and the
-affinity rule against a brute-force Jaccard over the request sets).
+tests/golden, invariants of the directory and of the counters, the
+affinity rule against a brute-force Jaccard over the request sets, and the
+compaction's packing against the connected components of the associated
+pairs built independently with networkx).
 """
 from __future__ import annotations
 
