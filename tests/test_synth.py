@@ -92,3 +92,28 @@ def test_update_workload():
     wl = synth.workload(3, scale=1 / 256)
     assert wl.new_emb.shape == (16, wl.dim) and wl.top_m == 32
     assert wl.new_component.max() <= wl.component.max()
+
+
+def test_request_trace():
+    """The Memory Manager's query trace: deterministic for a seed, unit-length
+    bf16 rows, each within the noise of one of the anchor chunks, and the
+    anchors' popularity falling with rank like Zipf(1.1) (the most popular
+    anchor draws about 1 / H_{512, 1.1} of the queries here)."""
+    wl = synth.workload(0)
+    a = synth.request_trace(wl, 4000, n_topics=512)
+    b = synth.request_trace(wl, 4000, n_topics=512)
+    assert a.dtype == np.uint16 and a.shape == (4000, wl.dim)
+    assert np.array_equal(a, b)
+    assert not np.array_equal(a, synth.request_trace(wl, 4000, n_topics=512, seed=1))
+    x = synth.bf16_to_f32(a).astype(np.float64)
+    assert np.allclose(np.linalg.norm(x, axis=1), 1.0, atol=1e-2)
+    e = synth.bf16_to_f32(wl.emb).astype(np.float64)
+    e /= np.linalg.norm(e, axis=1, keepdims=True)
+    nearest = (x @ e.T).argmax(axis=1)
+    cos = (x @ e.T).max(axis=1)
+    assert cos.min() > 0.99                     # noise 0.05 / sqrt(d) per dimension
+    counts = np.bincount(nearest, minlength=wl.n)
+    top = np.sort(counts)[::-1]
+    h = (1.0 / np.arange(1, 513) ** 1.1).sum()
+    assert abs(top[0] / 4000 - 1 / h) < 0.03
+    assert (counts > 0).sum() <= 512
