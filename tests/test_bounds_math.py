@@ -15,6 +15,8 @@ and widens them by the rounding bound of each sum; here the inequalities are
 checked without that margin.  A dropped term, a transposed R (out- instead
 of in-weights) or a wrong extreme makes one of them fail.
 """
+import math
+
 import numpy as np
 import pytest
 
@@ -104,3 +106,62 @@ def test_reach_coefficients_reproduce_propagated_scores(hops, alpha):
     # planted: out-weights in place of in-weights
     bad = u + sum(alpha ** (t + 1) * (u @ np.linalg.matrix_power(R.T, t + 1)) for t in range(hops))
     assert not np.allclose(bad, s, rtol=1e-6, atol=0)
+
+
+# --------------------------------------------------------------------------- fp32 margins
+F32 = np.float32
+
+
+def _x(n):
+    """The per-level rounding allowance of a row with n in-edges, as the
+    device computes it in fp32: 3.25 (n + 8) 2^-24."""
+    return F32(3.25) * F32(n + 8) * F32(5.9604645e-8)
+
+
+def _seq_sum_f32(w, a):
+    """A worse evaluation than the device's: every product rounded to fp32,
+    then one sequential fp32 chain over all n terms (the device fuses each
+    product into its sum and splits the chain over lanes and segments)."""
+    return np.cumsum((w * a).astype(F32), dtype=F32)[-1]
+
+
+@pytest.mark.parametrize("n", [1, 7, 256, 4096, 100_000, 818_357])
+@pytest.mark.parametrize("kind", ["uniform", "lognormal", "constant"])
+def test_level_margins_cover_fp32_sums(n, kind):
+    """One mass level in fp32: the device's widened sums, Σ·(1 + x + x²)·(1 + 4e-6)
+    above and Σ·(1 − x)·(1 − 4e-6) below, bracket the exact sum of the same fp32
+    inputs, for in-degrees up to the largest hub of the 1M-chunk graph."""
+    rng = np.random.default_rng(n)
+    if kind == "uniform":
+        w, a = rng.random(n).astype(F32), (1 + 10 * rng.random(n)).astype(F32)
+    elif kind == "lognormal":
+        w, a = rng.random(n).astype(F32), rng.lognormal(0, 2, n).astype(F32)
+    else:
+        w, a = np.full(n, 0.1, F32), np.full(n, 3.3, F32)
+    exact = math.fsum((w.astype(np.float64) * a.astype(np.float64)).tolist())
+    s = _seq_sum_f32(w, a)
+    x = _x(n)
+    up = F32(F32(s * F32(F32(1) + x + x * x)) * F32(1 + 4e-6))
+    dn = F32(F32(s * F32(F32(1) - x)) * F32(1 - 4e-6))
+    assert float(up) >= exact
+    assert float(dn) <= exact
+
+
+@pytest.mark.parametrize("hops", [1, 2, 16])
+def test_final_bound_margin_covers_fp32_horner(hops):
+    """The per-call bounds in fp32, ub = (U0 + Umax·Σ_t α^t M_t)(1 + 1e-5) by
+    Horner's rule and lb likewise with (1 − 1e-5), bracket the exact value of
+    the same fp32 inputs, up to sixteen hops."""
+    rng = np.random.default_rng(hops)
+    for _ in range(2000):
+        alpha = F32(rng.random())
+        M = rng.lognormal(2, 2, hops).astype(F32)
+        u0, umax = F32(rng.random() * 1e-3), F32(rng.random())
+        cu = F32(0)
+        for t in range(hops, 0, -1):
+            cu = F32(alpha * F32(cu + M[t - 1]))
+        ub = F32(F32(umax * cu + u0) * F32(1 + 1e-5))      # fmaf: one rounding, a
+        lb = F32(F32(umax * cu + u0) * F32(1 - 1e-5))      # second here is worse
+        exact = float(u0) + float(umax) * sum(float(alpha) ** t * float(M[t - 1])
+                                              for t in range(1, hops + 1))
+        assert float(ub) >= exact and float(lb) <= exact
