@@ -165,3 +165,28 @@ def test_final_bound_margin_covers_fp32_horner(hops):
         exact = float(u0) + float(umax) * sum(float(alpha) ** t * float(M[t - 1])
                                               for t in range(1, hops + 1))
         assert float(ub) >= exact and float(lb) <= exact
+
+
+def test_fp32_hops_never_lower_a_score():
+    """The fused filter's bound: with w >= 0 and alpha >= 0, s^(h) >= s^(h-1)
+    elementwise also in fp32 when every hop sums a row's in-edges in the same
+    order (each fma and add is monotone in its arguments), so the k-th
+    largest sampled value of s^(H-1) is a safe threshold for s^(H).  Emulated
+    with fp32 numpy, one sequential fma-free chain per row (product rounded,
+    then added), for 12 hops."""
+    out, R, u, row_ptr = _case(21, 150, 9, 0.9, 1, True)
+    n = R.shape[0]
+    u32 = u.astype(F32)
+    alpha = F32(0.9)
+    Rt = R.T.astype(F32)                                 # Rt[j][i] = w(i -> j)
+    prev = u32.copy()
+    for _ in range(12):
+        nxt = np.empty_like(prev)
+        for j in range(n):
+            src = np.nonzero(Rt[j])[0]
+            acc = np.zeros(prev.shape[0], F32)
+            for i in src:                                 # the same order every hop
+                acc = (acc + (Rt[j, i] * prev[:, i]).astype(F32)).astype(F32)
+            nxt[:, j] = (u32[:, j] + (alpha * acc).astype(F32)).astype(F32)
+        assert (nxt >= prev).all()
+        prev = nxt
