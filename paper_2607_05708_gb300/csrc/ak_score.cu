@@ -212,14 +212,7 @@ struct GemmCfg {
     static_assert(STAGES >= 2, "not enough shared memory for two stages");
 };
 
-// PAIR: clusters of two CTAs on the row tiles 2p and 2p+1 of the same
-// column tile.  Each loads its own row tile and one half of the column tile,
-// multicast to both, so the column operand crosses L2 once per pair; each
-// CTA's MMAs free a stage in both CTAs (the stage's empty barrier counts two
-// arrivals).  A pair whose second row tile lies past the end still runs it
-// (zero-filled rows that the epilogue ignores), so both CTAs walk the same
-// tiles and stages.
-template <int BP, int MODE, bool PAIR>
+template <int BP, int MODE>
 __global__ __launch_bounds__(GemmCfg<BP, MODE>::THREADS, 1) void k_gemm_umma(const __grid_constant__ CUtensorMap tmA,
                                                       const __grid_constant__ CUtensorMap tmB,
                                                       const __grid_constant__ CUtensorMap tmC,
@@ -249,18 +242,17 @@ __global__ __launch_bounds__(GemmCfg<BP, MODE>::THREADS, 1) void k_gemm_umma(con
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int64_t m_tiles = (n_rows + C::BM - 1) / C::BM;
-    // work units: (row tile, column tile), or (row tile pair, column tile)
-    const uint32_t crank = PAIR ? cluster_ctarank() : 0u;
-    const int64_t n_units = (PAIR ? (m_tiles + 1) / 2 : m_tiles) * n_ctiles;
-    const int64_t u_first = PAIR ? blockIdx.x / 2 : blockIdx.x;
-    const int64_t u_step = PAIR ? gridDim.x / 2 : gridDim.x;
+    // work units: (row tile, column tile)
+    const int64_t n_units = m_tiles * n_ctiles;
+    const int64_t u_first = blockIdx.x;
+    const int64_t u_step = gridDim.x;
     const int kb_n = dim / C::BK;
     int *status = ep.status;
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < C::STAGES; ++s) {
             mbar_init(&full[s], 1);
-            mbar_init(&empty[s], PAIR ? 2 : 1);
+            mbar_init(&empty[s], 1);
         }
         for (int a = 0; a < 2; ++a) {
             mbar_init(&tfull[a], 1);
@@ -278,9 +270,6 @@ __global__ __launch_bounds__(GemmCfg<BP, MODE>::THREADS, 1) void k_gemm_umma(con
     }
     tc_fence_before();
     __syncthreads();
-    // the peer's copies and commits reach this CTA's barriers only after
-    // both have initialised theirs
-    if (PAIR) cluster_sync();
     tc_fence_after();
     const uint32_t tmem_base = *tmem_slot;
 
@@ -293,7 +282,7 @@ __global__ __launch_bounds__(GemmCfg<BP, MODE>::THREADS, 1) void k_gemm_umma(con
             bool ok = true;
             for (int64_t u = u_first; u < n_units && ok; u += u_step) {
                 const int64_t ct = u % n_ctiles;
-                const int64_t mt = PAIR ? (u / n_ctiles) * 2 + crank : u / n_ctiles;
+                const int64_t mt = u / n_ctiles;
                 for (int kb = 0; kb < kb_n; ++kb) {
                     if (!mbar_wait(&empty[stage], phase ^ 1u, status)) {
                         ok = false;
@@ -302,13 +291,8 @@ __global__ __launch_bounds__(GemmCfg<BP, MODE>::THREADS, 1) void k_gemm_umma(con
                     mbar_expect_tx(&full[stage], C::STAGE_BYTES);
                     tma_load_2d(sA + stage * C::A_BYTES, &tmA, &full[stage], kb * C::BK,
                                 (int)(mt * C::BM));
-                    if (PAIR)
-                        tma_load_2d_mc(sB + stage * C::B_BYTES + crank * (C::B_BYTES / 2), &tmB,
-                                       &full[stage], kb * C::BK, (int)(ct * BP + crank * (BP / 2)),
-                                       (uint16_t)3);
-                    else
-                        tma_load_2d(sB + stage * C::B_BYTES, &tmB, &full[stage], kb * C::BK,
-                                    (int)(ct * BP));
+                    tma_load_2d(sB + stage * C::B_BYTES, &tmB, &full[stage], kb * C::BK,
+                                (int)(ct * BP));
                     last_par[stage] = (int)phase;
                     if (++stage == (uint32_t)C::STAGES) {
                         stage = 0;
@@ -320,16 +304,6 @@ __global__ __launch_bounds__(GemmCfg<BP, MODE>::THREADS, 1) void k_gemm_umma(con
                 // let every copy this thread issued land before the CTA exits
                 for (int s = 0; s < C::STAGES; ++s)
                     if (last_par[s] >= 0) mbar_wait(&full[s], (uint32_t)last_par[s], status);
-            } else if (PAIR) {
-                // every stage released by both CTAs' MMAs: the peer's last
-                // commits have reached this CTA's barriers before it leaves
-                for (int s = 0; s < C::STAGES; ++s) {
-                    if (!mbar_wait(&empty[stage], phase ^ 1u, status)) break;
-                    if (++stage == (uint32_t)C::STAGES) {
-                        stage = 0;
-                        phase ^= 1u;
-                    }
-                }
             }
         }
     } else if (warp == 1) {
@@ -357,8 +331,7 @@ __global__ __launch_bounds__(GemmCfg<BP, MODE>::THREADS, 1) void k_gemm_umma(con
                     for (int k = 0; k < C::BK / 16; ++k)
                         umma_bf16(d, ad + (uint64_t)(2 * k), bd + (uint64_t)(2 * k), idesc,
                                   (kb | k) != 0 ? 1u : 0u);
-                    if (PAIR) umma_commit_mc(&empty[stage], (uint16_t)3);
-                    else umma_commit(&empty[stage]);
+                    umma_commit(&empty[stage]);
                     if (++stage == (uint32_t)C::STAGES) {
                         stage = 0;
                         phase ^= 1u;
@@ -383,7 +356,7 @@ __global__ __launch_bounds__(GemmCfg<BP, MODE>::THREADS, 1) void k_gemm_umma(con
         int it = 0, cc = 0;
         for (int64_t u = u_first; u < n_units; u += u_step, ++it) {
             const int64_t ct = u % n_ctiles;
-            const int64_t mt = PAIR ? (u / n_ctiles) * 2 + crank : u / n_ctiles;
+            const int64_t mt = u / n_ctiles;
             const int acc = it & 1;
             const uint32_t aph = (uint32_t)(it >> 1) & 1u;
             // one thread polls, the barrier makes the outcome uniform
@@ -573,8 +546,6 @@ __global__ __launch_bounds__(GemmCfg<BP, MODE>::THREADS, 1) void k_gemm_umma(con
     }
     tc_fence_before();
     __syncthreads();
-    // no CTA of a pair leaves while the other may still signal its barriers
-    if (PAIR) cluster_sync();
     tc_fence_after();
     if (warp == 1) tmem_dealloc(tmem_base, C::TMEM_COLS);
 }
@@ -582,64 +553,27 @@ __global__ __launch_bounds__(GemmCfg<BP, MODE>::THREADS, 1) void k_gemm_umma(con
 int64_t score_tiles(int64_t n) { return ceil_div<int64_t>(n, 128); }
 
 // A: E rows (row_stride_rows apart: 1 = every row, s = every s-th row),
-// The relation filter GEMM runs as CTA pairs sharing the column tile
-// (AKASHIC_GEMM_PAIR=0 selects single CTAs).
-static bool gemm_pair_enabled() {
-    static int on = -1;
-    if (on < 0) {
-        const char *e = getenv("AKASHIC_GEMM_PAIR");
-        on = (e && e[0] == '0') ? 0 : 1;
-    }
-    return on == 1;
-}
-
 // B: n_ctiles * BP query rows, C: output [n_rows][n_ctiles * BP] (EXP/RAW).
 template <int BP, int MODE>
 static cudaError_t gemm_bp(const uint16_t *emb, int64_t n_rows, int64_t row_stride_rows, int dim,
                            const uint16_t *qp, int n_ctiles, float *out, const GemmEpi &ep,
                            cudaStream_t st, int *zrows) {
     using C = GemmCfg<BP, MODE>;
-    constexpr bool CAN_PAIR = MODE == GEMM_FILTER && BP == 256;
-    const bool pair = CAN_PAIR && gemm_pair_enabled();
     static bool attr[64] = {false};
-    static int pair_clusters[64] = {0};
     int dev = 0;
     cudaGetDevice(&dev);
     if (dev >= 0 && dev < 64 && !attr[dev]) {
-        cudaError_t e = cudaFuncSetAttribute(k_gemm_umma<BP, MODE, false>,
+        cudaError_t e = cudaFuncSetAttribute(k_gemm_umma<BP, MODE>,
                                              cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
-        if (e == cudaSuccess && CAN_PAIR)
-            e = cudaFuncSetAttribute(k_gemm_umma<BP, MODE, CAN_PAIR>,
-                                     cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
         if (e != cudaSuccess) return e;
-        if (CAN_PAIR) {
-            // clusters of two that fit at once (one CTA per SM)
-            cudaLaunchConfig_t cfg = {};
-            cudaLaunchAttribute at[1];
-            at[0].id = cudaLaunchAttributeClusterDimension;
-            at[0].val.clusterDim.x = 2;
-            at[0].val.clusterDim.y = 1;
-            at[0].val.clusterDim.z = 1;
-            cfg.gridDim = dim3((unsigned)(device_sm_count() & ~1));
-            cfg.blockDim = dim3(C::THREADS);
-            cfg.dynamicSmemBytes = C::SMEM;
-            cfg.attrs = at;
-            cfg.numAttrs = 1;
-            int ncl = 0;
-            e = cudaOccupancyMaxActiveClusters(&ncl, k_gemm_umma<BP, MODE, CAN_PAIR>, &cfg);
-            if (e != cudaSuccess) return e;
-            pair_clusters[dev] = ncl;
-        }
         attr[dev] = true;
     }
-    const bool use_pair = pair && dev >= 0 && dev < 64 && pair_clusters[dev] > 0;
     CUtensorMap ta, tb, tc;
     cudaError_t e = make_tmap_2d(&ta, emb, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, (uint64_t)dim,
                                  (uint64_t)n_rows, (uint64_t)dim * 2 * row_stride_rows, 64, 128);
     if (e == cudaSuccess)
         e = make_tmap_2d(&tb, qp, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, (uint64_t)dim,
-                         (uint64_t)n_ctiles * BP, (uint64_t)dim * 2, 64,
-                         use_pair ? BP / 2 : BP);
+                         (uint64_t)n_ctiles * BP, (uint64_t)dim * 2, 64, BP);
     if (e == cudaSuccess && MODE != GEMM_FILTER && MODE != GEMM_EXP_FILTER)
         e = make_tmap_2d(&tc, out, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, (uint64_t)n_ctiles * BP,
                          (uint64_t)n_rows, (uint64_t)n_ctiles * BP * 4, 32, 128);
@@ -647,30 +581,10 @@ static cudaError_t gemm_bp(const uint16_t *emb, int64_t n_rows, int64_t row_stri
         tc = ta;   // unused by the filter epilogue
     if (e != cudaSuccess) return e;
     const int64_t m_tiles = ceil_div<int64_t>(n_rows, 128);
-    if (use_pair) {
-        const int64_t units = (m_tiles + 1) / 2 * n_ctiles;
-        const int64_t ncl = units < pair_clusters[dev] ? units : pair_clusters[dev];
-        cudaLaunchConfig_t cfg = {};
-        cudaLaunchAttribute at[1];
-        at[0].id = cudaLaunchAttributeClusterDimension;
-        at[0].val.clusterDim.x = 2;
-        at[0].val.clusterDim.y = 1;
-        at[0].val.clusterDim.z = 1;
-        cfg.gridDim = dim3((unsigned)(2 * ncl));
-        cfg.blockDim = dim3(C::THREADS);
-        cfg.dynamicSmemBytes = C::SMEM;
-        cfg.stream = st;
-        cfg.attrs = at;
-        cfg.numAttrs = 1;
-        e = cudaLaunchKernelEx(&cfg, k_gemm_umma<BP, MODE, CAN_PAIR>, ta, tb, tc, n_rows, dim,
-                               n_ctiles, ep);
-        if (zrows) *zrows = (int)(2 * ncl);
-        return e == cudaSuccess ? cudaGetLastError() : e;
-    }
     const int64_t tiles = m_tiles * n_ctiles;
     const int grid = (int)(tiles < device_sm_count() ? tiles : device_sm_count());
-    k_gemm_umma<BP, MODE, false><<<grid, C::THREADS, C::SMEM, st>>>(ta, tb, tc, n_rows, dim,
-                                                                     n_ctiles, ep);
+    k_gemm_umma<BP, MODE><<<grid, C::THREADS, C::SMEM, st>>>(ta, tb, tc, n_rows, dim, n_ctiles,
+                                                             ep);
     if (zrows) *zrows = grid;
     return cudaGetLastError();
 }
