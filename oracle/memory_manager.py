@@ -22,13 +22,20 @@ their dense stand-ins (the same substitution as the Dense-only form, §5.5):
       slot of its page (a tombstone).
   Block compaction: every page B whose invalid ratio
       phi(B) = invalid / total >= theta (0.75, §4.2) is compacted: its live
-      chunks are partitioned by namespace, grouped within a partition by
-      LLMGroup's stand-in -- connected components of the pairs at or above
-      the affinity threshold (both chunks live on compacted pages, same
-      namespace) -- and repacked into fresh pages partition by partition,
-      group by group (groups ordered by their earliest chunk), chunk ID order
-      within a group, P slots per page, groups sharing a page when they fit;
-      B is released.
+      chunks are partitioned by namespace (PartitionByUserSession), grouped
+      within a partition by LLMGroup's stand-in -- connected components of
+      the pairs at or above the affinity threshold (both chunks live on
+      compacted pages, same namespace) -- and repacked into fresh pages
+      partition by partition, group by group (groups ordered by their
+      earliest chunk), chunk ID order within a group, P slots per page.
+      Every partition starts on a fresh page, so no page ever holds chunks
+      of two namespaces (§4.2: compaction never mixes tenants or sessions).
+      Within a partition the groups are packed back to back and may share a
+      page: Algorithm 2 packs each group "into one or more new blocks", but
+      a fresh page per group would give every singleton survivor (the
+      common case) a page of its own and multiply space by up to P, against
+      the reclamation §4.2 gives as compaction's first purpose.  B is
+      released.
   Deleted chunks (tombstones of a delete) are invalid slots of their pages;
       they are never relocated.
 
@@ -142,12 +149,15 @@ class MemoryManager:
         for p in cand:
             self.total[p] = 0
             self.live[p] = 0
-        for i, c in enumerate(order):
-            p = self.next_page + i // self.P
+        p, fill, prev_ns = self.next_page - 1, self.P, None
+        for c in order:
+            if fill == self.P or int(self.ns[c]) != prev_ns:
+                p, fill = p + 1, 0            # a full page, or a new partition
             self.page[c] = p
             self.total[p] = self.total.get(p, 0) + 1
             self.live[p] = self.live.get(p, 0) + 1
-        self.next_page += -(-len(order) // self.P)
+            fill, prev_ns = fill + 1, int(self.ns[c])
+        self.next_page = p + 1
         self.writes += len(order)
         return cand
 

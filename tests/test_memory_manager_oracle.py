@@ -120,7 +120,7 @@ def test_compaction_packs_connected_components(seed):
     request sets >= tau, computed here from the trace), its connected
     components (networkx), and the packing by (namespace, earliest chunk of
     the component, chunk ID), P chunks per fresh page from the next free
-    page on."""
+    page on, each namespace starting on a page of its own (§4.2)."""
     nx = pytest.importorskip("networkx")
     # relocation at 0.5 leaves tombstones; compaction groups at 0.2, so that
     # associated pairs remain among the chunks it moves
@@ -149,13 +149,49 @@ def test_compaction_packs_connected_components(seed):
                 g.add_edge(a, b)
     comps = sorted((sorted(cc) for cc in nx.connected_components(g)),
                    key=lambda cc: (int(ns[cc[0]]), cc[0]))
-    order = [c for cc in comps for c in cc]
     assert cand and max(len(cc) for cc in comps) >= 2          # not vacuous
     first = mm.next_page
+    expect, base = {}, first
+    for t in sorted({int(ns[c]) for c in moving}):
+        members = [c for cc in comps if int(ns[cc[0]]) == t for c in cc]
+        for i, c in enumerate(members):
+            expect[c] = base + i // P
+        base += -(-len(members) // P)
     released = mm.compact(theta, tau)
     assert released == cand
-    for i, c in enumerate(order):
-        assert mm.page[c] == first + i // P, (c, i)
-    assert mm.next_page == first + -(-len(order) // P)
+    for c, p in expect.items():
+        assert mm.page[c] == p, (c, p)
+    assert mm.next_page == base
     for p in cand:
         assert mm.total[p] == 0 and mm.live[p] == 0
+
+
+@pytest.mark.parametrize("seed", [5, 8, 9])
+def test_compaction_never_mixes_namespaces(seed):
+    """§4.2: block compaction partitions the survivors by user and session
+    (PartitionByUserSession, Algorithm 2), so it never mixes chunks of two
+    tenants or sessions on a page.  Three namespaces whose survivor counts
+    are not multiples of P: every page compaction writes holds a single
+    namespace, and each namespace fills exactly ceil(survivors / P) pages.
+    Packing the survivors back to back across namespaces fails this."""
+    tau_r, tau, theta, P = 0.5, 0.2, 0.75, 8
+    page_of, reqs, comp = _random_trace(seed)
+    ns = (comp * 7 + 3) % 5 % 3
+    mm = MemoryManager(page_of, P, ns_of=ns)
+    mm.relocate(reqs, tau_r)
+    rng = np.random.default_rng(seed + 100)
+    mm.delete(rng.choice(mm.n, 60, replace=False))
+    first = mm.next_page
+    released = mm.compact(theta, tau)
+    moved = [c for c in range(mm.n) if not mm.dead[c] and mm.page[c] >= first]
+    counts = {}
+    for c in moved:
+        counts[int(ns[c])] = counts.get(int(ns[c]), 0) + 1
+    assert released and len(counts) == 3                      # not vacuous
+    assert any(v % P for v in counts.values())
+    owner = {}
+    for c in moved:
+        assert owner.setdefault(int(mm.page[c]), int(ns[c])) == int(ns[c]), c
+    for t, v in counts.items():
+        assert len({int(mm.page[c]) for c in moved if ns[c] == t}) == -(-v // P)
+    assert mm.next_page - first == sum(-(-v // P) for v in counts.values())
