@@ -89,6 +89,10 @@ HOP_DRAM_BYTES = 11.16e9
 # 1.035 GB) from the same kind of capture, taken on the current epilogue (u's
 # row extremes, Z's column sums per warp).  None once that kernel changes.
 SCORE_DRAM_BYTES = 3.183e9
+# distinct query batches the retrieval steps rotate through
+QUERY_POOL = 8
+# timed steps of the hop_path record (the hops always run)
+HOP_PATH_STEPS = 40
 
 
 def score_bytes(n, d, b):
@@ -557,6 +561,9 @@ def main():
     ap.add_argument("--impl", default="native", choices=["native", "reference"])
     ap.add_argument("--cpu-queries", type=int, default=8)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-hop-path", action="store_true",
+                    help="skip the retrieve workload's hop_path record (the same retrieval "
+                         "with the hops always run)")
     ap.add_argument("--placement", default="clustered")
     ap.add_argument("--scale", type=float, default=1.0,
                     help="shrink N (profiling captures of a smaller case); 1.0 = the benchmark")
@@ -589,10 +596,11 @@ def main():
         return run_retrieve(args, k=5, hops=0, metric=DENSE_METRIC, workload=DENSE_WORKLOAD)
     if args.workload == "scoped":
         return run_retrieve(args, metric=SCOPED_METRIC, workload=SCOPED_WORKLOAD, scoped=True)
-    return run_retrieve(args)
+    return run_retrieve(args, hop_path=not args.no_hop_path)
 
 
-def run_retrieve(args, k=None, hops=None, metric=METRIC, workload=WORKLOAD, scoped=False):
+def run_retrieve(args, k=None, hops=None, metric=METRIC, workload=WORKLOAD, scoped=False,
+                 hop_path=False):
     """The retrieval pass on the gmm1m store (k / hops override the
     configuration: the Dense-only form uses k = 5, hops = 0; `scoped` tags
     chunks by component mod 64 and scopes each query to a namespace, with
@@ -630,7 +638,11 @@ def run_retrieve(args, k=None, hops=None, metric=METRIC, workload=WORKLOAD, scop
     k = wl.k if k is None else k
     hops = wl.hops if hops is None else hops
     st = torch.cuda.Stream(device=dev)
-    q_dev = torch.from_numpy(wl.queries.view(np.int16)).to(f"cuda:{dev}")
+    # a rotating pool of distinct seeded query batches (the workload's own
+    # batch first): step i retrieves batch i mod POOL
+    batches = [wl.queries] + synth.query_batches(wl, QUERY_POOL - 1)
+    q_pool = torch.from_numpy(np.stack(batches).view(np.int16)).to(f"cuda:{dev}")
+    q_dev = torch.empty_like(q_pool[0])
     ids = torch.empty((B, k), dtype=torch.int64, device=f"cuda:{dev}")
     scores = torch.empty((B, k), dtype=torch.float32, device=f"cuda:{dev}")
     pages = torch.empty((B, k), dtype=torch.int32, device=f"cuda:{dev}")
@@ -641,9 +653,10 @@ def run_retrieve(args, k=None, hops=None, metric=METRIC, workload=WORKLOAD, scop
         store.set_namespace(0, torch.from_numpy(ns_of).to(f"cuda:{dev}"))
         q_ns = torch.from_numpy(q_ns_host).to(f"cuda:{dev}")
 
-    def step():
-        store.retrieve(q_dev, k, wl.alpha, hops, ids, scores, pages, npages, stream=st,
-                       q_ns=q_ns, sort_by_time=scoped)
+    def step(i, q=None, target=None):
+        (target or store).retrieve(q_pool[i % QUERY_POOL] if q is None else q, k, wl.alpha, hops,
+                                   ids, scores, pages, npages, stream=st, q_ns=q_ns,
+                                   sort_by_time=scoped)
 
     def barrier():
         torch.cuda.synchronize(dev)
@@ -651,8 +664,8 @@ def run_retrieve(args, k=None, hops=None, metric=METRIC, workload=WORKLOAD, scop
             torch.distributed.barrier()
 
     with torch.cuda.stream(st):
-        for _ in range(args.warmup):
-            step()
+        for i in range(args.warmup):
+            step(i)
     store.sync(stream=st)
     # ---- timed region (device-resident inputs)
     store.set_profiling(True)
@@ -662,8 +675,8 @@ def run_retrieve(args, k=None, hops=None, metric=METRIC, workload=WORKLOAD, scop
     ev1 = torch.cuda.Event(enable_timing=True)
     with Clocks(dev) as clk:
         ev0.record(st)
-        for _ in range(args.steps):
-            step()
+        for i in range(args.steps):
+            step(i)
         ev1.record(st)
         barrier()
     store.sync(stream=st)
@@ -674,32 +687,32 @@ def run_retrieve(args, k=None, hops=None, metric=METRIC, workload=WORKLOAD, scop
     npg_clustered = npages.float().mean().item()
 
     # ---- end-to-end: host query buffer in, host results out, via the public API
-    q_host = torch.from_numpy(wl.queries.view(np.int16)).pin_memory()
+    q_host = torch.from_numpy(np.stack(batches).view(np.int16)).pin_memory()
     outs_host = [torch.empty((B, k), dtype=torch.int64).pin_memory(),
                  torch.empty((B, k), dtype=torch.float32).pin_memory(),
                  torch.empty((B, k), dtype=torch.int32).pin_memory(),
                  torch.empty((B,), dtype=torch.int32).pin_memory()]
 
-    def e2e_step():
+    def e2e_step(i):
         with torch.cuda.stream(st):
-            q_dev.copy_(q_host, non_blocking=True)
-            step()
+            q_dev.copy_(q_host[i % QUERY_POOL], non_blocking=True)
+            step(i, q=q_dev)
             for h, d in zip(outs_host, (ids, scores, pages, npages)):
                 h.copy_(d, non_blocking=True)
 
-    for _ in range(args.warmup):
-        e2e_step()
+    for i in range(args.warmup):
+        e2e_step(i)
     barrier()
     e0 = torch.cuda.Event(enable_timing=True)
     e1 = torch.cuda.Event(enable_timing=True)
     e0.record(st)
-    for _ in range(args.steps):
-        e2e_step()
+    for i in range(args.steps):
+        e2e_step(i)
     e1.record(st)
     barrier()
     ms_e2e = e0.elapsed_time(e1)
     store.sync(stream=st)
-    h2d = q_host.numel() * 2
+    h2d = q_host[0].numel() * 2
     d2h = sum(t.numel() * t.element_size() for t in outs_host)
 
     # max over ranks
@@ -733,14 +746,18 @@ def run_retrieve(args, k=None, hops=None, metric=METRIC, workload=WORKLOAD, scop
     # which propagation ran: the hops, or (two hops, every row that can reach
     # the top-k among the reach candidates) the candidates' scores from u
     if hops >= 1 and phases["propagate"][1] == 0 and phases["last_hop"][1] > 0:
+        moved = wl.n * wl.dim * 2 + 2 * wl.n * 256 * 4 + wl.n * 40 * 4
         path_note = {"propagation": "two-hop scores of the top-k candidates from graph-only "
                                     "reach coefficients, one pass over u (no hop run)",
-                     "bytes_moved_per_step": wl.n * wl.dim * 2 + 2 * wl.n * 256 * 4
-                                             + wl.n * 40 * 4,
+                     "bytes_moved_per_step": moved,
                      "note": "pass_roofline counts full hops (five slab passes); this path "
-                             "reads E, writes u and reads u and the candidates' coefficients"}
+                             "reads E, writes u and reads u and the candidates' coefficients "
+                             "(40 per row)"}
     else:
-        path_note = {"propagation": "hops (the last one skips rows below the top-k floor)"}
+        moved = total_ab
+        path_note = {"propagation": "hops (the last one skips rows below the top-k floor)",
+                     "bytes_moved_per_step": moved}
+    path_note["call_hbm_frac"] = moved / (per_step_ms * 1e-3) / 1e9 / hbm
     line = {
         "metric": metric,
         "value": job_throughput(B * args.steps, ws, ms),
@@ -757,6 +774,8 @@ def run_retrieve(args, k=None, hops=None, metric=METRIC, workload=WORKLOAD, scop
         "config": {"workload": workload if args.scale == 1.0 else f"{workload} scaled by {args.scale}",
                    "l2": "inputs larger than L2 (E 2.1 GB, score slabs 1.07 GB "
                    "each), no flush", "placement": args.placement,
+                   "queries": f"{QUERY_POOL} distinct seeded batches of {B}, step i takes batch "
+                              f"i mod {QUERY_POOL}",
                    "parallelism": "replicas" if ws > 1 else "single GPU"},
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": hbm, "unit": "GB/s",
                      "frac": achieved / hbm,
@@ -786,12 +805,70 @@ def run_retrieve(args, k=None, hops=None, metric=METRIC, workload=WORKLOAD, scop
         po = wl.page_of[other]
         sel = ids.cpu().numpy()
         line["pages_per_query"][other] = float(np.mean([len(set(po[r].tolist())) for r in sel]))
+    store.close()
+    if hop_path and hops >= 1 and not scoped and args.scale == 1.0:
+        line["hop_path"] = time_hop_path(args, wl, step, st, barrier, dev, ws, B, hbm, peak_kind)
     if rank == 0:
         print(json.dumps(line), flush=True)
-    store.close()
     if ws > 1:
         torch.distributed.destroy_process_group()
     return 0
+
+
+def time_hop_path(args, wl, step, st, barrier, dev, ws, B, hbm, peak_kind):
+    """The same retrieval with the hops always run (a store created with
+    AKASHIC_REACH=0), timed the same way over the same rotating batches:
+    its queries/s, and the full hop's roofline (graph once + two slab
+    passes per hop against the hop phase's event-timed duration) with its
+    ncu DRAM bytes."""
+    import torch
+    from paper_2607_05708_gb300 import MemStore
+    old = os.environ.get("AKASHIC_REACH")
+    os.environ["AKASHIC_REACH"] = "0"
+    try:
+        store = MemStore.from_arrays(wl.emb, wl.page_of[args.placement], wl.row_ptr, wl.col,
+                                     wl.aff, capacity=wl.n, chunks_per_page=wl.chunks_per_page,
+                                     temperature=wl.tau, device=dev)
+    finally:
+        if old is None:
+            del os.environ["AKASHIC_REACH"]
+        else:
+            os.environ["AKASHIC_REACH"] = old
+    steps = max(1, min(args.steps, HOP_PATH_STEPS))
+    with torch.cuda.stream(st):
+        for i in range(args.warmup):
+            step(i, target=store)
+    store.sync(stream=st)
+    store.set_profiling(True)
+    store.phase_times()
+    barrier()
+    ev0 = torch.cuda.Event(enable_timing=True)
+    ev1 = torch.cuda.Event(enable_timing=True)
+    ev0.record(st)
+    for i in range(steps):
+        step(i, target=store)
+    ev1.record(st)
+    barrier()
+    store.sync(stream=st)
+    ms = ev0.elapsed_time(ev1)
+    phases = store.phase_times()
+    store.close()
+    ms = max_over_ranks([ms], device=f"cuda:{dev}" if ws > 1 else None)[0]
+    hop_ms = phases["propagate"][0] / steps
+    per_hop = hop_bytes(wl.n, 256, wl.nnz)
+    achieved = per_hop / (hop_ms * 1e-3) / 1e9
+    return {
+        "value": job_throughput(B * steps, ws, ms), "unit": "queries/s", "steps": steps,
+        "ms_per_step": ms / steps,
+        "phases_ms_per_step": {p: phases[p][0] / steps
+                               for p in ("score", "propagate", "last_hop", "bound", "select")},
+        "roofline": {"bound": "hbm", "achieved": achieved, "peak": hbm, "unit": "GB/s",
+                     "frac": achieved / hbm, "traffic": HOP_DRAM_BYTES,
+                     "kernel": "propagate", "what": "full propagation hop (graph once + two "
+                     "slab passes), k_hop_segs + k_hop_rows", "peak_kind": peak_kind},
+        "note": "the same store and batches with AKASHIC_REACH=0: the first hop runs in full, "
+                "the last skips rows whose bound stays below the top-k floor",
+    }
 
 
 if __name__ == "__main__":

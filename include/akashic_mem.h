@@ -277,10 +277,11 @@ akashic_status_t akashic_mem_phase_times(akashic_mem_t *m, float *ms, int32_t *l
 
 /* Softmax scores for callers that cannot allocate device memory.
  *
- * The paper has no counterpart: this is a library convenience.  Code that
- * records work into a CUDA graph, runs inside a serving runtime's
- * pre-reserved memory pool, or has no device allocator cannot call
- * cudaMalloc when it needs scores, and akashic_mem_create allocates.  This
+ * The paper has no counterpart: this is a library convenience.  A serving
+ * runtime that works inside a memory pool it reserved up front, code that
+ * is recording a stream capture, or a host without a device allocator
+ * cannot call cudaMalloc when it needs scores, and akashic_mem_create
+ * allocates.  This
  * call needs no store and allocates nothing: it computes, over caller-owned
  * buffers, the score step of retrieval
  *   u[j*B + b] = exp(tau <e_j, q_b> - c_b),   z[b] = sum_j u[j*B + b],
@@ -299,9 +300,10 @@ akashic_status_t akashic_mem_phase_times(akashic_mem_t *m, float *ms, int32_t *l
  *          the kernels
  * Its scratch is a fixed 320 KiB array in device memory, present on every
  * GPU that runs this call until the process exits (no allocation ever
- * happens).  The first call on a device looks up that array's address with
- * cudaGetSymbolAddress while the device is current; make that first call
- * before capturing a stream.  Every call shares the array, so calls whose
+ * happens).  The first call on a device does a one-time set-up while the
+ * device is current: it looks up that array's address with
+ * cudaGetSymbolAddress and sets the score kernel's shared-memory limit for
+ * all four widths B; make that first call before capturing a stream.  Every call shares the array, so calls whose
  * work overlaps on the GPU (different streams without ordering) race and
  * must not be issued.  Stream-ordered; does not synchronise.
  * EINVAL for a NULL pointer, misalignment, n < 1, dim outside [64, 4096]

@@ -1001,15 +1001,24 @@ akashic_status_t akashic_mem_compact_pages(akashic_mem_t *m, float theta, float 
         CUDA_TRY(radix_sort_pairs(nsk, sid, nk, spare_v, count, 32, tmp, tb, st, &alt2,
                                   &ph.launches));
         const uint32_t *order = alt2 ? spare_v : sid;
-        AK_TRY(mm_ensure_pages(m, m->next_page + ceil_div<int64_t>(count, m->per_page) + 1, st));
-        CUDA_TRY(launch_mm_release_repack(mm_tables(m), pages, cand, order, count, row_of,
-                                          m->page_of.as<int32_t>(), m->next_page, m->per_page,
-                                          st));
-        ph.launches += 2 + (pages > 0) + 1;
-        m->next_page += ceil_div<int64_t>(count, m->per_page);
+        const uint32_t *ns_sorted = alt2 ? nk : nsk;
+        // every namespace starts on a fresh page (compaction never mixes
+        // tenants or sessions): pages per namespace run, scanned into each
+        // run's base page; `moving` and `pos` are free again
+        CUDA_TRY(launch_mm_part_pages(ns_sorted, count, m->per_page, moving, st));
+        CUDA_TRY(scan_exclusive(moving, pos, count, tmp, tb, st, &ph.launches));
+        int64_t new_pages = 0;
+        CUDA_TRY(cudaMemcpyAsync(&new_pages, pos + count, 8, cudaMemcpyDeviceToHost, st));
+        AK_TRY(check_status(m, st, "compact"));
+        AK_TRY(mm_ensure_pages(m, m->next_page + new_pages + 1, st));
+        CUDA_TRY(launch_mm_release_repack(mm_tables(m), pages, cand, order, ns_sorted, pos, count,
+                                          row_of, m->page_of.as<int32_t>(), m->next_page,
+                                          m->per_page, st));
+        ph.launches += 3 + (pages > 0) + 1;
+        m->next_page += new_pages;
         m->moves += count;
     } else if (n_rel > 0) {
-        CUDA_TRY(launch_mm_release_repack(t, pages, cand, nullptr, 0, row_of,
+        CUDA_TRY(launch_mm_release_repack(t, pages, cand, nullptr, nullptr, nullptr, 0, row_of,
                                           m->page_of.as<int32_t>(), m->next_page, m->per_page,
                                           st));
         ph.launches += 1;

@@ -81,6 +81,9 @@ int64_t score_tiles(int64_t n);
 // each row over the first n_real columns (the real queries), for the
 // propagation's row bounds; with them, ext (optional, [2], zeroed before)
 // gets their extremes in launch_final_bounds' encoding.
+// Raises the score kernel's shared-memory limit for every query width on the
+// current device now (launch_score does it lazily per width otherwise).
+cudaError_t prepare_score_gemm();
 cudaError_t launch_score(const uint16_t *emb, int64_t n, int dim, const uint16_t *qp, int bp,
                          const float *shift, float tau, float *u, float *zpart, int *status,
                          cudaStream_t st, int *launches, int *zrows,
@@ -275,8 +278,14 @@ cudaError_t launch_mm_union(const MmTables &t, const int64_t *moving, const int3
 cudaError_t launch_mm_keys(const int64_t *moving, const int64_t *pos, int64_t n,
                            const int32_t *parent, const int32_t *ns_by_id, uint32_t *ids,
                            uint32_t *root_key, uint32_t *ns_key, cudaStream_t st);
+// part_pages[i] = pages the namespace run starting at i fills (0 inside a run)
+cudaError_t launch_mm_part_pages(const uint32_t *ns_sorted, int64_t count, int per_page,
+                                 int64_t *part_pages, cudaStream_t st);
+// releases the candidate pages, then writes the ordered chunks into fresh
+// pages from first_page on, each namespace from its own base page
 cudaError_t launch_mm_release_repack(const MmTables &t, int64_t n_pages, const int32_t *cand,
-                                     const uint32_t *order_ids, int64_t count,
+                                     const uint32_t *order_ids, const uint32_t *ns_sorted,
+                                     const int64_t *part_base, int64_t count,
                                      const int32_t *row_of, int32_t *page_row, int64_t first_page,
                                      int per_page, cudaStream_t st);
 cudaError_t launch_mm_count_pages(const int32_t *page_row, int64_t first, int64_t n,

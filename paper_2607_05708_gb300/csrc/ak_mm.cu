@@ -293,12 +293,54 @@ __global__ void k_mm_release(MmTables t, int64_t n_pages, const int32_t *__restr
         }
 }
 
-__global__ void k_mm_repack(const uint32_t *__restrict__ order_ids, int64_t count,
+// first index of the sorted keys[0, count) holding a key >= v
+__device__ __forceinline__ int64_t lower_bound_u32(const uint32_t *__restrict__ keys, int64_t count,
+                                                   uint32_t v) {
+    int64_t lo = 0, hi = count;
+    while (lo < hi) {
+        const int64_t mid = (lo + hi) >> 1;
+        if (keys[mid] < v) lo = mid + 1;
+        else hi = mid;
+    }
+    return lo;
+}
+
+// Every namespace (partition) starts on a fresh page: at the first
+// position of each run of equal namespace keys, the pages that run fills
+// (ceil(run / P)); zero elsewhere.  An exclusive scan of these gives each
+// partition's first page relative to the first fresh page.
+__global__ void k_mm_part_pages(const uint32_t *__restrict__ ns_sorted, int64_t count,
+                                int per_page, int64_t *__restrict__ part_pages) {
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < count;
+         i += (int64_t)gridDim.x * blockDim.x) {
+        const uint32_t k = ns_sorted[i];
+        int64_t v = 0;
+        if (i == 0 || ns_sorted[i - 1] != k) {
+            const int64_t end = k == 0xffffffffu ? count : lower_bound_u32(ns_sorted, count, k + 1);
+            v = (end - i + per_page - 1) / per_page;
+        }
+        part_pages[i] = v;
+    }
+}
+
+cudaError_t launch_mm_part_pages(const uint32_t *ns_sorted, int64_t count, int per_page,
+                                 int64_t *part_pages, cudaStream_t st) {
+    if (count <= 0) return cudaSuccess;
+    k_mm_part_pages<<<device_sm_count() * 2, 256, 0, st>>>(ns_sorted, count, per_page, part_pages);
+    return cudaGetLastError();
+}
+
+// chunk i of the ordered list: page = first page + its partition's base
+// page + (offset inside the partition) / P
+__global__ void k_mm_repack(const uint32_t *__restrict__ order_ids,
+                            const uint32_t *__restrict__ ns_sorted,
+                            const int64_t *__restrict__ part_base, int64_t count,
                             const int32_t *__restrict__ row_of, int32_t *__restrict__ page_row,
                             MmTables t, int64_t first_page, int per_page) {
     for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < count;
          i += (int64_t)gridDim.x * blockDim.x) {
-        const int32_t p = (int32_t)(first_page + i / per_page);
+        const int64_t s = lower_bound_u32(ns_sorted, count, ns_sorted[i]);
+        const int32_t p = (int32_t)(first_page + part_base[s] + (i - s) / per_page);
         page_row[row_of[order_ids[i]]] = p;
         atomicAdd(&t.page_total[p], 1);
         atomicAdd(&t.page_live[p], 1);
@@ -418,15 +460,16 @@ cudaError_t launch_mm_keys(const int64_t *moving, const int64_t *pos, int64_t n,
 }
 
 cudaError_t launch_mm_release_repack(const MmTables &t, int64_t n_pages, const int32_t *cand,
-                                     const uint32_t *order_ids, int64_t count,
+                                     const uint32_t *order_ids, const uint32_t *ns_sorted,
+                                     const int64_t *part_base, int64_t count,
                                      const int32_t *row_of, int32_t *page_row, int64_t first_page,
                                      int per_page, cudaStream_t st) {
     const int sms = device_sm_count();
     if (n_pages > 0) k_mm_release<<<sms * 2, 256, 0, st>>>(t, n_pages, cand);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess || count <= 0) return e;
-    k_mm_repack<<<sms * 2, 256, 0, st>>>(order_ids, count, row_of, page_row, t, first_page,
-                                         per_page);
+    k_mm_repack<<<sms * 2, 256, 0, st>>>(order_ids, ns_sorted, part_base, count, row_of, page_row,
+                                         t, first_page, per_page);
     return cudaGetLastError();
 }
 

@@ -91,8 +91,10 @@ static akashic_status_t noalloc_fail(akashic_status_t code, const char *fmt, ...
     return code;
 }
 
-// Device address of the scratch array, looked up once per device (with that
-// device current) on the first call made on it.
+// Set-up on the first call made on a device (with that device current):
+// the device address of the scratch array, and the score kernel's
+// shared-memory limit for all four query widths, so that later calls with
+// any B do no set-up at all.
 static std::mutex g_noalloc_mu;
 static unsigned char *g_noalloc_ptr[64] = {nullptr};
 
@@ -101,6 +103,7 @@ static cudaError_t noalloc_scratch(int dev, unsigned char **out) {
     if (!g_noalloc_ptr[dev]) {
         void *p = nullptr;
         cudaError_t e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
+        if (e == cudaSuccess) e = prepare_score_gemm();
         if (e != cudaSuccess) return e;
         g_noalloc_ptr[dev] = (unsigned char *)p;
     }
@@ -142,7 +145,7 @@ extern "C" akashic_status_t akashic_mem_softmax_scores_noalloc(const uint16_t *e
     unsigned char *scr = nullptr;
     cudaError_t e = noalloc_scratch(dev, &scr);
     if (e != cudaSuccess)
-        return noalloc_fail(AKASHIC_ECUDA, "softmax_scores_noalloc: cudaGetSymbolAddress: %s",
+        return noalloc_fail(AKASHIC_ECUDA, "softmax_scores_noalloc: set-up on this device: %s",
                             cudaGetErrorString(e));
     cudaStream_t st = (cudaStream_t)stream;
     const float tau = temperature > 0.f ? temperature : 1.0f / sqrtf((float)dim);

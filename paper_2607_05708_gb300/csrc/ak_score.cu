@@ -552,12 +552,10 @@ __global__ __launch_bounds__(GemmCfg<BP, MODE>::THREADS, 1) void k_gemm_umma(con
 
 int64_t score_tiles(int64_t n) { return ceil_div<int64_t>(n, 128); }
 
-// A: E rows (row_stride_rows apart: 1 = every row, s = every s-th row),
-// B: n_ctiles * BP query rows, C: output [n_rows][n_ctiles * BP] (EXP/RAW).
+// The kernel's dynamic shared-memory limit, raised once per device (with
+// that device current) before its first launch there.
 template <int BP, int MODE>
-static cudaError_t gemm_bp(const uint16_t *emb, int64_t n_rows, int64_t row_stride_rows, int dim,
-                           const uint16_t *qp, int n_ctiles, float *out, const GemmEpi &ep,
-                           cudaStream_t st, int *zrows) {
+static cudaError_t gemm_attr() {
     using C = GemmCfg<BP, MODE>;
     static bool attr[64] = {false};
     int dev = 0;
@@ -568,8 +566,28 @@ static cudaError_t gemm_bp(const uint16_t *emb, int64_t n_rows, int64_t row_stri
         if (e != cudaSuccess) return e;
         attr[dev] = true;
     }
+    return cudaSuccess;
+}
+
+cudaError_t prepare_score_gemm() {
+    cudaError_t e = gemm_attr<32, GEMM_EXP>();
+    if (e == cudaSuccess) e = gemm_attr<64, GEMM_EXP>();
+    if (e == cudaSuccess) e = gemm_attr<128, GEMM_EXP>();
+    if (e == cudaSuccess) e = gemm_attr<256, GEMM_EXP>();
+    return e;
+}
+
+// A: E rows (row_stride_rows apart: 1 = every row, s = every s-th row),
+// B: n_ctiles * BP query rows, C: output [n_rows][n_ctiles * BP] (EXP/RAW).
+template <int BP, int MODE>
+static cudaError_t gemm_bp(const uint16_t *emb, int64_t n_rows, int64_t row_stride_rows, int dim,
+                           const uint16_t *qp, int n_ctiles, float *out, const GemmEpi &ep,
+                           cudaStream_t st, int *zrows) {
+    using C = GemmCfg<BP, MODE>;
+    cudaError_t e = gemm_attr<BP, MODE>();
+    if (e != cudaSuccess) return e;
     CUtensorMap ta, tb, tc;
-    cudaError_t e = make_tmap_2d(&ta, emb, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, (uint64_t)dim,
+    e = make_tmap_2d(&ta, emb, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, (uint64_t)dim,
                                  (uint64_t)n_rows, (uint64_t)dim * 2 * row_stride_rows, 64, 128);
     if (e == cudaSuccess)
         e = make_tmap_2d(&tb, qp, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, (uint64_t)dim,

@@ -394,6 +394,7 @@ def workload(index: int, scale: float = 1.0, placements=None) -> Workload:
         aff = np.log(u).astype(np.float32)                 # softmax(log u) = u / sum(u)
         queries = _iid_unit_bf16(s_query, cfg["queries"], d)
         comp = None
+        wl_centers = None
         recipe = ("iid N(0,1) rows, L2-normalised in fp32, rounded to bf16; 8 distinct uniform "
                   "out-neighbours per chunk (never itself); edge logit ln(U), U~U(0,1], so the row "
                   "softmax equals U row-normalised; queries from the same distribution; 16 chunks "
@@ -427,6 +428,7 @@ def workload(index: int, scale: float = 1.0, placements=None) -> Workload:
                       "(std 0.1/sqrt(d)); 64 chunks per page, clustered (by component) and random")
         if index == 1:
             aff = (10.0 * dots).astype(np.float32)
+        wl_centers = centers
         rng_q = np.random.default_rng(s_query)
         qc = rng_q.integers(0, n_comp, size=cfg["queries"])
         queries = _mixture_bf16(s_query.spawn(1)[0], centers, qc.astype(np.int32), 0.1 / math.sqrt(d))
@@ -436,7 +438,7 @@ def workload(index: int, scale: float = 1.0, placements=None) -> Workload:
         name=cfg["name"], dim=d, emb=emb, queries=queries, row_ptr=row_ptr, col=col, aff=aff,
         page_of=pages, chunks_per_page=cfg["per_page"], alpha=cfg["alpha"], hops=cfg["hops"],
         k=cfg["k"], component=comp, streams=cfg.get("streams", 1), recipe=recipe,
-        meta=dict(index=index, scale=scale, seed=cfg["seed"]),
+        meta=dict(index=index, scale=scale, seed=cfg["seed"], centers=wl_centers),
     )
     if "order_seed" in cfg:
         wl.stream_order = np.random.default_rng(cfg["order_seed"]).permutation(cfg["streams"])
@@ -453,6 +455,24 @@ def workload(index: int, scale: float = 1.0, placements=None) -> Workload:
                       "to its size), "
                       "top-32 cosine neighbours among the old store, reciprocal edges")
     return wl
+
+
+def query_batches(wl: Workload, count: int, seed: int = 2026) -> list:
+    """`count` further query batches of the workload's size, drawn by the
+    workload's own query recipe (mixture stores: a uniformly drawn centre +
+    N(0, (0.1/sqrt(d))^2 I); the iid store: iid unit rows), unit length,
+    bf16, from SeedSequence(seed).  Returns a list of uint16 [B, dim]."""
+    ss = np.random.SeedSequence(seed)
+    out = []
+    centers = wl.meta.get("centers")
+    for kid in ss.spawn(count):
+        if centers is None:
+            out.append(_iid_unit_bf16(kid, wl.n_queries, wl.dim))
+        else:
+            a, b = kid.spawn(2)
+            qc = np.random.default_rng(a).integers(0, centers.shape[0], size=wl.n_queries)
+            out.append(_mixture_bf16(b, centers, qc.astype(np.int32), 0.1 / math.sqrt(wl.dim)))
+    return out
 
 
 def request_trace(wl: Workload, n_queries: int, n_topics: int = 4096, s: float = 1.1,

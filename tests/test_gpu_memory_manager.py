@@ -156,11 +156,20 @@ def test_compaction_groups_associated_chunks():
     st.delete(torch.from_numpy(v).cuda())
     mm.delete(v)
     _check(st, mm)
-    w = mm.writes
+    w, first = mm.writes, mm.next_page
     rel = st.compact_pages(0.75, 0.5)
     assert rel == len(mm.compact(0.75, 0.5))
     _check(st, mm)
     assert mm.writes - w >= 100                 # survivors were moved, grouped
+    # §4.2: compaction never mixes namespaces on a page; the three
+    # namespaces' survivors do not fill whole pages
+    pages = st.export_pages().cpu().numpy()
+    moved = np.nonzero((pages >= first) & ~mm.dead)[0]
+    per_ns = np.bincount(ns[moved], minlength=3)
+    assert (per_ns > 0).all() and (per_ns % P != 0).any()
+    for p in np.unique(pages[moved]):
+        assert np.unique(ns[moved[pages[moved] == p]]).size == 1, p
+    assert mm.next_page - first == sum(-(-int(v) // P) for v in per_ns)
 
 
 def test_relocation_lowers_pages_per_request():
