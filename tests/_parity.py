@@ -68,6 +68,23 @@ def oracle_retrieve(wl, placement, queries=None, k=None, alpha=None, hops=None):
                            page_of=wl.page_of[placement], want_final=True)
 
 
+def oracle_retrieve_rows(wl, placement, rows, threads=None):
+    """The oracle on the query rows `rows`, a few rows per host thread (the
+    oracle's C code releases the interpreter lock; each call is the plain
+    single-threaded oracle on its rows).  Same dict as oracle_retrieve."""
+    import os
+    from concurrent.futures import ThreadPoolExecutor
+    rows = list(rows)
+    oracle_weights(wl)                         # once, before the threads
+    threads = max(1, min(len(rows), threads or os.cpu_count() or 1))
+    parts = [rows[i::threads] for i in range(threads)]
+    with ThreadPoolExecutor(max_workers=threads) as ex:
+        outs = list(ex.map(lambda r: oracle_retrieve(wl, placement, queries=wl.queries[r]),
+                           parts))
+    order = np.argsort(np.concatenate([np.asarray(p) for p in parts]), kind="stable")
+    return {key: np.concatenate([o[key] for o in outs])[order] for key in outs[0]}
+
+
 def assert_retrieval_parity(wl, placement, got, ref, rows=None):
     """got: GPU outputs (row r of got = query rows[r] of ref if rows is given)."""
     page_of = wl.page_of[placement]
@@ -135,9 +152,11 @@ def assert_scoped_parity(wl, placement, got, ref, ns_of, q_ns, sort_by_time):
 
 
 # --------------------------------------------------------------------------- relation update
-def check_update(wl, sample=None, M=None, seed=0):
+def check_update(wl, sample=None, M=None, seed=0, golden=None):
     """Append wl.new_emb to a store holding wl, run the update on the GPU and
-    compare with the oracle (all new rows, or a seeded sample of them)."""
+    compare with the oracle: all new rows (the oracle run here, or its
+    stored result `golden` = dict(nbr_ids, nbr_cos) for every new chunk),
+    or a seeded sample of them."""
     import torch
     from paper_2607_05708_gb300 import MemStore
     M = M or wl.top_m
@@ -151,8 +170,10 @@ def check_update(wl, sample=None, M=None, seed=0):
     store.update_relations(first, n_new, M, reciprocal=wl.reciprocal)
     store.sync()
     rp, col, aff, w = (t.cpu().numpy() for t in store.export_csr())
-    all_emb = np.concatenate([wl.emb, wl.new_emb])
-    if sample is None:
+    if golden is not None:
+        _compare_update(wl, M, rp, col, aff, w, golden, np.arange(n_new), full=True)
+    elif sample is None:
+        all_emb = np.concatenate([wl.emb, wl.new_emb])
         old_rp = np.concatenate([wl.row_ptr, np.full(n_new, wl.row_ptr[-1], np.int64)])
         ref = oracle.update_relations(all_emb, n_old, n_new, M, old_rp, wl.col, wl.aff,
                                       scale=wl.relation_scale, reciprocal=wl.reciprocal)
@@ -169,45 +190,96 @@ def check_update(wl, sample=None, M=None, seed=0):
     return store
 
 
-def _compare_update(wl, M, rp, col, aff, w, ref, picks, full):
+def _cosines(wl, nids, cols):
+    """fp64 <e_nid, e_col> of the widened stored values, pair by pair."""
+    all_emb = (wl.emb, wl.new_emb)
     n_old = wl.n
-    E = oracle_free_widen(np.concatenate([wl.emb, wl.new_emb]))
+
+    def rows(ids):
+        ids = np.asarray(ids, np.int64)
+        out = np.empty((ids.size, wl.dim), np.uint16)
+        old = ids < n_old
+        out[old] = all_emb[0][ids[old]]
+        out[~old] = all_emb[1][ids[~old] - n_old]
+        return oracle_free_widen(out)
+
+    res = np.empty(len(nids), np.float64)
+    for s in range(0, len(nids), 16384):
+        a, b = rows(nids[s:s + 16384]), rows(cols[s:s + 16384])
+        res[s:s + 16384] = np.einsum("ij,ij->i", a, b)
+    return res
+
+
+def _compare_update(wl, M, rp, col, aff, w, ref, picks, full):
+    """The picked new rows against the oracle's selection (swaps only among
+    near-ties at the M-th cosine), logits = scale * fp64 cosine, reciprocal
+    edges.  With `full`, every row of the exported CSR against the oracle's
+    CSR with those recorded swaps applied: the old edges of every row in
+    place and bit-exact, then the reciprocal edges of the new chunks that
+    chose the row, in ascending ID order; each new row its M neighbours in
+    ascending ID order; row pointers equal throughout."""
+    n_old, n_new = wl.n, len(wl.new_emb)
+    scale = wl.relation_scale
     assert (np.diff(rp) >= 0).all()
-    assert rp[-1] == wl.row_ptr[-1] + len(wl.new_emb) * M * (2 if wl.reciprocal else 1)
-    for t, a in enumerate(picks):
-        nid = n_old + a
-        g_cols = col[rp[nid]:rp[nid + 1]]
-        o_ids = ref["nbr_ids"][t]
-        o_cos = ref["nbr_cos"][t]
-        assert len(g_cols) == M and (np.diff(g_cols) > 0).all()
-        kth = o_cos[M - 1]
-        for x in set(g_cols.tolist()) ^ set(o_ids.tolist()):
-            cx = float(E[x] @ E[nid])
-            assert abs(cx - kth) < COS_ABS, f"new chunk {nid}: neighbour {x} swapped ({cx} vs {kth})"
-        for x, lg in zip(g_cols, aff[rp[nid]:rp[nid + 1]]):
-            cx = float(E[x] @ E[nid])
-            assert abs(lg - wl.relation_scale * cx) <= 1e-5 * max(1.0, abs(wl.relation_scale * cx)), \
-                f"logit of {nid}->{x}: {lg} vs {wl.relation_scale * cx}"
-            if wl.reciprocal:
+    assert rp[-1] == wl.row_ptr[-1] + n_new * M * (2 if wl.reciprocal else 1)
+    nid_all = n_old + np.asarray(picks, np.int64)
+    g_nbr = np.stack([col[rp[nid]:rp[nid + 1]] for nid in nid_all]).astype(np.int64)
+    assert g_nbr.shape == (len(picks), M), "a new row does not hold M neighbours"
+    assert (np.diff(g_nbr, axis=1) > 0).all() and (g_nbr < n_old).all()
+    swaps = 0
+    for t, nid in enumerate(nid_all):
+        o_ids = np.asarray(ref["nbr_ids"][t], np.int64)
+        kth = float(ref["nbr_cos"][t][M - 1])
+        diff = sorted(set(g_nbr[t].tolist()) ^ set(o_ids.tolist()))
+        if diff:
+            cx = _cosines(wl, np.full(len(diff), nid), np.array(diff))
+            for x, c in zip(diff, cx):
+                assert abs(c - kth) < COS_ABS, f"new chunk {nid}: neighbour {x} swapped ({c} vs {kth})"
+            swaps += len(diff) // 2
+    # logits of the new rows = scale * fp64 cosine; reciprocal edges carry the same
+    fwd_pos = np.concatenate([np.arange(rp[nid], rp[nid + 1]) for nid in nid_all])
+    cx = _cosines(wl, np.repeat(nid_all, M), g_nbr.ravel())
+    lg = aff[fwd_pos].astype(np.float64)
+    assert (np.abs(lg - scale * cx) <= 1e-5 * np.maximum(1.0, np.abs(scale * cx))).all(), \
+        "new-row logits differ from scale * cos"
+    if wl.reciprocal:
+        for t, nid in enumerate(nid_all):
+            for x, l in zip(g_nbr[t], aff[rp[nid]:rp[nid + 1]]):
                 row = col[rp[x]:rp[x + 1]]
                 pos = np.searchsorted(row, nid)
                 assert pos < len(row) and row[pos] == nid, f"missing reciprocal edge {x}->{nid}"
-                assert aff[rp[x] + pos] == lg
+                assert aff[rp[x] + pos] == l
     # weights: row softmax of the exported logits
     wr = oracle.row_softmax(rp, aff)
     assert np.allclose(w, wr, rtol=2e-3, atol=0)
-    if full:
-        # whole CSR identical to the oracle's, given no swaps were needed
-        if (ref["row_ptr"] == rp).all() and (ref["col"] == col).all():
-            assert np.allclose(aff, ref["aff"], rtol=1e-5, atol=1e-5)
-        else:
-            # a swap happened: row pointers can differ only through swapped reciprocal edges
-            assert ref["row_ptr"][-1] == rp[-1]
-        # old edges untouched
-        for i in range(0, n_old, max(1, n_old // 997)):
-            a, b = wl.row_ptr[i], wl.row_ptr[i + 1]
-            g = col[rp[i]:rp[i] + (b - a)]
-            assert (g == wl.col[a:b]).all()
+    if not full:
+        return swaps
+    # the whole CSR, row by row (vectorised)
+    orig_len = np.diff(wl.row_ptr)
+    js = g_nbr.ravel()
+    nids = np.repeat(nid_all, M)
+    cnt = np.bincount(js, minlength=n_old) if wl.reciprocal else np.zeros(n_old, np.int64)
+    exp_len = np.concatenate([orig_len + cnt, np.full(n_new, M, np.int64)])
+    exp_rp = np.concatenate([[0], np.cumsum(exp_len)])
+    assert (rp == exp_rp).all(), "row pointers differ from the oracle's CSR with its swaps"
+    exp_col = np.full(exp_rp[-1], -1, np.int64)
+    owner = np.repeat(np.arange(n_old), orig_len)
+    old_pos = exp_rp[owner] + (np.arange(wl.row_ptr[-1]) - wl.row_ptr[owner])
+    exp_col[old_pos] = wl.col
+    if wl.reciprocal:
+        order = np.lexsort((nids, js))
+        js_s, nid_s = js[order], nids[order]
+        rank = np.arange(js_s.size) - np.searchsorted(js_s, js_s, side="left")
+        exp_col[exp_rp[js_s] + orig_len[js_s] + rank] = nid_s
+    exp_col[fwd_pos] = js
+    assert (exp_col >= 0).all()
+    bad = np.nonzero(col != exp_col)[0]
+    assert bad.size == 0, f"{bad.size} CSR columns differ, first at edge {bad[:5]}"
+    assert (aff[old_pos] == wl.aff).all(), "old edges' logits changed"
+    if swaps == 0 and "row_ptr" in ref:
+        assert (ref["row_ptr"] == rp).all() and (ref["col"] == col).all()
+        assert np.allclose(aff, ref["aff"], rtol=1e-5, atol=1e-5)
+    return swaps
 
 
 def oracle_free_widen(h):

@@ -5,7 +5,7 @@ import pytest
 
 import synth
 from _parity import (assert_retrieval_parity, assert_scoped_parity, check_update, gpu_retrieve,
-                     gpu_store, oracle_retrieve, oracle_weights)
+                     gpu_store, oracle_retrieve, oracle_retrieve_rows, oracle_weights)
 
 pytestmark = pytest.mark.gpu
 
@@ -114,6 +114,29 @@ def test_last_hop_row_bounds_change_nothing(hops, k, monkeypatch):
         assert np.array_equal(full[key], pruned[key]), key
     np.testing.assert_allclose(pruned["scores"], full["scores"], rtol=1e-5, atol=0)
     assert_retrieval_parity(wl, "clustered", pruned, oracle_retrieve(wl, "clustered"))
+
+
+@pytest.mark.parametrize("hops", [0, 1, 2])
+def test_unfused_selection_switch(hops, monkeypatch):
+    """AKASHIC_FUSE_FILTER=0 (the measurement switch that writes the last
+    slab and selects from it in a separate pass, and with no hops leaves the
+    score GEMM unfiltered) against the oracle (gmm1m recipe at N = 16384)."""
+    import dataclasses
+    wl = dataclasses.replace(synth.workload(2, scale=1 / 64), hops=hops)
+    monkeypatch.setenv("AKASHIC_FUSE_FILTER", "0")
+    _, got = gpu_retrieve(wl, "random")
+    assert_retrieval_parity(wl, "random", got, oracle_retrieve(wl, "random"))
+
+
+def test_full_transpose_switch_after_update(monkeypatch):
+    """AKASHIC_FULL_TRANSPOSE=1 (the measurement switch that rebuilds the
+    in-edge transpose by radix sort after an update instead of patching
+    it): the update's whole CSR against the oracle, then retrieval on the
+    updated store against the oracle."""
+    monkeypatch.setenv("AKASHIC_FULL_TRANSPOSE", "1")
+    wl = synth.workload(3, scale=1 / 64)
+    store = check_update(wl)
+    _retrieval_on_store(wl, store, [wl.new_emb.shape[0]])
 
 
 def test_score_filter_overflow_falls_back():
@@ -431,19 +454,87 @@ def gmm1m():
     return synth.workload(2)
 
 
-def test_gmm1m_full_size_sampled(gmm1m):
-    """N=1,048,576, d=1024, B=256, two hops, k=32: the whole batch runs in the
-    launch configuration the benchmark times; the oracle recomputes a seeded
-    sample of 3 queries one by one."""
+@pytest.mark.parametrize("placement", ["clustered", "random"])
+def test_gmm1m_full_size_sampled(gmm1m, placement):
+    """N=1,048,576, d=1024, B=256, two hops, k=32, both placements (the
+    co-retrieval-clustered and the random page table): the whole batch runs
+    in the launch configuration the benchmark times; the oracle recomputes a
+    seeded sample of 3 queries."""
     wl = gmm1m
-    _, got = gpu_retrieve(wl, "clustered")
+    _, got = gpu_retrieve(wl, placement)
     rows = [0, 97, 255]
-    ref = oracle_retrieve(wl, "clustered", queries=wl.queries[rows])
+    ref = oracle_retrieve_rows(wl, placement, rows)
     sub = {k: v[rows] for k, v in got.items()}
-    assert_retrieval_parity(wl, "clustered", sub, ref)
+    assert_retrieval_parity(wl, placement, sub, ref)
     # properties at any size: page counts within [ceil(k/P), k]
     assert (got["n_pages"] >= int(np.ceil(wl.k / wl.chunks_per_page))).all()
     assert (got["n_pages"] <= wl.k).all()
+
+
+def test_gmm65k_full_size():
+    """The gmm65k workload at its stated size: N=65,536, d=768, exact top-16
+    cosine graph, B=64 queries near mixture centres, one hop, alpha=0.5,
+    k=16, 32 chunks per page by component; every query against the oracle."""
+    wl = synth.workload(1)
+    assert wl.n == 65536 and wl.n_queries == 64
+    _, got = gpu_retrieve(wl, "component")
+    ref = oracle_retrieve_rows(wl, "component", range(wl.n_queries))
+    assert_retrieval_parity(wl, "component", got, ref)
+
+
+def _streams_retrieve(wl, store, placement, per_stream, seed):
+    """The workload's queries as its streams of equal slices, issued in the
+    seeded arrival order and all in flight at once (each stream has its own
+    scratch); returns the sampled rows (per_stream per stream) with their
+    outputs, after checking every stream's page counts in [1, k]."""
+    import torch
+    per = wl.n_queries // wl.streams
+    streams = [torch.cuda.Stream() for _ in range(wl.streams)]
+    outs = {}
+    for i in wl.stream_order:
+        q = torch.from_numpy(np.ascontiguousarray(wl.queries[i * per:(i + 1) * per]).view(np.int16)).cuda()
+        torch.cuda.current_stream().synchronize()
+        outs[i] = store.retrieve(q, wl.k, wl.alpha, wl.hops, stream=streams[i]) + (q,)
+    torch.cuda.synchronize()
+    store.sync()
+    rng = np.random.default_rng(seed)
+    rows = []
+    got = {"ids": [], "scores": [], "page_ids": [], "n_pages": []}
+    for i in range(wl.streams):
+        ids, sc, pg, npg, _ = outs[i]
+        for r in sorted(rng.choice(per, size=per_stream, replace=False)):
+            rows.append(i * per + r)
+            got["ids"].append(ids[r].cpu().numpy())
+            got["scores"].append(sc[r].cpu().numpy())
+            got["page_ids"].append(pg[r].cpu().numpy())
+            got["n_pages"].append(int(npg[r]))
+        assert (npg.cpu().numpy() <= wl.k).all()
+        assert (npg.cpu().numpy() >= 1).all()
+    return rows, {k: np.array(v) for k, v in got.items()}
+
+
+@pytest.mark.parametrize("placement", ["clustered", "random"])
+def test_gmm4m_full_size_streams_sampled(placement):
+    """The gmm4m workload at its stated size: N=4,194,304, d=768,
+    16384-component mixture, 32-neighbour graph, 1024 queries as 8 streams
+    of 128 in the seeded arrival order, two hops, alpha=0.4, k=64, 64 chunks
+    per page; 2 sampled queries per stream against the oracle."""
+    wl = _gmm4m()
+    assert wl.n == 4194304 and wl.n_queries == 1024 and wl.streams == 8
+    store = gpu_store(wl, placement)
+    rows, got = _streams_retrieve(wl, store, placement, 2, seed=11)
+    store.close()
+    ref = oracle_retrieve_rows(wl, placement, rows)
+    assert_retrieval_parity(wl, placement, got, ref)
+
+
+_GMM4M = []
+
+
+def _gmm4m():
+    if not _GMM4M:
+        _GMM4M.append(synth.workload(4))
+    return _GMM4M[0]
 
 
 # --------------------------------------------------------------------------- relation update
@@ -583,44 +674,36 @@ def update_full():
     return synth.workload(3)
 
 
-def test_update_full_size_sampled(update_full):
+def test_update_full_size_whole_csr(update_full):
     """4096 new chunks linked into the N=1,048,576 store in one call (the
-    benchmark's update); the oracle recomputes 4 seeded new chunks (their
-    top-32 among all prior chunks, logits, reciprocal edges)."""
-    check_update(update_full, sample=4)
+    benchmark's update), and the whole exported CSR (every row's pointers,
+    columns and logits) against the oracle's: its top-32 of every new chunk
+    is stored in tests/golden/update_gmm1m_top32.npz by
+    tests/golden/make_update_golden.py (oracle/ only), with the SHA-256 of
+    the inputs it was computed on, checked here first."""
+    import os
+    path = os.path.join(os.path.dirname(__file__), "golden", "update_gmm1m_top32.npz")
+    g = np.load(path)
+    import importlib.util
+    spec = importlib.util.spec_from_file_location(
+        "make_update_golden", os.path.join(os.path.dirname(__file__), "golden",
+                                           "make_update_golden.py"))
+    mk = importlib.util.module_from_spec(spec)
+    spec.loader.exec_module(mk)
+    wl = update_full
+    assert str(g["inputs_sha256"]) == mk.input_digest(wl), "generated inputs differ from the golden's"
+    assert int(g["n_old"]) == wl.n and int(g["top_m"]) == wl.top_m
+    check_update(wl, golden={"nbr_ids": g["nbr_ids"], "nbr_cos": g["nbr_cos"]})
 
 
 def test_gmm4m_recipe_eight_concurrent_streams():
     """gmm4m recipe at N=65536 (d=768, k=64, alpha=0.4): 1024 queries issued
     as 8 streams of 128 in the seeded arrival order, all in flight at once
     (each stream has its own scratch); 2 sampled queries per stream against
-    the oracle, and every stream's page counts within [ceil(k/P), k]."""
-    import torch
+    the oracle, and every stream's page counts within [1, k]."""
     wl = synth.workload(4, scale=1 / 64)
     store = gpu_store(wl, "clustered")
-    per = wl.n_queries // wl.streams
-    streams = [torch.cuda.Stream() for _ in range(wl.streams)]
-    outs = {}
-    for i in wl.stream_order:
-        q = torch.from_numpy(np.ascontiguousarray(wl.queries[i * per:(i + 1) * per]).view(np.int16)).cuda()
-        torch.cuda.current_stream().synchronize()
-        outs[i] = store.retrieve(q, wl.k, wl.alpha, wl.hops, stream=streams[i]) + (q,)
-    torch.cuda.synchronize()
-    store.sync()
-    rng = np.random.default_rng(7)
-    rows = []
-    got = {"ids": [], "scores": [], "page_ids": [], "n_pages": []}
-    for i in range(wl.streams):
-        ids, sc, pg, npg, _ = outs[i]
-        for r in sorted(rng.choice(per, size=2, replace=False)):
-            rows.append(i * per + r)
-            got["ids"].append(ids[r].cpu().numpy())
-            got["scores"].append(sc[r].cpu().numpy())
-            got["page_ids"].append(pg[r].cpu().numpy())
-            got["n_pages"].append(int(npg[r]))
-        assert (npg.cpu().numpy() <= wl.k).all()
-        assert (npg.cpu().numpy() >= 1).all()
-    got = {k: np.array(v) for k, v in got.items()}
+    rows, got = _streams_retrieve(wl, store, "clustered", 2, seed=7)
     ref = oracle_retrieve(wl, "clustered", queries=wl.queries[rows])
     assert_retrieval_parity(wl, "clustered", got, ref)
 
