@@ -86,13 +86,22 @@ struct StreamScratch {
     DevBuf rmax_u, rmin_u;       // u's row maxima / minima over the real queries
     DevBuf ub, lb, ext, pfloor;  // the last hop's row bounds, extremes, floor
     DevBuf skip_split, skip_slot, kept_rows, kept_count, kept_segs, kflag, kpos, ktmp;
-    DevBuf reach_keep, reach_bad, reach_part;
-    // packed coefficients of the last flagged candidates, and their key
-    DevBuf coefK;
+    DevBuf reach_keep, reach_bad, reach_part, reach_plan;
+    DevBuf nsf;                  // scoped last hop: tags, their floors, their count
+    // every candidate's combined coefficients (bf16 hi, lo), and their key
+    DevBuf coef_hi, coef_lo;
     uint64_t coef_build = ~0ull;
     float coef_alpha = -1.f;
-    int coef_bp = 0;
-    ReachSlots coef_slots{};
+    int coef_H = 0;
+    int64_t coef_n = -1;
+    // the call's plan read back: pinned host words and the event after
+    // their copy (the host waits for that point only)
+    int32_t *plan_host = nullptr;
+    cudaEvent_t plan_ev = nullptr;
+    ~StreamScratch() {
+        if (plan_host) cudaFreeHost(plan_host);
+        if (plan_ev) cudaEventDestroy(plan_ev);
+    }
 };
 
 struct ProfRec {
@@ -1317,8 +1326,6 @@ static akashic_status_t retrieve_impl(akashic_mem *m, const uint16_t *q, int32_t
             bool reach_done = false;
             if (prune && eff_hops == 2 && !q_ns && m->reach_on && m->n_split > 0 &&
                 (bp == 256 || bp == 128)) {
-                int bad = -1;
-                int32_t keep[REACH_T] = {0};
                 {
                     PhaseScope ph(m, AKASHIC_PHASE_BOUND, st);
                     {
@@ -1327,6 +1334,10 @@ static akashic_status_t retrieve_impl(akashic_mem *m, const uint16_t *q, int32_t
                     }
                     AK_TRY(sc->reach_keep.ensure(REACH_T * 4));
                     AK_TRY(sc->reach_bad.ensure(16));
+                    AK_TRY(sc->reach_plan.ensure(REACH_PLAN_INTS * 4));
+                    if (!sc->plan_host) CUDA_TRY(cudaMallocHost((void **)&sc->plan_host, 16));
+                    if (!sc->plan_ev)
+                        CUDA_TRY(cudaEventCreateWithFlags(&sc->plan_ev, cudaEventDisableTiming));
                     const int64_t n_lb = m->n_split < 1024 ? m->n_split : 1024;
                     CUDA_TRY(launch_prune_floor(nullptr, 0, row_lb, hp.split_row, hp.split_order,
                                                 n_lb, k, sc->pfloor.as<float>(), st));
@@ -1334,39 +1345,48 @@ static akashic_status_t retrieve_impl(akashic_mem *m, const uint16_t *q, int32_t
                                                 m->reach_map.as<int32_t>(), n,
                                                 sc->reach_keep.as<int32_t>(),
                                                 sc->reach_bad.as<int>(), st));
-                    CUDA_TRY(cudaMemcpyAsync(&bad, sc->reach_bad.p, 4, cudaMemcpyDeviceToHost, st));
-                    CUDA_TRY(cudaMemcpyAsync(keep, sc->reach_keep.p, sizeof keep,
+                    CUDA_TRY(launch_reach_plan(sc->reach_keep.as<int32_t>(), sc->reach_bad.as<int>(),
+                                               m->reach_t.as<int>(), k,
+                                               sc->reach_plan.as<int32_t>(), st));
+                    CUDA_TRY(cudaMemcpyAsync(sc->plan_host, sc->reach_plan.p, 8,
                                              cudaMemcpyDeviceToHost, st));
-                    CUDA_TRY(cudaStreamSynchronize(st));
-                    ph.launches += 2;
+                    CUDA_TRY(cudaEventRecord(sc->plan_ev, st));
+                    ph.launches += 3;
                 }
-                ReachSlots rs{};
-                for (int t = 0; t < REACH_T; ++t)
-                    if (keep[t]) rs.slot[rs.nk++] = t;
-                if (bad == 0 && m->reach_T >= k && rs.nk >= k && reach_fits(bp, rs.nk)) {
+                {
+                    // The candidates' pass is queued before the host learns the
+                    // plan (its kernels return at once when the plan says the
+                    // hops run), so the GPU goes on while the host waits.
                     PhaseScope ph(m, AKASHIC_PHASE_LAST_HOP, st);
                     AK_TRY(sc->reach_part.ensure((size_t)reach_parts() * REACH_T * bp * 4));
-                    // packed coefficients, kept while the graph, alpha and the
-                    // flagged candidates stay the same
-                    bool same = sc->coef_build == m->reach_build && sc->coef_alpha == alpha &&
-                                sc->coef_bp == bp && sc->coef_slots.nk == rs.nk;
-                    for (int i = 0; same && i < rs.nk; ++i) same = sc->coef_slots.slot[i] == rs.slot[i];
-                    if (!same) {
-                        AK_TRY(sc->coefK.ensure(reach_coef_floats(n, bp, rs.nk) * 4));
-                        CUDA_TRY(launch_reach_coef(m->reach_c.as<float>(), n, eff_hops, alpha, rs,
-                                                   bp, sc->coefK.as<float>(), st));
+                    // every candidate's packed coefficients, kept while the
+                    // graph, alpha and the hop count stay the same
+                    if (sc->coef_build != m->reach_build || sc->coef_alpha != alpha ||
+                        sc->coef_H != eff_hops || sc->coef_n != n) {
+                        const size_t cb = (size_t)REACH_T * reach_pad_rows(n) * 2;
+                        AK_TRY(sc->coef_hi.ensure(cb));
+                        AK_TRY(sc->coef_lo.ensure(cb));
+                        CUDA_TRY(launch_reach_pack(m->reach_c.as<float>(), n, eff_hops, alpha,
+                                                   sc->coef_hi.as<uint16_t>(),
+                                                   sc->coef_lo.as<uint16_t>(), st));
                         ph.launches += 1;
-                        sc->coef_bp = bp;
                         sc->coef_build = m->reach_build;
                         sc->coef_alpha = alpha;
-                        sc->coef_slots = rs;
+                        sc->coef_H = eff_hops;
+                        sc->coef_n = n;
                     }
-                    CUDA_TRY(launch_reach_scores(sc->u.as<float>(), bp, b, n, sc->coefK.as<float>(),
-                                                 rs, m->reach_rows.as<int32_t>(),
+                    CUDA_TRY(launch_reach_scores(sc->u.as<float>(), bp, b, n,
+                                                 sc->coef_hi.as<uint16_t>(),
+                                                 sc->coef_lo.as<uint16_t>(),
+                                                 sc->reach_plan.as<int32_t>(),
+                                                 m->reach_rows.as<int32_t>(),
                                                  m->ext_of.as<int32_t>(),
                                                  sc->reach_part.as<float>(),
                                                  (unsigned int *)(ws + sp.off_cnt), ws + sp.off_buf,
-                                                 sp.cap, st, &ph.launches));
+                                                 sp.cap, m->status.as<int>(), st, &ph.launches));
+                }
+                CUDA_TRY(cudaEventSynchronize(sc->plan_ev));
+                if (sc->plan_host[0] == 1) {
                     rc = ColumnRecompute{};   // the buffers hold every candidate
                     reach_done = true;
                 }
@@ -1395,9 +1415,25 @@ static akashic_status_t retrieve_impl(akashic_mem *m, const uint16_t *q, int32_t
                                                     q_ns ? nullptr : hp.split_row,
                                                     hp.split_order, n_lb, k,
                                                     sc->pfloor.as<float>(), st));
+                        // with a scope, each namespace of the batch gets its own
+                        // floor (its rows can only be selected by its queries)
+                        NsFloors nf{};
+                        if (q_ns) {
+                            AK_TRY(sc->nsf.ensure(4096));
+                            int32_t *tags = sc->nsf.as<int32_t>();
+                            float *tag_floor = (float *)(tags + PF_TAGS);
+                            int *n_tags = (int *)(tag_floor + PF_TAGS);
+                            CUDA_TRY(launch_ns_floors(ws + sp.off_bound, sc->qns.as<int32_t>(), b,
+                                                      row_lb, m->ns_row.as<int32_t>(),
+                                                      hp.split_row, hp.split_order, m->n_split, k,
+                                                      tags, n_tags, tag_floor, st));
+                            nf = NsFloors{m->ns_row.as<int32_t>(), tags, n_tags, tag_floor};
+                            ps.launches += m->n_split > 0 ? 2 : 1;
+                        }
                         KeptScratch ks{sc->kflag.as<int64_t>(), sc->kpos.as<int64_t>(),
                                        sc->ktmp.p, sc->ktmp.cap};
                         CUDA_TRY(launch_split_flags(hp, row_ub, sc->pfloor.as<float>(),
+                                                    q_ns ? &nf : nullptr,
                                                     sc->skip_split.as<int32_t>(),
                                                     sc->skip_slot.as<int32_t>(),
                                                     sc->kept_rows.as<int32_t>(),

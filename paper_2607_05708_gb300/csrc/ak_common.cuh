@@ -411,10 +411,45 @@ cudaError_t launch_final_bounds(const float *u0, const float *l0, const float *m
                                 const float *mdn, int64_t n, int H, float alpha,
                                 unsigned int *ext, float *ub, float *lb, cudaStream_t st,
                                 int *launches, bool ext_ready = false);
+// Floors of a namespace-scoped last hop: a row can only be selected by the
+// batch's queries of its own namespace, so its floor is that namespace's
+// (tag_floor[i] for tags[i] == its tag; the tags are the batch's distinct
+// query namespaces, ascending), or +inf when no query of the batch has its
+// namespace.  ns_row == NULL: the one device floor applies to every row.
+struct NsFloors {
+    const int32_t *ns_row;    // [n] namespace tag of each row
+    const int32_t *tags;      // [<= PF_TAGS] distinct query tags, ascending
+    const int *n_tags;        // their number (device)
+    const float *tag_floor;   // [<= PF_TAGS]
+};
+constexpr int PF_TAGS = 256;
+__device__ __forceinline__ float row_floor(const NsFloors &f, float floor_, int64_t row) {
+    if (!f.ns_row) return floor_;
+    const int32_t t = f.ns_row[row];
+    int lo = 0, hi = *f.n_tags;
+    while (lo < hi) {
+        const int mid = (lo + hi) >> 1;
+        if (f.tags[mid] < t) lo = mid + 1;
+        else hi = mid;
+    }
+    if (lo < *f.n_tags && f.tags[lo] == t) return fmaxf(floor_, f.tag_floor[lo]);
+    return INFINITY;
+}
+// nf: the per-namespace floors, or NULL (one floor for all rows)
 cudaError_t launch_split_flags(const HopPlan &p, const float *row_ub, const float *floor_p,
-                               int32_t *split_skip, int32_t *slot_skip, int32_t *kept_rows,
-                               int64_t *kept_count, int32_t *kept_segs, KeptScratch &ks,
-                               cudaStream_t st, int *launches);
+                               const NsFloors *nf, int32_t *split_skip, int32_t *slot_skip,
+                               int32_t *kept_rows, int64_t *kept_count, int32_t *kept_segs,
+                               KeptScratch &ks, cudaStream_t st, int *launches);
+// The floors of a scoped batch: tags = the distinct q_ns of the n_real query
+// columns, and for each tag the largest of (a) the smallest score that the
+// filter bound of any of its queries admits and (b) the k-th largest lb over
+// the split rows of that namespace, taken heaviest first (split_order), at
+// most PF_ROWS of them (any subset of a namespace's rows gives a floor that
+// each of its queries' k-th largest final score reaches).
+cudaError_t launch_ns_floors(const unsigned long long *bound, const int32_t *q_ns, int n_real,
+                             const float *lb, const int32_t *ns_row, const int32_t *split_row,
+                             const int32_t *split_order, int64_t n_split, int k, int32_t *tags,
+                             int *n_tags, float *tag_floor, cudaStream_t st);
 // floor = max(the smallest score any real column's filter bound admits,
 // and, if lb_rows != NULL, the k-th largest lb over the rows
 // lb_rows[order[i]], i < n_lb_rows), written to floor_out.  The second term
@@ -450,27 +485,31 @@ cudaError_t launch_reach_build(const ReachBuild &rb, cudaStream_t st);
 // *bad counts the other rows that do (the candidates then do not suffice).
 cudaError_t launch_reach_check(const float *ub, const float *floor_p, const int32_t *map,
                                int64_t n, int32_t *keep, int *bad, cudaStream_t st);
-int reach_parts();                   // CTAs of the score pass (partial rows)
-// The flagged candidates (slots in ascending order), built on the host from
-// the check's flags.
-struct ReachSlots {
-    int32_t slot[REACH_T];
-    int nk;
-};
-// The flagged candidates' combined coefficients sum_t alpha^t C_t, packed
-// [n][nk rounded up to 8] (reach_coef_floats floats).
-size_t reach_coef_floats(int64_t n, int bp, int nk);
-cudaError_t launch_reach_coef(const float *C, int64_t n, int H, float alpha, const ReachSlots &rs,
-                              int bp, float *coefK, cudaStream_t st);
-// partial: [reach_parts()][REACH_T][bp] scratch; the flagged candidates'
-// keys are written to each real column's buffer (cnt[b] = their number).
-// Needs bp = 256 with at most 64 flagged candidates, or bp = 128 with at
-// most 128 (reach_fits).
-bool reach_fits(int bp, int nk);
-cudaError_t launch_reach_scores(const float *u, int bp, int B, int64_t n, const float *coefK,
-                                const ReachSlots &rs, const int32_t *rows, const int32_t *ext_of,
-                                float *partial, unsigned int *cnt, unsigned long long *buf,
-                                int64_t cap, cudaStream_t st, int *launches);
+int reach_parts();                   // CTAs of the candidates' pass (partial rows)
+// The call's plan on the device (int32[REACH_PLAN_INTS]): plan[0] = 1 when
+// the flagged candidates suffice for top-k (else the hops run), plan[1] =
+// their number nk, plan[2..] their slots in ascending order,
+// plan[REACH_PLAN_WIDE] = 1 when a flagged slot is 64 or above.
+constexpr int REACH_PLAN_WIDE = REACH_T + 2;
+constexpr int REACH_PLAN_INTS = REACH_T + 3;
+cudaError_t launch_reach_plan(const int32_t *keep, const int *bad, const int *t_cnt, int k,
+                              int32_t *plan, cudaStream_t st);
+// Rows of the packed coefficients: n rounded up to a whole 64-row stage.
+int64_t reach_pad_rows(int64_t n);
+// Every candidate's combined coefficients sum_t alpha^t C_t as bf16 hi + lo,
+// [REACH_T][reach_pad_rows(n)] each (graph-only; repacked when the graph,
+// alpha or H change).
+cudaError_t launch_reach_pack(const float *C, int64_t n, int H, float alpha, uint16_t *coef_hi,
+                              uint16_t *coef_lo, cudaStream_t st);
+// partial: [reach_parts()][REACH_T][bp] scratch; with plan[0] = 1 the
+// flagged candidates' keys are written to each real column's buffer
+// (cnt[b] = nk); with plan[0] = 0 both kernels return at once.  bp = 128
+// or 256.
+cudaError_t launch_reach_scores(const float *u, int bp, int B, int64_t n, const uint16_t *coef_hi,
+                                const uint16_t *coef_lo, const int32_t *plan, const int32_t *rows,
+                                const int32_t *ext_of, float *partial, unsigned int *cnt,
+                                unsigned long long *buf, int64_t cap, int *status, cudaStream_t st,
+                                int *launches);
 // slot_split[s] = r for every partial slot s of split row r.
 cudaError_t launch_slot_owner(const int64_t *split_slot0, int64_t n_split, int32_t *slot_split,
                               cudaStream_t st);

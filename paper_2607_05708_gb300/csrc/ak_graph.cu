@@ -882,12 +882,14 @@ __global__ void k_split_bound(const int64_t *__restrict__ in_ptr, int64_t n_spli
 __global__ void k_split_flags(int64_t n_split, const int32_t *__restrict__ split_row,
                               const int64_t *__restrict__ split_slot0,
                               const float *__restrict__ row_ub, const float *__restrict__ floor_p,
-                              int32_t *__restrict__ split_skip, int32_t *__restrict__ slot_skip) {
+                              const NsFloors nf, int32_t *__restrict__ split_skip,
+                              int32_t *__restrict__ slot_skip) {
     const float floor_ = *floor_p;
     const int lane = threadIdx.x & 31;
     const int64_t nw = ((int64_t)gridDim.x * blockDim.x) >> 5;
     for (int64_t r = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5; r < n_split; r += nw) {
-        const int32_t skip = row_ub[split_row[r]] < floor_ ? 1 : 0;
+        const int32_t j = split_row[r];
+        const int32_t skip = row_ub[j] < row_floor(nf, floor_, j) ? 1 : 0;
         if (lane == 0) split_skip[r] = skip;
         for (int64_t s = split_slot0[r] + lane; s < split_slot0[r + 1]; s += 32) slot_skip[s] = skip;
     }
@@ -1029,11 +1031,11 @@ cudaError_t launch_final_bounds(const float *u0, const float *l0, const float *m
 // that keeps gathered source rows in L2).
 __global__ void k_keep_rows(const int64_t *__restrict__ in_ptr, int64_t n, int64_t split_t,
                             const float *__restrict__ row_ub, const float *__restrict__ floor_p,
-                            int64_t *__restrict__ flag) {
+                            const NsFloors nf, int64_t *__restrict__ flag) {
     const float floor_ = *floor_p;
     for (int64_t j = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; j < n;
          j += (int64_t)gridDim.x * blockDim.x)
-        flag[j] = in_ptr[j + 1] - in_ptr[j] <= split_t && row_ub[j] >= floor_;
+        flag[j] = in_ptr[j + 1] - in_ptr[j] <= split_t && row_ub[j] >= row_floor(nf, floor_, j);
 }
 __global__ void k_keep_segs(const int32_t *__restrict__ seg_slot, int64_t n_segs,
                             const int32_t *__restrict__ slot_skip, int64_t *__restrict__ flag) {
@@ -1050,19 +1052,20 @@ __global__ void k_compact_kept(const int64_t *__restrict__ flag, const int64_t *
 }
 
 cudaError_t launch_split_flags(const HopPlan &p, const float *row_ub, const float *floor_p,
-                               int32_t *split_skip, int32_t *slot_skip, int32_t *kept_rows,
-                               int64_t *kept_count, int32_t *kept_segs, KeptScratch &ks,
-                               cudaStream_t st, int *launches) {
+                               const NsFloors *nf, int32_t *split_skip, int32_t *slot_skip,
+                               int32_t *kept_rows, int64_t *kept_count, int32_t *kept_segs,
+                               KeptScratch &ks, cudaStream_t st, int *launches) {
     const int sms = device_sm_count();
+    const NsFloors f = nf ? *nf : NsFloors{};
     if (p.n_split_rows > 0) {
         const int64_t want = ceil_div<int64_t>(p.n_split_rows, 8);
         const int g = (int)(want < (int64_t)sms * 4 ? want : (int64_t)sms * 4);
         k_split_flags<<<g, 256, 0, st>>>(p.n_split_rows, p.split_row, p.split_slot0, row_ub,
-                                         floor_p, split_skip, slot_skip);
+                                         floor_p, f, split_skip, slot_skip);
     }
     if (launches && p.n_split_rows > 0) *launches += 1;
     // kept_count[0]: rows, kept_count[1]: segments
-    k_keep_rows<<<sms * 4, 256, 0, st>>>(p.in_ptr, p.n, p.split.split_t, row_ub, floor_p,
+    k_keep_rows<<<sms * 4, 256, 0, st>>>(p.in_ptr, p.n, p.split.split_t, row_ub, floor_p, f,
                                          ks.flag);
     cudaError_t e = scan_exclusive(ks.flag, ks.pos, p.n, ks.tmp, ks.tmp_bytes, st, launches);
     if (e != cudaSuccess) return e;

@@ -11,7 +11,10 @@
 // final scores for every query come from one pass over the score slab u,
 // and the hops are not run.  The selection is the same as the hops' (the
 // values differ only by fp32 summation order).
+#include <cuda_bf16.h>
+
 #include "ak_common.cuh"
+#include "ak_sm100.cuh"
 
 namespace ak {
 
@@ -132,152 +135,364 @@ __global__ void k_reach_check(const float *__restrict__ ub, const float *__restr
     if (nb) atomicAdd(bad, nb);
 }
 
-// The flagged candidates' combined coefficients, contiguous:
-// coefK[k][i] = sum_t alpha^t C_t[k][slot_i] for i < nk, 0 up to NK8.
-__global__ void k_reach_coef(const float *__restrict__ C, int64_t n, int H, float alpha,
-                             const ReachSlots rs, int nk8, float *__restrict__ coefK) {
-    for (int64_t x = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; x < n * nk8;
-         x += (int64_t)gridDim.x * blockDim.x) {
-        const int64_t k = x / nk8;
-        const int i = (int)(x - k * nk8);
-        float c = 0.f;
-        if (i < rs.nk) {
-            const int64_t at = k * REACH_T + rs.slot[i];
-            for (int t = H; t >= 1; --t) c = alpha * (c + C[(int64_t)(t - 1) * n * REACH_T + at]);
-        }
-        coefK[x] = c;
+// The plan of a call, on the device: plan[0] = 1 when the candidates
+// suffice (no other row reaches the floor, at least k of them do, and at
+// least k candidates exist), else 0 and the hops run; plan[1] = nk, the
+// flagged count; plan[2 .. 2 + nk) the flagged slots in ascending order;
+// plan[REACH_PLAN_WIDE] = 1 when one of them is 64 or above.  One CTA of
+// REACH_T threads.
+__global__ __launch_bounds__(REACH_T) void k_reach_plan(const int32_t *__restrict__ keep,
+                                                        const int *__restrict__ bad,
+                                                        const int *__restrict__ t_cnt, int k,
+                                                        int32_t *__restrict__ plan) {
+    __shared__ int pre[REACH_T];
+    const int t = threadIdx.x;
+    const int f = keep[t] != 0 ? 1 : 0;
+    pre[t] = f;
+    __syncthreads();
+    for (int o = 1; o < REACH_T; o <<= 1) {          // inclusive scan
+        const int v = t >= o ? pre[t - o] : 0;
+        __syncthreads();
+        pre[t] += v;
+        __syncthreads();
+    }
+    if (f) plan[2 + pre[t] - 1] = t;
+    if (t == REACH_T - 1) {
+        const int nk = pre[t];
+        plan[1] = nk;
+        plan[0] = (*bad == 0 && nk >= k && *t_cnt >= k) ? 1 : 0;
+        // a flagged slot in the upper half: the candidates' pass loads all
+        // 128 coefficient rows, else the first 64
+        plan[REACH_PLAN_WIDE] = nk - pre[REACH_T / 2 - 1] > 0 ? 1 : 0;
     }
 }
 
-__device__ __forceinline__ void cp_async16(void *dst, const void *src) {
-    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(
-                     (uint32_t)__cvta_generic_to_shared(dst)),
-                 "l"(src)
-                 : "memory");
-}
-__device__ __forceinline__ void cp_async_commit() {
-    asm volatile("cp.async.commit_group;" ::: "memory");
-}
-template <int N>
-__device__ __forceinline__ void cp_async_wait() {
-    asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
+// ------------------------------------------------------------------ tensor-core terms
+// partial[cta][i][b] = sum over the CTA's rows k of coef[k][i] u[k][b] for
+// every candidate slot i, on tcgen05 with split-bf16 operands:
+//   coef = A_hi + A_lo,  u = B_hi + B_lo  (each lo the bf16 rounding of the
+//   rest, so hi + lo holds 16 significant bits),
+//   coef u ~= A_hi B_hi + A_hi B_lo + A_lo B_hi,
+// three MMAs per 16-row slice into an fp32 accumulator in TMEM (the
+// dropped A_lo B_lo term is below 2^-16 of the product).
+//   A = the combined coefficients sum_t alpha^t C_t, packed by
+//       k_reach_pack as [REACH_T slots][n_pad rows] bf16 (hi, lo), loaded
+//       by TMA as K-major tiles [128 slots][64 rows] in the 128-byte swizzle;
+//   B = u, loaded by converter warps from global memory (two float4 of one
+//       row per lane, one row per warp instruction), split into hi / lo and
+//       stored as MN-major tiles [64 rows][BP queries]: atoms of 8 rows x 64
+//       queries (128 bytes a row, 16-byte chunks swizzled by the row), four
+//       (BP = 256) or two such atom columns RM_BK * 128 bytes apart.
+// D[slot][query] (M = 128 slots = TMEM lanes, N = BP queries = columns).
+// The tensor core's accumulation of many positive terms drifts (each add
+// into the fp32 accumulator may round the same way), so an accumulator
+// takes only RM_CHUNK stages (1024 rows, 192 MMAs): two accumulators
+// alternate, and the converter warps add each finished one into the CTA's
+// partial with ordinary round-to-nearest fp32 adds (the partial rows stay
+// in L2) while the MMAs fill the other.
+// Warps: 0 TMA producer (A), 1 MMA issuer, 2..9 converters (and the flush:
+// warp w reads TMEM lanes 32 (w % 4) .., column half (w - 2) / 4).  Each
+// CTA takes a contiguous range of 64-row stages; 2 stages of 2 A + 2 B
+// tiles.
+constexpr int RM_BK = 64;                // store rows (K) per stage
+constexpr int RM_M = REACH_T;            // candidate slots (M)
+constexpr int RM_STAGES = 2;
+constexpr int RM_CONV_W = 8;             // converter warps
+constexpr int RM_THREADS = 64 + 32 * RM_CONV_W;
+constexpr int RM_CHUNK = 16;             // stages per accumulator
+
+template <int BP>
+struct RmCfg {
+    static constexpr int A_BYTES = RM_M * RM_BK * 2;             // one of hi / lo
+    static constexpr int B_BYTES = BP * RM_BK * 2;               // one of hi / lo
+    static constexpr int STAGE_BYTES = 2 * A_BYTES + 2 * B_BYTES;
+    static constexpr uint32_t LBO = RM_BK * 128;                 // between query atoms
+    static constexpr uint32_t SBO = 8 * 128;                     // between 8-row groups
+    static constexpr int SMEM = 1024 + RM_STAGES * STAGE_BYTES + 256;
+    static constexpr int CH = BP / 8;        // 16-byte bf16 chunks of a u row
+    static constexpr int RPI = 32 / CH;      // u rows per warp instruction
+    static constexpr int ITEMS = 8 / RPI;    // (row, chunk) items per lane per stage
+    static constexpr int TMEM_COLS = 2 * BP; // two accumulators
+    static_assert(BP == 128 || BP == 256, "query widths 128 and 256");
+    static_assert(SMEM <= 227 * 1024, "shared memory");
+};
+
+__device__ __forceinline__ uint32_t split_bf16_pair(float x, float y, uint32_t &lo) {
+    const __nv_bfloat16 hx = __float2bfloat16_rn(x), hy = __float2bfloat16_rn(y);
+    const __nv_bfloat16 lx = __float2bfloat16_rn(x - __bfloat162float(hx));   // exact rest
+    const __nv_bfloat16 ly = __float2bfloat16_rn(y - __bfloat162float(hy));
+    lo = (uint32_t)__bfloat16_as_ushort(lx) | ((uint32_t)__bfloat16_as_ushort(ly) << 16);
+    return (uint32_t)__bfloat16_as_ushort(hx) | ((uint32_t)__bfloat16_as_ushort(hy) << 16);
 }
 
-// partial[cta][i][b] = sum over this CTA's rows k of coefK[k][i] u[k][b]
-// (BP = 256 or 128 columns of u).  REACH_T_THREADS threads: thread t takes
-// columns 4 (t % (BP/4)) + 0..3 and one of G = 512 / BP slot groups
-// (t / (BP/4)), so that one shared load of four coefficients feeds sixteen
-// FMAs; REACH_ROWS rows at a time are copied to shared memory (u rows and
-// coefficient rows) with cp.async, double-buffered so that the next rows
-// load while these are summed; rows in order.
-constexpr int REACH_ROWS = 32;
-constexpr int REACH_T_THREADS = 128;
+template <int BP>
+__global__ __launch_bounds__(RM_THREADS, 1) void k_reach_mma(
+    const __grid_constant__ CUtensorMap tmAhi, const __grid_constant__ CUtensorMap tmAlo,
+    const __grid_constant__ CUtensorMap tmAhi64, const __grid_constant__ CUtensorMap tmAlo64,
+    const float *__restrict__ u, int64_t n, const int32_t *__restrict__ plan,
+    float *__restrict__ partial, int *status) {
+    using C = RmCfg<BP>;
+    if (plan[0] == 0) return;                          // the hops run instead
+    // every flagged slot below 64: only the first 64 coefficient rows are
+    // loaded (rows 64..127 of the A tiles keep whatever they hold, and
+    // the accumulator rows they feed are never read)
+    const bool wide = plan[REACH_PLAN_WIDE] != 0;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *smem = (uint8_t *)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+    uint64_t *afull = (uint64_t *)(smem + RM_STAGES * C::STAGE_BYTES);
+    uint64_t *bfull = afull + RM_STAGES;              // RM_CONV_W arrivals
+    uint64_t *empty = bfull + RM_STAGES;              // the MMAs' commit
+    uint64_t *dfull = empty + RM_STAGES;              // [2] accumulator complete
+    uint64_t *dfree = dfull + 2;                      // [2] accumulator flushed (RM_CONV_W)
+    uint32_t *tmem_slot = (uint32_t *)(dfree + 2);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    auto a_hi = [&](int s) { return smem + s * C::STAGE_BYTES; };
+    auto a_lo = [&](int s) { return smem + s * C::STAGE_BYTES + C::A_BYTES; };
+    auto b_hi = [&](int s) { return smem + s * C::STAGE_BYTES + 2 * C::A_BYTES; };
+    auto b_lo = [&](int s) { return smem + s * C::STAGE_BYTES + 2 * C::A_BYTES + C::B_BYTES; };
 
-template <int NK, int BP>
-__global__ __launch_bounds__(REACH_T_THREADS, 2) void k_reach_terms(
-    const float *__restrict__ u, int64_t n, const float *__restrict__ coefK, int nk,
-    float *__restrict__ partial) {
-    extern __shared__ __align__(16) float dyn[];
-    constexpr int TT = REACH_T_THREADS;
-    constexpr int G = TT / (BP / 4);                   // slot groups (= 512 / BP)
-    constexpr int HALF = NK / G;                       // slots per thread
-    static_assert(G * (BP / 4) == TT, "every thread one column quad and one slot group");
-    static_assert(HALF % 4 == 0, "four coefficients per shared load");
-    float *us = dyn;                                   // [2][REACH_ROWS][BP]
-    float *cs = dyn + 2 * REACH_ROWS * BP;             // [2][REACH_ROWS][NK]
-    const int cg = threadIdx.x % (BP / 4), sg = threadIdx.x / (BP / 4);
-    const int64_t per = (n + gridDim.x - 1) / gridDim.x;
-    const int64_t k0 = (int64_t)blockIdx.x * per;
-    const int64_t k1 = k0 + per < n ? k0 + per : n;
-    const int64_t n_chunks = (k1 - k0 + REACH_ROWS - 1) / REACH_ROWS;
-    auto stage = [&](int64_t c, int buf) {
-        const int64_t kb = k0 + c * REACH_ROWS;
-        const int rows = (int)(k1 - kb < REACH_ROWS ? k1 - kb : REACH_ROWS);
-        float *ud = us + buf * REACH_ROWS * BP;
-        float *cd = cs + buf * REACH_ROWS * NK;
-        // u rows: rows x BP/4 pieces of 16 bytes; coefficient rows: rows x NK/4
-        for (int x = threadIdx.x; x < rows * (BP / 4); x += TT)
-            cp_async16(ud + x * 4, u + kb * BP + (int64_t)x * 4);
-        for (int x = threadIdx.x; x < rows * (NK / 4); x += TT)
-            cp_async16(cd + x * 4, coefK + kb * NK + (int64_t)x * 4);
-        cp_async_commit();
-    };
-    float acc[HALF][4];
-#pragma unroll
-    for (int i = 0; i < HALF; ++i) acc[i][0] = acc[i][1] = acc[i][2] = acc[i][3] = 0.f;
-    if (n_chunks > 0) stage(0, 0);
-    for (int64_t c = 0; c < n_chunks; ++c) {
-        const int buf = (int)(c & 1);
-        if (c + 1 < n_chunks) {
-            stage(c + 1, buf ^ 1);
-            cp_async_wait<1>();
-        } else {
-            cp_async_wait<0>();
+    const int64_t stages_total = (n + RM_BK - 1) / RM_BK;
+    const int64_t per = (stages_total + gridDim.x - 1) / gridDim.x;
+    const int64_t s0 = (int64_t)blockIdx.x * per;
+    const int64_t s1 = s0 + per < stages_total ? s0 + per : stages_total;
+    const int64_t ns = s1 > s0 ? s1 - s0 : 0;
+    const int64_t n_chunks = (ns + RM_CHUNK - 1) / RM_CHUNK;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < RM_STAGES; ++s) {
+            mbar_init(&afull[s], 1);
+            mbar_init(&bfull[s], RM_CONV_W);
+            mbar_init(&empty[s], 1);
         }
-        __syncthreads();
-        const int64_t kb = k0 + c * REACH_ROWS;
-        const int rows = (int)(k1 - kb < REACH_ROWS ? k1 - kb : REACH_ROWS);
-        const float *ud = us + buf * REACH_ROWS * BP;
-        const float *cd = cs + buf * REACH_ROWS * NK;
-#pragma unroll 2
-        for (int r = 0; r < rows; ++r) {
-            const float4 x = *reinterpret_cast<const float4 *>(ud + r * BP + 4 * cg);
-            const float4 *c4 = reinterpret_cast<const float4 *>(cd + r * NK + sg * HALF);
+        for (int a = 0; a < 2; ++a) {
+            mbar_init(&dfull[a], 1);
+            mbar_init(&dfree[a], RM_CONV_W);
+        }
+        mbar_fence_init();
+    }
+    if (warp == 1) {
+        tmem_alloc(tmem_slot, C::TMEM_COLS);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem_base = *tmem_slot;
+
+    if (warp == 0) {
+        if (lane == 0 && ns > 0) {
+            // ---------------- TMA producer: A hi / lo [128 slots][64 rows]
+            uint32_t stage = 0, phase = 0;
+            int last_par[RM_STAGES];
+            for (int s = 0; s < RM_STAGES; ++s) last_par[s] = -1;
+            bool ok = true;
+            for (int64_t t = 0; t < ns; ++t) {
+                if (!mbar_wait(&empty[stage], phase ^ 1u, status)) {
+                    ok = false;
+                    break;
+                }
+                mbar_expect_tx(&afull[stage], wide ? 2 * C::A_BYTES : C::A_BYTES);
+                const int kx = (int)((s0 + t) * RM_BK);
+                tma_load_2d(a_hi(stage), wide ? &tmAhi : &tmAhi64, &afull[stage], kx, 0);
+                tma_load_2d(a_lo(stage), wide ? &tmAlo : &tmAlo64, &afull[stage], kx, 0);
+                last_par[stage] = (int)phase;
+                if (++stage == RM_STAGES) {
+                    stage = 0;
+                    phase ^= 1u;
+                }
+            }
+            if (!ok)   // let every copy this thread issued land before the CTA exits
+                for (int s = 0; s < RM_STAGES; ++s)
+                    if (last_par[s] >= 0) mbar_wait(&afull[s], (uint32_t)last_par[s], status);
+        }
+    } else if (warp == 1) {
+        if (lane == 0 && ns > 0) {
+            // ---------------- MMA issuer: three products per 16-row slice
+            const uint32_t idesc = idesc_bf16_m128(BP) | IDESC_B_MN_MAJOR;
+            uint32_t stage = 0, phase = 0;
+            bool ok = true;
+            for (int64_t t = 0; t < ns && ok; ++t) {
+                const int64_t c = t / RM_CHUNK;
+                const int acc = (int)(c & 1);
+                const bool first = t % RM_CHUNK == 0;
+                const bool last = t % RM_CHUNK == RM_CHUNK - 1 || t == ns - 1;
+                // the accumulator is free once the converters flushed its
+                // previous chunk (c - 2)
+                if (first && !mbar_wait(&dfree[acc], (uint32_t)((c >> 1) & 1) ^ 1u, status)) break;
+                if (!mbar_wait(&afull[stage], phase, status) ||
+                    !mbar_wait(&bfull[stage], phase, status)) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+                const uint32_t d = tmem_base + (uint32_t)(acc * BP);
+                const uint64_t ah = sdesc_sw128(smem_u32(a_hi(stage)));
+                const uint64_t al = sdesc_sw128(smem_u32(a_lo(stage)));
+                const uint64_t bh = sdesc_mn_sw128(smem_u32(b_hi(stage)), C::LBO, C::SBO);
+                const uint64_t bl = sdesc_mn_sw128(smem_u32(b_lo(stage)), C::LBO, C::SBO);
 #pragma unroll
-            for (int q = 0; q < HALF / 4; ++q) {
-                const float4 cq = c4[q];
-                const float cv[4] = {cq.x, cq.y, cq.z, cq.w};
-#pragma unroll
-                for (int i = 0; i < 4; ++i) {
-                    acc[4 * q + i][0] = fmaf(cv[i], x.x, acc[4 * q + i][0]);
-                    acc[4 * q + i][1] = fmaf(cv[i], x.y, acc[4 * q + i][1]);
-                    acc[4 * q + i][2] = fmaf(cv[i], x.z, acc[4 * q + i][2]);
-                    acc[4 * q + i][3] = fmaf(cv[i], x.w, acc[4 * q + i][3]);
+                for (int k = 0; k < RM_BK / 16; ++k) {
+                    // A: 16 K values = 32 bytes further along the row; B: two
+                    // 8-row groups further down
+                    const uint64_t ao = (uint64_t)(2 * k), bo = (uint64_t)(2 * C::SBO * k) >> 4;
+                    umma_bf16(d, ah + ao, bh + bo, idesc, (first && k == 0) ? 0u : 1u);
+                    umma_bf16(d, ah + ao, bl + bo, idesc, 1u);
+                    umma_bf16(d, al + ao, bh + bo, idesc, 1u);
+                }
+                umma_commit(&empty[stage]);
+                if (last) umma_commit(&dfull[acc]);
+                if (++stage == RM_STAGES) {
+                    stage = 0;
+                    phase ^= 1u;
                 }
             }
         }
-        __syncthreads();   // this buffer is restaged two chunks later
-    }
+    } else {
+        // ---------------- converters: u rows -> B hi / lo (MN-major)
+        const int cw = warp - 2;
+        const int c8 = lane % C::CH;                  // chunk: queries 8 c8 .. 8 c8 + 7
+        const int rl = lane / C::CH;                  // row within a warp instruction
+        const int q = warp & 3;                       // flush: TMEM lanes 32 q ..
+        const int half = cw >> 2;                     // flush: column half
+        const int slot = q * 32 + lane;
+        float *o = partial + ((int64_t)blockIdx.x * REACH_T + slot) * BP + half * (BP / 2);
+        float4 cur[C::ITEMS][2], nxt[C::ITEMS][2];
+        auto load = [&](int64_t t, float4 (&dst)[C::ITEMS][2]) {
 #pragma unroll
-    for (int i = 0; i < HALF; ++i) {
-        const int slot = sg * HALF + i;
-        if (slot < nk)
-            *reinterpret_cast<float4 *>(partial + ((int64_t)blockIdx.x * REACH_T + slot) * BP +
-                                        4 * cg) =
-                make_float4(acc[i][0], acc[i][1], acc[i][2], acc[i][3]);
+            for (int i = 0; i < C::ITEMS; ++i) {
+                const int64_t k = (s0 + t) * RM_BK + 8 * cw + i * C::RPI + rl;
+                if (k < n) {
+                    const float4 *src = reinterpret_cast<const float4 *>(u + k * BP + 8 * c8);
+                    dst[i][0] = __ldcs(src);
+                    dst[i][1] = __ldcs(src + 1);
+                } else {
+                    dst[i][0] = dst[i][1] = make_float4(0.f, 0.f, 0.f, 0.f);
+                }
+            }
+        };
+        // add the finished accumulator of chunk c into the partial (the
+        // first chunk stores); false if its wait gave up
+        auto flush = [&](int64_t c) -> bool {
+            const int acc = (int)(c & 1);
+            int f_ok = lane == 0 ? (mbar_wait(&dfull[acc], (uint32_t)((c >> 1) & 1), status) ? 1 : 0)
+                                 : 0;
+            f_ok = __shfl_sync(0xffffffffu, f_ok, 0);
+            if (!f_ok) return false;
+            tc_fence_after();
+#pragma unroll 1
+            for (int ch = 0; ch < BP / 64; ++ch) {
+                uint32_t r[32];
+                tmem_ld32(tmem_base + ((uint32_t)(q * 32) << 16) +
+                              (uint32_t)(acc * BP + half * (BP / 2) + ch * 32),
+                          r);
+                tmem_ld_wait();
+                float4 *dst = reinterpret_cast<float4 *>(o + ch * 32);
+#pragma unroll
+                for (int i = 0; i < 8; ++i) {
+                    float4 v = make_float4(__uint_as_float(r[4 * i]), __uint_as_float(r[4 * i + 1]),
+                                           __uint_as_float(r[4 * i + 2]),
+                                           __uint_as_float(r[4 * i + 3]));
+                    if (c > 0) {
+                        const float4 p = dst[i];
+                        v.x += p.x;
+                        v.y += p.y;
+                        v.z += p.z;
+                        v.w += p.w;
+                    }
+                    dst[i] = v;
+                }
+            }
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&dfree[acc]);
+            return true;
+        };
+        uint32_t stage = 0, phase = 0;
+        bool ok = true;
+        if (ns > 0) load(0, cur);
+        for (int64_t t = 0; t < ns; ++t) {
+            if (t + 1 < ns) load(t + 1, nxt);
+            int w_ok = lane == 0 ? (mbar_wait(&empty[stage], phase ^ 1u, status) ? 1 : 0) : 0;
+            w_ok = __shfl_sync(0xffffffffu, w_ok, 0);
+            if (!w_ok) {
+                ok = false;
+                break;
+            }
+            uint8_t *bh = b_hi(stage), *bl = b_lo(stage);
+#pragma unroll
+            for (int i = 0; i < C::ITEMS; ++i) {
+                const int r = 8 * cw + i * C::RPI + rl;     // row in the stage (K)
+                const uint32_t off = (uint32_t)(c8 >> 3) * C::LBO + (uint32_t)r * 128u +
+                                     ((uint32_t)((c8 & 7) ^ (r & 7)) << 4);
+                uint4 vh, vl;
+                vh.x = split_bf16_pair(cur[i][0].x, cur[i][0].y, vl.x);
+                vh.y = split_bf16_pair(cur[i][0].z, cur[i][0].w, vl.y);
+                vh.z = split_bf16_pair(cur[i][1].x, cur[i][1].y, vl.z);
+                vh.w = split_bf16_pair(cur[i][1].z, cur[i][1].w, vl.w);
+                *reinterpret_cast<uint4 *>(bh + off) = vh;
+                *reinterpret_cast<uint4 *>(bl + off) = vl;
+            }
+            fence_async_smem();                       // generic writes -> the MMA's reads
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&bfull[stage]);
+            if (++stage == RM_STAGES) {
+                stage = 0;
+                phase ^= 1u;
+            }
+            // the previous chunk is complete once the first stage of this
+            // one is handed over: flush it while the MMAs run on
+            if (t % RM_CHUNK == 0 && t > 0 && !flush(t / RM_CHUNK - 1)) {
+                ok = false;
+                break;
+            }
+#pragma unroll
+            for (int i = 0; i < C::ITEMS; ++i) {
+                cur[i][0] = nxt[i][0];
+                cur[i][1] = nxt[i][1];
+            }
+        }
+        if (ns == 0) {
+            for (int b = 0; b < BP / 2; b += 4)
+                *reinterpret_cast<float4 *>(o + b) = make_float4(0.f, 0.f, 0.f, 0.f);
+        } else if (ok) {
+            flush(n_chunks - 1);
+        }
     }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    if (warp == 1) tmem_dealloc(tmem_base, C::TMEM_COLS);
 }
 
-// Final score of each flagged candidate for each real query column: its u
-// plus the CTAs' partials, appended as a filter key (score bits, ~chunk ID)
-// to the column's buffer; the buffer then holds exactly them.  One block per
-// candidate: thread t takes column t % bp and every (1024 / bp)-th partial
-// from t / bp on (coalesced rows of the partials), and the groups are added
-// in group order (the same order on every run).
-__global__ __launch_bounds__(1024) void k_reach_emit(const float *__restrict__ u, int bp, int B,
-                                                     const float *__restrict__ partial,
-                                                     int n_parts, const ReachSlots rs,
-                                                     const int32_t *__restrict__ rows,
-                                                     const int32_t *__restrict__ ext_of,
-                                                     unsigned int *__restrict__ cnt,
-                                                     unsigned long long *__restrict__ buf,
-                                                     int64_t cap) {
-    __shared__ float red[1024];
-    const int i = blockIdx.x;
-    const int b = threadIdx.x % bp, g = threadIdx.x / bp, ng = blockDim.x / bp;
-    float acc = 0.f;
-#pragma unroll 16
-    for (int p = g; p < n_parts; p += ng) acc += partial[((int64_t)p * REACH_T + i) * bp + b];
-    red[threadIdx.x] = acc;
+// coef_hi / coef_lo [REACH_T][n_pad] bf16: row i = candidate slot i's
+// combined coefficient sum_t alpha^t C_t[k][i] (Horner over t) split into
+// hi + lo, zero for k >= n.  One CTA per 64 rows k: the rows' slots are
+// read contiguously (coalesced), transposed through shared memory and
+// written along k (coalesced).
+__global__ __launch_bounds__(256) void k_reach_pack(const float *__restrict__ C, int64_t n,
+                                                    int64_t n_pad, int H, float alpha,
+                                                    uint16_t *__restrict__ hi,
+                                                    uint16_t *__restrict__ lo) {
+    __shared__ float tile[64][REACH_T + 1];
+    const int64_t k0 = (int64_t)blockIdx.x * 64;
+    for (int x = threadIdx.x; x < 64 * REACH_T; x += blockDim.x) {
+        const int kk = x / REACH_T, i = x % REACH_T;
+        const int64_t k = k0 + kk;
+        float c = 0.f;
+        if (k < n) {
+            const int64_t at = k * REACH_T + i;
+            for (int t = H; t >= 1; --t) c = alpha * (c + C[(int64_t)(t - 1) * n * REACH_T + at]);
+        }
+        tile[kk][i] = c;
+    }
     __syncthreads();
-    if (g == 0 && b < B) {
-        float sum = red[b];
-        for (int h = 1; h < ng; ++h) sum += red[h * bp + b];
-        const int64_t j = rows[rs.slot[i]];
-        const float s = u[j * bp + b] + sum;
-        buf[(int64_t)b * cap + i] = ((unsigned long long)__float_as_uint(s) << 32) |
-                                    (unsigned long long)(~(uint32_t)ext_of[j]);
-        if (i == 0) cnt[b] = (unsigned int)rs.nk;
+    for (int x = threadIdx.x; x < 32 * REACH_T; x += blockDim.x) {
+        const int i = x / 32, kk = 2 * (x % 32);
+        const int64_t k = k0 + kk;
+        uint32_t l;
+        const uint32_t h = split_bf16_pair(tile[kk][i], tile[kk + 1][i], l);
+        *reinterpret_cast<uint32_t *>(hi + (int64_t)i * n_pad + k) = h;
+        *reinterpret_cast<uint32_t *>(lo + (int64_t)i * n_pad + k) = l;
     }
 }
 
@@ -290,77 +505,109 @@ cudaError_t launch_reach_check(const float *ub, const float *floor_p, const int3
     return cudaGetLastError();
 }
 
-int reach_parts() { return device_sm_count() * 2; }
+// Final score of each flagged candidate for each real query column: its u
+// plus the CTAs' partials, appended as a filter key (score bits, ~chunk ID)
+// to the column's buffer; the buffer then holds exactly them.  One block
+// per candidate slot of the plan (blocks past nk, and every block when the
+// plan says the hops run, return at once): thread t takes column t % bp
+// and every (1024 / bp)-th partial from t / bp on (coalesced rows of the
+// partials), and the groups are added in group order (the same order on
+// every run).
+__global__ __launch_bounds__(1024) void k_reach_emit(const float *__restrict__ u, int bp, int B,
+                                                     const float *__restrict__ partial,
+                                                     int n_parts, const int32_t *__restrict__ plan,
+                                                     const int32_t *__restrict__ rows,
+                                                     const int32_t *__restrict__ ext_of,
+                                                     unsigned int *__restrict__ cnt,
+                                                     unsigned long long *__restrict__ buf,
+                                                     int64_t cap) {
+    __shared__ float red[1024];
+    if (plan[0] == 0) return;
+    const int nk = plan[1];
+    const int i = blockIdx.x;
+    if (i >= nk) return;
+    const int slot = plan[2 + i];
+    const int b = threadIdx.x % bp, g = threadIdx.x / bp, ng = blockDim.x / bp;
+    float acc = 0.f;
+#pragma unroll 16
+    for (int p = g; p < n_parts; p += ng) acc += partial[((int64_t)p * REACH_T + slot) * bp + b];
+    red[threadIdx.x] = acc;
+    __syncthreads();
+    if (g == 0 && b < B) {
+        float sum = red[b];
+        for (int h = 1; h < ng; ++h) sum += red[h * bp + b];
+        const int64_t j = rows[slot];
+        const float s = u[j * bp + b] + sum;
+        buf[(int64_t)b * cap + i] = ((unsigned long long)__float_as_uint(s) << 32) |
+                                    (unsigned long long)(~(uint32_t)ext_of[j]);
+        if (i == 0) cnt[b] = (unsigned int)nk;
+    }
+}
 
-// The packed width: the flagged count rounded up to 8 (bp = 256) or 16.
-static int reach_width(int bp, int nk) { return bp == 256 ? (nk + 7) & ~7 : (nk + 15) & ~15; }
+int reach_parts() { return device_sm_count(); }
 
-size_t reach_coef_floats(int64_t n, int bp, int nk) { return (size_t)n * reach_width(bp, nk); }
+int64_t reach_pad_rows(int64_t n) { return (n + RM_BK - 1) / RM_BK * RM_BK; }
 
-cudaError_t launch_reach_coef(const float *C, int64_t n, int H, float alpha, const ReachSlots &rs,
-                              int bp, float *coefK, cudaStream_t st) {
-    const int nk8 = reach_width(bp, rs.nk);
-    k_reach_coef<<<device_sm_count() * 8, 256, 0, st>>>(C, n, H, alpha, rs, nk8, coefK);
+cudaError_t launch_reach_plan(const int32_t *keep, const int *bad, const int *t_cnt, int k,
+                              int32_t *plan, cudaStream_t st) {
+    k_reach_plan<<<1, REACH_T, 0, st>>>(keep, bad, t_cnt, k, plan);
     return cudaGetLastError();
 }
 
-template <int NK, int BP>
-static cudaError_t reach_terms_nk(const float *u, int64_t n, const float *coefK, int nk,
-                                  float *partial, int parts, cudaStream_t st) {
-    const size_t smem = (size_t)2 * REACH_ROWS * (BP + NK) * sizeof(float);
+cudaError_t launch_reach_pack(const float *C, int64_t n, int H, float alpha, uint16_t *coef_hi,
+                              uint16_t *coef_lo, cudaStream_t st) {
+    const int64_t n_pad = reach_pad_rows(n);
+    if (n_pad <= 0) return cudaSuccess;
+    k_reach_pack<<<(unsigned)(n_pad / 64), 256, 0, st>>>(C, n, n_pad, H, alpha, coef_hi, coef_lo);
+    return cudaGetLastError();
+}
+
+template <int BP>
+static cudaError_t reach_mma_bp(const uint16_t *coef_hi, const uint16_t *coef_lo, const float *u,
+                                int64_t n, const int32_t *plan, float *partial, int parts,
+                                int *status, cudaStream_t st) {
+    using C = RmCfg<BP>;
     static bool attr[64] = {false};
     int dev = 0;
     cudaGetDevice(&dev);
     if (dev >= 0 && dev < 64 && !attr[dev]) {
-        cudaError_t e = cudaFuncSetAttribute(k_reach_terms<NK, BP>,
-                                             cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        cudaError_t e = cudaFuncSetAttribute(k_reach_mma<BP>,
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
         if (e != cudaSuccess) return e;
         attr[dev] = true;
     }
-    k_reach_terms<NK, BP><<<parts, REACH_T_THREADS, smem, st>>>(u, n, coefK, nk, partial);
+    const int64_t n_pad = reach_pad_rows(n);
+    CUtensorMap thi, tlo, thi64, tlo64;
+    cudaError_t e = make_tmap_2d(&thi, coef_hi, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2,
+                                 (uint64_t)n_pad, RM_M, (uint64_t)n_pad * 2, RM_BK, RM_M);
+    if (e == cudaSuccess)
+        e = make_tmap_2d(&tlo, coef_lo, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, (uint64_t)n_pad, RM_M,
+                         (uint64_t)n_pad * 2, RM_BK, RM_M);
+    if (e == cudaSuccess)
+        e = make_tmap_2d(&thi64, coef_hi, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, (uint64_t)n_pad,
+                         RM_M, (uint64_t)n_pad * 2, RM_BK, RM_M / 2);
+    if (e == cudaSuccess)
+        e = make_tmap_2d(&tlo64, coef_lo, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, (uint64_t)n_pad,
+                         RM_M, (uint64_t)n_pad * 2, RM_BK, RM_M / 2);
+    if (e != cudaSuccess) return e;
+    k_reach_mma<BP><<<parts, RM_THREADS, C::SMEM, st>>>(thi, tlo, thi64, tlo64, u, n, plan,
+                                                         partial, status);
     return cudaGetLastError();
 }
 
-// Flagged counts the score pass takes: NK (rounded up to 8 / 16) at most 64
-// slots per thread group pair at BP = 256, 128 at BP = 128.
-bool reach_fits(int bp, int nk) {
-    return nk >= 1 && ((bp == 256 && nk <= 64) || (bp == 128 && nk <= 128));
-}
-
-cudaError_t launch_reach_scores(const float *u, int bp, int B, int64_t n, const float *coefK,
-                                const ReachSlots &rs, const int32_t *rows, const int32_t *ext_of,
-                                float *partial, unsigned int *cnt, unsigned long long *buf,
-                                int64_t cap, cudaStream_t st, int *launches) {
-    if (!reach_fits(bp, rs.nk)) return cudaErrorInvalidValue;
+cudaError_t launch_reach_scores(const float *u, int bp, int B, int64_t n, const uint16_t *coef_hi,
+                                const uint16_t *coef_lo, const int32_t *plan, const int32_t *rows,
+                                const int32_t *ext_of, float *partial, unsigned int *cnt,
+                                unsigned long long *buf, int64_t cap, int *status, cudaStream_t st,
+                                int *launches) {
+    if (n <= 0 || (bp != 128 && bp != 256)) return cudaErrorInvalidValue;
     const int parts = reach_parts();
-    cudaError_t e = cudaErrorInvalidValue;
-    if (bp == 256) {
-        switch ((rs.nk + 7) & ~7) {
-        case 8: e = reach_terms_nk<8, 256>(u, n, coefK, rs.nk, partial, parts, st); break;
-        case 16: e = reach_terms_nk<16, 256>(u, n, coefK, rs.nk, partial, parts, st); break;
-        case 24: e = reach_terms_nk<24, 256>(u, n, coefK, rs.nk, partial, parts, st); break;
-        case 32: e = reach_terms_nk<32, 256>(u, n, coefK, rs.nk, partial, parts, st); break;
-        case 40: e = reach_terms_nk<40, 256>(u, n, coefK, rs.nk, partial, parts, st); break;
-        case 48: e = reach_terms_nk<48, 256>(u, n, coefK, rs.nk, partial, parts, st); break;
-        case 56: e = reach_terms_nk<56, 256>(u, n, coefK, rs.nk, partial, parts, st); break;
-        case 64: e = reach_terms_nk<64, 256>(u, n, coefK, rs.nk, partial, parts, st); break;
-        default: break;
-        }
-    } else {
-        switch ((rs.nk + 15) & ~15) {
-        case 16: e = reach_terms_nk<16, 128>(u, n, coefK, rs.nk, partial, parts, st); break;
-        case 32: e = reach_terms_nk<32, 128>(u, n, coefK, rs.nk, partial, parts, st); break;
-        case 48: e = reach_terms_nk<48, 128>(u, n, coefK, rs.nk, partial, parts, st); break;
-        case 64: e = reach_terms_nk<64, 128>(u, n, coefK, rs.nk, partial, parts, st); break;
-        case 80: e = reach_terms_nk<80, 128>(u, n, coefK, rs.nk, partial, parts, st); break;
-        case 96: e = reach_terms_nk<96, 128>(u, n, coefK, rs.nk, partial, parts, st); break;
-        case 112: e = reach_terms_nk<112, 128>(u, n, coefK, rs.nk, partial, parts, st); break;
-        case 128: e = reach_terms_nk<128, 128>(u, n, coefK, rs.nk, partial, parts, st); break;
-        default: break;
-        }
-    }
+    cudaError_t e = bp == 256
+                        ? reach_mma_bp<256>(coef_hi, coef_lo, u, n, plan, partial, parts, status, st)
+                        : reach_mma_bp<128>(coef_hi, coef_lo, u, n, plan, partial, parts, status, st);
     if (e != cudaSuccess) return e;
-    k_reach_emit<<<rs.nk, 1024, 0, st>>>(u, bp, B, partial, parts, rs, rows, ext_of, cnt, buf, cap);
+    k_reach_emit<<<REACH_T, 1024, 0, st>>>(u, bp, B, partial, parts, plan, rows, ext_of, cnt, buf,
+                                           cap);
     if (launches) *launches += 2;
     return cudaGetLastError();
 }

@@ -609,6 +609,135 @@ __global__ __launch_bounds__(PF_ROWS) void k_prune_floor(
     }
 }
 
+// The batch's distinct query namespaces, ascending, and for each the
+// smallest score that the filter bound of any of its queries admits.  One
+// CTA of PF_TAGS threads: keys (valid, tag) sorted by a bitonic network in
+// shared memory, first occurrences numbered by a scan.
+__global__ __launch_bounds__(PF_TAGS) void k_ns_tags(const unsigned long long *__restrict__ bound,
+                                                     const int32_t *__restrict__ q_ns, int n_real,
+                                                     int32_t *__restrict__ tags,
+                                                     int *__restrict__ n_tags,
+                                                     float *__restrict__ tag_floor) {
+    __shared__ unsigned long long key[PF_TAGS];
+    __shared__ int pos[PF_TAGS];
+    __shared__ unsigned int mn[PF_TAGS];
+    const int t = threadIdx.x;
+    // valid tags first, in signed order; padding (1 << 32) last
+    key[t] = t < n_real ? (unsigned long long)((uint32_t)q_ns[t] ^ 0x80000000u) : (1ull << 32);
+    mn[t] = 0x7f800000u;
+    __syncthreads();
+    for (int size = 2; size <= PF_TAGS; size <<= 1)
+        for (int stride = size >> 1; stride > 0; stride >>= 1) {
+            const int o = t ^ stride;
+            if (o > t) {
+                const unsigned long long a = key[t], b = key[o];
+                const bool asc = (t & size) == 0;
+                if (asc ? a > b : a < b) {
+                    key[t] = b;
+                    key[o] = a;
+                }
+            }
+            __syncthreads();
+        }
+    const bool first = key[t] < (1ull << 32) && (t == 0 || key[t - 1] != key[t]);
+    pos[t] = first ? 1 : 0;
+    __syncthreads();
+    for (int o = 1; o < PF_TAGS; o <<= 1) {          // inclusive scan
+        const int v = t >= o ? pos[t - o] : 0;
+        __syncthreads();
+        pos[t] += v;
+        __syncthreads();
+    }
+    const int nt = pos[PF_TAGS - 1];
+    if (first) tags[pos[t] - 1] = (int32_t)((uint32_t)key[t] ^ 0x80000000u);
+    if (t == 0) *n_tags = nt;
+    __syncthreads();
+    if (t < n_real && bound) {
+        const int32_t mine = q_ns[t];
+        int lo = 0, hi = nt;
+        while (lo < hi) {
+            const int mid = (lo + hi) >> 1;
+            if (tags[mid] < mine) lo = mid + 1;
+            else hi = mid;
+        }
+        atomicMin(&mn[lo], (unsigned int)(bound[t] >> 32));
+    }
+    __syncthreads();
+    if (t < nt) tag_floor[t] = bound ? __uint_as_float(mn[t]) : 0.f;
+}
+
+// tag_floor[d] = max(tag_floor[d], k-th largest lb over the first PF_ROWS
+// split rows, heaviest first, of namespace tags[d]); one CTA per tag.
+__global__ __launch_bounds__(PF_ROWS) void k_ns_floor(const float *__restrict__ lb,
+                                                      const int32_t *__restrict__ ns_row,
+                                                      const int32_t *__restrict__ split_row,
+                                                      const int32_t *__restrict__ order,
+                                                      int64_t n_split, int k,
+                                                      const int32_t *__restrict__ tags,
+                                                      const int *__restrict__ n_tags,
+                                                      float *__restrict__ tag_floor) {
+    __shared__ unsigned int key[PF_ROWS];
+    __shared__ int wcount[PF_ROWS / 32];
+    __shared__ int got_s;
+    const int d = blockIdx.x;
+    if (d >= *n_tags) return;
+    const int t = threadIdx.x, lane = t & 31, w = t >> 5;
+    const int32_t tag = tags[d];
+    key[t] = 0u;
+    if (t == 0) got_s = 0;
+    __syncthreads();
+    for (int64_t c0 = 0; c0 < n_split; c0 += PF_ROWS) {
+        const int got = got_s;
+        if (got >= PF_ROWS) break;
+        const int64_t i = c0 + t;
+        int32_t r = 0;
+        const bool match = i < n_split && ns_row[r = split_row[order[i]]] == tag;
+        const unsigned int bal = __ballot_sync(0xffffffffu, match);
+        if (lane == 0) wcount[w] = __popc(bal);
+        __syncthreads();
+        int before = got;
+        for (int x = 0; x < w; ++x) before += wcount[x];
+        before += __popc(bal & ((1u << lane) - 1u));
+        if (match && before < PF_ROWS) key[before] = __float_as_uint(lb[r]);   // lb >= 0
+        __syncthreads();
+        if (t == 0) {
+            int tot = got;
+            for (int x = 0; x < PF_ROWS / 32; ++x) tot += wcount[x];
+            got_s = tot;
+        }
+        __syncthreads();
+    }
+    const int got = got_s < PF_ROWS ? got_s : PF_ROWS;
+    if (got < k) return;                              // too few rows for a floor of their own
+    // descending bitonic sort of the collected keys (absent ones are 0)
+    for (int size = 2; size <= PF_ROWS; size <<= 1)
+        for (int stride = size >> 1; stride > 0; stride >>= 1) {
+            const int o = t ^ stride;
+            if (o > t) {
+                const unsigned int a = key[t], b = key[o];
+                const bool desc = (t & size) == 0;
+                if (desc ? a < b : a > b) {
+                    key[t] = b;
+                    key[o] = a;
+                }
+            }
+            __syncthreads();
+        }
+    if (t == 0) tag_floor[d] = fmaxf(tag_floor[d], __uint_as_float(key[k - 1]));
+}
+
+cudaError_t launch_ns_floors(const unsigned long long *bound, const int32_t *q_ns, int n_real,
+                             const float *lb, const int32_t *ns_row, const int32_t *split_row,
+                             const int32_t *split_order, int64_t n_split, int k, int32_t *tags,
+                             int *n_tags, float *tag_floor, cudaStream_t st) {
+    if (n_real < 1 || n_real > PF_TAGS || k < 1) return cudaErrorInvalidValue;
+    k_ns_tags<<<1, PF_TAGS, 0, st>>>(bound, q_ns, n_real, tags, n_tags, tag_floor);
+    if (n_split > 0 && k <= PF_ROWS)
+        k_ns_floor<<<PF_TAGS, PF_ROWS, 0, st>>>(lb, ns_row, split_row, split_order, n_split, k,
+                                                tags, n_tags, tag_floor);
+    return cudaGetLastError();
+}
+
 cudaError_t launch_prune_floor(const unsigned long long *bound, int n_real, const float *lb,
                                const int32_t *lb_rows, const int32_t *order, int64_t n_lb_rows,
                                int k, float *floor_out, cudaStream_t st) {

@@ -133,6 +133,25 @@ __host__ __device__ constexpr uint32_t idesc_bf16_m128(int n) {
            | ((uint32_t)(128 >> 4) << 24);  // M >> 4
 }
 
+// Instruction-descriptor bit: the B operand is MN-major (N contiguous in
+// shared memory) instead of K-major.
+constexpr uint32_t IDESC_B_MN_MAJOR = 1u << 16;
+
+// Shared-memory matrix descriptor for an MN-major operand in the 128-byte
+// swizzle layout: atoms of 8 K-rows x 64 bf16 along MN (128 bytes a row,
+// the 16-byte chunk c of row r stored at chunk position c ^ (r % 8)), the
+// next 64 MN values `lbo` bytes further, the next 8 K-rows `sbo` bytes
+// further; descriptor version 1, layout SWIZZLE_128B.
+__device__ __forceinline__ uint64_t sdesc_mn_sw128(uint32_t saddr, uint32_t lbo, uint32_t sbo) {
+    uint64_t d = 0;
+    d |= (uint64_t)((saddr & 0x3FFFFu) >> 4);   // start address >> 4
+    d |= (uint64_t)((lbo >> 4) & 0x3FFFu) << 16; // leading offset: between MN atoms
+    d |= (uint64_t)((sbo >> 4) & 0x3FFFu) << 32; // stride offset: between 8-row K groups
+    d |= (uint64_t)1 << 46;                     // descriptor version for tcgen05
+    d |= (uint64_t)2 << 61;                     // SWIZZLE_128B
+    return d;
+}
+
 // Shared-memory matrix descriptor for a K-major operand stored in the
 // 128-byte swizzle layout TMA produces (rows of 64 bf16 = 128 B, 8-row
 // atoms of 1024 B): start address, stride between 8-row groups 1024 B,

@@ -190,3 +190,54 @@ def test_fp32_hops_never_lower_a_score():
             nxt[:, j] = (u32[:, j] + (alpha * acc).astype(F32)).astype(F32)
         assert (nxt >= prev).all()
         prev = nxt
+
+
+def _bf16_rne(x):
+    """float32 -> nearest bf16 (ties to even), as float32 (bit arithmetic)."""
+    b = np.ascontiguousarray(x, dtype=F32).view(np.uint32)
+    r = (b + np.uint32(0x7FFF) + ((b >> np.uint32(16)) & np.uint32(1))) & np.uint32(0xFFFF0000)
+    return r.view(F32)
+
+
+@pytest.mark.parametrize("seed", [0, 1])
+def test_split_bf16_products_keep_the_candidates_terms(seed):
+    """The candidates' two-hop terms sum_k coef[k][i] u[k][b] are computed on
+    the tensor cores from split-bf16 operands: x = hi + lo with hi = bf16(x)
+    and lo = bf16(x - hi) (x - hi is exact in fp32), and the three products
+    hi*hi + hi*lo + lo*hi.  bf16 rounds to 8 significant bits, so
+    |x - hi| <= 2^-8 |x| and |x - hi - lo| <= 2^-8 |x - hi| <= 2^-16 |x|; the
+    dropped lo*lo is at most 2^-16 of the product; every product is thus
+    within 3 * 2^-16 (4.6e-5) relative, and, all terms being non-negative,
+    so is the sum: inside the 1e-4 near-tie band of the selection, where a
+    single bf16 product (2^-8) is not.  The rounding errors have random
+    signs, so the sums land far closer (below 1e-5 here).  Emulated with the
+    products in fp64, on scores u = exp(tau <q, e> - c) of unit vectors
+    (tau = 1/sqrt(d)) and heavy-tailed non-negative coefficients."""
+    rng = np.random.default_rng(seed)
+    n, d, nq, nk = 4096, 256, 16, 40
+    e = rng.standard_normal((n, d)).astype(F32)
+    e /= np.linalg.norm(e, axis=1, keepdims=True)
+    q = rng.standard_normal((nq, d)).astype(F32)
+    q /= np.linalg.norm(q, axis=1, keepdims=True)
+    tau = 1.0 / math.sqrt(d)
+    u = np.exp((tau * (e @ q.T) - tau).astype(F32)).astype(F32)          # [n][nq]
+    coef = (rng.lognormal(-6.0, 2.0, (n, nk)) * (rng.random((n, nk)) < 0.3)).astype(F32)
+    exact = coef.astype(np.float64).T @ u.astype(np.float64)            # [nk][nq]
+
+    def split(x):
+        hi = _bf16_rne(x)
+        lo = _bf16_rne((x - hi).astype(F32))
+        return hi.astype(np.float64), lo.astype(np.float64)
+
+    ch, cl = split(coef)
+    uh, ul = split(u)
+    three = ch.T @ uh + ch.T @ ul + cl.T @ uh
+    one = ch.T @ uh
+    rel3 = np.abs(three - exact) / exact
+    rel1 = np.abs(one - exact) / exact
+    assert rel3.max() <= 3 * 2.0 ** -16, rel3.max()
+    assert rel3.max() < 1e-5
+    assert rel1.max() > 1e-4          # a single bf16 product would break the band
+    # the split itself: hi + lo within 2^-16 of every operand
+    assert (np.abs(ch + cl - coef) <= 2.0 ** -16 * coef).all()
+    assert (np.abs(uh + ul - u) <= 2.0 ** -16 * u).all()

@@ -103,9 +103,12 @@ def test_last_hop_row_bounds_change_nothing(hops, k, monkeypatch):
     and the oracle's (gmm1m recipe at N = 16384, hub rows split).  Scores may
     differ in the last bits only: without the skip more rows clear the
     filter's sample bound, a query's buffer can overflow, and its column is
-    then recomputed by the merge with another summation order."""
+    then recomputed by the merge with another summation order.  The two-hop
+    path from reach coefficients is switched off in both runs: it is tested
+    on its own below."""
     import dataclasses
     wl = dataclasses.replace(synth.workload(2, scale=1 / 64), hops=hops, k=k)
+    monkeypatch.setenv("AKASHIC_REACH", "0")
     monkeypatch.setenv("AKASHIC_HOP_PRUNE", "0")
     _, full = gpu_retrieve(wl, "clustered")
     monkeypatch.setenv("AKASHIC_HOP_PRUNE", "1")
@@ -157,29 +160,41 @@ def test_score_filter_overflow_falls_back():
 
 
 @pytest.mark.parametrize("hops,sort_by_time", [(0, False), (2, False), (2, True), (1, True)])
-def test_namespace_scoped_retrieval(hops, sort_by_time):
-    """Chunks tagged by component mod 5, plus a namespace of only 3 chunks;
-    each of the 256 queries scoped to a seeded namespace (every 17th to the
-    small one, which pads its list); scores and propagation over the whole
-    store, candidates from the namespace only; score order or SortByTime.
-    N = 16384 from the gmm1m recipe."""
+def test_namespace_scoped_retrieval(hops, sort_by_time, monkeypatch):
+    """Chunks tagged by component mod 6 (namespace 5 queried by no query),
+    plus a namespace of only 3 chunks; each of the 256 queries scoped to a
+    seeded namespace (every 17th to the small one, which pads its list);
+    scores and propagation over the whole store, candidates from the
+    namespace only; score order or SortByTime.  N = 16384 from the gmm1m
+    recipe.  The last hop's per-namespace floors (each namespace's k-th
+    largest lower bound; rows of unqueried namespaces skipped) must select
+    what the unpruned hops select."""
     import oracle
     import torch
     wl = synth.workload(2, scale=1 / 64)
     rng = np.random.default_rng(11)
-    ns_of = (wl.component % 5).astype(np.int32)
+    ns_of = (wl.component % 6).astype(np.int32)
     ns_of[rng.choice(wl.n, 3, replace=False)] = 7
     q_ns = rng.integers(0, 5, wl.n_queries).astype(np.int32)
     q_ns[::17] = 7
-    store = gpu_store(wl, "clustered")
-    store.set_namespace(0, torch.from_numpy(ns_of).cuda())
     q = torch.from_numpy(np.ascontiguousarray(wl.queries).view(np.int16)).cuda()
-    ids, sc, pg, npg = store.retrieve(q, wl.k, wl.alpha, hops,
-                                      q_ns=torch.from_numpy(q_ns).cuda(),
-                                      sort_by_time=sort_by_time)
-    store.sync()
-    got = dict(ids=ids.cpu().numpy(), scores=sc.cpu().numpy(), page_ids=pg.cpu().numpy(),
-               n_pages=npg.cpu().numpy())
+
+    def run():
+        store = gpu_store(wl, "clustered")
+        store.set_namespace(0, torch.from_numpy(ns_of).cuda())
+        ids, sc, pg, npg = store.retrieve(q, wl.k, wl.alpha, hops,
+                                          q_ns=torch.from_numpy(q_ns).cuda(),
+                                          sort_by_time=sort_by_time)
+        store.sync()
+        return dict(ids=ids.cpu().numpy(), scores=sc.cpu().numpy(), page_ids=pg.cpu().numpy(),
+                    n_pages=npg.cpu().numpy())
+
+    got = run()
+    if hops >= 1:
+        monkeypatch.setenv("AKASHIC_HOP_PRUNE", "0")
+        full = run()
+        for key in ("ids", "page_ids", "n_pages"):
+            assert np.array_equal(full[key], got[key]), key
     ref = oracle.retrieve(wl.emb, wl.queries, wl.row_ptr, wl.col, oracle_weights(wl), tau=wl.tau,
                           alpha=wl.alpha, hops=hops, k=wl.k, page_of=wl.page_of["clustered"],
                           want_final=True, ns_of=ns_of, q_ns=q_ns, sort_by_time=sort_by_time)
@@ -231,9 +246,13 @@ def test_two_hop_scores_from_reach_coefficients(placement, B, k, must, monkeypat
     top-k floor is one of the candidate rows with graph-only reach
     coefficients, s^(2) of those rows comes from one pass over u.  On the
     gmm1m recipe (N = 16384) that path must be taken where `must` (no
-    propagation hop is launched) and select what the hops select: equal IDs,
-    pages and counts, scores within fp32 reordering, and the oracle's
-    selection (B = 256 and 128 queries, k = 32 and 64)."""
+    propagation hop is launched) and select what the hops select: the same
+    IDs except near-ties (scores within REACH_REL of the k-th), pages from
+    the page table, scores of the common IDs within REACH_REL, and the
+    oracle's selection (B = 256 and 128 queries, k = 32 and 64).  REACH_REL
+    = 5e-5: the candidates' terms are split-bf16 products (each operand
+    hi + lo to 2^-16, the lo x lo term dropped: at most 3 * 2^-16 = 4.6e-5
+    relative per product, all products non-negative) with fp32 sums."""
     import dataclasses
     wl = dataclasses.replace(synth.workload(2, scale=1 / 64), k=k)
     wl = dataclasses.replace(wl, queries=wl.queries[:B])
@@ -250,9 +269,17 @@ def test_two_hop_scores_from_reach_coefficients(placement, B, k, must, monkeypat
     if must:
         assert ph["propagate"][1] == 0, ph            # no hop launched
         assert ph["last_hop"][1] > 0, ph              # the reach scores were
-    for key in ("ids", "page_ids", "n_pages"):
-        assert np.array_equal(hops_out[key], reach_out[key]), key
-    np.testing.assert_allclose(reach_out["scores"], hops_out["scores"], rtol=1e-5, atol=0)
+    REACH_REL = 5e-5
+    for b in range(B):
+        hi, ri = hops_out["ids"][b].tolist(), reach_out["ids"][b].tolist()
+        hs = dict(zip(hi, hops_out["scores"][b].astype(np.float64)))
+        rs = dict(zip(ri, reach_out["scores"][b].astype(np.float64)))
+        kth = min(hs.values())
+        for x in set(hi) ^ set(ri):
+            s = hs.get(x, rs.get(x))
+            assert abs(s - kth) <= REACH_REL * kth, f"query {b}: chunk {x} swapped ({s} vs {kth})"
+        for x in set(hi) & set(ri):
+            assert abs(rs[x] - hs[x]) <= REACH_REL * hs[x], f"query {b}: chunk {x} score"
     assert_retrieval_parity(wl, placement, reach_out, oracle_retrieve(wl, placement))
 
 
