@@ -746,13 +746,14 @@ def run_retrieve(args, k=None, hops=None, metric=METRIC, workload=WORKLOAD, scop
     # which propagation ran: the hops, or (two hops, every row that can reach
     # the top-k among the reach candidates) the candidates' scores from u
     if hops >= 1 and phases["propagate"][1] == 0 and phases["last_hop"][1] > 0:
-        moved = wl.n * wl.dim * 2 + 2 * wl.n * 256 * 4 + wl.n * 40 * 4
+        moved = wl.n * wl.dim * 2 + 2 * wl.n * 256 * 4 + wl.n * 64 * 2 * 2
         path_note = {"propagation": "two-hop scores of the top-k candidates from graph-only "
-                                    "reach coefficients, one pass over u (no hop run)",
+                                    "reach coefficients, one tensor-core pass over u (no hop run)",
                      "bytes_moved_per_step": moved,
                      "note": "pass_roofline counts full hops (five slab passes); this path "
-                             "reads E, writes u and reads u and the candidates' coefficients "
-                             "(40 per row)"}
+                             "reads E, writes u and reads u and 64 coefficient rows per store "
+                             "row (bf16 hi + lo; 128 when a flagged candidate is at slot 64 or "
+                             "above)"}
     else:
         moved = total_ab
         path_note = {"propagation": "hops (the last one skips rows below the top-k floor)",

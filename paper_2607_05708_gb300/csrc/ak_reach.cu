@@ -179,7 +179,7 @@ __global__ __launch_bounds__(REACH_T) void k_reach_plan(const int32_t *__restric
 //       k_reach_pack as [REACH_T slots][n_pad rows] bf16 (hi, lo), loaded
 //       by TMA as K-major tiles [128 slots][64 rows] in the 128-byte swizzle;
 //   B = u, loaded by converter warps from global memory (two float4 of one
-//       row per lane, one row per warp instruction), split into hi / lo and
+//       row per lane, one row per warp instruction at BP = 256), split into hi / lo and
 //       stored as MN-major tiles [64 rows][BP queries]: atoms of 8 rows x 64
 //       queries (128 bytes a row, 16-byte chunks swizzled by the row), four
 //       (BP = 256) or two such atom columns RM_BK * 128 bytes apart.
@@ -190,14 +190,17 @@ __global__ __launch_bounds__(REACH_T) void k_reach_plan(const int32_t *__restric
 // alternate, and the converter warps add each finished one into the CTA's
 // partial with ordinary round-to-nearest fp32 adds (the partial rows stay
 // in L2) while the MMAs fill the other.
-// Warps: 0 TMA producer (A), 1 MMA issuer, 2..9 converters (and the flush:
-// warp w reads TMEM lanes 32 (w % 4) .., column half (w - 2) / 4).  Each
+// Warps: 0 TMA producer (A), 1 MMA issuer, 2..9 converters, eight rows of
+// a stage each (and the flush: warp w reads TMEM lanes 32 (w % 4) ..,
+// column half (w - 2) / 4).  Sixteen converter warps with half the rows
+// each measured slower (290 against 260 us at full size), as did an L2
+// prefetch of u three stages ahead (280 us).  Each
 // CTA takes a contiguous range of 64-row stages; 2 stages of 2 A + 2 B
 // tiles.
 constexpr int RM_BK = 64;                // store rows (K) per stage
 constexpr int RM_M = REACH_T;            // candidate slots (M)
 constexpr int RM_STAGES = 2;
-constexpr int RM_CONV_W = 8;             // converter warps
+constexpr int RM_CONV_W = 8;             // converter warps (8 rows of a stage each)
 constexpr int RM_THREADS = 64 + 32 * RM_CONV_W;
 constexpr int RM_CHUNK = 16;             // stages per accumulator
 
@@ -211,7 +214,10 @@ struct RmCfg {
     static constexpr int SMEM = 1024 + RM_STAGES * STAGE_BYTES + 256;
     static constexpr int CH = BP / 8;        // 16-byte bf16 chunks of a u row
     static constexpr int RPI = 32 / CH;      // u rows per warp instruction
-    static constexpr int ITEMS = 8 / RPI;    // (row, chunk) items per lane per stage
+    static constexpr int RPW = RM_BK / RM_CONV_W;   // u rows per converter warp per stage
+    static constexpr int ITEMS = RPW / RPI;  // (row, chunk) items per lane per stage
+    static constexpr int PARTS = RM_CONV_W / 4;     // column parts of a flush
+    static_assert(ITEMS >= 1 && RPW % RPI == 0, "converter layout");
     static constexpr int TMEM_COLS = 2 * BP; // two accumulators
     static_assert(BP == 128 || BP == 256, "query widths 128 and 256");
     static_assert(SMEM <= 227 * 1024, "shared memory");
@@ -353,14 +359,15 @@ __global__ __launch_bounds__(RM_THREADS, 1) void k_reach_mma(
         const int c8 = lane % C::CH;                  // chunk: queries 8 c8 .. 8 c8 + 7
         const int rl = lane / C::CH;                  // row within a warp instruction
         const int q = warp & 3;                       // flush: TMEM lanes 32 q ..
-        const int half = cw >> 2;                     // flush: column half
+        const int part = cw >> 2;                     // flush: column part
         const int slot = q * 32 + lane;
-        float *o = partial + ((int64_t)blockIdx.x * REACH_T + slot) * BP + half * (BP / 2);
+        constexpr int PW = BP / C::PARTS;             // columns of a part
+        float *o = partial + ((int64_t)blockIdx.x * REACH_T + slot) * BP + part * PW;
         float4 cur[C::ITEMS][2], nxt[C::ITEMS][2];
         auto load = [&](int64_t t, float4 (&dst)[C::ITEMS][2]) {
 #pragma unroll
             for (int i = 0; i < C::ITEMS; ++i) {
-                const int64_t k = (s0 + t) * RM_BK + 8 * cw + i * C::RPI + rl;
+                const int64_t k = (s0 + t) * RM_BK + C::RPW * cw + i * C::RPI + rl;
                 if (k < n) {
                     const float4 *src = reinterpret_cast<const float4 *>(u + k * BP + 8 * c8);
                     dst[i][0] = __ldcs(src);
@@ -380,10 +387,10 @@ __global__ __launch_bounds__(RM_THREADS, 1) void k_reach_mma(
             if (!f_ok) return false;
             tc_fence_after();
 #pragma unroll 1
-            for (int ch = 0; ch < BP / 64; ++ch) {
+            for (int ch = 0; ch < PW / 32; ++ch) {
                 uint32_t r[32];
                 tmem_ld32(tmem_base + ((uint32_t)(q * 32) << 16) +
-                              (uint32_t)(acc * BP + half * (BP / 2) + ch * 32),
+                              (uint32_t)(acc * BP + part * PW + ch * 32),
                           r);
                 tmem_ld_wait();
                 float4 *dst = reinterpret_cast<float4 *>(o + ch * 32);
@@ -421,7 +428,7 @@ __global__ __launch_bounds__(RM_THREADS, 1) void k_reach_mma(
             uint8_t *bh = b_hi(stage), *bl = b_lo(stage);
 #pragma unroll
             for (int i = 0; i < C::ITEMS; ++i) {
-                const int r = 8 * cw + i * C::RPI + rl;     // row in the stage (K)
+                const int r = C::RPW * cw + i * C::RPI + rl;   // row in the stage (K)
                 const uint32_t off = (uint32_t)(c8 >> 3) * C::LBO + (uint32_t)r * 128u +
                                      ((uint32_t)((c8 & 7) ^ (r & 7)) << 4);
                 uint4 vh, vl;
@@ -452,7 +459,7 @@ __global__ __launch_bounds__(RM_THREADS, 1) void k_reach_mma(
             }
         }
         if (ns == 0) {
-            for (int b = 0; b < BP / 2; b += 4)
+            for (int b = 0; b < PW; b += 4)
                 *reinterpret_cast<float4 *>(o + b) = make_float4(0.f, 0.f, 0.f, 0.f);
         } else if (ok) {
             flush(n_chunks - 1);
