@@ -86,7 +86,7 @@ struct StreamScratch {
     DevBuf rmax_u, rmin_u;       // u's row maxima / minima over the real queries
     DevBuf ub, lb, ext, pfloor;  // the last hop's row bounds, extremes, floor
     DevBuf skip_split, skip_slot, kept_rows, kept_count, kept_segs, kflag, kpos, ktmp;
-    DevBuf reach_keep, reach_bad, reach_part, reach_plan;
+    DevBuf reach_keep, reach_part, reach_plan;   // flags + bad + done, partials, plan
     DevBuf nsf;                  // scoped last hop: tags, their floors, their count
     // every candidate's combined coefficients (bf16 hi, lo), and their key
     DevBuf coef_hi, coef_lo;
@@ -1304,13 +1304,13 @@ static akashic_status_t retrieve_impl(akashic_mem *m, const uint16_t *q, int32_t
             rc.in_w = hp.in_w;
             rc.alpha = alpha;
             // scalar row bounds of the last hop's output, from u's row extremes
+            // (the two-hop reach path evaluates them only where it needs them
+            // and writes the arrays only when the hops run after all)
             const float *row_ub = nullptr, *row_lb = nullptr;
-            if (prune) {
+            const bool reach_try = prune && eff_hops == 2 && !q_ns && m->reach_on &&
+                                   m->n_split > 0 && (bp == 256 || bp == 128);
+            auto row_bounds = [&]() -> akashic_status_t {
                 PhaseScope ph(m, AKASHIC_PHASE_BOUND, st);
-                {
-                    std::lock_guard<std::mutex> lk(m->table_mu);
-                    AK_TRY(ensure_mass(m, hp, eff_hops, st));
-                }
                 CUDA_TRY(launch_final_bounds(sc->rmax_u.as<float>(), sc->rmin_u.as<float>(),
                                              m->mass_up.as<float>(), m->mass_dn.as<float>(), n,
                                              eff_hops, alpha, sc->ext.as<unsigned int>(),
@@ -1318,40 +1318,54 @@ static akashic_status_t retrieve_impl(akashic_mem *m, const uint16_t *q, int32_t
                                              &ph.launches, true));
                 row_ub = sc->ub.as<float>();
                 row_lb = sc->lb.as<float>();
+                return AKASHIC_OK;
+            };
+            if (prune) {
+                {
+                    std::lock_guard<std::mutex> lk(m->table_mu);
+                    AK_TRY(ensure_mass(m, hp, eff_hops, st));
+                }
+                if (!reach_try) AK_TRY(row_bounds());
             }
             // Two hops without running them: when every row whose upper bound
             // reaches the floor (here the k-th largest lower bound) is a
             // candidate with reach coefficients, their final scores come from
             // one pass over u and they alone are the selection's candidates.
             bool reach_done = false;
-            if (prune && eff_hops == 2 && !q_ns && m->reach_on && m->n_split > 0 &&
-                (bp == 256 || bp == 128)) {
+            if (reach_try) {
                 {
                     PhaseScope ph(m, AKASHIC_PHASE_BOUND, st);
                     {
                         std::lock_guard<std::mutex> lk(m->table_mu);
                         AK_TRY(ensure_reach(m, hp, eff_hops, st));
                     }
-                    AK_TRY(sc->reach_keep.ensure(REACH_T * 4));
-                    AK_TRY(sc->reach_bad.ensure(16));
+                    AK_TRY(sc->reach_keep.ensure((REACH_T + 2) * 4));
                     AK_TRY(sc->reach_plan.ensure(REACH_PLAN_INTS * 4));
                     if (!sc->plan_host) CUDA_TRY(cudaMallocHost((void **)&sc->plan_host, 16));
                     if (!sc->plan_ev)
                         CUDA_TRY(cudaEventCreateWithFlags(&sc->plan_ev, cudaEventDisableTiming));
-                    const int64_t n_lb = m->n_split < 1024 ? m->n_split : 1024;
-                    CUDA_TRY(launch_prune_floor(nullptr, 0, row_lb, hp.split_row, hp.split_order,
-                                                n_lb, k, sc->pfloor.as<float>(), st));
-                    CUDA_TRY(launch_reach_check(row_ub, sc->pfloor.as<float>(),
-                                                m->reach_map.as<int32_t>(), n,
-                                                sc->reach_keep.as<int32_t>(),
-                                                sc->reach_bad.as<int>(), st));
-                    CUDA_TRY(launch_reach_plan(sc->reach_keep.as<int32_t>(), sc->reach_bad.as<int>(),
-                                               m->reach_t.as<int>(), k,
-                                               sc->reach_plan.as<int32_t>(), st));
+                    ReachFlags rf{};
+                    rf.u0 = sc->rmax_u.as<float>();
+                    rf.l0 = sc->rmin_u.as<float>();
+                    rf.mup = m->mass_up.as<float>();
+                    rf.mdn = m->mass_dn.as<float>();
+                    rf.ext = sc->ext.as<unsigned int>();
+                    rf.n = n;
+                    rf.H = eff_hops;
+                    rf.alpha = alpha;
+                    rf.split_row = hp.split_row;
+                    rf.split_order = hp.split_order;
+                    rf.n_lb = m->n_split < 1024 ? m->n_split : 1024;
+                    rf.k = k;
+                    rf.map = m->reach_map.as<int32_t>();
+                    rf.t_cnt = m->reach_t.as<int>();
+                    rf.floor_out = sc->pfloor.as<float>();
+                    rf.ws = sc->reach_keep.as<int32_t>();
+                    rf.plan = sc->reach_plan.as<int32_t>();
+                    CUDA_TRY(launch_reach_flags(rf, st, &ph.launches));
                     CUDA_TRY(cudaMemcpyAsync(sc->plan_host, sc->reach_plan.p, 8,
                                              cudaMemcpyDeviceToHost, st));
                     CUDA_TRY(cudaEventRecord(sc->plan_ev, st));
-                    ph.launches += 3;
                 }
                 {
                     // The candidates' pass is queued before the host learns the
@@ -1389,6 +1403,8 @@ static akashic_status_t retrieve_impl(akashic_mem *m, const uint16_t *q, int32_t
                 if (sc->plan_host[0] == 1) {
                     rc = ColumnRecompute{};   // the buffers hold every candidate
                     reach_done = true;
+                } else {
+                    AK_TRY(row_bounds());     // the hops run: they need every row's bounds
                 }
             }
             for (int h = 0; h < eff_hops && !reach_done; ++h) {

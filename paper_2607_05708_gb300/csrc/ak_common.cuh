@@ -402,6 +402,27 @@ struct KeptScratch {
 cudaError_t launch_mass_levels(const HopPlan &p, int t0, int t1, float *mup, float *mdn,
                                const float *zeros, float *split_vu, float *split_vl,
                                cudaStream_t st);
+// The row bounds of the last hop's output (one row; k_final_bounds writes
+// them for every row, the reach path evaluates them where it needs them):
+// ub_j = (U0_j + Umax sum_t alpha^t Mup[t]_j)(1 + 1e-5),
+// lb_j = (L0_j + Lmin sum_t alpha^t Mdn[t]_j)(1 - 1e-5), Horner over t.
+__device__ __forceinline__ float row_upper_bound(const float *u0, const float *mup, int64_t n,
+                                                 int H, float alpha, float umax, int64_t j) {
+    float c = 0.f;
+    for (int t = H; t >= 1; --t) c = alpha * (c + __ldg(mup + (int64_t)t * n + j));
+    return fmaf(umax, c, u0[j]) * (1.f + 1e-5f);
+}
+__device__ __forceinline__ float row_lower_bound(const float *l0, const float *mdn, int64_t n,
+                                                 int H, float alpha, float lmin, int64_t j) {
+    if (!(lmin < INFINITY)) return 0.f;
+    float c = 0.f;
+    for (int t = H; t >= 1; --t) c = alpha * (c + __ldg(mdn + (int64_t)t * n + j));
+    return fmaf(lmin, c, l0[j]) * (1.f - 1e-5f);
+}
+__device__ __forceinline__ float ext_umax(const unsigned int *ext) { return __uint_as_float(ext[0]); }
+__device__ __forceinline__ float ext_lmin(const unsigned int *ext) {
+    return __uint_as_float(0x7f800000u - ext[1]);
+}
 // Per call: ub / lb [n] from u's row extremes u0 / l0 and the mass levels
 // 1..H.  ext [2]: ext[0] the bits of Umax = max_j u0_j, ext[1] 0x7f800000
 // minus the bits of Lmin = min over u0_j > 0 of l0_j (both maxima, so zero
@@ -481,19 +502,37 @@ struct ReachBuild {
     float *C;                        // [H][n][REACH_T]
 };
 cudaError_t launch_reach_build(const ReachBuild &rb, cudaStream_t st);
-// keep[REACH_T] flags the candidates whose upper bound reaches the floor;
-// *bad counts the other rows that do (the candidates then do not suffice).
-cudaError_t launch_reach_check(const float *ub, const float *floor_p, const int32_t *map,
-                               int64_t n, int32_t *keep, int *bad, cudaStream_t st);
+// The reach path's floor, flags and plan, without the per-row bound arrays:
+// floor = the k-th largest lower bound over the (up to 1024) heaviest split
+// rows, computed for those rows only; then every row's upper bound against
+// it: keep[REACH_T] flags the candidates that reach it, *bad counts the
+// other rows that do, and the last CTA to finish writes the plan (see
+// launch_reach_plan).  ws: int32[REACH_T + 2] scratch (keep, bad, done).
+struct ReachFlags {
+    const float *u0, *l0;            // u's row maxima / minima [n]
+    const float *mup, *mdn;          // mass levels [H + 1][n]
+    const unsigned int *ext;         // Umax / Lmin (launch_final_bounds' encoding)
+    int64_t n;
+    int H;
+    float alpha;
+    const int32_t *split_row, *split_order;
+    int64_t n_lb;                    // heaviest split rows taken for the floor (<= 1024)
+    int k;
+    const int32_t *map;              // row -> candidate slot or -1
+    const int *t_cnt;                // candidates (device)
+    float *floor_out;
+    int32_t *ws;
+    int32_t *plan;                   // [REACH_PLAN_INTS]
+};
+cudaError_t launch_reach_flags(const ReachFlags &f, cudaStream_t st, int *launches);
 int reach_parts();                   // CTAs of the candidates' pass (partial rows)
-// The call's plan on the device (int32[REACH_PLAN_INTS]): plan[0] = 1 when
-// the flagged candidates suffice for top-k (else the hops run), plan[1] =
-// their number nk, plan[2..] their slots in ascending order,
-// plan[REACH_PLAN_WIDE] = 1 when a flagged slot is 64 or above.
+// The call's plan on the device (int32[REACH_PLAN_INTS], written by
+// launch_reach_flags): plan[0] = 1 when the flagged candidates suffice for
+// top-k (else the hops run), plan[1] = their number nk, plan[2..] their
+// slots in ascending order, plan[REACH_PLAN_WIDE] = 1 when a flagged slot
+// is 64 or above.
 constexpr int REACH_PLAN_WIDE = REACH_T + 2;
 constexpr int REACH_PLAN_INTS = REACH_T + 3;
-cudaError_t launch_reach_plan(const int32_t *keep, const int *bad, const int *t_cnt, int k,
-                              int32_t *plan, cudaStream_t st);
 // Rows of the packed coefficients: n rounded up to a whole 64-row stage.
 int64_t reach_pad_rows(int64_t n);
 // Every candidate's combined coefficients sum_t alpha^t C_t as bf16 hi + lo,

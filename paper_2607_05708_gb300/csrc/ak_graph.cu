@@ -992,16 +992,11 @@ __global__ void k_final_bounds(const float *__restrict__ u0, const float *__rest
                                const float *__restrict__ mup, const float *__restrict__ mdn,
                                int64_t n, int H, float alpha, const unsigned int *__restrict__ ext,
                                float *__restrict__ ub, float *__restrict__ lb) {
-    const float umax = __uint_as_float(ext[0]), lmin = __uint_as_float(0x7f800000u - ext[1]);
+    const float umax = ext_umax(ext), lmin = ext_lmin(ext);
     for (int64_t j = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; j < n;
          j += (int64_t)gridDim.x * blockDim.x) {
-        float cu = 0.f, cl = 0.f;
-        for (int t = H; t >= 1; --t) {
-            cu = alpha * (cu + __ldg(mup + (int64_t)t * n + j));
-            cl = alpha * (cl + __ldg(mdn + (int64_t)t * n + j));
-        }
-        ub[j] = fmaf(umax, cu, u0[j]) * (1.f + 1e-5f);
-        lb[j] = lmin < INFINITY ? fmaf(lmin, cl, l0[j]) * (1.f - 1e-5f) : 0.f;
+        ub[j] = row_upper_bound(u0, mup, n, H, alpha, umax, j);
+        lb[j] = row_lower_bound(l0, mdn, n, H, alpha, lmin, j);
     }
 }
 

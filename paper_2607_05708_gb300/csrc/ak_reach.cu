@@ -117,54 +117,108 @@ cudaError_t launch_reach_build(const ReachBuild &rb, cudaStream_t st) {
 }
 
 // ------------------------------------------------------------------ per call
-// Rows whose upper bound reaches the floor: a candidate's slot is flagged,
-// any other row counted in *bad (then the hops run instead).
-__global__ void k_reach_check(const float *__restrict__ ub, const float *__restrict__ floor_p,
-                              const int32_t *__restrict__ map, int64_t n,
-                              int32_t *__restrict__ keep, int *__restrict__ bad) {
-    const float floor_ = *floor_p;
-    int nb = 0;
-    for (int64_t j = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; j < n;
-         j += (int64_t)gridDim.x * blockDim.x) {
-        if (ub[j] >= floor_) {
-            const int32_t t = map[j];
-            if (t >= 0) keep[t] = 1;
-            else ++nb;
-        }
-    }
-    if (nb) atomicAdd(bad, nb);
-}
-
 // The plan of a call, on the device: plan[0] = 1 when the candidates
 // suffice (no other row reaches the floor, at least k of them do, and at
 // least k candidates exist), else 0 and the hops run; plan[1] = nk, the
 // flagged count; plan[2 .. 2 + nk) the flagged slots in ascending order;
-// plan[REACH_PLAN_WIDE] = 1 when one of them is 64 or above.  One CTA of
-// REACH_T threads.
-__global__ __launch_bounds__(REACH_T) void k_reach_plan(const int32_t *__restrict__ keep,
-                                                        const int *__restrict__ bad,
-                                                        const int *__restrict__ t_cnt, int k,
-                                                        int32_t *__restrict__ plan) {
+// plan[REACH_PLAN_WIDE] = 1 when one of them is 64 or above.  Run by one
+// CTA of at least REACH_T threads (every thread calls it).
+__device__ void reach_build_plan(const int32_t *keep, int bad, int t_cnt, int k, int32_t *plan) {
     __shared__ int pre[REACH_T];
     const int t = threadIdx.x;
-    const int f = keep[t] != 0 ? 1 : 0;
-    pre[t] = f;
+    const int f = t < REACH_T && keep[t] != 0 ? 1 : 0;
+    if (t < REACH_T) pre[t] = f;
     __syncthreads();
     for (int o = 1; o < REACH_T; o <<= 1) {          // inclusive scan
-        const int v = t >= o ? pre[t - o] : 0;
+        const int v = t < REACH_T && t >= o ? pre[t - o] : 0;
         __syncthreads();
-        pre[t] += v;
+        if (t < REACH_T) pre[t] += v;
         __syncthreads();
     }
     if (f) plan[2 + pre[t] - 1] = t;
     if (t == REACH_T - 1) {
         const int nk = pre[t];
         plan[1] = nk;
-        plan[0] = (*bad == 0 && nk >= k && *t_cnt >= k) ? 1 : 0;
+        plan[0] = (bad == 0 && nk >= k && t_cnt >= k) ? 1 : 0;
         // a flagged slot in the upper half: the candidates' pass loads all
         // 128 coefficient rows, else the first 64
         plan[REACH_PLAN_WIDE] = nk - pre[REACH_T / 2 - 1] > 0 ? 1 : 0;
     }
+}
+
+// The floor: the k-th largest lower bound over the n_lb heaviest split
+// rows (each query's k-th largest final score reaches it: those k rows
+// score at least their lb for every query), computed for those rows only;
+// one CTA, one (lb bits, position) key per thread, a descending bitonic
+// network (partners within a warp by shuffles, farther ones through a
+// ping-pong pair of shared arrays).  Also clears the flags' scratch.
+__global__ __launch_bounds__(1024) void k_reach_floor(const ReachFlags f) {
+    __shared__ unsigned long long xk[2][1024];
+    const int t = threadIdx.x;
+    if (t < REACH_T + 2) f.ws[t] = 0;                  // keep[], bad, done
+    const float lmin = ext_lmin(f.ext);
+    unsigned long long key =
+        t < f.n_lb ? ((unsigned long long)__float_as_uint(row_lower_bound(
+                          f.l0, f.mdn, f.n, f.H, f.alpha, lmin, f.split_row[f.split_order[t]]))
+                      << 32) | (unsigned long long)(uint32_t)t
+                   : 0ull;
+    int cur = 0;
+    for (int size = 2; size <= 1024; size <<= 1)
+        for (int stride = size >> 1; stride > 0; stride >>= 1) {
+            unsigned long long other;
+            if (stride >= 32) {
+                xk[cur][t] = key;
+                __syncthreads();
+                other = xk[cur][t ^ stride];
+                cur ^= 1;          // the next write goes to the other array
+            } else {
+                other = __shfl_xor_sync(0xffffffffu, key, stride);
+            }
+            const bool keep_max = ((t & size) == 0) == ((t & stride) == 0);
+            key = keep_max ? (key > other ? key : other) : (key < other ? key : other);
+        }
+    if (t == f.k - 1)   // keys now descend with the thread index
+        *f.floor_out = f.n_lb >= f.k ? __uint_as_float((uint32_t)(key >> 32)) : 0.f;
+}
+
+// Rows whose upper bound reaches the floor: a candidate's slot is flagged,
+// any other row counted in bad; the last CTA to finish builds the plan.
+__global__ __launch_bounds__(256) void k_reach_flags(const ReachFlags f) {
+    __shared__ int last;
+    int32_t *keep = f.ws, *bad = f.ws + REACH_T, *done = f.ws + REACH_T + 1;
+    const float floor_ = *f.floor_out, umax = ext_umax(f.ext);
+    int nb = 0;
+    for (int64_t j = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; j < f.n;
+         j += (int64_t)gridDim.x * blockDim.x) {
+        if (row_upper_bound(f.u0, f.mup, f.n, f.H, f.alpha, umax, j) >= floor_) {
+            const int32_t t = f.map[j];
+            if (t >= 0) keep[t] = 1;
+            else ++nb;
+        }
+    }
+    if (nb) atomicAdd(bad, nb);
+    __threadfence();                                   // flags before the count
+    __syncthreads();
+    if (threadIdx.x == 0) last = atomicAdd(done, 1) == (int)gridDim.x - 1;
+    __syncthreads();
+    if (!last) return;
+    __threadfence();                                   // every CTA's flags are visible
+    const volatile int32_t *vk = keep;
+    __shared__ int32_t kf[REACH_T];
+    if (threadIdx.x < REACH_T) kf[threadIdx.x] = vk[threadIdx.x];
+    __syncthreads();
+    reach_build_plan(kf, *(volatile int *)bad, *f.t_cnt, f.k, f.plan);
+}
+
+cudaError_t launch_reach_flags(const ReachFlags &f, cudaStream_t st, int *launches) {
+    if (f.n_lb > 1024 || f.k < 1) return cudaErrorInvalidValue;
+    k_reach_floor<<<1, 1024, 0, st>>>(f);
+    // one row per thread: a few independent loads per row, so the rows in
+    // flight set the rate
+    const int64_t g = ceil_div<int64_t>(f.n, 256);
+    k_reach_flags<<<(unsigned)(g > 0 ? g : 1), 256, 0, st>>>(f);
+    if (launches) *launches += 2;
+    return cudaGetLastError();
 }
 
 // ------------------------------------------------------------------ tensor-core terms
@@ -503,14 +557,6 @@ __global__ __launch_bounds__(256) void k_reach_pack(const float *__restrict__ C,
     }
 }
 
-cudaError_t launch_reach_check(const float *ub, const float *floor_p, const int32_t *map,
-                               int64_t n, int32_t *keep, int *bad, cudaStream_t st) {
-    cudaError_t e = cudaMemsetAsync(keep, 0, REACH_T * 4, st);
-    if (e == cudaSuccess) e = cudaMemsetAsync(bad, 0, 4, st);
-    if (e != cudaSuccess) return e;
-    k_reach_check<<<device_sm_count() * 4, 256, 0, st>>>(ub, floor_p, map, n, keep, bad);
-    return cudaGetLastError();
-}
 
 // Final score of each flagged candidate for each real query column: its u
 // plus the CTAs' partials, appended as a filter key (score bits, ~chunk ID)
@@ -555,11 +601,6 @@ int reach_parts() { return device_sm_count(); }
 
 int64_t reach_pad_rows(int64_t n) { return (n + RM_BK - 1) / RM_BK * RM_BK; }
 
-cudaError_t launch_reach_plan(const int32_t *keep, const int *bad, const int *t_cnt, int k,
-                              int32_t *plan, cudaStream_t st) {
-    k_reach_plan<<<1, REACH_T, 0, st>>>(keep, bad, t_cnt, k, plan);
-    return cudaGetLastError();
-}
 
 cudaError_t launch_reach_pack(const float *C, int64_t n, int H, float alpha, uint16_t *coef_hi,
                               uint16_t *coef_lo, cudaStream_t st) {
