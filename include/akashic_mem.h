@@ -141,11 +141,13 @@ akashic_status_t akashic_mem_update_relations(akashic_mem_t *m, int64_t first, i
  * akashic_mem_sync) if 2 c_b > 80, where exp would leave fp32 range.
  * EINVAL if B < 1, k < 1, k > 64, k > size, hops < 0, hops > 16, alpha < 0
  * or not finite.
- * Does not synchronise, with one exception: with hops = 2, alpha > 0 and
- * 65 to 256 queries in a batch of 256, the call waits on `stream` once per
- * such batch to read which candidate rows the bounds flag (the two-hop
- * path from reach coefficients); the first such call after the graph
- * changed also waits while it builds their graph-only tables.
+ * Does not synchronise, with one exception: with hops = 2, alpha > 0, no
+ * scope and 65 to 256 queries in a batch of 128 or 256, the host waits once
+ * per batch for the device's decision between the two-hop path from reach
+ * coefficients and the hops (an event recorded after a 12-byte copy, not the
+ * whole stream; the candidates' pass is already queued behind it, so the
+ * GPU does not idle); the first such call after the graph changed also waits
+ * while it builds their graph-only tables.
  * Graph-only tables built by a call on one stream are waited for (an event,
  * not a host wait) by calls on every other stream. */
 akashic_status_t akashic_mem_retrieve(akashic_mem_t *m, const uint16_t *q, int32_t B, int32_t k,
@@ -313,6 +315,19 @@ akashic_status_t akashic_mem_softmax_scores_noalloc(const uint16_t *emb, int64_t
                                                     const uint16_t *q, int32_t B,
                                                     float temperature, float *u, float *z,
                                                     float *shift, int32_t *status, void *stream);
+
+/* Check of the failure path of the bounded device waits.  The paper has no
+ * counterpart: this is a library self-test.  Every wait inside the library's
+ * kernels (on a barrier, a copy, a peer's flag) gives up after a bounded number
+ * of polls, records ETIMEOUT in the store's status word and lets its kernel
+ * return, so a fault shows up as an error code and the context stays usable.
+ * This call launches one thread that waits, with that same wait, for a barrier
+ * phase that nothing ever completes, and gives up after `polls` polls (the
+ * kernels' waits allow 2^26).  The next akashic_mem_sync() on `stream` then
+ * returns ETIMEOUT and clears the word; the store is otherwise untouched.
+ * Stream-ordered; does not synchronise.  EINVAL for a NULL store or polls
+ * outside [1, 2^26]. */
+akashic_status_t akashic_mem_check_wait_timeout(akashic_mem_t *m, uint32_t polls, void *stream);
 
 /* Thread-local description of the last failure on this thread ("" if none). */
 const char *akashic_mem_last_error(void);

@@ -32,7 +32,7 @@ EXPORTS = (
     "akashic_mem_phase_times", "akashic_mem_last_error", "akashic_mem_softmax_scores_noalloc",
     "akashic_mem_set_namespace", "akashic_mem_retrieve_scoped", "akashic_mem_delete",
     "akashic_mem_relocate", "akashic_mem_compact_pages", "akashic_mem_page_stats",
-    "akashic_mem_export_pages",
+    "akashic_mem_export_pages", "akashic_mem_check_wait_timeout",
 )
 
 
@@ -81,6 +81,7 @@ def load_library(path: str | None = None):
         "akashic_mem_export_csr": ([V, P64, P64, V, V, V, V, V], ctypes.c_int),
         "akashic_mem_size": ([V, P64, P64], ctypes.c_int),
         "akashic_mem_sync": ([V, V], ctypes.c_int),
+        "akashic_mem_check_wait_timeout": ([V, ctypes.c_uint32, V], ctypes.c_int),
         "akashic_mem_set_profiling": ([V, I32], ctypes.c_int),
         "akashic_mem_phase_times": ([V, ctypes.POINTER(ctypes.c_float), ctypes.POINTER(I32)],
                                     ctypes.c_int),
@@ -314,6 +315,11 @@ class MemStore:
 
     def sync(self, stream=None):
         _check(load_library().akashic_mem_sync(self._h, _stream(self._torch, stream, self.device)))
+
+    def check_wait_timeout(self, polls: int, stream=None):
+        """Queue the bounded-wait self-check: the next sync() raises ETIMEOUT."""
+        _check(load_library().akashic_mem_check_wait_timeout(
+            self._h, int(polls), _stream(self._torch, stream, self.device)))
 
     def set_profiling(self, on: bool):
         _check(load_library().akashic_mem_set_profiling(self._h, int(bool(on))))

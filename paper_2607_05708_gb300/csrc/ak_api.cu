@@ -550,6 +550,16 @@ akashic_status_t akashic_mem_sync(akashic_mem_t *m, void *stream) {
     return check_status(m, (cudaStream_t)stream, "sync");
 }
 
+akashic_status_t akashic_mem_check_wait_timeout(akashic_mem_t *m, uint32_t polls, void *stream) {
+    g_last_error.clear();
+    if (!m) return fail(AKASHIC_EINVAL, "check_wait_timeout: NULL store");
+    if (polls < 1 || polls > (1u << 26))
+        return fail(AKASHIC_EINVAL, "check_wait_timeout: polls must be in [1, 2^26]");
+    DeviceGuard g(m->device);
+    CUDA_TRY(launch_wait_timeout_check(m->status.as<int>(), polls, (cudaStream_t)stream));
+    return AKASHIC_OK;
+}
+
 akashic_status_t akashic_mem_append_chunks(akashic_mem_t *m, const uint16_t *emb, int64_t n,
                                            const int32_t *page_of, const int64_t *row_ptr,
                                            const int32_t *col, const float *aff,

@@ -81,6 +81,9 @@ int64_t score_tiles(int64_t n);
 // each row over the first n_real columns (the real queries), for the
 // propagation's row bounds; with them, ext (optional, [2], zeroed before)
 // gets their extremes in launch_final_bounds' encoding.
+// One thread waits on a barrier that nothing signals, giving up after
+// `polls` polls like every bounded wait (ETIMEOUT into *status).
+cudaError_t launch_wait_timeout_check(int *status, uint32_t polls, cudaStream_t st);
 // Raises the score kernel's shared-memory limit for every query width on the
 // current device now (launch_score does it lazily per width otherwise).
 cudaError_t prepare_score_gemm();

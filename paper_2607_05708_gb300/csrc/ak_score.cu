@@ -228,9 +228,7 @@ __global__ __launch_bounds__(GemmCfg<BP, MODE>::THREADS, 1) void k_gemm_umma(con
     uint8_t *sB = smem + C::STAGES * C::A_BYTES;
     float *sOut = (float *)(smem + C::STAGES * C::STAGE_BYTES);     // 2 x [128][32], swizzled
     uint8_t *misc = smem + C::STAGES * C::STAGE_BYTES + C::OUT_REGION;
-    float *shift_s = (float *)misc;                  // [BP]
-    float *zacc = shift_s + BP;                      // [BP]
-    float *zq = zacc + BP;                           // [4][32]  (ends below misc + 2560)
+    float *shift_s = (float *)misc;                  // [BP]  (ends below misc + 2560)
     int *go = (int *)(misc + 2560);                  // epilogue: the tile's accumulator is ready
     uint64_t *bars = (uint64_t *)(misc + 3072);      // full[S], empty[S], tfull[2], tempty[2]
     uint64_t *full = bars, *empty = bars + C::STAGES;
@@ -266,7 +264,6 @@ __global__ __launch_bounds__(GemmCfg<BP, MODE>::THREADS, 1) void k_gemm_umma(con
     }
     for (int i = threadIdx.x; i < BP; i += blockDim.x) {
         shift_s[i] = EXP ? ep.shift[i] : 0.f;
-        zacc[i] = 0.f;
     }
     tc_fence_before();
     __syncthreads();
@@ -551,6 +548,23 @@ __global__ __launch_bounds__(GemmCfg<BP, MODE>::THREADS, 1) void k_gemm_umma(con
 }
 
 int64_t score_tiles(int64_t n) { return ceil_div<int64_t>(n, 128); }
+
+// The give-up path of the bounded waits, on its own: one thread waits for
+// the first phase of a barrier that nothing arrives on, with the same wait
+// the tensor-core kernels use, and gives up after `polls` polls.
+__global__ void k_wait_timeout_check(int *status, uint32_t polls) {
+    __shared__ uint64_t bar;
+    if (threadIdx.x == 0) {
+        mbar_init(&bar, 1);
+        mbar_fence_init();
+        mbar_wait_n(&bar, 0u, status, polls);
+    }
+}
+
+cudaError_t launch_wait_timeout_check(int *status, uint32_t polls, cudaStream_t st) {
+    k_wait_timeout_check<<<1, 32, 0, st>>>(status, polls);
+    return cudaGetLastError();
+}
 
 // The kernel's dynamic shared-memory limit, raised once per device (with
 // that device current) before its first launch there.

@@ -43,12 +43,17 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t *bar, uint32_t parity) {
         : "memory");
     return ok != 0;
 }
-// Bounded wait for the phase of the given parity to complete.
-__device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity, int *status) {
-    for (uint32_t i = 0; i < WAIT_LIMIT; ++i)
+// Bounded wait for the phase of the given parity to complete: gives up
+// after `limit` polls, records ETIMEOUT in the status word and returns false.
+__device__ __forceinline__ bool mbar_wait_n(uint64_t *bar, uint32_t parity, int *status,
+                                            uint32_t limit) {
+    for (uint32_t i = 0; i < limit; ++i)
         if (mbar_try_wait(bar, parity)) return true;
     set_status(status, AKASHIC_ETIMEOUT);
     return false;
+}
+__device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity, int *status) {
+    return mbar_wait_n(bar, parity, status, WAIT_LIMIT);
 }
 
 // ------------------------------------------------------------------ TMA

@@ -806,3 +806,24 @@ def test_embedding_width_limits(dim):
     wl = dataclasses.replace(base, dim=dim, emb=unit(base.n), queries=unit(37), hops=2, k=16)
     _, got = gpu_retrieve(wl, "id")
     assert_retrieval_parity(wl, "id", got, oracle_retrieve(wl, "id"))
+
+
+def test_bounded_wait_gives_up_and_the_store_stays_usable():
+    """Every device-side wait in the library gives up after a bounded number
+    of polls, records ETIMEOUT and lets its kernel return.  A wait that
+    nothing ever releases (akashic_mem_check_wait_timeout, 1000 polls) must
+    surface as ETIMEOUT at the next sync, the status must then be clear, and
+    a retrieval on the same store must still match the oracle."""
+    from paper_2607_05708_gb300 import AkashicError
+    wl = synth.workload(0)
+    store = gpu_store(wl, "id")
+    store.check_wait_timeout(1000)
+    with pytest.raises(AkashicError) as err:
+        store.sync()
+    assert err.value.code == "ETIMEOUT"
+    store.sync()                                      # the word was cleared
+    _, got = gpu_retrieve(wl, "id", store=store)
+    assert_retrieval_parity(wl, "id", got, oracle_retrieve(wl, "id"))
+    with pytest.raises(AkashicError) as err:
+        store.check_wait_timeout(0)
+    assert err.value.code == "EINVAL"
