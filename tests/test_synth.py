@@ -117,3 +117,26 @@ def test_request_trace():
     h = (1.0 / np.arange(1, 513) ** 1.1).sum()
     assert abs(top[0] / 4000 - 1 / h) < 0.03
     assert (counts > 0).sum() <= 512
+
+
+def test_gmm1m_edge_logits_follow_the_stated_reading():
+    """gmm1m / gmm4m edge logits are 10 * [same mixture component] + ln U with
+    U ~ U(0, 1] (the reading recorded for these sampled graphs, standing in for
+    10 * cos: inside a component the cosine is about 0.9, across about 0): the
+    remainder aff - 10 * same is <= 0, finite and spread like ln U (mean -1,
+    standard deviation 1), and most edges stay inside their component (each
+    draw lands there with probability 0.75, less where a component is too
+    small to hold distinct targets: about 0.65 at this scale)."""
+    wl = synth.workload(2, scale=1 / 64)
+    src = np.repeat(np.arange(wl.n), np.diff(wl.row_ptr))
+    same = wl.component[src] == wl.component[wl.col]
+    rest = wl.aff.astype(np.float64) - 10.0 * same
+    assert np.isfinite(rest).all() and (rest <= 0).all()
+    assert abs(rest.mean() + 1.0) < 0.02            # E[ln U] = -1
+    assert abs(rest.std() - 1.0) < 0.02             # Var[ln U] = 1
+    assert 0.6 <= same.mean() < 0.9
+    # inside a component the cosine is high, across it is near zero
+    E = synth.bf16_to_f32(wl.emb).astype(np.float64)
+    pick = np.random.default_rng(1).choice(src.size, 2000, replace=False)
+    cos = np.einsum("ij,ij->i", E[src[pick]], E[wl.col[pick]])
+    assert cos[same[pick]].mean() > 0.8 and abs(cos[~same[pick]].mean()) < 0.05
