@@ -509,8 +509,8 @@ cudaError_t launch_reach_build(const ReachBuild &rb, cudaStream_t st);
 // floor = the k-th largest lower bound over the (up to 1024) heaviest split
 // rows, computed for those rows only; then every row's upper bound against
 // it: keep[REACH_T] flags the candidates that reach it, *bad counts the
-// other rows that do, and the last CTA to finish writes the plan (see
-// launch_reach_plan).  ws: int32[REACH_T + 2] scratch (keep, bad, done).
+// other rows that do, and the last CTA to finish writes the plan
+// (REACH_PLAN_INTS below).  ws: int32[REACH_T + 2] scratch (keep, bad, done).
 struct ReachFlags {
     const float *u0, *l0;            // u's row maxima / minima [n]
     const float *mup, *mdn;          // mass levels [H + 1][n]
