@@ -182,6 +182,27 @@ __device__ __forceinline__ float row_softmax_weight(float aff, float2 stat) {
 }
 cudaError_t launch_row_softmax(const int64_t *row_ptr, const float *aff, float *w, int64_t n_rows,
                                float2 *rstat, cudaStream_t st);
+// For a wave of 32 consecutive edges of a CSR (lane l holds edge e, all
+// lanes call it; e < ptr[n]): the row of e, given r0 with ptr[r0] <= the
+// wave's first edge.  The 32 row ends after r0 are loaded once (one per
+// lane) and searched by shuffles; an edge past them walks on row by row.
+__device__ __forceinline__ int64_t wave_row(const int64_t *__restrict__ ptr, int64_t n,
+                                            int64_t r0, int64_t e) {
+    const int lane = threadIdx.x & 31;
+    const int64_t idx = r0 + 1 + lane;
+    const int64_t bj = ptr[idx < n ? idx : n];        // end of row r0 + lane
+    int c = 0;                                        // row ends <= e among the first 31
+#pragma unroll
+    for (int step = 16; step >= 1; step >>= 1) {
+        const int64_t b = __shfl_sync(0xffffffffu, bj, c + step - 1);
+        if (b <= e) c += step;
+    }
+    const int64_t last = __shfl_sync(0xffffffffu, bj, 31);
+    if (last > e) return r0 + c;
+    int64_t r = r0 + 32;
+    while (ptr[r + 1] <= e) ++r;
+    return r;
+}
 // The store keeps chunks in HBM in page order: row r holds chunk ext_of[r],
 // chunk c lives in row row_of[c].  The out-edge CSR stays in chunk IDs; the
 // in-edge transpose used by propagation is in rows.
@@ -217,6 +238,8 @@ struct InEdgeUpdate {
     const int32_t *row_of, *ext_of;
     const float2 *rstat;                // per chunk ID: (max, inv) of its out-row
 };
+// The update writes in_w_new for every edge as it places it (old edges
+// moved, new edges placed): row_softmax_weight(aff, rstat[ext_of[src]]).
 struct InEdgeScratch {
     int64_t *inc, *deg, *fwd_off;       // [n+1] each
     uint32_t *keys, *vals, *keys2, *vals2;   // [n_new * M] each

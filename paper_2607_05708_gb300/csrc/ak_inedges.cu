@@ -41,16 +41,21 @@ __global__ void k_in_deg_recip(const int32_t *__restrict__ row_of, int64_t first
         deg[row_of[first + a]] += M;
 }
 
-// Old lists to their new offsets, in order.  Edge-parallel (a row-parallel
-// copy would leave one warp copying a hub's ~10^5..10^6 edges): each warp
-// takes 512 consecutive old edges, finds the row of the first by binary
-// search, and each lane then walks its row index forward with its edges.
+// Old lists to their new offsets, in order, each edge's weight recomputed
+// from its logit and its source's row statistics on the way (a moved edge
+// whose source row did not change gets its old weight back bit for bit).
+// Edge-parallel (a row-parallel copy would leave one warp copying a hub's
+// ~10^5..10^6 edges): each warp takes COPY_PER_LANE waves of 32
+// consecutive old edges; the row of the first comes from a binary search,
+// the rows of a wave from wave_row.
 constexpr int COPY_PER_LANE = 16;
 __global__ void k_copy_in_edges(const int64_t *__restrict__ in_ptr_old,
                                 const int32_t *__restrict__ src_old,
                                 const float *__restrict__ aff_old, int64_t n, int64_t nnz_old,
                                 const int64_t *__restrict__ in_ptr_new,
-                                int32_t *__restrict__ src_new, float *__restrict__ aff_new) {
+                                int32_t *__restrict__ src_new, float *__restrict__ aff_new,
+                                const int32_t *__restrict__ ext_of,
+                                const float2 *__restrict__ rstat, float *__restrict__ w_new) {
     const int lane = threadIdx.x & 31;
     const int64_t per_warp = 32 * COPY_PER_LANE;
     const int64_t w0 = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
@@ -68,15 +73,20 @@ __global__ void k_copy_in_edges(const int64_t *__restrict__ in_ptr_old,
             r = lo;
         }
         r = __shfl_sync(0xffffffffu, r, 0);
-        int64_t next = in_ptr_old[r + 1];
-#pragma unroll 4
         for (int i = 0; i < COPY_PER_LANE; ++i) {
-            const int64_t e = base + 32 * i + lane;
-            if (e >= nnz_old) break;
-            while (next <= e) next = in_ptr_old[++r + 1];
-            const int64_t pos = e + (in_ptr_new[r] - in_ptr_old[r]);
-            src_new[pos] = src_old[e];
-            aff_new[pos] = aff_old[e];
+            const int64_t e0 = base + 32 * i;
+            if (e0 >= nnz_old) break;
+            const int64_t e = e0 + lane < nnz_old ? e0 + lane : nnz_old - 1;
+            const int64_t row = wave_row(in_ptr_old, n, r, e);
+            if (e0 + lane < nnz_old) {
+                const int64_t pos = e + (in_ptr_new[row] - in_ptr_old[row]);
+                const int32_t src = src_old[e];
+                const float a = aff_old[e];
+                src_new[pos] = src;
+                aff_new[pos] = a;
+                w_new[pos] = row_softmax_weight(a, rstat[ext_of[src]]);
+            }
+            r = __shfl_sync(0xffffffffu, row, 31);
         }
     }
 }
@@ -98,14 +108,17 @@ __global__ void k_place_fwd(const uint32_t *__restrict__ order, int64_t pairs,
                             const int64_t *__restrict__ in_ptr_old,
                             const int64_t *__restrict__ in_ptr_new,
                             const int64_t *__restrict__ fwd_off, int32_t *__restrict__ src_new,
-                            float *__restrict__ aff_new) {
+                            float *__restrict__ aff_new, const float2 *__restrict__ rstat,
+                            float *__restrict__ w_new) {
     for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < pairs;
          i += (int64_t)gridDim.x * blockDim.x) {
         const uint32_t p = order[i];
         const int64_t rt = row_of[nbr_ids[p]];
         const int64_t pos = in_ptr_new[rt] + (in_ptr_old[rt + 1] - in_ptr_old[rt]) + (i - fwd_off[rt]);
+        const float a = scale * nbr_cos[p];
         src_new[pos] = row_of[first + p / M];
-        aff_new[pos] = scale * nbr_cos[p];
+        aff_new[pos] = a;
+        w_new[pos] = row_softmax_weight(a, rstat[first + p / M]);   // source: chunk first + p / M
     }
 }
 
@@ -115,7 +128,8 @@ __global__ void k_place_recip(const int32_t *__restrict__ nbr_ids, const float *
                               float scale, int64_t first, int64_t n_new, int M,
                               const int32_t *__restrict__ row_of,
                               const int64_t *__restrict__ in_ptr_new, int32_t *__restrict__ src_new,
-                              float *__restrict__ aff_new) {
+                              float *__restrict__ aff_new, const float2 *__restrict__ rstat,
+                              float *__restrict__ w_new) {
     const int lane = threadIdx.x & 31;
     int64_t a = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
     const int64_t stride = ((int64_t)gridDim.x * blockDim.x) >> 5;
@@ -126,8 +140,10 @@ __global__ void k_place_recip(const int32_t *__restrict__ nbr_ids, const float *
             const int32_t rt = row_of[ids[t]];
             int rank = 0;
             for (int u = 0; u < M; ++u) rank += row_of[ids[u]] < rt;
+            const float af = scale * nbr_cos[a * M + t];
             src_new[o + rank] = rt;
-            aff_new[o + rank] = scale * nbr_cos[a * M + t];
+            aff_new[o + rank] = af;
+            w_new[o + rank] = row_softmax_weight(af, rstat[ids[t]]);   // source: chunk ids[t]
         }
     }
 }
@@ -177,7 +193,8 @@ cudaError_t launch_in_edges_update(const InEdgeUpdate &u, const InEdgeScratch &s
         const int64_t grid = ceil_div<int64_t>(warps, 8);
         k_copy_in_edges<<<(unsigned)(grid < (int64_t)sms * 16 ? grid : (int64_t)sms * 16), 256, 0,
                           st>>>(u.in_ptr_old, u.in_src_old, u.in_aff_old, u.n, nnz_old,
-                                u.in_ptr_new, u.in_src_new, u.in_aff_new);
+                                u.in_ptr_new, u.in_src_new, u.in_aff_new, u.ext_of, u.rstat,
+                                u.in_w_new);
         ++L;
     }
     if (pairs > 0) {
@@ -200,21 +217,20 @@ cudaError_t launch_in_edges_update(const InEdgeUpdate &u, const InEdgeScratch &s
         if (e != cudaSuccess) return e;
         k_place_fwd<<<sms * 2, 256, 0, st>>>(alt2 ? v2 : v1, pairs, u.nbr_ids, u.nbr_cos, u.scale,
                                              u.first, u.M, u.row_of, u.in_ptr_old, u.in_ptr_new,
-                                             s.fwd_off, u.in_src_new, u.in_aff_new);
+                                             s.fwd_off, u.in_src_new, u.in_aff_new, u.rstat,
+                                             u.in_w_new);
         ++L;
         if (u.reciprocal) {
             k_place_recip<<<sms * 2, 256, 0, st>>>(u.nbr_ids, u.nbr_cos, u.scale, u.first, u.n_new,
                                                    u.M, u.row_of, u.in_ptr_new, u.in_src_new,
-                                                   u.in_aff_new);
+                                                   u.in_aff_new, u.rstat, u.in_w_new);
             ++L;
         }
         e = cudaGetLastError();
         if (e != cudaSuccess) return e;
     }
-    e = launch_in_weights(u.in_src_new, u.in_aff_new, u.nnz_new, u.ext_of, u.rstat, u.in_w_new, st);
-    ++L;
     if (launches) *launches += L;
-    return e;
+    return cudaGetLastError();
 }
 
 }  // namespace ak

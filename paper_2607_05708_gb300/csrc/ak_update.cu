@@ -199,18 +199,42 @@ __global__ void k_count_recip(const int32_t *__restrict__ nbr, int64_t pairs,
 }
 
 // Old edges keep their order at the front of each row (one warp per row).
+// Edge-parallel: each warp takes OLD_PER_LANE waves of 32 consecutive old
+// edges; the row of the first comes from a binary search, the rows of a
+// wave from wave_row; edge e of row r goes to nrp[r] + (e - rp[r]).
+constexpr int OLD_PER_LANE = 16;
 __global__ void k_copy_old_rows(const int64_t *__restrict__ rp, const int32_t *__restrict__ col,
                                 const float *__restrict__ aff, int64_t n_rows,
                                 const int64_t *__restrict__ nrp, int32_t *__restrict__ ncol,
                                 float *__restrict__ naff) {
     const int lane = threadIdx.x & 31;
-    int64_t r = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
-    const int64_t stride = ((int64_t)gridDim.x * blockDim.x) >> 5;
-    for (; r < n_rows; r += stride) {
-        const int64_t a = rp[r], b = rp[r + 1], o = nrp[r];
-        for (int64_t e = a + lane; e < b; e += 32) {
-            ncol[o + e - a] = col[e];
-            naff[o + e - a] = aff[e];
+    const int64_t nnz = rp[n_rows];
+    const int64_t per_warp = 32 * OLD_PER_LANE;
+    const int64_t w0 = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    const int64_t nw = ((int64_t)gridDim.x * blockDim.x) >> 5;
+    for (int64_t base = w0 * per_warp; base < nnz; base += nw * per_warp) {
+        int64_t r = 0;                                // largest r with rp[r] <= base
+        if (lane == 0) {
+            int64_t lo = 0, hi = n_rows;
+            while (hi - lo > 1) {
+                const int64_t mid = (lo + hi) >> 1;
+                if (rp[mid] <= base) lo = mid;
+                else hi = mid;
+            }
+            r = lo;
+        }
+        r = __shfl_sync(0xffffffffu, r, 0);
+        for (int i = 0; i < OLD_PER_LANE; ++i) {
+            const int64_t e0 = base + 32 * i;
+            if (e0 >= nnz) break;
+            const int64_t e = e0 + lane < nnz ? e0 + lane : nnz - 1;
+            const int64_t row = wave_row(rp, n_rows, r, e);
+            if (e0 + lane < nnz) {
+                const int64_t pos = nrp[row] + (e - rp[row]);
+                ncol[pos] = col[e];
+                naff[pos] = aff[e];
+            }
+            r = __shfl_sync(0xffffffffu, row, 31);
         }
     }
 }
@@ -289,7 +313,10 @@ akashic_status_t csr_insert(const UpdateArgs &a, const int64_t *rp, const int32_
         e = cudaGetLastError();
         if (e == cudaSuccess) e = scan_exclusive(deg, new_rp, n_rows, tmp, tmp_bytes, st);
         if (e == cudaSuccess) {
-            k_copy_old_rows<<<sms * 8, 256, 0, st>>>(rp, col, aff, n_rows, new_rp, new_col, new_aff);
+            const int64_t warps = ceil_div<int64_t>(nnz, 32 * OLD_PER_LANE);
+            const int64_t g = ceil_div<int64_t>(warps > 0 ? warps : 1, 8);
+            k_copy_old_rows<<<(unsigned)(g < (int64_t)sms * 16 ? g : (int64_t)sms * 16), 256, 0,
+                              st>>>(rp, col, aff, n_rows, new_rp, new_col, new_aff);
             k_fill_new_rows<<<sms * 2, 256, 0, st>>>(a.nbr_ids, a.nbr_cos, a.first, a.n_new, a.M,
                                                      a.scale, new_rp, new_col, new_aff);
             L += 2;
