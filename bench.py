@@ -279,7 +279,8 @@ def run_update(args):
                      "unit": "TFLOP/s", "frac": fl / (relate_ms * 1e-3) / 1e12 / bf16,
                      "traffic": None, "kernel": "relation GEMM + top-M (relate phase)",
                      "peak_kind": kind},
-        "phases_ms_per_step": {p: phases[p][0] / len(times) for p in ("relate", "graph")},
+        "phases_ms_per_step": {p: phases[p][0] / len(times)
+                               for p in ("relate", "graph", "csr_insert", "transpose", "hub_plan")},
         "tensor_frac_of_whole_update": fl / (ms * 1e-3) / 1e12 / bf16,
         "clocks": clk.summary(),
     }

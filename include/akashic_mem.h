@@ -272,7 +272,13 @@ enum {
     AKASHIC_PHASE_COMPACT = 6,   /* block compaction                            */
     AKASHIC_PHASE_BOUND = 7,     /* last hop's row bounds, floor and skip flags */
     AKASHIC_PHASE_LAST_HOP = 8,  /* last hop with the top-k filter fused        */
-    AKASHIC_PHASE_COUNT = 9
+    /* three parts of AKASHIC_PHASE_GRAPH in a relation update, also counted
+     * in it: */
+    AKASHIC_PHASE_CSR_INSERT = 9,  /* new CSR: old rows moved, new rows and
+                                      reciprocal edges placed                 */
+    AKASHIC_PHASE_TRANSPOSE = 10,  /* row softmax and the in-edge transpose   */
+    AKASHIC_PHASE_HUB_PLAN = 11,   /* the hop's hub segment plan rebuilt      */
+    AKASHIC_PHASE_COUNT = 12
 };
 akashic_status_t akashic_mem_set_profiling(akashic_mem_t *m, int32_t on);
 akashic_status_t akashic_mem_phase_times(akashic_mem_t *m, float *ms, int32_t *launches);
@@ -328,6 +334,20 @@ akashic_status_t akashic_mem_softmax_scores_noalloc(const uint16_t *emb, int64_t
  * Stream-ordered; does not synchronise.  EINVAL for a NULL store or polls
  * outside [1, 2^26]. */
 akashic_status_t akashic_mem_check_wait_timeout(akashic_mem_t *m, uint32_t polls, void *stream);
+
+/* Stable sort of n (key, value) pairs of 32-bit words in device memory of the
+ * current device, by the low `bits` bits of the keys (pairs with equal low
+ * bits keep their input order), in place: keys[i] and vals[i] travel
+ * together.  The paper has no counterpart: this is the sort primitive that the
+ * library's own steps use (the in-edge transpose of the relation CSR, the
+ * reciprocal edges of a relation update, the hub plan of the propagation
+ * hop), exported so that it can be checked on its own.  Allocates and frees
+ * its scratch (2n words and the digit histograms) and synchronises `stream`.
+ * EINVAL for n < 0, n > 2^31 - 1, NULL buffers with n > 1, or bits outside
+ * [0, 32]; ENOMEM if the scratch cannot be allocated; ECUDA if a launch fails.
+ * n <= 1 or bits = 0 leaves the buffers untouched. */
+akashic_status_t akashic_mem_sort_pairs(uint32_t *keys, uint32_t *vals, int64_t n, int32_t bits,
+                                        void *stream);
 
 /* Thread-local description of the last failure on this thread ("" if none). */
 const char *akashic_mem_last_error(void);

@@ -17,12 +17,12 @@ from ._build import LIB as LIB_PATH
 from ._build import build
 
 __all__ = ["MemStore", "AkashicError", "load_library", "build", "EXPORTS", "STATUS", "PHASES",
-           "softmax_scores_noalloc"]
+           "softmax_scores_noalloc", "sort_pairs"]
 
 STATUS = {0: "OK", 1: "EINVAL", 2: "ENOMEM", 3: "ECAPACITY", 4: "ECUDA", 5: "ETIMEOUT",
           6: "EDEVICE", 7: "ERANGE"}
 PHASES = ("score", "propagate", "select", "relate", "graph", "relocate", "compact", "bound",
-          "last_hop")
+          "last_hop", "csr_insert", "transpose", "hub_plan")
 
 # Every function declared in include/akashic_mem.h.
 EXPORTS = (
@@ -32,7 +32,7 @@ EXPORTS = (
     "akashic_mem_phase_times", "akashic_mem_last_error", "akashic_mem_softmax_scores_noalloc",
     "akashic_mem_set_namespace", "akashic_mem_retrieve_scoped", "akashic_mem_delete",
     "akashic_mem_relocate", "akashic_mem_compact_pages", "akashic_mem_page_stats",
-    "akashic_mem_export_pages", "akashic_mem_check_wait_timeout",
+    "akashic_mem_export_pages", "akashic_mem_check_wait_timeout", "akashic_mem_sort_pairs",
 )
 
 
@@ -82,6 +82,7 @@ def load_library(path: str | None = None):
         "akashic_mem_size": ([V, P64, P64], ctypes.c_int),
         "akashic_mem_sync": ([V, V], ctypes.c_int),
         "akashic_mem_check_wait_timeout": ([V, ctypes.c_uint32, V], ctypes.c_int),
+        "akashic_mem_sort_pairs": ([V, V, I64, I32, V], ctypes.c_int),
         "akashic_mem_set_profiling": ([V, I32], ctypes.c_int),
         "akashic_mem_phase_times": ([V, ctypes.POINTER(ctypes.c_float), ctypes.POINTER(I32)],
                                     ctypes.c_int),
@@ -127,6 +128,21 @@ def softmax_scores_noalloc(emb, q, u, z, temperature=0.0, shift=None, status=Non
     _check(load_library().akashic_mem_softmax_scores_noalloc(
         _ptr(emb), emb.shape[0], emb.shape[1], _ptr(q), q.shape[0], float(temperature), _ptr(u),
         _ptr(z), _ptr(shift), _ptr(status), ctypes.c_void_p(s.cuda_stream)))
+
+
+def sort_pairs(keys, vals, bits=32, stream=None):
+    """Stable in-place sort of (keys, vals), int32 CUDA tensors of equal
+    length, by the low `bits` bits of the keys, through akashic_mem_sort_pairs
+    (the library's own sort primitive)."""
+    import torch
+    for t, name in ((keys, "keys"), (vals, "vals")):
+        if not t.is_cuda or not t.is_contiguous() or t.dtype != torch.int32:
+            raise ValueError(f"{name} must be a contiguous int32 CUDA tensor")
+    if keys.numel() != vals.numel():
+        raise ValueError("keys and vals differ in length")
+    s = stream if stream is not None else torch.cuda.current_stream(keys.device)
+    _check(load_library().akashic_mem_sort_pairs(_ptr(keys), _ptr(vals), keys.numel(), int(bits),
+                                                 ctypes.c_void_p(s.cuda_stream)))
 
 
 class MemStore:

@@ -216,6 +216,17 @@ struct PhaseScope {
         }
         return e;
     }
+    // close the scope early (once); the destructor then does nothing
+    void end() {
+        if (!m->prof || !a) return;
+        cudaEvent_t b = take_event();
+        if (b) {
+            cudaEventRecord(b, st);
+            std::lock_guard<std::mutex> g(m->mu);
+            m->recs.push_back(ProfRec{phase, a, b, launches});
+        }
+        a = nullptr;
+    }
     ~PhaseScope() {
         if (!m->prof || !a) return;
         cudaEvent_t b = take_event();
@@ -417,11 +428,13 @@ static akashic_status_t build_split_plan(akashic_mem *m, cudaStream_t st) {
     m->n_segs = n_segs;
     m->n_split = n_split;
     if (n_split > 0) {
-        AK_TRY(m->split_row.ensure((size_t)n_split * 4));
-        AK_TRY(m->split_slot0.ensure((size_t)(n_split + 1) * 8));
-        AK_TRY(m->seg_e0.ensure((size_t)n_segs * 8));
-        AK_TRY(m->seg_e1.ensure((size_t)n_segs * 8));
-        AK_TRY(m->seg_slot.ensure((size_t)n_segs * 4));
+        // grown with headroom: every relation update adds a few segments, and
+        // a reallocation would synchronise the device
+        AK_TRY(ensure_spare(m->split_row, (size_t)n_split * 4));
+        AK_TRY(ensure_spare(m->split_slot0, (size_t)(n_split + 1) * 8));
+        AK_TRY(ensure_spare(m->seg_e0, (size_t)n_segs * 8));
+        AK_TRY(ensure_spare(m->seg_e1, (size_t)n_segs * 8));
+        AK_TRY(ensure_spare(m->seg_slot, (size_t)n_segs * 4));
         const Tmp e0 = get(5, (size_t)n_segs * 8), e1 = get(6, (size_t)n_segs * 8);
         const Tmp win = get(7, (size_t)n_segs * 4), order = get(8, (size_t)n_segs * 4);
         const Tmp win2 = get(9, (size_t)n_segs * 4), order2 = get(10, (size_t)n_segs * 4);
@@ -444,7 +457,7 @@ static akashic_status_t build_split_plan(akashic_mem *m, cudaStream_t st) {
                                     m->seg_e0.as<int64_t>(), m->seg_e1.as<int64_t>(),
                                     m->seg_slot.as<int32_t>(), st));
         // split rows heaviest first (the hop's fixup order)
-        AK_TRY(m->split_order.ensure((size_t)n_split * 4));
+        AK_TRY(ensure_spare(m->split_order, (size_t)n_split * 4));
         CUDA_TRY(launch_split_keys(m->split_slot0.as<int64_t>(), n_split, win.as<uint32_t>(),
                                    order.as<uint32_t>(), st));
         bool alt2 = false;
@@ -452,7 +465,7 @@ static akashic_status_t build_split_plan(akashic_mem *m, cudaStream_t st) {
                                   order2.as<uint32_t>(), n_split, 32, rtmp.p, rtmp.cap, st, &alt2));
         CUDA_TRY(cudaMemcpyAsync(m->split_order.p, alt2 ? order2.p : order.p, (size_t)n_split * 4,
                                  cudaMemcpyDeviceToDevice, st));
-        AK_TRY(m->slot_split.ensure((size_t)n_segs * 4));
+        AK_TRY(ensure_spare(m->slot_split, (size_t)n_segs * 4));
         CUDA_TRY(launch_slot_owner(m->split_slot0.as<int64_t>(), n_split,
                                    m->slot_split.as<int32_t>(), st));
         AK_TRY(check_status(m, st, "relation graph rebuild"));
@@ -557,6 +570,35 @@ akashic_status_t akashic_mem_check_wait_timeout(akashic_mem_t *m, uint32_t polls
         return fail(AKASHIC_EINVAL, "check_wait_timeout: polls must be in [1, 2^26]");
     DeviceGuard g(m->device);
     CUDA_TRY(launch_wait_timeout_check(m->status.as<int>(), polls, (cudaStream_t)stream));
+    return AKASHIC_OK;
+}
+
+akashic_status_t akashic_mem_sort_pairs(uint32_t *keys, uint32_t *vals, int64_t n, int32_t bits,
+                                        void *stream) {
+    g_last_error.clear();
+    if (n < 0 || n > 0x7fffffffLL || bits < 0 || bits > 32 || (n > 1 && (!keys || !vals)))
+        return fail(AKASHIC_EINVAL, "sort_pairs: bad n, bits or buffers");
+    if (n <= 1 || bits == 0) return AKASHIC_OK;
+    cudaStream_t st = (cudaStream_t)stream;
+    const size_t words = ((size_t)n * 8 + 255) & ~(size_t)255;
+    const size_t tb = radix_tmp_bytes(n) + 4096;
+    void *buf = nullptr;
+    if (cudaMalloc(&buf, words + tb) != cudaSuccess) {
+        cudaGetLastError();
+        return fail(AKASHIC_ENOMEM, "sort_pairs: %lld bytes of scratch", (long long)(words + tb));
+    }
+    uint32_t *k2 = (uint32_t *)buf, *v2 = k2 + n;
+    bool alt = false;
+    cudaError_t e = radix_sort_pairs(keys, vals, k2, v2, n, bits, (uint8_t *)buf + words, tb, st,
+                                     &alt);
+    if (e == cudaSuccess && alt)
+        e = cudaMemcpyAsync(keys, k2, (size_t)n * 4, cudaMemcpyDeviceToDevice, st);
+    if (e == cudaSuccess && alt)
+        e = cudaMemcpyAsync(vals, v2, (size_t)n * 4, cudaMemcpyDeviceToDevice, st);
+    const cudaError_t es = cudaStreamSynchronize(st);
+    if (e == cudaSuccess) e = es;
+    cudaFree(buf);
+    if (e != cudaSuccess) return fail(AKASHIC_ECUDA, "sort_pairs: %s", cudaGetErrorString(e));
     return AKASHIC_OK;
 }
 
@@ -730,11 +772,17 @@ akashic_status_t akashic_mem_update_relations(akashic_mem_t *m, int64_t first, i
     }
     {
         PhaseScope ph(m, AKASHIC_PHASE_GRAPH, st);
-        akashic_status_t r = csr_insert(ua, m->row_ptr.as<int64_t>(), m->col.as<int32_t>(),
-                                        m->aff.as<float>(), m->nnz, nrp.as<int64_t>(),
-                                        ncol.as<int32_t>(), naff.as<float>(), st, &ph.launches);
-        if (r != AKASHIC_OK) return fail(r, "update: CSR insert failed");
-        AK_TRY(check_status(m, st, "update"));
+        {
+            PhaseScope pc(m, AKASHIC_PHASE_CSR_INSERT, st);
+            akashic_status_t r = csr_insert(ua, m->row_ptr.as<int64_t>(), m->col.as<int32_t>(),
+                                            m->aff.as<float>(), m->nnz, nrp.as<int64_t>(),
+                                            ncol.as<int32_t>(), naff.as<float>(), st,
+                                            &pc.launches);
+            ph.launches += pc.launches;
+            if (r != AKASHIC_OK) return fail(r, "update: CSR insert failed");
+            AK_TRY(check_status(m, st, "update"));
+        }
+        PhaseScope pt(m, AKASHIC_PHASE_TRANSPOSE, st);
         std::swap(m->row_ptr.p, nrp.p);
         std::swap(m->row_ptr.cap, nrp.cap);
         std::swap(m->col.p, ncol.p);
@@ -746,6 +794,7 @@ akashic_status_t akashic_mem_update_relations(akashic_mem_t *m, int64_t first, i
         AK_TRY(m->w.ensure(m->col.cap, false));
         CUDA_TRY(launch_row_softmax(m->row_ptr.as<int64_t>(), m->aff.as<float>(), m->w.as<float>(),
                                     m->n, m->rstat.as<float2>(), st));
+        pt.launches += 1;
         if (!m->inc_transpose || nnz_old == 0) {
             AK_TRY(rebuild_in_edges(m, st));
         } else {
@@ -793,7 +842,7 @@ akashic_status_t akashic_mem_update_relations(akashic_mem_t *m, int64_t first, i
             InEdgeScratch sc{(int64_t *)p_inc, (int64_t *)p_deg, (int64_t *)p_off,
                              (uint32_t *)p_k, (uint32_t *)p_v, (uint32_t *)p_k2, (uint32_t *)p_v2,
                              p_tmp, tb};
-            CUDA_TRY(launch_in_edges_update(u, sc, st, &ph.launches));
+            CUDA_TRY(launch_in_edges_update(u, sc, st, &pt.launches));
             std::swap(m->in_ptr.p, ptr2.p);
             std::swap(m->in_ptr.cap, ptr2.cap);
             std::swap(m->in_src.p, src2.p);
@@ -802,6 +851,9 @@ akashic_status_t akashic_mem_update_relations(akashic_mem_t *m, int64_t first, i
             std::swap(m->in_aff.cap, aff2.cap);
             std::swap(m->in_w.p, w2.p);
             std::swap(m->in_w.cap, w2.cap);
+            pt.end();
+            ph.launches += pt.launches;
+            PhaseScope phub(m, AKASHIC_PHASE_HUB_PLAN, st);
             AK_TRY(build_split_plan(m, st));
         }
     }
@@ -1098,11 +1150,11 @@ static akashic_status_t ensure_mass(akashic_mem *m, const HopPlan &hp, int H, cu
     if (m->mass_levels >= H) return AKASHIC_OK;
     const size_t lv = (size_t)(AKASHIC_MAX_HOPS + 1) * n * 4;
     if (m->mass_levels < 0 || m->mass_up.cap < lv) {
-        AK_TRY(m->mass_up.ensure(lv));
-        AK_TRY(m->mass_dn.ensure(lv));
-        AK_TRY(m->mass_zero.ensure((size_t)n * 4));
-        AK_TRY(m->mass_vu.ensure((size_t)(m->n_split + 1) * 4));
-        AK_TRY(m->mass_vl.ensure((size_t)(m->n_split + 1) * 4));
+        AK_TRY(ensure_spare(m->mass_up, lv));
+        AK_TRY(ensure_spare(m->mass_dn, lv));
+        AK_TRY(ensure_spare(m->mass_zero, (size_t)n * 4));
+        AK_TRY(ensure_spare(m->mass_vu, (size_t)(m->n_split + 1) * 4));
+        AK_TRY(ensure_spare(m->mass_vl, (size_t)(m->n_split + 1) * 4));
         CUDA_TRY(cudaMemsetAsync(m->mass_zero.p, 0, (size_t)n * 4, st));
         CUDA_TRY(launch_fill_f32(m->mass_up.as<float>(), n, 1.f, st));
         CUDA_TRY(launch_fill_f32(m->mass_dn.as<float>(), n, 1.f, st));
@@ -1124,8 +1176,8 @@ static akashic_status_t ensure_reach(akashic_mem *m, const HopPlan &hp, int H, c
     if (m->reach_levels == H && m->reach_n == n) return AKASHIC_OK;
     AK_TRY(m->reach_rows.ensure(REACH_T * 4));
     AK_TRY(m->reach_t.ensure(16));
-    AK_TRY(m->reach_map.ensure((size_t)n * 4));
-    AK_TRY(m->reach_c.ensure((size_t)H * n * REACH_T * 4));
+    AK_TRY(ensure_spare(m->reach_map, (size_t)n * 4));
+    AK_TRY(ensure_spare(m->reach_c, (size_t)H * n * REACH_T * 4));
     ReachBuild rb{};
     rb.n = n;
     rb.n_split = m->n_split;
@@ -1182,30 +1234,30 @@ static akashic_status_t retrieve_impl(akashic_mem *m, const uint16_t *q, int32_t
         const SelectPlan sp = select_plan(n, bp, k, sms);
         AK_TRY(sc->qp.ensure((size_t)bp * m->dim * 2));
         AK_TRY(sc->shift.ensure((size_t)bp * 4));
-        AK_TRY(sc->u.ensure((size_t)n * bp * 4));
-        AK_TRY(sc->zpart.ensure((size_t)tiles * bp * 4));
-        AK_TRY(sc->cand.ensure((size_t)sp.words * 8));
-        if (eff_hops >= 1) AK_TRY(sc->sa.ensure((size_t)n * bp * 4));
-        if (eff_hops >= 2) AK_TRY(sc->sb.ensure((size_t)n * bp * 4));
-        if (eff_hops >= 1 && m->n_segs > 0) AK_TRY(sc->partial.ensure((size_t)m->n_segs * bp * 4));
+        AK_TRY(ensure_spare(sc->u, (size_t)n * bp * 4));
+        AK_TRY(ensure_spare(sc->zpart, (size_t)tiles * bp * 4));
+        AK_TRY(ensure_spare(sc->cand, (size_t)sp.words * 8));
+        if (eff_hops >= 1) AK_TRY(ensure_spare(sc->sa, (size_t)n * bp * 4));
+        if (eff_hops >= 2) AK_TRY(ensure_spare(sc->sb, (size_t)n * bp * 4));
+        if (eff_hops >= 1 && m->n_segs > 0) AK_TRY(ensure_spare(sc->partial, (size_t)m->n_segs * bp * 4));
         if (eff_hops >= 1) AK_TRY(sc->counters.ensure(64));
         // row bounds for the last hop (fused filter only)
         const bool prune = eff_hops >= 1 && m->fuse_filter && m->hop_prune;
         if (prune) {
-            AK_TRY(sc->rmax_u.ensure((size_t)n * 4));
-            AK_TRY(sc->rmin_u.ensure((size_t)n * 4));
-            AK_TRY(sc->ub.ensure((size_t)n * 4));
-            AK_TRY(sc->lb.ensure((size_t)n * 4));
+            AK_TRY(ensure_spare(sc->rmax_u, (size_t)n * 4));
+            AK_TRY(ensure_spare(sc->rmin_u, (size_t)n * 4));
+            AK_TRY(ensure_spare(sc->ub, (size_t)n * 4));
+            AK_TRY(ensure_spare(sc->lb, (size_t)n * 4));
             AK_TRY(sc->ext.ensure(16));
-            AK_TRY(sc->skip_split.ensure((size_t)(m->n_split + 1) * 4));
-            AK_TRY(sc->kept_rows.ensure((size_t)n * 4));
+            AK_TRY(ensure_spare(sc->skip_split, (size_t)(m->n_split + 1) * 4));
+            AK_TRY(ensure_spare(sc->kept_rows, (size_t)n * 4));
             AK_TRY(sc->kept_count.ensure(16));
-            AK_TRY(sc->kept_segs.ensure((size_t)(m->n_segs + 1) * 4));
+            AK_TRY(ensure_spare(sc->kept_segs, (size_t)(m->n_segs + 1) * 4));
             const int64_t nk = n > m->n_segs ? n : m->n_segs;
-            AK_TRY(sc->kflag.ensure((size_t)(nk + 1) * 8));
-            AK_TRY(sc->kpos.ensure((size_t)(nk + 1) * 8));
-            AK_TRY(sc->ktmp.ensure(scan_tmp_bytes(nk + 1) + 4096));
-            AK_TRY(sc->skip_slot.ensure((size_t)(m->n_segs + 1) * 4));
+            AK_TRY(ensure_spare(sc->kflag, (size_t)(nk + 1) * 8));
+            AK_TRY(ensure_spare(sc->kpos, (size_t)(nk + 1) * 8));
+            AK_TRY(ensure_spare(sc->ktmp, scan_tmp_bytes(nk + 1) + 4096));
+            AK_TRY(ensure_spare(sc->skip_slot, (size_t)(m->n_segs + 1) * 4));
             AK_TRY(sc->pfloor.ensure(16));
         }
         const uint16_t *qb = q + (int64_t)off * m->dim;
@@ -1249,20 +1301,20 @@ static akashic_status_t retrieve_impl(akashic_mem *m, const uint16_t *q, int32_t
         if (dense_fused) {
             {
                 PhaseScope ps(m, AKASHIC_PHASE_SELECT, st);
-                AK_TRY(sc->samp.ensure((size_t)sp.n_sample * bp * 4));
-                AK_TRY(sc->ext_s.ensure((size_t)sp.n_sample * 4));
-                AK_TRY(sc->zsamp.ensure((size_t)score_tiles(sp.n_sample) * bp * 4));
+                AK_TRY(ensure_spare(sc->samp, (size_t)sp.n_sample * bp * 4));
+                AK_TRY(ensure_spare(sc->ext_s, (size_t)sp.n_sample * 4));
+                AK_TRY(ensure_spare(sc->zsamp, (size_t)score_tiles(sp.n_sample) * bp * 4));
                 CUDA_TRY(launch_ext_sample(m->ext_of.as<int32_t>(), sp.n_sample, sp.stride,
                                            sc->ext_s.as<int32_t>(), st));
                 NsScope ns_samp{};
                 if (q_ns) {
-                    AK_TRY(sc->ns_s.ensure((size_t)sp.n_sample * 4));
+                    AK_TRY(ensure_spare(sc->ns_s, (size_t)sp.n_sample * 4));
                     CUDA_TRY(launch_ext_sample(m->ns_row.as<int32_t>(), sp.n_sample, sp.stride,
                                                sc->ns_s.as<int32_t>(), st));
                     ns_samp = NsScope{sc->ns_s.as<int32_t>(), sc->qns.as<int32_t>(), nullptr};
                 }
                 if (m->has_dead) {
-                    AK_TRY(sc->dead_s.ensure((size_t)sp.n_sample * 4));
+                    AK_TRY(ensure_spare(sc->dead_s, (size_t)sp.n_sample * 4));
                     CUDA_TRY(launch_ext_sample(m->dead_row.as<int32_t>(), sp.n_sample, sp.stride,
                                                sc->dead_s.as<int32_t>(), st));
                     ns_samp.dead = sc->dead_s.as<int32_t>();
@@ -1388,8 +1440,8 @@ static akashic_status_t retrieve_impl(akashic_mem *m, const uint16_t *q, int32_t
                     if (sc->coef_build != m->reach_build || sc->coef_alpha != alpha ||
                         sc->coef_H != eff_hops || sc->coef_n != n) {
                         const size_t cb = (size_t)REACH_T * reach_pad_rows(n) * 2;
-                        AK_TRY(sc->coef_hi.ensure(cb));
-                        AK_TRY(sc->coef_lo.ensure(cb));
+                        AK_TRY(ensure_spare(sc->coef_hi, cb));
+                        AK_TRY(ensure_spare(sc->coef_lo, cb));
                         CUDA_TRY(launch_reach_pack(m->reach_c.as<float>(), n, eff_hops, alpha,
                                                    sc->coef_hi.as<uint16_t>(),
                                                    sc->coef_lo.as<uint16_t>(), st));

@@ -129,6 +129,15 @@ cudaError_t launch_dots_filter(const uint16_t *emb, int64_t n, int dim, const ui
                                int *status, cudaStream_t st, int *launches,
                                const int32_t *dead_row = nullptr);
 
+// Sampled dots as selection keys, column-major: keys_t[c][j] for the rows
+// j < n (row j*row_stride of emb) and the n_ctiles*256 rows c of qp; the
+// key is the order-preserving bits of the signed dot, or 0 where row j is
+// deleted (dead_row[j], if given) or ext_of[j] >= id_limit.
+cudaError_t launch_dots_keys_t(const uint16_t *emb, int64_t n, int64_t row_stride_rows, int dim,
+                               const uint16_t *qp, int n_ctiles, const int32_t *ext_of,
+                               int64_t id_limit, const int32_t *dead_row, uint32_t *keys_t,
+                               int *status, cudaStream_t st, int *launches);
+
 // Query preparation: pad q (b rows) to bp rows of zeros and compute
 // shift[c] = tau * |q_c| * max_norm (0 for padding); flags ERANGE.
 // ext_zero (or NULL): two words set to 0 (the row extremes' initial value).
@@ -663,6 +672,12 @@ cudaError_t launch_sample_bound_signed(const SelectPlan &sp, const float *s, int
                                        const int32_t *ext_of, int64_t id_limit,
                                        unsigned long long *ws, unsigned long long *bound,
                                        cudaStream_t st, int *launches, NsScope ns = NsScope{});
+// bound[c] = the k-th largest of the n_sample keys keys_t[c][*] (k <= 64) as a
+// key with the chunk-ID half zero, 0 if fewer than k keys are nonzero; ~0
+// for the padding columns b <= c < bp; cnt[c] = 0.  One CTA a column.
+cudaError_t launch_sample_kth_keys(const uint32_t *keys_t, int64_t n_sample, int bp, int b, int k,
+                                   unsigned long long *bound, unsigned int *cnt, cudaStream_t st,
+                                   int *launches);
 // Top-k of each column's filter buffer (no overflow): nbr rows 0..n_cols-1.
 cudaError_t launch_buf_merge_signed(const unsigned int *cnt, const unsigned long long *buf,
                                     int64_t cap, int64_t n_cols, int k, int32_t *nbr_ids,

@@ -81,6 +81,72 @@ __global__ void k_scan_total(const int64_t *__restrict__ in, int64_t *__restrict
     out[n] = n > 0 ? out[n - 1] + in[n - 1] : 0;
 }
 
+// Flat form, for at most SCAN_FLAT_TILES tiles: the tile sums, then each CTA
+// adds up the sums of the tiles before it and scans its own tile; the last
+// CTA writes the total.  Two launches (one for a single tile).
+constexpr int64_t SCAN_FLAT_TILES = 1024;
+
+__device__ __forceinline__ int64_t block_sum_scan(int64_t v, int64_t *wsum) {
+    // the CTA's sum of v, on every thread (wsum: SCAN_THREADS / 32 slots)
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    __syncthreads();
+    if (lane == 0) wsum[warp] = v;
+    __syncthreads();
+    int64_t s = 0;
+#pragma unroll
+    for (int w = 0; w < SCAN_THREADS / 32; ++w) s += wsum[w];
+    return s;
+}
+
+__global__ __launch_bounds__(SCAN_THREADS) void k_scan_reduce(const int64_t *__restrict__ in,
+                                                              int64_t n,
+                                                              int64_t *__restrict__ tile_sum) {
+    __shared__ int64_t wsum[SCAN_THREADS / 32];
+    const int64_t base = (int64_t)blockIdx.x * SCAN_TILE;
+    int64_t s = 0;
+#pragma unroll
+    for (int i = 0; i < SCAN_ITEMS; ++i) {
+        const int64_t idx = base + i * SCAN_THREADS + threadIdx.x;
+        if (idx < n) s += in[idx];
+    }
+    s = block_sum_scan(s, wsum);
+    if (threadIdx.x == 0) tile_sum[blockIdx.x] = s;
+}
+
+__global__ __launch_bounds__(SCAN_THREADS) void k_scan_down(const int64_t *__restrict__ in,
+                                                            int64_t *__restrict__ out, int64_t n,
+                                                            const int64_t *__restrict__ tile_sum) {
+    __shared__ int64_t wsum[SCAN_THREADS / 32];
+    int64_t pre = 0;
+    for (int64_t t = threadIdx.x; t < (int64_t)blockIdx.x; t += SCAN_THREADS) pre += tile_sum[t];
+    pre = block_sum_scan(pre, wsum);
+    __syncthreads();   // wsum is reused below
+    const int64_t base = (int64_t)blockIdx.x * SCAN_TILE + (int64_t)threadIdx.x * SCAN_ITEMS;
+    int64_t v[SCAN_ITEMS];
+    int64_t run = 0;
+#pragma unroll
+    for (int i = 0; i < SCAN_ITEMS; ++i) {
+        const int64_t idx = base + i;
+        v[i] = idx < n ? in[idx] : 0;
+        run += v[i];
+    }
+    const int64_t incl = warp_incl_scan(run);
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    if (lane == 31) wsum[warp] = incl;
+    __syncthreads();
+    int64_t excl = pre + incl - run;
+    for (int w = 0; w < warp; ++w) excl += wsum[w];
+#pragma unroll
+    for (int i = 0; i < SCAN_ITEMS; ++i) {
+        const int64_t idx = base + i;
+        if (idx < n) out[idx] = excl;
+        excl += v[i];
+    }
+    if (blockIdx.x == gridDim.x - 1 && threadIdx.x == SCAN_THREADS - 1) out[n] = excl;
+}
+
 size_t scan_tmp_bytes(int64_t n) {
     size_t tot = 0;
     int64_t m = n;
@@ -111,6 +177,14 @@ static cudaError_t scan_rec(const int64_t *in, int64_t *out, int64_t n, int64_t 
 cudaError_t scan_exclusive(const int64_t *in, int64_t *out, int64_t n, void *tmp,
                            size_t tmp_bytes, cudaStream_t st, int *launches) {
     if (tmp_bytes < scan_tmp_bytes(n)) return cudaErrorInvalidValue;
+    const int64_t tiles = ceil_div<int64_t>(n, SCAN_TILE);
+    if (n > 0 && tiles <= SCAN_FLAT_TILES) {
+        int64_t *sums = (int64_t *)tmp;
+        if (tiles > 1) k_scan_reduce<<<(unsigned)tiles, SCAN_THREADS, 0, st>>>(in, n, sums);
+        k_scan_down<<<(unsigned)tiles, SCAN_THREADS, 0, st>>>(in, out, n, sums);
+        if (launches) *launches += tiles > 1 ? 2 : 1;
+        return cudaGetLastError();
+    }
     cudaError_t e = scan_rec(in, out, n, (int64_t *)tmp, st, launches);
     if (e != cudaSuccess) return e;
     k_scan_total<<<1, 1, 0, st>>>(in, out, n);
@@ -142,19 +216,19 @@ __global__ __launch_bounds__(RS_THREADS) void k_rs_hist(const uint32_t *__restri
     hist[(int64_t)threadIdx.x * n_tiles + blockIdx.x] = h[threadIdx.x];
 }
 
-__global__ __launch_bounds__(RS_THREADS) void k_rs_scatter(
-    const uint32_t *__restrict__ keys, const uint32_t *__restrict__ vals, int64_t n, int shift,
-    uint32_t mask, int64_t n_tiles, const int64_t *__restrict__ offs, uint32_t *__restrict__ okeys,
-    uint32_t *__restrict__ ovals) {
-    __shared__ int cnt[RS_WARPS][256];
-    __shared__ int pre[RS_WARPS][256];
+// Rank the warp's RS_PER_WARP keys of the tile stably by digit: loc[r] is
+// the key's rank among the warp's keys of its digit, cnt[warp][d] the
+// warp's count of digit d; then pre[w][d] = the counts of digit d in the
+// warps before w (one thread a digit).  Keys at or past n get no digit.
+__device__ __forceinline__ void rs_rank(const uint32_t *__restrict__ keys,
+                                        const uint32_t *__restrict__ vals, int64_t n,
+                                        int64_t base, int shift, uint32_t mask,
+                                        uint32_t (&k)[RS_ITEMS], uint32_t (&v)[RS_ITEMS],
+                                        int (&loc)[RS_ITEMS], int (*cnt)[256], int (*pre)[256]) {
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     for (int d = lane; d < 256; d += 32) cnt[warp][d] = 0;
     __syncwarp();
-    const int64_t base = (int64_t)blockIdx.x * RS_TILE + (int64_t)warp * RS_PER_WARP;
     const unsigned lt = (1u << lane) - 1u;
-    uint32_t k[RS_ITEMS], v[RS_ITEMS];
-    int loc[RS_ITEMS];
 #pragma unroll
     for (int r = 0; r < RS_ITEMS; ++r) {
         int64_t idx = base + r * 32 + lane;
@@ -181,6 +255,19 @@ __global__ __launch_bounds__(RS_THREADS) void k_rs_scatter(
         }
     }
     __syncthreads();
+}
+
+__global__ __launch_bounds__(RS_THREADS) void k_rs_scatter(
+    const uint32_t *__restrict__ keys, const uint32_t *__restrict__ vals, int64_t n, int shift,
+    uint32_t mask, int64_t n_tiles, const int64_t *__restrict__ offs, uint32_t *__restrict__ okeys,
+    uint32_t *__restrict__ ovals) {
+    __shared__ int cnt[RS_WARPS][256];
+    __shared__ int pre[RS_WARPS][256];
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int64_t base = (int64_t)blockIdx.x * RS_TILE + (int64_t)warp * RS_PER_WARP;
+    uint32_t k[RS_ITEMS], v[RS_ITEMS];
+    int loc[RS_ITEMS];
+    rs_rank(keys, vals, n, base, shift, mask, k, v, loc, cnt, pre);
 #pragma unroll
     for (int r = 0; r < RS_ITEMS; ++r) {
         int64_t idx = base + r * 32 + lane;
@@ -189,6 +276,90 @@ __global__ __launch_bounds__(RS_THREADS) void k_rs_scatter(
             int64_t pos = offs[(int64_t)d * n_tiles + blockIdx.x] + pre[warp][d] + loc[r];
             okeys[pos] = k[r];
             ovals[pos] = v[r];
+        }
+    }
+}
+
+// Small sorts (at most RS_SMALL_TILES tiles) take one launch a pass after a
+// first histogram launch.  Histograms are int32, digit-major [256][n_tiles].
+// Each scatter CTA derives its own offsets from the pass's histograms (the
+// totals of the smaller digits plus its digit's counts in the tiles before
+// it) and counts the next pass's digit of every key it places into the next
+// histograms, by destination tile.  Three histogram buffers rotate: pass p
+// reads H[p % 3], counts into H[(p+1) % 3] (zero by then) and zeroes its
+// column of H[(p+2) % 3], which pass p-1 read and pass p+1 counts into.
+constexpr int64_t RS_SMALL_TILES = 64;
+
+__global__ __launch_bounds__(RS_THREADS) void k_rs_hist32(const uint32_t *__restrict__ keys,
+                                                          int64_t n, int shift, uint32_t mask,
+                                                          int n_tiles, int *__restrict__ hist,
+                                                          int *__restrict__ zero1,
+                                                          int *__restrict__ zero2) {
+    __shared__ int h[256];
+    h[threadIdx.x] = 0;
+    __syncthreads();
+    const int64_t base = (int64_t)blockIdx.x * RS_TILE;
+    for (int i = threadIdx.x; i < RS_TILE; i += RS_THREADS) {
+        int64_t idx = base + i;
+        if (idx < n) atomicAdd(&h[(keys[idx] >> shift) & mask], 1);
+    }
+    __syncthreads();
+    const int64_t at = (int64_t)threadIdx.x * n_tiles + blockIdx.x;
+    hist[at] = h[threadIdx.x];
+    zero1[at] = 0;
+    zero2[at] = 0;
+}
+
+__global__ __launch_bounds__(RS_THREADS) void k_rs_scatter_small(
+    const uint32_t *__restrict__ keys, const uint32_t *__restrict__ vals, int64_t n, int shift,
+    uint32_t mask, int n_tiles, const int *__restrict__ hcur, int *__restrict__ hnext,
+    int shift_next, uint32_t mask_next, int *__restrict__ hzero, uint32_t *__restrict__ okeys,
+    uint32_t *__restrict__ ovals) {
+    __shared__ int cnt[RS_WARPS][256];
+    __shared__ int pre[RS_WARPS][256];
+    __shared__ int off_s[256];
+    __shared__ int wtot[RS_WARPS];
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    {
+        // thread d: digit d's total and its count in the tiles before this one
+        const int d = threadIdx.x;
+        const int *row = hcur + (int64_t)d * n_tiles;
+        int tot = 0, before = 0;
+#pragma unroll 8
+        for (int t = 0; t < n_tiles; ++t) {
+            const int c = row[t];
+            tot += c;
+            before += t < (int)blockIdx.x ? c : 0;
+        }
+        int incl = tot;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int x = __shfl_up_sync(0xffffffffu, incl, o);
+            if (lane >= o) incl += x;
+        }
+        if (lane == 31) wtot[warp] = incl;
+        __syncthreads();
+        int wpre = 0;
+        for (int w = 0; w < warp; ++w) wpre += wtot[w];
+        off_s[d] = wpre + incl - tot + before;
+        if (hzero) hzero[(int64_t)d * n_tiles + blockIdx.x] = 0;
+    }
+    const int64_t base = (int64_t)blockIdx.x * RS_TILE + (int64_t)warp * RS_PER_WARP;
+    uint32_t k[RS_ITEMS], v[RS_ITEMS];
+    int loc[RS_ITEMS];
+    rs_rank(keys, vals, n, base, shift, mask, k, v, loc, cnt, pre);   // syncs the CTA
+#pragma unroll
+    for (int r = 0; r < RS_ITEMS; ++r) {
+        int64_t idx = base + r * 32 + lane;
+        if (idx < n) {
+            uint32_t d = (k[r] >> shift) & mask;
+            const int pos = off_s[d] + pre[warp][d] + loc[r];
+            okeys[pos] = k[r];
+            ovals[pos] = v[r];
+            if (hnext)
+                atomicAdd(&hnext[(int64_t)((k[r] >> shift_next) & mask_next) * n_tiles +
+                                 pos / RS_TILE],
+                          1);
         }
     }
 }
@@ -213,6 +384,29 @@ cudaError_t radix_sort_pairs(uint32_t *keys, uint32_t *vals, uint32_t *keys_alt,
     void *stmp = (void *)(offs + m + 1);
     size_t stmp_bytes = tmp_bytes - (size_t)(2 * m + 1) * sizeof(int64_t);
     uint32_t *ki = keys, *vi = vals, *ko = keys_alt, *vo = vals_alt;
+    if (n_tiles <= RS_SMALL_TILES) {
+        int *h[3] = {(int *)tmp, (int *)tmp + m, (int *)tmp + 2 * m};
+        const int nt = (int)n_tiles;
+        k_rs_hist32<<<nt, RS_THREADS, 0, st>>>(ki, n, 0, bits < 8 ? (1u << bits) - 1u : 0xffu, nt,
+                                               h[0], h[1], h[2]);
+        if (launches) *launches += 1;
+        for (int p = 0, sh = 0; sh < bits; ++p, sh += 8) {
+            const int nb = bits - sh < 8 ? bits - sh : 8;
+            const int shn = sh + 8;
+            const int nbn = bits - shn < 8 ? bits - shn : 8;
+            k_rs_scatter_small<<<nt, RS_THREADS, 0, st>>>(
+                ki, vi, n, sh, (1u << nb) - 1u, nt, h[p % 3], shn < bits ? h[(p + 1) % 3] : nullptr,
+                shn, shn < bits ? (1u << nbn) - 1u : 0u, p >= 1 ? h[(p + 2) % 3] : nullptr, ko, vo);
+            if (launches) *launches += 1;
+            cudaError_t e = cudaGetLastError();
+            if (e != cudaSuccess) return e;
+            uint32_t *t;
+            t = ki; ki = ko; ko = t;
+            t = vi; vi = vo; vo = t;
+            *result_in_alt = !*result_in_alt;
+        }
+        return cudaSuccess;
+    }
     for (int sh = 0; sh < bits; sh += 8) {
         int nb = bits - sh < 8 ? bits - sh : 8;
         uint32_t mask = (1u << nb) - 1u;

@@ -151,7 +151,13 @@ cudaError_t make_tmap_2d(CUtensorMap *map, const void *base, CUtensorMapDataType
 //                  store: exp, column sums toward Z, and every value whose
 //                  key clears its query's bound appended to that query's
 //                  buffer (retrieval without hops)
-enum GemmMode { GEMM_EXP = 0, GEMM_RAW = 1, GEMM_FILTER = 2, GEMM_EXP_FILTER = 3 };
+//     GEMM_KEYS_T  the dots as signed selection keys, written column-major
+//                  (keys_t[col][row], plain coalesced stores: a warp writes
+//                  32 consecutive rows of one column at a time); rows that
+//                  are deleted or whose chunk ID is >= id_limit get key 0
+//                  (the sample of the relation update's bound)
+enum GemmMode { GEMM_EXP = 0, GEMM_RAW = 1, GEMM_FILTER = 2, GEMM_EXP_FILTER = 3,
+                GEMM_KEYS_T = 4 };
 
 struct GemmEpi {
     const float *shift;                 // EXP: [BP]
@@ -168,6 +174,7 @@ struct GemmEpi {
     NsScope ns;                         // EXP_FILTER: namespace scope of the queries
     const int32_t *dead_row;            // EXP, EXP_FILTER, FILTER: deleted rows (or NULL):
                                         // no score (u = 0) / never a filter candidate
+    uint32_t *keys_t;                   // KEYS_T: [n_ctiles * BP][n_rows]
     float *row_max, *row_min;           // EXP (or NULL): [n_rows] largest / smallest u of
     int n_real;                         // the row over the first n_real columns
     unsigned int *ext;                  // with row_max (or NULL), atomically maxed, zeroed
@@ -193,7 +200,8 @@ struct GemmCfg {
     static constexpr int OUT_BYTES = BM * 32 * 4;
     // the filter epilogue stores nothing: its region only holds the tile's
     // column bounds, and the freed space goes to pipeline stages
-    static constexpr int OUT_REGION = MODE == GEMM_FILTER ? (BP * 12 < 1024 ? 1024 : BP * 12)
+    static constexpr int OUT_REGION = (MODE == GEMM_FILTER || MODE == GEMM_KEYS_T)
+                                          ? (BP * 12 < 1024 ? 1024 : BP * 12)
                                       : MODE == GEMM_EXP_FILTER ? 2 * OUT_BYTES + BP * 12
                                                                 : 2 * OUT_BYTES;
     static constexpr int MISC = 4096;   // shift, Z sums, flags, barriers
@@ -204,7 +212,7 @@ struct GemmCfg {
     // epilogue warps: the filter epilogue is issue-bound (one compare per
     // dot), so it runs two warps per TMEM lane quarter, each on half the
     // columns; the storing epilogues run one
-    static constexpr int EPI_W = (MODE == GEMM_FILTER && BP >= 64) ? 8 : 4;
+    static constexpr int EPI_W = ((MODE == GEMM_FILTER || MODE == GEMM_KEYS_T) && BP >= 64) ? 8 : 4;
     static constexpr int EPI_T = 32 * EPI_W;
     static constexpr int THREADS = 64 + EPI_T;
     static constexpr int SMEM = 1024 + STAGES * STAGE_BYTES + OUT_REGION + MISC;
@@ -222,6 +230,7 @@ __global__ __launch_bounds__(GemmCfg<BP, MODE>::THREADS, 1) void k_gemm_umma(con
     constexpr bool EXPF = MODE == GEMM_EXP_FILTER;
     constexpr bool EXP = MODE == GEMM_EXP || EXPF;
     constexpr bool FILTER = MODE == GEMM_FILTER;
+    constexpr bool KEYST = MODE == GEMM_KEYS_T;
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = (uint8_t *)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
     uint8_t *sA = smem;
@@ -382,6 +391,7 @@ __global__ __launch_bounds__(GemmCfg<BP, MODE>::THREADS, 1) void k_gemm_umma(con
                 in_rows && (MODE == GEMM_RAW || !ep.dead_row || !ep.dead_row[grow]);
             uint32_t fid = 0;
             bool fok = false;
+            const bool kok = KEYST && valid && (int64_t)ep.ext_of[grow] < ep.id_limit;
             float rmax = 0.f, rmin = INFINITY;           // u >= 0
             if ((FILTER || EXPF) && valid) {
                 const int32_t id = ep.ext_of[grow];
@@ -394,7 +404,14 @@ __global__ __launch_bounds__(GemmCfg<BP, MODE>::THREADS, 1) void k_gemm_umma(con
                 uint32_t r[32];
                 tmem_ld32(tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * BP + ch * 32), r);
                 tmem_ld_wait();
-                if constexpr (FILTER) {
+                if constexpr (KEYST) {
+                    if (in_rows) {
+                        uint32_t *kt = ep.keys_t + (ct * BP + ch * 32) * n_rows + grow;
+#pragma unroll
+                        for (int i = 0; i < 32; ++i)
+                            kt[(int64_t)i * n_rows] = kok ? ordered_bits(__uint_as_float(r[i])) : 0u;
+                    }
+                } else if constexpr (FILTER) {
                     if (fok) {
                         // one float compare per dot, branch-free, into a mask;
                         // the exact key test only for the few flagged
@@ -606,7 +623,7 @@ static cudaError_t gemm_bp(const uint16_t *emb, int64_t n_rows, int64_t row_stri
     if (e == cudaSuccess)
         e = make_tmap_2d(&tb, qp, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, (uint64_t)dim,
                          (uint64_t)n_ctiles * BP, (uint64_t)dim * 2, 64, BP);
-    if (e == cudaSuccess && MODE != GEMM_FILTER && MODE != GEMM_EXP_FILTER)
+    if (e == cudaSuccess && MODE != GEMM_FILTER && MODE != GEMM_EXP_FILTER && MODE != GEMM_KEYS_T)
         e = make_tmap_2d(&tc, out, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, (uint64_t)n_ctiles * BP,
                          (uint64_t)n_rows, (uint64_t)n_ctiles * BP * 4, 32, 128);
     else
@@ -724,6 +741,22 @@ cudaError_t launch_dots_filter(const uint16_t *emb, int64_t n, int dim, const ui
     ep.cap = cap;
     cudaError_t e = gemm_dispatch<GEMM_FILTER>(emb, n, 1, dim, qp, 256, n_ctiles, nullptr, ep, st,
                                                nullptr);
+    if (launches) *launches += 1;
+    return e;
+}
+
+cudaError_t launch_dots_keys_t(const uint16_t *emb, int64_t n, int64_t row_stride_rows, int dim,
+                               const uint16_t *qp, int n_ctiles, const int32_t *ext_of,
+                               int64_t id_limit, const int32_t *dead_row, uint32_t *keys_t,
+                               int *status, cudaStream_t st, int *launches) {
+    GemmEpi ep{};
+    ep.dead_row = dead_row;
+    ep.status = status;
+    ep.ext_of = ext_of;
+    ep.id_limit = id_limit;
+    ep.keys_t = keys_t;
+    cudaError_t e = gemm_dispatch<GEMM_KEYS_T>(emb, n, row_stride_rows, dim, qp, 256, n_ctiles,
+                                               nullptr, ep, st, nullptr);
     if (launches) *launches += 1;
     return e;
 }

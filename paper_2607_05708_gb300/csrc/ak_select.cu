@@ -286,6 +286,166 @@ __global__ __launch_bounds__(SEL_THREADS) void k_sample_kth(
     }
 }
 
+// bound[c] from column c of keys_t, split over KS_WARPS warps.  Each warp
+// scans a contiguous share of the column and keeps, in its own shared
+// buffer, every key above a running threshold t (0 at first: key 0 marks a
+// row that is out of the selection).  When the buffer is full it is cut to
+// its k largest keys (the keys above its k-th largest key x, then copies of
+// x up to k) and t becomes x: every key outside the buffer is then <= t <=
+// every key inside, so the k-th largest of the buffer stays the k-th
+// largest of the warp's share.  At the end each warp cuts its buffer to at
+// most k keys, and warp 0 selects the k-th largest of their union.
+constexpr int KS_WARPS = 4, KS_BUF = 512, KS_U = 16, KS_KMAX = 64;
+
+// The k-th largest (1 <= k <= len) of a[0..len) by one warp: MSB-first
+// radix select, 8 bits a pass, on a 256-bin histogram h of the warp's own.
+__device__ uint32_t warp_kth(const uint32_t *a, int len, int k, int *h) {
+    const int lane = threadIdx.x & 31;
+    uint32_t prefix = 0u, pmask = 0u;
+    int rem = k;
+    for (int sh = 24; sh >= 0; sh -= 8) {
+        for (int i = lane; i < 256; i += 32) h[i] = 0;
+        __syncwarp();
+        for (int i = lane; i < len; i += 32) {
+            const uint32_t x = a[i];
+            if ((x & pmask) == prefix) atomicAdd(&h[(x >> sh) & 255u], 1);
+        }
+        __syncwarp();
+        // lane l owns digits 255 - 8l - j (j = 0..7), largest first
+        int c[8], tot = 0;
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+            c[j] = h[255 - 8 * lane - j];
+            tot += c[j];
+        }
+        int incl = tot;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int x = __shfl_up_sync(0xffffffffu, incl, o);
+            if (lane >= o) incl += x;
+        }
+        const int before = incl - tot;               // keys with a larger digit
+        const bool mine = before < rem && incl >= rem;
+        int dig = 0, run = before, above = 0;
+        bool hit = false;
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+            if (mine && !hit && run + c[j] >= rem) {
+                hit = true;
+                dig = 255 - 8 * lane - j;
+                above = run;
+            }
+            run += c[j];
+        }
+        const int src = __ffs(__ballot_sync(0xffffffffu, mine)) - 1;
+        dig = __shfl_sync(0xffffffffu, dig, src);
+        above = __shfl_sync(0xffffffffu, above, src);
+        prefix |= (uint32_t)dig << sh;
+        pmask |= 255u << sh;
+        rem -= above;
+        __syncwarp();
+    }
+    return prefix;
+}
+
+// Cut a[0..len) (len >= k) to its k largest; returns the k-th largest.
+__device__ uint32_t warp_cut(uint32_t *a, int len, int k, int *h) {
+    const int lane = threadIdx.x & 31;
+    const unsigned lt = (1u << lane) - 1u;
+    const uint32_t x = warp_kth(a, len, k, h);
+    int out = 0;
+    for (int i0 = 0; i0 < len; i0 += 32) {
+        const uint32_t v = i0 + lane < len ? a[i0 + lane] : 0u;
+        const bool keep = i0 + lane < len && v > x;
+        const unsigned bal = __ballot_sync(0xffffffffu, keep);
+        __syncwarp();
+        if (keep) a[out + __popc(bal & lt)] = v;   // out + rank <= i0 + lane: already read
+        out += __popc(bal);
+        __syncwarp();
+    }
+    for (int j = out + lane; j < k; j += 32) a[j] = x;
+    __syncwarp();
+    return x;
+}
+
+__global__ __launch_bounds__(KS_WARPS * 32) void k_sample_kth_split(
+    const uint32_t *__restrict__ keys_t, int64_t n_sample, int b, int k,
+    unsigned long long *__restrict__ bound, unsigned int *__restrict__ cnt) {
+    __shared__ uint32_t buf[KS_WARPS][KS_BUF];
+    __shared__ int hist[KS_WARPS][256];
+    __shared__ int lens[KS_WARPS];
+    const int c = blockIdx.x, warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    if (c >= b) {   // padding column: nothing passes the filter
+        if (threadIdx.x == 0) {
+            bound[c] = ~0ull;
+            cnt[c] = 0u;
+        }
+        return;
+    }
+    const unsigned lt = (1u << lane) - 1u;
+    const uint32_t *col = keys_t + (int64_t)c * n_sample;
+    const int64_t share = (n_sample + KS_WARPS - 1) / KS_WARPS;
+    const int64_t v_lo = warp * share;
+    const int64_t v_hi = v_lo + share < n_sample ? v_lo + share : n_sample;
+    uint32_t *a = buf[warp];
+    uint32_t t = 0u;
+    int len = 0;
+    for (int64_t v0 = v_lo; v0 < v_hi; v0 += 32 * KS_U) {
+        uint32_t x[KS_U];
+#pragma unroll
+        for (int u = 0; u < KS_U; ++u) {
+            const int64_t v = v0 + u * 32 + lane;
+            x[u] = v < v_hi ? __ldcs(col + v) : 0u;
+        }
+#pragma unroll
+        for (int u = 0; u < KS_U; ++u) {
+            const bool p = x[u] > t;
+            const unsigned bal = __ballot_sync(0xffffffffu, p);
+            if (bal) {
+                if (len + 32 > KS_BUF) {
+                    t = warp_cut(a, len, k, hist[warp]);
+                    len = k;
+                }
+                const bool q = p && x[u] > t;       // the cut may have raised t
+                const unsigned bq = __ballot_sync(0xffffffffu, q);
+                if (q) a[len + __popc(bq & lt)] = x[u];
+                len += __popc(bq);
+                __syncwarp();
+            }
+        }
+    }
+    if (len > k) {
+        warp_cut(a, len, k, hist[warp]);
+        len = k;
+    }
+    if (lane == 0) lens[warp] = len;
+    __syncthreads();
+    if (warp == 0) {
+        // the survivors of all warps, gathered behind warp 0's own
+        int tot = lens[0];
+        for (int w = 1; w < KS_WARPS; ++w) {
+            for (int i = lane; i < lens[w]; i += 32) a[tot + i] = buf[w][i];
+            tot += lens[w];
+        }
+        __syncwarp();
+        const uint32_t x = tot >= k ? warp_kth(a, tot, k, hist[0]) : 0u;
+        if (lane == 0) {
+            bound[c] = (unsigned long long)x << 32;
+            cnt[c] = 0u;
+        }
+    }
+}
+
+cudaError_t launch_sample_kth_keys(const uint32_t *keys_t, int64_t n_sample, int bp, int b, int k,
+                                   unsigned long long *bound, unsigned int *cnt, cudaStream_t st,
+                                   int *launches) {
+    if (k < 1 || k > KS_KMAX || bp < 1 || b > bp || KS_WARPS * KS_KMAX > KS_BUF)
+        return cudaErrorInvalidValue;
+    k_sample_kth_split<<<bp, KS_WARPS * 32, 0, st>>>(keys_t, n_sample, b, k, bound, cnt);
+    if (launches) *launches += 1;
+    return cudaGetLastError();
+}
+
 // ------------------------------------------------------------------ filter pass
 template <int BP>
 struct SelShape {

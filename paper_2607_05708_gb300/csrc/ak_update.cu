@@ -89,8 +89,9 @@ akashic_status_t relate_top_m(const UpdateArgs &a, cudaStream_t st, int *launche
     stride = stride < 1 ? 1 : (stride > 64 ? 64 : stride);
     const int64_t n_sample = ceil_div<int64_t>(n, stride);
     const int64_t cap = 4 * (int64_t)a.M * stride > 8192 ? 4 * (int64_t)a.M * stride : 8192;
-    // the sample bounds of G column tiles come from one dots GEMM, one
-    // transpose and one k-th launch (G tiles of sampled dots: <= 512 MB)
+    // the sample bounds of G column tiles come from one dots GEMM that
+    // writes the sampled keys column-major and one k-th launch (G tiles of
+    // sampled keys: <= 512 MB)
     const int64_t tile_bytes = n_sample * 256 * 4;
     int64_t G = ((int64_t)512 << 20) / tile_bytes;
     G = G < 1 ? 1 : (G > n_ct ? n_ct : G);
@@ -99,14 +100,13 @@ akashic_status_t relate_top_m(const UpdateArgs &a, cudaStream_t st, int *launche
     sp.off_tr = sp.off_buf;
     sp.words = sp.off_tr + ceil_div<int64_t>(sp.n_sample * sp.bp, 2);
     uint16_t *qp = (uint16_t *)a.get(SCR_QP, (size_t)n_pad * a.dim * 2);
-    float *sdots = (float *)a.get(SCR_SDOTS, (size_t)G * tile_bytes);
     int32_t *ext_s = (int32_t *)a.get(SCR_EXTS, (size_t)n_sample * 4);
     unsigned long long *ws = (unsigned long long *)a.get(SCR_WS, (size_t)sp.words * 8);
     unsigned long long *bound = (unsigned long long *)a.get(SCR_BOUND, (size_t)n_pad * 8);
     unsigned int *cnt = (unsigned int *)a.get(SCR_CNT, (size_t)n_pad * 4);
     unsigned long long *buf = (unsigned long long *)a.get(SCR_BUF, (size_t)a.n_new * cap * 8);
     akashic_status_t rc =
-        (qp && sdots && ext_s && ws && bound && cnt && buf) ? AKASHIC_OK : AKASHIC_ENOMEM;
+        (qp && ext_s && ws && bound && cnt && buf) ? AKASHIC_OK : AKASHIC_ENOMEM;
     cudaError_t e = cudaSuccess;
     bool overflow = false;
     if (rc == AKASHIC_OK) {
@@ -115,28 +115,27 @@ akashic_status_t relate_top_m(const UpdateArgs &a, cudaStream_t st, int *launche
         k_ext_sample<<<sms, 256, 0, st>>>(a.ext_of, n_sample, stride, ext_s);
         e = cudaGetLastError();
         // deleted chunks are never neighbours: their sample rows carry no key
-        NsScope dscope{};
+        const int32_t *dead_s = nullptr;
         if (e == cudaSuccess && a.dead_row) {
-            int32_t *dead_s = (int32_t *)a.get(SCR_DEAD_S, (size_t)n_sample * 4);
-            if (!dead_s) {
+            int32_t *ds = (int32_t *)a.get(SCR_DEAD_S, (size_t)n_sample * 4);
+            if (!ds) {
                 rc = AKASHIC_ENOMEM;
             } else {
-                k_ext_sample<<<sms, 256, 0, st>>>(a.dead_row, n_sample, stride, dead_s);
+                k_ext_sample<<<sms, 256, 0, st>>>(a.dead_row, n_sample, stride, ds);
                 e = cudaGetLastError();
-                dscope = NsScope{nullptr, nullptr, dead_s};
+                dead_s = ds;
             }
         }
         for (int64_t g0 = 0; rc == AKASHIC_OK && e == cudaSuccess && g0 < n_ct; g0 += G) {
             const int gt = (int)(n_ct - g0 < G ? n_ct - g0 : G);
             const int64_t left = a.n_new - g0 * 256;
             const int b = (int)(left < (int64_t)gt * 256 ? left : (int64_t)gt * 256);
-            SelectPlan spg = sp;
-            spg.bp = gt * 256;
-            e = launch_dots(a.emb, n_sample, stride, a.dim, qp + g0 * 256 * a.dim, 256, gt, sdots,
-                            a.status, st, launches);
+            uint32_t *keys_t = (uint32_t *)(ws + sp.off_tr);
+            e = launch_dots_keys_t(a.emb, n_sample, stride, a.dim, qp + g0 * 256 * a.dim, gt,
+                                   ext_s, a.first, dead_s, keys_t, a.status, st, launches);
             if (e == cudaSuccess)
-                e = launch_sample_bound_signed(spg, sdots, b, ext_s, a.first, ws, bound + g0 * 256,
-                                               st, launches, dscope);
+                e = launch_sample_kth_keys(keys_t, n_sample, gt * 256, b, a.M, bound + g0 * 256,
+                                           (unsigned int *)(ws + sp.off_cnt), st, launches);
         }
         if (rc == AKASHIC_OK && e == cudaSuccess) e = cudaMemsetAsync(cnt, 0, (size_t)n_pad * 4, st);
         if (rc == AKASHIC_OK && e == cudaSuccess)

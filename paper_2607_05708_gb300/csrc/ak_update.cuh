@@ -7,7 +7,7 @@ namespace ak {
 
 // Scratch slots of the store's grow-only update workspace.
 enum UpdateScratchSlot {
-    SCR_QP = 0, SCR_SDOTS, SCR_EXTS, SCR_WS, SCR_BOUND, SCR_CNT, SCR_BUF,   // relate (fused)
+    SCR_QP = 0, SCR_EXTS, SCR_WS, SCR_BOUND, SCR_CNT, SCR_BUF,              // relate (fused)
     SCR_DOTS, SCR_CAND,                                                      // relate (batched)
     SCR_DEG, SCR_RECIP, SCR_RECIP_OFF, SCR_KEYS, SCR_VALS, SCR_KEYS2, SCR_VALS2, SCR_TMP,
     SCR_NBR_IDS, SCR_NBR_COS,                                                // update results

@@ -66,3 +66,15 @@ def test_build_targets_sm103a_only(lib_path):
     flags = " ".join(_build.FLAGS)
     assert "gencode" not in flags and "arch=" not in flags
     assert os.path.exists(lib_path)
+
+
+def test_sort_pairs_rejects_bad_arguments_without_gpu_work(lib_path):
+    """sort_pairs validates n, bits and its buffers before any device call;
+    n <= 1 is a no-op."""
+    import paper_2607_05708_gb300 as pkg
+    lib = pkg.load_library()
+    for n, bits in ((-1, 8), (10, 8), (10, 33), (10, -1), (1 << 31, 8)):
+        assert lib.akashic_mem_sort_pairs(None, None, n, bits, None) == 1
+        assert b"sort_pairs" in lib.akashic_mem_last_error()
+    assert lib.akashic_mem_sort_pairs(None, None, 0, 8, None) == 0
+    assert lib.akashic_mem_sort_pairs(None, None, 1, 8, None) == 0
