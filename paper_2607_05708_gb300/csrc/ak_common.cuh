@@ -54,6 +54,10 @@ __host__ __device__ __forceinline__ bool scope_active(const NsScope &s) {
     return s.q_ns != nullptr || s.dead != nullptr;
 }
 
+// log2(e): scores exp(tau x - c) are evaluated as 2^(x tau log2(e) - c log2(e))
+// (one FMA and the hardware exp2).
+constexpr float LOG2E_F = 1.44269504088896340736f;
+
 // Keys for signed cosine values: order-preserving map of any finite fp32 to
 // uint32 (flip all bits of negatives, set the sign bit of non-negatives).
 __device__ __forceinline__ uint32_t ordered_bits(float v) {

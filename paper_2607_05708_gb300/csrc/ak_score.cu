@@ -191,42 +191,55 @@ __device__ __forceinline__ void zadd(float (&z)[N], int ch, float s) {
         if (i == ch) z[i] += s;
 }
 
-template <int BP, int MODE>
+// P2: the CTA-pair form.  Clusters of two CTAs compute 256-row tiles with
+// the two-SM MMA: each CTA stages its own 128 rows of A and half of the
+// BP-row B tile per stage (so a stage is a third smaller at BP = 256 and
+// more of them fit), and each CTA's TMEM holds its own rows' accumulators,
+// double-buffered.  The odd CTA's copies signal their completion on the
+// even CTA's (the MMA issuer's) barrier, whose arrival announces both
+// CTAs' bytes; the issuer commits each stage release and each ready
+// accumulator to both CTAs' barriers, and the odd CTA's epilogue releases
+// the accumulator on the even CTA's barrier by a remote arrive.
+template <int BP, int MODE, bool P2 = false>
 struct GemmCfg {
     static constexpr int BM = 128, BK = 64;
     static constexpr int A_BYTES = BM * BK * 2;
-    static constexpr int B_BYTES = BP * BK * 2;
+    static constexpr int B_BYTES = (P2 ? BP / 2 : BP) * BK * 2;
     static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
     static constexpr int OUT_BYTES = BM * 32 * 4;
     // the filter epilogue stores nothing: its region only holds the tile's
     // column bounds, and the freed space goes to pipeline stages
+    // epilogue warps: the filter epilogues are issue-bound (one compare per
+    // dot) and the score epilogue nearly so (exp, row extremes, column
+    // sums, staging), so they run two warps per TMEM lane quarter, each on
+    // half the columns (HALVES = 2); the others run one
+    static constexpr int EPI_W =
+        ((MODE == GEMM_FILTER || MODE == GEMM_KEYS_T || MODE == GEMM_EXP) && BP >= 64) ? 8 : 4;
+    static constexpr int HALVES = EPI_W / 4;
     static constexpr int OUT_REGION = (MODE == GEMM_FILTER || MODE == GEMM_KEYS_T)
                                           ? (BP * 12 < 1024 ? 1024 : BP * 12)
                                       : MODE == GEMM_EXP_FILTER ? 2 * OUT_BYTES + BP * 12
-                                                                : 2 * OUT_BYTES;
+                                                                : 2 * HALVES * OUT_BYTES;
     static constexpr int MISC = 4096;   // shift, Z sums, flags, barriers
     static constexpr int BUDGET = 227 * 1024 - 1024;
     static constexpr int S_FIT = (BUDGET - OUT_REGION - MISC) / STAGE_BYTES;
     static constexpr int STAGES = S_FIT > 8 ? 8 : S_FIT;
     static constexpr int TMEM_COLS = 2 * BP < 32 ? 32 : 2 * BP;
-    // epilogue warps: the filter epilogue is issue-bound (one compare per
-    // dot), so it runs two warps per TMEM lane quarter, each on half the
-    // columns; the storing epilogues run one
-    static constexpr int EPI_W = ((MODE == GEMM_FILTER || MODE == GEMM_KEYS_T) && BP >= 64) ? 8 : 4;
     static constexpr int EPI_T = 32 * EPI_W;
     static constexpr int THREADS = 64 + EPI_T;
     static constexpr int SMEM = 1024 + STAGES * STAGE_BYTES + OUT_REGION + MISC;
     static_assert(BP >= 32 && BP <= 256 && (BP & (BP - 1)) == 0, "BP must be 32..256, a power of 2");
     static_assert(STAGES >= 2, "not enough shared memory for two stages");
+    static_assert(!P2 || BP >= 128, "the pair form needs B halves of 64 rows or more");
 };
 
-template <int BP, int MODE>
-__global__ __launch_bounds__(GemmCfg<BP, MODE>::THREADS, 1) void k_gemm_umma(const __grid_constant__ CUtensorMap tmA,
+template <int BP, int MODE, bool P2 = false>
+__global__ __launch_bounds__(GemmCfg<BP, MODE, P2>::THREADS, 1) void k_gemm_umma(const __grid_constant__ CUtensorMap tmA,
                                                       const __grid_constant__ CUtensorMap tmB,
                                                       const __grid_constant__ CUtensorMap tmC,
                                                       int64_t n_rows, int dim, int n_ctiles,
                                                       const GemmEpi ep) {
-    using C = GemmCfg<BP, MODE>;
+    using C = GemmCfg<BP, MODE, P2>;
     constexpr bool EXPF = MODE == GEMM_EXP_FILTER;
     constexpr bool EXP = MODE == GEMM_EXP || EXPF;
     constexpr bool FILTER = MODE == GEMM_FILTER;
@@ -237,24 +250,34 @@ __global__ __launch_bounds__(GemmCfg<BP, MODE>::THREADS, 1) void k_gemm_umma(con
     uint8_t *sB = smem + C::STAGES * C::A_BYTES;
     float *sOut = (float *)(smem + C::STAGES * C::STAGE_BYTES);     // 2 x [128][32], swizzled
     uint8_t *misc = smem + C::STAGES * C::STAGE_BYTES + C::OUT_REGION;
-    float *shift_s = (float *)misc;                  // [BP]  (ends below misc + 2560)
+    float *shift_s = (float *)misc;                  // [BP]  (ends below misc + 1024)
+    float *xmax = (float *)(misc + 1024);            // [128] row extremes of the second
+    float *xmin = xmax + 128;                        // column half (ends at misc + 2048)
     int *go = (int *)(misc + 2560);                  // epilogue: the tile's accumulator is ready
     uint64_t *bars = (uint64_t *)(misc + 3072);      // full[S], empty[S], tfull[2], tempty[2]
     uint64_t *full = bars, *empty = bars + C::STAGES;
     uint64_t *tfull = bars + 2 * C::STAGES, *tempty = tfull + 2;
-    uint32_t *tmem_slot = (uint32_t *)(tempty + 2);
+    uint64_t *done_bar = tempty + 2;                 // the issuer's MMAs have all completed
+    uint32_t *tmem_slot = (uint32_t *)(done_bar + 1);
     // filters: the tile's column bounds and the same as float thresholds
     unsigned long long *bnd_s = (unsigned long long *)(sOut + (EXPF ? 2 * C::OUT_BYTES / 4 : 0));
     float *thr_s = (float *)(bnd_s + BP);
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int64_t m_tiles = (n_rows + C::BM - 1) / C::BM;
-    // work units: (row tile, column tile)
+    // the pair form: this CTA's rank in its cluster (0 issues the MMAs)
+    const uint32_t crank = P2 ? cluster_ctarank() : 0u;
+    const bool lead = crank == 0u;
+    constexpr int TM = P2 ? 2 * C::BM : C::BM;       // rows of a work unit
+    const int row_off = (int)crank * C::BM;          // this CTA's rows in a unit
+    const int b_off = (int)crank * (BP / 2);         // this CTA's half of the B tile (P2)
+    const int64_t m_tiles = (n_rows + TM - 1) / TM;
+    // work units: (row tile, column tile); the two CTAs of a pair share each
     const int64_t n_units = m_tiles * n_ctiles;
-    const int64_t u_first = blockIdx.x;
-    const int64_t u_step = gridDim.x;
+    const int64_t u_first = P2 ? blockIdx.x / 2 : blockIdx.x;
+    const int64_t u_step = P2 ? gridDim.x / 2 : gridDim.x;
     const int kb_n = dim / C::BK;
     int *status = ep.status;
+    const float tau_l2e = ep.tau * LOG2E_F;
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < C::STAGES; ++s) {
@@ -263,25 +286,34 @@ __global__ __launch_bounds__(GemmCfg<BP, MODE>::THREADS, 1) void k_gemm_umma(con
         }
         for (int a = 0; a < 2; ++a) {
             mbar_init(&tfull[a], 1);
-            mbar_init(&tempty[a], 1);
+            mbar_init(&tempty[a], P2 && lead ? 2 : 1);   // both CTAs' epilogues
         }
+        mbar_init(done_bar, 1);
         mbar_fence_init();
     }
     if (warp == 1) {
-        tmem_alloc(tmem_slot, C::TMEM_COLS);
-        tmem_relinquish();
+        if constexpr (P2) {
+            tmem_alloc2(tmem_slot, C::TMEM_COLS);
+            tmem_relinquish2();
+        } else {
+            tmem_alloc(tmem_slot, C::TMEM_COLS);
+            tmem_relinquish();
+        }
     }
     for (int i = threadIdx.x; i < BP; i += blockDim.x) {
-        shift_s[i] = EXP ? ep.shift[i] : 0.f;
+        // exp(tau x - c) evaluated as 2^(x tau log2(e) - c log2(e)): one FMA
+        // and the hardware exp2 per score
+        shift_s[i] = EXP ? ep.shift[i] * LOG2E_F : 0.f;
     }
     tc_fence_before();
     __syncthreads();
+    if constexpr (P2) cluster_sync();   // both CTAs' barriers exist before any remote arrive
     tc_fence_after();
     const uint32_t tmem_base = *tmem_slot;
 
     if (warp == 0) {
         if (lane == 0) {
-            // ---------------- TMA producer
+            // ---------------- TMA producer (each CTA loads its own share)
             uint32_t stage = 0, phase = 0;
             int last_par[8];
             for (int s = 0; s < 8; ++s) last_par[s] = -1;
@@ -290,15 +322,26 @@ __global__ __launch_bounds__(GemmCfg<BP, MODE>::THREADS, 1) void k_gemm_umma(con
                 const int64_t ct = u % n_ctiles;
                 const int64_t mt = u / n_ctiles;
                 for (int kb = 0; kb < kb_n; ++kb) {
-                    if (!mbar_wait(&empty[stage], phase ^ 1u, status)) {
+                    // (the odd CTA's releases arrive remotely: spin on them)
+                    if (!(P2 && !lead ? mbar_wait_spin(&empty[stage], phase ^ 1u, status)
+                                      : mbar_wait(&empty[stage], phase ^ 1u, status))) {
                         ok = false;
                         break;
                     }
-                    mbar_expect_tx(&full[stage], C::STAGE_BYTES);
-                    tma_load_2d(sA + stage * C::A_BYTES, &tmA, &full[stage], kb * C::BK,
-                                (int)(mt * C::BM));
-                    tma_load_2d(sB + stage * C::B_BYTES, &tmB, &full[stage], kb * C::BK,
-                                (int)(ct * BP));
+                    if (lead) {
+                        // the stage fills with both CTAs' bytes
+                        mbar_expect_tx(&full[stage], (P2 ? 2 : 1) * C::STAGE_BYTES);
+                        tma_load_2d(sA + stage * C::A_BYTES, &tmA, &full[stage], kb * C::BK,
+                                    (int)(mt * TM));
+                        tma_load_2d(sB + stage * C::B_BYTES, &tmB, &full[stage], kb * C::BK,
+                                    (int)(ct * BP));
+                    } else {
+                        // the odd CTA's copies complete on the even CTA's barrier
+                        tma_load_2d_pair(sA + stage * C::A_BYTES, &tmA, &full[stage], 0u,
+                                         kb * C::BK, (int)(mt * TM + row_off));
+                        tma_load_2d_pair(sB + stage * C::B_BYTES, &tmB, &full[stage], 0u,
+                                         kb * C::BK, (int)(ct * BP + b_off));
+                    }
                     last_par[stage] = (int)phase;
                     if (++stage == (uint32_t)C::STAGES) {
                         stage = 0;
@@ -308,21 +351,29 @@ __global__ __launch_bounds__(GemmCfg<BP, MODE>::THREADS, 1) void k_gemm_umma(con
             }
             if (!ok) {
                 // let every copy this thread issued land before the CTA exits
-                for (int s = 0; s < C::STAGES; ++s)
-                    if (last_par[s] >= 0) mbar_wait(&full[s], (uint32_t)last_par[s], status);
+                if (lead) {
+                    for (int s = 0; s < C::STAGES; ++s)
+                        if (last_par[s] >= 0) mbar_wait(&full[s], (uint32_t)last_par[s], status);
+                } else {
+                    // the odd CTA's copies report to the even CTA: give them
+                    // ample time (they land within microseconds)
+                    for (int i = 0; i < 200; ++i) __nanosleep(1000);
+                }
             }
         }
     } else if (warp == 1) {
-        if (lane == 0) {
+        if (lane == 0 && lead) {
             // ---------------- MMA issuer
-            const uint32_t idesc = idesc_bf16_m128(BP);
+            const uint32_t idesc = idesc_bf16(TM, BP);
             uint32_t stage = 0, phase = 0;
             int it = 0;
             bool ok = true;
             for (int64_t u = u_first; u < n_units && ok; u += u_step, ++it) {
                 const int acc = it & 1;
                 const uint32_t aph = (uint32_t)(it >> 1) & 1u;
-                if (!mbar_wait(&tempty[acc], aph ^ 1u, status)) break;
+                if (!(P2 ? mbar_wait_spin(&tempty[acc], aph ^ 1u, status)
+                         : mbar_wait(&tempty[acc], aph ^ 1u, status)))
+                    break;
                 tc_fence_after();
                 const uint32_t d = tmem_base + (uint32_t)(acc * BP);
                 for (int kb = 0; kb < kb_n; ++kb) {
@@ -334,17 +385,38 @@ __global__ __launch_bounds__(GemmCfg<BP, MODE>::THREADS, 1) void k_gemm_umma(con
                     const uint64_t ad = sdesc_sw128(smem_u32(sA + stage * C::A_BYTES));
                     const uint64_t bd = sdesc_sw128(smem_u32(sB + stage * C::B_BYTES));
 #pragma unroll
-                    for (int k = 0; k < C::BK / 16; ++k)
-                        umma_bf16(d, ad + (uint64_t)(2 * k), bd + (uint64_t)(2 * k), idesc,
-                                  (kb | k) != 0 ? 1u : 0u);
-                    umma_commit(&empty[stage]);
+                    for (int k = 0; k < C::BK / 16; ++k) {
+                        if constexpr (P2)
+                            umma2_bf16(d, ad + (uint64_t)(2 * k), bd + (uint64_t)(2 * k), idesc,
+                                       (kb | k) != 0 ? 1u : 0u);
+                        else
+                            umma_bf16(d, ad + (uint64_t)(2 * k), bd + (uint64_t)(2 * k), idesc,
+                                      (kb | k) != 0 ? 1u : 0u);
+                    }
+                    if constexpr (P2) {
+                        umma2_commit(&empty[stage]);
+                        umma2_commit_to(&empty[stage], 1u);
+                    } else {
+                        umma_commit(&empty[stage]);
+                    }
                     if (++stage == (uint32_t)C::STAGES) {
                         stage = 0;
                         phase ^= 1u;
                     }
                 }
-                if (ok) umma_commit(&tfull[acc]);
+                if (ok) {
+                    if constexpr (P2) {
+                        umma2_commit(&tfull[acc]);
+                        umma2_commit_to(&tfull[acc], 1u);
+                    } else {
+                        umma_commit(&tfull[acc]);
+                    }
+                }
             }
+            // every MMA issued has completed before the CTA (and its pair) may leave
+            if constexpr (P2) umma2_commit(done_bar);
+            else umma_commit(done_bar);
+            mbar_wait(done_bar, 0u, status);
         }
     } else {
         // ---------------- epilogue (EPI_T threads; warp w reads TMEM lanes 32*(w%4)..)
@@ -366,7 +438,11 @@ __global__ __launch_bounds__(GemmCfg<BP, MODE>::THREADS, 1) void k_gemm_umma(con
             const int acc = it & 1;
             const uint32_t aph = (uint32_t)(it >> 1) & 1u;
             // one thread polls, the barrier makes the outcome uniform
-            if (et == 0) *go = mbar_wait(&tfull[acc], aph, status) ? 1 : 0;
+            if (et == 0) {
+                const bool ok = P2 && !lead ? mbar_wait_spin(&tfull[acc], aph, status)
+                                            : mbar_wait(&tfull[acc], aph, status);
+                *go = ok ? 1 : 0;
+            }
             if (FILTER || EXPF) {
                 // threshold T with: v < T => key < bound; v > T => key > bound
                 // (signed keys order values like floats, -0 below +0; the
@@ -385,7 +461,7 @@ __global__ __launch_bounds__(GemmCfg<BP, MODE>::THREADS, 1) void k_gemm_umma(con
             named_bar(1, C::EPI_T);
             if (!*go) break;
             tc_fence_after();
-            const int64_t grow = mt * C::BM + row;
+            const int64_t grow = mt * TM + row_off + row;
             const bool in_rows = grow < n_rows;
             const bool valid =
                 in_rows && (MODE == GEMM_RAW || !ep.dead_row || !ep.dead_row[grow]);
@@ -444,7 +520,7 @@ __global__ __launch_bounds__(GemmCfg<BP, MODE>::THREADS, 1) void k_gemm_umma(con
 #pragma unroll
                 for (int i = 0; i < 32; ++i) {
                     const float x = __uint_as_float(r[i]);
-                    v[i] = valid ? (EXP ? expf(ep.tau * x - shift_s[ch * 32 + i]) : x) : 0.f;
+                    v[i] = valid ? (EXP ? exp2f(fmaf(x, tau_l2e, -shift_s[ch * 32 + i])) : x) : 0.f;
                 }
                 if (MODE == GEMM_EXP && ep.row_max) {
 #pragma unroll
@@ -471,15 +547,15 @@ __global__ __launch_bounds__(GemmCfg<BP, MODE>::THREADS, 1) void k_gemm_umma(con
                     }
                 }
                 // stage the row: EXP_FILTER in the warp's own 32 rows of
-                // buffer 0 (warp-private, no CTA barrier); EXP in buffer buf,
-                // shared with the TMA store
+                // buffer 0 (warp-private, no CTA barrier); EXP / RAW in the
+                // column half's buffer buf, shared with the TMA store
                 float *so_base;
                 if constexpr (EXPF) {
                     __syncwarp();                             // the warp's rows free again
                     so_base = sOut;
                 } else {
-                    named_bar(1, C::EPI_T);                   // staging[buf] free again
-                    so_base = sOut + buf * (C::OUT_BYTES / 4);
+                    named_bar(2 + hsel, 128);                 // staging[buf] free again
+                    so_base = sOut + (hsel * 2 + buf) * (C::OUT_BYTES / 4);
                 }
                 float4 *dst = (float4 *)(so_base + row * 32);
 #pragma unroll
@@ -513,24 +589,46 @@ __global__ __launch_bounds__(GemmCfg<BP, MODE>::THREADS, 1) void k_gemm_umma(con
                         }
                     }
                 } else {
-                    named_bar(1, C::EPI_T);                   // staging[buf] complete
-                    if (et == 0) {
-                        tma_store_2d(&tmC, so_base, (int)(ct * BP + ch * 32), (int)(mt * C::BM));
-                        bulk_commit();
+                    named_bar(2 + hsel, 128);                 // staging[buf] complete
+                    if ((et & 127) == 0) {
+                        // (the odd CTA's half of the last pair tile may lie
+                        // wholly past the last row: no store starts there)
+                        if (mt * TM + row_off < n_rows) {
+                            tma_store_2d(&tmC, so_base, (int)(ct * BP + ch * 32),
+                                         (int)(mt * TM + row_off));
+                            bulk_commit();
+                        }
                         bulk_wait_read<1>();                  // the other buffer is free
                     }
                 }
                 }
             }
-            if (MODE == GEMM_EXP && ep.row_max && in_rows) {
-                ep.row_max[grow] = rmax;
-                ep.row_min[grow] = rmin;
-                emx = fmaxf(emx, rmax);
-                if (rmax > 0.f) emn = fminf(emn, rmin);
+            if (MODE == GEMM_EXP && ep.row_max) {
+                if constexpr (C::HALVES == 2) {
+                    // the row's second column half hands its extremes over
+                    if (hsel == 1) {
+                        xmax[row] = rmax;
+                        xmin[row] = rmin;
+                    }
+                    named_bar(1, C::EPI_T);
+                    if (hsel == 0) {
+                        rmax = fmaxf(rmax, xmax[row]);
+                        rmin = fminf(rmin, xmin[row]);
+                    }
+                }
+                if (hsel == 0 && in_rows) {
+                    ep.row_max[grow] = rmax;
+                    ep.row_min[grow] = rmin;
+                    emx = fmaxf(emx, rmax);
+                    if (rmax > 0.f) emn = fminf(emn, rmin);
+                }
             }
             tc_fence_before();
             named_bar(1, C::EPI_T);
-            if (et == 0) mbar_arrive(&tempty[acc]);
+            if (et == 0) {
+                if (P2 && !lead) mbar_arrive_remote(&tempty[acc], 0u);
+                else mbar_arrive(&tempty[acc]);
+            }
         }
         if (MODE == GEMM_EXP && ep.ext) {
             // u >= 0: float bits order like the values
@@ -545,13 +643,15 @@ __global__ __launch_bounds__(GemmCfg<BP, MODE>::THREADS, 1) void k_gemm_umma(con
                 atomicMax(ep.ext + 1, mn);
             }
         }
-        if (!EXPF && et == 0) bulk_wait_all();
+        if (!EXPF && (et & 127) == 0) bulk_wait_all();
         named_bar(1, C::EPI_T);
         if (EXP && ep.zpart) {
-            // the four warps' column sums, added in a fixed order
+            // the four lane quarters' column sums, added in a fixed order
+            // (each chunk's sums come from the one warp of its column half)
             float *zred = sOut;                               // [4][BP], free now
 #pragma unroll
-            for (int i = 0; i < BP / 32; ++i) zred[q * BP + i * 32 + lane] = zl[i];
+            for (int i = 0; i < BP / 32; ++i)
+                if (i / CH_PER == hsel) zred[q * BP + i * 32 + lane] = zl[i];
             named_bar(1, C::EPI_T);
             for (int c = et; c < BP; c += C::EPI_T)
                 ep.zpart[(int64_t)blockIdx.x * BP + c] =
@@ -561,7 +661,15 @@ __global__ __launch_bounds__(GemmCfg<BP, MODE>::THREADS, 1) void k_gemm_umma(con
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
-    if (warp == 1) tmem_dealloc(tmem_base, C::TMEM_COLS);
+    if constexpr (P2) {
+        // neither CTA leaves while the other may still arrive on its
+        // barriers or the pair's MMAs read its shared memory
+        cluster_sync();
+        tc_fence_after();
+        if (warp == 1) tmem_dealloc2(tmem_base, C::TMEM_COLS);
+    } else {
+        if (warp == 1) tmem_dealloc(tmem_base, C::TMEM_COLS);
+    }
 }
 
 int64_t score_tiles(int64_t n) { return ceil_div<int64_t>(n, 128); }
@@ -584,20 +692,52 @@ cudaError_t launch_wait_timeout_check(int *status, uint32_t polls, cudaStream_t 
 }
 
 // The kernel's dynamic shared-memory limit, raised once per device (with
-// that device current) before its first launch there.
-template <int BP, int MODE>
-static cudaError_t gemm_attr() {
-    using C = GemmCfg<BP, MODE>;
+// that device current) before its first launch there; for the pair form
+// also the number of clusters of two that fit on the device at once (one
+// CTA per SM), or 0 if none does.
+template <int BP, int MODE, bool P2 = false>
+static cudaError_t gemm_attr(int *clusters = nullptr) {
+    using C = GemmCfg<BP, MODE, P2>;
     static bool attr[64] = {false};
+    static int ncl[64] = {0};
     int dev = 0;
     cudaGetDevice(&dev);
-    if (dev >= 0 && dev < 64 && !attr[dev]) {
-        cudaError_t e = cudaFuncSetAttribute(k_gemm_umma<BP, MODE>,
+    if (dev < 0 || dev >= 64) return cudaSuccess;
+    if (!attr[dev]) {
+        cudaError_t e = cudaFuncSetAttribute(k_gemm_umma<BP, MODE, P2>,
                                              cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
         if (e != cudaSuccess) return e;
+        if (P2) {
+            cudaLaunchConfig_t cfg = {};
+            cudaLaunchAttribute at[1];
+            at[0].id = cudaLaunchAttributeClusterDimension;
+            at[0].val.clusterDim.x = 2;
+            at[0].val.clusterDim.y = 1;
+            at[0].val.clusterDim.z = 1;
+            cfg.gridDim = dim3((unsigned)(device_sm_count() & ~1));
+            cfg.blockDim = dim3(C::THREADS);
+            cfg.dynamicSmemBytes = C::SMEM;
+            cfg.attrs = at;
+            cfg.numAttrs = 1;
+            int n = 0;
+            e = cudaOccupancyMaxActiveClusters(&n, k_gemm_umma<BP, MODE, P2>, &cfg);
+            if (e != cudaSuccess) return e;
+            ncl[dev] = n;
+        }
         attr[dev] = true;
     }
+    if (clusters) *clusters = ncl[dev];
     return cudaSuccess;
+}
+
+// The pair form is taken where it applies unless AKASHIC_GEMM_PAIR=0.
+static bool gemm_pair_enabled() {
+    static int v = -1;
+    if (v < 0) {
+        const char *e = getenv("AKASHIC_GEMM_PAIR");
+        v = (e && e[0] == '0') ? 0 : 1;
+    }
+    return v == 1;
 }
 
 cudaError_t prepare_score_gemm() {
@@ -605,30 +745,70 @@ cudaError_t prepare_score_gemm() {
     if (e == cudaSuccess) e = gemm_attr<64, GEMM_EXP>();
     if (e == cudaSuccess) e = gemm_attr<128, GEMM_EXP>();
     if (e == cudaSuccess) e = gemm_attr<256, GEMM_EXP>();
+    if (e == cudaSuccess) e = gemm_attr<128, GEMM_EXP, true>();
+    if (e == cudaSuccess) e = gemm_attr<256, GEMM_EXP, true>();
     return e;
 }
 
 // A: E rows (row_stride_rows apart: 1 = every row, s = every s-th row),
 // B: n_ctiles * BP query rows, C: output [n_rows][n_ctiles * BP] (EXP/RAW).
+// The grid: one CTA per SM at most (the single form), or clusters of two
+// on 256-row tiles (the pair form, B >= 128, taken when the rows fill every
+// cluster that fits, so that the grid never exceeds ceil(n_rows / 128) and
+// the Z partials keep at most one row per 128-row tile).  *zrows = grid.
 template <int BP, int MODE>
 static cudaError_t gemm_bp(const uint16_t *emb, int64_t n_rows, int64_t row_stride_rows, int dim,
                            const uint16_t *qp, int n_ctiles, float *out, const GemmEpi &ep,
                            cudaStream_t st, int *zrows) {
-    using C = GemmCfg<BP, MODE>;
-    cudaError_t e = gemm_attr<BP, MODE>();
-    if (e != cudaSuccess) return e;
+    constexpr bool CAN_P2 = BP >= 128;
+    int ncl = 0;
+    if constexpr (CAN_P2) {
+        if (gemm_pair_enabled()) {
+            cudaError_t e = gemm_attr<BP, MODE, true>(&ncl);
+            if (e != cudaSuccess) return e;
+        }
+    }
+    const bool p2 = CAN_P2 && ncl > 0 && n_rows >= (int64_t)256 * ncl;
+    if (!p2) {
+        cudaError_t e = gemm_attr<BP, MODE>();
+        if (e != cudaSuccess) return e;
+    }
     CUtensorMap ta, tb, tc;
-    e = make_tmap_2d(&ta, emb, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, (uint64_t)dim,
+    cudaError_t e = make_tmap_2d(&ta, emb, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, (uint64_t)dim,
                                  (uint64_t)n_rows, (uint64_t)dim * 2 * row_stride_rows, 64, 128);
     if (e == cudaSuccess)
         e = make_tmap_2d(&tb, qp, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, (uint64_t)dim,
-                         (uint64_t)n_ctiles * BP, (uint64_t)dim * 2, 64, BP);
+                         (uint64_t)n_ctiles * BP, (uint64_t)dim * 2, 64, p2 ? BP / 2 : BP);
     if (e == cudaSuccess && MODE != GEMM_FILTER && MODE != GEMM_EXP_FILTER && MODE != GEMM_KEYS_T)
         e = make_tmap_2d(&tc, out, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, (uint64_t)n_ctiles * BP,
                          (uint64_t)n_rows, (uint64_t)n_ctiles * BP * 4, 32, 128);
     else
         tc = ta;   // unused by the filter epilogue
     if (e != cudaSuccess) return e;
+    if constexpr (CAN_P2) {
+        if (p2) {
+            using C2 = GemmCfg<BP, MODE, true>;
+            const int64_t units = ceil_div<int64_t>(n_rows, 256) * n_ctiles;
+            const int64_t clusters = units < ncl ? units : ncl;
+            cudaLaunchConfig_t cfg = {};
+            cudaLaunchAttribute at[1];
+            at[0].id = cudaLaunchAttributeClusterDimension;
+            at[0].val.clusterDim.x = 2;
+            at[0].val.clusterDim.y = 1;
+            at[0].val.clusterDim.z = 1;
+            cfg.gridDim = dim3((unsigned)(2 * clusters));
+            cfg.blockDim = dim3(C2::THREADS);
+            cfg.dynamicSmemBytes = C2::SMEM;
+            cfg.stream = st;
+            cfg.attrs = at;
+            cfg.numAttrs = 1;
+            e = cudaLaunchKernelEx(&cfg, k_gemm_umma<BP, MODE, true>, ta, tb, tc, n_rows, dim,
+                                   n_ctiles, ep);
+            if (zrows) *zrows = (int)(2 * clusters);
+            return e == cudaSuccess ? cudaGetLastError() : e;
+        }
+    }
+    using C = GemmCfg<BP, MODE>;
     const int64_t m_tiles = ceil_div<int64_t>(n_rows, 128);
     const int64_t tiles = m_tiles * n_ctiles;
     const int grid = (int)(tiles < device_sm_count() ? tiles : device_sm_count());

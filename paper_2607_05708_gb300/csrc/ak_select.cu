@@ -585,7 +585,8 @@ __global__ __launch_bounds__(SEL_THREADS) void k_topk_merge(
             for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
             if (lane == 0)
                 rc.dst[j * bp + c] = rc.kind == 1 ? fmaf(rc.alpha, acc, rc.u[j * bp + c])
-                                                  : expf(rc.tau * acc - rc.shift[c]);
+                                                  : exp2f(fmaf(acc, rc.tau * LOG2E_F,
+                                                               -rc.shift[c] * LOG2E_F));
         }
         __threadfence_block();
         __syncthreads();

@@ -56,6 +56,48 @@ __device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity, int *s
     return mbar_wait_n(bar, parity, status, WAIT_LIMIT);
 }
 
+// Bounded spin on the non-blocking test (no suspension between polls), for
+// a barrier that another CTA of the cluster completes by a remote arrive.
+__device__ __forceinline__ bool mbar_test_wait(uint64_t *bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(smem_u32(bar)), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+constexpr uint32_t SPIN_LIMIT = 1u << 28;   // test_wait polls before a spin gives up
+__device__ __forceinline__ bool mbar_wait_spin(uint64_t *bar, uint32_t parity, int *status) {
+    for (uint32_t i = 0; i < SPIN_LIMIT; ++i)
+        if (mbar_test_wait(bar, parity)) return true;
+    set_status(status, AKASHIC_ETIMEOUT);
+    return false;
+}
+
+// ------------------------------------------------------------------ clusters
+__device__ __forceinline__ uint32_t cluster_ctarank() {
+    uint32_t r;
+    asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+    return r;
+}
+// Every thread of every CTA of the cluster (release / acquire).
+__device__ __forceinline__ void cluster_sync() {
+    asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;"
+                 ::: "memory");
+}
+// Arrive once on the barrier at the same shared-memory offset as `bar` in
+// the cluster's CTA `rank` (default semantics: release at CTA scope; the
+// signals sent this way order tensor-core and copy completions, which carry
+// their own ordering, not generic writes, so no cluster-scope fence).
+__device__ __forceinline__ void mbar_arrive_remote(uint64_t *bar, uint32_t rank) {
+    uint32_t ra;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(ra) : "r"(smem_u32(bar)), "r"(rank));
+    asm volatile("mbarrier.arrive.shared::cluster.b64 _, [%0];" ::"r"(ra) : "memory");
+}
+
 // ------------------------------------------------------------------ TMA
 __device__ __forceinline__ void tma_load_2d(void *dst, const CUtensorMap *map, uint64_t *bar,
                                             int x, int y) {
@@ -63,6 +105,19 @@ __device__ __forceinline__ void tma_load_2d(void *dst, const CUtensorMap *map, u
         "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
         " [%0], [%1, {%3, %4}], [%2];" ::"r"(smem_u32(dst)),
         "l"(map), "r"(smem_u32(bar)), "r"(x), "r"(y)
+        : "memory");
+}
+// The same load into this CTA's shared memory, its completion signalled on
+// the barrier at the same offset as `bar` in the pair's CTA `rank`
+// (cta_group::2: the barrier may be in the other CTA of the pair).
+__device__ __forceinline__ void tma_load_2d_pair(void *dst, const CUtensorMap *map, uint64_t *bar,
+                                                 uint32_t rank, int x, int y) {
+    uint32_t rb;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(rb) : "r"(smem_u32(bar)), "r"(rank));
+    asm volatile(
+        "cp.async.bulk.tensor.2d.cta_group::2.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+        " [%0], [%1, {%3, %4}], [%2];" ::"r"(smem_u32(dst)),
+        "l"(map), "r"(rb), "r"(x), "r"(y)
         : "memory");
 }
 __device__ __forceinline__ void tma_store_2d(const CUtensorMap *map, const void *src, int x,
@@ -126,6 +181,61 @@ __device__ __forceinline__ void umma_commit(uint64_t *bar) {
         "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
             smem_u32(bar))
         : "memory");
+}
+
+// The CTA-pair forms (cta_group::2): the pair's TMEM is allocated and freed
+// by one warp of each CTA together; the MMA, issued by the even CTA alone,
+// computes a 256-row tile whose rows 0-127 come from that CTA's A tile and
+// 128-255 from the odd CTA's A tile at the same shared-memory offset, B's
+// first N/2 rows from the even CTA and the rest from the odd one, and each
+// CTA's TMEM receives its own 128 rows x N columns.  A kernel that uses them
+// uses no cta_group::1 tcgen05 instruction.
+__device__ __forceinline__ void tmem_alloc2(uint32_t *dst_smem, uint32_t ncols) {
+    asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                     smem_u32(dst_smem)),
+                 "r"(ncols)
+                 : "memory");
+}
+__device__ __forceinline__ void tmem_relinquish2() {
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_dealloc2(uint32_t taddr, uint32_t ncols) {
+    asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols)
+                 : "memory");
+}
+__device__ __forceinline__ void umma2_bf16(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc,
+                                           uint32_t idesc, uint32_t accumulate) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "setp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+        "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+        : "memory");
+}
+// Arrive once on this CTA's `bar` when every tcgen05.mma this thread issued
+// has completed (in both CTAs of the pair).
+__device__ __forceinline__ void umma2_commit(uint64_t *bar) {
+    asm volatile(
+        "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
+            smem_u32(bar))
+        : "memory");
+}
+
+// The same arrive on the barrier at the same offset as `bar` in the pair's
+// CTA `rank` (a shared::cluster address from mapa).
+__device__ __forceinline__ void umma2_commit_to(uint64_t *bar, uint32_t rank) {
+    uint32_t ra;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(ra) : "r"(smem_u32(bar)), "r"(rank));
+    asm volatile("tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
+                     ra)
+                 : "memory");
+}
+
+// Instruction descriptor, kind::f16: D fp32, A and B bf16, both K-major,
+// M = m (128, or 256 for the pair form), N = n (multiple of 16, 16..256).
+__host__ __device__ constexpr uint32_t idesc_bf16(int m, int n) {
+    return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(n >> 3) << 17) |
+           ((uint32_t)(m >> 4) << 24);
 }
 
 // Instruction descriptor, kind::f16: D fp32, A and B bf16, both K-major,

@@ -46,6 +46,31 @@ def test_gmm1m_scaled_two_hops(placement):
     assert_retrieval_parity(wl, placement, got, ref)
 
 
+@pytest.mark.parametrize("hops", [0, 2])
+def test_pair_gemm_store(hops):
+    """A store large enough for the score GEMM's CTA-pair form (256-row
+    tiles on clusters of two, B = 256): the gmm1m recipe at N=32768 cut to
+    N=32700 (the last pair tile's odd half partly past the last row),
+    no hops (the fused top-k filter in the GEMM) and two hops, against the
+    oracle."""
+    base = synth.workload(2, scale=1 / 32)
+    n = 32700
+    keep = base.row_ptr[:n + 1]
+    cols = base.col[:keep[-1]]
+    ok = cols < n
+    rows = np.repeat(np.arange(n), np.diff(keep))
+    rp = np.concatenate([[0], np.cumsum(np.bincount(rows[ok], minlength=n))]).astype(np.int64)
+    wl = synth.Workload(name="pair", dim=base.dim, emb=base.emb[:n], queries=base.queries,
+                        row_ptr=rp, col=cols[ok].astype(np.int32),
+                        aff=base.aff[:keep[-1]][ok],
+                        page_of={"clustered": base.page_of["clustered"][:n]},
+                        chunks_per_page=64, alpha=base.alpha, hops=hops, k=base.k)
+    assert wl.queries.shape[0] == 256
+    _, got = gpu_retrieve(wl, "clustered")
+    ref = oracle_retrieve(wl, "clustered")
+    assert_retrieval_parity(wl, "clustered", got, ref)
+
+
 @pytest.mark.parametrize("B,k,hops,alpha", [
     (1, 1, 0, 0.0), (5, 64, 1, 0.5), (37, 13, 2, 0.3), (130, 32, 3, 0.7), (300, 8, 2, 0.5),
     (16, 10, 2, 0.0),
