@@ -350,16 +350,23 @@ __global__ __launch_bounds__(RS_THREADS) void k_rs_scatter_small(
     rs_rank(keys, vals, n, base, shift, mask, k, v, loc, cnt, pre);   // syncs the CTA
 #pragma unroll
     for (int r = 0; r < RS_ITEMS; ++r) {
-        int64_t idx = base + r * 32 + lane;
-        if (idx < n) {
-            uint32_t d = (k[r] >> shift) & mask;
-            const int pos = off_s[d] + pre[warp][d] + loc[r];
+        const int64_t idx = base + r * 32 + lane;
+        const bool ok = idx < n;
+        const uint32_t d = (k[r] >> shift) & mask;
+        const int pos = ok ? off_s[d] + pre[warp][d] + loc[r] : 0;
+        if (ok) {
             okeys[pos] = k[r];
             ovals[pos] = v[r];
-            if (hnext)
-                atomicAdd(&hnext[(int64_t)((k[r] >> shift_next) & mask_next) * n_tiles +
-                                 pos / RS_TILE],
-                          1);
+        }
+        if (hnext) {
+            // one atomic per distinct (next digit, destination tile) of the
+            // warp's round: a high digit has few values, whose counters
+            // would otherwise take the whole round's atomics each
+            const uint32_t slot =
+                ok ? ((k[r] >> shift_next) & mask_next) * (uint32_t)n_tiles + (uint32_t)(pos / RS_TILE)
+                   : 0xffffffffu;
+            const unsigned peers = __match_any_sync(0xffffffffu, slot);
+            if (ok && lane == __ffs(peers) - 1) atomicAdd(&hnext[slot], (int)__popc(peers));
         }
     }
 }

@@ -297,62 +297,38 @@ __global__ __launch_bounds__(SEL_THREADS) void k_sample_kth(
 // most k keys, and warp 0 selects the k-th largest of their union.
 constexpr int KS_WARPS = 4, KS_BUF = 512, KS_U = 16, KS_KMAX = 64;
 
-// The k-th largest (1 <= k <= len) of a[0..len) by one warp: MSB-first
-// radix select, 8 bits a pass, on a 256-bin histogram h of the warp's own.
-__device__ uint32_t warp_kth(const uint32_t *a, int len, int k, int *h) {
+// The k-th largest (1 <= k <= len <= KS_BUF) of a[0..len) by one warp: the
+// keys in registers (KS_BUF / 32 a lane, 0 past len, which ranks below
+// every candidate), then the answer's bits from the top, each kept when at
+// least k keys are >= the prefix with it set (the largest t with k keys
+// >= t is the k-th largest key).  No shared-memory atomics: the sampled
+// keys of one column share their top bits, so histogram bins would collide.
+__device__ uint32_t warp_kth(const uint32_t *a, int len, int k) {
     const int lane = threadIdx.x & 31;
-    uint32_t prefix = 0u, pmask = 0u;
-    int rem = k;
-    for (int sh = 24; sh >= 0; sh -= 8) {
-        for (int i = lane; i < 256; i += 32) h[i] = 0;
-        __syncwarp();
-        for (int i = lane; i < len; i += 32) {
-            const uint32_t x = a[i];
-            if ((x & pmask) == prefix) atomicAdd(&h[(x >> sh) & 255u], 1);
-        }
-        __syncwarp();
-        // lane l owns digits 255 - 8l - j (j = 0..7), largest first
-        int c[8], tot = 0;
+    uint32_t x[KS_BUF / 32];
 #pragma unroll
-        for (int j = 0; j < 8; ++j) {
-            c[j] = h[255 - 8 * lane - j];
-            tot += c[j];
-        }
-        int incl = tot;
+    for (int j = 0; j < KS_BUF / 32; ++j) {
+        const int i = j * 32 + lane;
+        x[j] = i < len ? a[i] : 0u;
+    }
+    uint32_t prefix = 0u;
+#pragma unroll 1
+    for (int b = 31; b >= 0; --b) {
+        const uint32_t cand = prefix | (1u << b);
+        unsigned c = 0u;
 #pragma unroll
-        for (int o = 1; o < 32; o <<= 1) {
-            const int x = __shfl_up_sync(0xffffffffu, incl, o);
-            if (lane >= o) incl += x;
-        }
-        const int before = incl - tot;               // keys with a larger digit
-        const bool mine = before < rem && incl >= rem;
-        int dig = 0, run = before, above = 0;
-        bool hit = false;
-#pragma unroll
-        for (int j = 0; j < 8; ++j) {
-            if (mine && !hit && run + c[j] >= rem) {
-                hit = true;
-                dig = 255 - 8 * lane - j;
-                above = run;
-            }
-            run += c[j];
-        }
-        const int src = __ffs(__ballot_sync(0xffffffffu, mine)) - 1;
-        dig = __shfl_sync(0xffffffffu, dig, src);
-        above = __shfl_sync(0xffffffffu, above, src);
-        prefix |= (uint32_t)dig << sh;
-        pmask |= 255u << sh;
-        rem -= above;
-        __syncwarp();
+        for (int j = 0; j < KS_BUF / 32; ++j) c += x[j] >= cand ? 1u : 0u;
+        c = __reduce_add_sync(0xffffffffu, c);
+        if (c >= (unsigned)k) prefix = cand;
     }
     return prefix;
 }
 
 // Cut a[0..len) (len >= k) to its k largest; returns the k-th largest.
-__device__ uint32_t warp_cut(uint32_t *a, int len, int k, int *h) {
+__device__ uint32_t warp_cut(uint32_t *a, int len, int k) {
     const int lane = threadIdx.x & 31;
     const unsigned lt = (1u << lane) - 1u;
-    const uint32_t x = warp_kth(a, len, k, h);
+    const uint32_t x = warp_kth(a, len, k);
     int out = 0;
     for (int i0 = 0; i0 < len; i0 += 32) {
         const uint32_t v = i0 + lane < len ? a[i0 + lane] : 0u;
@@ -372,7 +348,6 @@ __global__ __launch_bounds__(KS_WARPS * 32) void k_sample_kth_split(
     const uint32_t *__restrict__ keys_t, int64_t n_sample, int b, int k,
     unsigned long long *__restrict__ bound, unsigned int *__restrict__ cnt) {
     __shared__ uint32_t buf[KS_WARPS][KS_BUF];
-    __shared__ int hist[KS_WARPS][256];
     __shared__ int lens[KS_WARPS];
     const int c = blockIdx.x, warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     if (c >= b) {   // padding column: nothing passes the filter
@@ -403,7 +378,7 @@ __global__ __launch_bounds__(KS_WARPS * 32) void k_sample_kth_split(
             const unsigned bal = __ballot_sync(0xffffffffu, p);
             if (bal) {
                 if (len + 32 > KS_BUF) {
-                    t = warp_cut(a, len, k, hist[warp]);
+                    t = warp_cut(a, len, k);
                     len = k;
                 }
                 const bool q = p && x[u] > t;       // the cut may have raised t
@@ -415,7 +390,7 @@ __global__ __launch_bounds__(KS_WARPS * 32) void k_sample_kth_split(
         }
     }
     if (len > k) {
-        warp_cut(a, len, k, hist[warp]);
+        warp_cut(a, len, k);
         len = k;
     }
     if (lane == 0) lens[warp] = len;
@@ -428,7 +403,7 @@ __global__ __launch_bounds__(KS_WARPS * 32) void k_sample_kth_split(
             tot += lens[w];
         }
         __syncwarp();
-        const uint32_t x = tot >= k ? warp_kth(a, tot, k, hist[0]) : 0u;
+        const uint32_t x = tot >= k ? warp_kth(a, tot, k) : 0u;
         if (lane == 0) {
             bound[c] = (unsigned long long)x << 32;
             cnt[c] = 0u;
