@@ -213,8 +213,9 @@ struct GemmCfg {
     // dot) and the score epilogue nearly so (exp, row extremes, column
     // sums, staging), so they run two warps per TMEM lane quarter, each on
     // half the columns (HALVES = 2); the others run one
-    static constexpr int EPI_W =
-        ((MODE == GEMM_FILTER || MODE == GEMM_KEYS_T || MODE == GEMM_EXP) && BP >= 64) ? 8 : 4;
+    static constexpr int EPI_W = ((MODE == GEMM_FILTER || MODE == GEMM_KEYS_T ||
+                                   MODE == GEMM_EXP || MODE == GEMM_EXP_FILTER) && BP >= 64)
+                                     ? 8 : 4;
     static constexpr int HALVES = EPI_W / 4;
     static constexpr int OUT_REGION = (MODE == GEMM_FILTER || MODE == GEMM_KEYS_T)
                                           ? (BP * 12 < 1024 ? 1024 : BP * 12)
@@ -546,13 +547,13 @@ __global__ __launch_bounds__(GemmCfg<BP, MODE, P2>::THREADS, 1) void k_gemm_umma
                         }
                     }
                 }
-                // stage the row: EXP_FILTER in the warp's own 32 rows of
-                // buffer 0 (warp-private, no CTA barrier); EXP / RAW in the
-                // column half's buffer buf, shared with the TMA store
+                // stage the row: EXP_FILTER in the warp's own 32 rows of its
+                // column half's buffer (warp-private, no CTA barrier); EXP /
+                // RAW in the column half's buffer buf, shared with the TMA store
                 float *so_base;
                 if constexpr (EXPF) {
                     __syncwarp();                             // the warp's rows free again
-                    so_base = sOut;
+                    so_base = sOut + hsel * (C::OUT_BYTES / 4);
                 } else {
                     named_bar(2 + hsel, 128);                 // staging[buf] free again
                     so_base = sOut + (hsel * 2 + buf) * (C::OUT_BYTES / 4);
