@@ -811,12 +811,13 @@ akashic_status_t akashic_mem_update_relations(akashic_mem_t *m, int64_t first, i
             void *p_inc = store_scratch(m, SCR_IN_INC, (size_t)(rows + 1) * 8);
             void *p_deg = store_scratch(m, SCR_IN_DEG, (size_t)(rows + 1) * 8);
             void *p_off = store_scratch(m, SCR_IN_OFF, (size_t)(rows + 1) * 8);
+            void *p_rs = store_scratch(m, SCR_IN_RSTAT, (size_t)(rows > 0 ? rows : 1) * 8);
             void *p_k = store_scratch(m, SCR_KEYS, (size_t)pairs * 4 + 16);
             void *p_v = store_scratch(m, SCR_VALS, (size_t)pairs * 4 + 16);
             void *p_k2 = store_scratch(m, SCR_KEYS2, (size_t)pairs * 4 + 16);
             void *p_v2 = store_scratch(m, SCR_VALS2, (size_t)pairs * 4 + 16);
             void *p_tmp = store_scratch(m, SCR_TMP, tb);
-            if (!p_inc || !p_deg || !p_off || !p_k || !p_v || !p_k2 || !p_v2 || !p_tmp)
+            if (!p_inc || !p_deg || !p_off || !p_rs || !p_k || !p_v || !p_k2 || !p_v2 || !p_tmp)
                 return fail(AKASHIC_ENOMEM, "update: out of device memory");
             InEdgeUpdate u;
             u.n = rows;
@@ -841,7 +842,7 @@ akashic_status_t akashic_mem_update_relations(akashic_mem_t *m, int64_t first, i
             u.rstat = m->rstat.as<float2>();
             InEdgeScratch sc{(int64_t *)p_inc, (int64_t *)p_deg, (int64_t *)p_off,
                              (uint32_t *)p_k, (uint32_t *)p_v, (uint32_t *)p_k2, (uint32_t *)p_v2,
-                             p_tmp, tb};
+                             p_tmp, tb, (float2 *)p_rs};
             CUDA_TRY(launch_in_edges_update(u, sc, st, &pt.launches));
             std::swap(m->in_ptr.p, ptr2.p);
             std::swap(m->in_ptr.cap, ptr2.cap);

@@ -195,26 +195,60 @@ __device__ __forceinline__ float row_softmax_weight(float aff, float2 stat) {
 }
 cudaError_t launch_row_softmax(const int64_t *row_ptr, const float *aff, float *w, int64_t n_rows,
                                float2 *rstat, cudaStream_t st);
-// For a wave of 32 consecutive edges of a CSR (lane l holds edge e, all
-// lanes call it; e < ptr[n]): the row of e, given r0 with ptr[r0] <= the
-// wave's first edge.  The 32 row ends after r0 are loaded once (one per
-// lane) and searched by shuffles; an edge past them walks on row by row.
-__device__ __forceinline__ int64_t wave_row(const int64_t *__restrict__ ptr, int64_t n,
-                                            int64_t r0, int64_t e) {
+// Edge-parallel moves of CSR rows: a warp takes CHUNK_E consecutive edges
+// [base, base + CHUNK_E), lane l the edges base + 32 j + l (j < CHUNK_E / 32),
+// and finds their rows without a search per edge.  Given r_lo, the row of
+// edge `base` (ptr[r_lo] <= base < ptr[r_lo + 1]), the warp marks in its own
+// shared array rid[] the first edge of every later row that starts inside
+// the chunk, as row - r_lo (where several rows start at one edge, the empty
+// rows before it, the largest wins); a running maximum over the positions,
+// taken 32 at a time across the lanes, gives every edge its row:
+// rows[j] = row of edge base + 32 j + lane - r_lo.  ptr has n + 1 entries,
+// ptr[n] = nnz.
+// All 32 lanes call it.  Chunks are small (four edges a lane) so that the
+// moving kernels stay at high occupancy: their loads are latency-bound.
+constexpr int CHUNK_E = 128;
+__device__ __forceinline__ void chunk_rows(const int64_t *__restrict__ ptr, int64_t n,
+                                           int64_t nnz, int64_t base, int64_t r_lo, int *rid,
+                                           int (&rows)[CHUNK_E / 32]) {
     const int lane = threadIdx.x & 31;
-    const int64_t idx = r0 + 1 + lane;
-    const int64_t bj = ptr[idx < n ? idx : n];        // end of row r0 + lane
-    int c = 0;                                        // row ends <= e among the first 31
 #pragma unroll
-    for (int step = 16; step >= 1; step >>= 1) {
-        const int64_t b = __shfl_sync(0xffffffffu, bj, c + step - 1);
-        if (b <= e) c += step;
+    for (int j = 0; j < CHUNK_E / 32; ++j) rid[32 * j + lane] = 0;
+    __syncwarp();
+    // rows starting at or past nnz own no edge (the empty rows at the end)
+    const int64_t lim = base + CHUNK_E < nnz ? base + CHUNK_E : nnz;
+    for (int64_t r0 = r_lo + 1; r0 < n; r0 += 32) {
+        const int64_t r = r0 + lane;
+        const int64_t s = r < n ? ptr[r] : INT64_MAX;   // > base for every r > r_lo
+        if (s < lim) atomicMax(&rid[s - base], (int)(r - r_lo));
+        if (__shfl_sync(0xffffffffu, s, 31) >= lim) break;
     }
-    const int64_t last = __shfl_sync(0xffffffffu, bj, 31);
-    if (last > e) return r0 + c;
-    int64_t r = r0 + 32;
-    while (ptr[r + 1] <= e) ++r;
-    return r;
+    __syncwarp();
+    int carry = 0;
+#pragma unroll
+    for (int j = 0; j < CHUNK_E / 32; ++j) {
+        int x = max(rid[32 * j + lane], carry);
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int t = __shfl_up_sync(0xffffffffu, x, o);
+            if (lane >= o) x = max(x, t);
+        }
+        rows[j] = x;
+        carry = __shfl_sync(0xffffffffu, x, 31);
+    }
+    __syncwarp();
+}
+// The row of edge e (e < ptr[n]) by binary search: the largest r with
+// ptr[r] <= e.
+__device__ __forceinline__ int64_t edge_row(const int64_t *__restrict__ ptr, int64_t n,
+                                            int64_t e) {
+    int64_t lo = 0, hi = n;
+    while (hi - lo > 1) {
+        const int64_t mid = (lo + hi) >> 1;
+        if (ptr[mid] <= e) lo = mid;
+        else hi = mid;
+    }
+    return lo;
 }
 // The store keeps chunks in HBM in page order: row r holds chunk ext_of[r],
 // chunk c lives in row row_of[c].  The out-edge CSR stays in chunk IDs; the
@@ -258,6 +292,7 @@ struct InEdgeScratch {
     uint32_t *keys, *vals, *keys2, *vals2;   // [n_new * M] each
     void *tmp;
     size_t tmp_bytes;                   // >= radix and scan needs
+    float2 *rstat_row;                  // [n]: rstat[ext_of[r]], the statistics by row
 };
 cudaError_t launch_in_edges_update(const InEdgeUpdate &u, const InEdgeScratch &s, cudaStream_t st,
                                    int *launches);

@@ -45,50 +45,71 @@ __global__ void k_in_deg_recip(const int32_t *__restrict__ row_of, int64_t first
 // from its logit and its source's row statistics on the way (a moved edge
 // whose source row did not change gets its old weight back bit for bit).
 // Edge-parallel (a row-parallel copy would leave one warp copying a hub's
-// ~10^5..10^6 edges): each warp takes COPY_PER_LANE waves of 32
-// consecutive old edges; the row of the first comes from a binary search,
-// the rows of a wave from wave_row.
-constexpr int COPY_PER_LANE = 16;
-__global__ void k_copy_in_edges(const int64_t *__restrict__ in_ptr_old,
-                                const int32_t *__restrict__ src_old,
-                                const float *__restrict__ aff_old, int64_t n, int64_t nnz_old,
-                                const int64_t *__restrict__ in_ptr_new,
-                                int32_t *__restrict__ src_new, float *__restrict__ aff_new,
-                                const int32_t *__restrict__ ext_of,
-                                const float2 *__restrict__ rstat, float *__restrict__ w_new) {
+// ~10^5..10^6 edges): chunks of CHUNK_E edges are dealt
+// round-robin to the warps; a warp finds the rows of a chunk at once
+// (chunk_rows), then issues all of a lane's loads for the chunk before any
+// store.
+__global__ __launch_bounds__(256) void k_copy_in_edges(
+    const int64_t *__restrict__ in_ptr_old, const int32_t *__restrict__ src_old,
+    const float *__restrict__ aff_old, int64_t n, int64_t nnz_old,
+    const int64_t *__restrict__ in_ptr_new, int32_t *__restrict__ src_new,
+    float *__restrict__ aff_new, const float2 *__restrict__ rstat_row,
+    float *__restrict__ w_new) {
+    __shared__ int rid_s[8][CHUNK_E];
+    constexpr int PER = CHUNK_E / 32;
     const int lane = threadIdx.x & 31;
-    const int64_t per_warp = 32 * COPY_PER_LANE;
+    int *rid = rid_s[threadIdx.x >> 5];
     const int64_t w0 = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
     const int64_t nw = ((int64_t)gridDim.x * blockDim.x) >> 5;
-    for (int64_t base = w0 * per_warp; base < nnz_old; base += nw * per_warp) {
-        // largest r with in_ptr_old[r] <= base (in_ptr_old[n] = nnz_old > base)
-        int64_t r = 0;
-        if (lane == 0) {
-            int64_t lo = 0, hi = n;
-            while (hi - lo > 1) {
-                const int64_t mid = (lo + hi) >> 1;
-                if (in_ptr_old[mid] <= base) lo = mid;
-                else hi = mid;
-            }
-            r = lo;
+    const int64_t n_chunks = (nnz_old + CHUNK_E - 1) / CHUNK_E;
+    // chunks dealt round-robin to the warps; the lanes find the first rows
+    // of a warp's next 32 chunks at once, one binary search each
+    int64_t first = 0;
+    int i = 0;
+    for (int64_t c = w0; c < n_chunks; c += nw, ++i) {
+        if ((i & 31) == 0) {
+            const int64_t cl = c + (int64_t)lane * nw;
+            first = cl < n_chunks ? edge_row(in_ptr_old, n, cl * CHUNK_E) : 0;
         }
-        r = __shfl_sync(0xffffffffu, r, 0);
-        for (int i = 0; i < COPY_PER_LANE; ++i) {
-            const int64_t e0 = base + 32 * i;
-            if (e0 >= nnz_old) break;
-            const int64_t e = e0 + lane < nnz_old ? e0 + lane : nnz_old - 1;
-            const int64_t row = wave_row(in_ptr_old, n, r, e);
-            if (e0 + lane < nnz_old) {
-                const int64_t pos = e + (in_ptr_new[row] - in_ptr_old[row]);
-                const int32_t src = src_old[e];
-                const float a = aff_old[e];
-                src_new[pos] = src;
-                aff_new[pos] = a;
-                w_new[pos] = row_softmax_weight(a, rstat[ext_of[src]]);
+        const int64_t base = c * CHUNK_E;
+        const int64_t r_lo = __shfl_sync(0xffffffffu, first, i & 31);
+        {
+            int rows[PER];
+            chunk_rows(in_ptr_old, n, nnz_old, base, r_lo, rid, rows);
+            int32_t src[PER];
+            float a[PER];
+            int64_t pos[PER];
+#pragma unroll
+            for (int j = 0; j < PER; ++j) {
+                const int64_t e = base + 32 * j + lane;
+                const int64_t row = r_lo + rows[j];
+                const bool ok = e < nnz_old;
+                src[j] = ok ? src_old[e] : 0;
+                a[j] = ok ? aff_old[e] : 0.f;
+                pos[j] = ok ? e + (in_ptr_new[row] - in_ptr_old[row]) : -1;
             }
-            r = __shfl_sync(0xffffffffu, row, 31);
+            float2 st[PER];
+#pragma unroll
+            for (int j = 0; j < PER; ++j) st[j] = pos[j] >= 0 ? rstat_row[src[j]] : make_float2(0.f, 0.f);
+#pragma unroll
+            for (int j = 0; j < PER; ++j) {
+                if (pos[j] < 0) continue;
+                src_new[pos[j]] = src[j];
+                aff_new[pos[j]] = a[j];
+                w_new[pos[j]] = row_softmax_weight(a[j], st[j]);
+            }
+            __syncwarp();
         }
     }
+}
+
+// The row statistics by row: rstat_row[r] = rstat[ext_of[r]] (one gather
+// per moved in-edge instead of two).
+__global__ void k_rstat_rows(const int32_t *__restrict__ ext_of, const float2 *__restrict__ rstat,
+                             int64_t n, float2 *__restrict__ rstat_row) {
+    for (int64_t r = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; r < n;
+         r += (int64_t)gridDim.x * blockDim.x)
+        rstat_row[r] = rstat[ext_of[r]];
 }
 
 // keys[p] = row of the new chunk of pair p (pairs are [new chunk][slot]).
@@ -189,13 +210,14 @@ cudaError_t launch_in_edges_update(const InEdgeUpdate &u, const InEdgeScratch &s
     if (e != cudaSuccess) return e;
     const int64_t nnz_old = u.nnz_new - pairs * (u.reciprocal ? 2 : 1);
     if (nnz_old > 0) {
-        const int64_t warps = ceil_div<int64_t>(nnz_old, 32 * COPY_PER_LANE);
+        k_rstat_rows<<<sms * 4, 256, 0, st>>>(u.ext_of, u.rstat, u.n, s.rstat_row);
+        const int64_t warps = ceil_div<int64_t>(nnz_old, CHUNK_E);
         const int64_t grid = ceil_div<int64_t>(warps, 8);
-        k_copy_in_edges<<<(unsigned)(grid < (int64_t)sms * 16 ? grid : (int64_t)sms * 16), 256, 0,
+        k_copy_in_edges<<<(unsigned)(grid < (int64_t)sms * 6 ? grid : (int64_t)sms * 6), 256, 0,
                           st>>>(u.in_ptr_old, u.in_src_old, u.in_aff_old, u.n, nnz_old,
-                                u.in_ptr_new, u.in_src_new, u.in_aff_new, u.ext_of, u.rstat,
+                                u.in_ptr_new, u.in_src_new, u.in_aff_new, s.rstat_row,
                                 u.in_w_new);
-        ++L;
+        L += 2;
     }
     if (pairs > 0) {
         // forward pairs by (target row, source row): sort by source row,

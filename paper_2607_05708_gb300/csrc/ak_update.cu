@@ -167,16 +167,6 @@ akashic_status_t relate_top_m(const UpdateArgs &a, cudaStream_t st, int *launche
 }
 
 // ------------------------------------------------------------------ CSR insert
-// An existing edge into a new chunk would make a reciprocal edge a repeat.
-__global__ void k_check_no_edge_into(const int32_t *__restrict__ col, int64_t nnz, int64_t lo,
-                                     int64_t hi, int *status) {
-    for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < nnz;
-         e += (int64_t)gridDim.x * blockDim.x) {
-        const int64_t c = col[e];
-        if (c >= lo && c < hi) set_status(status, AKASHIC_EDEVICE);
-    }
-}
-
 // new degree of every row: old degree, + M for new rows, + reciprocal count
 __global__ void k_new_degree(const int64_t *__restrict__ rp, int64_t n_rows, int64_t first,
                              int64_t n_new, int M, const int64_t *__restrict__ recip,
@@ -197,43 +187,60 @@ __global__ void k_count_recip(const int32_t *__restrict__ nbr, int64_t pairs,
         atomicAdd(&recip[nbr[p]], 1ull);
 }
 
-// Old edges keep their order at the front of each row (one warp per row).
-// Edge-parallel: each warp takes OLD_PER_LANE waves of 32 consecutive old
-// edges; the row of the first comes from a binary search, the rows of a
-// wave from wave_row; edge e of row r goes to nrp[r] + (e - rp[r]).
-constexpr int OLD_PER_LANE = 16;
-__global__ void k_copy_old_rows(const int64_t *__restrict__ rp, const int32_t *__restrict__ col,
-                                const float *__restrict__ aff, int64_t n_rows,
-                                const int64_t *__restrict__ nrp, int32_t *__restrict__ ncol,
-                                float *__restrict__ naff) {
+// Old edges keep their order at the front of each row.  Edge-parallel:
+// chunks of CHUNK_E old edges are dealt round-robin to the warps; a warp
+// finds the rows of a chunk at once (chunk_rows), then issues all of a
+// lane's loads for the chunk before any store; edge e of row r goes to
+// nrp[r] + (e - rp[r]).
+__global__ __launch_bounds__(256) void k_copy_old_rows(
+    const int64_t *__restrict__ rp, const int32_t *__restrict__ col,
+    const float *__restrict__ aff, int64_t n_rows, const int64_t *__restrict__ nrp,
+    int32_t *__restrict__ ncol, float *__restrict__ naff, int64_t new_lo, int64_t new_hi,
+    int *status) {
+    __shared__ int rid_s[8][CHUNK_E];
+    constexpr int PER = CHUNK_E / 32;
     const int lane = threadIdx.x & 31;
+    int *rid = rid_s[threadIdx.x >> 5];
     const int64_t nnz = rp[n_rows];
-    const int64_t per_warp = 32 * OLD_PER_LANE;
     const int64_t w0 = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
     const int64_t nw = ((int64_t)gridDim.x * blockDim.x) >> 5;
-    for (int64_t base = w0 * per_warp; base < nnz; base += nw * per_warp) {
-        int64_t r = 0;                                // largest r with rp[r] <= base
-        if (lane == 0) {
-            int64_t lo = 0, hi = n_rows;
-            while (hi - lo > 1) {
-                const int64_t mid = (lo + hi) >> 1;
-                if (rp[mid] <= base) lo = mid;
-                else hi = mid;
-            }
-            r = lo;
+    const int64_t n_chunks = (nnz + CHUNK_E - 1) / CHUNK_E;
+    // chunks dealt round-robin to the warps; the lanes find the first rows
+    // of a warp's next 32 chunks at once, one binary search each
+    int64_t first = 0;
+    int i = 0;
+    for (int64_t c = w0; c < n_chunks; c += nw, ++i) {
+        if ((i & 31) == 0) {
+            const int64_t cl = c + (int64_t)lane * nw;
+            first = cl < n_chunks ? edge_row(rp, n_rows, cl * CHUNK_E) : 0;
         }
-        r = __shfl_sync(0xffffffffu, r, 0);
-        for (int i = 0; i < OLD_PER_LANE; ++i) {
-            const int64_t e0 = base + 32 * i;
-            if (e0 >= nnz) break;
-            const int64_t e = e0 + lane < nnz ? e0 + lane : nnz - 1;
-            const int64_t row = wave_row(rp, n_rows, r, e);
-            if (e0 + lane < nnz) {
-                const int64_t pos = nrp[row] + (e - rp[row]);
-                ncol[pos] = col[e];
-                naff[pos] = aff[e];
+        const int64_t base = c * CHUNK_E;
+        const int64_t r_lo = __shfl_sync(0xffffffffu, first, i & 31);
+        {
+            int rows[PER];
+            chunk_rows(rp, n_rows, nnz, base, r_lo, rid, rows);
+            int32_t cv[PER];
+            float av[PER];
+            int64_t pos[PER];
+#pragma unroll
+            for (int j = 0; j < PER; ++j) {
+                const int64_t e = base + 32 * j + lane;
+                const int64_t row = r_lo + rows[j];
+                const bool ok = e < nnz;
+                cv[j] = ok ? col[e] : 0;
+                av[j] = ok ? aff[e] : 0.f;
+                pos[j] = ok ? e + (nrp[row] - rp[row]) : -1;
             }
-            r = __shfl_sync(0xffffffffu, row, 31);
+#pragma unroll
+            for (int j = 0; j < PER; ++j) {
+                if (pos[j] < 0) continue;
+                // an existing edge into a new chunk would make a reciprocal
+                // edge a repeat
+                if (cv[j] >= new_lo && cv[j] < new_hi) set_status(status, AKASHIC_EDEVICE);
+                ncol[pos[j]] = cv[j];
+                naff[pos[j]] = av[j];
+            }
+            __syncwarp();
         }
     }
 }
@@ -302,20 +309,20 @@ akashic_status_t csr_insert(const UpdateArgs &a, const int64_t *rp, const int32_
     cudaError_t e = cudaSuccess;
     int L = 0;
     if (rc == AKASHIC_OK) {
-        k_check_no_edge_into<<<sms * 4, 256, 0, st>>>(col, nnz, a.first, a.first + a.n_new, a.status);
         cudaMemsetAsync(recip, 0, (size_t)(n_rows + 1) * 8, st);
         if (a.reciprocal)
             k_count_recip<<<sms * 4, 256, 0, st>>>(a.nbr_ids, pairs, (unsigned long long *)recip);
         k_new_degree<<<sms * 4, 256, 0, st>>>(rp, n_rows, a.first, a.n_new, a.M,
                                               a.reciprocal ? recip : nullptr, deg);
-        L += 4;
+        L += 3;
         e = cudaGetLastError();
         if (e == cudaSuccess) e = scan_exclusive(deg, new_rp, n_rows, tmp, tmp_bytes, st);
         if (e == cudaSuccess) {
-            const int64_t warps = ceil_div<int64_t>(nnz, 32 * OLD_PER_LANE);
+            const int64_t warps = ceil_div<int64_t>(nnz, CHUNK_E);
             const int64_t g = ceil_div<int64_t>(warps > 0 ? warps : 1, 8);
-            k_copy_old_rows<<<(unsigned)(g < (int64_t)sms * 16 ? g : (int64_t)sms * 16), 256, 0,
-                              st>>>(rp, col, aff, n_rows, new_rp, new_col, new_aff);
+            k_copy_old_rows<<<(unsigned)(g < (int64_t)sms * 6 ? g : (int64_t)sms * 6), 256, 0,
+                              st>>>(rp, col, aff, n_rows, new_rp, new_col, new_aff, a.first,
+                                    a.first + a.n_new, a.status);
             k_fill_new_rows<<<sms * 2, 256, 0, st>>>(a.nbr_ids, a.nbr_cos, a.first, a.n_new, a.M,
                                                      a.scale, new_rp, new_col, new_aff);
             L += 2;

@@ -11,7 +11,7 @@ enum UpdateScratchSlot {
     SCR_DOTS, SCR_CAND,                                                      // relate (batched)
     SCR_DEG, SCR_RECIP, SCR_RECIP_OFF, SCR_KEYS, SCR_VALS, SCR_KEYS2, SCR_VALS2, SCR_TMP,
     SCR_NBR_IDS, SCR_NBR_COS,                                                // update results
-    SCR_IN_INC, SCR_IN_DEG, SCR_IN_OFF,                                      // transpose patch
+    SCR_IN_INC, SCR_IN_DEG, SCR_IN_OFF, SCR_IN_RSTAT,                        // transpose patch
     SCR_DEAD_S,                                                              // relate sample
     SCR_DEL_KEEP, SCR_DEL_POS, SCR_DEL_TMP,                                  // deletion
     SCR_MM_G, SCR_MM_GN, SCR_MM_CAND, SCR_MM_MOVING, SCR_MM_POS, SCR_MM_PARENT,  // memory
