@@ -229,12 +229,17 @@ __device__ __forceinline__ void rs_rank(const uint32_t *__restrict__ keys,
     for (int d = lane; d < 256; d += 32) cnt[warp][d] = 0;
     __syncwarp();
     const unsigned lt = (1u << lane) - 1u;
+    // every load first, then the ranking (whose rounds depend on each other)
+#pragma unroll
+    for (int r = 0; r < RS_ITEMS; ++r) {
+        const int64_t idx = base + r * 32 + lane;
+        k[r] = idx < n ? keys[idx] : 0u;
+        v[r] = idx < n ? vals[idx] : 0u;
+    }
 #pragma unroll
     for (int r = 0; r < RS_ITEMS; ++r) {
         int64_t idx = base + r * 32 + lane;
         bool ok = idx < n;
-        k[r] = ok ? keys[idx] : 0u;
-        v[r] = ok ? vals[idx] : 0u;
         uint32_t d = ok ? ((k[r] >> shift) & mask) : 0x100u;   // 0x100: no digit
         unsigned peers = __match_any_sync(0xffffffffu, d);
         int leader = __ffs(peers) - 1;
@@ -325,7 +330,7 @@ __global__ __launch_bounds__(RS_THREADS) void k_rs_scatter_small(
         const int d = threadIdx.x;
         const int *row = hcur + (int64_t)d * n_tiles;
         int tot = 0, before = 0;
-#pragma unroll 8
+#pragma unroll 16
         for (int t = 0; t < n_tiles; ++t) {
             const int c = row[t];
             tot += c;

@@ -303,7 +303,7 @@ constexpr int KS_WARPS = 4, KS_BUF = 512, KS_U = 16, KS_KMAX = 64;
 // least k keys are >= the prefix with it set (the largest t with k keys
 // >= t is the k-th largest key).  No shared-memory atomics: the sampled
 // keys of one column share their top bits, so histogram bins would collide.
-__device__ uint32_t warp_kth(const uint32_t *a, int len, int k) {
+__device__ __noinline__ uint32_t warp_kth(const uint32_t *a, int len, int k) {
     const int lane = threadIdx.x & 31;
     uint32_t x[KS_BUF / 32];
 #pragma unroll
@@ -325,7 +325,9 @@ __device__ uint32_t warp_kth(const uint32_t *a, int len, int k) {
 }
 
 // Cut a[0..len) (len >= k) to its k largest; returns the k-th largest.
-__device__ uint32_t warp_cut(uint32_t *a, int len, int k) {
+// (Called out of line from the scan's unrolled loop, which it would
+// otherwise bloat past the instruction cache.)
+__device__ __noinline__ uint32_t warp_cut(uint32_t *a, int len, int k) {
     const int lane = threadIdx.x & 31;
     const unsigned lt = (1u << lane) - 1u;
     const uint32_t x = warp_kth(a, len, k);
