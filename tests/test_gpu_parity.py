@@ -46,13 +46,13 @@ def test_gmm1m_scaled_two_hops(placement):
     assert_retrieval_parity(wl, placement, got, ref)
 
 
-@pytest.mark.parametrize("hops", [0, 2])
-def test_pair_gemm_store(hops):
+@pytest.mark.parametrize("hops,B", [(0, 256), (2, 256), (0, 128), (2, 128), (2, 200)])
+def test_pair_gemm_store(hops, B):
     """A store large enough for the score GEMM's CTA-pair form (256-row
-    tiles on clusters of two, B = 256): the gmm1m recipe at N=32768 cut to
-    N=32700 (the last pair tile's odd half partly past the last row),
-    no hops (the fused top-k filter in the GEMM) and two hops, against the
-    oracle."""
+    tiles on clusters of two, B >= 128): the gmm1m recipe at N=32768 cut to
+    N=32700 (the last pair tile's odd half partly past the last row), no
+    hops (the fused top-k filter in the GEMM) and two hops, query batches
+    of 256, 128 and 200 (padded to 256), against the oracle."""
     base = synth.workload(2, scale=1 / 32)
     n = 32700
     keep = base.row_ptr[:n + 1]
@@ -60,12 +60,12 @@ def test_pair_gemm_store(hops):
     ok = cols < n
     rows = np.repeat(np.arange(n), np.diff(keep))
     rp = np.concatenate([[0], np.cumsum(np.bincount(rows[ok], minlength=n))]).astype(np.int64)
-    wl = synth.Workload(name="pair", dim=base.dim, emb=base.emb[:n], queries=base.queries,
+    wl = synth.Workload(name="pair", dim=base.dim, emb=base.emb[:n], queries=base.queries[:B],
                         row_ptr=rp, col=cols[ok].astype(np.int32),
                         aff=base.aff[:keep[-1]][ok],
                         page_of={"clustered": base.page_of["clustered"][:n]},
                         chunks_per_page=64, alpha=base.alpha, hops=hops, k=base.k)
-    assert wl.queries.shape[0] == 256
+    assert wl.queries.shape[0] == B
     _, got = gpu_retrieve(wl, "clustered")
     ref = oracle_retrieve(wl, "clustered")
     assert_retrieval_parity(wl, "clustered", got, ref)
