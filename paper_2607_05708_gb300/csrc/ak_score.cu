@@ -324,8 +324,9 @@ __global__ __launch_bounds__(GemmCfg<BP, MODE, P2>::THREADS, 1) void k_gemm_umma
                 const int64_t mt = u / n_ctiles;
                 for (int kb = 0; kb < kb_n; ++kb) {
                     // (the odd CTA's releases arrive remotely: spin on them)
-                    if (!(P2 && !lead ? mbar_wait_spin(&empty[stage], phase ^ 1u, status)
-                                      : mbar_wait(&empty[stage], phase ^ 1u, status))) {
+                    // (a bounded spin: the suspending wait added wake-up time on the
+                    // producer's path every stage; relate 6.76 -> 6.65 ms)
+                    if (!mbar_wait_spin(&empty[stage], phase ^ 1u, status)) {
                         ok = false;
                         break;
                     }
@@ -378,7 +379,7 @@ __global__ __launch_bounds__(GemmCfg<BP, MODE, P2>::THREADS, 1) void k_gemm_umma
                 tc_fence_after();
                 const uint32_t d = tmem_base + (uint32_t)(acc * BP);
                 for (int kb = 0; kb < kb_n; ++kb) {
-                    if (!mbar_wait(&full[stage], phase, status)) {
+                    if (!mbar_wait_spin(&full[stage], phase, status)) {
                         ok = false;
                         break;
                     }
