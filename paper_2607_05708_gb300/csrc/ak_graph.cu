@@ -489,14 +489,20 @@ __global__ void k_row_softmax(const int64_t *__restrict__ row_ptr, const float *
     constexpr int L = RSM_LANES, R = 32 / RSM_LANES;
     const int lane = threadIdx.x & 31, sub = lane % L, grp = lane / L;
     const int64_t nw = ((int64_t)gridDim.x * blockDim.x) >> 5;
-    for (int64_t r0 = (((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5) * R; r0 < n_rows;
-         r0 += nw * R) {
+    // the next step's row bounds are loaded while this step's rows are
+    // processed (they head each step's chain of dependent loads)
+    int64_t r0 = (((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5) * R;
+    int64_t na = 0, nb = 0;
+    if (r0 + grp < n_rows) {
+        na = row_ptr[r0 + grp];
+        nb = row_ptr[r0 + grp + 1];
+    }
+    for (; r0 < n_rows; r0 += nw * R) {
         const int64_t r = r0 + grp;
-        int64_t a = 0, b = 0;
-        if (r < n_rows) {
-            a = row_ptr[r];
-            b = row_ptr[r + 1];
-        }
+        const int64_t a = na, b = nb;
+        const int64_t rn = r + nw * R;
+        na = rn < n_rows ? row_ptr[rn] : 0;
+        nb = rn < n_rows ? row_ptr[rn + 1] : 0;
         float v[RSM_KEEP];
         float m = -INFINITY;
 #pragma unroll
