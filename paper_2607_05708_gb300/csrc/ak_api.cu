@@ -1280,6 +1280,22 @@ static akashic_status_t retrieve_impl(akashic_mem *m, const uint16_t *q, int32_t
                                  sp2.words <= sp.words;
         unsigned long long *ws = sc->cand.as<unsigned long long>();
         ColumnRecompute rc{};
+        // the two-hop reach path is tried (its plan may still send the call
+        // through the hops): the score GEMM then writes u as split bf16, the
+        // operand form the candidates' tensor-core pass loads, in the bytes
+        // of the fp32 slab (hi [n][bp], then lo [n][bp])
+        const bool reach_try = prune && eff_hops == 2 && !q_ns && m->reach_on &&
+                               m->n_split > 0 && (bp == 256 || bp == 128);
+        uint16_t *u_hi = reach_try ? sc->u.as<uint16_t>() : nullptr;
+        uint16_t *u_lo = reach_try ? u_hi + (size_t)n * bp : nullptr;
+        auto score_fp32 = [&](int *launches) -> cudaError_t {
+            return launch_score(m->emb.as<uint16_t>(), n, m->dim, sc->qp.as<uint16_t>(), bp,
+                                sc->shift.as<float>(), m->tau, sc->u.as<float>(),
+                                sc->zpart.as<float>(), m->status.as<int>(), st, launches, &zrows,
+                                ns.dead, prune ? sc->rmax_u.as<float>() : nullptr,
+                                prune ? sc->rmin_u.as<float>() : nullptr, b,
+                                prune ? sc->ext.as<unsigned int>() : nullptr);
+        };
         {
             PhaseScope ph(m, AKASHIC_PHASE_SCORE, st);
             // with the row bounds (never with the dense fused filter) the
@@ -1290,14 +1306,15 @@ static akashic_status_t retrieve_impl(akashic_mem *m, const uint16_t *q, int32_t
                                          m->status.as<int>(), st,
                                          prune ? sc->ext.as<unsigned int>() : nullptr));
             ph.launches += 1;
-            if (!dense_fused)
-                CUDA_TRY(launch_score(m->emb.as<uint16_t>(), n, m->dim, sc->qp.as<uint16_t>(), bp,
-                                      sc->shift.as<float>(), m->tau, sc->u.as<float>(),
-                                      sc->zpart.as<float>(), m->status.as<int>(), st,
-                                      &ph.launches, &zrows, ns.dead,
-                                      prune ? sc->rmax_u.as<float>() : nullptr,
-                                      prune ? sc->rmin_u.as<float>() : nullptr, b,
-                                      prune ? sc->ext.as<unsigned int>() : nullptr));
+            if (reach_try)
+                CUDA_TRY(launch_score_split(m->emb.as<uint16_t>(), n, m->dim,
+                                            sc->qp.as<uint16_t>(), bp, sc->shift.as<float>(),
+                                            m->tau, u_hi, u_lo, sc->zpart.as<float>(),
+                                            m->status.as<int>(), st, &ph.launches, &zrows, ns.dead,
+                                            sc->rmax_u.as<float>(), sc->rmin_u.as<float>(), b,
+                                            sc->ext.as<unsigned int>()));
+            else if (!dense_fused)
+                CUDA_TRY(score_fp32(&ph.launches));
         }
         if (dense_fused) {
             {
@@ -1370,8 +1387,6 @@ static akashic_status_t retrieve_impl(akashic_mem *m, const uint16_t *q, int32_t
             // (the two-hop reach path evaluates them only where it needs them
             // and writes the arrays only when the hops run after all)
             const float *row_ub = nullptr, *row_lb = nullptr;
-            const bool reach_try = prune && eff_hops == 2 && !q_ns && m->reach_on &&
-                                   m->n_split > 0 && (bp == 256 || bp == 128);
             auto row_bounds = [&]() -> akashic_status_t {
                 PhaseScope ph(m, AKASHIC_PHASE_BOUND, st);
                 CUDA_TRY(launch_final_bounds(sc->rmax_u.as<float>(), sc->rmin_u.as<float>(),
@@ -1452,7 +1467,7 @@ static akashic_status_t retrieve_impl(akashic_mem *m, const uint16_t *q, int32_t
                         sc->coef_H = eff_hops;
                         sc->coef_n = n;
                     }
-                    CUDA_TRY(launch_reach_scores(sc->u.as<float>(), bp, b, n,
+                    CUDA_TRY(launch_reach_scores(u_hi, u_lo, bp, b, n,
                                                  sc->coef_hi.as<uint16_t>(),
                                                  sc->coef_lo.as<uint16_t>(),
                                                  sc->reach_plan.as<int32_t>(),
@@ -1467,7 +1482,13 @@ static akashic_status_t retrieve_impl(akashic_mem *m, const uint16_t *q, int32_t
                     rc = ColumnRecompute{};   // the buffers hold every candidate
                     reach_done = true;
                 } else {
-                    AK_TRY(row_bounds());     // the hops run: they need every row's bounds
+                    // the hops run: they read u in fp32 (the same scores again)
+                    // and need every row's bounds
+                    {
+                        PhaseScope ph(m, AKASHIC_PHASE_SCORE, st);
+                        CUDA_TRY(score_fp32(&ph.launches));
+                    }
+                    AK_TRY(row_bounds());
                 }
             }
             for (int h = 0; h < eff_hops && !reach_done; ++h) {

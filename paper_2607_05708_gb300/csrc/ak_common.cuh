@@ -2,6 +2,7 @@
 // Nothing here is part of the public ABI (include/akashic_mem.h is).
 #pragma once
 
+#include <cuda_bf16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -54,6 +55,17 @@ __host__ __device__ __forceinline__ bool scope_active(const NsScope &s) {
     return s.q_ns != nullptr || s.dead != nullptr;
 }
 
+// Split-bf16 of two fp32 values: hi = bf16(x) (round to nearest), lo =
+// bf16(x - hi) (x - hi is exact in fp32), packed two to a word (x in the low
+// half); x = hi + lo to within 2^-17 relative.
+__device__ __forceinline__ uint32_t split_bf16_pair(float x, float y, uint32_t &lo) {
+    const __nv_bfloat16 hx = __float2bfloat16_rn(x), hy = __float2bfloat16_rn(y);
+    const __nv_bfloat16 lx = __float2bfloat16_rn(x - __bfloat162float(hx));   // exact rest
+    const __nv_bfloat16 ly = __float2bfloat16_rn(y - __bfloat162float(hy));
+    lo = (uint32_t)__bfloat16_as_ushort(lx) | ((uint32_t)__bfloat16_as_ushort(ly) << 16);
+    return (uint32_t)__bfloat16_as_ushort(hx) | ((uint32_t)__bfloat16_as_ushort(hy) << 16);
+}
+
 // log2(e): scores exp(tau x - c) are evaluated as 2^(x tau log2(e) - c log2(e))
 // (one FMA and the hardware exp2).
 constexpr float LOG2E_F = 1.44269504088896340736f;
@@ -96,6 +108,14 @@ cudaError_t launch_score(const uint16_t *emb, int64_t n, int dim, const uint16_t
                          cudaStream_t st, int *launches, int *zrows,
                          const int32_t *dead_row = nullptr, float *row_max = nullptr,
                          float *row_min = nullptr, int n_real = 0, unsigned int *ext = nullptr);
+// The same scores with u written as split bf16 instead of fp32: u_hi and u_lo
+// [n][bp] each, u = hi + lo to within 2^-17 relative (the operand form the
+// candidates' tensor-core pass reads); Z's column sums from the fp32 values.
+cudaError_t launch_score_split(const uint16_t *emb, int64_t n, int dim, const uint16_t *qp, int bp,
+                               const float *shift, float tau, uint16_t *u_hi, uint16_t *u_lo,
+                               float *zpart, int *status, cudaStream_t st, int *launches,
+                               int *zrows, const int32_t *dead_row, float *row_max,
+                               float *row_min, int n_real, unsigned int *ext);
 
 // The score on every stride-th row only: out[v, c] = u[v*stride, c] for
 // v < n_sample (same kernel and arithmetic as launch_score, so the values
@@ -617,8 +637,9 @@ cudaError_t launch_reach_pack(const float *C, int64_t n, int H, float alpha, uin
 // partial: [reach_parts()][REACH_T][bp] scratch; with plan[0] = 1 the
 // flagged candidates' keys are written to each real column's buffer
 // (cnt[b] = nk); with plan[0] = 0 both kernels return at once.  bp = 128
-// or 256.
-cudaError_t launch_reach_scores(const float *u, int bp, int B, int64_t n, const uint16_t *coef_hi,
+// or 256.  u_hi, u_lo: the score GEMM's split-bf16 u, [n][bp] each.
+cudaError_t launch_reach_scores(const uint16_t *u_hi, const uint16_t *u_lo, int bp, int B,
+                                int64_t n, const uint16_t *coef_hi,
                                 const uint16_t *coef_lo, const int32_t *plan, const int32_t *rows,
                                 const int32_t *ext_of, float *partial, unsigned int *cnt,
                                 unsigned long long *buf, int64_t cap, int *status, cudaStream_t st,

@@ -232,30 +232,28 @@ cudaError_t launch_reach_flags(const ReachFlags &f, cudaStream_t st, int *launch
 //   A = the combined coefficients sum_t alpha^t C_t, packed by
 //       k_reach_pack as [REACH_T slots][n_pad rows] bf16 (hi, lo), loaded
 //       by TMA as K-major tiles [128 slots][64 rows] in the 128-byte swizzle;
-//   B = u, loaded by converter warps from global memory (two float4 of one
-//       row per lane, one row per warp instruction at BP = 256), split into hi / lo and
-//       stored as MN-major tiles [64 rows][BP queries]: atoms of 8 rows x 64
-//       queries (128 bytes a row, 16-byte chunks swizzled by the row), four
-//       (BP = 256) or two such atom columns RM_BK * 128 bytes apart.
+//   B = u as the score GEMM wrote it, split bf16 [n rows][BP queries] (hi,
+//       lo), loaded by TMA as MN-major tiles [64 rows][BP queries]: boxes of
+//       64 rows x 64 queries in the 128-byte swizzle (128 bytes a row, the
+//       16-byte chunk c of row r at c ^ (r % 8)), i.e. atoms of 8 rows x 64
+//       queries, the BP / 64 boxes RM_BK * 128 bytes apart.
 // D[slot][query] (M = 128 slots = TMEM lanes, N = BP queries = columns).
 // The tensor core's accumulation of many positive terms drifts (each add
 // into the fp32 accumulator may round the same way), so an accumulator
 // takes only RM_CHUNK stages (1024 rows, 192 MMAs): two accumulators
-// alternate, and the converter warps add each finished one into the CTA's
+// alternate, and the flush warps add each finished one into the CTA's
 // partial with ordinary round-to-nearest fp32 adds (the partial rows stay
 // in L2) while the MMAs fill the other.
-// Warps: 0 TMA producer (A), 1 MMA issuer, 2..9 converters, eight rows of
-// a stage each (and the flush: warp w reads TMEM lanes 32 (w % 4) ..,
-// column half (w - 2) / 4).  Sixteen converter warps with half the rows
-// each measured slower (290 against 260 us at full size), as did an L2
-// prefetch of u three stages ahead (280 us).  Each
-// CTA takes a contiguous range of 64-row stages; 2 stages of 2 A + 2 B
-// tiles.
+// Warps: 0 TMA producer (A and B), 1 MMA issuer, 2..9 flush (warp w reads
+// TMEM lanes 32 (w % 4) .., column half (w - 2) / 4).  Both operands
+// arrive by TMA, so the bytes in flight are the two stages' 192 KB of
+// shared memory, not registers.  Each CTA takes a contiguous range of
+// 64-row stages.
 constexpr int RM_BK = 64;                // store rows (K) per stage
 constexpr int RM_M = REACH_T;            // candidate slots (M)
 constexpr int RM_STAGES = 2;
-constexpr int RM_CONV_W = 8;             // converter warps (8 rows of a stage each)
-constexpr int RM_THREADS = 64 + 32 * RM_CONV_W;
+constexpr int RM_FLUSH_W = 8;            // flush warps
+constexpr int RM_THREADS = 64 + 32 * RM_FLUSH_W;
 constexpr int RM_CHUNK = 16;             // stages per accumulator
 
 template <int BP>
@@ -266,31 +264,18 @@ struct RmCfg {
     static constexpr uint32_t LBO = RM_BK * 128;                 // between query atoms
     static constexpr uint32_t SBO = 8 * 128;                     // between 8-row groups
     static constexpr int SMEM = 1024 + RM_STAGES * STAGE_BYTES + 256;
-    static constexpr int CH = BP / 8;        // 16-byte bf16 chunks of a u row
-    static constexpr int RPI = 32 / CH;      // u rows per warp instruction
-    static constexpr int RPW = RM_BK / RM_CONV_W;   // u rows per converter warp per stage
-    static constexpr int ITEMS = RPW / RPI;  // (row, chunk) items per lane per stage
-    static constexpr int PARTS = RM_CONV_W / 4;     // column parts of a flush
-    static_assert(ITEMS >= 1 && RPW % RPI == 0, "converter layout");
+    static constexpr int PARTS = RM_FLUSH_W / 4;     // column parts of a flush
     static constexpr int TMEM_COLS = 2 * BP; // two accumulators
     static_assert(BP == 128 || BP == 256, "query widths 128 and 256");
     static_assert(SMEM <= 227 * 1024, "shared memory");
 };
 
-__device__ __forceinline__ uint32_t split_bf16_pair(float x, float y, uint32_t &lo) {
-    const __nv_bfloat16 hx = __float2bfloat16_rn(x), hy = __float2bfloat16_rn(y);
-    const __nv_bfloat16 lx = __float2bfloat16_rn(x - __bfloat162float(hx));   // exact rest
-    const __nv_bfloat16 ly = __float2bfloat16_rn(y - __bfloat162float(hy));
-    lo = (uint32_t)__bfloat16_as_ushort(lx) | ((uint32_t)__bfloat16_as_ushort(ly) << 16);
-    return (uint32_t)__bfloat16_as_ushort(hx) | ((uint32_t)__bfloat16_as_ushort(hy) << 16);
-}
-
 template <int BP>
 __global__ __launch_bounds__(RM_THREADS, 1) void k_reach_mma(
     const __grid_constant__ CUtensorMap tmAhi, const __grid_constant__ CUtensorMap tmAlo,
     const __grid_constant__ CUtensorMap tmAhi64, const __grid_constant__ CUtensorMap tmAlo64,
-    const float *__restrict__ u, int64_t n, const int32_t *__restrict__ plan,
-    float *__restrict__ partial, int *status) {
+    const __grid_constant__ CUtensorMap tmBhi, const __grid_constant__ CUtensorMap tmBlo,
+    int64_t n, const int32_t *__restrict__ plan, float *__restrict__ partial, int *status) {
     using C = RmCfg<BP>;
     if (plan[0] == 0) return;                          // the hops run instead
     // every flagged slot below 64: only the first 64 coefficient rows are
@@ -299,11 +284,10 @@ __global__ __launch_bounds__(RM_THREADS, 1) void k_reach_mma(
     const bool wide = plan[REACH_PLAN_WIDE] != 0;
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = (uint8_t *)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
-    uint64_t *afull = (uint64_t *)(smem + RM_STAGES * C::STAGE_BYTES);
-    uint64_t *bfull = afull + RM_STAGES;              // RM_CONV_W arrivals
-    uint64_t *empty = bfull + RM_STAGES;              // the MMAs' commit
+    uint64_t *full = (uint64_t *)(smem + RM_STAGES * C::STAGE_BYTES);
+    uint64_t *empty = full + RM_STAGES;               // the MMAs' commit
     uint64_t *dfull = empty + RM_STAGES;              // [2] accumulator complete
-    uint64_t *dfree = dfull + 2;                      // [2] accumulator flushed (RM_CONV_W)
+    uint64_t *dfree = dfull + 2;                      // [2] accumulator flushed (RM_FLUSH_W)
     uint32_t *tmem_slot = (uint32_t *)(dfree + 2);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     auto a_hi = [&](int s) { return smem + s * C::STAGE_BYTES; };
@@ -320,13 +304,12 @@ __global__ __launch_bounds__(RM_THREADS, 1) void k_reach_mma(
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < RM_STAGES; ++s) {
-            mbar_init(&afull[s], 1);
-            mbar_init(&bfull[s], RM_CONV_W);
+            mbar_init(&full[s], 1);
             mbar_init(&empty[s], 1);
         }
         for (int a = 0; a < 2; ++a) {
             mbar_init(&dfull[a], 1);
-            mbar_init(&dfree[a], RM_CONV_W);
+            mbar_init(&dfree[a], RM_FLUSH_W);
         }
         mbar_fence_init();
     }
@@ -341,20 +324,27 @@ __global__ __launch_bounds__(RM_THREADS, 1) void k_reach_mma(
 
     if (warp == 0) {
         if (lane == 0 && ns > 0) {
-            // ---------------- TMA producer: A hi / lo [128 slots][64 rows]
+            // ---------------- TMA producer: A hi / lo [128 slots][64 rows],
+            // B hi / lo [64 rows][BP queries] as BP / 64 boxes each
             uint32_t stage = 0, phase = 0;
             int last_par[RM_STAGES];
             for (int s = 0; s < RM_STAGES; ++s) last_par[s] = -1;
             bool ok = true;
             for (int64_t t = 0; t < ns; ++t) {
-                if (!mbar_wait(&empty[stage], phase ^ 1u, status)) {
+                if (!mbar_wait_spin(&empty[stage], phase ^ 1u, status)) {
                     ok = false;
                     break;
                 }
-                mbar_expect_tx(&afull[stage], wide ? 2 * C::A_BYTES : C::A_BYTES);
+                mbar_expect_tx(&full[stage],
+                               (wide ? 2 * C::A_BYTES : C::A_BYTES) + 2 * C::B_BYTES);
                 const int kx = (int)((s0 + t) * RM_BK);
-                tma_load_2d(a_hi(stage), wide ? &tmAhi : &tmAhi64, &afull[stage], kx, 0);
-                tma_load_2d(a_lo(stage), wide ? &tmAlo : &tmAlo64, &afull[stage], kx, 0);
+                tma_load_2d(a_hi(stage), wide ? &tmAhi : &tmAhi64, &full[stage], kx, 0);
+                tma_load_2d(a_lo(stage), wide ? &tmAlo : &tmAlo64, &full[stage], kx, 0);
+#pragma unroll
+                for (int c = 0; c < BP / 64; ++c) {
+                    tma_load_2d(b_hi(stage) + c * C::LBO, &tmBhi, &full[stage], 64 * c, kx);
+                    tma_load_2d(b_lo(stage) + c * C::LBO, &tmBlo, &full[stage], 64 * c, kx);
+                }
                 last_par[stage] = (int)phase;
                 if (++stage == RM_STAGES) {
                     stage = 0;
@@ -363,7 +353,7 @@ __global__ __launch_bounds__(RM_THREADS, 1) void k_reach_mma(
             }
             if (!ok)   // let every copy this thread issued land before the CTA exits
                 for (int s = 0; s < RM_STAGES; ++s)
-                    if (last_par[s] >= 0) mbar_wait(&afull[s], (uint32_t)last_par[s], status);
+                    if (last_par[s] >= 0) mbar_wait(&full[s], (uint32_t)last_par[s], status);
         }
     } else if (warp == 1) {
         if (lane == 0 && ns > 0) {
@@ -376,11 +366,10 @@ __global__ __launch_bounds__(RM_THREADS, 1) void k_reach_mma(
                 const int acc = (int)(c & 1);
                 const bool first = t % RM_CHUNK == 0;
                 const bool last = t % RM_CHUNK == RM_CHUNK - 1 || t == ns - 1;
-                // the accumulator is free once the converters flushed its
+                // the accumulator is free once the flush warps emptied its
                 // previous chunk (c - 2)
                 if (first && !mbar_wait(&dfree[acc], (uint32_t)((c >> 1) & 1) ^ 1u, status)) break;
-                if (!mbar_wait(&afull[stage], phase, status) ||
-                    !mbar_wait(&bfull[stage], phase, status)) {
+                if (!mbar_wait_spin(&full[stage], phase, status)) {
                     ok = false;
                     break;
                 }
@@ -408,37 +397,24 @@ __global__ __launch_bounds__(RM_THREADS, 1) void k_reach_mma(
             }
         }
     } else {
-        // ---------------- converters: u rows -> B hi / lo (MN-major)
-        const int cw = warp - 2;
-        const int c8 = lane % C::CH;                  // chunk: queries 8 c8 .. 8 c8 + 7
-        const int rl = lane / C::CH;                  // row within a warp instruction
-        const int q = warp & 3;                       // flush: TMEM lanes 32 q ..
-        const int part = cw >> 2;                     // flush: column part
+        // ---------------- flush warps: each finished accumulator into the
+        // CTA's partial rows (the first chunk stores, the later ones add)
+        const int fw = warp - 2;
+        const int q = warp & 3;                       // TMEM lanes 32 q ..
+        const int part = fw >> 2;                     // column part
         const int slot = q * 32 + lane;
         constexpr int PW = BP / C::PARTS;             // columns of a part
         float *o = partial + ((int64_t)blockIdx.x * REACH_T + slot) * BP + part * PW;
-        float4 cur[C::ITEMS][2], nxt[C::ITEMS][2];
-        auto load = [&](int64_t t, float4 (&dst)[C::ITEMS][2]) {
-#pragma unroll
-            for (int i = 0; i < C::ITEMS; ++i) {
-                const int64_t k = (s0 + t) * RM_BK + C::RPW * cw + i * C::RPI + rl;
-                if (k < n) {
-                    const float4 *src = reinterpret_cast<const float4 *>(u + k * BP + 8 * c8);
-                    dst[i][0] = __ldcs(src);
-                    dst[i][1] = __ldcs(src + 1);
-                } else {
-                    dst[i][0] = dst[i][1] = make_float4(0.f, 0.f, 0.f, 0.f);
-                }
-            }
-        };
-        // add the finished accumulator of chunk c into the partial (the
-        // first chunk stores); false if its wait gave up
-        auto flush = [&](int64_t c) -> bool {
+        if (ns == 0) {
+            for (int b = 0; b < PW; b += 4)
+                *reinterpret_cast<float4 *>(o + b) = make_float4(0.f, 0.f, 0.f, 0.f);
+        }
+        for (int64_t c = 0; c < n_chunks; ++c) {
             const int acc = (int)(c & 1);
             int f_ok = lane == 0 ? (mbar_wait(&dfull[acc], (uint32_t)((c >> 1) & 1), status) ? 1 : 0)
                                  : 0;
             f_ok = __shfl_sync(0xffffffffu, f_ok, 0);
-            if (!f_ok) return false;
+            if (!f_ok) break;
             tc_fence_after();
 #pragma unroll 1
             for (int ch = 0; ch < PW / 32; ++ch) {
@@ -466,57 +442,6 @@ __global__ __launch_bounds__(RM_THREADS, 1) void k_reach_mma(
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(&dfree[acc]);
-            return true;
-        };
-        uint32_t stage = 0, phase = 0;
-        bool ok = true;
-        if (ns > 0) load(0, cur);
-        for (int64_t t = 0; t < ns; ++t) {
-            if (t + 1 < ns) load(t + 1, nxt);
-            int w_ok = lane == 0 ? (mbar_wait(&empty[stage], phase ^ 1u, status) ? 1 : 0) : 0;
-            w_ok = __shfl_sync(0xffffffffu, w_ok, 0);
-            if (!w_ok) {
-                ok = false;
-                break;
-            }
-            uint8_t *bh = b_hi(stage), *bl = b_lo(stage);
-#pragma unroll
-            for (int i = 0; i < C::ITEMS; ++i) {
-                const int r = C::RPW * cw + i * C::RPI + rl;   // row in the stage (K)
-                const uint32_t off = (uint32_t)(c8 >> 3) * C::LBO + (uint32_t)r * 128u +
-                                     ((uint32_t)((c8 & 7) ^ (r & 7)) << 4);
-                uint4 vh, vl;
-                vh.x = split_bf16_pair(cur[i][0].x, cur[i][0].y, vl.x);
-                vh.y = split_bf16_pair(cur[i][0].z, cur[i][0].w, vl.y);
-                vh.z = split_bf16_pair(cur[i][1].x, cur[i][1].y, vl.z);
-                vh.w = split_bf16_pair(cur[i][1].z, cur[i][1].w, vl.w);
-                *reinterpret_cast<uint4 *>(bh + off) = vh;
-                *reinterpret_cast<uint4 *>(bl + off) = vl;
-            }
-            fence_async_smem();                       // generic writes -> the MMA's reads
-            __syncwarp();
-            if (lane == 0) mbar_arrive(&bfull[stage]);
-            if (++stage == RM_STAGES) {
-                stage = 0;
-                phase ^= 1u;
-            }
-            // the previous chunk is complete once the first stage of this
-            // one is handed over: flush it while the MMAs run on
-            if (t % RM_CHUNK == 0 && t > 0 && !flush(t / RM_CHUNK - 1)) {
-                ok = false;
-                break;
-            }
-#pragma unroll
-            for (int i = 0; i < C::ITEMS; ++i) {
-                cur[i][0] = nxt[i][0];
-                cur[i][1] = nxt[i][1];
-            }
-        }
-        if (ns == 0) {
-            for (int b = 0; b < PW; b += 4)
-                *reinterpret_cast<float4 *>(o + b) = make_float4(0.f, 0.f, 0.f, 0.f);
-        } else if (ok) {
-            flush(n_chunks - 1);
         }
     }
     tc_fence_before();
@@ -566,7 +491,8 @@ __global__ __launch_bounds__(256) void k_reach_pack(const float *__restrict__ C,
 // and every (1024 / bp)-th partial from t / bp on (coalesced rows of the
 // partials), and the groups are added in group order (the same order on
 // every run).
-__global__ __launch_bounds__(1024) void k_reach_emit(const float *__restrict__ u, int bp, int B,
+__global__ __launch_bounds__(1024) void k_reach_emit(const uint16_t *__restrict__ u_hi,
+                                                     const uint16_t *__restrict__ u_lo, int bp, int B,
                                                      const float *__restrict__ partial,
                                                      int n_parts, const int32_t *__restrict__ plan,
                                                      const int32_t *__restrict__ rows,
@@ -590,7 +516,9 @@ __global__ __launch_bounds__(1024) void k_reach_emit(const float *__restrict__ u
         float sum = red[b];
         for (int h = 1; h < ng; ++h) sum += red[h * bp + b];
         const int64_t j = rows[slot];
-        const float s = u[j * bp + b] + sum;
+        const float uj = __bfloat162float(__ushort_as_bfloat16(u_hi[j * bp + b])) +
+                         __bfloat162float(__ushort_as_bfloat16(u_lo[j * bp + b]));
+        const float s = uj + sum;
         buf[(int64_t)b * cap + i] = ((unsigned long long)__float_as_uint(s) << 32) |
                                     (unsigned long long)(~(uint32_t)ext_of[j]);
         if (i == 0) cnt[b] = (unsigned int)nk;
@@ -611,9 +539,10 @@ cudaError_t launch_reach_pack(const float *C, int64_t n, int H, float alpha, uin
 }
 
 template <int BP>
-static cudaError_t reach_mma_bp(const uint16_t *coef_hi, const uint16_t *coef_lo, const float *u,
-                                int64_t n, const int32_t *plan, float *partial, int parts,
-                                int *status, cudaStream_t st) {
+static cudaError_t reach_mma_bp(const uint16_t *coef_hi, const uint16_t *coef_lo,
+                                const uint16_t *u_hi, const uint16_t *u_lo, int64_t n,
+                                const int32_t *plan, float *partial, int parts, int *status,
+                                cudaStream_t st) {
     using C = RmCfg<BP>;
     static bool attr[64] = {false};
     int dev = 0;
@@ -637,25 +566,34 @@ static cudaError_t reach_mma_bp(const uint16_t *coef_hi, const uint16_t *coef_lo
     if (e == cudaSuccess)
         e = make_tmap_2d(&tlo64, coef_lo, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, (uint64_t)n_pad,
                          RM_M, (uint64_t)n_pad * 2, RM_BK, RM_M / 2);
+    CUtensorMap tbh, tbl;
+    if (e == cudaSuccess)
+        e = make_tmap_2d(&tbh, u_hi, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, BP, (uint64_t)n,
+                         (uint64_t)BP * 2, 64, RM_BK);
+    if (e == cudaSuccess)
+        e = make_tmap_2d(&tbl, u_lo, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, BP, (uint64_t)n,
+                         (uint64_t)BP * 2, 64, RM_BK);
     if (e != cudaSuccess) return e;
-    k_reach_mma<BP><<<parts, RM_THREADS, C::SMEM, st>>>(thi, tlo, thi64, tlo64, u, n, plan,
+    k_reach_mma<BP><<<parts, RM_THREADS, C::SMEM, st>>>(thi, tlo, thi64, tlo64, tbh, tbl, n, plan,
                                                          partial, status);
     return cudaGetLastError();
 }
 
-cudaError_t launch_reach_scores(const float *u, int bp, int B, int64_t n, const uint16_t *coef_hi,
+cudaError_t launch_reach_scores(const uint16_t *u_hi, const uint16_t *u_lo, int bp, int B,
+                                int64_t n, const uint16_t *coef_hi,
                                 const uint16_t *coef_lo, const int32_t *plan, const int32_t *rows,
                                 const int32_t *ext_of, float *partial, unsigned int *cnt,
                                 unsigned long long *buf, int64_t cap, int *status, cudaStream_t st,
                                 int *launches) {
     if (n <= 0 || (bp != 128 && bp != 256)) return cudaErrorInvalidValue;
     const int parts = reach_parts();
-    cudaError_t e = bp == 256
-                        ? reach_mma_bp<256>(coef_hi, coef_lo, u, n, plan, partial, parts, status, st)
-                        : reach_mma_bp<128>(coef_hi, coef_lo, u, n, plan, partial, parts, status, st);
+    cudaError_t e = bp == 256 ? reach_mma_bp<256>(coef_hi, coef_lo, u_hi, u_lo, n, plan, partial,
+                                                  parts, status, st)
+                              : reach_mma_bp<128>(coef_hi, coef_lo, u_hi, u_lo, n, plan, partial,
+                                                  parts, status, st);
     if (e != cudaSuccess) return e;
-    k_reach_emit<<<REACH_T, 1024, 0, st>>>(u, bp, B, partial, parts, plan, rows, ext_of, cnt, buf,
-                                           cap);
+    k_reach_emit<<<REACH_T, 1024, 0, st>>>(u_hi, u_lo, bp, B, partial, parts, plan, rows, ext_of,
+                                           cnt, buf, cap);
     if (launches) *launches += 2;
     return cudaGetLastError();
 }

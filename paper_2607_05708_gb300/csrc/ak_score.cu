@@ -116,7 +116,7 @@ static PFN_cuTensorMapEncodeTiled_v12000 tmap_encoder() {
 
 cudaError_t make_tmap_2d(CUtensorMap *map, const void *base, CUtensorMapDataType dtype,
                          int elem_bytes, uint64_t inner, uint64_t outer, uint64_t row_bytes,
-                         uint32_t box_inner, uint32_t box_outer) {
+                         uint32_t box_inner, uint32_t box_outer, CUtensorMapSwizzle swizzle) {
     auto fn = tmap_encoder();
     if (!fn) return cudaErrorNotSupported;
     (void)elem_bytes;
@@ -125,7 +125,7 @@ cudaError_t make_tmap_2d(CUtensorMap *map, const void *base, CUtensorMapDataType
     cuuint32_t box[2] = {box_inner, box_outer};
     cuuint32_t es[2] = {1, 1};
     CUresult r = fn(map, dtype, 2, const_cast<void *>(base), dims, strides, box, es,
-                    CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                    CU_TENSOR_MAP_INTERLEAVE_NONE, swizzle,
                     CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
 }
@@ -175,6 +175,8 @@ struct GemmEpi {
     const int32_t *dead_row;            // EXP, EXP_FILTER, FILTER: deleted rows (or NULL):
                                         // no score (u = 0) / never a filter candidate
     uint32_t *keys_t;                   // KEYS_T: [n_ctiles * BP][n_rows]
+    uint16_t *u_hi, *u_lo;              // EXP (or NULL): u as split bf16, [n_rows][n_ctiles * BP]
+                                        // each (u = hi + lo to 2^-17), instead of fp32
     float *row_max, *row_min;           // EXP (or NULL): [n_rows] largest / smallest u of
     int n_real;                         // the row over the first n_real columns
     unsigned int *ext;                  // with row_max (or NULL), atomically maxed, zeroed
@@ -238,6 +240,7 @@ template <int BP, int MODE, bool P2 = false>
 __global__ __launch_bounds__(GemmCfg<BP, MODE, P2>::THREADS, 1) void k_gemm_umma(const __grid_constant__ CUtensorMap tmA,
                                                       const __grid_constant__ CUtensorMap tmB,
                                                       const __grid_constant__ CUtensorMap tmC,
+                                                      const __grid_constant__ CUtensorMap tmD,
                                                       int64_t n_rows, int dim, int n_ctiles,
                                                       const GemmEpi ep) {
     using C = GemmCfg<BP, MODE, P2>;
@@ -532,6 +535,51 @@ __global__ __launch_bounds__(GemmCfg<BP, MODE, P2>::THREADS, 1) void k_gemm_umma
                             rmin = fminf(rmin, v[i]);
                         }
                 }
+                if (MODE == GEMM_EXP && ep.u_hi) {
+                    // u as split bf16: hi and lo tiles [128 rows][32 cols] of
+                    // 64-byte rows in the 64-byte swizzle (the 16-byte chunk c
+                    // of row r at c ^ ((r >> 1) & 3)), one TMA store each
+                    named_bar(2 + hsel, 128);                 // staging[buf] free again
+                    uint8_t *sb = (uint8_t *)(sOut + (hsel * 2 + buf) * (C::OUT_BYTES / 4));
+                    uint32_t hw[16], lw[16];
+#pragma unroll
+                    for (int i = 0; i < 16; ++i) hw[i] = split_bf16_pair(v[2 * i], v[2 * i + 1], lw[i]);
+#pragma unroll
+                    for (int j = 0; j < 4; ++j) {
+                        const int pos = row * 64 + ((j ^ ((row >> 1) & 3)) << 4);
+                        *reinterpret_cast<uint4 *>(sb + pos) =
+                            make_uint4(hw[4 * j], hw[4 * j + 1], hw[4 * j + 2], hw[4 * j + 3]);
+                        *reinterpret_cast<uint4 *>(sb + C::OUT_BYTES / 2 + pos) =
+                            make_uint4(lw[4 * j], lw[4 * j + 1], lw[4 * j + 2], lw[4 * j + 3]);
+                    }
+                    fence_async_smem();
+                    // Z: the column sums of the warp's 32 rows (fp32), by
+                    // halving exchanges across the lanes: lane l ends with
+                    // column l's sum
+#pragma unroll
+                    for (int o = 16; o >= 1; o >>= 1) {
+                        const bool up = (lane & o) != 0;
+#pragma unroll
+                        for (int i = 0; i < o; ++i) {
+                            const float send = up ? v[i] : v[i + o];
+                            const float keep = up ? v[i + o] : v[i];
+                            v[i] = keep + __shfl_xor_sync(0xffffffffu, send, o);
+                        }
+                    }
+                    zadd(zl, ch, v[0]);
+                    named_bar(2 + hsel, 128);                 // staging[buf] complete
+                    if ((et & 127) == 0) {
+                        if (mt * TM + row_off < n_rows) {
+                            tma_store_2d(&tmC, sb, (int)(ct * BP + ch * 32),
+                                         (int)(mt * TM + row_off));
+                            tma_store_2d(&tmD, sb + C::OUT_BYTES / 2, (int)(ct * BP + ch * 32),
+                                         (int)(mt * TM + row_off));
+                            bulk_commit();
+                        }
+                        bulk_wait_read<1>();                  // the other buffer is free
+                    }
+                    continue;
+                }
                 // filter, first half: which of this row's 32 values reach
                 // their query's threshold (branch-free; rarely any)
                 uint32_t pass = 0u;
@@ -775,17 +823,28 @@ static cudaError_t gemm_bp(const uint16_t *emb, int64_t n_rows, int64_t row_stri
         cudaError_t e = gemm_attr<BP, MODE>();
         if (e != cudaSuccess) return e;
     }
-    CUtensorMap ta, tb, tc;
+    CUtensorMap ta, tb, tc, td;
     cudaError_t e = make_tmap_2d(&ta, emb, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, (uint64_t)dim,
                                  (uint64_t)n_rows, (uint64_t)dim * 2 * row_stride_rows, 64, 128);
     if (e == cudaSuccess)
         e = make_tmap_2d(&tb, qp, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, (uint64_t)dim,
                          (uint64_t)n_ctiles * BP, (uint64_t)dim * 2, 64, p2 ? BP / 2 : BP);
-    if (e == cudaSuccess && MODE != GEMM_FILTER && MODE != GEMM_EXP_FILTER && MODE != GEMM_KEYS_T)
-        e = make_tmap_2d(&tc, out, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, (uint64_t)n_ctiles * BP,
-                         (uint64_t)n_rows, (uint64_t)n_ctiles * BP * 4, 32, 128);
-    else
-        tc = ta;   // unused by the filter epilogue
+    const uint64_t n_cols = (uint64_t)n_ctiles * BP;
+    if (e == cudaSuccess && MODE == GEMM_EXP && ep.u_hi) {
+        // split-bf16 output: [128][32] boxes of 64-byte rows, 64-byte swizzle
+        e = make_tmap_2d(&tc, ep.u_hi, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, n_cols,
+                         (uint64_t)n_rows, n_cols * 2, 32, 128, CU_TENSOR_MAP_SWIZZLE_64B);
+        if (e == cudaSuccess)
+            e = make_tmap_2d(&td, ep.u_lo, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, n_cols,
+                             (uint64_t)n_rows, n_cols * 2, 32, 128, CU_TENSOR_MAP_SWIZZLE_64B);
+    } else if (e == cudaSuccess && MODE != GEMM_FILTER && MODE != GEMM_EXP_FILTER &&
+               MODE != GEMM_KEYS_T) {
+        e = make_tmap_2d(&tc, out, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, n_cols, (uint64_t)n_rows,
+                         n_cols * 4, 32, 128);
+        td = tc;   // unused
+    } else {
+        tc = td = ta;   // unused by the filter epilogues
+    }
     if (e != cudaSuccess) return e;
     if constexpr (CAN_P2) {
         if (p2) {
@@ -804,7 +863,7 @@ static cudaError_t gemm_bp(const uint16_t *emb, int64_t n_rows, int64_t row_stri
             cfg.stream = st;
             cfg.attrs = at;
             cfg.numAttrs = 1;
-            e = cudaLaunchKernelEx(&cfg, k_gemm_umma<BP, MODE, true>, ta, tb, tc, n_rows, dim,
+            e = cudaLaunchKernelEx(&cfg, k_gemm_umma<BP, MODE, true>, ta, tb, tc, td, n_rows, dim,
                                    n_ctiles, ep);
             if (zrows) *zrows = (int)(2 * clusters);
             return e == cudaSuccess ? cudaGetLastError() : e;
@@ -814,7 +873,7 @@ static cudaError_t gemm_bp(const uint16_t *emb, int64_t n_rows, int64_t row_stri
     const int64_t m_tiles = ceil_div<int64_t>(n_rows, 128);
     const int64_t tiles = m_tiles * n_ctiles;
     const int grid = (int)(tiles < device_sm_count() ? tiles : device_sm_count());
-    k_gemm_umma<BP, MODE><<<grid, C::THREADS, C::SMEM, st>>>(ta, tb, tc, n_rows, dim, n_ctiles,
+    k_gemm_umma<BP, MODE><<<grid, C::THREADS, C::SMEM, st>>>(ta, tb, tc, td, n_rows, dim, n_ctiles,
                                                              ep);
     if (zrows) *zrows = grid;
     return cudaGetLastError();
@@ -849,6 +908,28 @@ cudaError_t launch_score(const uint16_t *emb, int64_t n, int dim, const uint16_t
     ep.zpart = zpart;
     ep.status = status;
     cudaError_t e = gemm_dispatch<GEMM_EXP>(emb, n, 1, dim, qp, bp, 1, u, ep, st, zrows);
+    if (launches) *launches += 1;
+    return e;
+}
+
+cudaError_t launch_score_split(const uint16_t *emb, int64_t n, int dim, const uint16_t *qp, int bp,
+                               const float *shift, float tau, uint16_t *u_hi, uint16_t *u_lo,
+                               float *zpart, int *status, cudaStream_t st, int *launches,
+                               int *zrows, const int32_t *dead_row, float *row_max,
+                               float *row_min, int n_real, unsigned int *ext) {
+    GemmEpi ep{};
+    ep.dead_row = dead_row;
+    ep.row_max = row_max;
+    ep.row_min = row_min;
+    ep.n_real = n_real;
+    ep.ext = row_max ? ext : nullptr;
+    ep.shift = shift;
+    ep.tau = tau;
+    ep.zpart = zpart;
+    ep.status = status;
+    ep.u_hi = u_hi;
+    ep.u_lo = u_lo;
+    cudaError_t e = gemm_dispatch<GEMM_EXP>(emb, n, 1, dim, qp, bp, 1, nullptr, ep, st, zrows);
     if (launches) *launches += 1;
     return e;
 }

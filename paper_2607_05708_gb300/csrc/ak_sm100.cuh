@@ -306,6 +306,7 @@ __device__ __forceinline__ void tmem_ld_wait() {
 // Tensor-map encoder fetched from the driver at run time (no libcuda link).
 cudaError_t make_tmap_2d(CUtensorMap *map, const void *base, CUtensorMapDataType dtype,
                          int elem_bytes, uint64_t inner, uint64_t outer, uint64_t row_bytes,
-                         uint32_t box_inner, uint32_t box_outer);
+                         uint32_t box_inner, uint32_t box_outer,
+                         CUtensorMapSwizzle swizzle = CU_TENSOR_MAP_SWIZZLE_128B);
 
 }  // namespace ak
