@@ -242,8 +242,11 @@ cudaError_t launch_reach_flags(const ReachFlags &f, cudaStream_t st, int *launch
 // into the fp32 accumulator may round the same way), so an accumulator
 // takes only RM_CHUNK stages (1024 rows, 192 MMAs): two accumulators
 // alternate, and the flush warps add each finished one into the CTA's
-// partial with ordinary round-to-nearest fp32 adds (the partial rows stay
-// in L2) while the MMAs fill the other.
+// partial with ordinary round-to-nearest fp32 adds while the MMAs fill the
+// other.  The operands' loads carry an L2 evict-first hint and the partial
+// rows' loads and stores an evict-last one, so that the partials stay in L2
+// while u streams past; slots 64 and above are flushed only when the plan
+// is wide.
 // Warps: 0 TMA producer (A and B), 1 MMA issuer, 2..9 flush (warp w reads
 // TMEM lanes 32 (w % 4) .., column half (w - 2) / 4).  Both operands
 // arrive by TMA, so the bytes in flight are the two stages' 192 KB of
@@ -330,6 +333,9 @@ __global__ __launch_bounds__(RM_THREADS, 1) void k_reach_mma(
             int last_par[RM_STAGES];
             for (int s = 0; s < RM_STAGES; ++s) last_par[s] = -1;
             bool ok = true;
+            // both operands are read once a call: evict them first, so that
+            // they do not push the CTAs' partial rows out of L2
+            const uint64_t pol = l2_evict_first_policy();
             for (int64_t t = 0; t < ns; ++t) {
                 if (!mbar_wait_spin(&empty[stage], phase ^ 1u, status)) {
                     ok = false;
@@ -338,12 +344,14 @@ __global__ __launch_bounds__(RM_THREADS, 1) void k_reach_mma(
                 mbar_expect_tx(&full[stage],
                                (wide ? 2 * C::A_BYTES : C::A_BYTES) + 2 * C::B_BYTES);
                 const int kx = (int)((s0 + t) * RM_BK);
-                tma_load_2d(a_hi(stage), wide ? &tmAhi : &tmAhi64, &full[stage], kx, 0);
-                tma_load_2d(a_lo(stage), wide ? &tmAlo : &tmAlo64, &full[stage], kx, 0);
+                tma_load_2d_hint(a_hi(stage), wide ? &tmAhi : &tmAhi64, &full[stage], kx, 0, pol);
+                tma_load_2d_hint(a_lo(stage), wide ? &tmAlo : &tmAlo64, &full[stage], kx, 0, pol);
 #pragma unroll
                 for (int c = 0; c < BP / 64; ++c) {
-                    tma_load_2d(b_hi(stage) + c * C::LBO, &tmBhi, &full[stage], 64 * c, kx);
-                    tma_load_2d(b_lo(stage) + c * C::LBO, &tmBlo, &full[stage], 64 * c, kx);
+                    tma_load_2d_hint(b_hi(stage) + c * C::LBO, &tmBhi, &full[stage], 64 * c, kx,
+                                     pol);
+                    tma_load_2d_hint(b_lo(stage) + c * C::LBO, &tmBlo, &full[stage], 64 * c, kx,
+                                     pol);
                 }
                 last_par[stage] = (int)phase;
                 if (++stage == RM_STAGES) {
@@ -405,7 +413,11 @@ __global__ __launch_bounds__(RM_THREADS, 1) void k_reach_mma(
         const int slot = q * 32 + lane;
         constexpr int PW = BP / C::PARTS;             // columns of a part
         float *o = partial + ((int64_t)blockIdx.x * REACH_T + slot) * BP + part * PW;
-        if (ns == 0) {
+        // slots 64..127 are read only when the plan is wide
+        const bool live = wide || q < 2;
+        // the partial rows are re-read every chunk: keep them in L2
+        const uint64_t pol = l2_evict_last_policy();
+        if (ns == 0 && live) {
             for (int b = 0; b < PW; b += 4)
                 *reinterpret_cast<float4 *>(o + b) = make_float4(0.f, 0.f, 0.f, 0.f);
         }
@@ -417,7 +429,7 @@ __global__ __launch_bounds__(RM_THREADS, 1) void k_reach_mma(
             if (!f_ok) break;
             tc_fence_after();
 #pragma unroll 1
-            for (int ch = 0; ch < PW / 32; ++ch) {
+            for (int ch = 0; ch < (live ? PW / 32 : 0); ++ch) {
                 uint32_t r[32];
                 tmem_ld32(tmem_base + ((uint32_t)(q * 32) << 16) +
                               (uint32_t)(acc * BP + part * PW + ch * 32),
@@ -430,13 +442,13 @@ __global__ __launch_bounds__(RM_THREADS, 1) void k_reach_mma(
                                            __uint_as_float(r[4 * i + 2]),
                                            __uint_as_float(r[4 * i + 3]));
                     if (c > 0) {
-                        const float4 p = dst[i];
+                        const float4 p = ld_f4_hint(dst + i, pol);
                         v.x += p.x;
                         v.y += p.y;
                         v.z += p.z;
                         v.w += p.w;
                     }
-                    dst[i] = v;
+                    st_f4_hint(dst + i, v, pol);
                 }
             }
             tc_fence_before();
