@@ -154,6 +154,7 @@ __device__ void reach_build_plan(const int32_t *keep, int bad, int t_cnt, int k,
 // ping-pong pair of shared arrays).  Also clears the flags' scratch.
 __global__ __launch_bounds__(1024) void k_reach_floor(const ReachFlags f) {
     __shared__ unsigned long long xk[2][1024];
+    griddep_wait();
     const int t = threadIdx.x;
     if (t < REACH_T + 2) f.ws[t] = 0;                  // keep[], bad, done
     const float lmin = ext_lmin(f.ext);
@@ -185,6 +186,7 @@ __global__ __launch_bounds__(1024) void k_reach_floor(const ReachFlags f) {
 // any other row counted in bad; the last CTA to finish builds the plan.
 __global__ __launch_bounds__(256) void k_reach_flags(const ReachFlags f) {
     __shared__ int last;
+    griddep_wait();
     int32_t *keep = f.ws, *bad = f.ws + REACH_T, *done = f.ws + REACH_T + 1;
     const float floor_ = *f.floor_out, umax = ext_umax(f.ext);
     int nb = 0;
@@ -212,13 +214,14 @@ __global__ __launch_bounds__(256) void k_reach_flags(const ReachFlags f) {
 
 cudaError_t launch_reach_flags(const ReachFlags &f, cudaStream_t st, int *launches) {
     if (f.n_lb > 1024 || f.k < 1) return cudaErrorInvalidValue;
-    k_reach_floor<<<1, 1024, 0, st>>>(f);
+    cudaError_t e = launch_pdl(k_reach_floor, dim3(1), dim3(1024), 0, st, f);
+    if (e != cudaSuccess) return e;
     // one row per thread: a few independent loads per row, so the rows in
     // flight set the rate
     const int64_t g = ceil_div<int64_t>(f.n, 256);
-    k_reach_flags<<<(unsigned)(g > 0 ? g : 1), 256, 0, st>>>(f);
+    e = launch_pdl(k_reach_flags, dim3((unsigned)(g > 0 ? g : 1)), dim3(256), 0, st, f);
     if (launches) *launches += 2;
-    return cudaGetLastError();
+    return e == cudaSuccess ? cudaGetLastError() : e;
 }
 
 // ------------------------------------------------------------------ tensor-core terms
@@ -280,6 +283,7 @@ __global__ __launch_bounds__(RM_THREADS, 1) void k_reach_mma(
     const __grid_constant__ CUtensorMap tmBhi, const __grid_constant__ CUtensorMap tmBlo,
     int64_t n, const int32_t *__restrict__ plan, float *__restrict__ partial, int *status) {
     using C = RmCfg<BP>;
+    griddep_wait();
     if (plan[0] == 0) return;                          // the hops run instead
     // every flagged slot below 64: only the first 64 coefficient rows are
     // loaded (rows 64..127 of the A tiles keep whatever they hold, and
@@ -513,6 +517,7 @@ __global__ __launch_bounds__(1024) void k_reach_emit(const uint16_t *__restrict_
                                                      unsigned long long *__restrict__ buf,
                                                      int64_t cap) {
     __shared__ float red[1024];
+    griddep_wait();
     if (plan[0] == 0) return;
     const int nk = plan[1];
     const int i = blockIdx.x;
@@ -604,10 +609,10 @@ cudaError_t launch_reach_scores(const uint16_t *u_hi, const uint16_t *u_lo, int 
                               : reach_mma_bp<128>(coef_hi, coef_lo, u_hi, u_lo, n, plan, partial,
                                                   parts, status, st);
     if (e != cudaSuccess) return e;
-    k_reach_emit<<<REACH_T, 1024, 0, st>>>(u_hi, u_lo, bp, B, partial, parts, plan, rows, ext_of,
-                                           cnt, buf, cap);
+    e = launch_pdl(k_reach_emit, dim3(REACH_T), dim3(1024), 0, st, u_hi, u_lo, bp, B,
+                   (const float *)partial, parts, plan, rows, ext_of, cnt, buf, cap);
     if (launches) *launches += 2;
-    return cudaGetLastError();
+    return e == cudaSuccess ? cudaGetLastError() : e;
 }
 
 }  // namespace ak

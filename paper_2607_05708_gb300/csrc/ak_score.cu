@@ -18,6 +18,7 @@ __global__ void k_prep_queries(const uint16_t *__restrict__ q, int b, int dim, f
                                const float *__restrict__ max_norm, uint16_t *__restrict__ qp,
                                float *__restrict__ shift, int *status,
                                unsigned int *__restrict__ ext_zero) {
+    griddep_wait();
     const int c = blockIdx.x;
     if (ext_zero && c == 0 && threadIdx.x < 2) ext_zero[threadIdx.x] = 0u;
     __shared__ float red[32];
@@ -59,13 +60,11 @@ __global__ void k_prep_queries(const uint16_t *__restrict__ q, int b, int dim, f
 cudaError_t launch_prep_queries(const uint16_t *q, int b, int bp, int dim, float tau,
                                 const float *max_norm, uint16_t *qp, float *shift, int *status,
                                 cudaStream_t st, unsigned int *ext_zero) {
-    if (((uintptr_t)q & 15) == 0 && dim % 8 == 0)
-        k_prep_queries<true><<<bp, 128, 0, st>>>(q, b, dim, tau, max_norm, qp, shift, status,
-                                                 ext_zero);
-    else
-        k_prep_queries<false><<<bp, 128, 0, st>>>(q, b, dim, tau, max_norm, qp, shift, status,
-                                                  ext_zero);
-    return cudaGetLastError();
+    const bool vec = ((uintptr_t)q & 15) == 0 && dim % 8 == 0;
+    cudaError_t e = launch_pdl(vec ? k_prep_queries<true> : k_prep_queries<false>, dim3(bp),
+                               dim3(128), 0, st, q, b, dim, tau, max_norm, qp, shift, status,
+                               ext_zero);
+    return e == cudaSuccess ? cudaGetLastError() : e;
 }
 
 // ------------------------------------------------------------------ norm max
@@ -244,6 +243,7 @@ __global__ __launch_bounds__(GemmCfg<BP, MODE, P2>::THREADS, 1) void k_gemm_umma
                                                       int64_t n_rows, int dim, int n_ctiles,
                                                       const GemmEpi ep) {
     using C = GemmCfg<BP, MODE, P2>;
+    griddep_wait();
     constexpr bool EXPF = MODE == GEMM_EXP_FILTER;
     constexpr bool EXP = MODE == GEMM_EXP || EXPF;
     constexpr bool FILTER = MODE == GEMM_FILTER;
@@ -852,17 +852,19 @@ static cudaError_t gemm_bp(const uint16_t *emb, int64_t n_rows, int64_t row_stri
             const int64_t units = ceil_div<int64_t>(n_rows, 256) * n_ctiles;
             const int64_t clusters = units < ncl ? units : ncl;
             cudaLaunchConfig_t cfg = {};
-            cudaLaunchAttribute at[1];
+            cudaLaunchAttribute at[2];
             at[0].id = cudaLaunchAttributeClusterDimension;
             at[0].val.clusterDim.x = 2;
             at[0].val.clusterDim.y = 1;
             at[0].val.clusterDim.z = 1;
+            at[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;   // see griddep_wait
+            at[1].val.programmaticStreamSerializationAllowed = 1;
             cfg.gridDim = dim3((unsigned)(2 * clusters));
             cfg.blockDim = dim3(C2::THREADS);
             cfg.dynamicSmemBytes = C2::SMEM;
             cfg.stream = st;
             cfg.attrs = at;
-            cfg.numAttrs = 1;
+            cfg.numAttrs = 2;
             e = cudaLaunchKernelEx(&cfg, k_gemm_umma<BP, MODE, true>, ta, tb, tc, td, n_rows, dim,
                                    n_ctiles, ep);
             if (zrows) *zrows = (int)(2 * clusters);
@@ -873,10 +875,10 @@ static cudaError_t gemm_bp(const uint16_t *emb, int64_t n_rows, int64_t row_stri
     const int64_t m_tiles = ceil_div<int64_t>(n_rows, 128);
     const int64_t tiles = m_tiles * n_ctiles;
     const int grid = (int)(tiles < device_sm_count() ? tiles : device_sm_count());
-    k_gemm_umma<BP, MODE><<<grid, C::THREADS, C::SMEM, st>>>(ta, tb, tc, td, n_rows, dim, n_ctiles,
-                                                             ep);
+    e = launch_pdl(k_gemm_umma<BP, MODE, false>, dim3(grid), dim3(C::THREADS), C::SMEM, st, ta, tb,
+                   tc, td, n_rows, dim, n_ctiles, ep);
     if (zrows) *zrows = grid;
-    return cudaGetLastError();
+    return e == cudaSuccess ? cudaGetLastError() : e;
 }
 
 template <int MODE>

@@ -542,6 +542,7 @@ __global__ __launch_bounds__(SEL_THREADS) void k_topk_merge(
     __shared__ int s_remaining, win_n;
     __shared__ double zred[SEL_THREADS / 32];
     __shared__ int pg[64];
+    griddep_wait();
     const int c = blockIdx.x;
     const int tid = threadIdx.x;
     if (rc.kind != 0 && (int64_t)cnt[c] > cap) {
@@ -986,13 +987,13 @@ cudaError_t launch_topk_merge(const SelectPlan &sp, const float *s, int b,
                               cudaStream_t st, int *launches) {
     ColumnRecompute r{};
     if (rc) r = *rc;
-    k_topk_merge<<<b, SEL_THREADS, 0, st>>>(s, sp.n, sp.bp, sp.k, ext_of,
-                                            (const unsigned int *)(ws + sp.off_cnt),
-                                            ws + sp.off_buf, sp.cap, zpart, n_ztiles, row_of,
-                                            page_row, ids, scores, page_ids, n_pages, status, r,
-                                            ns, sort_by_time);
+    cudaError_t e = launch_pdl(k_topk_merge, dim3(b), dim3(SEL_THREADS), 0, st, s, sp.n, sp.bp,
+                               sp.k, ext_of, (const unsigned int *)(ws + sp.off_cnt),
+                               (const unsigned long long *)(ws + sp.off_buf), sp.cap, zpart,
+                               n_ztiles, row_of, page_row, ids, scores, page_ids, n_pages, status,
+                               r, ns, sort_by_time);
     if (launches) *launches += 1;
-    return cudaGetLastError();
+    return e == cudaSuccess ? cudaGetLastError() : e;
 }
 
 cudaError_t launch_select_signed(const SelectPlan &sp, const float *s, int b,
