@@ -190,13 +190,38 @@ __global__ __launch_bounds__(256) void k_reach_flags(const ReachFlags f) {
     int32_t *keep = f.ws, *bad = f.ws + REACH_T, *done = f.ws + REACH_T + 1;
     const float floor_ = *f.floor_out, umax = ext_umax(f.ext);
     int nb = 0;
-    for (int64_t j = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; j < f.n;
-         j += (int64_t)gridDim.x * blockDim.x) {
-        if (row_upper_bound(f.u0, f.mup, f.n, f.H, f.alpha, umax, j) >= floor_) {
+    auto visit = [&](int64_t j, float ub) {
+        if (ub >= floor_) {
             const int32_t t = f.map[j];
             if (t >= 0) keep[t] = 1;
             else ++nb;
         }
+    };
+    const int64_t tid = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    if ((f.n & 3) == 0) {
+        // four rows a thread: 16-byte loads of u's row maxima and of each
+        // mass level, the bound evaluated per row as row_upper_bound does
+        const int64_t n4 = f.n >> 2;
+        for (int64_t q = tid; q < n4; q += stride) {
+            float4 c = make_float4(0.f, 0.f, 0.f, 0.f);
+            for (int t = f.H; t >= 1; --t) {
+                const float4 m =
+                    __ldg(reinterpret_cast<const float4 *>(f.mup + (int64_t)t * f.n) + q);
+                c.x = f.alpha * (c.x + m.x);
+                c.y = f.alpha * (c.y + m.y);
+                c.z = f.alpha * (c.z + m.z);
+                c.w = f.alpha * (c.w + m.w);
+            }
+            const float4 u = reinterpret_cast<const float4 *>(f.u0)[q];
+            visit(4 * q, fmaf(umax, c.x, u.x) * (1.f + 1e-5f));
+            visit(4 * q + 1, fmaf(umax, c.y, u.y) * (1.f + 1e-5f));
+            visit(4 * q + 2, fmaf(umax, c.z, u.z) * (1.f + 1e-5f));
+            visit(4 * q + 3, fmaf(umax, c.w, u.w) * (1.f + 1e-5f));
+        }
+    } else {
+        for (int64_t j = tid; j < f.n; j += stride)
+            visit(j, row_upper_bound(f.u0, f.mup, f.n, f.H, f.alpha, umax, j));
     }
     if (nb) atomicAdd(bad, nb);
     __threadfence();                                   // flags before the count
@@ -216,9 +241,11 @@ cudaError_t launch_reach_flags(const ReachFlags &f, cudaStream_t st, int *launch
     if (f.n_lb > 1024 || f.k < 1) return cudaErrorInvalidValue;
     cudaError_t e = launch_pdl(k_reach_floor, dim3(1), dim3(1024), 0, st, f);
     if (e != cudaSuccess) return e;
-    // one row per thread: a few independent loads per row, so the rows in
-    // flight set the rate
-    const int64_t g = ceil_div<int64_t>(f.n, 256);
+    // four rows per thread (one where n is not a multiple of 4): a few
+    // independent loads per row, so the rows in flight set the rate; a
+    // quarter of the CTAs also takes three quarters of the done counter's
+    // atomics off the tail
+    const int64_t g = ceil_div<int64_t>(f.n, (f.n & 3) == 0 ? 1024 : 256);
     e = launch_pdl(k_reach_flags, dim3((unsigned)(g > 0 ? g : 1)), dim3(256), 0, st, f);
     if (launches) *launches += 2;
     return e == cudaSuccess ? cudaGetLastError() : e;
