@@ -216,28 +216,29 @@ __global__ __launch_bounds__(RS_THREADS) void k_rs_hist(const uint32_t *__restri
     hist[(int64_t)threadIdx.x * n_tiles + blockIdx.x] = h[threadIdx.x];
 }
 
-// Rank the warp's RS_PER_WARP keys of the tile stably by digit: loc[r] is
+// Rank the warp's 32 * ITEMS keys of the tile stably by digit: loc[r] is
 // the key's rank among the warp's keys of its digit, cnt[warp][d] the
 // warp's count of digit d; then pre[w][d] = the counts of digit d in the
 // warps before w (one thread a digit).  Keys at or past n get no digit.
+template <int ITEMS>
 __device__ __forceinline__ void rs_rank(const uint32_t *__restrict__ keys,
                                         const uint32_t *__restrict__ vals, int64_t n,
                                         int64_t base, int shift, uint32_t mask,
-                                        uint32_t (&k)[RS_ITEMS], uint32_t (&v)[RS_ITEMS],
-                                        int (&loc)[RS_ITEMS], int (*cnt)[256], int (*pre)[256]) {
+                                        uint32_t (&k)[ITEMS], uint32_t (&v)[ITEMS],
+                                        int (&loc)[ITEMS], int (*cnt)[256], int (*pre)[256]) {
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     for (int d = lane; d < 256; d += 32) cnt[warp][d] = 0;
     __syncwarp();
     const unsigned lt = (1u << lane) - 1u;
     // every load first, then the ranking (whose rounds depend on each other)
 #pragma unroll
-    for (int r = 0; r < RS_ITEMS; ++r) {
+    for (int r = 0; r < ITEMS; ++r) {
         const int64_t idx = base + r * 32 + lane;
         k[r] = idx < n ? keys[idx] : 0u;
         v[r] = idx < n ? vals[idx] : 0u;
     }
 #pragma unroll
-    for (int r = 0; r < RS_ITEMS; ++r) {
+    for (int r = 0; r < ITEMS; ++r) {
         int64_t idx = base + r * 32 + lane;
         bool ok = idx < n;
         uint32_t d = ok ? ((k[r] >> shift) & mask) : 0x100u;   // 0x100: no digit
@@ -272,7 +273,7 @@ __global__ __launch_bounds__(RS_THREADS) void k_rs_scatter(
     const int64_t base = (int64_t)blockIdx.x * RS_TILE + (int64_t)warp * RS_PER_WARP;
     uint32_t k[RS_ITEMS], v[RS_ITEMS];
     int loc[RS_ITEMS];
-    rs_rank(keys, vals, n, base, shift, mask, k, v, loc, cnt, pre);
+    rs_rank<RS_ITEMS>(keys, vals, n, base, shift, mask, k, v, loc, cnt, pre);
 #pragma unroll
     for (int r = 0; r < RS_ITEMS; ++r) {
         int64_t idx = base + r * 32 + lane;
@@ -285,15 +286,18 @@ __global__ __launch_bounds__(RS_THREADS) void k_rs_scatter(
     }
 }
 
-// Small sorts (at most RS_SMALL_TILES tiles) take one launch a pass after a
-// first histogram launch.  Histograms are int32, digit-major [256][n_tiles].
+// Small sorts (at most RS_SMALL_TILES tiles of RS_SMALL_TILE keys: four a
+// thread, so that a sort of ~100k pairs still spreads over ~100 CTAs) take
+// one launch a pass after a first histogram launch.  Histograms are int32,
+// digit-major [256][n_tiles].
 // Each scatter CTA derives its own offsets from the pass's histograms (the
 // totals of the smaller digits plus its digit's counts in the tiles before
 // it) and counts the next pass's digit of every key it places into the next
 // histograms, by destination tile.  Three histogram buffers rotate: pass p
 // reads H[p % 3], counts into H[(p+1) % 3] (zero by then) and zeroes its
 // column of H[(p+2) % 3], which pass p-1 read and pass p+1 counts into.
-constexpr int64_t RS_SMALL_TILES = 64;
+constexpr int RS_SMALL_ITEMS = 4, RS_SMALL_TILE = RS_THREADS * RS_SMALL_ITEMS;
+constexpr int64_t RS_SMALL_TILES = 256;
 
 __global__ __launch_bounds__(RS_THREADS) void k_rs_hist32(const uint32_t *__restrict__ keys,
                                                           int64_t n, int shift, uint32_t mask,
@@ -303,8 +307,8 @@ __global__ __launch_bounds__(RS_THREADS) void k_rs_hist32(const uint32_t *__rest
     __shared__ int h[256];
     h[threadIdx.x] = 0;
     __syncthreads();
-    const int64_t base = (int64_t)blockIdx.x * RS_TILE;
-    for (int i = threadIdx.x; i < RS_TILE; i += RS_THREADS) {
+    const int64_t base = (int64_t)blockIdx.x * RS_SMALL_TILE;
+    for (int i = threadIdx.x; i < RS_SMALL_TILE; i += RS_THREADS) {
         int64_t idx = base + i;
         if (idx < n) atomicAdd(&h[(keys[idx] >> shift) & mask], 1);
     }
@@ -349,12 +353,13 @@ __global__ __launch_bounds__(RS_THREADS) void k_rs_scatter_small(
         off_s[d] = wpre + incl - tot + before;
         if (hzero) hzero[(int64_t)d * n_tiles + blockIdx.x] = 0;
     }
-    const int64_t base = (int64_t)blockIdx.x * RS_TILE + (int64_t)warp * RS_PER_WARP;
-    uint32_t k[RS_ITEMS], v[RS_ITEMS];
-    int loc[RS_ITEMS];
-    rs_rank(keys, vals, n, base, shift, mask, k, v, loc, cnt, pre);   // syncs the CTA
+    const int64_t base =
+        (int64_t)blockIdx.x * RS_SMALL_TILE + (int64_t)warp * (32 * RS_SMALL_ITEMS);
+    uint32_t k[RS_SMALL_ITEMS], v[RS_SMALL_ITEMS];
+    int loc[RS_SMALL_ITEMS];
+    rs_rank<RS_SMALL_ITEMS>(keys, vals, n, base, shift, mask, k, v, loc, cnt, pre);   // syncs the CTA
 #pragma unroll
-    for (int r = 0; r < RS_ITEMS; ++r) {
+    for (int r = 0; r < RS_SMALL_ITEMS; ++r) {
         const int64_t idx = base + r * 32 + lane;
         const bool ok = idx < n;
         const uint32_t d = (k[r] >> shift) & mask;
@@ -368,7 +373,8 @@ __global__ __launch_bounds__(RS_THREADS) void k_rs_scatter_small(
             // warp's round: a high digit has few values, whose counters
             // would otherwise take the whole round's atomics each
             const uint32_t slot =
-                ok ? ((k[r] >> shift_next) & mask_next) * (uint32_t)n_tiles + (uint32_t)(pos / RS_TILE)
+                ok ? ((k[r] >> shift_next) & mask_next) * (uint32_t)n_tiles +
+                         (uint32_t)(pos / RS_SMALL_TILE)
                    : 0xffffffffu;
             const unsigned peers = __match_any_sync(0xffffffffu, slot);
             if (ok && lane == __ffs(peers) - 1) atomicAdd(&hnext[slot], (int)__popc(peers));
@@ -379,7 +385,10 @@ __global__ __launch_bounds__(RS_THREADS) void k_rs_scatter_small(
 size_t radix_tmp_bytes(int64_t n) {
     int64_t n_tiles = ceil_div<int64_t>(n, RS_TILE);
     int64_t m = 256 * n_tiles;
-    return (size_t)(2 * m + 1) * sizeof(int64_t) + scan_tmp_bytes(m) + 256;
+    const size_t big = (size_t)(2 * m + 1) * sizeof(int64_t) + scan_tmp_bytes(m) + 256;
+    const int64_t st = ceil_div<int64_t>(n, RS_SMALL_TILE);
+    const size_t small = st <= RS_SMALL_TILES ? (size_t)3 * 256 * st * sizeof(int) + 256 : 0;
+    return big > small ? big : small;
 }
 
 cudaError_t radix_sort_pairs(uint32_t *keys, uint32_t *vals, uint32_t *keys_alt,
@@ -396,9 +405,11 @@ cudaError_t radix_sort_pairs(uint32_t *keys, uint32_t *vals, uint32_t *keys_alt,
     void *stmp = (void *)(offs + m + 1);
     size_t stmp_bytes = tmp_bytes - (size_t)(2 * m + 1) * sizeof(int64_t);
     uint32_t *ki = keys, *vi = vals, *ko = keys_alt, *vo = vals_alt;
-    if (n_tiles <= RS_SMALL_TILES) {
-        int *h[3] = {(int *)tmp, (int *)tmp + m, (int *)tmp + 2 * m};
-        const int nt = (int)n_tiles;
+    const int64_t s_tiles = ceil_div<int64_t>(n, RS_SMALL_TILE);
+    if (s_tiles <= RS_SMALL_TILES) {
+        const int64_t ms = 256 * s_tiles;
+        int *h[3] = {(int *)tmp, (int *)tmp + ms, (int *)tmp + 2 * ms};
+        const int nt = (int)s_tiles;
         k_rs_hist32<<<nt, RS_THREADS, 0, st>>>(ki, n, 0, bits < 8 ? (1u << bits) - 1u : 0xffu, nt,
                                                h[0], h[1], h[2]);
         if (launches) *launches += 1;

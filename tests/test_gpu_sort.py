@@ -1,16 +1,17 @@
 """The library's stable radix sort (akashic_mem_sort_pairs) against numpy's
-stable argsort: both the small form (at most 64 tiles of 4096 pairs: one
+stable argsort: both the small form (at most 256 tiles of 1024 pairs: one
 launch a pass, offsets and next-pass histograms built by the scatter) and
-the large form (tile histograms, a scan, a scatter per pass), at ragged
-sizes on both sides of the switch, with narrow and full key widths and
-many equal keys (stability)."""
+the large form (tiles of 4096 pairs: tile histograms, a scan, a scatter per
+pass), at ragged sizes on both sides of the switch and of a small tile,
+with narrow and full key widths and many equal keys (stability)."""
 import numpy as np
 import pytest
 
 pytestmark = pytest.mark.gpu
 
 TILE = 4096
-SMALL_MAX = 64 * TILE
+SMALL_TILE = 1024
+SMALL_MAX = 256 * SMALL_TILE
 
 
 @pytest.fixture(scope="module", autouse=True)
@@ -39,7 +40,8 @@ def _check(n, bits, key_hi, seed):
     np.testing.assert_array_equal(got_v, vals[order])
 
 
-@pytest.mark.parametrize("n", [2, 31, TILE - 1, TILE, TILE + 1, 32 * TILE, 131_071,
+@pytest.mark.parametrize("n", [2, 31, SMALL_TILE - 1, SMALL_TILE, SMALL_TILE + 1, TILE - 1, TILE,
+                               TILE + 1, 32 * TILE, 131_071,
                                SMALL_MAX - 1, SMALL_MAX, SMALL_MAX + 1, 1_000_003])
 @pytest.mark.parametrize("bits", [5, 8, 20, 32])
 def test_sort_pairs_matches_stable_argsort(n, bits):
