@@ -528,12 +528,13 @@ __global__ __launch_bounds__(256) void k_reach_pack(const float *__restrict__ C,
 
 // Final score of each flagged candidate for each real query column: its u
 // plus the CTAs' partials, appended as a filter key (score bits, ~chunk ID)
-// to the column's buffer; the buffer then holds exactly them.  One block
-// per candidate slot of the plan (blocks past nk, and every block when the
-// plan says the hops run, return at once): thread t takes column t % bp
-// and every (1024 / bp)-th partial from t / bp on (coalesced rows of the
-// partials), and the groups are added in group order (the same order on
-// every run).
+// to the column's buffer; the buffer then holds exactly them.  bp / 64
+// blocks per candidate slot of the plan, each on 64 query columns (blocks
+// past nk, and every block when the plan says the hops run, return at
+// once): thread t takes column t % 64 of its block's and every 16th
+// partial from t / 64 on (coalesced rows of the partials), and the groups
+// are added in group order (the same order on every run).
+constexpr int EMIT_Q = 64, EMIT_G = 1024 / EMIT_Q;
 __global__ __launch_bounds__(1024) void k_reach_emit(const uint16_t *__restrict__ u_hi,
                                                      const uint16_t *__restrict__ u_lo, int bp, int B,
                                                      const float *__restrict__ partial,
@@ -547,18 +548,20 @@ __global__ __launch_bounds__(1024) void k_reach_emit(const uint16_t *__restrict_
     griddep_wait();
     if (plan[0] == 0) return;
     const int nk = plan[1];
-    const int i = blockIdx.x;
+    const int qb_n = bp / EMIT_Q;
+    const int i = blockIdx.x / qb_n;
     if (i >= nk) return;
     const int slot = plan[2 + i];
-    const int b = threadIdx.x % bp, g = threadIdx.x / bp, ng = blockDim.x / bp;
+    const int b = (blockIdx.x % qb_n) * EMIT_Q + threadIdx.x % EMIT_Q;
+    const int g = threadIdx.x / EMIT_Q;
     float acc = 0.f;
-#pragma unroll 16
-    for (int p = g; p < n_parts; p += ng) acc += partial[((int64_t)p * REACH_T + slot) * bp + b];
+#pragma unroll 4
+    for (int p = g; p < n_parts; p += EMIT_G) acc += partial[((int64_t)p * REACH_T + slot) * bp + b];
     red[threadIdx.x] = acc;
     __syncthreads();
     if (g == 0 && b < B) {
-        float sum = red[b];
-        for (int h = 1; h < ng; ++h) sum += red[h * bp + b];
+        float sum = red[threadIdx.x];
+        for (int h = 1; h < EMIT_G; ++h) sum += red[h * EMIT_Q + threadIdx.x];
         const int64_t j = rows[slot];
         const float uj = __bfloat162float(__ushort_as_bfloat16(u_hi[j * bp + b])) +
                          __bfloat162float(__ushort_as_bfloat16(u_lo[j * bp + b]));
@@ -636,7 +639,7 @@ cudaError_t launch_reach_scores(const uint16_t *u_hi, const uint16_t *u_lo, int 
                               : reach_mma_bp<128>(coef_hi, coef_lo, u_hi, u_lo, n, plan, partial,
                                                   parts, status, st);
     if (e != cudaSuccess) return e;
-    e = launch_pdl(k_reach_emit, dim3(REACH_T), dim3(1024), 0, st, u_hi, u_lo, bp, B,
+    e = launch_pdl(k_reach_emit, dim3(REACH_T * (bp / EMIT_Q)), dim3(1024), 0, st, u_hi, u_lo, bp, B,
                    (const float *)partial, parts, plan, rows, ext_of, cnt, buf, cap);
     if (launches) *launches += 2;
     return e == cudaSuccess ? cudaGetLastError() : e;
