@@ -504,6 +504,29 @@ __device__ void column_top(const float *__restrict__ s, int64_t n, int bp, int k
                            int *hist, unsigned long long *s_prefix, int *s_remaining,
                            NsScope ns = NsScope{}) {
     const int64_t m = cnt[c];
+    if (m <= SEL_THREADS) {
+        // few candidates: each thread ranks one key against the others (the
+        // keys are unique but for the padding 0, never selected), and the
+        // keys ranked below k are the ones radix_select would leave in win[]
+        const unsigned long long *bc = buf + (int64_t)c * cap;
+        const int tid = threadIdx.x;
+        if (tid == 0) *win_n = 0;
+        if (tid < m) stage[tid] = bc[tid];
+        __syncthreads();
+        if (tid < m) {
+            const unsigned long long x = stage[tid];
+            if (x != 0ull) {
+                int r = 0;
+                for (int j = 0; j < (int)m; ++j) r += stage[j] > x ? 1 : 0;
+                if (r < k) {
+                    const int p = atomicAdd(win_n, 1);
+                    if (p < 64) win[p] = x;
+                }
+            }
+        }
+        __syncthreads();
+        return;
+    }
     if (m <= cap) {
         const unsigned long long *bc = buf + (int64_t)c * cap;
         if (m <= SEL_STAGE) {
